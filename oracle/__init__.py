@@ -1,0 +1,185 @@
+"""CPU oracle for the latency-aware router -- test infrastructure only.
+
+A ctypes front end to ``sfs_oracle.c``: the literal per-candidate serving
+simulation of Sec. 4.1 (Eq. 7-9) and brute-force routing (Eq. 2, 3, 5).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this package.  The product path (the CUDA library and
+its binding) never does.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+from typing import Optional
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "sfs_oracle.c")
+_LIBDIR = os.path.join(_HERE, "_lib")
+_LIB = os.path.join(_LIBDIR, "libsfs_oracle.so")
+_lib = None
+
+FIRST_TOKEN_SEPARATE_DECODE = 0
+FIRST_TOKEN_WITH_LAST_CHUNK = 1
+DEFAULT_MAX_BATCHES = 1 << 40
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (no fp contraction, no fast-math)."""
+    os.makedirs(_LIBDIR, exist_ok=True)
+    hdr = os.path.join(_HERE, "sfs_oracle.h")
+    if (not force and os.path.exists(_LIB)
+            and os.path.getmtime(_LIB) >= max(os.path.getmtime(_SRC), os.path.getmtime(hdr))):
+        return _LIB
+    tmp = _LIB + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-std=c11", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared",
+           "-o", tmp, _SRC, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        build()
+        lib = ctypes.CDLL(_LIB)
+        P = ctypes.c_void_p
+        i32, i64 = ctypes.c_int32, ctypes.c_int64
+        lib.orc_sfs_candidate.argtypes = [P, i32, i32, i32, i32, i32, i64, P, P, P]
+        lib.orc_sfs_candidate.restype = ctypes.c_int
+        lib.orc_ttft_f32.argtypes = [P, P]
+        lib.orc_ttft_f32.restype = ctypes.c_float
+        lib.orc_ttft_f64.argtypes = [P, P]
+        lib.orc_ttft_f64.restype = ctypes.c_double
+        lib.orc_estimate_candidates.argtypes = [i32, P, P, P, P, i32, i32, P, P, P, P, P, P, P, i32, P, P,
+                                                i32, i64, i64, P, P, P, P, P, P]
+        lib.orc_estimate_candidates.restype = ctypes.c_int
+        lib.orc_route.argtypes = [i32, i32, i32, P, P, P, P, P, P, P, P, i32, P, P, P, P, P]
+        lib.orc_route.restype = ctypes.c_int
+        lib.orc_frontier.argtypes = [i32, i32, i32, P, P, P, P, P, P, i32, P, P, P]
+        lib.orc_frontier.restype = ctypes.c_int
+        lib.orc_utility.argtypes = [ctypes.c_float, ctypes.c_float, i32, i32, ctypes.c_float, ctypes.c_float]
+        lib.orc_utility.restype = ctypes.c_float
+        _lib = lib
+    return _lib
+
+
+def _p(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+class _Instance(ctypes.Structure):
+    _fields_ = [("n_run", ctypes.c_int32), ("run_ctx", ctypes.c_void_p), ("run_pre", ctypes.c_void_p),
+                ("run_dec", ctypes.c_void_p), ("n_wait", ctypes.c_int32), ("wait_pre", ctypes.c_void_p),
+                ("wait_dec", ctypes.c_void_p)]
+
+
+def simulate(running, waiting, B: int, S: int, p: int, d: int = 1, mode: int = FIRST_TOKEN_SEPARATE_DECODE,
+             max_batches: int = DEFAULT_MAX_BATCHES):
+    """One candidate.  running: list of (ctx, pre, dec); waiting: list of (pre, dec).
+
+    Returns (F[5] int64, admit batch, first-token batch)."""
+    run = np.asarray(running, dtype=np.int32).reshape(-1, 3)
+    wt = np.asarray(waiting, dtype=np.int32).reshape(-1, 2)
+    rc_, rp_, rd_ = (_c(run[:, k], np.int32) for k in range(3))
+    wp_, wd_ = (_c(wt[:, k], np.int32) for k in range(2))
+    inst = _Instance(run.shape[0], _p(rc_), _p(rp_), _p(rd_), wt.shape[0], _p(wp_), _p(wd_))
+    F = np.zeros(5, np.int64)
+    la = ctypes.c_int64(0)
+    lt = ctypes.c_int64(0)
+    rc = _load().orc_sfs_candidate(ctypes.byref(inst), B, S, mode, p, d, max_batches, _p(F),
+                                   ctypes.byref(la), ctypes.byref(lt))
+    if rc != 0:
+        raise RuntimeError(f"oracle simulation failed with code {rc}")
+    return F, int(la.value), int(lt.value)
+
+
+def ttft_f32(coef, F) -> np.float32:
+    c = _c(coef, np.float32)
+    f = _c(F, np.int64)
+    return np.float32(_load().orc_ttft_f32(_p(c), _p(f)))
+
+
+def ttft_f64(coef, F) -> float:
+    c = _c(coef, np.float32)
+    f = _c(F, np.int64)
+    return float(_load().orc_ttft_f64(_p(c), _p(f)))
+
+
+def utility(acc, lam, p, dec_hat, price_in, price_out) -> np.float32:
+    return np.float32(_load().orc_utility(float(np.float32(acc)), float(np.float32(lam)), int(p), int(dec_hat),
+                                          float(np.float32(price_in)), float(np.float32(price_out))))
+
+
+def estimate_candidates(wl, cand_q, cand_j, max_batches: int = DEFAULT_MAX_BATCHES):
+    """F[C,5], first-token batch [C], canonical fp32 TTFT [C], fp64 TTFT [C]."""
+    cq = _c(cand_q, np.int32)
+    cj = _c(cand_j, np.int32)
+    C = cq.shape[0]
+    F = np.zeros((C, 5), np.int64)
+    lt = np.zeros(C, np.int64)
+    t32 = np.zeros(C, np.float32)
+    t64 = np.zeros(C, np.float64)
+    arrs = [_c(a, np.int32) for a in (wl.model_of_instance, wl.max_batched_tokens, wl.max_seqs, wl.n_run,
+                                      wl.run_ctx, wl.run_pre, wl.run_dec, wl.n_wait, wl.wait_pre,
+                                      wl.wait_dec, wl.prompt_len, wl.dec_hat)]
+    coef = _c(wl.coef, np.float32)
+    moi, B, S, n_run, run_ctx, run_pre, run_dec, n_wait, wait_pre, wait_dec, p, dh = arrs
+    rc = _load().orc_estimate_candidates(
+        wl.num_instances, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running, wl.cap_waiting, _p(n_run),
+        _p(run_ctx), _p(run_pre), _p(run_dec), _p(n_wait), _p(wait_pre), _p(wait_dec), wl.num_models, _p(p),
+        _p(dh), wl.first_token_mode, max_batches, C, _p(cq), _p(cj), _p(F), _p(lt), _p(t32), _p(t64))
+    if rc != 0:
+        raise RuntimeError(f"oracle estimate failed with code {rc}")
+    return F, lt, t32, t64
+
+
+def estimate_matrix(wl, max_batches: int = DEFAULT_MAX_BATCHES):
+    """Every candidate: F[Q,I,5], first-token batch [Q,I], fp32 [Q,I], fp64 [Q,I]."""
+    Q, I = wl.num_queries, wl.num_instances
+    qq, jj = np.meshgrid(np.arange(Q), np.arange(I), indexing="ij")
+    F, lt, t32, t64 = estimate_candidates(wl, qq.ravel(), jj.ravel(), max_batches)
+    return F.reshape(Q, I, 5), lt.reshape(Q, I), t32.reshape(Q, I), t64.reshape(Q, I)
+
+
+def route(wl, ttft32: np.ndarray, lam=None, mu=None, tau=None):
+    """Brute-force routing over full TTFT rows: assign/util/ttft_chosen [P,Q]."""
+    lam = _c(wl.lam if lam is None else lam, np.float32)
+    P = lam.shape[0]
+    mu_a = _c(np.zeros(P, np.float32) if (mu is None and tau is not None) else (wl.mu if mu is None else mu),
+              np.float32)
+    t = _c(ttft32, np.float32)
+    Q, I = t.shape
+    tau_a = None if tau is None else _c(tau, np.float32)
+    assign = np.zeros((P, Q), np.int32)
+    util = np.zeros((P, Q), np.float32)
+    tch = np.zeros((P, Q), np.float32)
+    moi, p, dh = (_c(a, np.int32) for a in (wl.model_of_instance, wl.prompt_len, wl.dec_hat))
+    acc, pin, pout = (_c(a, np.float32) for a in (wl.acc, wl.price_in, wl.price_out))
+    rc = _load().orc_route(Q, I, wl.num_models, _p(moi), _p(pin), _p(pout), _p(p), _p(dh), _p(acc), _p(t),
+                           _p(tau_a), P, _p(lam), _p(mu_a), _p(assign), _p(util), _p(tch))
+    if rc != 0:
+        raise RuntimeError(f"oracle route failed with code {rc}")
+    return assign, util, tch
+
+
+def frontier(wl, assign: np.ndarray, ttft_chosen: np.ndarray) -> np.ndarray:
+    a = _c(assign, np.int32)
+    tch = _c(ttft_chosen, np.float32)
+    P, Q = a.shape
+    out = np.zeros((P, 3), np.float64)
+    moi, p, dh = (_c(x, np.int32) for x in (wl.model_of_instance, wl.prompt_len, wl.dec_hat))
+    acc, pin, pout = (_c(x, np.float32) for x in (wl.acc, wl.price_in, wl.price_out))
+    rc = _load().orc_frontier(Q, wl.num_instances, wl.num_models, _p(moi), _p(pin), _p(pout), _p(p), _p(dh),
+                              _p(acc), P, _p(a), _p(tch), _p(out))
+    if rc != 0:
+        raise RuntimeError(f"oracle frontier failed with code {rc}")
+    return out

@@ -1,0 +1,284 @@
+/*
+ * CPU oracle for the latency-aware router -- test infrastructure only.
+ *
+ * Literal restatement of the paper's Serving Framework Simulation (Sec. 4.1)
+ * and routing objectives (Sec. 3).  Nothing here is blocked, fused or
+ * reordered: each candidate is simulated on its own, one token batch after
+ * another, with the whole resident set in a plain array.  Built with
+ * -ffp-contract=off so that the only fused multiply-adds are the explicit
+ * fmaf() calls of the canonical expressions below.
+ *
+ * Readings of points the paper leaves open (each is a stated convention):
+ *  - Scheduler step (Sec. 2 "chunked prefills", App. F "queue order, admission
+ *    limits, token-budget constraints"): a batch starts with budget B; the
+ *    running list is served in order, a request with remaining prefill taking
+ *    min(remaining, budget) tokens and a decoding request one token, until the
+ *    budget is spent; then, while budget remains, the waiting list is non-empty
+ *    and fewer than S requests run, the waiting head is admitted FCFS with a
+ *    prefill chunk of min(prompt, budget).  Requests whose decode count reaches
+ *    zero leave after the batch.
+ *  - First output token: by default a separate decode batch after the last
+ *    prefill chunk (Sec. 4.1 "the decode stage ... begins only after all
+ *    prefill tokens"); optionally sampled in the batch of the last chunk.
+ *  - Context of a decode token = tokens in the KV cache before the batch.
+ *  - KV capacity is unbounded and nothing is preempted.
+ *  - Canonical fp32 order for Eq. 9 summed over batches: intercept, decode
+ *    tokens, prefill tokens, decode context, prefill attention.
+ *
+ * parity pins: tests/test_oracle_pins.py (closed forms, hand traces, invariants).
+ */
+#include "sfs_oracle.h"
+
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+typedef struct {
+    int64_t ctx;  /* tokens already in the KV cache */
+    int64_t pre;  /* remaining prefill tokens */
+    int64_t dec;  /* remaining decode tokens */
+    int is_query; /* the new query q_i */
+} orc_req;
+
+enum { SCHED_NONE = 0, SCHED_PREFILL = 1, SCHED_DECODE = 2 };
+
+static int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
+
+/*
+ * The augmented workload X_{i,j} (Sec. 4.1): the resident set R_j = Q_j u A_j
+ * plus q_i at the tail of the waiting queue.  Simulate token batches
+ * l = 1, 2, ... until q_i produces its first output token (Eq. 7) and return
+ * the batch features whose Eq. 9 weighted sum, added over those batches,
+ * is the SFS TTFT of Eq. 8.
+ */
+int orc_sfs_candidate(const orc_instance *inst, int32_t B, int32_t S, int32_t mode,
+                      int32_t p, int32_t d, int64_t max_batches,
+                      int64_t F[5], int64_t *l_admit, int64_t *l_ttft)
+{
+    if (!inst || !F || B < 1 || S < 1 || p < 1 || d < 1 || inst->n_run < 0 || inst->n_wait < 0)
+        return ORC_EINVAL;
+    if (mode != ORC_FIRST_TOKEN_SEPARATE_DECODE && mode != ORC_FIRST_TOKEN_WITH_LAST_CHUNK)
+        return ORC_EINVAL;
+    const int64_t total = (int64_t)inst->n_run + inst->n_wait + 1;
+    orc_req *run = (orc_req *)calloc((size_t)total, sizeof(orc_req));
+    orc_req *wait = (orc_req *)calloc((size_t)total, sizeof(orc_req));
+    int64_t *alloc = (int64_t *)calloc((size_t)total, sizeof(int64_t));
+    int *kind = (int *)calloc((size_t)total, sizeof(int));
+    if (!run || !wait || !alloc || !kind) {
+        free(run); free(wait); free(alloc); free(kind);
+        return ORC_ENOMEM;
+    }
+    int64_t nr = 0, nw = 0, wh = 0;
+    for (int32_t r = 0; r < inst->n_run; ++r) {
+        run[nr].ctx = inst->run_ctx[r];
+        run[nr].pre = inst->run_pre[r];
+        run[nr].dec = inst->run_dec[r];
+        run[nr].is_query = 0;
+        if (run[nr].ctx < 0 || run[nr].pre < 0 || run[nr].dec < 1) goto bad;
+        ++nr;
+    }
+    for (int32_t w = 0; w < inst->n_wait; ++w) {
+        wait[nw].ctx = 0;
+        wait[nw].pre = inst->wait_pre[w];
+        wait[nw].dec = inst->wait_dec[w];
+        wait[nw].is_query = 0;
+        if (wait[nw].pre < 1 || wait[nw].dec < 1) goto bad;
+        ++nw;
+    }
+    wait[nw].ctx = 0; wait[nw].pre = p; wait[nw].dec = d; wait[nw].is_query = 1;
+    ++nw;
+
+    for (int k = 0; k < 5; ++k) F[k] = 0;
+    int64_t admitted_at = 0;
+    for (int64_t l = 1; l <= max_batches; ++l) {
+        /* 1. serve the running list in order until the token budget is spent */
+        int64_t budget = B;
+        for (int64_t r = 0; r < nr; ++r) { kind[r] = SCHED_NONE; alloc[r] = 0; }
+        for (int64_t r = 0; r < nr && budget > 0; ++r) {
+            if (run[r].pre > 0) {
+                alloc[r] = min64(run[r].pre, budget);
+                kind[r] = SCHED_PREFILL;
+            } else {
+                alloc[r] = 1;
+                kind[r] = SCHED_DECODE;
+            }
+            budget -= alloc[r];
+        }
+        /* 2. admit from the waiting head while budget and a sequence slot remain */
+        while (budget > 0 && wh < nw && nr < S) {
+            run[nr] = wait[wh++];
+            alloc[nr] = min64(run[nr].pre, budget);
+            kind[nr] = SCHED_PREFILL;
+            budget -= alloc[nr];
+            if (run[nr].is_query) admitted_at = l;
+            ++nr;
+        }
+        /* 3. account the batch: the feature vector of Eq. 9 */
+        int done = 0;
+        F[0] += 1;
+        for (int64_t r = 0; r < nr; ++r) {
+            if (kind[r] == SCHED_PREFILL) {
+                const int64_t x = alloc[r];
+                F[1] += x;
+                F[4] += x * run[r].ctx + x * (x + 1) / 2;
+                run[r].ctx += x;
+                run[r].pre -= x;
+                if (run[r].pre == 0 && mode == ORC_FIRST_TOKEN_WITH_LAST_CHUNK) {
+                    run[r].dec -= 1;              /* first token sampled with the last chunk */
+                    if (run[r].is_query) done = 1;
+                }
+            } else if (kind[r] == SCHED_DECODE) {
+                F[2] += 1;
+                F[3] += run[r].ctx;
+                run[r].ctx += 1;
+                run[r].dec -= 1;
+                if (run[r].is_query) done = 1;    /* Eq. 7: first batch with a decode token of q_i */
+            }
+        }
+        if (done) {
+            if (l_admit) *l_admit = admitted_at;
+            if (l_ttft) *l_ttft = l;
+            free(run); free(wait); free(alloc); free(kind);
+            return ORC_OK;
+        }
+        /* 4. finished requests leave the running list (order kept) */
+        int64_t keep = 0;
+        for (int64_t r = 0; r < nr; ++r)
+            if (run[r].dec > 0) run[keep++] = run[r];
+        nr = keep;
+    }
+    free(run); free(wait); free(alloc); free(kind);
+    return ORC_ELIMIT;
+bad:
+    free(run); free(wait); free(alloc); free(kind);
+    return ORC_EINVAL;
+}
+
+/* Eq. 9 summed over the batches up to the first-token batch (Eq. 8):
+ * T = b0*F0 + b1p*F1 + b1d*F2 + b2*F3 + b3*F4, evaluated in this fixed fp32 order. */
+float orc_ttft_f32(const float coef[5], const int64_t F[5])
+{
+    const float f0 = (float)F[0], f1 = (float)F[1], f2 = (float)F[2];
+    const float f3 = (float)F[3], f4 = (float)F[4];
+    float t = coef[0] * f0;
+    t = fmaf(coef[2], f2, t);
+    t = fmaf(coef[1], f1, t);
+    t = fmaf(coef[3], f3, t);
+    t = fmaf(coef[4], f4, t);
+    return t;
+}
+
+double orc_ttft_f64(const float coef[5], const int64_t F[5])
+{
+    return (double)coef[0] * (double)F[0] + (double)coef[1] * (double)F[1] +
+           (double)coef[2] * (double)F[2] + (double)coef[3] * (double)F[3] +
+           (double)coef[4] * (double)F[4];
+}
+
+int orc_estimate_candidates(int32_t num_instances, const int32_t *model_of_instance,
+                            const float *coef, const int32_t *B, const int32_t *S,
+                            int32_t cap_running, int32_t cap_waiting,
+                            const int32_t *n_run, const int32_t *run_ctx, const int32_t *run_pre,
+                            const int32_t *run_dec, const int32_t *n_wait, const int32_t *wait_pre,
+                            const int32_t *wait_dec, int32_t num_models, const int32_t *prompt_len,
+                            const int32_t *dec_hat, int32_t mode, int64_t max_batches,
+                            int64_t num_cand, const int32_t *cand_q, const int32_t *cand_j,
+                            int64_t *F, int64_t *l_ttft, float *ttft32, double *ttft64)
+{
+    for (int64_t c = 0; c < num_cand; ++c) {
+        const int32_t i = cand_q[c], j = cand_j[c];
+        if (j < 0 || j >= num_instances) return ORC_EINVAL;
+        const int32_t m = model_of_instance[j];
+        if (m < 0 || m >= num_models) return ORC_EINVAL;
+        orc_instance inst;
+        inst.n_run = n_run[j];
+        inst.run_ctx = run_ctx + (int64_t)j * cap_running;
+        inst.run_pre = run_pre + (int64_t)j * cap_running;
+        inst.run_dec = run_dec + (int64_t)j * cap_running;
+        inst.n_wait = n_wait[j];
+        inst.wait_pre = wait_pre + (int64_t)j * cap_waiting;
+        inst.wait_dec = wait_dec + (int64_t)j * cap_waiting;
+        if (inst.n_run > cap_running || inst.n_wait > cap_waiting) return ORC_EINVAL;
+        int64_t Fc[5], la = 0, lt = 0;
+        const int rc = orc_sfs_candidate(&inst, B[j], S[j], mode, prompt_len[i],
+                                         dec_hat[(int64_t)i * num_models + m], max_batches, Fc, &la, &lt);
+        if (rc != ORC_OK) return rc;
+        for (int k = 0; k < 5; ++k) F[c * 5 + k] = Fc[k];
+        if (l_ttft) l_ttft[c] = lt;
+        if (ttft32) ttft32[c] = orc_ttft_f32(coef + 5 * m, Fc);
+        if (ttft64) ttft64[c] = orc_ttft_f64(coef + 5 * m, Fc);
+    }
+    return ORC_OK;
+}
+
+/* Eq. 2 with the predicted cost of App. B.4:
+ * cost = p * price_in + dec_hat * price_out, U = acc - lambda * cost (fp32, explicit fma). */
+float orc_utility(float acc, float lambda, int32_t p, int32_t dec_hat, float price_in, float price_out)
+{
+    const float cost = fmaf((float)dec_hat, price_out, (float)p * price_in);
+    return fmaf(-lambda, cost, acc);
+}
+
+int orc_route(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instance,
+              const float *price_in, const float *price_out, const int32_t *prompt_len,
+              const int32_t *dec_hat, const float *acc, const float *ttft, const float *tau,
+              int32_t P, const float *lambda, const float *mu,
+              int32_t *assign, float *util, float *ttft_chosen)
+{
+    if (Q < 0 || I < 1 || M < 1 || P < 1) return ORC_EINVAL;
+    for (int32_t pp = 0; pp < P; ++pp) {
+        for (int32_t i = 0; i < Q; ++i) {
+            const float *row = ttft + (int64_t)i * I;
+            int32_t best_j = -1, fast_j = -1;
+            float best = 0.0f, best_u = 0.0f, fast_t = 0.0f;
+            for (int32_t j = 0; j < I; ++j) {
+                const int32_t m = model_of_instance[j];
+                const float u = orc_utility(acc[(int64_t)i * M + m], lambda[pp], prompt_len[i],
+                                            dec_hat[(int64_t)i * M + m], price_in[m], price_out[m]);
+                const float t = row[j];
+                if (tau == NULL) {
+                    /* Eq. 5: argmax_j U - mu * L, ties to the lowest index */
+                    const float J = fmaf(-mu[pp], t, u);
+                    if (best_j < 0 || J > best) { best = J; best_j = j; best_u = u; }
+                } else {
+                    /* Eq. 3: argmax U over {j : L <= tau}; empty set -> least latency */
+                    if (t <= tau[i] && (best_j < 0 || u > best_u)) { best_u = u; best_j = j; }
+                    if (fast_j < 0 || t < fast_t) { fast_t = t; fast_j = j; }
+                }
+            }
+            int32_t pick = best_j;
+            if (tau != NULL && best_j < 0) pick = fast_j;
+            const int32_t m = model_of_instance[pick];
+            assign[(int64_t)pp * Q + i] = pick;
+            util[(int64_t)pp * Q + i] = orc_utility(acc[(int64_t)i * M + m], lambda[pp], prompt_len[i],
+                                                    dec_hat[(int64_t)i * M + m], price_in[m], price_out[m]);
+            if (ttft_chosen) ttft_chosen[(int64_t)pp * Q + i] = row[pick];
+        }
+    }
+    return ORC_OK;
+}
+
+int orc_frontier(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instance,
+                 const float *price_in, const float *price_out, const int32_t *prompt_len,
+                 const int32_t *dec_hat, const float *acc, int32_t P, const int32_t *assign,
+                 const float *ttft_chosen, double *out)
+{
+    if (Q < 1 || P < 1) return ORC_EINVAL;
+    for (int32_t pp = 0; pp < P; ++pp) {
+        double sa = 0.0, sc = 0.0, st = 0.0;
+        for (int32_t i = 0; i < Q; ++i) {
+            const int32_t j = assign[(int64_t)pp * Q + i];
+            if (j < 0 || j >= I) return ORC_EINVAL;
+            const int32_t m = model_of_instance[j];
+            const float cost = fmaf((float)dec_hat[(int64_t)i * M + m], price_out[m],
+                                    (float)prompt_len[i] * price_in[m]);
+            sa += (double)acc[(int64_t)i * M + m];
+            sc += (double)cost;
+            st += (double)ttft_chosen[(int64_t)pp * Q + i];
+        }
+        out[pp * 3 + 0] = sa / Q;
+        out[pp * 3 + 1] = sc / Q;
+        out[pp * 3 + 2] = st / Q;
+    }
+    return ORC_OK;
+}

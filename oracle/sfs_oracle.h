@@ -1,0 +1,82 @@
+/*
+ * CPU oracle for the latency-aware router (test infrastructure only).
+ *
+ * Plain, slow, literal C: for every (query, instance) candidate it copies the
+ * instance's resident set, appends the query at the FCFS waiting tail and
+ * steps the serving scheduler one token batch at a time until the query's
+ * first output token (Sec. 4.1, Eq. 7 and Eq. 8), accumulating the five batch
+ * features that Eq. 9 is linear in.  Routing is brute-force enumeration over
+ * instances (Eq. 2, Eq. 3, Eq. 5).
+ *
+ * Only the test suite, the package smoke check and the benchmark's CPU
+ * baseline use this library.  It shares no code, header or constant with the
+ * CUDA library and is never on the product path.
+ */
+#ifndef SFS_ORACLE_H
+#define SFS_ORACLE_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum { ORC_OK = 0, ORC_EINVAL = 1, ORC_ELIMIT = 2, ORC_ENOMEM = 3 };
+enum { ORC_FIRST_TOKEN_SEPARATE_DECODE = 0, ORC_FIRST_TOKEN_WITH_LAST_CHUNK = 1 };
+
+/* One instance's snapshot: running list (admission order) and waiting list (FCFS order). */
+typedef struct {
+    int32_t n_run;
+    const int32_t *run_ctx, *run_pre, *run_dec;
+    int32_t n_wait;
+    const int32_t *wait_pre, *wait_dec;
+} orc_instance;
+
+/* Simulate one candidate: instance `inst` with budget B and sequence cap S plus a new
+ * query of prompt p and predicted decode d appended at the waiting tail.
+ * Writes F[5] = (batches, prefill tokens, decode tokens, sum ctx*dec, sum prefill
+ * attention pairs) over batches 1..l_ttft, the batch index that admitted the query
+ * and the query's first-token batch.  Returns ORC_ELIMIT after max_batches. */
+int orc_sfs_candidate(const orc_instance *inst, int32_t B, int32_t S, int32_t mode,
+                      int32_t p, int32_t d, int64_t max_batches,
+                      int64_t F[5], int64_t *l_admit, int64_t *l_ttft);
+
+/* Canonical single-precision batch-time sum (Eq. 9 summed per Eq. 8) and its fp64 value. */
+float orc_ttft_f32(const float coef[5], const int64_t F[5]);
+double orc_ttft_f64(const float coef[5], const int64_t F[5]);
+
+/* Every candidate of a list: cand_q[c], cand_j[c] index the queries / instances.
+ * State arrays are [I][cap] row-major.  Outputs per candidate: F[c][5],
+ * l_ttft[c], ttft32[c], ttft64[c]. */
+int orc_estimate_candidates(int32_t num_instances, const int32_t *model_of_instance,
+                            const float *coef, const int32_t *B, const int32_t *S,
+                            int32_t cap_running, int32_t cap_waiting,
+                            const int32_t *n_run, const int32_t *run_ctx, const int32_t *run_pre,
+                            const int32_t *run_dec, const int32_t *n_wait, const int32_t *wait_pre,
+                            const int32_t *wait_dec, int32_t num_models, const int32_t *prompt_len,
+                            const int32_t *dec_hat, int32_t mode, int64_t max_batches,
+                            int64_t num_cand, const int32_t *cand_q, const int32_t *cand_j,
+                            int64_t *F, int64_t *l_ttft, float *ttft32, double *ttft64);
+
+/* Brute-force routing of Q queries given their full TTFT rows ttft[Q][I] (canonical fp32).
+ * tau == NULL: Lagrangian objective (Eq. 5) for each of the P (lambda, mu) pairs.
+ * tau != NULL: constrained objective (Eq. 3) for each lambda; mu is ignored.
+ * Outputs [P][Q]: assign, util (U of the chosen instance), ttft_chosen. */
+int orc_route(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instance,
+              const float *price_in, const float *price_out, const int32_t *prompt_len,
+              const int32_t *dec_hat, const float *acc, const float *ttft, const float *tau,
+              int32_t P, const float *lambda, const float *mu,
+              int32_t *assign, float *util, float *ttft_chosen);
+
+/* Per-pair means of accuracy, cost and TTFT of the chosen instances: out[P][3]. */
+int orc_frontier(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instance,
+                 const float *price_in, const float *price_out, const int32_t *prompt_len,
+                 const int32_t *dec_hat, const float *acc, int32_t P, const int32_t *assign,
+                 const float *ttft_chosen, double *out);
+
+/* Utility of Eq. 2 with the cost of App. B.4 in canonical fp32. */
+float orc_utility(float acc, float lambda, int32_t p, int32_t dec_hat, float price_in, float price_out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif
