@@ -1,0 +1,347 @@
+"""Benchmark of the router hot path on one GB300 (or N independent replicas).
+
+A step is one pass of the whole hot path over one batch: ingest the instance
+snapshot (copy + per-instance trajectory summary) and route every query of the
+batch -- SFS TTFT for every (query, instance) candidate written as the full
+estimate matrix, utility, Lagrangian argmax.  Workload: "pool256", 256
+instances (8 models x 32 replicas) and 65,536 queries, seeded synthetic.
+
+value      = candidates (query x instance) per second, device time, inputs resident
+e2e        = same metric through the public API from pinned host buffers, with the
+             host->device copy of the snapshot and queries and the device->host copy
+             of the routing result inside each timed step
+roofline   = the dominant kernel against measured HBM bandwidth
+cpu_baseline / --impl reference = the CPU oracle (literal per-candidate simulation)
+"""
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "TTFT estimates/sec (query×instance) on 1 GB300; p50 per-batch route latency"
+UNIT = "estimates/s"
+WORKLOAD = "pool256"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _dist():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def _config_desc(wl, extra=None):
+    d = {"workload": f"{WORKLOAD}: {wl.num_instances} instances ({wl.num_models} models x "
+                     f"{wl.num_instances // wl.num_models} replicas) x {wl.num_queries} queries, "
+                     f"B={int(wl.max_batched_tokens[0])}, S={int(wl.max_seqs[0])}, prompts <= {wl.max_prompt_len}",
+         "instances": wl.num_instances, "queries_per_batch": wl.num_queries,
+         "step": "lr_load_state + lr_route (full TTFT matrix, Lagrangian argmax)",
+         "l2": "flushed (256 MiB write) between timed steps",
+         "parallelism": "replicas"}
+    if extra:
+        d.update(extra)
+    return d
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}",
+                 "--query-gpu=index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap",
+                 "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        try:
+            for line in open(self.path):
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax = float(parts[2])
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        except OSError:
+            pass
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax, "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    import __graft_entry__
+    from paper_2607_18253_gb300 import router as R
+    from paper_2607_18253_gb300 import workloads as W
+
+    rank, world, local = _dist()
+    if world > 1:
+        dist.init_process_group("gloo")
+    torch.cuda.set_device(local)
+    if rank == 0:
+        __graft_entry__.build()
+    if world > 1:
+        dist.barrier()
+    dev = torch.device("cuda", local)
+
+    wl = W.make_workload(WORKLOAD)
+    Q, I, M = wl.num_queries, wl.num_instances, wl.num_models
+    rt = R.LatencyRouter.from_workload(wl)
+    state = R.state_tensors(wl, dev)
+    p, dh, acc, _ = R.query_tensors(wl, dev)
+    mat = torch.empty((Q, I), dtype=torch.float32, device=dev)
+    out = {"assign": torch.empty((1, Q), dtype=torch.int32, device=dev),
+           "util": torch.empty((1, Q), dtype=torch.float32, device=dev),
+           "ttft_chosen": torch.empty((1, Q), dtype=torch.float32, device=dev)}
+    flush = torch.empty(64 << 20, dtype=torch.float32, device=dev)  # 256 MiB > L2
+    stream = torch.cuda.current_stream()
+
+    def step():
+        rt.load_state(*state)
+        rt.route(p, dh, acc, wl.lam, wl.mu, ttft_matrix=mat, out=out)
+
+    for _ in range(args.warmup):
+        flush.fill_(1.0)
+        step()
+    torch.cuda.synchronize()
+    st = rt.status()
+    if st != R.LR_OK:
+        raise RuntimeError(f"device status {st} after warm-up")
+
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with Clocks(local) as clk:
+        t_wall0 = time.perf_counter()
+        for k in range(K):
+            flush.fill_(float(k))
+            ev[k][0].record(stream)
+            rt.load_state(*state)
+            ev[k][1].record(stream)
+            rt.route(p, dh, acc, wl.lam, wl.mu, ttft_matrix=mat, out=out)
+            ev[k][2].record(stream)
+        torch.cuda.synchronize()
+        t_wall = time.perf_counter() - t_wall0
+    if world > 1:
+        dist.barrier()
+    load_ms = [ev[k][0].elapsed_time(ev[k][1]) for k in range(K)]
+    route_ms = [ev[k][1].elapsed_time(ev[k][2]) for k in range(K)]
+    step_ms = [a + b for a, b in zip(load_ms, route_ms)]
+    total_ms = sum(step_ms)
+    if world > 1:
+        tt = torch.tensor([total_ms], dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    ms_per_step = total_ms / K
+    cands = Q * I
+    value = cands * world / (ms_per_step * 1e-3)
+
+    # end to end: pinned host buffers -> device, load + route, result -> host
+    host_state = [t.cpu().pin_memory() for t in state]
+    host_q = [t.cpu().pin_memory() for t in (p, dh, acc)]
+    dstate = [torch.empty_like(t) for t in state]
+    dq = [torch.empty_like(t) for t in (p, dh, acc)]
+    host_out = {k: torch.empty(v.shape, dtype=v.dtype).pin_memory() for k, v in out.items()}
+    h2d = sum(t.numel() * t.element_size() for t in host_state + host_q)
+    d2h = sum(t.numel() * t.element_size() for t in host_out.values())
+
+    def e2e_step():
+        for d, h in zip(dstate + dq, host_state + host_q):
+            d.copy_(h, non_blocking=True)
+        rt.load_state(*dstate)
+        rt.route(dq[0], dq[1], dq[2], wl.lam, wl.mu, ttft_matrix=mat, out=out)
+        for k, v in out.items():
+            host_out[k].copy_(v, non_blocking=True)
+
+    for _ in range(args.warmup):
+        e2e_step()
+    torch.cuda.synchronize()
+    KE = max(3, min(K, 200))
+    e2e_ms = []
+    for k in range(KE):
+        flush.fill_(float(k))
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        e2e_step()
+        e1.record(stream)
+        e1.synchronize()  # the result is on the host after this
+        e2e_ms.append(e0.elapsed_time(e1))
+    e2e_mean = sum(e2e_ms) / KE
+    if world > 1:
+        tt = torch.tensor([e2e_mean], dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_mean = float(tt.item())
+    assert rt.status() == R.LR_OK
+
+    # roofline of the dominant kernel (algorithmic bytes / event-timed duration)
+    hbm, peak_src = _peaks()
+    load_avg = sum(load_ms) / K
+    route_avg = sum(route_ms) / K
+    route_bytes = cands * 4 + Q * (4 + 8 * M) + Q * 12
+    load_bytes = 2 * 4 * (I * (3 * wl.cap_running + 2 * wl.cap_waiting) + 2 * I)
+    kernels = {
+        "k_route (TTFT matrix + utility + argmax)": {"ms": route_avg, "share": route_avg / ms_per_step,
+                                                      "algorithmic_bytes": route_bytes},
+        "k_trajectory (snapshot copy + summary)": {"ms": load_avg, "share": load_avg / ms_per_step,
+                                                    "algorithmic_bytes": load_bytes},
+    }
+    if route_avg >= load_avg:
+        ach = route_bytes / (route_avg * 1e-3) / 1e9
+        roof = {"kernel": "k_route", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+                "frac": ach / hbm, "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs, copy)",
+                "traffic": args.traffic}
+    else:
+        ach = load_bytes / (load_avg * 1e-3) / 1e9
+        roof = {"kernel": "k_trajectory", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+                "frac": ach / hbm, "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs, copy)",
+                "traffic": None, "note": "latency-bound event loop; bytes fraction shown for reference"}
+
+    if rank == 0:
+        cpu = cpu_baseline(wl, args.cpu_seconds) if (world == 1 and not args.no_cpu) else None
+        srt = sorted(step_ms)
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
+            "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32+i64", "data": "synthetic (seeded lognormal/uniform stand-ins, see DESIGN.md)",
+            "config": _config_desc(wl),
+            "p50_step_ms": srt[len(srt) // 2], "p99_step_ms": srt[min(len(srt) - 1, int(0.99 * len(srt)))],
+            "kernels": kernels, "roofline": roof, "cpu_baseline": cpu,
+            "e2e": {"value": cands * world / (e2e_mean * 1e-3), "unit": UNIT, "ms_per_step": e2e_mean,
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": 2 * K, "clocks": clk.summary(), "wall_s_timed_region": t_wall,
+        }
+        print(json.dumps(line), flush=True)
+    rt.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def _oracle_rows(wl, nq, seed):
+    """Full TTFT rows for nq sampled queries, then the oracle's argmax over them."""
+    import oracle
+    rng = np.random.default_rng(seed)
+    qs = np.sort(rng.choice(wl.num_queries, nq, replace=False))
+    sub = wl.with_queries(qs)
+    t0 = time.perf_counter()
+    _, _, t32, _ = oracle.estimate_matrix(sub)
+    oracle.route(sub, t32)
+    return nq * wl.num_instances, time.perf_counter() - t0
+
+
+def cpu_baseline(wl, seconds: float):
+    """The oracle as it stands, one host core, on a bounded sample of the workload."""
+    cands, dt = _oracle_rows(wl, 8, 1)
+    per = dt / cands
+    nq = max(8, min(wl.num_queries, int(seconds / (per * wl.num_instances))))
+    cands, dt = _oracle_rows(wl, nq, 2)
+    return {"value": cands / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{nq} random queries of {WORKLOAD} x all {wl.num_instances} instances "
+                      f"({cands} candidates, {dt:.1f} s): literal per-candidate simulation + brute-force argmax"}
+
+
+def run_reference(args):
+    rank, world, _ = _dist()
+    if rank != 0:
+        return
+    import oracle
+    from paper_2607_18253_gb300 import workloads as W
+    oracle.build()
+    wl = W.make_workload(WORKLOAD)
+    cands, dt = _oracle_rows(wl, 4, 0)
+    per_row = dt / 4
+    # about two minutes in total, whatever K and W are
+    step_s = min(args.ref_step_seconds, 120.0 / max(1, args.steps + args.warmup))
+    nq = max(2, min(wl.num_queries, int(step_s / per_row)))
+    for w in range(args.warmup):
+        _oracle_rows(wl, nq, 100 + w)
+    times = []
+    for k in range(args.steps):
+        c, t = _oracle_rows(wl, nq, 1000 + k)
+        times.append(t)
+    ms = 1e3 * sum(times) / len(times)
+    v = nq * wl.num_instances / (ms * 1e-3)
+    sample = (f"each step: {nq} random queries of {WORKLOAD} x all {wl.num_instances} instances, literal "
+              f"per-candidate simulation + brute-force argmax, 1 host core")
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32+i64", "data": "synthetic", "config": _config_desc(wl),
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--ref-step-seconds", type=float, default=2.0)
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--traffic", type=float, default=None,
+                    help="dram bytes per launch of the dominant kernel from an ncu capture of this build")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,175 @@
+/*
+ * latency_router.h -- C ABI of the GB300 latency-aware router hot path.
+ *
+ * The library estimates, for every (query, model instance) candidate, the
+ * time to first token by the Serving Framework Simulation of Sec. 4.1: the
+ * instance's resident requests plus the new query at the tail of its FCFS
+ * waiting queue are stepped through token batches (chunked prefill under a
+ * token budget and a sequence cap) until the query's first output token
+ * (Eq. 7); the estimate is the sum over those batches (Eq. 8) of the batch
+ * time model of Eq. 9.  It then scores each candidate with the accuracy-cost
+ * utility of Eq. 2 and picks one instance per query by the Lagrangian
+ * objective of Eq. 5 or the latency-constrained objective of Eq. 3.
+ *
+ * Conventions for every call:
+ *  - All integers are int32 unless stated; all arrays are dense, row-major.
+ *  - Configuration arrays passed to lr_create are host pointers, copied.
+ *  - Per-call arrays are DEVICE pointers owned by the caller; the library
+ *    reads or writes them only inside work enqueued on `cuda_stream`
+ *    (a cudaStream_t; NULL means the legacy default stream).
+ *  - Calls are asynchronous on that stream.  Calls on one context must be
+ *    ordered by the caller (one stream, or events between streams).
+ *  - Errors a host can see (null pointers, sizes beyond capacity, invalid
+ *    limits) are returned immediately and nothing is enqueued.  Errors found
+ *    on the device (an invalid snapshot, a trajectory longer than max_iters,
+ *    a prompt length out of range) are recorded in a device status word that
+ *    lr_status() returns; affected outputs are NaN (times) or -1 (indices).
+ *  - The library never aborts, throws or leaves a device loop unbounded.
+ */
+#ifndef LATENCY_ROUTER_H
+#define LATENCY_ROUTER_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define LR_API __attribute__((visibility("default")))
+#else
+#define LR_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Return codes. */
+enum lr_code {
+    LR_OK = 0,
+    LR_EINVAL = 1,      /* invalid argument or invalid input value */
+    LR_ENOMEM = 2,      /* device or host allocation failed */
+    LR_ECUDA = 3,       /* a CUDA runtime call failed (see lr_last_error) */
+    LR_ECAPACITY = 4,   /* a size exceeds what the context was created for */
+    LR_ETRAJ = 5,       /* a simulated trajectory exceeded max_iters (device) */
+    LR_ESTATE = 6,      /* a snapshot violates the state preconditions (device) */
+    LR_ENOSTATE = 7     /* no snapshot has been loaded successfully yet (device) */
+};
+
+/* When the first output token is produced (Sec. 4.1: the decode stage begins only
+ * after all prefill tokens have been processed). */
+enum lr_first_token_mode {
+    LR_FIRST_TOKEN_SEPARATE_DECODE = 0,  /* its own decode batch after the last prefill chunk (default) */
+    LR_FIRST_TOKEN_WITH_LAST_CHUNK = 1   /* sampled in the batch that completes the prompt */
+};
+
+/* Pool description (Sec. 3 "System model"; Eq. 9 coefficients; App. B.4 prices). */
+typedef struct {
+    int32_t num_instances;             /* I >= 1 model instances j */
+    int32_t num_models;                /* M >= 1 distinct models */
+    const int32_t *model_of_instance;  /* [I] in [0, M) */
+    const float *coef;                 /* [M][5] Eq. 9 coefficients in seconds:
+                                          beta0 (per batch), beta1p (per prefill token),
+                                          beta1d (per decode token), beta2 (per decode token
+                                          and token of context), beta3 (per prefill attention
+                                          pair); the paper's form has beta1p == beta1d.
+                                          Finite and >= 0. */
+    const float *price_in;             /* [M] $ per prompt token, finite >= 0 */
+    const float *price_out;            /* [M] $ per response token, finite >= 0 */
+    const int32_t *max_batched_tokens; /* [I] token budget B_j per batch, 1..2^24 */
+    const int32_t *max_seqs;           /* [I] sequence cap S_j, 1 <= S_j <= B_j */
+    int32_t cap_running;               /* row stride of the running arrays (>= 1) */
+    int32_t cap_waiting;               /* row stride of the waiting arrays (>= 1) */
+    int32_t max_queries;               /* largest Q of any call */
+    int32_t max_pairs;                 /* largest P of lr_route, 1..64 */
+    int32_t max_prompt_len;            /* largest prompt length of any query, 1..2^20 */
+    int32_t first_token_mode;          /* enum lr_first_token_mode */
+    int32_t max_iters;                 /* bound on simulation steps per instance and load */
+} lr_config;
+
+/* One snapshot of every instance (Sec. 4 "Setup": resident set R_j = Q_j u A_j with
+ * remaining prefill and predicted decode tokens; App. F "Query workload snapshots").
+ * DEVICE pointers.  Per-instance arrays are [I]; per-request arrays are
+ * [I][cap] with row stride cap_running / cap_waiting; entries beyond a row's
+ * count are ignored.
+ * Preconditions, checked on the device (LR_ESTATE): 0 <= n_run[j] <= min(cap_running,
+ * S_j); 0 <= n_wait[j] <= cap_waiting; run_ctx in [0, 2^28]; run_pre in [0, 2^24];
+ * run_dec and wait_dec in [1, 2^24]; wait_pre in [1, 2^24]; only the LAST running
+ * request of a row may have run_pre > 0 (the state a chunked-prefill FCFS engine is in
+ * after any batch). */
+typedef struct {
+    const int32_t *n_run;      /* [I] running requests (admission order) */
+    const int32_t *run_ctx;    /* [I][cap_running] tokens already in the KV cache */
+    const int32_t *run_pre;    /* [I][cap_running] remaining prefill tokens */
+    const int32_t *run_dec;    /* [I][cap_running] remaining predicted decode tokens */
+    const int32_t *n_wait;     /* [I] waiting requests (FCFS order) */
+    const int32_t *wait_pre;   /* [I][cap_waiting] prompt tokens */
+    const int32_t *wait_dec;   /* [I][cap_waiting] predicted decode tokens */
+} lr_state_view;
+
+typedef struct lr_ctx lr_ctx;  /* opaque, owned by the library */
+
+/* Create a context on the current CUDA device.  Copies the configuration and
+ * allocates all device memory the other calls need.  *out is set on LR_OK. */
+LR_API int lr_create(const lr_config *cfg, lr_ctx **out);
+
+/* Free everything lr_create allocated.  Synchronizes the device first.  NULL is a no-op. */
+LR_API int lr_destroy(lr_ctx *ctx);
+
+/* Ingest a snapshot (App. F): copies it into library memory and summarizes, per
+ * instance, the query-independent part of the simulation -- the batch at which a
+ * query appended now would be admitted, the budget left to it in that and the
+ * following batches, and the resident batch features up to each of them.  The
+ * snapshot is written to a back buffer and becomes the live one only if every
+ * instance is valid and simulates within max_iters; otherwise the previous live
+ * snapshot stays in use (App. F: the router keeps its last complete copy) and the
+ * status word records LR_ESTATE or LR_ETRAJ. */
+LR_API int lr_load_state(lr_ctx *ctx, const lr_state_view *state, void *cuda_stream);
+
+/* SFS TTFT estimates (Eq. 8 with Eq. 9) for every candidate of Q queries.
+ * prompt_len: [Q] device, each in [1, max_prompt_len] (else that row is NaN and the
+ * status word records LR_EINVAL).  ttft_out: [Q][I] device fp32 seconds.
+ * first_batch_out: [Q][I] device int32 index of the first-token batch (Eq. 7), or NULL.
+ * Q may be 0. */
+LR_API int lr_estimate_ttft(lr_ctx *ctx, int32_t Q, const int32_t *prompt_len, float *ttft_out,
+                     int32_t *first_batch_out, void *cuda_stream);
+
+/* The integer batch features behind each estimate: features_out [Q][I][5] int64 device,
+ * F = (batches, prefill tokens, decode tokens, sum of decode-token context, sum over
+ * prefill chunks of x*c + x(x+1)/2) summed over batches 1..l_TTFT (Eq. 7-9), so that
+ * TTFT = beta . F.  Rows with an invalid prompt length are -1. */
+LR_API int lr_estimate_features(lr_ctx *ctx, int32_t Q, const int32_t *prompt_len, int64_t *features_out,
+                         void *cuda_stream);
+
+/* Route Q queries for each of P trade-off pairs.
+ *  prompt_len [Q], dec_hat [Q][M] (predicted response tokens, >= 0), acc [Q][M]
+ *  (predicted accuracy, finite): device.
+ *  cost_{i,j} = p_i * price_in_m + dec_hat_{i,m} * price_out_m (App. B.4),
+ *  U = acc - lambda * cost (Eq. 2).
+ *  tau == NULL: Lagrangian objective (Eq. 5), argmax_j U - mu * TTFT.
+ *  tau != NULL ([Q] device, seconds): constrained objective (Eq. 3), argmax U over
+ *  {j : TTFT <= tau_i}, or the least TTFT when that set is empty; mu is then unused
+ *  and may be NULL.  Ties go to the lowest instance index.
+ *  lambda, mu: [P] HOST arrays, finite and >= 0, 1 <= P <= max_pairs.
+ *  Outputs, device: assign_out [P][Q] int32, util_out [P][Q] fp32 U of the chosen
+ *  instance, ttft_chosen_out [P][Q] fp32 or NULL, frontier_out [P][3] fp64 means of
+ *  (accuracy, cost, TTFT) of the chosen instances or NULL, ttft_matrix_out [Q][I] fp32
+ *  (the full estimate matrix, as lr_estimate_ttft writes it) or NULL.
+ *  Requires I <= 1024. */
+LR_API int lr_route(lr_ctx *ctx, int32_t Q, const int32_t *prompt_len, const int32_t *dec_hat, const float *acc,
+             const float *tau, int32_t P, const float *lambda, const float *mu, int32_t *assign_out,
+             float *util_out, float *ttft_chosen_out, double *frontier_out, float *ttft_matrix_out,
+             void *cuda_stream);
+
+/* Synchronize `cuda_stream`, return the first device-side error code recorded since
+ * the last call (LR_OK if none) and clear it. */
+LR_API int lr_status(lr_ctx *ctx, void *cuda_stream);
+
+/* Static description of a return code. */
+LR_API const char *lr_strerror(int code);
+
+/* Text of the last host-side failure on this context (CUDA error string or the
+ * validation that failed); empty if none.  Valid until the next call on ctx. */
+LR_API const char *lr_last_error(const lr_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LATENCY_ROUTER_H */

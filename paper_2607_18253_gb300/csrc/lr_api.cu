@@ -1,0 +1,390 @@
+// Host side of the C ABI declared in include/latency_router.h: validation,
+// device memory, launch shapes and the status word.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "latency_router.h"
+#include "lr_internal.cuh"
+
+struct lr_ctx {
+    int device = 0;
+    int sms = 0;
+    lr::DevConfig cfg{};
+    lr::StateBuf buf[2]{};
+    lr::DevCtl *ctl = nullptr;
+    float *scratch_tch = nullptr;
+    std::vector<void *> allocs;
+    std::string err;
+    int max_queries = 0, max_pairs = 0;
+    // K1
+    size_t k1_smem = 0;
+    // estimate
+    int est_IT = 0, est_QS = 0, est_QT = 0, est_block = 0, est_occ = 0;
+    size_t est_smem = 0;
+    // route
+    bool route_ok = false;
+    int rt_QS = 0, rt_QT = 0, rt_TPR = 0, rt_block = 0, rt_occ = 0;
+    size_t rt_smem = 0;
+};
+
+namespace {
+
+int fail(lr_ctx *c, int code, const std::string &msg) {
+    if (c) c->err = msg;
+    return code;
+}
+
+int cuda_fail(lr_ctx *c, cudaError_t e, const char *what) {
+    if (c) c->err = std::string(what) + ": " + cudaGetErrorString(e);
+    return LR_ECUDA;
+}
+
+template <typename T>
+cudaError_t dev_alloc(lr_ctx *c, T **p, size_t count) {
+    void *v = nullptr;
+    const size_t bytes = count * sizeof(T) > 0 ? count * sizeof(T) : 16;
+    cudaError_t e = cudaMalloc(&v, bytes);
+    if (e != cudaSuccess) return e;
+    c->allocs.push_back(v);
+    e = cudaMemset(v, 0, bytes);
+    *p = static_cast<T *>(v);
+    return e;
+}
+
+int floor_log2(long long x) {
+    int s = 0;
+    while ((2LL << s) <= x) ++s;
+    return s;
+}
+
+int round_up(int x, int m) { return ((x + m - 1) / m) * m; }
+
+int pow2_floor(int x) {
+    int p = 1;
+    while (p * 2 <= x) p *= 2;
+    return p;
+}
+
+bool finite_nonneg(float v) { return std::isfinite(v) && v >= 0.0f; }
+
+void free_all(lr_ctx *c) {
+    for (void *p : c->allocs) cudaFree(p);
+    c->allocs.clear();
+}
+
+// Shared-memory layout of the estimate / route kernels (16-byte objects first).
+size_t est_smem_bytes(const lr::DevConfig &cfg, int IT, int QT) {
+    return (size_t)IT * cfg.kph * 16 + (size_t)QT * 16 + (size_t)IT * cfg.nbh * 8;
+}
+
+size_t route_smem_bytes(const lr::DevConfig &cfg, int QT, int TPR) {
+    const int I = cfg.I;
+    const int ST = round_up(I, 32) + TPR;
+    return est_smem_bytes(cfg, I, QT) + (size_t)QT * cfg.M * 8 + (size_t)QT * ST * 4 + (size_t)QT * 4 +
+           (size_t)I * 4;
+}
+
+lr::K2Launch k2_base(const lr_ctx *c) {
+    lr::K2Launch a;
+    std::memset(&a, 0, sizeof(a));
+    a.cfg = c->cfg;
+    a.buf0 = c->buf[0];
+    a.buf1 = c->buf[1];
+    a.ctl = c->ctl;
+    return a;
+}
+
+}  // namespace
+
+extern "C" {
+
+int lr_create(const lr_config *cfg, lr_ctx **out) {
+    if (!cfg || !out) return LR_EINVAL;
+    *out = nullptr;
+    lr_ctx *c = new (std::nothrow) lr_ctx();
+    if (!c) return LR_ENOMEM;
+    auto bail = [&](int code, const std::string &msg) {
+        std::fprintf(stderr, "lr_create: %s\n", msg.c_str());
+        free_all(c);
+        delete c;
+        return code;
+    };
+    const int I = cfg->num_instances, M = cfg->num_models;
+    if (I < 1 || I > (1 << 16) || M < 1 || M > 1024) return bail(LR_EINVAL, "num_instances or num_models out of range");
+    if (!cfg->model_of_instance || !cfg->coef || !cfg->price_in || !cfg->price_out || !cfg->max_batched_tokens ||
+        !cfg->max_seqs)
+        return bail(LR_EINVAL, "null configuration array");
+    if (cfg->cap_running < 1 || cfg->cap_waiting < 1 || cfg->cap_running > 4096 || cfg->cap_waiting > 4096)
+        return bail(LR_EINVAL, "cap_running / cap_waiting out of range");
+    if (cfg->max_queries < 1 || cfg->max_pairs < 1 || cfg->max_pairs > lr::kMaxPairs)
+        return bail(LR_EINVAL, "max_queries / max_pairs out of range");
+    if (cfg->max_prompt_len < 1 || cfg->max_prompt_len > (1 << 20)) return bail(LR_EINVAL, "max_prompt_len out of range");
+    if (cfg->first_token_mode != LR_FIRST_TOKEN_SEPARATE_DECODE && cfg->first_token_mode != LR_FIRST_TOKEN_WITH_LAST_CHUNK)
+        return bail(LR_EINVAL, "first_token_mode");
+    if (cfg->max_iters < 1) return bail(LR_EINVAL, "max_iters");
+    for (int m = 0; m < M; ++m) {
+        for (int k = 0; k < 5; ++k)
+            if (!finite_nonneg(cfg->coef[m * 5 + k])) return bail(LR_EINVAL, "coefficients must be finite and >= 0");
+        if (!finite_nonneg(cfg->price_in[m]) || !finite_nonneg(cfg->price_out[m]))
+            return bail(LR_EINVAL, "prices must be finite and >= 0");
+    }
+    std::vector<int32_t> shift(I), nb(I);
+    int kph = 1, nbh = 1, smax = 1;
+    for (int j = 0; j < I; ++j) {
+        const int B = cfg->max_batched_tokens[j], S = cfg->max_seqs[j], m = cfg->model_of_instance[j];
+        if (m < 0 || m >= M) return bail(LR_EINVAL, "model_of_instance out of range");
+        if (B < 1 || B > (1 << 24) || S < 1 || S > B) return bail(LR_EINVAL, "need 1 <= max_seqs <= max_batched_tokens <= 2^24");
+        const long long gap = (long long)B - S + 1;  // least budget a query gets after admission
+        shift[j] = floor_log2(gap);
+        nb[j] = (cfg->max_prompt_len >> shift[j]) + 1;
+        const long long kp = (cfg->max_prompt_len - 1 + gap - 1) / gap + 1;
+        if (kp > lr::kKMax || nb[j] > lr::kNBMax)
+            return bail(LR_ECAPACITY, "max_prompt_len too large for max_batched_tokens - max_seqs + 1 of instance " +
+                                          std::to_string(j));
+        kph = std::max(kph, (int)kp);
+        nbh = std::max(nbh, nb[j]);
+        smax = std::max(smax, S);
+    }
+    cudaError_t e = cudaGetDevice(&c->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, c->device);
+    if (e != cudaSuccess) return bail(LR_ECUDA, std::string("cuda device: ") + cudaGetErrorString(e));
+
+    lr::DevConfig &d = c->cfg;
+    d.I = I;
+    d.M = M;
+    d.capR = cfg->cap_running;
+    d.capW = cfg->cap_waiting;
+    d.pmax = cfg->max_prompt_len;
+    d.mode = cfg->first_token_mode;
+    d.max_iters = cfg->max_iters;
+    d.slots = std::max(32, round_up(std::min(smax, cfg->cap_running + cfg->cap_waiting), 32));
+    d.kph = kph;
+    d.nbh = nbh;
+    c->max_queries = cfg->max_queries;
+    c->max_pairs = cfg->max_pairs;
+
+    int32_t *moi, *B, *S, *sh, *nbd;
+    float *coef, *pin, *pout;
+    const size_t R = (size_t)I * d.capR, W = (size_t)I * d.capW;
+#define LR_ALLOC(ptr, n)                                                            \
+    do {                                                                            \
+        cudaError_t ee = dev_alloc(c, &(ptr), (n));                                 \
+        if (ee != cudaSuccess) return bail(LR_ENOMEM, cudaGetErrorString(ee));      \
+    } while (0)
+    LR_ALLOC(moi, I);
+    LR_ALLOC(B, I);
+    LR_ALLOC(S, I);
+    LR_ALLOC(sh, I);
+    LR_ALLOC(nbd, I);
+    LR_ALLOC(coef, (size_t)M * 5);
+    LR_ALLOC(pin, M);
+    LR_ALLOC(pout, M);
+    for (int b = 0; b < 2; ++b) {
+        lr::StateBuf &s = c->buf[b];
+        LR_ALLOC(s.n_run, I);
+        LR_ALLOC(s.run_ctx, R);
+        LR_ALLOC(s.run_pre, R);
+        LR_ALLOC(s.run_dec, R);
+        LR_ALLOC(s.n_wait, I);
+        LR_ALLOC(s.wait_pre, W);
+        LR_ALLOC(s.wait_dec, W);
+        LR_ALLOC(s.inst, I);
+        LR_ALLOC(s.bkt, (size_t)nbh * I);
+        LR_ALLOC(s.ent, (size_t)kph * I);
+        LR_ALLOC(s.f2, (size_t)kph * I);
+        LR_ALLOC(s.f3, (size_t)kph * I);
+        LR_ALLOC(s.rcum, (size_t)kph * I);
+    }
+    LR_ALLOC(c->ctl, 1);
+    LR_ALLOC(c->scratch_tch, (size_t)cfg->max_pairs * cfg->max_queries);
+#undef LR_ALLOC
+    e = cudaMemcpy(moi, cfg->model_of_instance, I * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(B, cfg->max_batched_tokens, I * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(S, cfg->max_seqs, I * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(sh, shift.data(), I * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(nbd, nb.data(), I * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(coef, cfg->coef, (size_t)M * 20, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(pin, cfg->price_in, M * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(pout, cfg->price_out, M * 4, cudaMemcpyHostToDevice);
+    lr::DevCtl ctl0{-1, 0, 0, 0u};
+    if (e == cudaSuccess) e = cudaMemcpy(c->ctl, &ctl0, sizeof(ctl0), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return bail(LR_ECUDA, cudaGetErrorString(e));
+    d.moi = moi;
+    d.B = B;
+    d.S = S;
+    d.shift = sh;
+    d.nb = nbd;
+    d.coef = coef;
+    d.pin = pin;
+    d.pout = pout;
+
+    // K1: one warp per instance.
+    c->k1_smem = lr::kK1Warps * lr::trajectory_smem_per_warp(d);
+    if (c->k1_smem > 200 * 1024) return bail(LR_ECAPACITY, "snapshot capacities too large for one K1 warp");
+    // Estimate: threads own instances of a tile, QS query rows in flight.
+    c->est_IT = I <= 256 ? I : 256;
+    c->est_QS = I <= 256 ? 256 / I : 1;
+    c->est_block = round_up(c->est_IT * c->est_QS, 32);
+    c->est_QT = std::max(c->est_QS, (std::min(c->est_block, 128) / c->est_QS) * c->est_QS);
+    c->est_smem = est_smem_bytes(d, c->est_IT, c->est_QT);
+    if (c->est_smem > 200 * 1024) return bail(LR_ECAPACITY, "summary tables too large for shared memory");
+    // Route: one CTA holds every instance of a row.
+    if (I <= 1024) {
+        c->rt_QS = I <= 256 ? 256 / I : 1;
+        c->rt_block = round_up(I * c->rt_QS, 32);
+        const int want = std::min(256, std::max(1, 8192 / (I + 1)));
+        c->rt_QT = std::max(c->rt_QS, (want / c->rt_QS) * c->rt_QS);
+        c->rt_QT = std::min(c->rt_QT, c->rt_block);
+        c->rt_TPR = std::min(32, std::max(1, pow2_floor(c->rt_block / c->rt_QT)));
+        c->rt_smem = route_smem_bytes(d, c->rt_QT, c->rt_TPR);
+        c->route_ok = c->rt_smem <= 200 * 1024;
+    }
+    e = lr::set_k1_smem(c->k1_smem);
+    if (e == cudaSuccess) e = lr::set_k2_smem(c->est_smem, c->route_ok ? c->rt_smem : c->est_smem);
+    if (e == cudaSuccess) e = lr::estimate_occupancy(0, d.mode, c->est_block, c->est_smem, &c->est_occ);
+    if (e == cudaSuccess && c->route_ok) e = lr::route_occupancy(d.mode, c->rt_block, c->rt_smem, &c->rt_occ);
+    if (e != cudaSuccess) return bail(LR_ECUDA, cudaGetErrorString(e));
+    c->est_occ = std::max(1, c->est_occ);
+    c->rt_occ = std::max(1, c->rt_occ);
+    *out = c;
+    return LR_OK;
+}
+
+int lr_destroy(lr_ctx *c) {
+    if (!c) return LR_OK;
+    cudaDeviceSynchronize();
+    free_all(c);
+    delete c;
+    return LR_OK;
+}
+
+int lr_load_state(lr_ctx *c, const lr_state_view *v, void *stream) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    if (!v || !v->n_run || !v->run_ctx || !v->run_pre || !v->run_dec || !v->n_wait || !v->wait_pre || !v->wait_dec)
+        return fail(c, LR_EINVAL, "null snapshot array");
+    lr::K1Launch a;
+    std::memset(&a, 0, sizeof(a));
+    a.cfg = c->cfg;
+    a.buf0 = c->buf[0];
+    a.buf1 = c->buf[1];
+    a.ctl = c->ctl;
+    a.in = lr::StateIn{v->n_run, v->run_ctx, v->run_pre, v->run_dec, v->n_wait, v->wait_pre, v->wait_dec};
+    const int grid = (c->cfg.I + lr::kK1Warps - 1) / lr::kK1Warps;
+    cudaError_t e = lr::launch_trajectory(a, grid, lr::kK1Warps * 32, c->k1_smem, (cudaStream_t)stream);
+    return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "trajectory launch");
+}
+
+static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, int32_t *iters, int64_t *feat,
+                           void *stream) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    if (Q < 0) return fail(c, LR_EINVAL, "Q < 0");
+    if (Q > c->max_queries) return fail(c, LR_ECAPACITY, "Q exceeds max_queries");
+    if (Q == 0) return LR_OK;
+    if (!p || (!ttft && !feat)) return fail(c, LR_EINVAL, "null array");
+    lr::K2Launch a = k2_base(c);
+    a.Q = Q;
+    a.prompt = p;
+    a.ttft = ttft;
+    a.first_batch = iters;
+    a.features = reinterpret_cast<long long *>(feat);
+    a.IT = c->est_IT;
+    a.QS = c->est_QS;
+    a.QT = c->est_QT;
+    dim3 grid(std::min(c->sms * c->est_occ, Q), (c->cfg.I + c->est_IT - 1) / c->est_IT);
+    cudaError_t e = lr::launch_estimate(a, feat ? lr::kEstFeatures : lr::kEstTtft, grid, c->est_block, c->est_smem,
+                                        (cudaStream_t)stream);
+    return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "estimate launch");
+}
+
+int lr_estimate_ttft(lr_ctx *c, int32_t Q, const int32_t *prompt_len, float *ttft_out, int32_t *first_batch_out,
+                     void *stream) {
+    if (c && Q > 0 && !ttft_out) return fail(c, LR_EINVAL, "null ttft_out");
+    return estimate_common(c, Q, prompt_len, ttft_out, first_batch_out, nullptr, stream);
+}
+
+int lr_estimate_features(lr_ctx *c, int32_t Q, const int32_t *prompt_len, int64_t *features_out, void *stream) {
+    if (c && Q > 0 && !features_out) return fail(c, LR_EINVAL, "null features_out");
+    return estimate_common(c, Q, prompt_len, nullptr, nullptr, features_out, stream);
+}
+
+int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec_hat, const float *acc, const float *tau,
+             int32_t P, const float *lambda, const float *mu, int32_t *assign_out, float *util_out,
+             float *ttft_chosen_out, double *frontier_out, float *ttft_matrix_out, void *stream) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    if (Q < 0) return fail(c, LR_EINVAL, "Q < 0");
+    if (Q > c->max_queries) return fail(c, LR_ECAPACITY, "Q exceeds max_queries");
+    if (P < 1) return fail(c, LR_EINVAL, "P < 1");
+    if (P > c->max_pairs) return fail(c, LR_ECAPACITY, "P exceeds max_pairs");
+    if (!c->route_ok) return fail(c, LR_ECAPACITY, "routing needs num_instances <= 1024 and its tiles in shared memory");
+    if (!lambda || (!tau && !mu)) return fail(c, LR_EINVAL, "null lambda / mu");
+    for (int k = 0; k < P; ++k) {
+        if (!finite_nonneg(lambda[k])) return fail(c, LR_EINVAL, "lambda must be finite and >= 0");
+        if (!tau && !finite_nonneg(mu[k])) return fail(c, LR_EINVAL, "mu must be finite and >= 0");
+    }
+    if (Q == 0) return LR_OK;
+    if (!prompt_len || !dec_hat || !acc || !assign_out || !util_out) return fail(c, LR_EINVAL, "null array");
+    lr::K2Launch a = k2_base(c);
+    a.Q = Q;
+    a.prompt = prompt_len;
+    a.dec_hat = dec_hat;
+    a.acc = acc;
+    a.tau = tau;
+    a.P = P;
+    for (int k = 0; k < P; ++k) {
+        a.lam[k] = lambda[k];
+        a.mu[k] = tau ? 0.0f : mu[k];
+    }
+    a.assign = assign_out;
+    a.util = util_out;
+    a.ttft_chosen = ttft_chosen_out ? ttft_chosen_out : (frontier_out ? c->scratch_tch : nullptr);
+    a.ttft = ttft_matrix_out;
+    a.IT = c->cfg.I;
+    a.QS = c->rt_QS;
+    a.QT = c->rt_QT;
+    a.TPR = c->rt_TPR;
+    dim3 grid(std::min(c->sms * c->rt_occ, Q), 1);
+    cudaError_t e = lr::launch_route(a, grid, c->rt_block, c->rt_smem, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "route launch");
+    if (frontier_out) {
+        e = lr::launch_frontier(a, frontier_out, (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(c, e, "frontier launch");
+    }
+    return LR_OK;
+}
+
+int lr_status(lr_ctx *c, void *stream) {
+    if (!c) return LR_EINVAL;
+    int32_t h = 0;
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e = cudaMemcpyAsync(&h, &c->ctl->status, sizeof(int32_t), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(&c->ctl->status, 0, sizeof(int32_t), st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "status");
+    return h;
+}
+
+const char *lr_strerror(int code) {
+    switch (code) {
+        case LR_OK: return "ok";
+        case LR_EINVAL: return "invalid argument or input value";
+        case LR_ENOMEM: return "out of memory";
+        case LR_ECUDA: return "CUDA runtime error";
+        case LR_ECAPACITY: return "size exceeds the context's capacity";
+        case LR_ETRAJ: return "simulated trajectory exceeded max_iters";
+        case LR_ESTATE: return "snapshot violates the state preconditions";
+        case LR_ENOSTATE: return "no snapshot loaded";
+        default: return "unknown error";
+    }
+}
+
+const char *lr_last_error(const lr_ctx *c) { return c ? c->err.c_str() : ""; }
+
+}  // extern "C"

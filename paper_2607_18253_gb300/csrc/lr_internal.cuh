@@ -1,0 +1,138 @@
+// Library-internal layout shared by the host API and the kernels.
+//
+// Data layout in HBM (all per-instance tables are [row][I], instance-minor, so
+// that consecutive threads of a CTA -- which own consecutive instances -- read
+// consecutive words):
+//
+//   config      : model_of_instance[I], B[I], S[I], shift[I], nb[I], coef[M][5],
+//                 price_in[M], price_out[M]
+//   buffer 0/1  : a snapshot copy (SoA, row stride cap) plus its summary:
+//                 inst[I]           InstParams (admission batch, totals, splits)
+//                 bkt[NBH][I]       int2 (in-bucket boundary, boundaries below)
+//                 ent[KPH][I]       float4 (T_k, H3_k, L3_k, f3_k)
+//                 f2[KPH][I], f3[KPH][I], rcum[KPH][I]
+//   control     : live buffer index, sticky status word, load error, CTA counter
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace lr {
+
+constexpr int kKMax = 64;               // table entries per instance (k = 0..kp-1)
+constexpr int kNBMax = 2 * kKMax + 2;   // prompt-length buckets per instance
+constexpr int kBig = 0x7fffffff;        // "never" / "no boundary"
+constexpr int kSplitBits = 20;          // low part of the exact fp32 splits
+constexpr long long kFastLimit = 1LL << 44;  // integers below this split exactly
+constexpr int kMaxPairs = 64;
+
+// Return codes (mirror include/latency_router.h).
+enum : int { kOk = 0, kEInval = 1, kENoMem = 2, kECuda = 3, kECapacity = 4, kETraj = 5, kEState = 6,
+             kENoState = 7 };
+
+struct InstParams {      // 64 bytes
+    int32_t la;          // batch at which a query appended now is admitted
+    int32_t kp;          // number of table entries
+    int32_t shift;       // log2 of the bucket width
+    int32_t fast;        // 1: every feature of this instance splits exactly into fp32
+    long long f1tot;     // prefill tokens of all residents
+    long long f4tot;     // prefill attention pairs of all residents
+    float h1, l1, h4, l4;  // exact fp32 high/low parts of f1tot and f4tot
+    int32_t r0;          // budget left to the query in its admission batch
+    int32_t pad[3];
+};
+
+struct DevConfig {
+    int32_t I, M, capR, capW;
+    int32_t pmax, mode, max_iters, slots;  // slots: decoder slots per instance in K1
+    int32_t kph, nbh;                       // table row counts (host bounds over instances)
+    const int32_t *moi, *B, *S, *shift, *nb;
+    const float *coef, *pin, *pout;
+};
+
+struct StateBuf {
+    int32_t *n_run, *run_ctx, *run_pre, *run_dec, *n_wait, *wait_pre, *wait_dec;
+    InstParams *inst;
+    int2 *bkt;
+    float4 *ent;
+    long long *f2, *f3;
+    int32_t *rcum;
+};
+
+struct DevCtl {
+    int32_t active;      // live buffer, -1 before the first successful load
+    int32_t status;      // first error since the last lr_status
+    int32_t load_err;    // error of the load in progress
+    uint32_t done_ctas;  // K1 completion counter
+};
+
+struct StateIn {
+    const int32_t *n_run, *run_ctx, *run_pre, *run_dec, *n_wait, *wait_pre, *wait_dec;
+};
+
+__device__ __forceinline__ void record_status(DevCtl *ctl, int code) {
+    atomicCAS(&ctl->status, 0, code);
+}
+
+__device__ __forceinline__ unsigned lanemask_lt() {
+    unsigned m;
+    asm volatile("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+    return m;
+}
+
+__device__ __forceinline__ long long warp_sum64(long long v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Launch helpers implemented in the kernel translation units.
+struct K1Launch {
+    DevConfig cfg;
+    StateBuf buf0, buf1;
+    DevCtl *ctl;
+    StateIn in;
+};
+cudaError_t launch_trajectory(const K1Launch &a, int grid, int block, size_t smem, cudaStream_t st);
+cudaError_t set_k1_smem(size_t bytes);
+constexpr int kK1Warps = 4;
+
+// Shared memory of one K1 warp: decoder slots (s, f, cb, free list), the
+// waiting queue and the cumulative budgets.
+__host__ __device__ inline size_t trajectory_smem_per_warp(const DevConfig &c) {
+    return sizeof(int32_t) * (4 * (size_t)c.slots + 2 * (size_t)c.capW + (size_t)c.kph);
+}
+
+struct K2Launch {
+    DevConfig cfg;
+    StateBuf buf0, buf1;
+    DevCtl *ctl;
+    int32_t Q;
+    const int32_t *prompt;
+    // estimate outputs
+    float *ttft;
+    int32_t *first_batch;
+    long long *features;
+    // route inputs / outputs
+    const int32_t *dec_hat;
+    const float *acc;
+    const float *tau;
+    int32_t P;
+    float lam[kMaxPairs];
+    float mu[kMaxPairs];
+    int32_t *assign;
+    float *util;
+    float *ttft_chosen;
+    // launch shape
+    int32_t IT, QS, QT, TPR;
+};
+cudaError_t launch_estimate(const K2Launch &a, int kind, dim3 grid, int block, size_t smem, cudaStream_t st);
+cudaError_t launch_route(const K2Launch &a, dim3 grid, int block, size_t smem, cudaStream_t st);
+cudaError_t launch_frontier(const K2Launch &a, double *out, cudaStream_t st);
+cudaError_t estimate_occupancy(int kind, int mode, int block, size_t smem, int *blocks_per_sm);
+cudaError_t route_occupancy(int mode, int block, size_t smem, int *blocks_per_sm);
+cudaError_t set_k2_smem(size_t estimate_bytes, size_t route_bytes);
+
+enum : int { kEstTtft = 0, kEstFeatures = 1 };
+
+}  // namespace lr

@@ -134,8 +134,9 @@ def coefficients(alpha_ms, beta_ms, gamma_ms) -> np.ndarray:
 def ttft_targets(rng: np.random.Generator, prompt_len: np.ndarray) -> np.ndarray:
     """TTFT targets of App. B.2: clip(u + (155 + 3.5e-3 p) v, 150, 1120) ms, in seconds."""
     n = prompt_len.shape[0]
-    u = rng.uniform(1.0, 5.0, n)
-    v = rng.uniform(0.98, 1.02, n)
+    uv = rng.uniform(0.0, 1.0, (n, 2))  # row-wise draws keep a prefix of queries unchanged
+    u = 1.0 + 4.0 * uv[:, 0]
+    v = 0.98 + 0.04 * uv[:, 1]
     t_ms = np.minimum(1120.0, np.maximum(150.0, u + (155.0 + 3.5e-3 * prompt_len.astype(np.float64)) * v))
     return (t_ms * 1e-3).astype(np.float32)
 
@@ -226,16 +227,16 @@ def sweep_pairs():
 
 def random_small_state(rng: np.random.Generator, num_instances: int, cap_running: int, cap_waiting: int,
                        budget_range=(4, 64), with_tail_prefill: bool = True,
-                       max_ctx: int = 300, max_pre: int = 200, max_dec: int = 40):
+                       max_ctx: int = 300, max_pre: int = 200, max_dec: int = 40, min_gap: int = 1):
     """Small random pools for property tests.
 
-    Returns per-instance budget B, cap S (1 <= S <= B), and a state whose
-    running list holds at most one request with remaining prefill, placed
-    last, and never more requests than S.
+    Returns per-instance budget B, cap S (1 <= S <= B - min_gap + 1), and a
+    state whose running list holds at most one request with remaining
+    prefill, placed last, and never more requests than S.
     """
     I = num_instances
-    B = rng.integers(budget_range[0], budget_range[1] + 1, I).astype(np.int32)
-    S = np.array([rng.integers(1, b + 1) for b in B], np.int32)
+    B = rng.integers(max(budget_range[0], min_gap), budget_range[1] + 1, I).astype(np.int32)
+    S = np.array([rng.integers(1, b - min_gap + 2) for b in B], np.int32)
     S = np.minimum(S, cap_running).astype(np.int32)
     n_run = np.array([rng.integers(0, s + 1) for s in S], np.int32)
     n_wait = rng.integers(0, cap_waiting + 1, I).astype(np.int32)
@@ -259,12 +260,12 @@ def random_small_state(rng: np.random.Generator, num_instances: int, cap_running
 def small_workload(seed: int, num_instances: int = 6, num_models: int = 3, num_queries: int = 24,
                    cap_running: int = 8, cap_waiting: int = 8, max_prompt_len: int = 160,
                    first_token_mode: int = FIRST_TOKEN_SEPARATE_DECODE, budget_range=(4, 64),
-                   with_tail_prefill: bool = True) -> Workload:
+                   with_tail_prefill: bool = True, min_gap: int = 1) -> Workload:
     """A random small pool (for property and parity tests on tiny inputs)."""
     rng = np.random.default_rng(seed)
     B, S, n_run, run_ctx, run_pre, run_dec, n_wait, wait_pre, wait_dec = random_small_state(
         rng, num_instances, cap_running, cap_waiting, budget_range=budget_range,
-        with_tail_prefill=with_tail_prefill)
+        with_tail_prefill=with_tail_prefill, min_gap=min_gap)
     alpha = rng.uniform(1.0, 10.0, num_models)
     beta = rng.uniform(0.01, 0.2, num_models)
     gamma = beta + rng.uniform(0.05, 0.5, num_models)
