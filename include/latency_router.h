@@ -91,9 +91,9 @@ typedef struct {
  * count are ignored.
  * Preconditions, checked on the device (LR_ESTATE): 0 <= n_run[j] <= min(cap_running,
  * S_j); 0 <= n_wait[j] <= cap_waiting; run_ctx in [0, 2^28]; run_pre in [0, 2^24];
- * run_dec and wait_dec in [1, 2^24]; wait_pre in [1, 2^24]; only the LAST running
- * request of a row may have run_pre > 0 (the state a chunked-prefill FCFS engine is in
- * after any batch). */
+ * run_dec and wait_dec in [1, 2^24]; wait_pre in [1, 2^24] and at most 2^30 in total per
+ * instance; only the LAST running request of a row may have run_pre > 0 (the state a
+ * chunked-prefill FCFS engine is in after any batch). */
 typedef struct {
     const int32_t *n_run;      /* [I] running requests (admission order) */
     const int32_t *run_ctx;    /* [I][cap_running] tokens already in the KV cache */

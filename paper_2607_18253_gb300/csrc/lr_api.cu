@@ -1,6 +1,7 @@
 // Host side of the C ABI declared in include/latency_router.h: validation,
 // device memory, launch shapes and the status word.
 #include <cmath>
+#include <cstdint>
 #include <cstdio>
 #include <cstring>
 #include <new>
@@ -22,13 +23,13 @@ struct lr_ctx {
     int max_queries = 0, max_pairs = 0;
     // K1
     size_t k1_smem = 0;
-    // estimate
-    int est_IT = 0, est_QS = 0, est_QT = 0, est_block = 0, est_occ = 0;
-    size_t est_smem = 0;
-    // route
-    bool route_ok = false;
-    int rt_QS = 0, rt_QT = 0, rt_TPR = 0, rt_block = 0, rt_occ = 0;
-    size_t rt_smem = 0;
+    // candidate kernel shapes: estimate (instances may span several tiles) and
+    // route (all instances of a row in one CTA)
+    struct Shape {
+        int Gp = 0, QS = 0, QT = 0, tiles = 1, occ = 1;
+        size_t smem = 0;
+        bool ok = false;
+    } est, rt;
 };
 
 namespace {
@@ -63,12 +64,6 @@ int floor_log2(long long x) {
 
 int round_up(int x, int m) { return ((x + m - 1) / m) * m; }
 
-int pow2_floor(int x) {
-    int p = 1;
-    while (p * 2 <= x) p *= 2;
-    return p;
-}
-
 bool finite_nonneg(float v) { return std::isfinite(v) && v >= 0.0f; }
 
 void free_all(lr_ctx *c) {
@@ -76,16 +71,38 @@ void free_all(lr_ctx *c) {
     c->allocs.clear();
 }
 
-// Shared-memory layout of the estimate / route kernels (16-byte objects first).
-size_t est_smem_bytes(const lr::DevConfig &cfg, int IT, int QT) {
-    return (size_t)IT * cfg.kph * 16 + (size_t)QT * 16 + (size_t)IT * cfg.nbh * 8;
+int pow2_ceil(int x) {
+    int p = 1;
+    while (p < x) p *= 2;
+    return p;
 }
 
-size_t route_smem_bytes(const lr::DevConfig &cfg, int QT, int TPR) {
-    const int I = cfg.I;
-    const int ST = round_up(I, 32) + TPR;
-    return est_smem_bytes(cfg, I, QT) + (size_t)QT * cfg.M * 8 + (size_t)QT * ST * 4 + (size_t)QT * 4 +
-           (size_t)I * 4;
+// Launch shape of the candidate kernel: threads own four consecutive instances;
+// Gp groups per row (power of two up to 32, else a multiple of 32); the
+// summary tables of the tile and QT staged query rows fit the shared-memory
+// target so that four CTAs share an SM.
+lr_ctx::Shape make_shape(const lr::DevConfig &d, bool route, int max_pairs) {
+    lr_ctx::Shape s;
+    const int G = (d.I + 3) / 4;
+    s.Gp = G <= 32 ? pow2_ceil(G) : round_up(G, 32);
+    if (s.Gp > lr::kK2Block) {
+        if (route) return s;
+        s.Gp = lr::kK2Block;
+    }
+    s.tiles = (d.I + 4 * s.Gp - 1) / (4 * s.Gp);
+    s.QS = lr::kK2Block / s.Gp;
+    const int wpr = s.Gp > 32 ? s.Gp / 32 : 1;
+    const size_t tables = (size_t)d.kph * 4 * s.Gp * 16 + (size_t)d.nbh * 4 * s.Gp * 8;
+    const size_t part = s.Gp > 32 ? 2 * (size_t)wpr * 16 * max_pairs : 0;  // wide-row partials per pair
+    const size_t per_row = 16 + (route ? part + (size_t)d.M * 8 + 4 : 0);
+    const size_t room = lr::kK2SmemTarget > tables ? lr::kK2SmemTarget - tables : 0;
+    int qt = (int)std::min<size_t>(256, room / per_row);
+    if (route && (size_t)qt * per_row + tables > 200 * 1024) qt = 0;
+    qt = std::max(s.QS, (qt / s.QS) * s.QS);
+    s.QT = qt;
+    s.smem = tables + (size_t)qt * per_row;
+    s.ok = s.smem <= 200 * 1024;
+    return s;
 }
 
 lr::K2Launch k2_base(const lr_ctx *c) {
@@ -133,7 +150,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
             return bail(LR_EINVAL, "prices must be finite and >= 0");
     }
     std::vector<int32_t> shift(I), nb(I);
-    int kph = 1, nbh = 1, smax = 1;
+    int kph = 1, nbh = 1;
     for (int j = 0; j < I; ++j) {
         const int B = cfg->max_batched_tokens[j], S = cfg->max_seqs[j], m = cfg->model_of_instance[j];
         if (m < 0 || m >= M) return bail(LR_EINVAL, "model_of_instance out of range");
@@ -147,7 +164,6 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
                                           std::to_string(j));
         kph = std::max(kph, (int)kp);
         nbh = std::max(nbh, nb[j]);
-        smax = std::max(smax, S);
     }
     cudaError_t e = cudaGetDevice(&c->device);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, c->device);
@@ -161,7 +177,6 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     d.pmax = cfg->max_prompt_len;
     d.mode = cfg->first_token_mode;
     d.max_iters = cfg->max_iters;
-    d.slots = std::max(32, round_up(std::min(smax, cfg->cap_running + cfg->cap_waiting), 32));
     d.kph = kph;
     d.nbh = nbh;
     c->max_queries = cfg->max_queries;
@@ -225,31 +240,16 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     // K1: one warp per instance.
     c->k1_smem = lr::kK1Warps * lr::trajectory_smem_per_warp(d);
     if (c->k1_smem > 200 * 1024) return bail(LR_ECAPACITY, "snapshot capacities too large for one K1 warp");
-    // Estimate: threads own instances of a tile, QS query rows in flight.
-    c->est_IT = I <= 256 ? I : 256;
-    c->est_QS = I <= 256 ? 256 / I : 1;
-    c->est_block = round_up(c->est_IT * c->est_QS, 32);
-    c->est_QT = std::max(c->est_QS, (std::min(c->est_block, 128) / c->est_QS) * c->est_QS);
-    c->est_smem = est_smem_bytes(d, c->est_IT, c->est_QT);
-    if (c->est_smem > 200 * 1024) return bail(LR_ECAPACITY, "summary tables too large for shared memory");
-    // Route: one CTA holds every instance of a row.
-    if (I <= 1024) {
-        c->rt_QS = I <= 256 ? 256 / I : 1;
-        c->rt_block = round_up(I * c->rt_QS, 32);
-        const int want = std::min(256, std::max(1, 8192 / (I + 1)));
-        c->rt_QT = std::max(c->rt_QS, (want / c->rt_QS) * c->rt_QS);
-        c->rt_QT = std::min(c->rt_QT, c->rt_block);
-        c->rt_TPR = std::min(32, std::max(1, pow2_floor(c->rt_block / c->rt_QT)));
-        c->rt_smem = route_smem_bytes(d, c->rt_QT, c->rt_TPR);
-        c->route_ok = c->rt_smem <= 200 * 1024;
-    }
+    c->est = make_shape(d, false, 1);
+    c->rt = make_shape(d, true, cfg->max_pairs);
+    if (!c->est.ok) return bail(LR_ECAPACITY, "summary tables too large for shared memory");
     e = lr::set_k1_smem(c->k1_smem);
-    if (e == cudaSuccess) e = lr::set_k2_smem(c->est_smem, c->route_ok ? c->rt_smem : c->est_smem);
-    if (e == cudaSuccess) e = lr::estimate_occupancy(0, d.mode, c->est_block, c->est_smem, &c->est_occ);
-    if (e == cudaSuccess && c->route_ok) e = lr::route_occupancy(d.mode, c->rt_block, c->rt_smem, &c->rt_occ);
+    if (e == cudaSuccess) e = lr::set_k2_smem(std::max(c->est.smem, c->rt.ok ? c->rt.smem : 0));
+    if (e == cudaSuccess) e = lr::cand_occupancy(d.mode, false, lr::kK2Block, c->est.smem, &c->est.occ);
+    if (e == cudaSuccess && c->rt.ok) e = lr::cand_occupancy(d.mode, true, lr::kK2Block, c->rt.smem, &c->rt.occ);
     if (e != cudaSuccess) return bail(LR_ECUDA, cudaGetErrorString(e));
-    c->est_occ = std::max(1, c->est_occ);
-    c->rt_occ = std::max(1, c->rt_occ);
+    c->est.occ = std::max(1, c->est.occ);
+    c->rt.occ = std::max(1, c->rt.occ);
     *out = c;
     return LR_OK;
 }
@@ -290,15 +290,21 @@ static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, 
     lr::K2Launch a = k2_base(c);
     a.Q = Q;
     a.prompt = p;
+    cudaError_t e;
+    if (feat) {
+        a.features = reinterpret_cast<long long *>(feat);
+        e = lr::launch_features(a, c->sms, (cudaStream_t)stream);
+        return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "features launch");
+    }
     a.ttft = ttft;
     a.first_batch = iters;
-    a.features = reinterpret_cast<long long *>(feat);
-    a.IT = c->est_IT;
-    a.QS = c->est_QS;
-    a.QT = c->est_QT;
-    dim3 grid(std::min(c->sms * c->est_occ, Q), (c->cfg.I + c->est_IT - 1) / c->est_IT);
-    cudaError_t e = lr::launch_estimate(a, feat ? lr::kEstFeatures : lr::kEstTtft, grid, c->est_block, c->est_smem,
-                                        (cudaStream_t)stream);
+    a.Gp = c->est.Gp;
+    a.QS = c->est.QS;
+    a.QT = c->est.QT;
+    a.vec_ok = (c->cfg.I % 4 == 0) && ((uintptr_t)ttft % 16 == 0);
+    dim3 grid(std::min(c->sms * c->est.occ, (Q + a.QS - 1) / a.QS), c->est.tiles);
+    e = lr::launch_cand(a, lr::cand_out_flags(true, iters != nullptr, false, false, 1), grid, lr::kK2Block,
+                        c->est.smem, (cudaStream_t)stream);
     return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "estimate launch");
 }
 
@@ -322,7 +328,7 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
     if (Q > c->max_queries) return fail(c, LR_ECAPACITY, "Q exceeds max_queries");
     if (P < 1) return fail(c, LR_EINVAL, "P < 1");
     if (P > c->max_pairs) return fail(c, LR_ECAPACITY, "P exceeds max_pairs");
-    if (!c->route_ok) return fail(c, LR_ECAPACITY, "routing needs num_instances <= 1024 and its tiles in shared memory");
+    if (!c->rt.ok) return fail(c, LR_ECAPACITY, "routing needs num_instances <= 1024 and its tiles in shared memory");
     if (!lambda || (!tau && !mu)) return fail(c, LR_EINVAL, "null lambda / mu");
     for (int k = 0; k < P; ++k) {
         if (!finite_nonneg(lambda[k])) return fail(c, LR_EINVAL, "lambda must be finite and >= 0");
@@ -345,12 +351,13 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
     a.util = util_out;
     a.ttft_chosen = ttft_chosen_out ? ttft_chosen_out : (frontier_out ? c->scratch_tch : nullptr);
     a.ttft = ttft_matrix_out;
-    a.IT = c->cfg.I;
-    a.QS = c->rt_QS;
-    a.QT = c->rt_QT;
-    a.TPR = c->rt_TPR;
-    dim3 grid(std::min(c->sms * c->rt_occ, Q), 1);
-    cudaError_t e = lr::launch_route(a, grid, c->rt_block, c->rt_smem, (cudaStream_t)stream);
+    a.Gp = c->rt.Gp;
+    a.QS = c->rt.QS;
+    a.QT = c->rt.QT;
+    a.vec_ok = (c->cfg.I % 4 == 0) && ((uintptr_t)ttft_matrix_out % 16 == 0);
+    dim3 grid(std::min(c->sms * c->rt.occ, (Q + a.QS - 1) / a.QS), 1);
+    cudaError_t e = lr::launch_cand(a, lr::cand_out_flags(ttft_matrix_out != nullptr, false, true, tau != nullptr, P),
+                                    grid, lr::kK2Block, c->rt.smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(c, e, "route launch");
     if (frontier_out) {
         e = lr::launch_frontier(a, frontier_out, (cudaStream_t)stream);

@@ -1,9 +1,9 @@
 // K2: per-candidate SFS TTFT (Sec. 4.1, Eq. 7-9), utility (Eq. 2) and the
 // per-query argmax (Eq. 3, Eq. 5).
 //
-// Each thread owns one instance j of its CTA's instance tile and walks the
-// CTA's query rows; the instance's summary (written by K1) sits in shared
-// memory, its scalars in registers.  For a query of prompt p:
+// Each thread owns four consecutive instances of its CTA's instance tile and
+// walks the CTA's query rows; the instances' summaries (written by K1) sit in
+// shared memory, their scalars in registers.  For a query of prompt p:
 //
 //   k* = #{k : R_k < p}          cumulative budget after the admission batch;
 //                                found with one bucket lookup (bucket width
@@ -18,10 +18,12 @@
 // X + y with X = H + L (H a multiple of 2^20 below 2^44, L < 2^20) rounds as
 // fadd(H, fadd(L, y)) because the inner sum is an exact integer below 2^24
 // and the outer add rounds the exact total once.  This keeps the hot loop on
-// the FMA pipe; instances whose totals reach 2^44 take the int64 path.
+// the FMA pipe; instances whose totals reach 2^44 take an int64 path.
 //
-// The estimate matrix is write-only (4 bytes per candidate) and streamed out
-// with evict-first stores; this kernel is bound by HBM bandwidth.
+// The estimate matrix is write-only (4 bytes per candidate) and leaves as one
+// 16-byte evict-first store per thread and row.  Routing reduces each row with
+// redux.sync over order-preserving integer keys of the objective: the lowest
+// lane (lowest instance) among the maximal keys wins, as in a first-max scan.
 #include <math.h>
 
 #include "lr_internal.cuh"
@@ -32,18 +34,13 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr long long kLowMask = (1LL << kSplitBits) - 1;
+constexpr float kNaN = __builtin_nanf("");
 
 struct __align__(16) QRec {
     int p;     // prompt length, clamped into [1, pmax] for table lookups
     float fp;  // p as fp32, NaN if p was out of range
     float ph;  // p(p+1)/2 high part (multiple of 2^20)
     float pl;  // p(p+1)/2 low part
-};
-
-struct InstRegs {
-    int jl, la, shift;
-    float h1, l1, h4, l4, b1p, b2, b3;
-    long long f1tot, f4tot;
 };
 
 __device__ __forceinline__ QRec make_qrec(int p, int pmax, bool *ok) {
@@ -53,172 +50,170 @@ __device__ __forceinline__ QRec make_qrec(int p, int pmax, bool *ok) {
     const long long pp = ((long long)p * (p + 1)) / 2;
     const long long pl = pp & kLowMask;
     q.p = p;
-    q.fp = *ok ? (float)p : __int_as_float(0x7fc00000);
+    q.fp = *ok ? (float)p : kNaN;
     q.ph = __ll2float_rn(pp - pl);
     q.pl = __ll2float_rn(pl);
     return q;
 }
 
-__device__ __forceinline__ InstRegs load_inst(const DevConfig &c, const StateBuf &sb, int j, int jl) {
-    InstRegs r;
+// Order-preserving key of a float (no NaN): larger float <-> larger key, and
+// -0 and +0 share a key.  Zero is below every key.
+__device__ __forceinline__ unsigned order_key(float x) {
+    const unsigned u = __float_as_uint(__fadd_rn(x, 0.0f));
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// ---------------------------------------------------------------------------
+// Integer features (exact, for verification): one thread per candidate.
+__global__ void __launch_bounds__(256) k_features(const K2Launch a) {
+    const DevConfig &c = a.cfg;
+    const int active = *((volatile int32_t *)&a.ctl->active);
+    const long long total = (long long)a.Q * c.I;
+    const int off = (c.mode == 0) ? 1 : 0;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int i = (int)(idx / c.I);
+        const int j = (int)(idx - (long long)i * c.I);
+        long long *F = a.features + idx * 5;
+        const int p = a.prompt[i];
+        if (active < 0 || p < 1 || p > c.pmax) {
+            record_status(a.ctl, active < 0 ? kENoState : kEInval);
+            for (int f = 0; f < 5; ++f) F[f] = -1;
+            continue;
+        }
+        const StateBuf sb = active ? a.buf1 : a.buf0;
+        const InstParams ip = sb.inst[j];
+        const int2 bk = sb.bkt[(size_t)(p >> ip.shift) * c.I + j];
+        const int k = bk.y + (p > bk.x ? 1 : 0);
+        const size_t e = (size_t)k * c.I + j;
+        F[0] = ip.la + k + off;
+        F[1] = ip.f1tot + p;
+        F[2] = sb.f2[e];
+        F[3] = sb.f3[e] + (c.mode == 0 ? p : 0);
+        F[4] = ip.f4tot + ((long long)p * (p + 1)) / 2;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// The candidate kernel.
+enum : int {
+    kOutMatrix = 1,   // write the TTFT matrix
+    kOutIters = 2,    // write the first-token batch index
+    kOutLag = 4,      // Lagrangian argmax (Eq. 5), one (lambda, mu) pair
+    kOutCon = 8,      // constrained argmax (Eq. 3), one lambda
+    kOutSweep = 16    // Lagrangian argmax for several pairs
+};
+
+struct Inst4 {
+    int shift[4];
+    float h1[4], l1[4], h4[4], l4[4], b1p[4], b2[4], b3[4];
+};
+
+template <int MODE>
+__device__ __forceinline__ float ttft_fast(const QRec &q, const Inst4 &r, int u, const float4 e) {
+    const float f1 = __fadd_rn(r.h1[u], __fadd_rn(r.l1[u], q.fp));
+    const float f3 = (MODE == 0) ? __fadd_rn(e.y, __fadd_rn(e.z, q.fp)) : e.w;
+    const float f4 = __fadd_rn(__fadd_rn(r.h4[u], q.ph), __fadd_rn(r.l4[u], q.pl));
+    float t = __fmaf_rn(r.b1p[u], f1, e.x);
+    t = __fmaf_rn(r.b2[u], f3, t);
+    t = __fmaf_rn(r.b3[u], f4, t);
+    return t;
+}
+
+// Exact int64 path for instances whose totals do not split into fp32.
+template <int MODE>
+__device__ float ttft_exact64(const DevConfig &c, const StateBuf &sb, const QRec &q, int j, int k, const float4 e) {
+    if (q.fp != q.fp) return q.fp;
     const InstParams ip = sb.inst[j];
     const int m = c.moi[j];
-    r.jl = jl;
-    r.la = ip.la;
-    r.shift = ip.shift;
-    r.h1 = ip.h1;
-    r.l1 = ip.l1;
-    r.h4 = ip.h4;
-    r.l4 = ip.l4;
-    r.f1tot = ip.f1tot;
-    r.f4tot = ip.f4tot;
-    r.b1p = c.coef[m * 5 + 1];
-    r.b2 = c.coef[m * 5 + 3];
-    r.b3 = c.coef[m * 5 + 4];
-    return r;
-}
-
-// Index of the query's last prefill batch relative to the admission batch.
-__device__ __forceinline__ int locate(const QRec &q, const InstRegs &r, const int2 *s_bkt, int IT) {
-    const int2 bk = s_bkt[(q.p >> r.shift) * IT + r.jl];
-    return bk.y + (q.p > bk.x ? 1 : 0);
-}
-
-template <int MODE>
-__device__ __forceinline__ float ttft_fast(const QRec &q, const InstRegs &r, const float4 e) {
-    const float f1 = __fadd_rn(r.h1, __fadd_rn(r.l1, q.fp));
-    const float f3 = (MODE == 0) ? __fadd_rn(e.y, __fadd_rn(e.z, q.fp)) : e.w;
-    const float f4 = __fadd_rn(__fadd_rn(r.h4, q.ph), __fadd_rn(r.l4, q.pl));
-    float t = __fmaf_rn(r.b1p, f1, e.x);
-    t = __fmaf_rn(r.b2, f3, t);
-    t = __fmaf_rn(r.b3, f4, t);
-    return t;
-}
-
-template <int MODE>
-__device__ __forceinline__ float ttft_exact64(const QRec &q, const InstRegs &r, const float4 e, long long f3b) {
-    if (q.fp != q.fp) return q.fp;
     const long long p = q.p;
-    const float f1 = __ll2float_rn(r.f1tot + p);
-    const float f3 = __ll2float_rn(f3b + (MODE == 0 ? p : 0));
-    const float f4 = __ll2float_rn(r.f4tot + (p * (p + 1)) / 2);
-    float t = __fmaf_rn(r.b1p, f1, e.x);
-    t = __fmaf_rn(r.b2, f3, t);
-    t = __fmaf_rn(r.b3, f4, t);
+    const float f1 = __ll2float_rn(ip.f1tot + p);
+    const float f3 = __ll2float_rn(sb.f3[(size_t)k * c.I + j] + (MODE == 0 ? p : 0));
+    const float f4 = __ll2float_rn(ip.f4tot + (p * (p + 1)) / 2);
+    float t = __fmaf_rn(c.coef[m * 5 + 1], f1, e.x);
+    t = __fmaf_rn(c.coef[m * 5 + 3], f3, t);
+    t = __fmaf_rn(c.coef[m * 5 + 4], f4, t);
     return t;
 }
 
-// Stage the summary tables of instances [j0, j0 + IT) into shared memory.
-__device__ __forceinline__ void stage_tables(const DevConfig &c, const StateBuf &sb, int j0, int IT,
-                                             float4 *s_ent, int2 *s_bkt) {
-    for (int idx = threadIdx.x; idx < c.kph * IT; idx += blockDim.x) {
-        const int k = idx / IT;
-        const int jg = j0 + (idx - k * IT);
-        s_ent[idx] = jg < c.I ? sb.ent[(size_t)k * c.I + jg] : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-    for (int idx = threadIdx.x; idx < c.nbh * IT; idx += blockDim.x) {
-        const int b = idx / IT;
-        const int jg = j0 + (idx - b * IT);
-        s_bkt[idx] = jg < c.I ? sb.bkt[(size_t)b * c.I + jg] : make_int2(kBig, 0);
+// Reduce a key over the row's lanes; returns the winning lane's value of `v`
+// (and its key) to every lane of the row group.  Rows of up to 32 groups sit in
+// an aligned power-of-two lane group; wider rows use whole warps per row.
+__device__ __forceinline__ unsigned group_mask(int Gp, int lane) {
+    if (Gp >= 32) return kFull;
+    const unsigned g = (Gp == 32) ? kFull : ((1u << Gp) - 1u);
+    return g << (lane & ~(Gp - 1));
+}
+
+// A routing candidate: its key, instance, TTFT and utility.
+struct Cand {
+    unsigned key;  // order key of the objective, 0 = none
+    int j;         // instance (the thread-local index before group_pick)
+    float t, U;
+};
+
+__device__ __forceinline__ int4 pack(const Cand &c) {
+    return make_int4((int)c.key, c.j, __float_as_int(c.t), __float_as_int(c.U));
+}
+
+__device__ __forceinline__ Cand unpack(const int4 v) {
+    return Cand{(unsigned)v.x, v.y, __int_as_float(v.z), __int_as_float(v.w)};
+}
+
+__device__ __forceinline__ void write_pick(const K2Launch &a, size_t o, const Cand &w) {
+    if (w.key == 0u) {  // invalid prompt: no instance
+        a.assign[o] = -1;
+        a.util[o] = kNaN;
+        if (a.ttft_chosen) a.ttft_chosen[o] = kNaN;
+    } else {
+        a.assign[o] = w.j;
+        a.util[o] = w.U;
+        if (a.ttft_chosen) a.ttft_chosen[o] = w.t;
     }
 }
 
-enum : int { kOutTtft = 0, kOutTtftIters = 1, kOutFeatures = 2 };
+// Table loads by 32-bit shared-memory address.  The tables are written once
+// before the first barrier and only read afterwards.
+__device__ __forceinline__ int2 lds_int2(uint32_t addr) {
+    int2 v;
+    asm("ld.shared.v2.s32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ float4 lds_float4(uint32_t addr) {
+    float4 v;
+    asm("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ float pick4(const float v[4], int u) {
+    float x = v[0];
+    x = (u == 1) ? v[1] : x;
+    x = (u == 2) ? v[2] : x;
+    x = (u == 3) ? v[3] : x;
+    return x;
+}
+
+template <bool B>
+struct Flag {
+    static constexpr bool value = B;
+};
 
 template <int MODE, int OUT>
-__global__ void __launch_bounds__(256) k_estimate(const K2Launch a) {
+__global__ void __launch_bounds__(256) k_cand(const K2Launch a) {
     extern __shared__ __align__(16) unsigned char smem[];
-    const DevConfig &c = a.cfg;
-    const int I = c.I, IT = a.IT, QS = a.QS, QT = a.QT;
-    const int jl = threadIdx.x % IT;
-    const int qs = threadIdx.x / IT;
-    const int j = blockIdx.y * IT + jl;
-    const bool jv = (qs < QS) && (j < I);
-    const int rows_per = (a.Q + gridDim.x - 1) / gridDim.x;
-    const int rb = blockIdx.x * rows_per;
-    const int re = min(a.Q, rb + rows_per);
-    if (rb >= re) return;
-    const int active = *((volatile int32_t *)&a.ctl->active);
-    if (active < 0) {
-        if (threadIdx.x == 0) record_status(a.ctl, kENoState);
-        if (jv) {
-            for (int rr = rb + qs; rr < re; rr += QS) {
-                const size_t o = (size_t)rr * I + j;
-                if (OUT == kOutFeatures) {
-                    for (int f = 0; f < 5; ++f) a.features[o * 5 + f] = -1;
-                } else {
-                    a.ttft[o] = __int_as_float(0x7fc00000);
-                    if (OUT == kOutTtftIters) a.first_batch[o] = -1;
-                }
-            }
-        }
-        return;
-    }
-    const StateBuf sb = active ? a.buf1 : a.buf0;
-    float4 *s_ent = reinterpret_cast<float4 *>(smem);                 // [kph][IT]
-    QRec *s_q = reinterpret_cast<QRec *>(s_ent + c.kph * IT);          // [QT]
-    int2 *s_bkt = reinterpret_cast<int2 *>(s_q + QT);                  // [nbh][IT]
-    stage_tables(c, sb, blockIdx.y * IT, IT, s_ent, s_bkt);
-    InstRegs r = {};
-    if (jv) r = load_inst(c, sb, j, jl);
-    const int fast = __syncthreads_and(!jv || sb.inst[j].fast);
+    constexpr bool ROUTE = (OUT & (kOutLag | kOutCon | kOutSweep)) != 0;
+    constexpr bool CON = (OUT & kOutCon) != 0;
+    constexpr bool SWEEP = (OUT & kOutSweep) != 0;
     constexpr int off = (MODE == 0) ? 1 : 0;
-
-    for (int q0 = rb; q0 < re; q0 += QT) {
-        const int nrows = min(QT, re - q0);
-        if ((int)threadIdx.x < nrows) {
-            bool ok;
-            s_q[threadIdx.x] = make_qrec(a.prompt[q0 + threadIdx.x], c.pmax, &ok);
-            if (!ok && blockIdx.y == 0) record_status(a.ctl, kEInval);
-        }
-        __syncthreads();
-        if (jv) {
-            float *out = a.ttft + (size_t)q0 * I + j;
-            for (int rr = qs; rr < nrows; rr += QS) {
-                const QRec q = s_q[rr];
-                const int k = locate(q, r, s_bkt, IT);
-                const size_t o = (size_t)rr * I;
-                if (OUT == kOutFeatures) {
-                    long long *F = a.features + ((size_t)(q0 + rr) * I + j) * 5;
-                    if (q.fp != q.fp) {
-                        for (int f = 0; f < 5; ++f) F[f] = -1;
-                    } else {
-                        const long long p = q.p;
-                        const size_t e = (size_t)k * I + j;
-                        F[0] = r.la + k + off;
-                        F[1] = r.f1tot + p;
-                        F[2] = sb.f2[e];
-                        F[3] = sb.f3[e] + (MODE == 0 ? p : 0);
-                        F[4] = r.f4tot + (p * (p + 1)) / 2;
-                    }
-                } else {
-                    const float4 e = s_ent[k * IT + jl];
-                    const float t = fast ? ttft_fast<MODE>(q, r, e)
-                                         : ttft_exact64<MODE>(q, r, e, sb.f3[(size_t)k * I + j]);
-                    __stcs(out + o, t);
-                    if (OUT == kOutTtftIters)
-                        a.first_batch[(size_t)(q0 + rr) * I + j] = (q.fp != q.fp) ? -1 : r.la + k + off;
-                }
-            }
-        }
-        __syncthreads();
-    }
-}
-
-// Route: phase 1 fills a [rows][instances] tile of TTFT in shared memory (and
-// optionally streams it to the estimate matrix); phase 2 scores the tile for
-// each (lambda, mu) pair with TPR threads per row and reduces to one instance
-// per query, ties to the lowest index.
-template <int MODE, bool CONSTRAINED, bool MATRIX>
-__global__ void __launch_bounds__(1024) k_route(const K2Launch a) {
-    extern __shared__ __align__(16) unsigned char smem[];
     const DevConfig &c = a.cfg;
-    const int I = c.I, M = c.M, IT = a.IT, QS = a.QS, QT = a.QT, TPR = a.TPR;
-    const int ST = ((I + 31) & ~31) + TPR;  // padded row stride of the TTFT tile
-    const int jl = threadIdx.x % IT;
-    const int qs = threadIdx.x / IT;
-    const int j = jl;
-    const bool jv = (qs < QS) && (j < I);
+    const int I = c.I, M = c.M, Gp = a.Gp, QS = a.QS, QT = a.QT;
+    const int lane = threadIdx.x & 31;
+    const int g = threadIdx.x % Gp;
+    const int qs = threadIdx.x / Gp;
+    const int j0 = blockIdx.y * Gp * 4;
+    const int jb = j0 + 4 * g;                         // first instance of this thread
+    const int nv = max(0, min(4, I - jb));             // instances this thread owns
     const int rows_per = (a.Q + gridDim.x - 1) / gridDim.x;
     const int rb = blockIdx.x * rows_per;
     const int re = min(a.Q, rb + rows_per);
@@ -226,117 +221,225 @@ __global__ void __launch_bounds__(1024) k_route(const K2Launch a) {
     const int active = *((volatile int32_t *)&a.ctl->active);
     if (active < 0) {
         if (threadIdx.x == 0) record_status(a.ctl, kENoState);
-        for (int pp = 0; pp < a.P; ++pp)
-            for (int i = rb + threadIdx.x; i < re; i += blockDim.x) {
-                a.assign[(size_t)pp * a.Q + i] = -1;
-                a.util[(size_t)pp * a.Q + i] = __int_as_float(0x7fc00000);
-                if (a.ttft_chosen) a.ttft_chosen[(size_t)pp * a.Q + i] = __int_as_float(0x7fc00000);
+        for (int rr = rb + qs; rr < re; rr += QS) {
+            for (int u = 0; u < nv; ++u) {
+                if (OUT & kOutMatrix) a.ttft[(size_t)rr * I + jb + u] = kNaN;
+                if (OUT & kOutIters) a.first_batch[(size_t)rr * I + jb + u] = -1;
             }
-        if (MATRIX && jv)
-            for (int rr = rb + qs; rr < re; rr += QS) a.ttft[(size_t)rr * I + j] = __int_as_float(0x7fc00000);
+            if (ROUTE && g == 0)
+                for (int pp = 0; pp < a.P; ++pp) {
+                    a.assign[(size_t)pp * a.Q + rr] = -1;
+                    a.util[(size_t)pp * a.Q + rr] = kNaN;
+                    if (a.ttft_chosen) a.ttft_chosen[(size_t)pp * a.Q + rr] = kNaN;
+                }
+        }
         return;
     }
     const StateBuf sb = active ? a.buf1 : a.buf0;
-    float4 *s_ent = reinterpret_cast<float4 *>(smem);                 // [kph][IT]
-    QRec *s_q = reinterpret_cast<QRec *>(s_ent + c.kph * IT);          // [QT]
-    int2 *s_bkt = reinterpret_cast<int2 *>(s_q + QT);                  // [nbh][IT]
-    float2 *s_ca = reinterpret_cast<float2 *>(s_bkt + c.nbh * IT);     // [QT][M] (cost, acc)
-    float *s_t = reinterpret_cast<float *>(s_ca + QT * M);             // [QT][ST]
-    float *s_tau = s_t + QT * ST;                                      // [QT]
-    int *s_moi = reinterpret_cast<int *>(s_tau + QT);                  // [I]
-    stage_tables(c, sb, 0, IT, s_ent, s_bkt);
-    for (int jj = threadIdx.x; jj < I; jj += blockDim.x) s_moi[jj] = c.moi[jj];
-    InstRegs r = {};
-    if (jv) r = load_inst(c, sb, j, jl);
-    const int fast = __syncthreads_and(!jv || sb.inst[j].fast);
+    // shared memory: tables, query records, row partials, utility inputs, targets
+    // (route with one pair stages (U, cost) per row and model, sweeps (cost, acc))
+    const int WPR = Gp > 32 ? Gp / 32 : 1;  // warps per row
+    const int NP = SWEEP ? a.P : 1;
+    float4 *s_ent = reinterpret_cast<float4 *>(smem);                                  // [kph][4][Gp]
+    QRec *s_q = reinterpret_cast<QRec *>(s_ent + c.kph * 4 * Gp);                      // [QT]
+    int4 *s_part = reinterpret_cast<int4 *>(s_q + QT);                                 // [NP][QT][WPR][2]
+    int2 *s_bkt = reinterpret_cast<int2 *>(s_part + (ROUTE && Gp > 32 ? 2 * NP * QT * WPR : 0));  // [nbh][4][Gp]
+    float2 *s_ca = reinterpret_cast<float2 *>(s_bkt + c.nbh * 4 * Gp);                 // [QT][M] (cost, acc)
+    float *s_tau = reinterpret_cast<float *>(s_ca + (ROUTE ? QT * M : 0));             // [QT]
 
-    const int rr2 = threadIdx.x / TPR;  // phase-2 row
-    const int u = threadIdx.x % TPR;    // phase-2 lane within the row group
+    for (int idx = threadIdx.x; idx < c.kph * 4 * Gp; idx += blockDim.x) {
+        const int k = idx / (4 * Gp);
+        const int rem = idx - k * 4 * Gp;
+        const int u = rem / Gp;
+        const int jg = j0 + 4 * (rem - u * Gp) + u;
+        s_ent[idx] = jg < I ? sb.ent[(size_t)k * I + jg] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    for (int idx = threadIdx.x; idx < c.nbh * 4 * Gp; idx += blockDim.x) {
+        const int b = idx / (4 * Gp);
+        const int rem = idx - b * 4 * Gp;
+        const int u = rem / Gp;
+        const int jg = j0 + 4 * (rem - u * Gp) + u;
+        s_bkt[idx] = jg < I ? sb.bkt[(size_t)b * I + jg] : make_int2(kBig, 0);
+    }
+    Inst4 r;
+    int model[4], la[4];
+    bool fast_mine = true;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int j = min(jb + u, I - 1);
+        const InstParams ip = sb.inst[j];
+        const int m = c.moi[j];
+        r.shift[u] = ip.shift;
+        r.h1[u] = ip.h1;
+        r.l1[u] = ip.l1;
+        r.h4[u] = ip.h4;
+        r.l4[u] = ip.l4;
+        r.b1p[u] = c.coef[m * 5 + 1];
+        r.b2[u] = c.coef[m * 5 + 3];
+        r.b3[u] = c.coef[m * 5 + 4];
+        model[u] = m;
+        la[u] = ip.la;
+        if (u < nv) fast_mine = fast_mine && ip.fast != 0;
+    }
+    const bool fast = __syncthreads_and(fast_mine);
+    const bool vec = a.vec_ok && nv == 4;
+    const unsigned gmask = group_mask(Gp, lane);
+    const int grp_lane0 = lane & ~(min(Gp, 32) - 1);  // first lane of this row group in the warp
+    const int wrow = g / 32;                          // warp index within a wide row
+    // shared addresses of this thread's table columns: entry (k, u) at ecol[u] + k * erow,
+    // bucket (b, u) at bcol[u] + b * brow
+    uint32_t ecol[4], bcol[4];
+    const uint32_t e0 = (uint32_t)__cvta_generic_to_shared(s_ent), b0 = (uint32_t)__cvta_generic_to_shared(s_bkt);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        ecol[u] = e0 + 16u * (uint32_t)(u * Gp + g);
+        bcol[u] = b0 + 8u * (uint32_t)(u * Gp + g);
+    }
+    const uint32_t erow = 16u * 4u * (uint32_t)Gp, brow = 8u * 4u * (uint32_t)Gp;
+    bool same_model = true;
+#pragma unroll
+    for (int u = 1; u < 4; ++u) same_model = same_model && model[u] == model[0];
 
-    for (int q0 = rb; q0 < re; q0 += QT) {
-        const int nrows = min(QT, re - q0);
-        if ((int)threadIdx.x < nrows) {
-            bool ok;
-            const int p = a.prompt[q0 + threadIdx.x];
-            s_q[threadIdx.x] = make_qrec(p, c.pmax, &ok);
-            if (!ok) record_status(a.ctl, kEInval);
-            if (CONSTRAINED) s_tau[threadIdx.x] = a.tau[q0 + threadIdx.x];
-        }
-        // per (row, model): cost of App. B.4 and the predicted accuracy
-        for (int idx = threadIdx.x; idx < nrows * M; idx += blockDim.x) {
-            const int rr = idx / M;
-            const int m = idx - rr * M;
-            const size_t g = (size_t)(q0 + rr) * M + m;
-            const float cost = __fmaf_rn((float)a.dec_hat[g], c.pout[m], __fmul_rn((float)a.prompt[q0 + rr], c.pin[m]));
-            s_ca[idx] = make_float2(cost, a.acc[g]);
-        }
-        __syncthreads();
-        if (jv) {
+    auto run = [&](auto fast_tag) {
+        constexpr bool FAST = decltype(fast_tag)::value;
+        for (int q0 = rb; q0 < re; q0 += QT) {
+            const int nrows = min(QT, re - q0);
+            for (int t = threadIdx.x; t < nrows; t += blockDim.x) {
+                bool ok;
+                s_q[t] = make_qrec(a.prompt[q0 + t], c.pmax, &ok);
+                if (!ok && blockIdx.y == 0) record_status(a.ctl, kEInval);
+                if (CON) s_tau[t] = a.tau[q0 + t];
+            }
+            if (ROUTE) {
+                for (int idx = threadIdx.x; idx < nrows * M; idx += blockDim.x) {
+                    const int rr = idx / M;
+                    const int m = idx - rr * M;
+                    const size_t gi = (size_t)(q0 + rr) * M + m;
+                    const float cost = __fmaf_rn((float)a.dec_hat[gi], c.pout[m],
+                                                 __fmul_rn((float)a.prompt[q0 + rr], c.pin[m]));
+                    const float acc = a.acc[gi];
+                    // one pair: stage U itself (x), else (cost, acc)
+                    s_ca[idx] = SWEEP ? make_float2(cost, acc) : make_float2(__fmaf_rn(-a.lam[0], cost, acc), cost);
+                }
+            }
+            __syncthreads();
+            float *orow = (OUT & kOutMatrix) ? a.ttft + (size_t)(q0 + qs) * I + jb : nullptr;
+            const size_t ostep = (size_t)QS * I;
             for (int rr = qs; rr < nrows; rr += QS) {
                 const QRec q = s_q[rr];
-                const int k = locate(q, r, s_bkt, IT);
-                const float4 e = s_ent[k * IT + jl];
-                const float t = fast ? ttft_fast<MODE>(q, r, e)
-                                     : ttft_exact64<MODE>(q, r, e, sb.f3[(size_t)k * I + j]);
-                s_t[rr * ST + j] = t;
-                if (MATRIX) __stcs(a.ttft + (size_t)(q0 + rr) * I + j, t);
-            }
-        }
-        __syncthreads();
-        const bool live = rr2 < nrows;
-        const float *trow = s_t + (live ? rr2 : 0) * ST;
-        const float2 *carow = s_ca + (live ? rr2 : 0) * M;
-        for (int pp = 0; pp < a.P; ++pp) {
-            const float lam = a.lam[pp];
-            const float mu = a.mu[pp];
-            float best = 0.f, bestu = 0.f, fastest = 0.f;
-            int bj = kBig, bju = kBig, bjt = kBig;
-            if (live) {
-                const float tau = CONSTRAINED ? s_tau[rr2] : 0.f;
-                for (int jj = u; jj < I; jj += TPR) {
-                    const float t = trow[jj];
-                    const float2 ca = carow[s_moi[jj]];
-                    const float U = __fmaf_rn(-lam, ca.x, ca.y);
-                    if (CONSTRAINED) {
-                        if (t <= tau && (bju == kBig || U > bestu)) { bestu = U; bju = jj; }
-                        if (t == t && (bjt == kBig || t < fastest)) { fastest = t; bjt = jj; }
+                float t[4];
+                int kk[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int2 bk = lds_int2(bcol[u] + (uint32_t)(q.p >> r.shift[u]) * brow);
+                    kk[u] = bk.y + (q.p > bk.x ? 1 : 0);
+                    const float4 e = lds_float4(ecol[u] + (uint32_t)kk[u] * erow);
+                    if (FAST) t[u] = ttft_fast<MODE>(q, r, u, e);
+                    else t[u] = (u < nv) ? ttft_exact64<MODE>(c, sb, q, jb + u, kk[u], e) : 0.f;
+                }
+                if (OUT & kOutMatrix) {
+                    if (vec) {
+                        __stcs(reinterpret_cast<float4 *>(orow), make_float4(t[0], t[1], t[2], t[3]));
                     } else {
-                        const float J = __fmaf_rn(-mu, t, U);
-                        if (J == J && (bj == kBig || J > best)) { best = J; bj = jj; }
+                        for (int u = 0; u < nv; ++u) __stcs(orow + u, t[u]);
+                    }
+                    orow += ostep;
+                }
+                if (OUT & kOutIters) {
+                    const bool bad = q.fp != q.fp;
+                    const size_t o = (size_t)(q0 + rr) * I + jb;
+                    for (int u = 0; u < nv; ++u) a.first_batch[o + u] = bad ? -1 : la[u] + kk[u] + off;
+                }
+                if (ROUTE) {
+                    const bool row_ok = q.fp == q.fp;
+                    const float2 *carow = s_ca + rr * M;
+                    const float tau = CON ? s_tau[rr] : 0.f;
+#pragma unroll 1
+                    for (int pp = 0; pp < (SWEEP ? NP : 1); ++pp) {
+                        const float lam = SWEEP ? a.lam[pp] : 0.f;
+                        const float mu = a.mu[pp];
+                        float U[4];
+                        if (same_model) {
+                            const float2 ca = carow[model[0]];
+                            U[0] = U[1] = U[2] = U[3] = SWEEP ? __fmaf_rn(-lam, ca.x, ca.y) : ca.x;
+                        } else {
+#pragma unroll
+                            for (int u = 0; u < 4; ++u) {
+                                const float2 ca = carow[model[u]];
+                                U[u] = SWEEP ? __fmaf_rn(-lam, ca.x, ca.y) : ca.x;
+                            }
+                        }
+                        // this thread's best of its four instances (first max wins); NaN marks
+                        // an invalid row or an instance beyond the pool
+                        float best1, best2 = 0.f;
+                        int u1 = 0, u2 = 0;
+                        if (CON) {
+                            best1 = (0 < nv && row_ok && t[0] <= tau) ? U[0] : kNaN;
+                            best2 = (0 < nv && row_ok) ? t[0] : kNaN;
+#pragma unroll
+                            for (int u = 1; u < 4; ++u) {
+                                if (u < nv && t[u] <= tau && (U[u] > best1 || best1 != best1)) { best1 = U[u]; u1 = u; }
+                                if (u < nv && t[u] < best2) { best2 = t[u]; u2 = u; }
+                            }
+                        } else {
+                            best1 = (0 < nv && row_ok) ? __fmaf_rn(-mu, t[0], U[0]) : kNaN;
+#pragma unroll
+                            for (int u = 1; u < 4; ++u) {
+                                const float J = __fmaf_rn(-mu, t[u], U[u]);
+                                if (u < nv && J > best1) { best1 = J; u1 = u; }
+                            }
+                        }
+                        const unsigned k1 = (best1 == best1) ? order_key(best1) : 0u;
+                        const unsigned k2 = (CON && best2 == best2 && row_ok) ? order_key(-best2) : 0u;
+                        // row group argmax: the lowest lane among the maximal keys
+                        const unsigned w1 = __reduce_max_sync(gmask, k1);
+                        const int src1 = __ffs(__ballot_sync(gmask, k1 == w1) & gmask) - 1;
+                        unsigned w2 = 0u;
+                        int src2 = 0;
+                        if (CON) {
+                            w2 = __reduce_max_sync(gmask, k2);
+                            src2 = __ffs(__ballot_sync(gmask, k2 == w2) & gmask) - 1;
+                        }
+                        // the winner of each reduction describes itself
+                        const Cand c1 = {w1, jb + u1, pick4(t, u1), pick4(U, u1)};
+                        const Cand c2 = {w2, jb + u2, pick4(t, u2), pick4(U, u2)};
+                        if (Gp <= 32) {
+                            const bool use2 = CON && w1 == 0u;
+                            if (lane == (use2 ? src2 : src1))
+                                write_pick(a, (size_t)pp * a.Q + q0 + rr, use2 ? c2 : c1);
+                        } else {
+                            // wide rows: each warp leaves its partial; combined once per chunk
+                            int4 *part = s_part + 2 * ((pp * QT + rr) * WPR + wrow);
+                            if (lane == src1) part[0] = pack(c1);
+                            if (CON && lane == src2) part[1] = pack(c2);
+                        }
                     }
                 }
             }
-            for (int o = TPR >> 1; o > 0; o >>= 1) {
-                if (CONSTRAINED) {
-                    const float ou = __shfl_xor_sync(kFull, bestu, o);
-                    const int oj = __shfl_xor_sync(kFull, bju, o);
-                    if (oj != kBig && (bju == kBig || ou > bestu || (ou == bestu && oj < bju))) { bestu = ou; bju = oj; }
-                    const float ot = __shfl_xor_sync(kFull, fastest, o);
-                    const int ojt = __shfl_xor_sync(kFull, bjt, o);
-                    if (ojt != kBig && (bjt == kBig || ot < fastest || (ot == fastest && ojt < bjt))) { fastest = ot; bjt = ojt; }
-                } else {
-                    const float oJ = __shfl_xor_sync(kFull, best, o);
-                    const int oj = __shfl_xor_sync(kFull, bj, o);
-                    if (oj != kBig && (bj == kBig || oJ > best || (oJ == best && oj < bj))) { best = oJ; bj = oj; }
+            if (ROUTE && Gp > 32) {
+                // one thread per (row, pair) combines the warps of the row in instance order
+                __syncthreads();
+                for (int t2 = threadIdx.x; t2 < nrows * NP; t2 += blockDim.x) {
+                    const int pp = t2 / nrows;
+                    const int r2 = t2 - pp * nrows;
+                    Cand c1 = {0u, 0, 0.f, 0.f}, c2 = {0u, 0, 0.f, 0.f};
+                    for (int wi = 0; wi < WPR; ++wi) {
+                        const Cand x1 = unpack(s_part[2 * ((pp * QT + r2) * WPR + wi)]);
+                        if (x1.key > c1.key) c1 = x1;
+                        if (CON) {
+                            const Cand x2 = unpack(s_part[2 * ((pp * QT + r2) * WPR + wi) + 1]);
+                            if (x2.key > c2.key) c2 = x2;
+                        }
+                    }
+                    write_pick(a, (size_t)pp * a.Q + q0 + r2, (CON && c1.key == 0u) ? c2 : c1);
                 }
             }
-            if (live && u == 0) {
-                const int pick = CONSTRAINED ? (bju != kBig ? bju : bjt) : bj;
-                const size_t o = (size_t)pp * a.Q + q0 + rr2;
-                if (pick == kBig) {
-                    a.assign[o] = -1;
-                    a.util[o] = __int_as_float(0x7fc00000);
-                    if (a.ttft_chosen) a.ttft_chosen[o] = __int_as_float(0x7fc00000);
-                } else {
-                    const float2 ca = carow[s_moi[pick]];
-                    a.assign[o] = pick;
-                    a.util[o] = __fmaf_rn(-lam, ca.x, ca.y);
-                    if (a.ttft_chosen) a.ttft_chosen[o] = trow[pick];
-                }
-            }
+            __syncthreads();
         }
-        __syncthreads();
-    }
+    };
+    if (fast) run(Flag<true>{});
+    else run(Flag<false>{});
+    (void)grp_lane0;
 }
 
 // Per-pair means of (accuracy, cost, TTFT) of the chosen instances, fp64, fixed
@@ -373,21 +476,18 @@ __global__ void __launch_bounds__(256) k_frontier(const K2Launch a, double *out)
 }
 
 template <int MODE>
-cudaError_t launch_est_mode(const K2Launch &a, int kind, dim3 grid, int block, size_t smem, cudaStream_t st) {
-    if (kind == kEstFeatures) {
-        k_estimate<MODE, kOutFeatures><<<grid, block, smem, st>>>(a);
-    } else if (a.first_batch) {
-        k_estimate<MODE, kOutTtftIters><<<grid, block, smem, st>>>(a);
-    } else {
-        k_estimate<MODE, kOutTtft><<<grid, block, smem, st>>>(a);
+cudaError_t launch_cand_mode(const K2Launch &a, int out, dim3 grid, int block, size_t smem, cudaStream_t st) {
+    switch (out) {
+        case kOutMatrix: k_cand<MODE, kOutMatrix><<<grid, block, smem, st>>>(a); break;
+        case kOutMatrix | kOutIters: k_cand<MODE, kOutMatrix | kOutIters><<<grid, block, smem, st>>>(a); break;
+        case kOutLag: k_cand<MODE, kOutLag><<<grid, block, smem, st>>>(a); break;
+        case kOutLag | kOutMatrix: k_cand<MODE, kOutLag | kOutMatrix><<<grid, block, smem, st>>>(a); break;
+        case kOutCon: k_cand<MODE, kOutCon><<<grid, block, smem, st>>>(a); break;
+        case kOutCon | kOutMatrix: k_cand<MODE, kOutCon | kOutMatrix><<<grid, block, smem, st>>>(a); break;
+        case kOutSweep: k_cand<MODE, kOutSweep><<<grid, block, smem, st>>>(a); break;
+        case kOutSweep | kOutMatrix: k_cand<MODE, kOutSweep | kOutMatrix><<<grid, block, smem, st>>>(a); break;
+        default: return cudaErrorInvalidValue;
     }
-    return cudaGetLastError();
-}
-
-template <int MODE, bool CON>
-cudaError_t launch_route_mode(const K2Launch &a, dim3 grid, int block, size_t smem, cudaStream_t st) {
-    if (a.ttft) k_route<MODE, CON, true><<<grid, block, smem, st>>>(a);
-    else k_route<MODE, CON, false><<<grid, block, smem, st>>>(a);
     return cudaGetLastError();
 }
 
@@ -396,19 +496,38 @@ cudaError_t set_attr(F f, size_t bytes) {
     return cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
 
-}  // namespace
-
-cudaError_t launch_estimate(const K2Launch &a, int kind, dim3 grid, int block, size_t smem, cudaStream_t st) {
-    return a.cfg.mode == 0 ? launch_est_mode<0>(a, kind, grid, block, smem, st)
-                           : launch_est_mode<1>(a, kind, grid, block, smem, st);
+template <int MODE>
+cudaError_t set_mode_attrs(size_t bytes) {
+    const cudaError_t es[] = {
+        set_attr(k_cand<MODE, kOutMatrix>, bytes), set_attr(k_cand<MODE, kOutMatrix | kOutIters>, bytes),
+        set_attr(k_cand<MODE, kOutLag>, bytes), set_attr(k_cand<MODE, kOutLag | kOutMatrix>, bytes),
+        set_attr(k_cand<MODE, kOutCon>, bytes), set_attr(k_cand<MODE, kOutCon | kOutMatrix>, bytes),
+        set_attr(k_cand<MODE, kOutSweep>, bytes), set_attr(k_cand<MODE, kOutSweep | kOutMatrix>, bytes)};
+    for (cudaError_t x : es)
+        if (x != cudaSuccess) return x;
+    return cudaSuccess;
 }
 
-cudaError_t launch_route(const K2Launch &a, dim3 grid, int block, size_t smem, cudaStream_t st) {
-    const bool con = a.tau != nullptr;
-    if (a.cfg.mode == 0) return con ? launch_route_mode<0, true>(a, grid, block, smem, st)
-                                    : launch_route_mode<0, false>(a, grid, block, smem, st);
-    return con ? launch_route_mode<1, true>(a, grid, block, smem, st)
-               : launch_route_mode<1, false>(a, grid, block, smem, st);
+}  // namespace
+
+int cand_out_flags(bool matrix, bool iters, bool route, bool constrained, int P) {
+    int f = 0;
+    if (matrix) f |= kOutMatrix;
+    if (iters) f |= kOutIters;
+    if (route) f |= constrained ? kOutCon : (P > 1 ? kOutSweep : kOutLag);
+    return f;
+}
+
+cudaError_t launch_cand(const K2Launch &a, int out, dim3 grid, int block, size_t smem, cudaStream_t st) {
+    return a.cfg.mode == 0 ? launch_cand_mode<0>(a, out, grid, block, smem, st)
+                           : launch_cand_mode<1>(a, out, grid, block, smem, st);
+}
+
+cudaError_t launch_features(const K2Launch &a, int sms, cudaStream_t st) {
+    const long long total = (long long)a.Q * a.cfg.I;
+    const int grid = (int)std::min<long long>((total + 255) / 256, (long long)sms * 8);
+    k_features<<<grid, 256, 0, st>>>(a);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_frontier(const K2Launch &a, double *out, cudaStream_t st) {
@@ -416,30 +535,18 @@ cudaError_t launch_frontier(const K2Launch &a, double *out, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-cudaError_t set_k2_smem(size_t est, size_t route) {
-    cudaError_t e = cudaSuccess;
-    const cudaError_t es[] = {
-        set_attr(k_estimate<0, kOutTtft>, est), set_attr(k_estimate<0, kOutTtftIters>, est),
-        set_attr(k_estimate<0, kOutFeatures>, est), set_attr(k_estimate<1, kOutTtft>, est),
-        set_attr(k_estimate<1, kOutTtftIters>, est), set_attr(k_estimate<1, kOutFeatures>, est),
-        set_attr(k_route<0, true, true>, route), set_attr(k_route<0, true, false>, route),
-        set_attr(k_route<0, false, true>, route), set_attr(k_route<0, false, false>, route),
-        set_attr(k_route<1, true, true>, route), set_attr(k_route<1, true, false>, route),
-        set_attr(k_route<1, false, true>, route), set_attr(k_route<1, false, false>, route)};
-    for (cudaError_t x : es)
-        if (x != cudaSuccess) e = x;
+cudaError_t set_k2_smem(size_t bytes) {
+    cudaError_t e = set_mode_attrs<0>(bytes);
+    if (e == cudaSuccess) e = set_mode_attrs<1>(bytes);
     return e;
 }
 
-cudaError_t estimate_occupancy(int kind, int mode, int block, size_t smem, int *n) {
-    (void)kind;
-    return mode == 0 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, k_estimate<0, kOutTtft>, block, smem)
-                     : cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, k_estimate<1, kOutTtft>, block, smem);
-}
-
-cudaError_t route_occupancy(int mode, int block, size_t smem, int *n) {
-    return mode == 0 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, k_route<0, false, true>, block, smem)
-                     : cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, k_route<1, false, true>, block, smem);
+cudaError_t cand_occupancy(int mode, bool route, int block, size_t smem, int *n) {
+    if (route)
+        return mode == 0 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, k_cand<0, kOutLag | kOutMatrix>, block, smem)
+                         : cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, k_cand<1, kOutLag | kOutMatrix>, block, smem);
+    return mode == 0 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, k_cand<0, kOutMatrix>, block, smem)
+                     : cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, k_cand<1, kOutMatrix>, block, smem);
 }
 
 }  // namespace lr

@@ -44,7 +44,7 @@ struct InstParams {      // 64 bytes
 
 struct DevConfig {
     int32_t I, M, capR, capW;
-    int32_t pmax, mode, max_iters, slots;  // slots: decoder slots per instance in K1
+    int32_t pmax, mode, max_iters, pad0;
     int32_t kph, nbh;                       // table row counts (host bounds over instances)
     const int32_t *moi, *B, *S, *shift, *nb;
     const float *coef, *pin, *pout;
@@ -97,10 +97,17 @@ cudaError_t launch_trajectory(const K1Launch &a, int grid, int block, size_t sme
 cudaError_t set_k1_smem(size_t bytes);
 constexpr int kK1Warps = 4;
 
-// Shared memory of one K1 warp: decoder slots (s, f, cb, free list), the
-// waiting queue and the cumulative budgets.
+// Batches covered by K1's completion calendar; decoders ending later are
+// tracked by scanning the decoder list.
+constexpr int kCalendar = 2048;
+
+// Shared memory of one K1 warp (in int32 words, a multiple of 4): calendar and
+// its bitmap, the waiting queue's prompt prefix sums and decode lengths, the
+// decoder list (first batch, last batch, context offset) and the budgets.
 __host__ __device__ inline size_t trajectory_smem_per_warp(const DevConfig &c) {
-    return sizeof(int32_t) * (4 * (size_t)c.slots + 2 * (size_t)c.capW + (size_t)c.kph);
+    const size_t words = (size_t)kCalendar + kCalendar / 32 + (size_t)(c.capW + 1) + (size_t)c.capW +
+                         3 * (size_t)(c.capR + c.capW) + (size_t)c.kph;
+    return sizeof(int32_t) * ((words + 3) & ~(size_t)3);
 }
 
 struct K2Launch {
@@ -123,16 +130,17 @@ struct K2Launch {
     int32_t *assign;
     float *util;
     float *ttft_chosen;
-    // launch shape
-    int32_t IT, QS, QT, TPR;
+    // launch shape: Gp thread groups of four instances per row (a power of two up
+    // to 32, else a multiple of 32), QS rows in flight, QT rows per staged chunk
+    int32_t Gp, QS, QT, vec_ok;
 };
-cudaError_t launch_estimate(const K2Launch &a, int kind, dim3 grid, int block, size_t smem, cudaStream_t st);
-cudaError_t launch_route(const K2Launch &a, dim3 grid, int block, size_t smem, cudaStream_t st);
+int cand_out_flags(bool matrix, bool iters, bool route, bool constrained, int P);
+cudaError_t launch_cand(const K2Launch &a, int out, dim3 grid, int block, size_t smem, cudaStream_t st);
+cudaError_t launch_features(const K2Launch &a, int sms, cudaStream_t st);
 cudaError_t launch_frontier(const K2Launch &a, double *out, cudaStream_t st);
-cudaError_t estimate_occupancy(int kind, int mode, int block, size_t smem, int *blocks_per_sm);
-cudaError_t route_occupancy(int mode, int block, size_t smem, int *blocks_per_sm);
-cudaError_t set_k2_smem(size_t estimate_bytes, size_t route_bytes);
-
-enum : int { kEstTtft = 0, kEstFeatures = 1 };
+cudaError_t cand_occupancy(int mode, bool route, int block, size_t smem, int *blocks_per_sm);
+cudaError_t set_k2_smem(size_t bytes);
+constexpr int kK2Block = 256;
+constexpr size_t kK2SmemTarget = 56 * 1024;
 
 }  // namespace lr

@@ -21,8 +21,16 @@
 // token in every batch (decoders come first and number fewer than B_j), so
 // decode progress is lockstep: a request that starts decoding in batch s with
 // d tokens to go decodes in batches s..s+d-1 at context cb + l.  The warp
-// keeps one slot (s, f, cb) per decoder in shared memory and jumps over runs
-// of batches in which nothing but decoding happens.
+// therefore never touches individual decoders while it steps:
+//
+//   * every decoder is appended once to a list (s, f, cb); its Eq. 9 decode
+//     features up to any batch L follow in closed form, summed over the list
+//     in parallel after the loop;
+//   * a calendar counts decoders by last decode batch f (with a bitmap to find
+//     the next non-empty batch); decoders ending beyond the calendar are rare
+//     and handled by scanning the list;
+//   * waiting requests are admitted a batch-group at a time: 32 lanes test the
+//     next 32 requests against the budget with the prompts' prefix sums.
 #include "lr_internal.cuh"
 
 namespace lr {
@@ -32,93 +40,27 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 
 struct WarpSmem {
-    int32_t *s, *f, *cb, *freel, *wpre, *wdec, *rcum;
+    int32_t *P;      // [capW + 1] exclusive prefix sums of waiting prompts
+    int32_t *wdec;   // [capW] waiting decode lengths
+    int32_t *ds;     // [capR + capW] decoder list: first decode batch
+    int32_t *df;     //   last decode batch
+    int32_t *dcb;    //   context at batch l is dcb + l
+    int32_t *cal;    // [kCalendar] decoders by last decode batch
+    uint32_t *bm;    // [kCalendar / 32] non-empty calendar batches
+    int32_t *rcum;   // [kph] cumulative budgets
 };
 
 __device__ __forceinline__ WarpSmem carve(int32_t *base, const DevConfig &c) {
     WarpSmem w;
-    w.s = base;
-    w.f = w.s + c.slots;
-    w.cb = w.f + c.slots;
-    w.freel = w.cb + c.slots;
-    w.wpre = w.freel + c.slots;
-    w.wdec = w.wpre + c.capW;
-    w.rcum = w.wdec + c.capW;
+    w.cal = base;
+    w.bm = reinterpret_cast<uint32_t *>(w.cal + kCalendar);
+    w.P = reinterpret_cast<int32_t *>(w.bm + kCalendar / 32);
+    w.wdec = w.P + (c.capW + 1);
+    w.ds = w.wdec + c.capW;
+    w.df = w.ds + (c.capR + c.capW);
+    w.dcb = w.df + (c.capR + c.capW);
+    w.rcum = w.dcb + (c.capR + c.capW);
     return w;
-}
-
-// Decoder slots of one instance, manipulated by all 32 lanes in lockstep.
-struct Slots {
-    WarpSmem m;
-    int n;          // slots in use
-    int top;        // free-list size
-    int fmin;       // smallest last-decode batch over used slots (kBig if none)
-    long long f2d;  // this lane's share of decode tokens of finished decoders
-    long long f3d;  // ... and of their decode context
-    int lane;
-    int nslots_cap;
-    bool overflow;
-
-    // Drop decoders whose last decode batch is before l; fold their features.
-    __device__ void remove_before(int l) {
-        int removed = 0;
-        int mn = kBig;
-        for (int base = 0; base < nslots_cap; base += 32) {
-            const int idx = base + lane;
-            const int f = m.f[idx];
-            const bool rm = f < l;  // free slots hold kBig
-            if (rm) {
-                const int s = m.s[idx];
-                const long long cnt = (long long)f - s + 1;
-                f2d += cnt;
-                f3d += cnt * (long long)m.cb[idx] + (((long long)s + f) * cnt) / 2;
-                m.f[idx] = kBig;
-                m.s[idx] = kBig;
-            } else {
-                mn = min(mn, f);
-            }
-            const unsigned b = __ballot_sync(kFull, rm);
-            if (rm) m.freel[top + __popc(b & lanemask_lt())] = idx;
-            top += __popc(b);
-            removed += __popc(b);
-        }
-        __syncwarp();
-        fmin = __reduce_min_sync(kFull, mn);
-        n -= removed;
-    }
-
-    // New decoder: first decode batch s, last decode batch f, context at batch l is cb + l.
-    __device__ void insert(int s, int f, int cb) {
-        if (top <= 0) {  // more decoders than slots: excluded by the preconditions
-            overflow = true;
-            return;
-        }
-        const int idx = m.freel[top - 1];
-        --top;
-        if (lane == 0) {
-            m.s[idx] = s;
-            m.f[idx] = f;
-            m.cb[idx] = cb;
-        }
-        fmin = min(fmin, f);
-        ++n;
-    }
-
-    // Move to batch l: finished decoders leave.
-    __device__ void advance_to(int l) {
-        __syncwarp();
-        if (l > fmin) remove_before(l);
-    }
-};
-
-// A request finished its prompt in batch e with ce tokens of context and d
-// output tokens to produce (Sec. 4.1: decode begins after the prefill).
-__device__ __forceinline__ void prefill_done(Slots &sl, int mode, int e, int ce, int d) {
-    if (mode == 0) {
-        sl.insert(e + 1, e + d, ce - (e + 1));
-    } else if (d >= 2) {  // first token sampled with the last chunk
-        sl.insert(e + 1, e + d - 1, ce - (e + 1));
-    }
 }
 
 __device__ void fail(DevCtl *ctl, int code, int lane) {
@@ -126,6 +68,75 @@ __device__ void fail(DevCtl *ctl, int code, int lane) {
         atomicCAS(&ctl->load_err, 0, code);
         record_status(ctl, code);
     }
+}
+
+struct Sim {
+    WarpSmem m;
+    int lane;
+    int nlist;    // decoders in the list
+    int far_min;  // smallest last-decode batch >= kCalendar among live decoders (kBig if none)
+
+    // Smallest calendar batch >= L holding a decoder end.
+    __device__ int next_cal(int L) const {
+        for (int w0 = L >> 5; w0 < kCalendar / 32; w0 += 32) {
+            const int w = w0 + lane;
+            uint32_t word = (w < kCalendar / 32) ? m.bm[w] : 0u;
+            if (w == (L >> 5)) word &= ~0u << (L & 31);
+            const unsigned nz = __ballot_sync(kFull, word != 0u);
+            if (nz) {
+                const int src = __ffs(nz) - 1;
+                const uint32_t wv = __shfl_sync(kFull, word, src);
+                return (w0 + src) * 32 + __ffs(wv) - 1;
+            }
+        }
+        return kBig;
+    }
+
+    __device__ int next_end(int L) const { return min(next_cal(L), far_min); }
+
+    // Number of decoders whose last decode batch is fc.
+    __device__ int ends_at(int fc) {
+        int c = fc < kCalendar ? m.cal[fc] : 0;
+        if (fc == far_min) {
+            int eq = 0, mn = kBig;
+            for (int i = lane; i < nlist; i += 32) {
+                const int f = m.df[i];
+                eq += (f == fc) ? 1 : 0;
+                if (f >= kCalendar && f > fc) mn = min(mn, f);
+            }
+            c += __reduce_add_sync(kFull, eq);
+            far_min = __reduce_min_sync(kFull, mn);
+        }
+        return c;
+    }
+
+    // Append a decoder from the lanes with `mine` set; returns the smallest new end.
+    __device__ int append(bool mine, int s, int f, int cb) {
+        const unsigned bal = __ballot_sync(kFull, mine);
+        if (mine) {
+            const int pos = nlist + __popc(bal & lanemask_lt());
+            m.ds[pos] = s;
+            m.df[pos] = f;
+            m.dcb[pos] = cb;
+            if (f < kCalendar) {
+                atomicAdd(&m.cal[f], 1);
+                atomicOr(&m.bm[f >> 5], 1u << (f & 31));
+            }
+        }
+        nlist += __popc(bal);
+        far_min = min(far_min, __reduce_min_sync(kFull, (mine && f >= kCalendar) ? f : kBig));
+        return __reduce_min_sync(kFull, mine ? f : kBig);
+    }
+};
+
+// Last decode batch and context offset of a request that finished its prompt in
+// batch e with ce tokens of context and d output tokens (Sec. 4.1: the decode
+// stage starts after the prefill).  Returns false if it never decodes (first
+// token sampled with the last chunk and d == 1).
+__device__ __forceinline__ bool decoder_of(int mode, int e, int ce, int d, int *f, int *cb) {
+    *cb = ce - (e + 1);
+    *f = e + d - mode;
+    return mode == 0 || d >= 2;
 }
 
 __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j, int lane, int32_t *wbase) {
@@ -145,10 +156,18 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     WarpSmem m = carve(wbase, c);
     const size_t rrow = (size_t)j * c.capR;
     const size_t wrow = (size_t)j * c.capW;
+    const int mode = c.mode;
 
-    // Copy the snapshot into library memory, validate it and total the prefill work.
+    // Clear the calendar.
+    for (int i = lane; i < kCalendar / 4; i += 32) reinterpret_cast<int4 *>(m.cal)[i] = make_int4(0, 0, 0, 0);
+    for (int i = lane; i < kCalendar / 32; i += 32) m.bm[i] = 0u;
+    __syncwarp();
+
+    // Copy the snapshot into library memory, validate it, total the prefill work
+    // and list the running decoders (decoding from batch 1).
     bool bad = false;
     long long f1 = 0, f4 = 0;
+    int fmin0 = kBig;
     for (int t = lane; t < c.capR; t += 32) {
         const int ctx = a.in.run_ctx[rrow + t];
         const int pre = a.in.run_pre[rrow + t];
@@ -161,68 +180,63 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             bad |= pre > 0 && t != nr - 1;
             f1 += pre;
             f4 += (long long)pre * ctx + ((long long)pre * (pre + 1)) / 2;
+            if (pre == 0 && !bad) {
+                m.ds[t] = 1;
+                m.df[t] = dec;
+                m.dcb[t] = ctx - 1;
+                if (dec < kCalendar) {
+                    atomicAdd(&m.cal[dec], 1);
+                    atomicOr(&m.bm[dec >> 5], 1u << (dec & 31));
+                } else {
+                    fmin0 = min(fmin0, dec);
+                }
+            }
         }
     }
-    for (int t = lane; t < c.capW; t += 32) {
-        const int pre = a.in.wait_pre[wrow + t];
-        const int dec = a.in.wait_dec[wrow + t];
-        out.wait_pre[wrow + t] = pre;
-        out.wait_dec[wrow + t] = dec;
-        m.wpre[t] = pre;
-        m.wdec[t] = dec;
-        if (t < nw) {
+    long long wsum = 0;
+    int carry = 0;
+    for (int base = 0; base < c.capW; base += 32) {
+        const int t = base + lane;
+        int pre = 0, dec = 0;
+        if (t < c.capW) {
+            pre = a.in.wait_pre[wrow + t];
+            dec = a.in.wait_dec[wrow + t];
+            out.wait_pre[wrow + t] = pre;
+            out.wait_dec[wrow + t] = dec;
+            m.wdec[t] = dec;
+        }
+        const bool live = t < nw;
+        if (live) {
             bad |= pre < 1 || pre > (1 << 24) || dec < 1 || dec > (1 << 24);
             f1 += pre;
             f4 += ((long long)pre * (pre + 1)) / 2;
+            wsum += pre;
         }
+        // exclusive prefix sums of the prompts (valid while the total stays below 2^30)
+        int x = live ? min(pre, 1 << 24) : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(kFull, x, o);
+            if (lane >= o) x += y;
+        }
+        const int incl = carry + x;
+        if (t < c.capW) m.P[t + 1] = incl;
+        carry = __shfl_sync(kFull, incl, 31);
     }
-    if (__any_sync(kFull, bad)) {
+    if (lane == 0) m.P[0] = 0;
+    wsum = warp_sum64(wsum);
+    if (__any_sync(kFull, bad) || wsum > (1LL << 30)) {
         fail(a.ctl, kEState, lane);
         return;
     }
     f1 = warp_sum64(f1);
     f4 = warp_sum64(f4);
-
-    // Decoder slots: running request t (decoding from batch 1) takes slot t.
-    for (int idx = lane; idx < c.slots; idx += 32) {
-        int s = kBig, f = kBig, cb = 0;
-        if (idx < nr) {
-            const int pre = a.in.run_pre[rrow + idx];
-            if (pre == 0) {
-                s = 1;
-                f = a.in.run_dec[rrow + idx];
-                cb = a.in.run_ctx[rrow + idx] - 1;
-            }
-        }
-        m.s[idx] = s;
-        m.f[idx] = f;
-        m.cb[idx] = cb;
-    }
     __syncwarp();
-    Slots sl;
-    sl.m = m;
-    sl.lane = lane;
-    sl.nslots_cap = c.slots;
-    sl.f2d = 0;
-    sl.f3d = 0;
-    sl.top = 0;
-    sl.n = 0;
-    sl.overflow = false;
-    int mn = kBig;
-    for (int base = 0; base < c.slots; base += 32) {
-        const int idx = base + lane;
-        const int f = m.f[idx];
-        const bool fr = f == kBig;
-        const unsigned b = __ballot_sync(kFull, fr);
-        if (fr) m.freel[sl.top + __popc(b & lanemask_lt())] = idx;
-        sl.top += __popc(b);
-        sl.n += 32 - __popc(b);
-        if (!fr) mn = min(mn, f);
-    }
-    __syncwarp();
-    sl.fmin = __reduce_min_sync(kFull, mn);
 
-    // The request still in prefill, if any (always the last running one).
+    Sim sim;
+    sim.m = m;
+    sim.lane = lane;
+    // the request still in prefill, if any, is the last running one
     bool pf = false;
     int pfR = 0, pfC = 0, pfD = 0;
     if (nr > 0) {
@@ -234,57 +248,83 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             pfD = a.in.run_dec[rrow + nr - 1];
         }
     }
+    sim.nlist = nr - (pf ? 1 : 0);
+    sim.far_min = __reduce_min_sync(kFull, fmin0);
 
-    const int mode = c.mode;
+    int n = sim.nlist;  // decoders alive at the start of batch l
     int l = 1, head = 0, iters = 0;
+    int fnext = sim.next_end(1);
     bool found = false;
     int la = 0, r0 = 0;
     while (iters < c.max_iters && l < (1 << 30)) {
         ++iters;
-        int cnt = sl.n + (pf ? 1 : 0);  // requests running in batch l
+        int cnt = n + (pf ? 1 : 0);  // requests running in batch l
         if (!pf && cnt >= S) {
             // Every sequence slot is taken: nothing but decoding until one frees.
-            l = sl.fmin + 1;
-            sl.advance_to(l);
+            n -= sim.ends_at(fnext);
+            l = fnext + 1;
+            fnext = sim.next_end(l);
             continue;
         }
-        int budget = B - sl.n;  // every decoder takes one token first
+        int budget = B - n;  // every decoder takes one token first
+        int pend = 0;        // decoders that start in batch l + 1
         if (pf) {
             if (budget <= 0) break;  // excluded by the preconditions
             if (pfR > budget) {
                 // The prefill continues; skip the batches in which it cannot
                 // finish and the number of decoders stays the same.
-                const int m1 = (pfR - 1) / budget;
-                const int m2 = (sl.fmin == kBig) ? kBig : (sl.fmin + 1 - l);
-                const int step = min(m1, m2);
+                const int step = min((pfR - 1) / budget, fnext == kBig ? kBig : fnext + 1 - l);
                 pfR -= step * budget;
                 pfC += step * budget;
                 l += step;
-                sl.advance_to(l);
+                if (l - 1 == fnext) {
+                    n -= sim.ends_at(fnext);
+                    fnext = sim.next_end(l);
+                }
                 continue;
             }
             budget -= pfR;
             pfC += pfR;
-            pfR = 0;
             pf = false;
-            prefill_done(sl, mode, l, pfC, pfD);
+            int f, cb;
+            const bool dec = decoder_of(mode, l, pfC, pfD, &f, &cb);
+            const int fm = sim.append(dec && lane == 0, l + 1, f, cb);
+            fnext = min(fnext, fm);
+            pend += dec ? 1 : 0;
         }
-        // FCFS admission while budget and a sequence slot remain.
+        // FCFS admission, 32 waiting requests at a time, while budget and a
+        // sequence slot remain.
         while (budget > 0 && head < nw && cnt < S) {
-            const int p = m.wpre[head];
-            const int d = m.wdec[head];
-            ++head;
-            ++cnt;
-            if (p <= budget) {
-                budget -= p;
-                prefill_done(sl, mode, l, p, d);
-            } else {
+            const int idx = head + lane;
+            const bool inb = lane < S - cnt && idx < nw;
+            const int ph = m.P[head];
+            const int st = inb ? m.P[idx] - ph : kBig;
+            const int en = inb ? m.P[idx + 1] - ph : kBig;
+            const bool adm = inb && st < budget;
+            const bool full = adm && en <= budget;
+            const int na = __popc(__ballot_sync(kFull, adm));
+            const int d = inb ? m.wdec[idx] : 1;
+            int f, cb;
+            const bool dec = decoder_of(mode, l, en - st, d, &f, &cb) && full;
+            const int fm = sim.append(dec, l + 1, f, cb);
+            fnext = min(fnext, fm);
+            pend += __popc(__ballot_sync(kFull, dec));
+            const int last = na - 1;
+            const int st_l = __shfl_sync(kFull, st, last);
+            const int en_l = __shfl_sync(kFull, en, last);
+            const int d_l = __shfl_sync(kFull, d, last);
+            head += na;
+            cnt += na;
+            if (en_l > budget) {  // the last admitted request continues in later batches
                 pf = true;
-                pfR = p - budget;
-                pfC = budget;
-                pfD = d;
+                pfR = en_l - budget;
+                pfC = budget - st_l;
+                pfD = d_l;
                 budget = 0;
+            } else {
+                budget -= en_l;
             }
+            if (na < 32) break;
         }
         if (!pf && head == nw && budget > 0 && cnt < S) {
             found = true;
@@ -292,24 +332,30 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             r0 = budget;
             break;
         }
+        n += pend;
+        if (l == fnext) {
+            n -= sim.ends_at(l);
+            fnext = sim.next_end(l + 1);
+        }
         ++l;
-        sl.advance_to(l);
     }
     __syncwarp();
-    if (!found || sl.overflow) {
+    if (!found) {
         fail(a.ctl, kETraj, lane);
         return;
     }
 
-    // Budgets left to the query after its admission batch: cumulative sums until
-    // they cover the longest prompt.
+    // Budgets left to the query after its admission batch, and the residents'
+    // decode features up to each batch its first token can fall in.
+    const int off = (mode == 0) ? 1 : 0;
+    const int nl = sim.nlist;
     int kp = 1;
     long long rc = r0;
     if (lane == 0) m.rcum[0] = r0;
     while (rc < c.pmax && kp < c.kph) {
         const int lk = la + kp;
         int nd = 0;
-        for (int idx = lane; idx < c.slots; idx += 32) nd += (m.s[idx] <= lk && lk <= m.f[idx]) ? 1 : 0;
+        for (int i = lane; i < nl; i += 32) nd += (m.ds[i] <= lk && lk <= m.df[i]) ? 1 : 0;
         nd = __reduce_add_sync(kFull, nd);
         rc += B - nd;
         if (lane == 0) m.rcum[kp] = (int)min(rc, (long long)kBig - 1);
@@ -320,11 +366,6 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         fail(a.ctl, kETraj, lane);
         return;
     }
-
-    // Residents' decode features up to each batch the query's first token can fall in.
-    const int off = (mode == 0) ? 1 : 0;
-    const long long f2done = warp_sum64(sl.f2d);
-    const long long f3done = warp_sum64(sl.f3d);
     const int m_j = c.moi[j];
     const float b0 = c.coef[m_j * 5 + 0];
     const float b1d = c.coef[m_j * 5 + 2];
@@ -334,17 +375,17 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     for (int k = 0; k < kp; ++k) {
         const int L = la + k + off;
         long long a2 = 0, a3 = 0;
-        for (int idx = lane; idx < c.slots; idx += 32) {
-            const int s = m.s[idx];
+        for (int i = lane; i < nl; i += 32) {
+            const int s = m.ds[i];
             if (s <= L) {
-                const int e = min(m.f[idx], L);
+                const int e = min(m.df[i], L);
                 const long long cnt = (long long)e - s + 1;
                 a2 += cnt;
-                a3 += cnt * (long long)m.cb[idx] + (((long long)s + e) * cnt) / 2;
+                a3 += cnt * (long long)m.dcb[i] + (((long long)s + e) * cnt) / 2;
             }
         }
-        const long long F2 = f2done + warp_sum64(a2) + off;  // + the query's own first decode token
-        const long long F3 = f3done + warp_sum64(a3);
+        const long long F2 = warp_sum64(a2) + off;  // + the query's own first decode token
+        const long long F3 = warp_sum64(a3);
         fast = fast && (F3 + c.pmax < kFastLimit);
         if (lane == (k & 31)) {
             const float t = __fmaf_rn(b1d, __ll2float_rn(F2), __fmul_rn(b0, __int2float_rn(L)));
@@ -396,7 +437,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
 }
 
 __global__ void __launch_bounds__(kK1Warps * 32) k_trajectory(const K1Launch a) {
-    extern __shared__ int32_t k1_smem[];
+    extern __shared__ __align__(16) int32_t k1_smem[];
     const int lane = threadIdx.x & 31;
     const int wid = threadIdx.x >> 5;
     const int j = blockIdx.x * kK1Warps + wid;
