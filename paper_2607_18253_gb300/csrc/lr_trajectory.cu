@@ -21,16 +21,17 @@
 // token in every batch (decoders come first and number fewer than B_j), so
 // decode progress is lockstep: a request that starts decoding in batch s with
 // d tokens to go decodes in batches s..s+d-1 at context cb + l.  The warp
-// therefore never touches individual decoders while it steps:
+// never touches individual decoders while it steps:
 //
 //   * every decoder is appended once to a list (s, f, cb); its Eq. 9 decode
 //     features up to any batch L follow in closed form, summed over the list
-//     in parallel after the loop;
+//     by the whole warp after the loop;
 //   * a calendar counts decoders by last decode batch f (with a bitmap to find
 //     the next non-empty batch); decoders ending beyond the calendar are rare
 //     and handled by scanning the list;
-//   * waiting requests are admitted a batch-group at a time: 32 lanes test the
-//     next 32 requests against the budget with the prompts' prefix sums.
+//   * the step loop itself -- a chain of dependent scheduling decisions --
+//     runs on one lane as scalar code over shared memory (prompt prefix sums,
+//     calendar, list), with runs of batches that only decode skipped in one step.
 #include "lr_internal.cuh"
 
 namespace lr {
@@ -48,6 +49,7 @@ struct WarpSmem {
     int32_t *cal;    // [kCalendar] decoders by last decode batch
     uint32_t *bm;    // [kCalendar / 32] non-empty calendar batches
     int32_t *rcum;   // [kph] cumulative budgets
+    int32_t *scr;    // [32] scratch of the seat-limited step
 };
 
 __device__ __forceinline__ WarpSmem carve(int32_t *base, const DevConfig &c) {
@@ -60,6 +62,7 @@ __device__ __forceinline__ WarpSmem carve(int32_t *base, const DevConfig &c) {
     w.df = w.ds + (c.capR + c.capW);
     w.dcb = w.df + (c.capR + c.capW);
     w.rcum = w.dcb + (c.capR + c.capW);
+    w.scr = w.rcum + c.kph;
     return w;
 }
 
@@ -70,62 +73,56 @@ __device__ void fail(DevCtl *ctl, int code, int lane) {
     }
 }
 
-struct Sim {
-    WarpSmem m;
-    int lane;
-    int nlist;    // decoders in the list
-    int far_min;  // smallest last-decode batch >= kCalendar among live decoders (kBig if none)
-
-    // Smallest calendar batch >= L holding a decoder end.
-    __device__ int next_cal(int L) const {
-        for (int w0 = L >> 5; w0 < kCalendar / 32; w0 += 32) {
-            const int w = w0 + lane;
-            uint32_t word = (w < kCalendar / 32) ? m.bm[w] : 0u;
-            if (w == (L >> 5)) word &= ~0u << (L & 31);
-            const unsigned nz = __ballot_sync(kFull, word != 0u);
-            if (nz) {
-                const int src = __ffs(nz) - 1;
-                const uint32_t wv = __shfl_sync(kFull, word, src);
-                return (w0 + src) * 32 + __ffs(wv) - 1;
-            }
-        }
-        return kBig;
+__device__ __forceinline__ int warp_incl_sum(int x, int lane) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(kFull, x, o);
+        if (lane >= o) x += y;
     }
+    return x;
+}
 
-    __device__ int next_end(int L) const { return min(next_cal(L), far_min); }
+// Scalar view of one instance's trajectory state, used by a single lane: the
+// step loop is a chain of dependent decisions, so it runs as plain scalar
+// code over shared memory without warp-wide round trips.
+struct Track {
+    WarpSmem m;
+    int nlist;  // decoders in the list
+
+    // Smallest last-decode batch >= L of any decoder; ends beyond the calendar
+    // (always later than every calendar end) are found in the list.
+    __device__ int next_end(int L) const {
+        if (L < kCalendar) {
+            int w = L >> 5;
+            uint32_t word = m.bm[w] & (~0u << (L & 31));
+            while (word == 0u && ++w < kCalendar / 32) word = m.bm[w];
+            if (word != 0u) return (w << 5) + __ffs(word) - 1;
+        }
+        int mn = kBig;
+        for (int i = 0; i < nlist; ++i) {
+            const int f = m.df[i];
+            if (f >= L && f < mn) mn = f;
+        }
+        return mn;
+    }
 
     // Number of decoders whose last decode batch is fc.
-    __device__ int ends_at(int fc) {
-        int c = fc < kCalendar ? m.cal[fc] : 0;
-        if (fc == far_min) {
-            int eq = 0, mn = kBig;
-            for (int i = lane; i < nlist; i += 32) {
-                const int f = m.df[i];
-                eq += (f == fc) ? 1 : 0;
-                if (f >= kCalendar && f > fc) mn = min(mn, f);
-            }
-            c += __reduce_add_sync(kFull, eq);
-            far_min = __reduce_min_sync(kFull, mn);
-        }
-        return c;
+    __device__ int ends_at(int fc) const {
+        if (fc < kCalendar) return m.cal[fc];
+        int eq = 0;
+        for (int i = 0; i < nlist; ++i) eq += (m.df[i] == fc) ? 1 : 0;
+        return eq;
     }
 
-    // Append a decoder from the lanes with `mine` set; returns the smallest new end.
-    __device__ int append(bool mine, int s, int f, int cb) {
-        const unsigned bal = __ballot_sync(kFull, mine);
-        if (mine) {
-            const int pos = nlist + __popc(bal & lanemask_lt());
-            m.ds[pos] = s;
-            m.df[pos] = f;
-            m.dcb[pos] = cb;
-            if (f < kCalendar) {
-                atomicAdd(&m.cal[f], 1);
-                atomicOr(&m.bm[f >> 5], 1u << (f & 31));
-            }
+    __device__ void append(int s, int f, int cb) {
+        m.ds[nlist] = s;
+        m.df[nlist] = f;
+        m.dcb[nlist] = cb;
+        ++nlist;
+        if (f < kCalendar) {
+            m.cal[f] += 1;
+            m.bm[f >> 5] |= 1u << (f & 31);
         }
-        nlist += __popc(bal);
-        far_min = min(far_min, __reduce_min_sync(kFull, (mine && f >= kCalendar) ? f : kBig));
-        return __reduce_min_sync(kFull, mine ? f : kBig);
     }
 };
 
@@ -164,66 +161,81 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     __syncwarp();
 
     // Copy the snapshot into library memory, validate it, total the prefill work
-    // and list the running decoders (decoding from batch 1).
+    // and list the running decoders (decoding from batch 1).  Loads and stores
+    // go through non-aliasing row pointers so that loads of later elements can
+    // be issued ahead of earlier stores.
     bool bad = false;
-    long long f1 = 0, f4 = 0;
-    int fmin0 = kBig;
-    for (int t = lane; t < c.capR; t += 32) {
-        const int ctx = a.in.run_ctx[rrow + t];
-        const int pre = a.in.run_pre[rrow + t];
-        const int dec = a.in.run_dec[rrow + t];
-        out.run_ctx[rrow + t] = ctx;
-        out.run_pre[rrow + t] = pre;
-        out.run_dec[rrow + t] = dec;
-        if (t < nr) {
-            bad |= ctx < 0 || ctx > (1 << 28) || pre < 0 || pre > (1 << 24) || dec < 1 || dec > (1 << 24);
-            bad |= pre > 0 && t != nr - 1;
-            f1 += pre;
-            f4 += (long long)pre * ctx + ((long long)pre * (pre + 1)) / 2;
-            if (pre == 0 && !bad) {
-                m.ds[t] = 1;
-                m.df[t] = dec;
-                m.dcb[t] = ctx - 1;
-                if (dec < kCalendar) {
-                    atomicAdd(&m.cal[dec], 1);
-                    atomicOr(&m.bm[dec >> 5], 1u << (dec & 31));
-                } else {
-                    fmin0 = min(fmin0, dec);
+    long long f1 = 0, f4 = 0, wsum = 0;
+    int pf_pre = 0, pf_ctx = 0, pf_dec = 0;
+    {
+        const int32_t *__restrict__ ic = a.in.run_ctx + rrow;
+        const int32_t *__restrict__ ip = a.in.run_pre + rrow;
+        const int32_t *__restrict__ id = a.in.run_dec + rrow;
+        int32_t *__restrict__ oc = out.run_ctx + rrow;
+        int32_t *__restrict__ op = out.run_pre + rrow;
+        int32_t *__restrict__ od = out.run_dec + rrow;
+#pragma unroll 4
+        for (int t = lane; t < c.capR; t += 32) {
+            const int ctx = __ldg(ic + t);
+            const int pre = __ldg(ip + t);
+            const int dec = __ldg(id + t);
+            oc[t] = ctx;
+            op[t] = pre;
+            od[t] = dec;
+            if (t < nr) {
+                bad |= ctx < 0 || ctx > (1 << 28) || pre < 0 || pre > (1 << 24) || dec < 1 || dec > (1 << 24);
+                bad |= pre > 0 && t != nr - 1;
+                f1 += pre;
+                f4 += (long long)pre * ctx + ((long long)pre * (pre + 1)) / 2;
+                if (t == nr - 1) {
+                    pf_pre = pre;
+                    pf_ctx = ctx;
+                    pf_dec = dec;
+                }
+                if (pre == 0 && !bad) {
+                    m.ds[t] = 1;
+                    m.df[t] = dec;
+                    m.dcb[t] = ctx - 1;
+                    if (dec < kCalendar) {
+                        atomicAdd(&m.cal[dec], 1);
+                        atomicOr(&m.bm[dec >> 5], 1u << (dec & 31));
+                    }
                 }
             }
         }
-    }
-    long long wsum = 0;
-    int carry = 0;
-    for (int base = 0; base < c.capW; base += 32) {
-        const int t = base + lane;
-        int pre = 0, dec = 0;
-        if (t < c.capW) {
-            pre = a.in.wait_pre[wrow + t];
-            dec = a.in.wait_dec[wrow + t];
-            out.wait_pre[wrow + t] = pre;
-            out.wait_dec[wrow + t] = dec;
+        const int32_t *__restrict__ iwp = a.in.wait_pre + wrow;
+        const int32_t *__restrict__ iwd = a.in.wait_dec + wrow;
+        int32_t *__restrict__ owp = out.wait_pre + wrow;
+        int32_t *__restrict__ owd = out.wait_dec + wrow;
+#pragma unroll 4
+        for (int t = lane; t < c.capW; t += 32) {
+            const int pre = __ldg(iwp + t);
+            const int dec = __ldg(iwd + t);
+            owp[t] = pre;
+            owd[t] = dec;
             m.wdec[t] = dec;
+            const bool live = t < nw;
+            if (live) {
+                bad |= pre < 1 || pre > (1 << 24) || dec < 1 || dec > (1 << 24);
+                f1 += pre;
+                f4 += ((long long)pre * (pre + 1)) / 2;
+                wsum += pre;
+            }
+            m.P[t + 1] = live ? min(max(pre, 0), 1 << 24) : 0;
         }
-        const bool live = t < nw;
-        if (live) {
-            bad |= pre < 1 || pre > (1 << 24) || dec < 1 || dec > (1 << 24);
-            f1 += pre;
-            f4 += ((long long)pre * (pre + 1)) / 2;
-            wsum += pre;
-        }
-        // exclusive prefix sums of the prompts (valid while the total stays below 2^30)
-        int x = live ? min(pre, 1 << 24) : 0;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(kFull, x, o);
-            if (lane >= o) x += y;
-        }
-        const int incl = carry + x;
-        if (t < c.capW) m.P[t + 1] = incl;
-        carry = __shfl_sync(kFull, incl, 31);
     }
-    if (lane == 0) m.P[0] = 0;
+    __syncwarp();
+    // exclusive prefix sums of the prompts, in place (valid while the total stays below 2^30)
+    {
+        int carry = 0;
+        for (int base = 0; base < c.capW; base += 32) {
+            const int t = base + lane;
+            const int incl = carry + warp_incl_sum(t < c.capW ? m.P[t + 1] : 0, lane);
+            if (t < c.capW) m.P[t + 1] = incl;
+            carry = __shfl_sync(kFull, incl, 31);
+        }
+        if (lane == 0) m.P[0] = 0;
+    }
     wsum = warp_sum64(wsum);
     if (__any_sync(kFull, bad) || wsum > (1LL << 30)) {
         fail(a.ctl, kEState, lane);
@@ -233,120 +245,121 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     f4 = warp_sum64(f4);
     __syncwarp();
 
-    Sim sim;
-    sim.m = m;
-    sim.lane = lane;
     // the request still in prefill, if any, is the last running one
-    bool pf = false;
     int pfR = 0, pfC = 0, pfD = 0;
     if (nr > 0) {
-        const int pre = a.in.run_pre[rrow + nr - 1];
-        if (pre > 0) {
-            pf = true;
-            pfR = pre;
-            pfC = a.in.run_ctx[rrow + nr - 1];
-            pfD = a.in.run_dec[rrow + nr - 1];
-        }
+        const int src = (nr - 1) & 31;
+        pfR = __shfl_sync(kFull, pf_pre, src);
+        pfC = __shfl_sync(kFull, pf_ctx, src);
+        pfD = __shfl_sync(kFull, pf_dec, src);
     }
-    sim.nlist = nr - (pf ? 1 : 0);
-    sim.far_min = __reduce_min_sync(kFull, fmin0);
+    const int n0 = nr - (pfR > 0 ? 1 : 0);
 
-    int n = sim.nlist;  // decoders alive at the start of batch l
-    int l = 1, head = 0, iters = 0;
-    int fnext = sim.next_end(1);
-    bool found = false;
-    int la = 0, r0 = 0;
-    while (iters < c.max_iters && l < (1 << 30)) {
-        ++iters;
-        int cnt = n + (pf ? 1 : 0);  // requests running in batch l
-        if (!pf && cnt >= S) {
-            // Every sequence slot is taken: nothing but decoding until one frees.
-            n -= sim.ends_at(fnext);
-            l = fnext + 1;
-            fnext = sim.next_end(l);
-            continue;
-        }
-        int budget = B - n;  // every decoder takes one token first
-        int pend = 0;        // decoders that start in batch l + 1
-        if (pf) {
-            if (budget <= 0) break;  // excluded by the preconditions
-            if (pfR > budget) {
-                // The prefill continues; skip the batches in which it cannot
-                // finish and the number of decoders stays the same.
-                const int step = min((pfR - 1) / budget, fnext == kBig ? kBig : fnext + 1 - l);
-                pfR -= step * budget;
-                pfC += step * budget;
-                l += step;
-                if (l - 1 == fnext) {
-                    n -= sim.ends_at(fnext);
-                    fnext = sim.next_end(l);
-                }
+    // Step the scheduler on lane 0 until a query appended now would be admitted.
+    if (lane == 0) {
+        Track tr;
+        tr.m = m;
+        tr.nlist = n0;
+        bool pf = pfR > 0;
+        int n = n0;  // decoders alive at the start of batch l
+        int l = 1, head = 0, iters = 0;
+        int ph = 0;  // prompt prefix sum at the waiting head
+        int fnext = tr.next_end(1);
+        int la = 0, r0 = 0;
+        while (iters < c.max_iters && l < (1 << 30)) {
+            ++iters;
+            int cnt = n + (pf ? 1 : 0);  // requests running in batch l
+            if (!pf && cnt >= S) {
+                // Every sequence slot is taken: nothing but decoding until one frees.
+                n -= tr.ends_at(fnext);
+                l = fnext + 1;
+                fnext = tr.next_end(l);
                 continue;
             }
-            budget -= pfR;
-            pfC += pfR;
-            pf = false;
-            int f, cb;
-            const bool dec = decoder_of(mode, l, pfC, pfD, &f, &cb);
-            const int fm = sim.append(dec && lane == 0, l + 1, f, cb);
-            fnext = min(fnext, fm);
-            pend += dec ? 1 : 0;
-        }
-        // FCFS admission, 32 waiting requests at a time, while budget and a
-        // sequence slot remain.
-        while (budget > 0 && head < nw && cnt < S) {
-            const int idx = head + lane;
-            const bool inb = lane < S - cnt && idx < nw;
-            const int ph = m.P[head];
-            const int st = inb ? m.P[idx] - ph : kBig;
-            const int en = inb ? m.P[idx + 1] - ph : kBig;
-            const bool adm = inb && st < budget;
-            const bool full = adm && en <= budget;
-            const int na = __popc(__ballot_sync(kFull, adm));
-            const int d = inb ? m.wdec[idx] : 1;
-            int f, cb;
-            const bool dec = decoder_of(mode, l, en - st, d, &f, &cb) && full;
-            const int fm = sim.append(dec, l + 1, f, cb);
-            fnext = min(fnext, fm);
-            pend += __popc(__ballot_sync(kFull, dec));
-            const int last = na - 1;
-            const int st_l = __shfl_sync(kFull, st, last);
-            const int en_l = __shfl_sync(kFull, en, last);
-            const int d_l = __shfl_sync(kFull, d, last);
-            head += na;
-            cnt += na;
-            if (en_l > budget) {  // the last admitted request continues in later batches
-                pf = true;
-                pfR = en_l - budget;
-                pfC = budget - st_l;
-                pfD = d_l;
-                budget = 0;
-            } else {
-                budget -= en_l;
+            int budget = B - n;  // every decoder takes one token first
+            int pend = 0;        // decoders that start in batch l + 1
+            if (pf) {
+                if (budget <= 0) break;  // excluded by the preconditions
+                if (pfR > budget) {
+                    // The prefill continues; skip the batches in which it cannot
+                    // finish and the number of decoders stays the same.
+                    const int step = min((pfR - 1) / budget, fnext == kBig ? kBig : fnext + 1 - l);
+                    pfR -= step * budget;
+                    pfC += step * budget;
+                    l += step;
+                    if (l - 1 == fnext) {
+                        n -= tr.ends_at(fnext);
+                        fnext = tr.next_end(l);
+                    }
+                    continue;
+                }
+                budget -= pfR;
+                pfC += pfR;
+                pf = false;
+                int f, cb;
+                if (decoder_of(mode, l, pfC, pfD, &f, &cb)) {
+                    tr.append(l + 1, f, cb);
+                    ++pend;
+                    fnext = min(fnext, f);
+                }
             }
-            if (na < 32) break;
+            // FCFS admission while budget and a sequence slot remain.
+            while (budget > 0 && head < nw && cnt < S) {
+                const int pn = m.P[head + 1];
+                const int d = m.wdec[head];
+                const int p = pn - ph;
+                ++head;
+                ph = pn;
+                ++cnt;
+                if (p <= budget) {
+                    budget -= p;
+                    int f, cb;
+                    if (decoder_of(mode, l, p, d, &f, &cb)) {
+                        tr.append(l + 1, f, cb);
+                        ++pend;
+                        fnext = min(fnext, f);
+                    }
+                } else {  // the prompt continues in later batches
+                    pf = true;
+                    pfR = p - budget;
+                    pfC = budget;
+                    pfD = d;
+                    budget = 0;
+                }
+            }
+            if (!pf && head == nw && budget > 0 && cnt < S) {
+                la = l;
+                r0 = budget;
+                break;
+            }
+            n += pend;
+            if (l == fnext) {
+                n -= tr.ends_at(l);
+                fnext = tr.next_end(l + 1);
+            }
+            ++l;
         }
-        if (!pf && head == nw && budget > 0 && cnt < S) {
-            found = true;
-            la = l;
-            r0 = budget;
-            break;
-        }
-        n += pend;
-        if (l == fnext) {
-            n -= sim.ends_at(l);
-            fnext = sim.next_end(l + 1);
-        }
-        ++l;
+        m.scr[0] = la;
+        m.scr[1] = r0;
+        m.scr[2] = tr.nlist;
+        m.scr[3] = iters;
     }
     __syncwarp();
-    if (!found) {
+    const int la = m.scr[0];
+    const int r0 = m.scr[1];
+    const int iters = m.scr[3];  // simulation steps taken
+    (void)iters;
+    if (la == 0) {
         fail(a.ctl, kETraj, lane);
         return;
     }
+    struct {
+        int nlist;
+    } sim = {m.scr[2]};
 
     // Budgets left to the query after its admission batch, and the residents'
-    // decode features up to each batch its first token can fall in.
+    // decode features up to each batch its first token can fall in (one
+    // parallel pass over the decoder list per batch).
     const int off = (mode == 0) ? 1 : 0;
     const int nl = sim.nlist;
     int kp = 1;
