@@ -62,6 +62,9 @@ def _load():
         lib.orc_route.restype = ctypes.c_int
         lib.orc_frontier.argtypes = [i32, i32, i32, P, P, P, P, P, P, i32, P, P, P]
         lib.orc_frontier.restype = ctypes.c_int
+        lib.orc_advance.argtypes = [i32, P, P, P, P, i32, i32, P, P, P, P, P, P, P, P, i32, P, P, P, i32,
+                                    ctypes.c_double, i64]
+        lib.orc_advance.restype = ctypes.c_int
         lib.orc_utility.argtypes = [ctypes.c_float, ctypes.c_float, i32, i32, ctypes.c_float, ctypes.c_float]
         lib.orc_utility.restype = ctypes.c_float
         _lib = lib
@@ -183,3 +186,25 @@ def frontier(wl, assign: np.ndarray, ttft_chosen: np.ndarray) -> np.ndarray:
     if rc != 0:
         raise RuntimeError(f"oracle frontier failed with code {rc}")
     return out
+
+
+def advance(wl, clock, assign, prompt_len, dec, t_now: float, max_batches: int = 1 << 30):
+    """Online stream step on a copy of the workload's state.
+
+    Returns (new workload with the advanced state, new clocks)."""
+    import dataclasses
+    st = {k: np.array(getattr(wl, k), dtype=np.int32, copy=True)
+          for k in ("n_run", "run_ctx", "run_pre", "run_dec", "n_wait", "wait_pre", "wait_dec")}
+    clk = np.array(clock, dtype=np.float64, copy=True)
+    a = _c(assign, np.int32)
+    p = _c(prompt_len, np.int32)
+    d = _c(dec, np.int32)
+    moi, B, S = (_c(x, np.int32) for x in (wl.model_of_instance, wl.max_batched_tokens, wl.max_seqs))
+    coef = _c(wl.coef, np.float32)
+    rc = _load().orc_advance(wl.num_instances, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running, wl.cap_waiting,
+                             _p(st["n_run"]), _p(st["run_ctx"]), _p(st["run_pre"]), _p(st["run_dec"]),
+                             _p(st["n_wait"]), _p(st["wait_pre"]), _p(st["wait_dec"]), _p(clk), int(a.shape[0]),
+                             _p(a), _p(p), _p(d), wl.first_token_mode, float(t_now), int(max_batches))
+    if rc != 0:
+        raise RuntimeError(f"oracle advance failed with code {rc}")
+    return dataclasses.replace(wl, **st), clk

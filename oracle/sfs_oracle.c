@@ -282,3 +282,125 @@ int orc_frontier(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instan
     }
     return ORC_OK;
 }
+
+/*
+ * Online stream step.  The engine behind each instance keeps executing token
+ * batches (Sec. 2, continuous batching) and publishes its state after each one
+ * (App. F); the router sees the state after the last batch completed by the
+ * current time.  Batch times follow Eq. 9 for the batch actually executed.
+ */
+int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, const int32_t *B,
+                const int32_t *S, int32_t cap_running, int32_t cap_waiting, int32_t *n_run,
+                int32_t *run_ctx, int32_t *run_pre, int32_t *run_dec, int32_t *n_wait, int32_t *wait_pre,
+                int32_t *wait_dec, double *clock, int32_t Q, const int32_t *assign,
+                const int32_t *prompt_len, const int32_t *dec, int32_t mode, double t_now,
+                int64_t max_batches)
+{
+    int rc_all = ORC_OK;
+    for (int32_t j = 0; j < I; ++j) {
+        const int64_t total = (int64_t)cap_running + cap_waiting + Q + 1;
+        orc_req *run = (orc_req *)calloc((size_t)total, sizeof(orc_req));
+        orc_req *wait = (orc_req *)calloc((size_t)total, sizeof(orc_req));
+        int64_t *alloc = (int64_t *)calloc((size_t)total, sizeof(int64_t));
+        int *kind = (int *)calloc((size_t)total, sizeof(int));
+        if (!run || !wait || !alloc || !kind) {
+            free(run); free(wait); free(alloc); free(kind);
+            return ORC_ENOMEM;
+        }
+        int64_t nr = 0, nw = 0, wh = 0;
+        for (int32_t r = 0; r < n_run[j]; ++r) {
+            const int64_t o = (int64_t)j * cap_running + r;
+            run[nr].ctx = run_ctx[o]; run[nr].pre = run_pre[o]; run[nr].dec = run_dec[o]; run[nr].is_query = 0;
+            ++nr;
+        }
+        for (int32_t w = 0; w < n_wait[j]; ++w) {
+            const int64_t o = (int64_t)j * cap_waiting + w;
+            wait[nw].ctx = 0; wait[nw].pre = wait_pre[o]; wait[nw].dec = wait_dec[o]; wait[nw].is_query = 0;
+            ++nw;
+        }
+        /* 1. the routed queries join the waiting tail in query order */
+        for (int32_t i = 0; i < Q; ++i) {
+            if (assign[i] != j) continue;
+            wait[nw].ctx = 0; wait[nw].pre = prompt_len[i]; wait[nw].dec = dec[i]; wait[nw].is_query = 0;
+            ++nw;
+        }
+        int rc = (nw > cap_waiting) ? ORC_ELIMIT : ORC_OK;
+        const float *cf = coef + 5 * model_of_instance[j];
+        double t = clock[j];
+        /* 2. execute whole batches that end by t_now */
+        for (int64_t step = 0; rc == ORC_OK; ++step) {
+            if (nr == 0 && wh == nw) { t = t_now; break; }   /* idle: nothing to run */
+            if (step >= max_batches) { rc = ORC_ELIMIT; break; }
+            /* plan the batch with the scheduler step (running list, then FCFS admission) */
+            int64_t budget = B[j];
+            for (int64_t r = 0; r < nr; ++r) { kind[r] = SCHED_NONE; alloc[r] = 0; }
+            for (int64_t r = 0; r < nr && budget > 0; ++r) {
+                if (run[r].pre > 0) { alloc[r] = min64(run[r].pre, budget); kind[r] = SCHED_PREFILL; }
+                else { alloc[r] = 1; kind[r] = SCHED_DECODE; }
+                budget -= alloc[r];
+            }
+            int64_t na = 0;
+            int64_t wbud = budget;
+            while (wbud > 0 && wh + na < nw && nr + na < S[j]) {
+                alloc[nr + na] = min64(wait[wh + na].pre, wbud);
+                kind[nr + na] = SCHED_PREFILL;
+                wbud -= alloc[nr + na];
+                ++na;
+            }
+            int64_t F[5] = {1, 0, 0, 0, 0};
+            for (int64_t r = 0; r < nr + na; ++r) {
+                const orc_req *q = (r < nr) ? &run[r] : &wait[wh + r - nr];
+                if (kind[r] == SCHED_PREFILL) {
+                    const int64_t x = alloc[r];
+                    F[1] += x;
+                    F[4] += x * q->ctx + x * (x + 1) / 2;
+                } else if (kind[r] == SCHED_DECODE) {
+                    F[2] += 1;
+                    F[3] += q->ctx;
+                }
+            }
+            const float T = orc_ttft_f32(cf, F);   /* Eq. 9 for this one batch */
+            if (t + (double)T > t_now) break;       /* still running at t_now */
+            /* apply the batch */
+            for (int64_t k = 0; k < na; ++k) run[nr + k] = wait[wh + k];
+            nr += na;
+            wh += na;
+            if (nr > cap_running) { rc = ORC_ELIMIT; break; }
+            for (int64_t r = 0; r < nr; ++r) {
+                if (kind[r] == SCHED_PREFILL) {
+                    run[r].ctx += alloc[r];
+                    run[r].pre -= alloc[r];
+                    if (run[r].pre == 0 && mode == ORC_FIRST_TOKEN_WITH_LAST_CHUNK) run[r].dec -= 1;
+                } else if (kind[r] == SCHED_DECODE) {
+                    run[r].ctx += 1;
+                    run[r].dec -= 1;
+                }
+            }
+            int64_t keep = 0;
+            for (int64_t r = 0; r < nr; ++r)
+                if (run[r].dec > 0) run[keep++] = run[r];
+            nr = keep;
+            t += (double)T;
+        }
+        if (rc == ORC_OK) {
+            n_run[j] = (int32_t)nr;
+            for (int64_t r = 0; r < cap_running; ++r) {
+                const int64_t o = (int64_t)j * cap_running + r;
+                run_ctx[o] = r < nr ? (int32_t)run[r].ctx : 0;
+                run_pre[o] = r < nr ? (int32_t)run[r].pre : 0;
+                run_dec[o] = r < nr ? (int32_t)run[r].dec : 0;
+            }
+            n_wait[j] = (int32_t)(nw - wh);
+            for (int64_t w = 0; w < cap_waiting; ++w) {
+                const int64_t o = (int64_t)j * cap_waiting + w;
+                wait_pre[o] = w < nw - wh ? (int32_t)wait[wh + w].pre : 0;
+                wait_dec[o] = w < nw - wh ? (int32_t)wait[wh + w].dec : 0;
+            }
+            clock[j] = t;
+        } else {
+            rc_all = rc;
+        }
+        free(run); free(wait); free(alloc); free(kind);
+    }
+    return rc_all;
+}

@@ -73,6 +73,19 @@ int orc_frontier(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instan
                  const int32_t *dec_hat, const float *acc, int32_t P, const int32_t *assign,
                  const float *ttft_chosen, double *out);
 
+/* Online stream step: append the routed queries (assign[i] >= 0) to their instances'
+ * waiting queues in query order, then advance every instance by the whole token batches
+ * that end by t_now, each taking the Eq. 9 time of its own composition (canonical fp32,
+ * accumulated in fp64 clocks).  An instance with nothing to run jumps to t_now.  State
+ * arrays ([I][cap] row-major) and clocks are updated in place.  Returns ORC_ELIMIT if a
+ * queue would exceed its capacity or an instance needs more than max_batches batches. */
+int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, const int32_t *B,
+                const int32_t *S, int32_t cap_running, int32_t cap_waiting, int32_t *n_run,
+                int32_t *run_ctx, int32_t *run_pre, int32_t *run_dec, int32_t *n_wait, int32_t *wait_pre,
+                int32_t *wait_dec, double *clock, int32_t Q, const int32_t *assign,
+                const int32_t *prompt_len, const int32_t *dec, int32_t mode, double t_now,
+                int64_t max_batches);
+
 /* Utility of Eq. 2 with the cost of App. B.4 in canonical fp32. */
 float orc_utility(float acc, float lambda, int32_t p, int32_t dec_hat, float price_in, float price_out);
 

@@ -161,12 +161,14 @@ def _round_up(x: int, m: int) -> int:
 
 def make_workload(name: str, num_queries: Optional[int] = None, seed: Optional[int] = None,
                   lam: Optional[np.ndarray] = None, mu: Optional[np.ndarray] = None,
-                  first_token_mode: int = FIRST_TOKEN_SEPARATE_DECODE) -> Workload:
+                  first_token_mode: int = FIRST_TOKEN_SEPARATE_DECODE, cap_running: Optional[int] = None,
+                  cap_waiting: Optional[int] = None) -> Workload:
     """Build one of the named workloads ("tiny", "pool64", "pool256").
 
     The instance state and the queries come from independent child streams of
     the seed, so changing the query count leaves the state unchanged and keeps
-    the query prefix unchanged.
+    the query prefix unchanged.  Larger capacities (row strides) only pad the
+    state arrays; the drawn values do not change.
     """
     r = RECIPES[name]
     seed = r["seed"] if seed is None else seed
@@ -180,15 +182,23 @@ def make_workload(name: str, num_queries: Optional[int] = None, seed: Optional[i
     coef = coefficients(alpha, beta, gamma)
     price_tok = (price * 1e-6).astype(np.float32)
 
-    capR = _round_up(r["run_max"], 32)
-    capW = _round_up(r["wait_max"], 32)
+    dR = _round_up(r["run_max"], 32)
+    dW = _round_up(r["wait_max"], 32)
+    capR = max(dR, int(cap_running or 0))
+    capW = max(dW, int(cap_waiting or 0))
     n_run = g_state.integers(0, r["run_max"] + 1, I).astype(np.int32)
     n_wait = g_state.integers(0, r["wait_max"] + 1, I).astype(np.int32)
-    run_ctx = g_state.integers(128, 2048 + 1, (I, capR)).astype(np.int32)
-    run_dec = _lognormal_int(g_state, 128, 2048, (I, capR))
+
+    def pad(a, cap):
+        out = np.zeros((I, cap), np.int32)
+        out[:, :a.shape[1]] = a
+        return out
+
+    run_ctx = pad(g_state.integers(128, 2048 + 1, (I, dR)).astype(np.int32), capR)
+    run_dec = pad(_lognormal_int(g_state, 128, 2048, (I, dR)), capR)
     run_pre = np.zeros((I, capR), np.int32)
-    wait_pre = _lognormal_int(g_state, r["p_median"], r["p_cap"], (I, capW))
-    wait_dec = _lognormal_int(g_state, 256, 2048, (I, capW))
+    wait_pre = pad(_lognormal_int(g_state, r["p_median"], r["p_cap"], (I, dW)), capW)
+    wait_dec = pad(_lognormal_int(g_state, 256, 2048, (I, dW)), capW)
     # zero the padding beyond each row's count
     cols_r = np.arange(capR)[None, :]
     cols_w = np.arange(capW)[None, :]
@@ -227,7 +237,8 @@ def sweep_pairs():
 
 def random_small_state(rng: np.random.Generator, num_instances: int, cap_running: int, cap_waiting: int,
                        budget_range=(4, 64), with_tail_prefill: bool = True,
-                       max_ctx: int = 300, max_pre: int = 200, max_dec: int = 40, min_gap: int = 1):
+                       max_ctx: int = 300, max_pre: int = 200, max_dec: int = 40, min_gap: int = 1,
+                       wait_max: Optional[int] = None):
     """Small random pools for property tests.
 
     Returns per-instance budget B, cap S (1 <= S <= B - min_gap + 1), and a
@@ -239,7 +250,7 @@ def random_small_state(rng: np.random.Generator, num_instances: int, cap_running
     S = np.array([rng.integers(1, b - min_gap + 2) for b in B], np.int32)
     S = np.minimum(S, cap_running).astype(np.int32)
     n_run = np.array([rng.integers(0, s + 1) for s in S], np.int32)
-    n_wait = rng.integers(0, cap_waiting + 1, I).astype(np.int32)
+    n_wait = rng.integers(0, (cap_waiting if wait_max is None else wait_max) + 1, I).astype(np.int32)
     run_ctx = np.zeros((I, cap_running), np.int32)
     run_pre = np.zeros((I, cap_running), np.int32)
     run_dec = np.zeros((I, cap_running), np.int32)
@@ -260,12 +271,12 @@ def random_small_state(rng: np.random.Generator, num_instances: int, cap_running
 def small_workload(seed: int, num_instances: int = 6, num_models: int = 3, num_queries: int = 24,
                    cap_running: int = 8, cap_waiting: int = 8, max_prompt_len: int = 160,
                    first_token_mode: int = FIRST_TOKEN_SEPARATE_DECODE, budget_range=(4, 64),
-                   with_tail_prefill: bool = True, min_gap: int = 1) -> Workload:
+                   with_tail_prefill: bool = True, min_gap: int = 1, wait_max: Optional[int] = None) -> Workload:
     """A random small pool (for property and parity tests on tiny inputs)."""
     rng = np.random.default_rng(seed)
     B, S, n_run, run_ctx, run_pre, run_dec, n_wait, wait_pre, wait_dec = random_small_state(
         rng, num_instances, cap_running, cap_waiting, budget_range=budget_range,
-        with_tail_prefill=with_tail_prefill, min_gap=min_gap)
+        with_tail_prefill=with_tail_prefill, min_gap=min_gap, wait_max=wait_max)
     alpha = rng.uniform(1.0, 10.0, num_models)
     beta = rng.uniform(0.01, 0.2, num_models)
     gamma = beta + rng.uniform(0.05, 0.5, num_models)
