@@ -158,6 +158,28 @@ LR_API int lr_route(lr_ctx *ctx, int32_t Q, const int32_t *prompt_len, const int
              float *util_out, float *ttft_chosen_out, double *frontier_out, float *ttft_matrix_out,
              void *cuda_stream);
 
+/* Online stream step (Sec. 5: queries arrive over time and are routed as they come;
+ * App. F: every instance keeps executing token batches and publishes its state after each).
+ * The queries with assign[i] >= 0 join instance assign[i]'s waiting tail in query order
+ * (prompt_len[i] prompt tokens, dec[i] output tokens, both in [1, 2^24]); then every
+ * instance executes the whole token batches -- the scheduler step the estimator simulates --
+ * that end by t_now (seconds), each taking the Eq. 9 time of its own composition, evaluated
+ * in fp32 and accumulated into a per-instance fp64 clock (an instance with nothing to run
+ * jumps to t_now; no clock ever runs backwards).  Entries of assign outside [0, I), e.g. -1
+ * for a query routed elsewhere, are skipped.  The advanced snapshot is then summarized and published as by
+ * lr_load_state; clocks start at 0 when a snapshot is loaded.  assign, prompt_len, dec:
+ * [Q] device arrays (Q may be 0).  Requires cap_running >= every max_seqs (LR_ECAPACITY
+ * otherwise).  A waiting queue that would exceed cap_waiting records LR_ECAPACITY, an
+ * out-of-range length LR_EINVAL; either leaves the previous snapshot live. */
+LR_API int lr_advance(lr_ctx *ctx, int32_t Q, const int32_t *assign, const int32_t *prompt_len,
+                      const int32_t *dec, double t_now, void *cuda_stream);
+
+/* Copy the live snapshot (as advanced so far) into caller arrays: device pointers with the
+ * shapes of lr_state_view plus clock [I] fp64; any pointer may be NULL to skip it. */
+LR_API int lr_read_state(const lr_ctx *ctx, int32_t *n_run, int32_t *run_ctx, int32_t *run_pre,
+                         int32_t *run_dec, int32_t *n_wait, int32_t *wait_pre, int32_t *wait_dec,
+                         double *clock, void *cuda_stream);
+
 /* Synchronize `cuda_stream`, return the first device-side error code recorded since
  * the last call (LR_OK if none) and clear it. */
 LR_API int lr_status(lr_ctx *ctx, void *cuda_stream);

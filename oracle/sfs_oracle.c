@@ -329,7 +329,10 @@ int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, 
         double t = clock[j];
         /* 2. execute whole batches that end by t_now */
         for (int64_t step = 0; rc == ORC_OK; ++step) {
-            if (nr == 0 && wh == nw) { t = t_now; break; }   /* idle: nothing to run */
+            if (nr == 0 && wh == nw) {                        /* idle: nothing to run */
+                if (t < t_now) t = t_now;                     /* a clock never runs backwards */
+                break;
+            }
             if (step >= max_batches) { rc = ORC_ELIMIT; break; }
             /* plan the batch with the scheduler step (running list, then FCFS admission) */
             int64_t budget = B[j];

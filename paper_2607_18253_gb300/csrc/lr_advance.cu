@@ -1,0 +1,306 @@
+// K3: online stream step (Sec. 5: queries arrive by a Poisson process and are
+// routed as they come; App. F: every instance keeps executing token batches
+// and publishes its state after each one).
+//
+// One warp per instance: the queries routed to it join its waiting tail in
+// query order (a stable ballot compaction over the assignment vector), then
+// the instance executes whole token batches -- the same scheduler step the
+// estimator simulates -- as long as each ends by t_now.  Each batch takes the
+// Eq. 9 time of its own composition, evaluated in the same fp32 order as the
+// estimate and accumulated into an fp64 clock.  An instance with nothing to
+// run jumps to t_now.  The advanced snapshot goes to a scratch buffer, which
+// K1 then summarizes and publishes like any snapshot.
+//
+// Unlike K1 this kernel does not rely on decode being lockstep: every batch
+// serves the running list in order with a prefix sum of the token needs, so
+// any list (including prefills ahead of decoders) advances exactly.
+#include "lr_internal.cuh"
+
+namespace lr {
+
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+
+__device__ __forceinline__ long long warp_incl_sum64(long long x, int lane) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const long long y = __shfl_up_sync(kFull, x, o);
+        if (lane >= o) x += y;
+    }
+    return x;
+}
+
+__device__ void fail3(DevCtl *ctl, int code, int lane) {
+    if (lane == 0) {
+        atomicCAS(&ctl->load_err, 0, code);
+        record_status(ctl, code);
+    }
+}
+
+__device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, int lane, int32_t *wbase) {
+    const DevConfig &c = a.cfg;
+    const StateBuf &dst = a.scratch;
+    const int B = c.B[j];
+    const int S = c.S[j];
+    const int capR = c.capR, capW = c.capW;
+    int32_t *rc0 = wbase, *rp0 = rc0 + capR, *rd0 = rp0 + capR;
+    int32_t *rc1 = rd0 + capR, *rp1 = rc1 + capR, *rd1 = rp1 + capR;
+    int32_t *wp = rd1 + capR, *wd = wp + capW;
+    const size_t rrow = (size_t)j * capR, wrow = (size_t)j * capW;
+    int nr = src.n_run[j];
+    int nw = src.n_wait[j];
+    for (int t = lane; t < nr; t += 32) {
+        rc0[t] = src.run_ctx[rrow + t];
+        rp0[t] = src.run_pre[rrow + t];
+        rd0[t] = src.run_dec[rrow + t];
+    }
+    for (int t = lane; t < nw; t += 32) {
+        wp[t] = src.wait_pre[wrow + t];
+        wd[t] = src.wait_dec[wrow + t];
+    }
+    // routed queries join the waiting tail in query order
+    for (int base = 0; base < a.Q; base += 32) {
+        const int i = base + lane;
+        const bool mine = i < a.Q && a.assign[i] == j;
+        const unsigned bal = __ballot_sync(kFull, mine);
+        if (mine) {
+            const int pos = nw + __popc(bal & lanemask_lt());
+            if (pos < capW) {
+                wp[pos] = a.prompt[i];
+                wd[pos] = a.dec[i];
+            }
+        }
+        nw += __popc(bal);
+    }
+    const bool over = nw > capW;
+    bool bad = false;
+    for (int t = lane; t < min(nw, capW); t += 32)
+        bad |= wp[t] < 1 || wp[t] > (1 << 24) || wd[t] < 1 || wd[t] > (1 << 24);
+    if (over) {
+        fail3(a.ctl, kECapacity, lane);
+        return;
+    }
+    if (__any_sync(kFull, bad)) {
+        fail3(a.ctl, kEInval, lane);
+        return;
+    }
+    __syncwarp();
+
+    const float *cf = c.coef + 5 * c.moi[j];
+    const float b0 = cf[0], b1p = cf[1], b1d = cf[2], b2 = cf[3], b3 = cf[4];
+    double t = src.clock[j];
+    int wh = 0, iters = 0;
+    bool ok = true;
+    int32_t *rc = rc0, *rp = rp0, *rd = rd0, *nc = rc1, *np = rp1, *nd = rd1;
+    while (true) {
+        if (nr == 0 && wh == nw) {  // nothing to run: idle until t_now (never backwards)
+            t = fmax(t, a.t_now);
+            break;
+        }
+        if (++iters > c.max_iters) {
+            ok = false;
+            break;
+        }
+        // Plan the batch: the running list in order, each request taking
+        // min(need, budget left) where need is its remaining prompt or one
+        // decode token; then FCFS admission while budget and a slot remain.
+        long long used = 0;  // tokens given to the running list so far
+        long long f1 = 0, f2 = 0, f3 = 0, f4 = 0;
+        for (int base = 0; base < nr; base += 32) {
+            const int r = base + lane;
+            const bool live = r < nr;
+            const int need = live ? (rp[r] > 0 ? rp[r] : 1) : 0;
+            const long long incl = used + warp_incl_sum64(need, lane);
+            const long long excl = incl - need;
+            const long long x = live ? max(0LL, min((long long)need, (long long)B - excl)) : 0;
+            if (live && x > 0) {
+                if (rp[r] > 0) {
+                    f1 += x;
+                    f4 += x * rc[r] + x * (x + 1) / 2;
+                } else {
+                    f2 += 1;
+                    f3 += rc[r];
+                }
+            }
+            used = __shfl_sync(kFull, incl, 31);
+        }
+        const long long budget = max(0LL, (long long)B - used);
+        // admissions: the k-th waiting request is admitted if its prompt starts
+        // inside the budget and a sequence slot is free
+        int na = 0;
+        long long wused = 0;
+        for (int base = 0; budget - wused > 0 && wh + base < nw && nr + base < S; base += 32) {
+            const int k = base + lane;
+            const bool cand = wh + k < nw && nr + k < S;
+            const int p = cand ? wp[wh + k] : 0;
+            const long long incl = wused + warp_incl_sum64(p, lane);
+            const long long st = incl - p;
+            const bool adm = cand && st < budget;
+            const long long x = adm ? min((long long)p, budget - st) : 0;
+            f1 += x;
+            f4 += x * (x + 1) / 2;
+            const int nadm = __popc(__ballot_sync(kFull, adm));
+            na += nadm;
+            wused = __shfl_sync(kFull, incl, 31);
+            if (nadm < 32) break;
+        }
+        f1 = warp_sum64(f1);
+        f2 = warp_sum64(f2);
+        f3 = warp_sum64(f3);
+        f4 = warp_sum64(f4);
+        // Eq. 9 for this batch, in the estimator's fp32 order
+        float T = __fmul_rn(b0, 1.0f);
+        T = __fmaf_rn(b1d, __ll2float_rn(f2), T);
+        T = __fmaf_rn(b1p, __ll2float_rn(f1), T);
+        T = __fmaf_rn(b2, __ll2float_rn(f3), T);
+        T = __fmaf_rn(b3, __ll2float_rn(f4), T);
+        if (t + (double)T > a.t_now) break;  // still running at t_now
+        if (nr + na > capR) {
+            ok = false;
+            break;
+        }
+        // Execute it: update the running list and the admitted requests, then
+        // keep (in order) every request with decode tokens left.
+        int kept = 0;
+        used = 0;
+        const int total = nr + na;
+        long long wst = 0;
+        for (int base = 0; base < total; base += 32) {
+            const int r = base + lane;
+            int ctx = 0, pre = 0, dec = 0;
+            long long need = 0;
+            const bool live = r < total;
+            if (live) {
+                if (r < nr) {
+                    ctx = rc[r];
+                    pre = rp[r];
+                    dec = rd[r];
+                    need = pre > 0 ? pre : 1;
+                } else {
+                    pre = wp[wh + r - nr];
+                    dec = wd[wh + r - nr];
+                    need = pre;
+                }
+            }
+            const long long inr = (live && r < nr) ? need : 0;
+            const long long incl_r = used + warp_incl_sum64(inr, lane);
+            const long long inw = (live && r >= nr) ? need : 0;
+            const long long incl_w = wst + warp_incl_sum64(inw, lane);
+            long long x = 0;
+            if (live && r < nr) x = max(0LL, min(need, (long long)B - (incl_r - inr)));
+            if (live && r >= nr) x = min(need, budget - (incl_w - inw));
+            if (live && x > 0) {
+                if (pre > 0) {
+                    ctx += (int)x;
+                    pre -= (int)x;
+                    if (pre == 0 && c.mode == 1) dec -= 1;  // first token with the last chunk
+                } else {
+                    ctx += 1;
+                    dec -= 1;
+                }
+            }
+            const bool keep = live && dec > 0;
+            const unsigned bal = __ballot_sync(kFull, keep);
+            if (keep) {
+                const int pos = kept + __popc(bal & lanemask_lt());
+                nc[pos] = ctx;
+                np[pos] = pre;
+                nd[pos] = dec;
+            }
+            kept += __popc(bal);
+            used = __shfl_sync(kFull, incl_r, 31);
+            wst = __shfl_sync(kFull, incl_w, 31);
+        }
+        __syncwarp();
+        int32_t *x0 = rc, *x1 = rp, *x2 = rd;
+        rc = nc;
+        rp = np;
+        rd = nd;
+        nc = x0;
+        np = x1;
+        nd = x2;
+        nr = kept;
+        wh += na;
+        t += (double)T;
+    }
+    if (!ok) {
+        fail3(a.ctl, kETraj, lane);
+        return;
+    }
+    const int nw2 = nw - wh;
+    for (int q = lane; q < capR; q += 32) {
+        dst.run_ctx[rrow + q] = q < nr ? rc[q] : 0;
+        dst.run_pre[rrow + q] = q < nr ? rp[q] : 0;
+        dst.run_dec[rrow + q] = q < nr ? rd[q] : 0;
+    }
+    for (int q = lane; q < capW; q += 32) {
+        dst.wait_pre[wrow + q] = q < nw2 ? wp[wh + q] : 0;
+        dst.wait_dec[wrow + q] = q < nw2 ? wd[wh + q] : 0;
+    }
+    if (lane == 0) {
+        dst.n_run[j] = nr;
+        dst.n_wait[j] = nw2;
+        dst.clock[j] = t;
+    }
+}
+
+__global__ void __launch_bounds__(kK3Warps * 32) k_advance(const K3Launch a) {
+    extern __shared__ __align__(16) int32_t k3_smem[];
+    const int lane = threadIdx.x & 31;
+    const int wid = threadIdx.x >> 5;
+    const int j = blockIdx.x * kK3Warps + wid;
+    const int active = *((volatile int32_t *)&a.ctl->active);
+    if (j >= a.cfg.I) return;
+    if (active < 0) {
+        fail3(a.ctl, kENoState, lane);
+        return;
+    }
+    const StateBuf src = active ? a.buf1 : a.buf0;
+    const size_t per_warp = advance_smem_per_warp(a.cfg) / sizeof(int32_t);
+    advance_instance(a, src, j, lane, k3_smem + wid * per_warp);
+}
+
+// Copy of the live snapshot into caller arrays (the live buffer is known only on
+// the device).
+__global__ void k_read_state(const DevConfig c, const StateBuf b0, const StateBuf b1, const DevCtl *ctl,
+                             const StateOut o) {
+    const int active = *((volatile const int32_t *)&ctl->active);
+    const StateBuf s = active == 1 ? b1 : b0;
+    const size_t R = (size_t)c.I * c.capR, W = (size_t)c.I * c.capW;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < R + W + c.I;
+         i += (size_t)gridDim.x * blockDim.x) {
+        if (i < R) {
+            if (o.run_ctx) o.run_ctx[i] = s.run_ctx[i];
+            if (o.run_pre) o.run_pre[i] = s.run_pre[i];
+            if (o.run_dec) o.run_dec[i] = s.run_dec[i];
+        } else if (i < R + W) {
+            if (o.wait_pre) o.wait_pre[i - R] = s.wait_pre[i - R];
+            if (o.wait_dec) o.wait_dec[i - R] = s.wait_dec[i - R];
+        } else {
+            const size_t k = i - R - W;
+            if (o.n_run) o.n_run[k] = s.n_run[k];
+            if (o.n_wait) o.n_wait[k] = s.n_wait[k];
+            if (o.clock) o.clock[k] = s.clock[k];
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_read_state(const DevConfig &c, const StateBuf &b0, const StateBuf &b1, DevCtl *ctl,
+                              const StateOut &o, cudaStream_t st) {
+    k_read_state<<<128, 256, 0, st>>>(c, b0, b1, ctl, o);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_advance(const K3Launch &a, int grid, size_t smem, cudaStream_t st) {
+    k_advance<<<grid, kK3Warps * 32, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t set_k3_smem(size_t bytes) {
+    return cudaFuncSetAttribute(k_advance, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
+}  // namespace lr

@@ -16,7 +16,10 @@ struct lr_ctx {
     int sms = 0;
     lr::DevConfig cfg{};
     lr::StateBuf buf[2]{};
+    lr::StateBuf scratch{};  // advanced snapshot before it is summarized
     lr::DevCtl *ctl = nullptr;
+    int max_seqs = 0;
+    size_t k3_smem = 0;
     float *scratch_tch = nullptr;
     std::vector<void *> allocs;
     std::string err;
@@ -164,6 +167,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
                                           std::to_string(j));
         kph = std::max(kph, (int)kp);
         nbh = std::max(nbh, nb[j]);
+        c->max_seqs = std::max(c->max_seqs, S);
     }
     cudaError_t e = cudaGetDevice(&c->device);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, c->device);
@@ -207,12 +211,24 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
         LR_ALLOC(s.n_wait, I);
         LR_ALLOC(s.wait_pre, W);
         LR_ALLOC(s.wait_dec, W);
+        LR_ALLOC(s.clock, I);
         LR_ALLOC(s.inst, I);
         LR_ALLOC(s.bkt, (size_t)nbh * I);
         LR_ALLOC(s.ent, (size_t)kph * I);
         LR_ALLOC(s.f2, (size_t)kph * I);
         LR_ALLOC(s.f3, (size_t)kph * I);
         LR_ALLOC(s.rcum, (size_t)kph * I);
+    }
+    {
+        lr::StateBuf &s = c->scratch;
+        LR_ALLOC(s.n_run, I);
+        LR_ALLOC(s.run_ctx, R);
+        LR_ALLOC(s.run_pre, R);
+        LR_ALLOC(s.run_dec, R);
+        LR_ALLOC(s.n_wait, I);
+        LR_ALLOC(s.wait_pre, W);
+        LR_ALLOC(s.wait_dec, W);
+        LR_ALLOC(s.clock, I);
     }
     LR_ALLOC(c->ctl, 1);
     LR_ALLOC(c->scratch_tch, (size_t)cfg->max_pairs * cfg->max_queries);
@@ -243,7 +259,9 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     c->est = make_shape(d, false, 1);
     c->rt = make_shape(d, true, cfg->max_pairs);
     if (!c->est.ok) return bail(LR_ECAPACITY, "summary tables too large for shared memory");
+    c->k3_smem = lr::kK3Warps * lr::advance_smem_per_warp(d);
     e = lr::set_k1_smem(c->k1_smem);
+    if (e == cudaSuccess && c->k3_smem <= 200 * 1024) e = lr::set_k3_smem(c->k3_smem);
     if (e == cudaSuccess) e = lr::set_k2_smem(std::max(c->est.smem, c->rt.ok ? c->rt.smem : 0));
     if (e == cudaSuccess) e = lr::cand_occupancy(d.mode, false, lr::kK2Block, c->est.smem, &c->est.occ);
     if (e == cudaSuccess && c->rt.ok) e = lr::cand_occupancy(d.mode, true, lr::kK2Block, c->rt.smem, &c->rt.occ);
@@ -273,7 +291,7 @@ int lr_load_state(lr_ctx *c, const lr_state_view *v, void *stream) {
     a.buf0 = c->buf[0];
     a.buf1 = c->buf[1];
     a.ctl = c->ctl;
-    a.in = lr::StateIn{v->n_run, v->run_ctx, v->run_pre, v->run_dec, v->n_wait, v->wait_pre, v->wait_dec};
+    a.in = lr::StateIn{v->n_run, v->run_ctx, v->run_pre, v->run_dec, v->n_wait, v->wait_pre, v->wait_dec, nullptr};
     const int grid = (c->cfg.I + lr::kK1Warps - 1) / lr::kK1Warps;
     cudaError_t e = lr::launch_trajectory(a, grid, lr::kK1Warps * 32, c->k1_smem, (cudaStream_t)stream);
     return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "trajectory launch");
@@ -364,6 +382,52 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
         if (e != cudaSuccess) return cuda_fail(c, e, "frontier launch");
     }
     return LR_OK;
+}
+
+int lr_advance(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_t *prompt_len, const int32_t *dec,
+               double t_now, void *stream) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    if (Q < 0) return fail(c, LR_EINVAL, "Q < 0");
+    if (Q > 0 && (!assign || !prompt_len || !dec)) return fail(c, LR_EINVAL, "null array");
+    if (!std::isfinite(t_now)) return fail(c, LR_EINVAL, "t_now must be finite");
+    if (c->cfg.capR < c->max_seqs) return fail(c, LR_ECAPACITY, "advancing needs cap_running >= every max_seqs");
+    if (c->k3_smem > 200 * 1024) return fail(c, LR_ECAPACITY, "queue capacities too large for one advance warp");
+    lr::K3Launch k;
+    std::memset(&k, 0, sizeof(k));
+    k.cfg = c->cfg;
+    k.buf0 = c->buf[0];
+    k.buf1 = c->buf[1];
+    k.scratch = c->scratch;
+    k.ctl = c->ctl;
+    k.Q = Q;
+    k.assign = assign;
+    k.prompt = prompt_len;
+    k.dec = dec;
+    k.t_now = t_now;
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e = lr::launch_advance(k, (c->cfg.I + lr::kK3Warps - 1) / lr::kK3Warps, c->k3_smem, st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "advance launch");
+    // summarize and publish the advanced snapshot exactly as a loaded one
+    lr::K1Launch a;
+    std::memset(&a, 0, sizeof(a));
+    a.cfg = c->cfg;
+    a.buf0 = c->buf[0];
+    a.buf1 = c->buf[1];
+    a.ctl = c->ctl;
+    const lr::StateBuf &sc = c->scratch;
+    a.in = lr::StateIn{sc.n_run, sc.run_ctx, sc.run_pre, sc.run_dec, sc.n_wait, sc.wait_pre, sc.wait_dec, sc.clock};
+    const int grid = (c->cfg.I + lr::kK1Warps - 1) / lr::kK1Warps;
+    e = lr::launch_trajectory(a, grid, lr::kK1Warps * 32, c->k1_smem, st);
+    return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "trajectory launch");
+}
+
+int lr_read_state(const lr_ctx *c, int32_t *n_run, int32_t *run_ctx, int32_t *run_pre, int32_t *run_dec,
+                  int32_t *n_wait, int32_t *wait_pre, int32_t *wait_dec, double *clock, void *stream) {
+    if (!c) return LR_EINVAL;
+    lr::StateOut o{n_run, run_ctx, run_pre, run_dec, n_wait, wait_pre, wait_dec, clock};
+    cudaError_t e = lr::launch_read_state(c->cfg, c->buf[0], c->buf[1], c->ctl, o, (cudaStream_t)stream);
+    return e == cudaSuccess ? LR_OK : LR_ECUDA;
 }
 
 int lr_status(lr_ctx *c, void *stream) {

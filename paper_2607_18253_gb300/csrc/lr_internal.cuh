@@ -52,6 +52,7 @@ struct DevConfig {
 
 struct StateBuf {
     int32_t *n_run, *run_ctx, *run_pre, *run_dec, *n_wait, *wait_pre, *wait_dec;
+    double *clock;  // [I] end time of the instance's last completed batch (s)
     InstParams *inst;
     int2 *bkt;
     float4 *ent;
@@ -68,6 +69,7 @@ struct DevCtl {
 
 struct StateIn {
     const int32_t *n_run, *run_ctx, *run_pre, *run_dec, *n_wait, *wait_pre, *wait_dec;
+    const double *clock;  // may be null: clocks start at 0
 };
 
 __device__ __forceinline__ void record_status(DevCtl *ctl, int code) {
@@ -142,5 +144,30 @@ cudaError_t cand_occupancy(int mode, bool route, int block, size_t smem, int *bl
 cudaError_t set_k2_smem(size_t bytes);
 constexpr int kK2Block = 256;
 constexpr size_t kK2SmemTarget = 56 * 1024;
+
+// K3: append routed queries and advance every instance to t_now (online stream).
+struct K3Launch {
+    DevConfig cfg;
+    StateBuf buf0, buf1;  // the live one is read
+    StateBuf scratch;     // receives the advanced snapshot (then summarized by K1)
+    DevCtl *ctl;
+    int32_t Q;
+    const int32_t *assign, *prompt, *dec;
+    double t_now;
+};
+constexpr int kK3Warps = 4;
+// Shared memory of one K3 warp: the running list twice (ctx, pre, dec; the
+// batch's survivors are compacted into the other copy) and the waiting queue.
+__host__ __device__ inline size_t advance_smem_per_warp(const DevConfig &c) {
+    return sizeof(int32_t) * ((size_t)6 * c.capR + (size_t)2 * c.capW + 32);
+}
+cudaError_t launch_advance(const K3Launch &a, int grid, size_t smem, cudaStream_t st);
+cudaError_t set_k3_smem(size_t bytes);
+struct StateOut {
+    int32_t *n_run, *run_ctx, *run_pre, *run_dec, *n_wait, *wait_pre, *wait_dec;
+    double *clock;
+};
+cudaError_t launch_read_state(const DevConfig &c, const StateBuf &b0, const StateBuf &b1, DevCtl *ctl,
+                              const StateOut &o, cudaStream_t st);
 
 }  // namespace lr

@@ -145,6 +145,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     if (lane == 0) {
         out.n_run[j] = nr;
         out.n_wait[j] = nw;
+        out.clock[j] = a.in.clock ? a.in.clock[j] : 0.0;
     }
     if (!(nr >= 0 && nr <= c.capR && nr <= S && nw >= 0 && nw <= c.capW)) {
         fail(a.ctl, kEState, lane);

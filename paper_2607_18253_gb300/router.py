@@ -22,7 +22,7 @@ FIRST_TOKEN_SEPARATE_DECODE = 0
 FIRST_TOKEN_WITH_LAST_CHUNK = 1
 
 EXPORTED_SYMBOLS = ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
-                    "lr_route", "lr_status", "lr_strerror", "lr_last_error")
+                    "lr_route", "lr_advance", "lr_read_state", "lr_status", "lr_strerror", "lr_last_error")
 
 _P = ctypes.c_void_p
 _I32 = ctypes.c_int32
@@ -57,13 +57,15 @@ def load_library(path: str = LIB_PATH):
     lib.lr_estimate_ttft.argtypes = [_P, _I32, _P, _P, _P, _P]
     lib.lr_estimate_features.argtypes = [_P, _I32, _P, _P, _P]
     lib.lr_route.argtypes = [_P, _I32, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P, _P, _P]
+    lib.lr_advance.argtypes = [_P, _I32, _P, _P, _P, ctypes.c_double, _P]
+    lib.lr_read_state.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.lr_status.argtypes = [_P, _P]
     lib.lr_strerror.argtypes = [ctypes.c_int]
     lib.lr_strerror.restype = ctypes.c_char_p
     lib.lr_last_error.argtypes = [_P]
     lib.lr_last_error.restype = ctypes.c_char_p
     for name in ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
-                 "lr_route", "lr_status"):
+                 "lr_route", "lr_advance", "lr_read_state", "lr_status"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -207,6 +209,32 @@ class LatencyRouter:
             _dev(ttft_matrix, torch.float32, "ttft_matrix_out", Q * self.num_instances), _stream(stream))
         self._check(rc, "lr_route")
         return o
+
+    def advance(self, assign: torch.Tensor, prompt_len: torch.Tensor, dec: torch.Tensor, t_now: float,
+                stream=None):
+        """Append routed queries (assign[i] >= 0) and advance every instance to t_now."""
+        Q = int(assign.numel())
+        self._check(self._lib.lr_advance(self._h, Q, _dev(assign, torch.int32, "assign"),
+                                         _dev(prompt_len, torch.int32, "prompt_len", Q),
+                                         _dev(dec, torch.int32, "dec", Q), float(t_now), _stream(stream)),
+                    "lr_advance")
+
+    def read_state(self, device="cuda", stream=None) -> dict:
+        """The live snapshot as device tensors (n_run, run_ctx, ..., wait_dec, clock)."""
+        I, R, W = self.num_instances, self.cap_running, self.cap_waiting
+        out = {"n_run": torch.empty(I, dtype=torch.int32, device=device),
+               "run_ctx": torch.empty((I, R), dtype=torch.int32, device=device),
+               "run_pre": torch.empty((I, R), dtype=torch.int32, device=device),
+               "run_dec": torch.empty((I, R), dtype=torch.int32, device=device),
+               "n_wait": torch.empty(I, dtype=torch.int32, device=device),
+               "wait_pre": torch.empty((I, W), dtype=torch.int32, device=device),
+               "wait_dec": torch.empty((I, W), dtype=torch.int32, device=device),
+               "clock": torch.empty(I, dtype=torch.float64, device=device)}
+        rc = self._lib.lr_read_state(self._h, *(ctypes.c_void_p(out[k].data_ptr()) for k in
+                                                ("n_run", "run_ctx", "run_pre", "run_dec", "n_wait", "wait_pre",
+                                                 "wait_dec", "clock")), _stream(stream))
+        self._check(rc, "lr_read_state")
+        return out
 
     def status(self, stream=None) -> int:
         """Synchronize the stream; return and clear the device status word."""

@@ -38,6 +38,8 @@ def test_idle_instance_jumps_to_now():
     wl = _one_instance([], [], 16, 4, COEF)
     w2, clk = oracle.advance(wl, [3.0], NONE, NONE, NONE, 7.5)
     assert clk[0] == 7.5 and w2.n_run[0] == 0 and w2.n_wait[0] == 0
+    w3, clk3 = oracle.advance(wl, [9.0], NONE, NONE, NONE, 7.5)
+    assert clk3[0] == 9.0  # a clock never runs backwards
 
 
 def test_hand_trace_batch_times():
