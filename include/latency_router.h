@@ -145,8 +145,9 @@ LR_API int lr_estimate_features(lr_ctx *ctx, int32_t Q, const int32_t *prompt_le
  *  U = acc - lambda * cost (Eq. 2).
  *  tau == NULL: Lagrangian objective (Eq. 5), argmax_j U - mu * TTFT.
  *  tau != NULL ([Q] device, seconds): constrained objective (Eq. 3), argmax U over
- *  {j : TTFT <= tau_i}, or the least TTFT when that set is empty; mu is then unused
- *  and may be NULL.  Ties go to the lowest instance index.
+ *  {j : TTFT <= tau_i}, or the least TTFT when that set is empty; it takes one
+ *  lambda (P == 1, else LR_EINVAL), and mu is then unused and may be NULL.
+ *  Ties go to the lowest instance index.
  *  lambda, mu: [P] HOST arrays, finite and >= 0, 1 <= P <= max_pairs.
  *  Outputs, device: assign_out [P][Q] int32, util_out [P][Q] fp32 U of the chosen
  *  instance, ttft_chosen_out [P][Q] fp32 or NULL, frontier_out [P][3] fp64 means of

@@ -348,6 +348,7 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
     if (P > c->max_pairs) return fail(c, LR_ECAPACITY, "P exceeds max_pairs");
     if (!c->rt.ok) return fail(c, LR_ECAPACITY, "routing needs num_instances <= 1024 and its tiles in shared memory");
     if (!lambda || (!tau && !mu)) return fail(c, LR_EINVAL, "null lambda / mu");
+    if (tau && P != 1) return fail(c, LR_EINVAL, "the constrained objective takes one lambda (P == 1)");
     for (int k = 0; k < P; ++k) {
         if (!finite_nonneg(lambda[k])) return fail(c, LR_EINVAL, "lambda must be finite and >= 0");
         if (!tau && !finite_nonneg(mu[k])) return fail(c, LR_EINVAL, "mu must be finite and >= 0");

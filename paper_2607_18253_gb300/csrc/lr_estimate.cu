@@ -452,7 +452,7 @@ __global__ void __launch_bounds__(256) k_frontier(const K2Launch a, double *out)
     for (int i = threadIdx.x; i < a.Q; i += blockDim.x) {
         const size_t o = (size_t)pp * a.Q + i;
         const int jj = a.assign[o];
-        if (jj < 0) {
+        if (jj < 0 || jj >= c.I) {
             sa = sc = st = __longlong_as_double(0x7ff8000000000000LL);
             continue;
         }

@@ -260,6 +260,9 @@ def test_host_side_errors():
     with pytest.raises(R().LRError) as e:
         rt.route(p16, dh, acc, [-1.0], [0.1])
     assert e.value.code == R().LR_EINVAL
+    with pytest.raises(R().LRError) as e:  # the constrained objective takes one lambda
+        rt.route(p16, dh, acc, [1.0, 2.0], None, tau=torch.ones(16, dtype=torch.float32, device="cuda"))
+    assert e.value.code == R().LR_EINVAL
     with pytest.raises(R().LRError):
         R().LatencyRouter(model_of_instance=[0], coef=np.ones((1, 5)), price_in=[0], price_out=[0],
                           max_batched_tokens=[8], max_seqs=[9], cap_running=4, cap_waiting=4, max_queries=4,
