@@ -159,6 +159,29 @@ LR_API int lr_route(lr_ctx *ctx, int32_t Q, const int32_t *prompt_len, const int
              float *util_out, float *ttft_chosen_out, double *frontier_out, float *ttft_matrix_out,
              void *cuda_stream);
 
+/* lr_route with the frontier, for callers that must not allocate device memory while
+ * serving (the paper has no counterpart: it is a memory-management variant of lr_route).
+ * A serving loop that runs inside a fixed device-memory reservation, or that cannot let
+ * an allocation synchronize the device between its launches, cannot call cudaMalloc (or
+ * an allocating library routine) on the request path.  This call allocates nothing: the
+ * per-(pair, query) chosen-TTFT values that the frontier averages live in one fixed array
+ * of the library's static device memory (LR_STATIC_ROUTE_CAP fp32 entries, 1 MiB) instead
+ * of memory taken from the context.  Arguments and outputs are those of lr_route with
+ * ttft_chosen_out and ttft_matrix_out absent; frontier_out is required.
+ *  - Requires P * Q <= LR_STATIC_ROUTE_CAP, else LR_ECAPACITY before any launch.
+ *  - Set-up: the first call on each device (which must be current, and the context's
+ *    device) looks the array up once; make that first call before any stream capture.
+ *  - Nothing in the array needs to start at zero: every entry the frontier reads is
+ *    written earlier in the same call, in stream order.
+ *  - The array is shared by every context on a device: two of these calls in flight at
+ *    once on one device (different streams, or different contexts) race on it, so order
+ *    them (one stream, or events). */
+#define LR_STATIC_ROUTE_CAP (1 << 18)
+LR_API int lr_route_frontier_static(lr_ctx *ctx, int32_t Q, const int32_t *prompt_len, const int32_t *dec_hat,
+                                    const float *acc, const float *tau, int32_t P, const float *lambda,
+                                    const float *mu, int32_t *assign_out, float *util_out, double *frontier_out,
+                                    void *cuda_stream);
+
 /* Online stream step (Sec. 5: queries arrive over time and are routed as they come;
  * App. F: every instance keeps executing token batches and publishes its state after each).
  * The queries with assign[i] >= 0 join instance assign[i]'s waiting tail in query order

@@ -22,7 +22,8 @@ FIRST_TOKEN_SEPARATE_DECODE = 0
 FIRST_TOKEN_WITH_LAST_CHUNK = 1
 
 EXPORTED_SYMBOLS = ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
-                    "lr_route", "lr_advance", "lr_read_state", "lr_status", "lr_strerror", "lr_last_error")
+                    "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
+                    "lr_strerror", "lr_last_error")
 
 _P = ctypes.c_void_p
 _I32 = ctypes.c_int32
@@ -57,6 +58,7 @@ def load_library(path: str = LIB_PATH):
     lib.lr_estimate_ttft.argtypes = [_P, _I32, _P, _P, _P, _P]
     lib.lr_estimate_features.argtypes = [_P, _I32, _P, _P, _P]
     lib.lr_route.argtypes = [_P, _I32, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P, _P, _P]
+    lib.lr_route_frontier_static.argtypes = [_P, _I32, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P]
     lib.lr_advance.argtypes = [_P, _I32, _P, _P, _P, ctypes.c_double, _P]
     lib.lr_read_state.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.lr_status.argtypes = [_P, _P]
@@ -65,7 +67,7 @@ def load_library(path: str = LIB_PATH):
     lib.lr_last_error.argtypes = [_P]
     lib.lr_last_error.restype = ctypes.c_char_p
     for name in ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
-                 "lr_route", "lr_advance", "lr_read_state", "lr_status"):
+                 "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -208,6 +210,35 @@ class LatencyRouter:
             _dev(o.get("frontier") if frontier else None, torch.float64, "frontier_out", P * 3),
             _dev(ttft_matrix, torch.float32, "ttft_matrix_out", Q * self.num_instances), _stream(stream))
         self._check(rc, "lr_route")
+        return o
+
+    def route_frontier_static(self, prompt_len: torch.Tensor, dec_hat: torch.Tensor, acc: torch.Tensor,
+                              lam: Sequence[float], mu: Optional[Sequence[float]] = None,
+                              tau: Optional[torch.Tensor] = None, out: Optional[dict] = None, stream=None) -> dict:
+        """route(..., frontier=True, ttft_chosen=False) whose intermediate lives in static device memory.
+
+        The C call allocates nothing; pass preallocated tensors in `out` ("assign",
+        "util", "frontier") to keep this wrapper from allocating them."""
+        Q, M = int(prompt_len.numel()), self.num_models
+        lam_h = np.ascontiguousarray(np.atleast_1d(np.asarray(lam, np.float32)))
+        P = int(lam_h.shape[0])
+        mu_h = None if mu is None else np.ascontiguousarray(np.atleast_1d(np.asarray(mu, np.float32)))
+        if mu_h is not None and mu_h.shape[0] != P:
+            raise ValueError("lam and mu must have the same length")
+        dev = prompt_len.device
+        o = {} if out is None else out
+        if "assign" not in o:
+            o["assign"] = torch.empty((P, Q), dtype=torch.int32, device=dev)
+            o["util"] = torch.empty((P, Q), dtype=torch.float32, device=dev)
+        if "frontier" not in o:
+            o["frontier"] = torch.empty((P, 3), dtype=torch.float64, device=dev)
+        rc = self._lib.lr_route_frontier_static(
+            self._h, Q, _dev(prompt_len, torch.int32, "prompt_len"), _dev(dec_hat, torch.int32, "dec_hat", Q * M),
+            _dev(acc, torch.float32, "acc", Q * M), _dev(tau, torch.float32, "tau", Q), P,
+            lam_h.ctypes.data_as(_P), None if mu_h is None else mu_h.ctypes.data_as(_P),
+            _dev(o["assign"], torch.int32, "assign_out", P * Q), _dev(o["util"], torch.float32, "util_out", P * Q),
+            _dev(o["frontier"], torch.float64, "frontier_out", P * 3), _stream(stream))
+        self._check(rc, "lr_route_frontier_static")
         return o
 
     def advance(self, assign: torch.Tensor, prompt_len: torch.Tensor, dec: torch.Tensor, t_now: float,
