@@ -272,6 +272,8 @@ def run_gpu(args):
                 "frac": ach / hbm, "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs, copy)",
                 "traffic": None, "note": "latency-bound event loop; bytes fraction shown for reference"}
 
+    stream = None if args.no_stream else run_stream(args, dev)
+
     if rank == 0:
         cpu = cpu_baseline(wl, args.cpu_seconds) if (world == 1 and not args.no_cpu) else None
         srt = sorted(step_ms)
@@ -285,11 +287,146 @@ def run_gpu(args):
             "e2e": {"value": cands * world / (e2e_mean * 1e-3), "unit": UNIT, "ms_per_step": e2e_mean,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": 2 * K, "clocks": clk.summary(), "wall_s_timed_region": t_wall,
+            "stream": stream,
         }
         print(json.dumps(line), flush=True)
     rt.close()
     if world > 1:
         dist.destroy_process_group()
+
+
+STREAM_WORKLOAD = "pool64"
+STREAM_SEED = 3
+STREAM_QUERIES = 1_000_000
+STREAM_SIZES = (1, 16, 256)
+
+
+def pool_capacity(R, W, wl, dev, horizon=300.0, warm=30.0, dt=2.0, depth=256):
+    """Completions/s of every instance fed a saturating FCFS stream of the workload's queries.
+
+    Each instance starts empty.  Before every advance of dt seconds its waiting queue
+    is topped up to `depth` with the workload's next queries (each with the predicted
+    output length of the instance's model), so the scheduler never runs dry;
+    completions are counted between t = warm and t = horizon.  The simulation is the
+    library's own stream step (lr_advance)."""
+    import dataclasses
+
+    import torch
+    I, M = wl.num_instances, wl.num_models
+    z = np.zeros(I, np.int32)
+    empty = dataclasses.replace(wl, n_run=z, n_wait=z.copy(), cap_waiting=depth,
+                                run_ctx=np.zeros((I, wl.cap_running), np.int32),
+                                run_pre=np.zeros((I, wl.cap_running), np.int32),
+                                run_dec=np.zeros((I, wl.cap_running), np.int32),
+                                wait_pre=np.zeros((I, depth), np.int32), wait_dec=np.zeros((I, depth), np.int32))
+    rt = R.LatencyRouter.from_workload(empty, max_queries=I * depth)
+    rt.load_state(*R.state_tensors(empty, dev))
+    appended = np.zeros(I, np.int64)
+    nq = wl.num_queries
+    nxt, t, c_warm = 0, 0.0, None
+    while True:
+        st = rt.read_state(device=dev)
+        n_run, n_wait = st["n_run"].cpu().numpy(), st["n_wait"].cpu().numpy()
+        completed = appended - n_run - n_wait
+        if c_warm is None and t >= warm:
+            c_warm = completed.copy()
+        if t >= horizon:
+            break
+        need = depth - n_wait
+        a = np.repeat(np.arange(I, dtype=np.int32), need)
+        idx = (nxt + np.arange(a.shape[0])) % nq
+        nxt += a.shape[0]
+        appended += need
+        t += dt
+        rt.advance(torch.from_numpy(a).to(dev), torch.from_numpy(wl.prompt_len[idx]).to(dev),
+                   torch.from_numpy(np.ascontiguousarray(wl.dec_hat[idx, wl.model_of_instance[a]])).to(dev), t)
+    torch.cuda.synchronize()
+    if rt.status() != R.LR_OK:
+        raise RuntimeError("capacity run failed")
+    rt.close()
+    return (completed - c_warm) / (horizon - warm)
+
+
+def run_stream(args, dev):
+    """Online stream: Poisson arrivals at 0.8 x pool capacity, routed in micro-batches.
+
+    At each decision time (the arrival of the batch's last query) the pool is advanced
+    to that time with the previous batch appended to its chosen instances (K3 + K1),
+    then the batch is routed on the new snapshot (K2, Lagrangian argmax).  The latency
+    of a batch is the device time of those three launches, from CUDA events around them;
+    the arguments are marshalled once, so the loop issues the C calls directly."""
+    import ctypes
+
+    import torch
+    from paper_2607_18253_gb300 import router as R
+    from paper_2607_18253_gb300 import workloads as W
+
+    wl = W.make_workload(STREAM_WORKLOAD, num_queries=STREAM_QUERIES, seed=STREAM_SEED, cap_waiting=512)
+    I, M = wl.num_instances, wl.num_models
+    cap = pool_capacity(R, W, wl, dev)
+    rate = 0.8 * float(cap.sum())
+    arr = W.poisson_arrivals(STREAM_QUERIES, rate, STREAM_SEED)
+    mmax = max(STREAM_SIZES)
+    rt = R.LatencyRouter.from_workload(wl, max_queries=mmax)
+    state = R.state_tensors(wl, dev)
+    p, dh, acc, _ = R.query_tensors(wl, dev)
+    assign = torch.full((2, mmax), -1, dtype=torch.int32, device=dev)  # ping-pong: batch b, batch b-1
+    util = torch.empty((1, mmax), dtype=torch.float32, device=dev)
+    lam = np.ascontiguousarray(wl.lam[:1], np.float32)
+    mu = np.ascontiguousarray(wl.mu[:1], np.float32)
+    lib, h = rt._lib, rt._h
+    sp = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    pp, dhp, accp = p.data_ptr(), dh.data_ptr(), acc.data_ptr()
+    ap = [assign[0].data_ptr(), assign[1].data_ptr()]
+    lamp, mup = lam.ctypes.data_as(ctypes.c_void_p), mu.ctypes.data_as(ctypes.c_void_p)
+    V = ctypes.c_void_p
+    out = {"workload": f"{STREAM_WORKLOAD} state and pool (seed {STREAM_SEED}), {STREAM_QUERIES} Poisson arrivals",
+           "capacity_qps": float(cap.sum()), "arrival_qps": rate,
+           "capacity_reading": "completions/s of each instance under a saturating FCFS stream, t = 30..300 s",
+           "latency": "device time of advance (K3 + K1) + route (K2) per micro-batch, CUDA events",
+           "sizes": {}}
+    launches = 0
+    for m in STREAM_SIZES:
+        nq = STREAM_QUERIES if (m > 1 or args.stream_full) else min(STREAM_QUERIES, args.stream_queries_b1)
+        nb = nq // m
+        rt.load_state(*state)
+        chunk = 4096
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(chunk)]
+        lat = []
+        torch.cuda.synchronize()
+        w0 = time.perf_counter()
+        for b in range(nb):
+            lo = b * m
+            cur, prev = ap[b & 1], ap[(b - 1) & 1]
+            e0, e1 = ev[b % chunk]
+            e0.record()
+            # previous batch joins its instances' queues; every instance advances to now
+            pm = m if b > 0 else 0
+            plo = (b - 1) * m
+            rc = lib.lr_advance(h, pm, V(prev), V(pp + 4 * max(plo, 0)), V(dhp + 4 * M * max(plo, 0)), M,
+                                ctypes.c_double(float(arr[lo + m - 1])), sp)
+            rc |= lib.lr_route(h, m, V(pp + 4 * lo), V(dhp + 4 * M * lo), V(accp + 4 * M * lo), None, 1, lamp,
+                               mup, V(cur), V(util.data_ptr()), None, None, None, sp)
+            e1.record()
+            if rc:
+                raise RuntimeError(f"stream call failed: {lib.lr_last_error(h).decode()}")
+            if b % chunk == chunk - 1 or b == nb - 1:
+                torch.cuda.synchronize()
+                lat += [ev[k][0].elapsed_time(ev[k][1]) for k in range(b % chunk + 1)]
+        wall = time.perf_counter() - w0
+        st = rt.status()
+        if st != R.LR_OK:
+            raise RuntimeError(f"stream run (micro-batch {m}) ended with device status {st}")
+        launches += 3 * nb
+        q = np.percentile(np.asarray(lat) * 1e3, [50, 99])
+        fin = rt.read_state(device=dev)
+        out["sizes"][str(m)] = {"batches": nb, "queries": nb * m, "p50_us": float(q[0]), "p99_us": float(q[1]),
+                                "mean_us": float(np.mean(lat) * 1e3), "wall_s": wall,
+                                "simulated_s": float(arr[nb * m - 1]),
+                                "final_mean_waiting": float(fin["n_wait"].float().mean().item())}
+    out["gpu_launches"] = launches
+    rt.close()
+    return out
 
 
 def _oracle_rows(wl, nq, seed):
@@ -355,6 +492,11 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--ref-step-seconds", type=float, default=2.0)
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-stream", action="store_true", help="skip the online-stream latency run")
+    ap.add_argument("--stream-full", action="store_true",
+                    help="route the whole 10^6-query trace at micro-batch 1 too (about a minute)")
+    ap.add_argument("--stream-queries-b1", type=int, default=50_000,
+                    help="queries of the trace routed one at a time (default: the first 50,000)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="dram bytes per launch of the dominant kernel from an ncu capture of this build")
     args = ap.parse_args()

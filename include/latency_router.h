@@ -191,12 +191,14 @@ LR_API int lr_route_frontier_static(lr_ctx *ctx, int32_t Q, const int32_t *promp
  * in fp32 and accumulated into a per-instance fp64 clock (an instance with nothing to run
  * jumps to t_now; no clock ever runs backwards).  Entries of assign outside [0, I), e.g. -1
  * for a query routed elsewhere, are skipped.  The advanced snapshot is then summarized and published as by
- * lr_load_state; clocks start at 0 when a snapshot is loaded.  assign, prompt_len, dec:
- * [Q] device arrays (Q may be 0).  Requires cap_running >= every max_seqs (LR_ECAPACITY
+ * lr_load_state; clocks start at 0 when a snapshot is loaded.  assign, prompt_len: [Q]
+ * device arrays (Q may be 0); dec: [Q][dec_cols] device, dec_cols 1 (one length per query)
+ * or num_models (the column of the chosen instance's model is used, e.g. the dec_hat
+ * matrix given to lr_route).  Requires cap_running >= every max_seqs (LR_ECAPACITY
  * otherwise).  A waiting queue that would exceed cap_waiting records LR_ECAPACITY, an
  * out-of-range length LR_EINVAL; either leaves the previous snapshot live. */
 LR_API int lr_advance(lr_ctx *ctx, int32_t Q, const int32_t *assign, const int32_t *prompt_len,
-                      const int32_t *dec, double t_now, void *cuda_stream);
+                      const int32_t *dec, int32_t dec_cols, double t_now, void *cuda_stream);
 
 /* Copy the live snapshot (as advanced so far) into caller arrays: device pointers with the
  * shapes of lr_state_view plus clock [I] fp64; any pointer may be NULL to skip it. */

@@ -68,7 +68,7 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
             const int pos = nw + __popc(bal & lanemask_lt());
             if (pos < capW) {
                 wp[pos] = a.prompt[i];
-                wd[pos] = a.dec[i];
+                wd[pos] = a.dec[(size_t)i * a.dec_cols + (a.dec_cols == 1 ? 0 : c.moi[j])];
             }
         }
         nw += __popc(bal);

@@ -434,11 +434,12 @@ int lr_route_frontier_static(lr_ctx *c, int32_t Q, const int32_t *prompt_len, co
 }
 
 int lr_advance(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_t *prompt_len, const int32_t *dec,
-               double t_now, void *stream) {
+               int32_t dec_cols, double t_now, void *stream) {
     if (!c) return LR_EINVAL;
     c->err.clear();
     if (Q < 0) return fail(c, LR_EINVAL, "Q < 0");
     if (Q > 0 && (!assign || !prompt_len || !dec)) return fail(c, LR_EINVAL, "null array");
+    if (dec_cols != 1 && dec_cols != c->cfg.M) return fail(c, LR_EINVAL, "dec_cols must be 1 or num_models");
     if (!std::isfinite(t_now)) return fail(c, LR_EINVAL, "t_now must be finite");
     if (c->cfg.capR < c->max_seqs) return fail(c, LR_ECAPACITY, "advancing needs cap_running >= every max_seqs");
     if (c->k3_smem > 200 * 1024) return fail(c, LR_ECAPACITY, "queue capacities too large for one advance warp");
@@ -453,6 +454,7 @@ int lr_advance(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_t *promp
     k.assign = assign;
     k.prompt = prompt_len;
     k.dec = dec;
+    k.dec_cols = dec_cols;
     k.t_now = t_now;
     cudaStream_t st = (cudaStream_t)stream;
     cudaError_t e = lr::launch_advance(k, (c->cfg.I + lr::kK3Warps - 1) / lr::kK3Warps, c->k3_smem, st);

@@ -152,6 +152,7 @@ struct K3Launch {
     StateBuf scratch;     // receives the advanced snapshot (then summarized by K1)
     DevCtl *ctl;
     int32_t Q;
+    int32_t dec_cols;  // 1: dec[i]; M: dec[i][model of the chosen instance]
     const int32_t *assign, *prompt, *dec;
     double t_now;
 };

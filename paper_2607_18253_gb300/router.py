@@ -59,7 +59,7 @@ def load_library(path: str = LIB_PATH):
     lib.lr_estimate_features.argtypes = [_P, _I32, _P, _P, _P]
     lib.lr_route.argtypes = [_P, _I32, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.lr_route_frontier_static.argtypes = [_P, _I32, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P]
-    lib.lr_advance.argtypes = [_P, _I32, _P, _P, _P, ctypes.c_double, _P]
+    lib.lr_advance.argtypes = [_P, _I32, _P, _P, _P, _I32, ctypes.c_double, _P]
     lib.lr_read_state.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.lr_status.argtypes = [_P, _P]
     lib.lr_strerror.argtypes = [ctypes.c_int]
@@ -243,11 +243,15 @@ class LatencyRouter:
 
     def advance(self, assign: torch.Tensor, prompt_len: torch.Tensor, dec: torch.Tensor, t_now: float,
                 stream=None):
-        """Append routed queries (assign[i] >= 0) and advance every instance to t_now."""
+        """Append routed queries (assign[i] >= 0) and advance every instance to t_now.
+
+        dec is [Q] (one output length per query) or [Q, M] (the chosen model's column is used)."""
         Q = int(assign.numel())
+        cols = 1 if dec.dim() == 1 else int(dec.shape[1])
         self._check(self._lib.lr_advance(self._h, Q, _dev(assign, torch.int32, "assign"),
                                          _dev(prompt_len, torch.int32, "prompt_len", Q),
-                                         _dev(dec, torch.int32, "dec", Q), float(t_now), _stream(stream)),
+                                         _dev(dec, torch.int32, "dec", Q * cols), cols, float(t_now),
+                                         _stream(stream)),
                     "lr_advance")
 
     def read_state(self, device="cuda", stream=None) -> dict:

@@ -227,6 +227,12 @@ def make_workload(name: str, num_queries: Optional[int] = None, seed: Optional[i
         lam=lam, mu=mu, max_prompt_len=int(r["p_cap"]), first_token_mode=first_token_mode, seed=seed)
 
 
+def poisson_arrivals(num_queries: int, rate_qps: float, seed: int) -> np.ndarray:
+    """Arrival times (s, fp64) of a Poisson process: exponential gaps with mean 1/rate."""
+    rng = np.random.default_rng(np.random.SeedSequence([seed, 0x5eed]))
+    return np.cumsum(rng.exponential(1.0 / rate_qps, num_queries))
+
+
 def sweep_pairs():
     """The trade-off grid: 4 lambda values (log 0.1..10) x 8 mu values (log 0.01..1 /s), lambda-major."""
     lam = np.logspace(-1, 1, 4)

@@ -127,9 +127,10 @@ def test_route_advance_loop_pool64(mode):
         np.testing.assert_array_equal(out["assign"].cpu().numpy(), a)
         np.testing.assert_array_equal(bits(out["util"].cpu().numpy()), bits(u))
         a0 = a[0]
-        d = q.dec_hat[np.arange(per), q.model_of_instance[a0]]
+        d = q.dec_hat[np.arange(per), q.model_of_instance[a0]]  # the chosen model's predicted length
         t_now = 0.02 * (s + 1)
-        rt.advance(dev(a0), dev(q.prompt_len), dev(d), t_now)
+        # the advance reads that column itself from the [Q, M] matrix on even steps
+        rt.advance(dev(a0), dev(q.prompt_len), dev(q.dec_hat if s % 2 == 0 else d), t_now)
         torch.cuda.synchronize()
         assert rt.status() == R().LR_OK
         wl, clk = oracle.advance(q, clk, a0, q.prompt_len, d, t_now)
@@ -187,6 +188,10 @@ def test_advance_host_side_errors():
     rt2 = make_router(wl2)
     with pytest.raises(R().LRError) as e:
         rt2.advance(z, z, z, float("nan"))
+    assert e.value.code == R().LR_EINVAL
+    one = dev(np.zeros(1, np.int32))
+    with pytest.raises(R().LRError) as e:  # dec must have 1 or num_models columns
+        rt2.advance(one, dev(np.ones(1)), dev(np.ones((1, wl2.num_models + 1))), 1.0)
     assert e.value.code == R().LR_EINVAL
     rt3 = R().LatencyRouter.from_workload(wl2)
     rt3.advance(z, z, z, 1.0)
