@@ -98,6 +98,67 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
             t = fmax(t, a.t_now);
             break;
         }
+        // A run of decode-only batches: with no request in prefill and no admission
+        // possible (waiting queue empty, or every seat taken), every batch decodes one
+        // token of each running request, so consecutive batches differ only in their
+        // context sum until the first request finishes.  Each batch is still timed on
+        // its own, with the general path's fp32 expression.
+        {
+            bool pre = false;
+            int dmin = kBig;
+            long long csum = 0;
+            for (int r = lane; r < nr; r += 32) {
+                pre |= rp[r] > 0;
+                dmin = min(dmin, rd[r]);
+                csum += rc[r];
+            }
+            if (!__any_sync(kFull, pre) && nr > 0 && (wh == nw || nr >= S) && iters < c.max_iters) {
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) dmin = min(dmin, __shfl_xor_sync(kFull, dmin, o));
+                csum = warp_sum64(csum);
+                const int run = (int)min((long long)dmin, (long long)c.max_iters - iters);
+                const float f1 = 0.0f, f2 = __int2float_rn(nr), f4 = 0.0f;
+                int done = 0;
+                for (; done < run; ++done) {
+                    float T = __fmul_rn(b0, 1.0f);
+                    T = __fmaf_rn(b1d, f2, T);
+                    T = __fmaf_rn(b1p, f1, T);
+                    T = __fmaf_rn(b2, __ll2float_rn(csum + (long long)done * nr), T);
+                    T = __fmaf_rn(b3, f4, T);
+                    if (t + (double)T > a.t_now) break;
+                    t += (double)T;
+                }
+                iters += done;
+                if (done > 0) {
+                    int kept = 0;
+                    for (int base = 0; base < nr; base += 32) {
+                        const int r = base + lane;
+                        const bool live = r < nr;
+                        const int dec = live ? rd[r] - done : 0;
+                        const bool keep = live && dec > 0;
+                        const unsigned bal = __ballot_sync(kFull, keep);
+                        if (keep) {
+                            const int pos = kept + __popc(bal & lanemask_lt());
+                            nc[pos] = rc[r] + done;
+                            np[pos] = 0;
+                            nd[pos] = dec;
+                        }
+                        kept += __popc(bal);
+                    }
+                    __syncwarp();
+                    int32_t *x0 = rc, *x1 = rp, *x2 = rd;
+                    rc = nc;
+                    rp = np;
+                    rd = nd;
+                    nc = x0;
+                    np = x1;
+                    nd = x2;
+                    nr = kept;
+                }
+                if (done < run) break;  // the next batch would end after t_now
+                continue;               // a request finished (or max_iters is reached)
+            }
+        }
         if (++iters > c.max_iters) {
             ok = false;
             break;

@@ -196,3 +196,23 @@ def test_advance_host_side_errors():
     rt3 = R().LatencyRouter.from_workload(wl2)
     rt3.advance(z, z, z, 1.0)
     assert rt3.status() == R().LR_ENOSTATE
+
+
+def test_advance_beyond_max_iters_keeps_previous_snapshot():
+    wl = W.make_workload("tiny", cap_running=64)
+    wl.n_wait[:] = 0  # the load needs few steps; draining the decoders needs thousands
+    rt = make_router(wl, max_iters=200)
+    torch.cuda.synchronize()
+    assert rt.status() == R().LR_OK
+    before = read(rt)
+    z = dev(np.zeros(0, np.int32))
+    rt.advance(z, z, z, 1e9)
+    assert rt.status() == R().LR_ETRAJ
+    after = read(rt)
+    for k in STATE + ("clock",):
+        np.testing.assert_array_equal(after[k], before[k], err_msg=k)
+    # a short advance within the limit still matches the oracle
+    rt.advance(z, z, z, 0.05)
+    assert rt.status() == R().LR_OK
+    w2, c2 = oracle.advance(wl, np.zeros(wl.num_instances), [], [], [], 0.05)
+    check_state(read(rt), w2, c2)
