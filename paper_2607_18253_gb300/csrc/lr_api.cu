@@ -98,7 +98,9 @@ lr_ctx::Shape make_shape(const lr::DevConfig &d, bool route, int max_pairs) {
     const int wpr = s.Gp > 32 ? s.Gp / 32 : 1;
     const size_t tables = (size_t)d.kph * 4 * s.Gp * 16 + (size_t)d.nbh * 4 * s.Gp * 8;
     const size_t part = s.Gp > 32 ? 2 * (size_t)wpr * 16 * max_pairs : 0;  // wide-row partials per pair
-    const size_t per_row = 16 + (route ? part + (size_t)d.M * 8 + 4 : 0);
+    // staged row (16 B) and two raw copies of its prompt; routing adds the wide-row
+    // partials, (cost, acc) per model, tau, and two raw copies of tau, dec_hat and acc
+    const size_t per_row = 16 + 8 + (route ? part + (size_t)d.M * 8 + 4 + 8 + (size_t)d.M * 16 : 0);
     const size_t room = lr::kK2SmemTarget > tables ? lr::kK2SmemTarget - tables : 0;
     int qt = (int)std::min<size_t>(256, room / per_row);
     if (route && (size_t)qt * per_row + tables > 200 * 1024) qt = 0;

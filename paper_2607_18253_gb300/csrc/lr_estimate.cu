@@ -194,13 +194,26 @@ __device__ __forceinline__ float pick4(const float v[4], int u) {
     return x;
 }
 
+// Asynchronous 4-byte global -> shared copies (the staging of the next chunk of
+// query rows overlaps the current chunk's compute).
+__device__ __forceinline__ void cp_async4(void *smem_dst, const void *gmem_src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"((uint32_t)__cvta_generic_to_shared(smem_dst)),
+                 "l"(gmem_src)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
 template <bool B>
 struct Flag {
     static constexpr bool value = B;
 };
 
 template <int MODE, int OUT>
-__global__ void __launch_bounds__(256) k_cand(const K2Launch a) {
+__global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     extern __shared__ __align__(16) unsigned char smem[];
     constexpr bool ROUTE = (OUT & (kOutLag | kOutCon | kOutSweep)) != 0;
     constexpr bool CON = (OUT & kOutCon) != 0;
@@ -246,6 +259,12 @@ __global__ void __launch_bounds__(256) k_cand(const K2Launch a) {
     int2 *s_bkt = reinterpret_cast<int2 *>(s_part + (ROUTE && Gp > 32 ? 2 * NP * QT * WPR : 0));  // [nbh][4][Gp]
     float2 *s_ca = reinterpret_cast<float2 *>(s_bkt + c.nbh * 4 * Gp);                 // [QT][M] (cost, acc)
     float *s_tau = reinterpret_cast<float *>(s_ca + (ROUTE ? QT * M : 0));             // [QT]
+    // raw query rows as copied from global memory, two chunks in flight:
+    // prompt [2][QT], and for routing tau [2][QT], dec_hat [2][QT][M], acc [2][QT][M]
+    int32_t *r_p = reinterpret_cast<int32_t *>(s_tau + (ROUTE ? QT : 0));
+    float *r_t = reinterpret_cast<float *>(r_p + 2 * QT);
+    int32_t *r_d = reinterpret_cast<int32_t *>(r_t + (ROUTE ? 2 * QT : 0));
+    float *r_a = reinterpret_cast<float *>(r_d + (ROUTE ? 2 * QT * M : 0));
 
     for (int idx = threadIdx.x; idx < c.kph * 4 * Gp; idx += blockDim.x) {
         const int k = idx / (4 * Gp);
@@ -302,22 +321,47 @@ __global__ void __launch_bounds__(256) k_cand(const K2Launch a) {
 
     auto run = [&](auto fast_tag) {
         constexpr bool FAST = decltype(fast_tag)::value;
-        for (int q0 = rb; q0 < re; q0 += QT) {
-            const int nrows = min(QT, re - q0);
+        // copies of chunk [q0, q0 + nrows) into raw buffer b
+        auto issue = [&](int q0, int nrows, int b) {
             for (int t = threadIdx.x; t < nrows; t += blockDim.x) {
-                bool ok;
-                s_q[t] = make_qrec(a.prompt[q0 + t], c.pmax, &ok);
-                if (!ok && blockIdx.y == 0) record_status(a.ctl, kEInval);
-                if (CON) s_tau[t] = a.tau[q0 + t];
+                cp_async4(r_p + b * QT + t, a.prompt + q0 + t);
+                if (CON) cp_async4(r_t + b * QT + t, a.tau + q0 + t);
             }
             if (ROUTE) {
+                const size_t g0 = (size_t)q0 * M;
+                for (int idx = threadIdx.x; idx < nrows * M; idx += blockDim.x) {
+                    cp_async4(r_d + b * QT * M + idx, a.dec_hat + g0 + idx);
+                    cp_async4(r_a + b * QT * M + idx, a.acc + g0 + idx);
+                }
+            }
+            cp_async_commit();
+        };
+        issue(rb, min(QT, re - rb), 0);
+        int buf = 0;
+        for (int q0 = rb; q0 < re; q0 += QT, buf ^= 1) {
+            const int nrows = min(QT, re - q0);
+            if (q0 + QT < re) {
+                issue(q0 + QT, min(QT, re - q0 - QT), buf ^ 1);
+                cp_async_wait<1>();
+            } else {
+                cp_async_wait<0>();
+            }
+            __syncthreads();  // every thread's copies of this chunk have landed
+            const int32_t *bp = r_p + buf * QT;
+            for (int t = threadIdx.x; t < nrows; t += blockDim.x) {
+                bool ok;
+                s_q[t] = make_qrec(bp[t], c.pmax, &ok);
+                if (!ok && blockIdx.y == 0) record_status(a.ctl, kEInval);
+                if (CON) s_tau[t] = r_t[buf * QT + t];
+            }
+            if (ROUTE) {
+                const int32_t *bd = r_d + buf * QT * M;
+                const float *ba = r_a + buf * QT * M;
                 for (int idx = threadIdx.x; idx < nrows * M; idx += blockDim.x) {
                     const int rr = idx / M;
                     const int m = idx - rr * M;
-                    const size_t gi = (size_t)(q0 + rr) * M + m;
-                    const float cost = __fmaf_rn((float)a.dec_hat[gi], c.pout[m],
-                                                 __fmul_rn((float)a.prompt[q0 + rr], c.pin[m]));
-                    const float acc = a.acc[gi];
+                    const float cost = __fmaf_rn((float)bd[idx], c.pout[m], __fmul_rn((float)bp[rr], c.pin[m]));
+                    const float acc = ba[idx];
                     // one pair: stage U itself (x), else (cost, acc)
                     s_ca[idx] = SWEEP ? make_float2(cost, acc) : make_float2(__fmaf_rn(-a.lam[0], cost, acc), cost);
                 }

@@ -143,7 +143,7 @@ cudaError_t launch_frontier(const K2Launch &a, double *out, cudaStream_t st);
 cudaError_t cand_occupancy(int mode, bool route, int block, size_t smem, int *blocks_per_sm);
 cudaError_t set_k2_smem(size_t bytes);
 constexpr int kK2Block = 256;
-constexpr size_t kK2SmemTarget = 56 * 1024;
+constexpr size_t kK2SmemTarget = 72 * 1024;  // three CTAs per SM
 
 // K3: append routed queries and advance every instance to t_now (online stream).
 struct K3Launch {

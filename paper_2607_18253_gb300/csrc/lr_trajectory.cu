@@ -82,25 +82,50 @@ __device__ __forceinline__ int warp_incl_sum(int x, int lane) {
     return x;
 }
 
+// Shared-memory accesses of the step loop by 32-bit shared address: the loop is
+// a chain of dependent decisions on one lane, so every address computation and
+// every generic-to-shared translation sits on its critical path.  The volatile
+// statements keep their program order, which the loop relies on.
+__device__ __forceinline__ uint32_t saddr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ int lds(uint32_t a) {
+    int v;
+    asm volatile("ld.shared.s32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ void sts(uint32_t a, int v) {
+    asm volatile("st.shared.s32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+__device__ __forceinline__ void red_add(uint32_t a, int v) {
+    asm volatile("red.shared.add.s32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+__device__ __forceinline__ void red_or(uint32_t a, uint32_t v) {
+    asm volatile("red.shared.or.b32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+
 // Scalar view of one instance's trajectory state, used by a single lane: the
 // step loop is a chain of dependent decisions, so it runs as plain scalar
 // code over shared memory without warp-wide round trips.
 struct Track {
-    WarpSmem m;
-    int nlist;  // decoders in the list
+    uint32_t cal, bm, ds, df, dcb;  // shared addresses of the calendar, its bitmap and the decoder list
+    int nlist;                      // decoders in the list
+    unsigned long long words;       // bit w set: calendar word w has a non-empty batch
 
     // Smallest last-decode batch >= L of any decoder; ends beyond the calendar
     // (always later than every calendar end) are found in the list.
     __device__ int next_end(int L) const {
         if (L < kCalendar) {
-            int w = L >> 5;
-            uint32_t word = m.bm[w] & (~0u << (L & 31));
-            while (word == 0u && ++w < kCalendar / 32) word = m.bm[w];
+            const int w = L >> 5;
+            const uint32_t word = (uint32_t)lds(bm + 4u * w) & (~0u << (L & 31));
             if (word != 0u) return (w << 5) + __ffs(word) - 1;
+            const unsigned long long rest = (w + 1 < 64) ? (words & (~0ull << (w + 1))) : 0ull;
+            if (rest != 0ull) {
+                const int w2 = __ffsll((long long)rest) - 1;
+                return (w2 << 5) + __ffs(lds(bm + 4u * w2)) - 1;
+            }
         }
         int mn = kBig;
         for (int i = 0; i < nlist; ++i) {
-            const int f = m.df[i];
+            const int f = lds(df + 4u * i);
             if (f >= L && f < mn) mn = f;
         }
         return mn;
@@ -108,20 +133,23 @@ struct Track {
 
     // Number of decoders whose last decode batch is fc.
     __device__ int ends_at(int fc) const {
-        if (fc < kCalendar) return m.cal[fc];
+        if (fc < kCalendar) return lds(cal + 4u * fc);
         int eq = 0;
-        for (int i = 0; i < nlist; ++i) eq += (m.df[i] == fc) ? 1 : 0;
+        for (int i = 0; i < nlist; ++i) eq += (lds(df + 4u * i) == fc) ? 1 : 0;
         return eq;
     }
 
+    // The calendar updates are reductions whose results are not returned, so the
+    // step loop does not wait for a load-modify-store round trip.
     __device__ void append(int s, int f, int cb) {
-        m.ds[nlist] = s;
-        m.df[nlist] = f;
-        m.dcb[nlist] = cb;
+        sts(ds + 4u * nlist, s);
+        sts(df + 4u * nlist, f);
+        sts(dcb + 4u * nlist, cb);
         ++nlist;
         if (f < kCalendar) {
-            m.cal[f] += 1;
-            m.bm[f >> 5] |= 1u << (f & 31);
+            red_add(cal + 4u * f, 1);
+            red_or(bm + 4u * (f >> 5), 1u << (f & 31));
+            words |= 1ull << (f >> 5);
         }
     }
 };
@@ -256,17 +284,30 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     }
     const int n0 = nr - (pfR > 0 ? 1 : 0);
 
+    // non-empty calendar words after the running decoders were entered
+    const unsigned long long words0 =
+        (unsigned long long)__ballot_sync(kFull, m.bm[lane] != 0u) |
+        ((unsigned long long)__ballot_sync(kFull, m.bm[lane + 32] != 0u) << 32);
+
     // Step the scheduler on lane 0 until a query appended now would be admitted.
     if (lane == 0) {
         Track tr;
-        tr.m = m;
+        tr.cal = saddr(m.cal);
+        tr.bm = saddr(m.bm);
+        tr.ds = saddr(m.ds);
+        tr.df = saddr(m.df);
+        tr.dcb = saddr(m.dcb);
         tr.nlist = n0;
+        tr.words = words0;
+        const uint32_t sP = saddr(m.P), sW = saddr(m.wdec);
         bool pf = pfR > 0;
         int n = n0;  // decoders alive at the start of batch l
         int l = 1, head = 0, iters = 0;
         int ph = 0;  // prompt prefix sum at the waiting head
         int fnext = tr.next_end(1);
         int la = 0, r0 = 0;
+        int pn_head = lds(sP + 4u * min(1, c.capW));
+        int d_head = lds(sW);
         while (iters < c.max_iters && l < (1 << 30)) {
             ++iters;
             int cnt = n + (pf ? 1 : 0);  // requests running in batch l
@@ -306,12 +347,16 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             }
             // FCFS admission while budget and a sequence slot remain.
             while (budget > 0 && head < nw && cnt < S) {
-                const int pn = m.P[head + 1];
-                const int d = m.wdec[head];
+                const int pn = pn_head;
+                const int d = d_head;
                 const int p = pn - ph;
                 ++head;
                 ph = pn;
                 ++cnt;
+                // the next head's prompt sum and length, loaded ahead of their use
+                // (P has capW + 1 entries; wdec's entries past nw are in bounds too)
+                pn_head = lds(sP + 4u * min(head + 1, c.capW));
+                d_head = lds(sW + 4u * min(head, c.capW - 1));
                 if (p <= budget) {
                     budget -= p;
                     int f, cb;
