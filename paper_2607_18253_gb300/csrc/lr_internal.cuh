@@ -104,11 +104,11 @@ constexpr int kK1Warps = 4;
 constexpr int kCalendar = 2048;
 
 // Shared memory of one K1 warp (in int32 words, a multiple of 4): calendar and
-// its bitmap, the waiting queue's prompt prefix sums and decode lengths, the
-// decoder list (first batch, last batch, context offset) and the budgets.
+// its bitmap, the decoder list (first batch, last batch, context offset, pad),
+// the waiting queue's prompt prefix sums and decode lengths, and the budgets.
 __host__ __device__ inline size_t trajectory_smem_per_warp(const DevConfig &c) {
-    const size_t words = (size_t)kCalendar + kCalendar / 32 + (size_t)(c.capW + 1) + (size_t)c.capW +
-                         3 * (size_t)(c.capR + c.capW) + (size_t)c.kph + 32;
+    const size_t words = (size_t)kCalendar + kCalendar / 32 + 4 * (size_t)(c.capR + c.capW) +
+                         (size_t)(c.capW + 1) + (size_t)c.capW + (size_t)c.kph + 32;
     return sizeof(int32_t) * ((words + 3) & ~(size_t)3);
 }
 

@@ -41,27 +41,24 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 
 struct WarpSmem {
-    int32_t *P;      // [capW + 1] exclusive prefix sums of waiting prompts
-    int32_t *wdec;   // [capW] waiting decode lengths
-    int32_t *ds;     // [capR + capW] decoder list: first decode batch
-    int32_t *df;     //   last decode batch
-    int32_t *dcb;    //   context at batch l is dcb + l
     int32_t *cal;    // [kCalendar] decoders by last decode batch
     uint32_t *bm;    // [kCalendar / 32] non-empty calendar batches
+    int4 *dl;        // [capR + capW] decoder list: (first decode batch s, last decode
+                     //   batch f, context offset cb: context at batch l is cb + l, 0)
+    int32_t *P;      // [capW + 1] exclusive prefix sums of waiting prompts
+    int32_t *wdec;   // [capW] waiting decode lengths
     int32_t *rcum;   // [kph] cumulative budgets
-    int32_t *scr;    // [32] scratch of the seat-limited step
+    int32_t *scr;    // [32] results of the step loop
 };
 
 __device__ __forceinline__ WarpSmem carve(int32_t *base, const DevConfig &c) {
     WarpSmem w;
     w.cal = base;
     w.bm = reinterpret_cast<uint32_t *>(w.cal + kCalendar);
-    w.P = reinterpret_cast<int32_t *>(w.bm + kCalendar / 32);
+    w.dl = reinterpret_cast<int4 *>(w.bm + kCalendar / 32);  // 16-byte aligned
+    w.P = reinterpret_cast<int32_t *>(w.dl + (c.capR + c.capW));
     w.wdec = w.P + (c.capW + 1);
-    w.ds = w.wdec + c.capW;
-    w.df = w.ds + (c.capR + c.capW);
-    w.dcb = w.df + (c.capR + c.capW);
-    w.rcum = w.dcb + (c.capR + c.capW);
+    w.rcum = w.wdec + c.capW;
     w.scr = w.rcum + c.kph;
     return w;
 }
@@ -92,9 +89,6 @@ __device__ __forceinline__ int lds(uint32_t a) {
     asm volatile("ld.shared.s32 %0, [%1];" : "=r"(v) : "r"(a));
     return v;
 }
-__device__ __forceinline__ void sts(uint32_t a, int v) {
-    asm volatile("st.shared.s32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
-}
 __device__ __forceinline__ void red_add(uint32_t a, int v) {
     asm volatile("red.shared.add.s32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
 }
@@ -102,13 +96,17 @@ __device__ __forceinline__ void red_or(uint32_t a, uint32_t v) {
     asm volatile("red.shared.or.b32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
 }
 
+__device__ __forceinline__ void sts4(uint32_t a, int x, int y, int z, int w) {
+    asm volatile("st.shared.v4.s32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(x), "r"(y), "r"(z), "r"(w) : "memory");
+}
+
 // Scalar view of one instance's trajectory state, used by a single lane: the
 // step loop is a chain of dependent decisions, so it runs as plain scalar
 // code over shared memory without warp-wide round trips.
 struct Track {
-    uint32_t cal, bm, ds, df, dcb;  // shared addresses of the calendar, its bitmap and the decoder list
-    int nlist;                      // decoders in the list
-    unsigned long long words;       // bit w set: calendar word w has a non-empty batch
+    uint32_t cal, bm, dl;       // shared addresses of the calendar, its bitmap and the decoder list
+    int nlist;                  // decoders in the list
+    unsigned long long words;   // bit w set: calendar word w has a non-empty batch
 
     // Smallest last-decode batch >= L of any decoder; ends beyond the calendar
     // (always later than every calendar end) are found in the list.
@@ -125,7 +123,7 @@ struct Track {
         }
         int mn = kBig;
         for (int i = 0; i < nlist; ++i) {
-            const int f = lds(df + 4u * i);
+            const int f = lds(dl + 16u * i + 4u);
             if (f >= L && f < mn) mn = f;
         }
         return mn;
@@ -135,16 +133,15 @@ struct Track {
     __device__ int ends_at(int fc) const {
         if (fc < kCalendar) return lds(cal + 4u * fc);
         int eq = 0;
-        for (int i = 0; i < nlist; ++i) eq += (lds(df + 4u * i) == fc) ? 1 : 0;
+        for (int i = 0; i < nlist; ++i) eq += (lds(dl + 16u * i + 4u) == fc) ? 1 : 0;
         return eq;
     }
 
-    // The calendar updates are reductions whose results are not returned, so the
-    // step loop does not wait for a load-modify-store round trip.
+    // A new decoder with first decode batch s and last decode batch f.  The
+    // calendar updates are reductions whose results are not returned, so the
+    // loop does not wait for a load-modify-store round trip.
     __device__ void append(int s, int f, int cb) {
-        sts(ds + 4u * nlist, s);
-        sts(df + 4u * nlist, f);
-        sts(dcb + 4u * nlist, cb);
+        sts4(dl + 16u * nlist, s, f, cb, 0);
         ++nlist;
         if (f < kCalendar) {
             red_add(cal + 4u * f, 1);
@@ -158,12 +155,14 @@ struct Track {
 // batch e with ce tokens of context and d output tokens (Sec. 4.1: the decode
 // stage starts after the prefill).  Returns false if it never decodes (first
 // token sampled with the last chunk and d == 1).
-__device__ __forceinline__ bool decoder_of(int mode, int e, int ce, int d, int *f, int *cb) {
+template <int MODE>
+__device__ __forceinline__ bool decoder_of(int e, int ce, int d, int *f, int *cb) {
     *cb = ce - (e + 1);
-    *f = e + d - mode;
-    return mode == 0 || d >= 2;
+    *f = e + d - MODE;
+    return MODE == 0 || d >= 2;
 }
 
+template <int MODE>
 __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j, int lane, int32_t *wbase) {
     const DevConfig &c = a.cfg;
     const int B = c.B[j];
@@ -182,7 +181,6 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     WarpSmem m = carve(wbase, c);
     const size_t rrow = (size_t)j * c.capR;
     const size_t wrow = (size_t)j * c.capW;
-    const int mode = c.mode;
 
     // Clear the calendar.
     for (int i = lane; i < kCalendar / 4; i += 32) reinterpret_cast<int4 *>(m.cal)[i] = make_int4(0, 0, 0, 0);
@@ -222,9 +220,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                     pf_dec = dec;
                 }
                 if (pre == 0 && !bad) {
-                    m.ds[t] = 1;
-                    m.df[t] = dec;
-                    m.dcb[t] = ctx - 1;
+                    m.dl[t] = make_int4(1, dec, ctx - 1, 0);
                     if (dec < kCalendar) {
                         atomicAdd(&m.cal[dec], 1);
                         atomicOr(&m.bm[dec >> 5], 1u << (dec & 31));
@@ -294,9 +290,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         Track tr;
         tr.cal = saddr(m.cal);
         tr.bm = saddr(m.bm);
-        tr.ds = saddr(m.ds);
-        tr.df = saddr(m.df);
-        tr.dcb = saddr(m.dcb);
+        tr.dl = saddr(m.dl);
         tr.nlist = n0;
         tr.words = words0;
         const uint32_t sP = saddr(m.P), sW = saddr(m.wdec);
@@ -313,6 +307,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             int cnt = n + (pf ? 1 : 0);  // requests running in batch l
             if (!pf && cnt >= S) {
                 // Every sequence slot is taken: nothing but decoding until one frees.
+                if (fnext == kBig) break;  // excluded: a decoder is running
                 n -= tr.ends_at(fnext);
                 l = fnext + 1;
                 fnext = tr.next_end(l);
@@ -339,7 +334,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                 pfC += pfR;
                 pf = false;
                 int f, cb;
-                if (decoder_of(mode, l, pfC, pfD, &f, &cb)) {
+                if (decoder_of<MODE>(l, pfC, pfD, &f, &cb)) {
                     tr.append(l + 1, f, cb);
                     ++pend;
                     fnext = min(fnext, f);
@@ -360,7 +355,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                 if (p <= budget) {
                     budget -= p;
                     int f, cb;
-                    if (decoder_of(mode, l, p, d, &f, &cb)) {
+                    if (decoder_of<MODE>(l, p, d, &f, &cb)) {
                         tr.append(l + 1, f, cb);
                         ++pend;
                         fnext = min(fnext, f);
@@ -406,7 +401,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     // Budgets left to the query after its admission batch, and the residents'
     // decode features up to each batch its first token can fall in (one
     // parallel pass over the decoder list per batch).
-    const int off = (mode == 0) ? 1 : 0;
+    constexpr int off = (MODE == 0) ? 1 : 0;
     const int nl = sim.nlist;
     int kp = 1;
     long long rc = r0;
@@ -414,7 +409,10 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     while (rc < c.pmax && kp < c.kph) {
         const int lk = la + kp;
         int nd = 0;
-        for (int i = lane; i < nl; i += 32) nd += (m.ds[i] <= lk && lk <= m.df[i]) ? 1 : 0;
+        for (int i = lane; i < nl; i += 32) {
+            const int4 dd = m.dl[i];
+            nd += (dd.x <= lk && lk <= dd.y) ? 1 : 0;
+        }
         nd = __reduce_add_sync(kFull, nd);
         rc += B - nd;
         if (lane == 0) m.rcum[kp] = (int)min(rc, (long long)kBig - 1);
@@ -435,12 +433,13 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         const int L = la + k + off;
         long long a2 = 0, a3 = 0;
         for (int i = lane; i < nl; i += 32) {
-            const int s = m.ds[i];
+            const int4 dd = m.dl[i];
+            const int s = dd.x;
             if (s <= L) {
-                const int e = min(m.df[i], L);
+                const int e = min(dd.y, L);
                 const long long cnt = (long long)e - s + 1;
                 a2 += cnt;
-                a3 += cnt * (long long)m.dcb[i] + (((long long)s + e) * cnt) / 2;
+                a3 += cnt * (long long)dd.z + (((long long)s + e) * cnt) / 2;
             }
         }
         const long long F2 = warp_sum64(a2) + off;  // + the query's own first decode token
@@ -495,6 +494,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     }
 }
 
+template <int MODE>
 __global__ void __launch_bounds__(kK1Warps * 32) k_trajectory(const K1Launch a) {
     extern __shared__ __align__(16) int32_t k1_smem[];
     const int lane = threadIdx.x & 31;
@@ -504,7 +504,7 @@ __global__ void __launch_bounds__(kK1Warps * 32) k_trajectory(const K1Launch a) 
     const int dst = (active == 0) ? 1 : 0;
     const StateBuf out = dst ? a.buf1 : a.buf0;
     const size_t per_warp = trajectory_smem_per_warp(a.cfg) / sizeof(int32_t);
-    if (j < a.cfg.I) summarize_instance(a, out, j, lane, k1_smem + wid * per_warp);
+    if (j < a.cfg.I) summarize_instance<MODE>(a, out, j, lane, k1_smem + wid * per_warp);
 
     // The last CTA to finish publishes the new snapshot if every instance succeeded.
     __syncthreads();
@@ -524,12 +524,15 @@ __global__ void __launch_bounds__(kK1Warps * 32) k_trajectory(const K1Launch a) 
 }  // namespace
 
 cudaError_t launch_trajectory(const K1Launch &a, int grid, int block, size_t smem, cudaStream_t st) {
-    k_trajectory<<<grid, block, smem, st>>>(a);
+    if (a.cfg.mode == 0) k_trajectory<0><<<grid, block, smem, st>>>(a);
+    else k_trajectory<1><<<grid, block, smem, st>>>(a);
     return cudaGetLastError();
 }
 
 cudaError_t set_k1_smem(size_t bytes) {
-    return cudaFuncSetAttribute(k_trajectory, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    cudaError_t e = cudaFuncSetAttribute(k_trajectory<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_trajectory<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    return e;
 }
 
 }  // namespace lr
