@@ -67,6 +67,14 @@ def _load():
         lib.orc_advance.restype = ctypes.c_int
         lib.orc_utility.argtypes = [ctypes.c_float, ctypes.c_float, i32, i32, ctypes.c_float, ctypes.c_float]
         lib.orc_utility.restype = ctypes.c_float
+        lib.orc_pow_int.argtypes = [ctypes.c_double, i32]
+        lib.orc_pow_int.restype = ctypes.c_double
+        lib.orc_lps_wait.argtypes = [ctypes.c_double, ctypes.c_double, i32, ctypes.c_double, ctypes.c_double]
+        lib.orc_lps_wait.restype = ctypes.c_double
+        lib.orc_throughput_wait.argtypes = [P, ctypes.c_double]
+        lib.orc_throughput_wait.restype = ctypes.c_double
+        lib.orc_avgcase_ttft.argtypes = [i32, i32, P, P, P, P, P, P]
+        lib.orc_avgcase_ttft.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -208,3 +216,42 @@ def advance(wl, clock, assign, prompt_len, dec, t_now: float, max_batches: int =
     if rc != 0:
         raise RuntimeError(f"oracle advance failed with code {rc}")
     return dataclasses.replace(wl, **st), clk
+
+
+# ---------------------------------------------------------------------------
+# Average-case estimators (Sec. 4 "Average-case TTFT estimation"; App. E)
+
+def pow_int(x: float, k: int) -> float:
+    """x**k by binary exponentiation in fp64 (the order both sides use)."""
+    return float(_load().orc_pow_int(float(x), int(k)))
+
+
+def lps_wait(alpha: float, mu: float, k: int, ca2: float = 1.0, cs2: float = 1.0) -> float:
+    """Expected LPS queueing delay ((ca2 + cs2)/2) * (alpha/mu)^k / (mu - alpha) (App. E)."""
+    return float(_load().orc_lps_wait(float(alpha), float(mu), int(k), float(ca2), float(cs2)))
+
+
+def throughput_wait(wl, theta) -> np.ndarray:
+    """Per instance: remaining prefill tokens of the residents / theta (Sec. 4)."""
+    th = np.broadcast_to(np.asarray(theta, np.float64), (wl.num_instances,))
+    out = np.zeros(wl.num_instances)
+    lib = _load()
+    for j in range(wl.num_instances):
+        rc = _c(wl.run_pre[j], np.int32)
+        wp = _c(wl.wait_pre[j], np.int32)
+        inst = _Instance(int(wl.n_run[j]), None, _p(rc), None, int(wl.n_wait[j]), _p(wp), None)
+        out[j] = lib.orc_throughput_wait(ctypes.byref(inst), float(th[j]))
+    return out
+
+
+def avgcase_matrix(wl, W, theta, tdec):
+    """TTFT[Q][I] = W_j + p_i/theta_j + Tdec_j: canonical fp32 and fp64."""
+    I, Q = wl.num_instances, wl.num_queries
+    Wd, th, td = (np.ascontiguousarray(np.broadcast_to(np.asarray(x, np.float64), (I,))) for x in (W, theta, tdec))
+    p = _c(wl.prompt_len, np.int32)
+    t32 = np.zeros((Q, I), np.float32)
+    t64 = np.zeros((Q, I), np.float64)
+    rc = _load().orc_avgcase_ttft(I, Q, _p(Wd), _p(th), _p(td), _p(p), _p(t32), _p(t64))
+    if rc != 0:
+        raise ValueError(f"oracle average-case estimate failed with code {rc}")
+    return t32, t64

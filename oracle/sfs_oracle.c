@@ -407,3 +407,56 @@ int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, 
     }
     return rc_all;
 }
+
+/* ------------------------------------------------------------------------- */
+/* Average-case estimators (Sec. 4 "Average-case TTFT estimation"; App. E).   */
+
+double orc_pow_int(double x, int32_t k)
+{
+    double r = 1.0, b = x;
+    int32_t e = k;
+    while (e > 0) {
+        if (e & 1) r = r * b;
+        e >>= 1;
+        if (e > 0) b = b * b;
+    }
+    return r;
+}
+
+/* Limited processor sharing: Poisson arrivals at alpha, aggregate service rate mu
+ * shared by at most k active requests, FIFO beyond them.  An arrival that sees n >= k
+ * residents waits for n - k + 1 completions at rate mu; averaging over the M/M/1
+ * stationary law gives rho^k / (mu - alpha).  The G/G/k form scales it by
+ * (ca2 + cs2) / 2, with E[Q] = 1 / mu. */
+double orc_lps_wait(double alpha, double mu, int32_t k, double ca2, double cs2)
+{
+    if (!(mu > 0.0) || !(alpha >= 0.0) || !(alpha < mu) || k < 1) return NAN;
+    const double rho = alpha / mu;
+    const double c = (ca2 + cs2) * 0.5;
+    return (c * orc_pow_int(rho, k)) / (mu - alpha);
+}
+
+double orc_throughput_wait(const orc_instance *inst, double theta)
+{
+    int64_t tokens = 0;
+    for (int32_t r = 0; r < inst->n_run; ++r) tokens += inst->run_pre[r];
+    for (int32_t w = 0; w < inst->n_wait; ++w) tokens += inst->wait_pre[w];
+    return (double)tokens / theta;
+}
+
+int orc_avgcase_ttft(int32_t I, int32_t Q, const double *W, const double *theta, const double *tdec,
+                     const int32_t *prompt_len, float *t32, double *t64)
+{
+    for (int32_t j = 0; j < I; ++j)
+        if (!(theta[j] > 0.0) || !(tdec[j] >= 0.0) || !(W[j] >= 0.0)) return ORC_EINVAL;
+    for (int32_t i = 0; i < Q; ++i) {
+        const int32_t p = prompt_len[i];
+        for (int32_t j = 0; j < I; ++j) {
+            const float g = (float)(1.0 / theta[j]);
+            const float c = (float)(W[j] + tdec[j]);
+            t32[(int64_t)i * I + j] = fmaf((float)p, g, c);
+            t64[(int64_t)i * I + j] = W[j] + (double)p / theta[j] + tdec[j];
+        }
+    }
+    return ORC_OK;
+}

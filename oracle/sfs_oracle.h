@@ -89,6 +89,26 @@ int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, 
 /* Utility of Eq. 2 with the cost of App. B.4 in canonical fp32. */
 float orc_utility(float acc, float lambda, int32_t p, int32_t dec_hat, float price_in, float price_out);
 
+/* ---- Average-case TTFT estimators (Sec. 4 "Average-case TTFT estimation"; App. E) ---- */
+
+/* x^k for an integer k >= 0 by binary exponentiation (bits of k from the least
+ * significant; a fixed sequence of IEEE products). */
+double orc_pow_int(double x, int32_t k);
+
+/* Expected LPS queueing delay (App. E, boxed result; G/G/k correction at its end):
+ * rho = alpha / mu, E[W] = ((ca2 + cs2) / 2) * rho^k / (mu - alpha).  NaN unless
+ * 0 <= alpha < mu, k >= 1. */
+double orc_lps_wait(double alpha, double mu, int32_t k, double ca2, double cs2);
+
+/* Throughput-based waiting time (Sec. 4, prefill-throughput estimator): remaining
+ * prefill tokens of every resident request / theta. */
+double orc_throughput_wait(const orc_instance *inst, double theta);
+
+/* TTFT = W_j + p_i / theta_j + Tdec_j for every query i and instance j (outputs [Q][I]):
+ * canonical fp32 fmaf((float)p, (float)(1 / theta), (float)(W + Tdec)) and fp64. */
+int orc_avgcase_ttft(int32_t I, int32_t Q, const double *W, const double *theta, const double *tdec,
+                     const int32_t *prompt_len, float *t32, double *t64);
+
 #ifdef __cplusplus
 }
 #endif
