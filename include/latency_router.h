@@ -182,6 +182,40 @@ LR_API int lr_route_frontier_static(lr_ctx *ctx, int32_t Q, const int32_t *promp
                                     const float *mu, int32_t *assign_out, float *util_out, double *frontier_out,
                                     void *cuda_stream);
 
+/* Where the TTFT of lr_estimate_ttft and lr_route (and lr_route_frontier_static) comes from. */
+enum lr_ttft_source {
+    LR_TTFT_SFS = 0,         /* Serving Framework Simulation of the live snapshot (Sec. 4.1), the default */
+    LR_TTFT_THROUGHPUT = 1,  /* prefill-throughput estimator (Sec. 4): W_j = remaining prefill tokens of
+                                the snapshot's residents / theta_j */
+    LR_TTFT_LPS = 2          /* average-case estimator (Sec. 4, App. E): W_j = ((ca2 + cs2) / 2) *
+                                (alpha_j / mu_j)^k_j / (mu_j - alpha_j); needs no snapshot */
+};
+
+/* Per-instance parameters of the average-case sources; host arrays of length I, copied.
+ * TTFT_ij = W_j + p_i / theta_j + Tdec_j, evaluated as
+ * fmaf((float)p, fp32(1 / theta_j), fp32(W_j + Tdec_j)) with W_j and the divisions in fp64
+ * ((alpha/mu)^k by binary exponentiation over the bits of k from the least significant). */
+typedef struct {
+    const double *prefill_tput;       /* theta_j, prefill tokens per second, finite > 0 */
+    const double *decode_batch_time;  /* Tdec_j, average decode-batch time (s), finite >= 0 */
+    const double *arrival_rate;       /* alpha_j, queries/s, 0 <= alpha_j < mu_j; NULL: no LPS source */
+    const double *service_rate;       /* mu_j, queries/s (App. E: from peak output throughput) */
+    const int32_t *parallelism;       /* k_j, concurrent sequences, 1 .. 2^20 */
+    const double *arrival_scv;        /* ca^2_j >= 0 of inter-arrival times, NULL: 1 (Poisson) */
+    const double *service_scv;        /* cs^2_j >= 0 of service requirements, NULL: 1 (exponential) */
+} lr_queue_params;
+
+/* Validate and upload the queue parameters (LR_EINVAL, nothing changed, on a bad value);
+ * ordered on cuda_stream like the other calls. */
+LR_API int lr_set_queue_params(lr_ctx *ctx, const lr_queue_params *params, void *cuda_stream);
+
+/* Select the TTFT source (lr_ttft_source).  The average-case sources need
+ * lr_set_queue_params first (LPS: with rates), else LR_EINVAL.  first_batch_out of
+ * lr_estimate_ttft and lr_estimate_features describe the SFS only; first_batch_out with
+ * another source is LR_EINVAL.  The throughput source reads the live snapshot
+ * (LR_ENOSTATE before one is loaded); the LPS source reads none. */
+LR_API int lr_set_ttft_source(lr_ctx *ctx, int32_t source);
+
 /* Online stream step (Sec. 5: queries arrive over time and are routed as they come;
  * App. F: every instance keeps executing token batches and publishes its state after each).
  * The queries with assign[i] >= 0 join instance assign[i]'s waiting tail in query order

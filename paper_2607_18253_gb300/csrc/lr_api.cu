@@ -22,6 +22,11 @@ struct lr_ctx {
     int max_seqs = 0;
     size_t k3_smem = 0;
     float *scratch_tch = nullptr;
+    // average-case TTFT sources
+    lr::QueueRaw *qraw = nullptr;
+    lr::QueueDev *qd = nullptr;
+    int source = lr::kSrcSfs;
+    bool have_qp = false, have_lps = false;
     std::vector<void *> allocs;
     std::string err;
     int max_queries = 0, max_pairs = 0;
@@ -118,6 +123,8 @@ lr::K2Launch k2_base(const lr_ctx *c) {
     a.buf0 = c->buf[0];
     a.buf1 = c->buf[1];
     a.ctl = c->ctl;
+    a.src = c->source;
+    a.qd = c->qd;
     return a;
 }
 
@@ -235,6 +242,8 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     }
     LR_ALLOC(c->ctl, 1);
     LR_ALLOC(c->scratch_tch, (size_t)cfg->max_pairs * cfg->max_queries);
+    LR_ALLOC(c->qraw, I);
+    LR_ALLOC(c->qd, I);
 #undef LR_ALLOC
     e = cudaMemcpy(moi, cfg->model_of_instance, I * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(B, cfg->max_batched_tokens, I * 4, cudaMemcpyHostToDevice);
@@ -308,6 +317,8 @@ static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, 
     if (Q > c->max_queries) return fail(c, LR_ECAPACITY, "Q exceeds max_queries");
     if (Q == 0) return LR_OK;
     if (!p || (!ttft && !feat)) return fail(c, LR_EINVAL, "null array");
+    if (iters && c->source != lr::kSrcSfs)
+        return fail(c, LR_EINVAL, "first_batch_out exists only for the SFS source");
     lr::K2Launch a = k2_base(c);
     a.Q = Q;
     a.prompt = p;
@@ -433,6 +444,60 @@ int lr_route_frontier_static(lr_ctx *c, int32_t Q, const int32_t *prompt_len, co
     // the intermediate's storage differs
     return lr_route(c, Q, prompt_len, dec_hat, acc, tau, P, lambda, mu, assign_out, util_out, tch, frontier_out,
                     nullptr, stream);
+}
+
+int lr_set_queue_params(lr_ctx *c, const lr_queue_params *qp, void *stream) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    if (!qp || !qp->prefill_tput || !qp->decode_batch_time) return fail(c, LR_EINVAL, "null queue parameters");
+    const bool lps = qp->arrival_rate != nullptr;
+    if (lps && (!qp->service_rate || !qp->parallelism))
+        return fail(c, LR_EINVAL, "arrival_rate needs service_rate and parallelism");
+    const int I = c->cfg.I;
+    std::vector<lr::QueueRaw> raw(I);
+    for (int j = 0; j < I; ++j) {
+        lr::QueueRaw r;
+        std::memset(&r, 0, sizeof(r));
+        r.theta = qp->prefill_tput[j];
+        r.tdec = qp->decode_batch_time[j];
+        if (!(std::isfinite(r.theta) && r.theta > 0.0)) return fail(c, LR_EINVAL, "prefill_tput must be finite and > 0");
+        if (!(std::isfinite(r.tdec) && r.tdec >= 0.0))
+            return fail(c, LR_EINVAL, "decode_batch_time must be finite and >= 0");
+        if (lps) {
+            r.alpha = qp->arrival_rate[j];
+            r.mu = qp->service_rate[j];
+            r.k = qp->parallelism[j];
+            r.ca2 = qp->arrival_scv ? qp->arrival_scv[j] : 1.0;
+            r.cs2 = qp->service_scv ? qp->service_scv[j] : 1.0;
+            r.has_lps = 1;
+            if (!(std::isfinite(r.alpha) && r.alpha >= 0.0 && std::isfinite(r.mu) && r.alpha < r.mu))
+                return fail(c, LR_EINVAL, "rates must satisfy 0 <= arrival_rate < service_rate (finite)");
+            if (r.k < 1 || r.k > (1 << 20)) return fail(c, LR_EINVAL, "parallelism must be in [1, 2^20]");
+            if (!(std::isfinite(r.ca2) && r.ca2 >= 0.0 && std::isfinite(r.cs2) && r.cs2 >= 0.0))
+                return fail(c, LR_EINVAL, "squared coefficients of variation must be finite and >= 0");
+        }
+        raw[j] = r;
+    }
+    cudaStream_t st = (cudaStream_t)stream;
+    // pageable source: the copy has read the vector when the call returns
+    cudaError_t e = cudaMemcpyAsync(c->qraw, raw.data(), sizeof(lr::QueueRaw) * I, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) e = lr::launch_queue_params(I, c->qraw, c->qd, st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "queue parameters");
+    c->have_qp = true;
+    c->have_lps = lps;
+    if (c->source == lr::kSrcLps && !lps) c->source = lr::kSrcSfs;
+    return LR_OK;
+}
+
+int lr_set_ttft_source(lr_ctx *c, int32_t source) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    if (source != LR_TTFT_SFS && source != LR_TTFT_THROUGHPUT && source != LR_TTFT_LPS)
+        return fail(c, LR_EINVAL, "unknown TTFT source");
+    if (source != LR_TTFT_SFS && !c->have_qp) return fail(c, LR_EINVAL, "set the queue parameters first");
+    if (source == LR_TTFT_LPS && !c->have_lps) return fail(c, LR_EINVAL, "the LPS source needs arrival and service rates");
+    c->source = source;
+    return LR_OK;
 }
 
 int lr_advance(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_t *prompt_len, const int32_t *dec,

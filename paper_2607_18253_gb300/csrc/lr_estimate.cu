@@ -212,9 +212,13 @@ struct Flag {
     static constexpr bool value = B;
 };
 
+// MODE 0 / 1: SFS with the first output token in its own batch / with the last
+// prompt chunk.  MODE 2: an average-case source (Sec. 4, App. E), affine in p:
+// t = fma(p, g_j, C_j) with g_j = fp32(1/theta_j) and C_j = fp32(W_j + Tdec_j).
 template <int MODE, int OUT>
 __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     extern __shared__ __align__(16) unsigned char smem[];
+    constexpr bool AFF = MODE == 2;
     constexpr bool ROUTE = (OUT & (kOutLag | kOutCon | kOutSweep)) != 0;
     constexpr bool CON = (OUT & kOutCon) != 0;
     constexpr bool SWEEP = (OUT & kOutSweep) != 0;
@@ -232,7 +236,8 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     const int re = min(a.Q, rb + rows_per);
     if (rb >= re) return;
     const int active = *((volatile int32_t *)&a.ctl->active);
-    if (active < 0) {
+    // the LPS source needs no live snapshot; every other source does
+    if (active < 0 && !(AFF && a.src == kSrcLps)) {
         if (threadIdx.x == 0) record_status(a.ctl, kENoState);
         for (int rr = rb + qs; rr < re; rr += QS) {
             for (int u = 0; u < nv; ++u) {
@@ -266,14 +271,14 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     int32_t *r_d = reinterpret_cast<int32_t *>(r_t + (ROUTE ? 2 * QT : 0));
     float *r_a = reinterpret_cast<float *>(r_d + (ROUTE ? 2 * QT * M : 0));
 
-    for (int idx = threadIdx.x; idx < c.kph * 4 * Gp; idx += blockDim.x) {
+    for (int idx = threadIdx.x; !AFF && idx < c.kph * 4 * Gp; idx += blockDim.x) {
         const int k = idx / (4 * Gp);
         const int rem = idx - k * 4 * Gp;
         const int u = rem / Gp;
         const int jg = j0 + 4 * (rem - u * Gp) + u;
         s_ent[idx] = jg < I ? sb.ent[(size_t)k * I + jg] : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    for (int idx = threadIdx.x; idx < c.nbh * 4 * Gp; idx += blockDim.x) {
+    for (int idx = threadIdx.x; !AFF && idx < c.nbh * 4 * Gp; idx += blockDim.x) {
         const int b = idx / (4 * Gp);
         const int rem = idx - b * 4 * Gp;
         const int u = rem / Gp;
@@ -282,10 +287,21 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     }
     Inst4 r;
     int model[4], la[4];
+    float ag[4], ac[4];  // average-case sources: t = fma(p, ag, ac)
     bool fast_mine = true;
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
         const int j = min(jb + u, I - 1);
+        model[u] = c.moi[j];
+        if (AFF) {
+            const QueueDev qd = a.qd[j];
+            ag[u] = qd.g;
+            // throughput source: residents' remaining prefill tokens / theta + Tdec
+            ac[u] = (a.src == kSrcLps)
+                        ? qd.clps
+                        : __double2float_rn(__dadd_rn(__ddiv_rn((double)sb.inst[j].f1tot, qd.theta), qd.tdec));
+            continue;
+        }
         const InstParams ip = sb.inst[j];
         const int m = c.moi[j];
         r.shift[u] = ip.shift;
@@ -375,6 +391,11 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                 int kk[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
+                    if (AFF) {
+                        t[u] = __fmaf_rn(q.fp, ag[u], ac[u]);
+                        kk[u] = 0;
+                        continue;
+                    }
                     const int2 bk = lds_int2(bcol[u] + (uint32_t)(q.p >> r.shift[u]) * brow);
                     kk[u] = bk.y + (q.p > bk.x ? 1 : 0);
                     const float4 e = lds_float4(ecol[u] + (uint32_t)kk[u] * erow);
@@ -523,7 +544,10 @@ template <int MODE>
 cudaError_t launch_cand_mode(const K2Launch &a, int out, dim3 grid, int block, size_t smem, cudaStream_t st) {
     switch (out) {
         case kOutMatrix: k_cand<MODE, kOutMatrix><<<grid, block, smem, st>>>(a); break;
-        case kOutMatrix | kOutIters: k_cand<MODE, kOutMatrix | kOutIters><<<grid, block, smem, st>>>(a); break;
+        case kOutMatrix | kOutIters:
+            if (MODE == 2) return cudaErrorInvalidValue;  // the batch index exists only for SFS
+            k_cand<(MODE == 2 ? 0 : MODE), kOutMatrix | kOutIters><<<grid, block, smem, st>>>(a);
+            break;
         case kOutLag: k_cand<MODE, kOutLag><<<grid, block, smem, st>>>(a); break;
         case kOutLag | kOutMatrix: k_cand<MODE, kOutLag | kOutMatrix><<<grid, block, smem, st>>>(a); break;
         case kOutCon: k_cand<MODE, kOutCon><<<grid, block, smem, st>>>(a); break;
@@ -543,7 +567,7 @@ cudaError_t set_attr(F f, size_t bytes) {
 template <int MODE>
 cudaError_t set_mode_attrs(size_t bytes) {
     const cudaError_t es[] = {
-        set_attr(k_cand<MODE, kOutMatrix>, bytes), set_attr(k_cand<MODE, kOutMatrix | kOutIters>, bytes),
+        set_attr(k_cand<MODE, kOutMatrix>, bytes), set_attr(k_cand<(MODE == 2 ? 0 : MODE), kOutMatrix | kOutIters>, bytes),
         set_attr(k_cand<MODE, kOutLag>, bytes), set_attr(k_cand<MODE, kOutLag | kOutMatrix>, bytes),
         set_attr(k_cand<MODE, kOutCon>, bytes), set_attr(k_cand<MODE, kOutCon | kOutMatrix>, bytes),
         set_attr(k_cand<MODE, kOutSweep>, bytes), set_attr(k_cand<MODE, kOutSweep | kOutMatrix>, bytes)};
@@ -563,8 +587,50 @@ int cand_out_flags(bool matrix, bool iters, bool route, bool constrained, int P)
 }
 
 cudaError_t launch_cand(const K2Launch &a, int out, dim3 grid, int block, size_t smem, cudaStream_t st) {
+    if (a.src != kSrcSfs) return launch_cand_mode<2>(a, out, grid, block, smem, st);
     return a.cfg.mode == 0 ? launch_cand_mode<0>(a, out, grid, block, smem, st)
                            : launch_cand_mode<1>(a, out, grid, block, smem, st);
+}
+
+namespace {
+
+// x^k, k >= 0, by binary exponentiation (the bits of k from the least significant).
+__device__ double pow_int(double x, int k) {
+    double r = 1.0, b = x;
+    while (k > 0) {
+        if (k & 1) r = __dmul_rn(r, b);
+        k >>= 1;
+        if (k > 0) b = __dmul_rn(b, b);
+    }
+    return r;
+}
+
+// Per instance: the LPS expected wait of App. E, ((ca2 + cs2) / 2) rho^k / (mu - alpha)
+// with rho = alpha / mu, and the fp32 constants of the affine TTFT.
+__global__ void k_queue_params(int I, const QueueRaw *raw, QueueDev *qd) {
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= I) return;
+    const QueueRaw r = raw[j];
+    double w = __longlong_as_double(0x7ff8000000000000LL);
+    if (r.has_lps) {
+        const double rho = __ddiv_rn(r.alpha, r.mu);
+        const double c = __dmul_rn(__dadd_rn(r.ca2, r.cs2), 0.5);
+        w = __ddiv_rn(__dmul_rn(c, pow_int(rho, r.k)), __dsub_rn(r.mu, r.alpha));
+    }
+    QueueDev o;
+    o.theta = r.theta;
+    o.tdec = r.tdec;
+    o.wlps = w;
+    o.g = __double2float_rn(__ddiv_rn(1.0, r.theta));
+    o.clps = __double2float_rn(__dadd_rn(w, r.tdec));
+    qd[j] = o;
+}
+
+}  // namespace
+
+cudaError_t launch_queue_params(int I, const QueueRaw *raw, QueueDev *qd, cudaStream_t st) {
+    k_queue_params<<<(I + 127) / 128, 128, 0, st>>>(I, raw, qd);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_features(const K2Launch &a, int sms, cudaStream_t st) {
@@ -582,6 +648,7 @@ cudaError_t launch_frontier(const K2Launch &a, double *out, cudaStream_t st) {
 cudaError_t set_k2_smem(size_t bytes) {
     cudaError_t e = set_mode_attrs<0>(bytes);
     if (e == cudaSuccess) e = set_mode_attrs<1>(bytes);
+    if (e == cudaSuccess) e = set_mode_attrs<2>(bytes);
     return e;
 }
 

@@ -112,6 +112,22 @@ __host__ __device__ inline size_t trajectory_smem_per_warp(const DevConfig &c) {
     return sizeof(int32_t) * ((words + 3) & ~(size_t)3);
 }
 
+// Average-case TTFT sources (Sec. 4, App. E): per-instance parameters as given
+// and the derived constants of t = fma(p, g, C).
+enum : int { kSrcSfs = 0, kSrcThroughput = 1, kSrcLps = 2 };
+struct QueueRaw {      // 64 bytes, copied from the caller's arrays
+    double theta, tdec, alpha, mu, ca2, cs2;
+    int32_t k, has_lps;
+    int32_t pad[2];
+};
+struct QueueDev {      // 32 bytes
+    double theta, tdec;
+    double wlps;       // LPS expected wait (NaN without queue rates)
+    float g;           // fp32(1 / theta)
+    float clps;        // fp32(wlps + tdec)
+};
+cudaError_t launch_queue_params(int I, const QueueRaw *raw, QueueDev *qd, cudaStream_t st);
+
 struct K2Launch {
     DevConfig cfg;
     StateBuf buf0, buf1;
@@ -135,6 +151,9 @@ struct K2Launch {
     // launch shape: Gp thread groups of four instances per row (a power of two up
     // to 32, else a multiple of 32), QS rows in flight, QT rows per staged chunk
     int32_t Gp, QS, QT, vec_ok;
+    // TTFT source (kSrc*) and, for the average-case ones, the instance constants
+    int32_t src;
+    const QueueDev *qd;
 };
 int cand_out_flags(bool matrix, bool iters, bool route, bool constrained, int P);
 cudaError_t launch_cand(const K2Launch &a, int out, dim3 grid, int block, size_t smem, cudaStream_t st);

@@ -20,10 +20,11 @@ LIB_PATH = os.path.join(_PKG, "_lib", "liblr.so")
 LR_OK, LR_EINVAL, LR_ENOMEM, LR_ECUDA, LR_ECAPACITY, LR_ETRAJ, LR_ESTATE, LR_ENOSTATE = range(8)
 FIRST_TOKEN_SEPARATE_DECODE = 0
 FIRST_TOKEN_WITH_LAST_CHUNK = 1
+LR_TTFT_SFS, LR_TTFT_THROUGHPUT, LR_TTFT_LPS = 0, 1, 2
 
 EXPORTED_SYMBOLS = ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
                     "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
-                    "lr_strerror", "lr_last_error")
+                    "lr_set_queue_params", "lr_set_ttft_source", "lr_strerror", "lr_last_error")
 
 _P = ctypes.c_void_p
 _I32 = ctypes.c_int32
@@ -34,6 +35,11 @@ class _Config(ctypes.Structure):
                 ("price_in", _P), ("price_out", _P), ("max_batched_tokens", _P), ("max_seqs", _P),
                 ("cap_running", _I32), ("cap_waiting", _I32), ("max_queries", _I32), ("max_pairs", _I32),
                 ("max_prompt_len", _I32), ("first_token_mode", _I32), ("max_iters", _I32)]
+
+
+class _QueueParams(ctypes.Structure):
+    _fields_ = [("prefill_tput", _P), ("decode_batch_time", _P), ("arrival_rate", _P), ("service_rate", _P),
+                ("parallelism", _P), ("arrival_scv", _P), ("service_scv", _P)]
 
 
 class _StateView(ctypes.Structure):
@@ -60,6 +66,8 @@ def load_library(path: str = LIB_PATH):
     lib.lr_route.argtypes = [_P, _I32, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.lr_route_frontier_static.argtypes = [_P, _I32, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P]
     lib.lr_advance.argtypes = [_P, _I32, _P, _P, _P, _I32, ctypes.c_double, _P]
+    lib.lr_set_queue_params.argtypes = [_P, ctypes.POINTER(_QueueParams), _P]
+    lib.lr_set_ttft_source.argtypes = [_P, _I32]
     lib.lr_read_state.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.lr_status.argtypes = [_P, _P]
     lib.lr_strerror.argtypes = [ctypes.c_int]
@@ -67,7 +75,8 @@ def load_library(path: str = LIB_PATH):
     lib.lr_last_error.argtypes = [_P]
     lib.lr_last_error.restype = ctypes.c_char_p
     for name in ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
-                 "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status"):
+                 "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
+                 "lr_set_queue_params", "lr_set_ttft_source"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -240,6 +249,24 @@ class LatencyRouter:
             _dev(o["frontier"], torch.float64, "frontier_out", P * 3), _stream(stream))
         self._check(rc, "lr_route_frontier_static")
         return o
+
+    def set_queue_params(self, prefill_tput, decode_batch_time, arrival_rate=None, service_rate=None,
+                         parallelism=None, arrival_scv=None, service_scv=None, stream=None):
+        """Per-instance parameters of the average-case TTFT sources (host arrays of length I)."""
+        I = self.num_instances
+
+        def arr(x, dt):
+            return None if x is None else np.ascontiguousarray(np.broadcast_to(np.asarray(x, dt), (I,)))
+
+        keep = [arr(prefill_tput, np.float64), arr(decode_batch_time, np.float64), arr(arrival_rate, np.float64),
+                arr(service_rate, np.float64), arr(parallelism, np.int32), arr(arrival_scv, np.float64),
+                arr(service_scv, np.float64)]
+        qp = _QueueParams(*(None if k is None else k.ctypes.data_as(_P) for k in keep))
+        self._check(self._lib.lr_set_queue_params(self._h, ctypes.byref(qp), _stream(stream)), "lr_set_queue_params")
+
+    def set_ttft_source(self, source: int):
+        """LR_TTFT_SFS (default), LR_TTFT_THROUGHPUT or LR_TTFT_LPS."""
+        self._check(self._lib.lr_set_ttft_source(self._h, int(source)), "lr_set_ttft_source")
 
     def advance(self, assign: torch.Tensor, prompt_len: torch.Tensor, dec: torch.Tensor, t_now: float,
                 stream=None):
