@@ -405,7 +405,7 @@ def pool_capacity(R, W, wl, dev, horizon=300.0, warm=30.0, dt=2.0, depth=256):
 
 
 def run_stream(args, dev):
-    """Online stream: Poisson arrivals at 0.8 x pool capacity, routed in micro-batches.
+    """Online stream: arrivals at 0.8 x pool capacity (Poisson, and bursty MMPP-2), routed in micro-batches.
 
     At each decision time (the arrival of the batch's last query) the pool is advanced
     to that time with the previous batch appended to its chosen instances (K3 + K1),
@@ -422,7 +422,8 @@ def run_stream(args, dev):
     I, M = wl.num_instances, wl.num_models
     cap = pool_capacity(R, W, wl, dev)
     rate = 0.8 * float(cap.sum())
-    arr = W.poisson_arrivals(STREAM_QUERIES, rate, STREAM_SEED)
+    traces = [("poisson", W.poisson_arrivals(STREAM_QUERIES, rate, STREAM_SEED), STREAM_SIZES),
+              ("mmpp2_r6", W.mmpp2_arrivals(STREAM_QUERIES, rate, 6.0, STREAM_SEED), (16, 256))]
     mmax = max(STREAM_SIZES)
     rt = R.LatencyRouter.from_workload(wl, max_queries=mmax)
     state = R.state_tensors(wl, dev)
@@ -437,50 +438,52 @@ def run_stream(args, dev):
     ap = [assign[0].data_ptr(), assign[1].data_ptr()]
     lamp, mup = lam.ctypes.data_as(ctypes.c_void_p), mu.ctypes.data_as(ctypes.c_void_p)
     V = ctypes.c_void_p
-    out = {"workload": f"{STREAM_WORKLOAD} state and pool (seed {STREAM_SEED}), {STREAM_QUERIES} Poisson arrivals",
+    out = {"workload": f"{STREAM_WORKLOAD} state and pool (seed {STREAM_SEED}), {STREAM_QUERIES} arrivals: Poisson, "
+                       f"and MMPP-2 (rate ratio 6, 20% of time in the high state, switching 0.1/s and 0.4/s)",
            "capacity_qps": float(cap.sum()), "arrival_qps": rate,
            "capacity_reading": "completions/s of each instance under a saturating FCFS stream, t = 30..300 s",
            "latency": "device time of advance (K3 + K1) + route (K2) per micro-batch, CUDA events",
-           "sizes": {}}
+           "sizes": {}, "mmpp2_r6": {}}
     launches = 0
-    for m in STREAM_SIZES:
-        nq = STREAM_QUERIES if (m > 1 or args.stream_full) else min(STREAM_QUERIES, args.stream_queries_b1)
-        nb = nq // m
-        rt.load_state(*state)
-        chunk = 4096
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(chunk)]
-        lat = []
-        torch.cuda.synchronize()
-        w0 = time.perf_counter()
-        for b in range(nb):
-            lo = b * m
-            cur, prev = ap[b & 1], ap[(b - 1) & 1]
-            e0, e1 = ev[b % chunk]
-            e0.record()
-            # previous batch joins its instances' queues; every instance advances to now
-            pm = m if b > 0 else 0
-            plo = (b - 1) * m
-            rc = lib.lr_advance(h, pm, V(prev), V(pp + 4 * max(plo, 0)), V(dhp + 4 * M * max(plo, 0)), M,
-                                ctypes.c_double(float(arr[lo + m - 1])), sp)
-            rc |= lib.lr_route(h, m, V(pp + 4 * lo), V(dhp + 4 * M * lo), V(accp + 4 * M * lo), None, 1, lamp,
-                               mup, V(cur), V(util.data_ptr()), None, None, None, sp)
-            e1.record()
-            if rc:
-                raise RuntimeError(f"stream call failed: {lib.lr_last_error(h).decode()}")
-            if b % chunk == chunk - 1 or b == nb - 1:
-                torch.cuda.synchronize()
-                lat += [ev[k][0].elapsed_time(ev[k][1]) for k in range(b % chunk + 1)]
-        wall = time.perf_counter() - w0
-        st = rt.status()
-        if st != R.LR_OK:
-            raise RuntimeError(f"stream run (micro-batch {m}) ended with device status {st}")
-        launches += 3 * nb
-        q = np.percentile(np.asarray(lat) * 1e3, [50, 99])
-        fin = rt.read_state(device=dev)
-        out["sizes"][str(m)] = {"batches": nb, "queries": nb * m, "p50_us": float(q[0]), "p99_us": float(q[1]),
-                                "mean_us": float(np.mean(lat) * 1e3), "wall_s": wall,
-                                "simulated_s": float(arr[nb * m - 1]),
-                                "final_mean_waiting": float(fin["n_wait"].float().mean().item())}
+    for label, arr, sizes in traces:
+        for m in sizes:
+            nq = STREAM_QUERIES if (m > 1 or args.stream_full) else min(STREAM_QUERIES, args.stream_queries_b1)
+            nb = nq // m
+            rt.load_state(*state)
+            chunk = 4096
+            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(chunk)]
+            lat = []
+            torch.cuda.synchronize()
+            w0 = time.perf_counter()
+            for b in range(nb):
+                lo = b * m
+                cur, prev = ap[b & 1], ap[(b - 1) & 1]
+                e0, e1 = ev[b % chunk]
+                e0.record()
+                # previous batch joins its instances' queues; every instance advances to now
+                pm = m if b > 0 else 0
+                plo = (b - 1) * m
+                rc = lib.lr_advance(h, pm, V(prev), V(pp + 4 * max(plo, 0)), V(dhp + 4 * M * max(plo, 0)), M,
+                                    ctypes.c_double(float(arr[lo + m - 1])), sp)
+                rc |= lib.lr_route(h, m, V(pp + 4 * lo), V(dhp + 4 * M * lo), V(accp + 4 * M * lo), None, 1, lamp,
+                                   mup, V(cur), V(util.data_ptr()), None, None, None, sp)
+                e1.record()
+                if rc:
+                    raise RuntimeError(f"stream call failed: {lib.lr_last_error(h).decode()}")
+                if b % chunk == chunk - 1 or b == nb - 1:
+                    torch.cuda.synchronize()
+                    lat += [ev[k][0].elapsed_time(ev[k][1]) for k in range(b % chunk + 1)]
+            wall = time.perf_counter() - w0
+            st = rt.status()
+            if st != R.LR_OK:
+                raise RuntimeError(f"stream run ({label}, micro-batch {m}) ended with device status {st}")
+            launches += 3 * nb
+            q = np.percentile(np.asarray(lat) * 1e3, [50, 99])
+            fin = rt.read_state(device=dev)
+            res = {"batches": nb, "queries": nb * m, "p50_us": float(q[0]), "p99_us": float(q[1]),
+                   "mean_us": float(np.mean(lat) * 1e3), "wall_s": wall, "simulated_s": float(arr[nb * m - 1]),
+                   "final_mean_waiting": float(fin["n_wait"].float().mean().item())}
+            out["sizes" if label == "poisson" else label][str(m)] = res
     out["gpu_launches"] = launches
     rt.close()
     return out

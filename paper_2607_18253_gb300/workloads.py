@@ -233,6 +233,37 @@ def poisson_arrivals(num_queries: int, rate_qps: float, seed: int) -> np.ndarray
     return np.cumsum(rng.exponential(1.0 / rate_qps, num_queries))
 
 
+def mmpp2_rates(mean_qps: float, ratio: float, p_high: float = 0.2):
+    """Low- and high-state rates of a two-state MMPP with long-run mean `mean_qps`,
+    high/low rate ratio `ratio` and a fraction `p_high` of time in the high state."""
+    low = mean_qps / ((1.0 - p_high) + p_high * ratio)
+    return low, ratio * low
+
+
+def mmpp2_arrivals(num_queries: int, mean_qps: float, ratio: float, seed: int, z_lh: float = 0.1,
+                   z_hl: float = 0.4) -> np.ndarray:
+    """Arrival times (s, fp64) of a two-state Markov-modulated Poisson process.
+
+    The latent state switches low->high at rate z_lh and high->low at z_hl (so it
+    spends z_lh / (z_lh + z_hl) of the time high); within a sojourn of length d at
+    rate a, the arrivals are a Poisson(a d) count of uniform times.  The state
+    starts from its stationary law."""
+    p_high = z_lh / (z_lh + z_hl)
+    low, high_rate = mmpp2_rates(mean_qps, ratio, p_high)
+    rng = np.random.default_rng(np.random.SeedSequence([seed, 0x3A77]))
+    high = bool(rng.random() < p_high)
+    t, total, parts = 0.0, 0, []
+    while total < num_queries:
+        d = rng.exponential(1.0 / (z_hl if high else z_lh))
+        k = int(rng.poisson((high_rate if high else low) * d))
+        if k:
+            parts.append(t + np.sort(rng.uniform(0.0, d, k)))
+            total += k
+        t += d
+        high = not high
+    return np.concatenate(parts)[:num_queries]
+
+
 def sweep_pairs():
     """The trade-off grid: 4 lambda values (log 0.1..10) x 8 mu values (log 0.01..1 /s), lambda-major."""
     lam = np.logspace(-1, 1, 4)
