@@ -101,7 +101,8 @@ lr_ctx::Shape make_shape(const lr::DevConfig &d, bool route, int max_pairs) {
     s.tiles = (d.I + 4 * s.Gp - 1) / (4 * s.Gp);
     s.QS = lr::kK2Block / s.Gp;
     const int wpr = s.Gp > 32 ? s.Gp / 32 : 1;
-    const size_t tables = (size_t)d.kph * 4 * s.Gp * 16 + (size_t)d.nbh * 4 * s.Gp * 8;
+    // the tile block (tables and per-instance scalars), brought in by one bulk copy
+    const size_t tables = (size_t)d.kph * 4 * s.Gp * 16 + (size_t)d.nbh * 4 * s.Gp * 8 + (size_t)lr::kScal * 4 * s.Gp * 4;
     const size_t part = s.Gp > 32 ? 2 * (size_t)wpr * 16 * max_pairs : 0;  // wide-row partials per pair
     // staged row (16 B) and two raw copies of its prompt; routing adds the wide-row
     // partials, (cost, acc) per model, tau, and two raw copies of tau, dec_hat and acc
@@ -193,6 +194,11 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     d.max_iters = cfg->max_iters;
     d.kph = kph;
     d.nbh = nbh;
+    {
+        // thread groups per instance tile of the candidate kernel (as make_shape chooses)
+        const int G = (I + 3) / 4;
+        d.tgp = std::min(G <= 32 ? pow2_ceil(G) : round_up(G, 32), lr::kK2Block);
+    }
     c->max_queries = cfg->max_queries;
     c->max_pairs = cfg->max_pairs;
 
@@ -224,7 +230,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
         LR_ALLOC(s.clock, I);
         LR_ALLOC(s.inst, I);
         LR_ALLOC(s.bkt, (size_t)nbh * I);
-        LR_ALLOC(s.ent, (size_t)kph * I);
+        LR_ALLOC(s.tile, (size_t)lr::tile_count(d) * lr::tile_bytes(d));
         LR_ALLOC(s.f2, (size_t)kph * I);
         LR_ALLOC(s.f3, (size_t)kph * I);
         LR_ALLOC(s.rcum, (size_t)kph * I);
@@ -264,6 +270,12 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     d.coef = coef;
     d.pin = pin;
     d.pout = pout;
+    if (I % (4 * d.tgp) != 0) {
+        e = lr::launch_tile_pad(d, c->buf[0].tile, 0);
+        if (e == cudaSuccess) e = lr::launch_tile_pad(d, c->buf[1].tile, 0);
+        if (e == cudaSuccess) e = cudaDeviceSynchronize();
+        if (e != cudaSuccess) return bail(LR_ECUDA, cudaGetErrorString(e));
+    }
 
     // K1: one warp per instance.
     c->k1_smem = lr::kK1Warps * lr::trajectory_smem_per_warp(d);

@@ -207,6 +207,17 @@ __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
+// One poll of an mbarrier's phase 0 (true once the bulk copy it tracks has landed).
+__device__ __forceinline__ bool mbar_test(uint32_t mbar) {
+    uint32_t done;
+    asm volatile(
+        "{\n .reg .pred P;\n mbarrier.try_wait.parity.shared::cta.b64 P, [%1], 0;\n selp.u32 %0, 1, 0, P;\n}"
+        : "=r"(done)
+        : "r"(mbar)
+        : "memory");
+    return done != 0;
+}
+
 template <bool B>
 struct Flag {
     static constexpr bool value = B;
@@ -254,15 +265,18 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
         return;
     }
     const StateBuf sb = active ? a.buf1 : a.buf0;
-    // shared memory: tables, query records, row partials, utility inputs, targets
-    // (route with one pair stages (U, cost) per row and model, sweeps (cost, acc))
+    // Shared memory: the tile block (tables and per-instance scalars, exactly as K1
+    // laid it out for this tile), query records, row partials, utility inputs,
+    // targets and the raw query rows (route with one pair stages (U, cost) per row
+    // and model, sweeps (cost, acc)).
     const int WPR = Gp > 32 ? Gp / 32 : 1;  // warps per row
     const int NP = SWEEP ? a.P : 1;
     float4 *s_ent = reinterpret_cast<float4 *>(smem);                                  // [kph][4][Gp]
-    QRec *s_q = reinterpret_cast<QRec *>(s_ent + c.kph * 4 * Gp);                      // [QT]
+    int2 *s_bkt = reinterpret_cast<int2 *>(s_ent + c.kph * 4 * Gp);                    // [nbh][4][Gp]
+    const int32_t *s_scal = reinterpret_cast<const int32_t *>(s_bkt + c.nbh * 4 * Gp);  // [kScal][4][Gp]
+    QRec *s_q = reinterpret_cast<QRec *>(smem + tile_bytes(c));                        // [QT]
     int4 *s_part = reinterpret_cast<int4 *>(s_q + QT);                                 // [NP][QT][WPR][2]
-    int2 *s_bkt = reinterpret_cast<int2 *>(s_part + (ROUTE && Gp > 32 ? 2 * NP * QT * WPR : 0));  // [nbh][4][Gp]
-    float2 *s_ca = reinterpret_cast<float2 *>(s_bkt + c.nbh * 4 * Gp);                 // [QT][M] (cost, acc)
+    float2 *s_ca = reinterpret_cast<float2 *>(s_part + (ROUTE && Gp > 32 ? 2 * NP * QT * WPR : 0));  // [QT][M]
     float *s_tau = reinterpret_cast<float *>(s_ca + (ROUTE ? QT * M : 0));             // [QT]
     // raw query rows as copied from global memory, two chunks in flight:
     // prompt [2][QT], and for routing tau [2][QT], dec_hat [2][QT][M], acc [2][QT][M]
@@ -271,29 +285,66 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     int32_t *r_d = reinterpret_cast<int32_t *>(r_t + (ROUTE ? 2 * QT : 0));
     float *r_a = reinterpret_cast<float *>(r_d + (ROUTE ? 2 * QT * M : 0));
 
-    for (int idx = threadIdx.x; !AFF && idx < c.kph * 4 * Gp; idx += blockDim.x) {
-        const int k = idx / (4 * Gp);
-        const int rem = idx - k * 4 * Gp;
-        const int u = rem / Gp;
-        const int jg = j0 + 4 * (rem - u * Gp) + u;
-        s_ent[idx] = jg < I ? sb.ent[(size_t)k * I + jg] : make_float4(0.f, 0.f, 0.f, 0.f);
+    // The tile block arrives with one bulk copy (TMA) completing on an mbarrier:
+    // every CTA reads the same few tens of KB, and one large request per CTA is far
+    // cheaper than thousands of scattered loads of the same lines.
+    __shared__ __align__(8) unsigned long long s_mbar;
+    const uint32_t mbar = (uint32_t)__cvta_generic_to_shared(&s_mbar);
+    if (!AFF) {
+        if (threadIdx.x == 0) {
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar) : "memory");
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const uint32_t bytes = (uint32_t)tile_bytes(c);
+            const unsigned char *src = sb.tile + (size_t)blockIdx.y * tile_bytes(c);
+            asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(mbar), "r"(bytes) : "memory");
+            asm volatile(
+                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                    (uint32_t)__cvta_generic_to_shared(smem)),
+                "l"(src), "r"(bytes), "r"(mbar)
+                : "memory");
+        }
     }
-    for (int idx = threadIdx.x; !AFF && idx < c.nbh * 4 * Gp; idx += blockDim.x) {
-        const int b = idx / (4 * Gp);
-        const int rem = idx - b * 4 * Gp;
-        const int u = rem / Gp;
-        const int jg = j0 + 4 * (rem - u * Gp) + u;
-        s_bkt[idx] = jg < I ? sb.bkt[(size_t)b * I + jg] : make_int2(kBig, 0);
+    // copies of query rows [q0, q0 + nrows) into raw buffer b
+    auto issue = [&](int q0, int nrows, int b) {
+        for (int t = threadIdx.x; t < nrows; t += blockDim.x) {
+            cp_async4(r_p + b * QT + t, a.prompt + q0 + t);
+            if (CON) cp_async4(r_t + b * QT + t, a.tau + q0 + t);
+        }
+        if (ROUTE) {
+            const size_t g0 = (size_t)q0 * M;
+            for (int idx = threadIdx.x; idx < nrows * M; idx += blockDim.x) {
+                cp_async4(r_d + b * QT * M + idx, a.dec_hat + g0 + idx);
+                cp_async4(r_a + b * QT * M + idx, a.acc + g0 + idx);
+            }
+        }
+        cp_async_commit();
+    };
+    issue(rb, min(QT, re - rb), 0);  // the first chunk travels while the tile block lands
+    if (!AFF) {
+        // bounded wait for the tile block; a copy that never lands is reported, not waited out
+        bool landed = false;
+        for (int it = 0; it < (1 << 22) && !landed; ++it) landed = mbar_test(mbar);
+        if (__syncthreads_or(!landed)) {
+            if (threadIdx.x == 0) record_status(a.ctl, kECuda);
+            for (int it = 0; it < (1 << 22) && !mbar_test(mbar); ++it) {
+            }
+            cp_async_wait<0>();
+            return;
+        }
     }
     Inst4 r;
     int model[4], la[4];
     float ag[4], ac[4];  // average-case sources: t = fma(p, ag, ac)
     bool fast_mine = true;
+    const int fs = 4 * Gp;  // scalar field stride
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-        const int j = min(jb + u, I - 1);
-        model[u] = c.moi[j];
         if (AFF) {
+            const int j = min(jb + u, I - 1);
+            model[u] = c.moi[j];
             const QueueDev qd = a.qd[j];
             ag[u] = qd.g;
             // throughput source: residents' remaining prefill tokens / theta + Tdec
@@ -302,19 +353,18 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                         : __double2float_rn(__dadd_rn(__ddiv_rn((double)sb.inst[j].f1tot, qd.theta), qd.tdec));
             continue;
         }
-        const InstParams ip = sb.inst[j];
-        const int m = c.moi[j];
-        r.shift[u] = ip.shift;
-        r.h1[u] = ip.h1;
-        r.l1[u] = ip.l1;
-        r.h4[u] = ip.h4;
-        r.l4[u] = ip.l4;
-        r.b1p[u] = c.coef[m * 5 + 1];
-        r.b2[u] = c.coef[m * 5 + 3];
-        r.b3[u] = c.coef[m * 5 + 4];
-        model[u] = m;
-        la[u] = ip.la;
-        if (u < nv) fast_mine = fast_mine && ip.fast != 0;
+        const int col = u * Gp + g;
+        r.shift[u] = s_scal[kScShift * fs + col];
+        r.h1[u] = __int_as_float(s_scal[kScH1 * fs + col]);
+        r.l1[u] = __int_as_float(s_scal[kScL1 * fs + col]);
+        r.h4[u] = __int_as_float(s_scal[kScH4 * fs + col]);
+        r.l4[u] = __int_as_float(s_scal[kScL4 * fs + col]);
+        r.b1p[u] = __int_as_float(s_scal[kScB1p * fs + col]);
+        r.b2[u] = __int_as_float(s_scal[kScB2 * fs + col]);
+        r.b3[u] = __int_as_float(s_scal[kScB3 * fs + col]);
+        model[u] = s_scal[kScModel * fs + col];
+        la[u] = s_scal[kScLa * fs + col];
+        if (u < nv) fast_mine = fast_mine && s_scal[kScFast * fs + col] != 0;
     }
     const bool fast = __syncthreads_and(fast_mine);
     const bool vec = a.vec_ok && nv == 4;
@@ -337,22 +387,6 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
 
     auto run = [&](auto fast_tag) {
         constexpr bool FAST = decltype(fast_tag)::value;
-        // copies of chunk [q0, q0 + nrows) into raw buffer b
-        auto issue = [&](int q0, int nrows, int b) {
-            for (int t = threadIdx.x; t < nrows; t += blockDim.x) {
-                cp_async4(r_p + b * QT + t, a.prompt + q0 + t);
-                if (CON) cp_async4(r_t + b * QT + t, a.tau + q0 + t);
-            }
-            if (ROUTE) {
-                const size_t g0 = (size_t)q0 * M;
-                for (int idx = threadIdx.x; idx < nrows * M; idx += blockDim.x) {
-                    cp_async4(r_d + b * QT * M + idx, a.dec_hat + g0 + idx);
-                    cp_async4(r_a + b * QT * M + idx, a.acc + g0 + idx);
-                }
-            }
-            cp_async_commit();
-        };
-        issue(rb, min(QT, re - rb), 0);
         int buf = 0;
         for (int q0 = rb; q0 < re; q0 += QT, buf ^= 1) {
             const int nrows = min(QT, re - q0);

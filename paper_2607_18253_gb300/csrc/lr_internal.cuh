@@ -9,8 +9,9 @@
 //   buffer 0/1  : a snapshot copy (SoA, row stride cap) plus its summary:
 //                 inst[I]           InstParams (admission batch, totals, splits)
 //                 bkt[NBH][I]       int2 (in-bucket boundary, boundaries below)
-//                 ent[KPH][I]       float4 (T_k, H3_k, L3_k, f3_k)
 //                 f2[KPH][I], f3[KPH][I], rcum[KPH][I]
+//                 tile[T]           per tile of 4*tgp instances, the candidate
+//                                   kernel's shared-memory image (see below)
 //   control     : live buffer index, sticky status word, load error, CTA counter
 #pragma once
 
@@ -44,7 +45,7 @@ struct InstParams {      // 64 bytes
 
 struct DevConfig {
     int32_t I, M, capR, capW;
-    int32_t pmax, mode, max_iters, pad0;
+    int32_t pmax, mode, max_iters, tgp;     // tgp: thread groups per instance tile of the candidate kernel
     int32_t kph, nbh;                       // table row counts (host bounds over instances)
     const int32_t *moi, *B, *S, *shift, *nb;
     const float *coef, *pin, *pout;
@@ -55,7 +56,7 @@ struct StateBuf {
     double *clock;  // [I] end time of the instance's last completed batch (s)
     InstParams *inst;
     int2 *bkt;
-    float4 *ent;
+    unsigned char *tile;  // candidate-kernel tile blocks
     long long *f2, *f3;
     int32_t *rcum;
 };
@@ -87,6 +88,29 @@ __device__ __forceinline__ long long warp_sum64(long long v) {
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     return v;
 }
+
+// Candidate-kernel tile block: everything one CTA of the candidate kernel needs about
+// its tile of 4 * tgp instances, laid out as that CTA's shared memory so that a single
+// bulk copy brings it in.  Instance j0 + 4g + u of the tile sits in column u * tgp + g:
+//   ent  [kph][4][tgp]    float4 (T_k, H3_k, L3_k, f3_k)
+//   bkt  [nbh][4][tgp]    int2 (in-bucket boundary, boundaries below)
+//   scal [kScal][4][tgp]  32-bit scalars, fields kSc*
+constexpr int kScal = 12;
+enum : int { kScShift = 0, kScH1, kScL1, kScH4, kScL4, kScB1p, kScB2, kScB3, kScModel, kScLa, kScFast };
+__host__ __device__ inline size_t tile_ent_bytes(const DevConfig &c) { return (size_t)c.kph * 4 * c.tgp * 16; }
+__host__ __device__ inline size_t tile_bkt_bytes(const DevConfig &c) { return (size_t)c.nbh * 4 * c.tgp * 8; }
+__host__ __device__ inline size_t tile_bytes(const DevConfig &c) {
+    return tile_ent_bytes(c) + tile_bkt_bytes(c) + (size_t)kScal * 4 * c.tgp * 4;
+}
+__host__ __device__ inline int tile_count(const DevConfig &c) { return (c.I + 4 * c.tgp - 1) / (4 * c.tgp); }
+// Byte offset of instance j's column within its tile block, and the tile's base.
+__host__ __device__ inline size_t tile_base(const DevConfig &c, int j) { return (size_t)(j / (4 * c.tgp)) * tile_bytes(c); }
+__host__ __device__ inline int tile_col(const DevConfig &c, int j) {
+    const int jj = j % (4 * c.tgp);
+    return (jj & 3) * c.tgp + (jj >> 2);
+}
+// Columns past the last instance, written once so that they read as empty instances.
+cudaError_t launch_tile_pad(const DevConfig &c, unsigned char *tile, cudaStream_t st);
 
 // Launch helpers implemented in the kernel translation units.
 struct K1Launch {

@@ -454,7 +454,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             e.z = __ll2float_rn(lo);
             e.w = __ll2float_rn(F3);
             const size_t o = (size_t)k * c.I + j;
-            out.ent[o] = e;
+            reinterpret_cast<float4 *>(out.tile + tile_base(c, j))[(size_t)k * 4 * c.tgp + tile_col(c, j)] = e;
             out.f2[o] = F2;
             out.f3[o] = F3;
             out.rcum[o] = m.rcum[k];
@@ -475,6 +475,8 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             else if (rk <= hi) bnd = (int)rk;
         }
         out.bkt[(size_t)b * c.I + j] = make_int2(bnd, below);
+        reinterpret_cast<int2 *>(out.tile + tile_base(c, j) + tile_ent_bytes(c))[(size_t)b * 4 * c.tgp + tile_col(c, j)] =
+            make_int2(bnd, below);
     }
     if (lane == 0) {
         InstParams ip;
@@ -491,6 +493,22 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         ip.r0 = r0;
         ip.pad[0] = ip.pad[1] = ip.pad[2] = 0;
         out.inst[j] = ip;
+        // the candidate kernel's per-instance scalars
+        int32_t *sc = reinterpret_cast<int32_t *>(out.tile + tile_base(c, j) + tile_ent_bytes(c) + tile_bkt_bytes(c)) +
+                      tile_col(c, j);
+        const size_t fs = 4 * (size_t)c.tgp;  // field stride
+        const float *cf = c.coef + 5 * m_j;
+        sc[kScShift * fs] = sh;
+        sc[kScH1 * fs] = __float_as_int(ip.h1);
+        sc[kScL1 * fs] = __float_as_int(ip.l1);
+        sc[kScH4 * fs] = __float_as_int(ip.h4);
+        sc[kScL4 * fs] = __float_as_int(ip.l4);
+        sc[kScB1p * fs] = __float_as_int(cf[1]);
+        sc[kScB2 * fs] = __float_as_int(cf[3]);
+        sc[kScB3 * fs] = __float_as_int(cf[4]);
+        sc[kScModel * fs] = m_j;
+        sc[kScLa * fs] = la;
+        sc[kScFast * fs] = ip.fast;
     }
 }
 
@@ -522,6 +540,33 @@ __global__ void __launch_bounds__(kK1Warps * 32) k_trajectory(const K1Launch a) 
 }
 
 }  // namespace
+
+namespace {
+
+// Padding columns of the last tile: no boundary in any bucket, zero tables, an
+// exact ("fast") instance of model 0, and a bucket shift of 30 so that every
+// allowed prompt (at most 2^20 tokens) looks up bucket 0 and entry 0.
+__global__ void k_tile_pad(const DevConfig c, unsigned char *tile) {
+    const int first = c.I;
+    const int last = tile_count(c) * 4 * c.tgp;
+    for (int j = first + blockIdx.x * blockDim.x + threadIdx.x; j < last; j += gridDim.x * blockDim.x) {
+        unsigned char *base = tile + tile_base(c, j);
+        const int col = tile_col(c, j);
+        for (int k = 0; k < c.kph; ++k)
+            reinterpret_cast<float4 *>(base)[(size_t)k * 4 * c.tgp + col] = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int b = 0; b < c.nbh; ++b)
+            reinterpret_cast<int2 *>(base + tile_ent_bytes(c))[(size_t)b * 4 * c.tgp + col] = make_int2(kBig, 0);
+        int32_t *sc = reinterpret_cast<int32_t *>(base + tile_ent_bytes(c) + tile_bkt_bytes(c)) + col;
+        for (int f = 0; f < kScal; ++f) sc[(size_t)f * 4 * c.tgp] = (f == kScFast) ? 1 : (f == kScShift) ? 30 : 0;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_tile_pad(const DevConfig &c, unsigned char *tile, cudaStream_t st) {
+    k_tile_pad<<<1, 256, 0, st>>>(c, tile);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_trajectory(const K1Launch &a, int grid, int block, size_t smem, cudaStream_t st) {
     if (a.cfg.mode == 0) k_trajectory<0><<<grid, block, smem, st>>>(a);
