@@ -246,7 +246,12 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     const int rb = blockIdx.x * rows_per;
     const int re = min(a.Q, rb + rows_per);
     if (rb >= re) return;
-    const int active = *((volatile int32_t *)&a.ctl->active);
+    // one read of the live-buffer index per CTA (every thread reading the same word
+    // would queue them all on one L2 line)
+    __shared__ int s_active;
+    if (threadIdx.x == 0) s_active = *((volatile int32_t *)&a.ctl->active);
+    __syncthreads();
+    const int active = s_active;
     // the LPS source needs no live snapshot; every other source does
     if (active < 0 && !(AFF && a.src == kSrcLps)) {
         if (threadIdx.x == 0) record_status(a.ctl, kENoState);

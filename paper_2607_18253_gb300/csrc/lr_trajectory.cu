@@ -518,7 +518,12 @@ __global__ void __launch_bounds__(kK1Warps * 32) k_trajectory(const K1Launch a) 
     const int lane = threadIdx.x & 31;
     const int wid = threadIdx.x >> 5;
     const int j = blockIdx.x * kK1Warps + wid;
-    const int active = *((volatile int32_t *)&a.ctl->active);
+    // one read of the live-buffer index per CTA (every thread reading the same word
+    // would queue them all on one L2 line)
+    __shared__ int s_active;
+    if (threadIdx.x == 0) s_active = *((volatile int32_t *)&a.ctl->active);
+    __syncthreads();
+    const int active = s_active;
     const int dst = (active == 0) ? 1 : 0;
     const StateBuf out = dst ? a.buf1 : a.buf0;
     const size_t per_warp = trajectory_smem_per_warp(a.cfg) / sizeof(int32_t);
