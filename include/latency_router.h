@@ -120,7 +120,15 @@ LR_API int lr_destroy(lr_ctx *ctx);
  * snapshot is written to a back buffer and becomes the live one only if every
  * instance is valid and simulates within max_iters; otherwise the previous live
  * snapshot stays in use (App. F: the router keeps its last complete copy) and the
- * status word records LR_ESTATE or LR_ETRAJ. */
+ * status word records LR_ESTATE or LR_ETRAJ.
+ * Overlap: a load (or lr_advance) may run on one stream while lr_estimate_ttft /
+ * lr_route run on another; each CTA of those calls uses the snapshot that is live
+ * when it starts, so every query row is computed against one complete snapshot, the
+ * previous or the new one (App. F: the router estimates from its most recent complete
+ * copy while the next is prepared).  The back buffer a load writes is the one the
+ * snapshot before the live one occupied, so order the next load after every
+ * estimate or route call issued before the previous load finished (at most one load
+ * in flight). */
 LR_API int lr_load_state(lr_ctx *ctx, const lr_state_view *state, void *cuda_stream);
 
 /* SFS TTFT estimates (Eq. 8 with Eq. 9) for every candidate of Q queries.

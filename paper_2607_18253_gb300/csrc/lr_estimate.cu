@@ -249,7 +249,7 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     // one read of the live-buffer index per CTA (every thread reading the same word
     // would queue them all on one L2 line)
     __shared__ int s_active;
-    if (threadIdx.x == 0) s_active = *((volatile int32_t *)&a.ctl->active);
+    if (threadIdx.x == 0) s_active = load_acquire(&a.ctl->active);
     __syncthreads();
     const int active = s_active;
     // the LPS source needs no live snapshot; every other source does
@@ -304,6 +304,9 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
         if (threadIdx.x == 0) {
             const uint32_t bytes = (uint32_t)tile_bytes(c);
             const unsigned char *src = sb.tile + (size_t)blockIdx.y * tile_bytes(c);
+            // the block was written by generic stores (possibly of a load on another
+            // stream, acquired above); order them before the bulk copy's reads
+            asm volatile("fence.proxy.async.global;" ::: "memory");
             asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(mbar), "r"(bytes) : "memory");
             asm volatile(
                 "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(

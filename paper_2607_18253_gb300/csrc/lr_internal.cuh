@@ -73,6 +73,14 @@ struct StateIn {
     const double *clock;  // may be null: clocks start at 0
 };
 
+// The live-buffer index with acquire ordering: reads of the buffer it names see
+// everything the load that published it wrote (it may have finished on another stream).
+__device__ __forceinline__ int32_t load_acquire(const int32_t *p) {
+    int32_t v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
 __device__ __forceinline__ void record_status(DevCtl *ctl, int code) {
     atomicCAS(&ctl->status, 0, code);
 }

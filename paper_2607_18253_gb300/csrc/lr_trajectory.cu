@@ -521,7 +521,7 @@ __global__ void __launch_bounds__(kK1Warps * 32) k_trajectory(const K1Launch a) 
     // one read of the live-buffer index per CTA (every thread reading the same word
     // would queue them all on one L2 line)
     __shared__ int s_active;
-    if (threadIdx.x == 0) s_active = *((volatile int32_t *)&a.ctl->active);
+    if (threadIdx.x == 0) s_active = load_acquire(&a.ctl->active);
     __syncthreads();
     const int active = s_active;
     const int dst = (active == 0) ? 1 : 0;

@@ -6,6 +6,8 @@ oracle's canonical fp32 evaluation bit for bit (both sides evaluate the same
 fixed sequence of IEEE operations), which in turn is within 1e-5 relative of
 the oracle's fp64 value.
 """
+import dataclasses
+
 import numpy as np
 import pytest
 
@@ -267,3 +269,35 @@ def test_host_side_errors():
         R().LatencyRouter(model_of_instance=[0], coef=np.ones((1, 5)), price_in=[0], price_out=[0],
                           max_batched_tokens=[8], max_seqs=[9], cap_running=4, cap_waiting=4, max_queries=4,
                           max_prompt_len=16)
+
+
+def test_load_overlapping_estimates_sees_whole_snapshots():
+    # A snapshot load on one stream overlapping estimates on another: every query row
+    # must be exactly the oracle's row under the previous or under the new snapshot.
+    old = W.make_workload("pool64", num_queries=2048)
+    new = W.make_workload("pool64", num_queries=2048, seed=7)
+    rt = make_router(old)
+    p = R().query_tensors(old)[0]
+    _, _, t_old, _ = oracle.estimate_matrix(old)
+    _, _, t_new, _ = oracle.estimate_matrix(dataclasses.replace(new, prompt_len=old.prompt_len))
+    s_load, s_est = torch.cuda.Stream(), torch.cuda.Stream()
+    new_state = R().state_tensors(new)
+    outs = [torch.empty((2048, 64), dtype=torch.float32, device="cuda") for _ in range(6)]
+    torch.cuda.synchronize()
+    with torch.cuda.stream(s_est):
+        for o in outs[:3]:
+            rt.estimate_ttft(p, out=o, stream=s_est)
+    rt.load_state(*new_state, stream=s_load)
+    with torch.cuda.stream(s_est):
+        for o in outs[3:]:
+            rt.estimate_ttft(p, out=o, stream=s_est)
+    torch.cuda.synchronize()
+    assert rt.status() == R().LR_OK
+    b_old, b_new = bits(t_old), bits(t_new)
+    for o in outs:
+        got = bits(o.cpu().numpy())
+        is_old = np.all(got == b_old, axis=1)
+        is_new = np.all(got == b_new, axis=1)
+        assert np.all(is_old | is_new)
+    # after both streams finished, the new snapshot is live everywhere
+    np.testing.assert_array_equal(bits(rt.estimate_ttft(p).cpu().numpy()), b_new)
