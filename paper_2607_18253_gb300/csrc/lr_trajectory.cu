@@ -398,67 +398,158 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         int nlist;
     } sim = {m.scr[2]};
 
-    // Budgets left to the query after its admission batch, and the residents'
-    // decode features up to each batch its first token can fall in (one
-    // parallel pass over the decoder list per batch).
+    // Budgets left to the query after its admission batch, and the residents' decode
+    // features up to each batch its first token can fall in.  One pass over the
+    // decoder list serves eight table rows k: the decoders alive in batch la + k (so
+    // r_k = B - alive) and the decode tokens and context they contribute up to batch
+    // L_k = la + k + off.  A decoder alive over the whole window of a pass adds to
+    // row q in closed form (u + q tokens, and context sum up to L_0 plus
+    // q cb + q L_0 + q(q+1)/2, with u its tokens up to L_0), so only decoders that
+    // start or end inside the window take the per-row loop (one finished before it
+    // adds the same to every row).  Lane partials are
+    // reduced through shared memory (the calendar is free after the step loop).
     constexpr int off = (MODE == 0) ? 1 : 0;
+    constexpr int kRows = 8;
+    constexpr int kCols = 3 * kRows + 4;  // per-row partials of window decoders, then N, A2, A3, CB
     const int nl = sim.nlist;
-    int kp = 1;
-    long long rc = r0;
-    if (lane == 0) m.rcum[0] = r0;
-    while (rc < c.pmax && kp < c.kph) {
-        const int lk = la + kp;
-        int nd = 0;
-        for (int i = lane; i < nl; i += 32) {
-            const int4 dd = m.dl[i];
-            nd += (dd.x <= lk && lk <= dd.y) ? 1 : 0;
-        }
-        nd = __reduce_add_sync(kFull, nd);
-        rc += B - nd;
-        if (lane == 0) m.rcum[kp] = (int)min(rc, (long long)kBig - 1);
-        ++kp;
-    }
-    __syncwarp();
-    if (rc < c.pmax) {
-        fail(a.ctl, kETraj, lane);
-        return;
-    }
+    long long *red = reinterpret_cast<long long *>(m.cal);  // [kCols][32] lane partials (7 KB)
+    // after them, up to the end of the calendar bitmap: the window decoders' indices
+    constexpr int kWinList = (int)((kCalendar * 4 + kCalendar / 8 - kCols * 32 * 8) / 4);
+    int32_t *wlist = reinterpret_cast<int32_t *>(red + kCols * 32);
     const int m_j = c.moi[j];
     const float b0 = c.coef[m_j * 5 + 0];
     const float b1d = c.coef[m_j * 5 + 2];
     const long long ppmax = ((long long)c.pmax * (c.pmax + 1)) / 2;
     bool fast = (f1 + c.pmax < kFastLimit) && (f4 + ppmax < kFastLimit);
     const long long lowmask = (1LL << kSplitBits) - 1;
-    for (int k = 0; k < kp; ++k) {
-        const int L = la + k + off;
-        long long a2 = 0, a3 = 0;
-        for (int i = lane; i < nl; i += 32) {
-            const int4 dd = m.dl[i];
+    int kp = 0;          // table rows kept
+    long long rc = r0;   // cumulative budget R_k
+    bool more = true;
+    for (int k0 = 0; more && k0 < c.kph; k0 += kRows) {
+        const int lk0 = la + k0;             // first batch of the alive counts
+        const int L0 = lk0 + off;            // first feature horizon
+        const int Lend = lk0 + kRows - 1 + off;
+        int nd[kRows];
+        long long a2[kRows], a3[kRows];
+#pragma unroll
+        for (int q = 0; q < kRows; ++q) {
+            nd[q] = 0;
+            a2[q] = 0;
+            a3[q] = 0;
+        }
+        int nreg = 0;                        // decoders alive over the whole window
+        long long A2 = 0, A3 = 0, CB = 0;    // their tokens and context sums up to L0 (plus those of
+                                             // decoders finished before the window), and their cb sum
+        // a decoder that starts or ends inside the window adds to each row separately
+        auto rows = [&](const int4 dd) {
             const int s = dd.x;
-            if (s <= L) {
-                const int e = min(dd.y, L);
-                const long long cnt = (long long)e - s + 1;
-                a2 += cnt;
-                a3 += cnt * (long long)dd.z + (((long long)s + e) * cnt) / 2;
+#pragma unroll
+            for (int q = 0; q < kRows; ++q) {
+                const int lk = lk0 + q;
+                nd[q] += (s <= lk && lk <= dd.y) ? 1 : 0;
+                const int L = lk + off;
+                if (s <= L) {
+                    const int e = min(dd.y, L);
+                    const long long cnt = (long long)e - s + 1;
+                    a2[q] += cnt;
+                    a3[q] += cnt * (long long)dd.z + (((long long)s + e) * cnt) / 2;
+                }
+            }
+        };
+        // Window decoders are few but scattered, so they are first gathered into a
+        // list (stable ballot compaction) and then taken 32 at a time: a warp would
+        // otherwise run the per-row path in almost every step over the list.
+        int nwin = 0;
+        for (int base = 0; base < nl; base += 32) {
+            const int i = base + lane;
+            bool win = false;
+            if (i < nl) {
+                const int4 dd = m.dl[i];
+                const int s = dd.x;
+                // u tokens at contexts cb + s .. cb + e: u cb + (s + e) u / 2, where
+                // (s + e) u is twice a sum of consecutive integers, so the halving is exact
+                if (s <= lk0 && dd.y >= Lend) {
+                    const int u = L0 - s + 1;
+                    ++nreg;
+                    A2 += u;
+                    A3 += (long long)u * dd.z + (((long long)s + L0) * u >> 1);
+                    CB += dd.z;
+                } else if (dd.y < lk0) {
+                    // finished before the window: all of its tokens, in every row
+                    const int u = dd.y - s + 1;
+                    A2 += u;
+                    A3 += (long long)u * dd.z + (((long long)s + dd.y) * u >> 1);
+                } else {
+                    win = true;
+                }
+            }
+            const unsigned bal = __ballot_sync(kFull, win);
+            if (win) {
+                const int slot = nwin + __popc(bal & lanemask_lt());
+                if (slot < kWinList) wlist[slot] = i;
+                else rows(m.dl[i]);  // list full: on the spot
+            }
+            nwin += __popc(bal);
+        }
+        __syncwarp();
+        for (int t = lane; t < min(nwin, kWinList); t += 32) rows(m.dl[wlist[t]]);
+        __syncwarp();
+#pragma unroll
+        for (int q = 0; q < kRows; ++q) {
+            red[(0 * kRows + q) * 32 + lane] = nd[q];
+            red[(1 * kRows + q) * 32 + lane] = a2[q];
+            red[(2 * kRows + q) * 32 + lane] = a3[q];
+        }
+        red[(3 * kRows + 0) * 32 + lane] = nreg;
+        red[(3 * kRows + 1) * 32 + lane] = A2;
+        red[(3 * kRows + 2) * 32 + lane] = A3;
+        red[(3 * kRows + 3) * 32 + lane] = CB;
+        __syncwarp();
+        long long tot = 0;
+        if (lane < kCols)
+            for (int l = 0; l < 32; ++l) tot += red[lane * 32 + l];
+        __syncwarp();
+        if (lane < kCols) red[lane * 32] = tot;  // each column's head holds its sum
+        __syncwarp();
+        const long long Nw = red[(3 * kRows + 0) * 32], A2w = red[(3 * kRows + 1) * 32];
+        const long long A3w = red[(3 * kRows + 2) * 32], CBw = red[(3 * kRows + 3) * 32];
+        // the rows of this pass in order; row k >= 1 is needed while R_{k-1} < pmax
+        for (int q = 0; q < kRows && more; ++q) {
+            const int k = k0 + q;
+            if (k >= c.kph || (k >= 1 && rc >= c.pmax)) {
+                more = false;
+                break;
+            }
+            if (k >= 1) rc += B - (Nw + red[(0 * kRows + q) * 32]);
+            const int rk = (int)min(rc, (long long)kBig - 1);
+            if (lane == 0) m.rcum[k] = rk;
+            kp = k + 1;
+            const int L = la + k + off;
+            // + the query's own first decode token
+            const long long F2 = A2w + Nw * q + red[(1 * kRows + q) * 32] + off;
+            const long long F3 = A3w + q * CBw + Nw * ((long long)q * L0 + (long long)q * (q + 1) / 2) +
+                                 red[(2 * kRows + q) * 32];
+            fast = fast && (F3 + c.pmax < kFastLimit);
+            if (lane == (k & 31)) {
+                const float t = __fmaf_rn(b1d, __ll2float_rn(F2), __fmul_rn(b0, __int2float_rn(L)));
+                const long long lo = F3 & lowmask;
+                float4 e;
+                e.x = t;
+                e.y = __ll2float_rn(F3 - lo);
+                e.z = __ll2float_rn(lo);
+                e.w = __ll2float_rn(F3);
+                const size_t o = (size_t)k * c.I + j;
+                reinterpret_cast<float4 *>(out.tile + tile_base(c, j))[(size_t)k * 4 * c.tgp + tile_col(c, j)] = e;
+                out.f2[o] = F2;
+                out.f3[o] = F3;
+                out.rcum[o] = rk;
             }
         }
-        const long long F2 = warp_sum64(a2) + off;  // + the query's own first decode token
-        const long long F3 = warp_sum64(a3);
-        fast = fast && (F3 + c.pmax < kFastLimit);
-        if (lane == (k & 31)) {
-            const float t = __fmaf_rn(b1d, __ll2float_rn(F2), __fmul_rn(b0, __int2float_rn(L)));
-            const long long lo = F3 & lowmask;
-            float4 e;
-            e.x = t;
-            e.y = __ll2float_rn(F3 - lo);
-            e.z = __ll2float_rn(lo);
-            e.w = __ll2float_rn(F3);
-            const size_t o = (size_t)k * c.I + j;
-            reinterpret_cast<float4 *>(out.tile + tile_base(c, j))[(size_t)k * 4 * c.tgp + tile_col(c, j)] = e;
-            out.f2[o] = F2;
-            out.f3[o] = F3;
-            out.rcum[o] = m.rcum[k];
-        }
+        __syncwarp();
+    }
+    if (rc < c.pmax) {
+        fail(a.ctl, kETraj, lane);
+        return;
     }
 
     // Prompt-length buckets of width 2^shift <= B_j - S_j + 1 <= every r_k (k >= 1):
