@@ -140,7 +140,7 @@ constexpr int kCalendar = 2048;
 // the waiting queue's prompt prefix sums and decode lengths, and the budgets.
 __host__ __device__ inline size_t trajectory_smem_per_warp(const DevConfig &c) {
     const size_t words = (size_t)kCalendar + kCalendar / 32 + 4 * (size_t)(c.capR + c.capW) +
-                         (size_t)(c.capW + 1) + (size_t)c.capW + (size_t)c.kph + 32;
+                         (size_t)(c.capW + 2) + (size_t)(c.capW + 1) + (size_t)c.kph + 32;
     return sizeof(int32_t) * ((words + 3) & ~(size_t)3);
 }
 

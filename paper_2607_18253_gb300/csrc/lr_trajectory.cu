@@ -45,8 +45,8 @@ struct WarpSmem {
     uint32_t *bm;    // [kCalendar / 32] non-empty calendar batches
     int4 *dl;        // [capR + capW] decoder list: (first decode batch s, last decode
                      //   batch f, context offset cb: context at batch l is cb + l, 0)
-    int32_t *P;      // [capW + 1] exclusive prefix sums of waiting prompts
-    int32_t *wdec;   // [capW] waiting decode lengths
+    int32_t *P;      // [capW + 2] exclusive prefix sums of waiting prompts (+1 unread pad)
+    int32_t *wdec;   // [capW + 1] waiting decode lengths (+1 unread pad)
     int32_t *rcum;   // [kph] cumulative budgets
     int32_t *scr;    // [32] results of the step loop
 };
@@ -57,8 +57,8 @@ __device__ __forceinline__ WarpSmem carve(int32_t *base, const DevConfig &c) {
     w.bm = reinterpret_cast<uint32_t *>(w.cal + kCalendar);
     w.dl = reinterpret_cast<int4 *>(w.bm + kCalendar / 32);  // 16-byte aligned
     w.P = reinterpret_cast<int32_t *>(w.dl + (c.capR + c.capW));
-    w.wdec = w.P + (c.capW + 1);
-    w.rcum = w.wdec + c.capW;
+    w.wdec = w.P + (c.capW + 2);
+    w.rcum = w.wdec + (c.capW + 1);
     w.scr = w.rcum + c.kph;
     return w;
 }
@@ -300,7 +300,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         int ph = 0;  // prompt prefix sum at the waiting head
         int fnext = tr.next_end(1);
         int la = 0, r0 = 0;
-        int pn_head = lds(sP + 4u * min(1, c.capW));
+        int pn_head = lds(sP + 4u);
         int d_head = lds(sW);
         while (iters < c.max_iters && l < (1 << 30)) {
             ++iters;
@@ -341,7 +341,9 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                 }
             }
             // FCFS admission while budget and a sequence slot remain.
-            while (budget > 0 && head < nw && cnt < S) {
+            // requests this batch can admit at most: the queue and the free seats
+            const int lim = min(nw, head + (S - cnt));
+            while (budget > 0 && head < lim) {
                 const int pn = pn_head;
                 const int d = d_head;
                 const int p = pn - ph;
@@ -349,9 +351,9 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                 ph = pn;
                 ++cnt;
                 // the next head's prompt sum and length, loaded ahead of their use
-                // (P has capW + 1 entries; wdec's entries past nw are in bounds too)
-                pn_head = lds(sP + 4u * min(head + 1, c.capW));
-                d_head = lds(sW + 4u * min(head, c.capW - 1));
+                // (head <= nw <= capW here: both reads are in bounds, the pads included)
+                pn_head = lds(sP + 4u * (head + 1));
+                d_head = lds(sW + 4u * head);
                 if (p <= budget) {
                     budget -= p;
                     int f, cb;
