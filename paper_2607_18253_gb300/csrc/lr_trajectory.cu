@@ -314,7 +314,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                 continue;
             }
             int budget = B - n;  // every decoder takes one token first
-            int pend = 0;        // decoders that start in batch l + 1
+            const int nl0 = tr.nlist;  // decoders appended in this batch start in batch l + 1
             if (pf) {
                 if (budget <= 0) break;  // excluded by the preconditions
                 if (pfR > budget) {
@@ -336,20 +336,19 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                 int f, cb;
                 if (decoder_of<MODE>(l, pfC, pfD, &f, &cb)) {
                     tr.append(l + 1, f, cb);
-                    ++pend;
                     fnext = min(fnext, f);
                 }
             }
             // FCFS admission while budget and a sequence slot remain.
             // requests this batch can admit at most: the queue and the free seats
             const int lim = min(nw, head + (S - cnt));
+            const int head0 = head;
             while (budget > 0 && head < lim) {
                 const int pn = pn_head;
                 const int d = d_head;
                 const int p = pn - ph;
                 ++head;
                 ph = pn;
-                ++cnt;
                 // the next head's prompt sum and length, loaded ahead of their use
                 // (head <= nw <= capW here: both reads are in bounds, the pads included)
                 pn_head = lds(sP + 4u * (head + 1));
@@ -359,7 +358,6 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                     int f, cb;
                     if (decoder_of<MODE>(l, p, d, &f, &cb)) {
                         tr.append(l + 1, f, cb);
-                        ++pend;
                         fnext = min(fnext, f);
                     }
                 } else {  // the prompt continues in later batches
@@ -370,12 +368,13 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                     budget = 0;
                 }
             }
+            cnt += head - head0;  // every request taken from the queue holds a seat
             if (!pf && head == nw && budget > 0 && cnt < S) {
                 la = l;
                 r0 = budget;
                 break;
             }
-            n += pend;
+            n += tr.nlist - nl0;
             if (l == fnext) {
                 n -= tr.ends_at(l);
                 fnext = tr.next_end(l + 1);
