@@ -255,3 +255,33 @@ def avgcase_matrix(wl, W, theta, tdec):
     if rc != 0:
         raise ValueError(f"oracle average-case estimate failed with code {rc}")
     return t32, t64
+
+
+# ---------------------------------------------------------------------------
+# Calibration of the batch-time model (Sec. 4.1, "Token-batch processing time
+# estimator": the coefficients are calibrated from observed batch times)
+
+def calibrate(features, model, time, num_models: int, shared_beta1: bool = True) -> np.ndarray:
+    """Least-squares Eq. 9 coefficients per model from per-batch (F, observed time) rows.
+
+    features [N][5] (F0 .. F4 of each executed batch), model [N], time [N] seconds.
+    shared_beta1: the paper's four-coefficient form, one beta1 for prefill and
+    decode tokens (regressor F1 + F2); otherwise five coefficients.
+    Returns [M][5] fp64 (beta0, beta1p, beta1d, beta2, beta3); NaN rows for models
+    with fewer rows than unknowns or a rank-deficient design."""
+    F = np.asarray(features, np.float64)
+    mdl = np.asarray(model, np.int64)
+    y = np.asarray(time, np.float64)
+    out = np.full((num_models, 5), np.nan)
+    for m in range(num_models):
+        sel = mdl == m
+        X = F[sel]
+        if shared_beta1:
+            X = np.stack([X[:, 0], X[:, 1] + X[:, 2], X[:, 3], X[:, 4]], axis=1)
+        if X.shape[0] < X.shape[1]:
+            continue
+        beta, _, rank, _ = np.linalg.lstsq(X, y[sel], rcond=None)
+        if rank < X.shape[1]:
+            continue
+        out[m] = [beta[0], beta[1], beta[1], beta[2], beta[3]] if shared_beta1 else beta
+    return out

@@ -264,6 +264,38 @@ def mmpp2_arrivals(num_queries: int, mean_qps: float, ratio: float, seed: int, z
     return np.concatenate(parts)[:num_queries]
 
 
+def batch_log(num_batches: int, num_models: int, seed: int, coef: np.ndarray, noise: float = 0.04,
+              grouped: bool = True):
+    """A synthetic log of executed token batches, as calibration input.
+
+    Each row is one batch of some model: F0 = 1, up to 256 decode tokens at
+    contexts 128..4096 (F2, F3), and up to two prefill chunks of 1..2048 tokens at
+    contexts 0..8192 (F1, F4 = sum of x c + x(x+1)/2).  The synthetic engine's
+    observed time is coef[model] . F (the batch-time form being calibrated) times
+    (1 + noise * N(0, 1)).  grouped: rows sorted by model, as per-instance logs are.
+    Returns features [N][5] int64, model [N] int32, time [N] fp64."""
+    rng = np.random.default_rng(np.random.SeedSequence([seed, 0xCA1B]))
+    n = num_batches
+    mdl = rng.integers(0, num_models, n)
+    if grouped:
+        mdl = np.sort(mdl)
+    ndec = rng.integers(0, 257, n)
+    ctx = rng.integers(128, 4097, n)
+    F = np.zeros((n, 5), np.int64)
+    F[:, 0] = 1
+    F[:, 2] = ndec
+    F[:, 3] = ndec * ctx
+    for _ in range(2):
+        has = rng.random(n) < 0.5
+        x = np.where(has, rng.integers(1, 2049, n), 0)
+        c = rng.integers(0, 8193, n)
+        F[:, 1] += x
+        F[:, 4] += x * c + x * (x + 1) // 2
+    cf = np.asarray(coef, np.float64)[mdl]
+    t = np.einsum("nk,nk->n", cf, F.astype(np.float64)) * (1.0 + noise * rng.standard_normal(n))
+    return F, mdl.astype(np.int32), t
+
+
 def sweep_pairs():
     """The trade-off grid: 4 lambda values (log 0.1..10) x 8 mu values (log 0.01..1 /s), lambda-major."""
     lam = np.logspace(-1, 1, 4)
