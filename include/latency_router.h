@@ -224,6 +224,20 @@ LR_API int lr_set_queue_params(lr_ctx *ctx, const lr_queue_params *params, void 
  * (LR_ENOSTATE before one is loaded); the LPS source reads none. */
 LR_API int lr_set_ttft_source(lr_ctx *ctx, int32_t source);
 
+/* Least-squares calibration of the Eq. 9 coefficients per model from a log of executed
+ * token batches (Sec. 4.1: calibrated from observed token-batch processing times).
+ * features: [N][5] int64 device, each batch's (F0 = 1, prefill tokens, decode tokens, sum of
+ * decode-token contexts, sum over prefill chunks of x*c + x(x+1)/2); model: [N] int32 device
+ * in [0, M); time: [N] fp64 device, observed seconds.  shared_beta1 != 0 fits the paper's
+ * four-coefficient form (one beta1, regressor F1 + F2), otherwise five coefficients.
+ * coef_out: [M][5] fp64 device (beta0, beta1p, beta1d, beta2, beta3), NaN for a model with
+ * fewer rows than unknowns or a rank-deficient design.  Rows with a model outside [0, M)
+ * or a non-finite time are skipped and record LR_EINVAL.  Sums are fp64 atomics, so the
+ * last bits may differ between runs.  Rows grouped by model are the fast case.
+ * Requires num_models <= 256. */
+LR_API int lr_calibrate(lr_ctx *ctx, int64_t N, const int64_t *features, const int32_t *model, const double *time,
+                        int32_t shared_beta1, double *coef_out, void *cuda_stream);
+
 /* Online stream step (Sec. 5: queries arrive over time and are routed as they come;
  * App. F: every instance keeps executing token batches and publishes its state after each).
  * The queries with assign[i] >= 0 join instance assign[i]'s waiting tail in query order

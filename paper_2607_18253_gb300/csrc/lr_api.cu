@@ -25,6 +25,7 @@ struct lr_ctx {
     // average-case TTFT sources
     lr::QueueRaw *qraw = nullptr;
     lr::QueueDev *qd = nullptr;
+    double *cal_acc = nullptr;  // calibration sums [M][kCalAcc]
     int source = lr::kSrcSfs;
     bool have_qp = false, have_lps = false;
     std::vector<void *> allocs;
@@ -250,6 +251,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     LR_ALLOC(c->scratch_tch, (size_t)cfg->max_pairs * cfg->max_queries);
     LR_ALLOC(c->qraw, I);
     LR_ALLOC(c->qd, I);
+    LR_ALLOC(c->cal_acc, (size_t)M * lr::kCalAcc);
 #undef LR_ALLOC
     e = cudaMemcpy(moi, cfg->model_of_instance, I * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(B, cfg->max_batched_tokens, I * 4, cudaMemcpyHostToDevice);
@@ -286,6 +288,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     c->k3_smem = lr::kK3Warps * lr::advance_smem_per_warp(d);
     e = lr::set_k1_smem(c->k1_smem);
     if (e == cudaSuccess && c->k3_smem <= 200 * 1024) e = lr::set_k3_smem(c->k3_smem);
+    if (e == cudaSuccess && M <= lr::kCalMaxModels) e = lr::set_calib_smem(M);
     if (e == cudaSuccess) e = lr::set_k2_smem(std::max(c->est.smem, c->rt.ok ? c->rt.smem : 0));
     if (e == cudaSuccess) e = lr::cand_occupancy(d.mode, false, lr::kK2Block, c->est.smem, &c->est.occ);
     if (e == cudaSuccess && c->rt.ok) e = lr::cand_occupancy(d.mode, true, lr::kK2Block, c->rt.smem, &c->rt.occ);
@@ -510,6 +513,19 @@ int lr_set_ttft_source(lr_ctx *c, int32_t source) {
     if (source == LR_TTFT_LPS && !c->have_lps) return fail(c, LR_EINVAL, "the LPS source needs arrival and service rates");
     c->source = source;
     return LR_OK;
+}
+
+int lr_calibrate(lr_ctx *c, int64_t N, const int64_t *features, const int32_t *model, const double *time,
+                 int32_t shared_beta1, double *coef_out, void *stream) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    if (N < 0) return fail(c, LR_EINVAL, "N < 0");
+    if (!coef_out || (N > 0 && (!features || !model || !time))) return fail(c, LR_EINVAL, "null array");
+    if (c->cfg.M > lr::kCalMaxModels) return fail(c, LR_ECAPACITY, "calibration supports at most 256 models");
+    cudaError_t e = lr::launch_calibrate(N, reinterpret_cast<const long long *>(features), model, time, c->cfg.M,
+                                         shared_beta1 ? 1 : 0, c->cal_acc, coef_out, c->ctl, 2 * c->sms,
+                                         (cudaStream_t)stream);
+    return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "calibration launch");
 }
 
 int lr_advance(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_t *prompt_len, const int32_t *dec,

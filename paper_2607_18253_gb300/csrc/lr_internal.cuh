@@ -120,6 +120,14 @@ __host__ __device__ inline int tile_col(const DevConfig &c, int j) {
 // Columns past the last instance, written once so that they read as empty instances.
 cudaError_t launch_tile_pad(const DevConfig &c, unsigned char *tile, cudaStream_t st);
 
+// Calibration of the batch-time coefficients (lr_calibrate.cu).
+constexpr int kCalCols = 5;
+constexpr int kCalAcc = 21;        // per model: 15 sums of the upper triangle of G, 5 of b, the row count
+constexpr int kCalMaxModels = 256;  // shared-memory sums of one CTA
+cudaError_t launch_calibrate(long long N, const long long *F, const int32_t *model, const double *time, int M,
+                             int shared_beta1, double *acc, double *coef, DevCtl *ctl, int grid, cudaStream_t st);
+cudaError_t set_calib_smem(int M);
+
 // Launch helpers implemented in the kernel translation units.
 struct K1Launch {
     DevConfig cfg;

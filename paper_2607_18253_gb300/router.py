@@ -24,7 +24,7 @@ LR_TTFT_SFS, LR_TTFT_THROUGHPUT, LR_TTFT_LPS = 0, 1, 2
 
 EXPORTED_SYMBOLS = ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
                     "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
-                    "lr_set_queue_params", "lr_set_ttft_source", "lr_strerror", "lr_last_error")
+                    "lr_set_queue_params", "lr_set_ttft_source", "lr_calibrate", "lr_strerror", "lr_last_error")
 
 _P = ctypes.c_void_p
 _I32 = ctypes.c_int32
@@ -68,6 +68,7 @@ def load_library(path: str = LIB_PATH):
     lib.lr_advance.argtypes = [_P, _I32, _P, _P, _P, _I32, ctypes.c_double, _P]
     lib.lr_set_queue_params.argtypes = [_P, ctypes.POINTER(_QueueParams), _P]
     lib.lr_set_ttft_source.argtypes = [_P, _I32]
+    lib.lr_calibrate.argtypes = [_P, ctypes.c_int64, _P, _P, _P, _I32, _P, _P]
     lib.lr_read_state.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.lr_status.argtypes = [_P, _P]
     lib.lr_strerror.argtypes = [ctypes.c_int]
@@ -76,7 +77,7 @@ def load_library(path: str = LIB_PATH):
     lib.lr_last_error.restype = ctypes.c_char_p
     for name in ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
                  "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
-                 "lr_set_queue_params", "lr_set_ttft_source"):
+                 "lr_set_queue_params", "lr_set_ttft_source", "lr_calibrate"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -267,6 +268,18 @@ class LatencyRouter:
     def set_ttft_source(self, source: int):
         """LR_TTFT_SFS (default), LR_TTFT_THROUGHPUT or LR_TTFT_LPS."""
         self._check(self._lib.lr_set_ttft_source(self._h, int(source)), "lr_set_ttft_source")
+
+    def calibrate(self, features: torch.Tensor, model: torch.Tensor, time: torch.Tensor, shared_beta1: bool = True,
+                  out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+        """Least-squares batch-time coefficients per model, [M, 5] fp64, from a batch log."""
+        N = int(model.numel())
+        if out is None:
+            out = torch.empty((self.num_models, 5), dtype=torch.float64, device=model.device)
+        self._check(self._lib.lr_calibrate(self._h, N, _dev(features, torch.int64, "features", N * 5),
+                                           _dev(model, torch.int32, "model", N), _dev(time, torch.float64, "time", N),
+                                           1 if shared_beta1 else 0, _dev(out, torch.float64, "coef_out", self.num_models * 5),
+                                           _stream(stream)), "lr_calibrate")
+        return out
 
     def advance(self, assign: torch.Tensor, prompt_len: torch.Tensor, dec: torch.Tensor, t_now: float,
                 stream=None):
