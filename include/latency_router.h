@@ -231,10 +231,10 @@ LR_API int lr_set_ttft_source(lr_ctx *ctx, int32_t source);
  * in [0, M); time: [N] fp64 device, observed seconds.  shared_beta1 != 0 fits the paper's
  * four-coefficient form (one beta1, regressor F1 + F2), otherwise five coefficients.
  * coef_out: [M][5] fp64 device (beta0, beta1p, beta1d, beta2, beta3), NaN for a model with
- * fewer rows than unknowns or a rank-deficient design.  Rows with a model outside [0, M)
- * or a non-finite time are skipped and record LR_EINVAL.  Sums are fp64 atomics, so the
- * last bits may differ between runs.  Rows grouped by model are the fast case.
- * Requires num_models <= 256. */
+ * fewer rows than unknowns or a rank-deficient design.  The sums are exact integers
+ * (features must lie in [0, 2^32), times in [0, 2^19) s, kept to 2^-44 s, N < 2^32); rows
+ * outside those ranges or with a model outside [0, M) are skipped and record LR_EINVAL.
+ * Rows grouped by model are the fast case.  Requires num_models <= 128. */
 LR_API int lr_calibrate(lr_ctx *ctx, int64_t N, const int64_t *features, const int32_t *model, const double *time,
                         int32_t shared_beta1, double *coef_out, void *cuda_stream);
 

@@ -25,7 +25,7 @@ struct lr_ctx {
     // average-case TTFT sources
     lr::QueueRaw *qraw = nullptr;
     lr::QueueDev *qd = nullptr;
-    double *cal_acc = nullptr;  // calibration sums [M][kCalAcc]
+    unsigned long long *cal_acc = nullptr;  // calibration sums [M][kCalAcc][2] (128-bit)
     int source = lr::kSrcSfs;
     bool have_qp = false, have_lps = false;
     std::vector<void *> allocs;
@@ -251,7 +251,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     LR_ALLOC(c->scratch_tch, (size_t)cfg->max_pairs * cfg->max_queries);
     LR_ALLOC(c->qraw, I);
     LR_ALLOC(c->qd, I);
-    LR_ALLOC(c->cal_acc, (size_t)M * lr::kCalAcc);
+    LR_ALLOC(c->cal_acc, (size_t)M * lr::kCalAcc * 2);
 #undef LR_ALLOC
     e = cudaMemcpy(moi, cfg->model_of_instance, I * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(B, cfg->max_batched_tokens, I * 4, cudaMemcpyHostToDevice);
@@ -521,9 +521,9 @@ int lr_calibrate(lr_ctx *c, int64_t N, const int64_t *features, const int32_t *m
     c->err.clear();
     if (N < 0) return fail(c, LR_EINVAL, "N < 0");
     if (!coef_out || (N > 0 && (!features || !model || !time))) return fail(c, LR_EINVAL, "null array");
-    if (c->cfg.M > lr::kCalMaxModels) return fail(c, LR_ECAPACITY, "calibration supports at most 256 models");
+    if (c->cfg.M > lr::kCalMaxModels) return fail(c, LR_ECAPACITY, "calibration supports at most 128 models");
     cudaError_t e = lr::launch_calibrate(N, reinterpret_cast<const long long *>(features), model, time, c->cfg.M,
-                                         shared_beta1 ? 1 : 0, c->cal_acc, coef_out, c->ctl, 2 * c->sms,
+                                         shared_beta1 ? 1 : 0, c->cal_acc, coef_out, c->ctl, c->sms,
                                          (cudaStream_t)stream);
     return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "calibration launch");
 }

@@ -123,9 +123,18 @@ cudaError_t launch_tile_pad(const DevConfig &c, unsigned char *tile, cudaStream_
 // Calibration of the batch-time coefficients (lr_calibrate.cu).
 constexpr int kCalCols = 5;
 constexpr int kCalAcc = 21;        // per model: 15 sums of the upper triangle of G, 5 of b, the row count
-constexpr int kCalMaxModels = 256;  // shared-memory sums of one CTA
+constexpr int kCalMaxModels = 128;  // shared-memory sums of one CTA (128-bit each)
+constexpr double kCalTimeScale = 17592186044416.0;  // 2^44: times in 2^-44 s fixed point
+constexpr double kCalTimeMax = 524288.0;            // 2^19 s
+constexpr int kCalTile = 512;                       // rows per staged tile
+constexpr int kCalStages = 4;                       // tiles in flight per CTA
+constexpr size_t kCalStageBytes = (size_t)kCalTile * (kCalCols * 8 + 8 + 4);
+// copies of the shared 128-bit sums: one per warp of the 256-thread CTA up to 16 models
+__host__ __device__ inline int cal_copies(int M) { return M <= 16 ? 8 : 1; }
+__host__ __device__ inline size_t cal_sums_bytes(int M) { return (size_t)cal_copies(M) * M * kCalAcc * 16; }
 cudaError_t launch_calibrate(long long N, const long long *F, const int32_t *model, const double *time, int M,
-                             int shared_beta1, double *acc, double *coef, DevCtl *ctl, int grid, cudaStream_t st);
+                             int shared_beta1, unsigned long long *acc, double *coef, DevCtl *ctl, int grid,
+                             cudaStream_t st);
 cudaError_t set_calib_smem(int M);
 
 // Launch helpers implemented in the kernel translation units.

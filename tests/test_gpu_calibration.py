@@ -93,3 +93,17 @@ def test_missing_models_and_bad_rows():
     keep = np.ones(len(m), bool)
     keep[[10, 11]] = False
     np.testing.assert_allclose(got[:2], oracle.calibrate(F[keep], m[keep], t[keep], M)[:2], rtol=RTOL)
+
+
+def test_unaligned_inputs_take_the_direct_path():
+    # arrays starting one row in are not 16-byte aligned: the kernel reads rows directly
+    M = 4
+    coef = coef_of(M, 7)
+    F, m, t = W.batch_log(100_001, M, seed=8, coef=coef, noise=0.03)
+    Fd, md, td = dev(F), dev(m), dev(t)
+    rt = router_for(M)
+    got = rt.calibrate(Fd[1:], md[1:], td[1:], shared_beta1=False).cpu().numpy()
+    assert rt.status() == R().LR_OK
+    np.testing.assert_allclose(got, oracle.calibrate(F[1:], m[1:], t[1:], M, shared_beta1=False), rtol=RTOL)
+    aligned = rt.calibrate(Fd, md, td, shared_beta1=False).cpu().numpy()
+    np.testing.assert_allclose(aligned, oracle.calibrate(F, m, t, M, shared_beta1=False), rtol=RTOL)
