@@ -30,8 +30,11 @@
 //     the next non-empty batch); decoders ending beyond the calendar are rare
 //     and handled by scanning the list;
 //   * the step loop itself -- a chain of dependent scheduling decisions --
-//     runs on one lane as scalar code over shared memory (prompt prefix sums,
-//     calendar, list), with runs of batches that only decode skipped in one step.
+//     is scalar code over shared memory (prompt prefix sums, calendar, list)
+//     that every lane runs on the same values, with runs of batches that only
+//     decode skipped in one step;
+//   * where only the sequence cap limits admission (every freed seat is
+//     refilled at once), up to 32 end batches are taken in one warp-wide step.
 #include "lr_internal.cuh"
 
 namespace lr {
@@ -79,6 +82,42 @@ __device__ __forceinline__ int warp_incl_sum(int x, int lane) {
     return x;
 }
 
+// Exclusive prefix sum over the warp of values in [0, 63]: one ballot per bit,
+// all independent of each other.
+__device__ __forceinline__ int warp_excl_sum6(int v, unsigned lt) {
+    int r = 0;
+#pragma unroll
+    for (int b = 0; b < 6; ++b) r += __popc(__ballot_sync(kFull, (v >> b) & 1) & lt) << b;
+    return r;
+}
+
+// Number of lanes whose key is <= x, for keys that do not decrease over the
+// lanes and a last key above x: a binary search by shuffles.
+__device__ __forceinline__ int warp_rank(int key, int x) {
+    int j = 0;
+#pragma unroll
+    for (int step = 16; step >= 1; step >>= 1) {
+        const int v = __shfl_sync(kFull, key, j + step - 1);
+        if (v <= x) j += step;
+    }
+    return j;
+}
+
+// Position of set bit number r (from 0) of x, which has more than r set bits.
+__device__ __forceinline__ int select_bit(uint32_t x, int r) {
+    int pos = 0;
+#pragma unroll
+    for (int half = 16; half >= 1; half >>= 1) {
+        const int c = __popc(x & ((1u << half) - 1u));
+        if (r >= c) {
+            r -= c;
+            x >>= half;
+            pos += half;
+        }
+    }
+    return pos;
+}
+
 // Shared-memory accesses of the step loop by 32-bit shared address: the loop is
 // a chain of dependent decisions on one lane, so every address computation and
 // every generic-to-shared translation sits on its critical path.  The volatile
@@ -99,18 +138,35 @@ __device__ __forceinline__ void red_or(uint32_t a, uint32_t v) {
 __device__ __forceinline__ void sts4(uint32_t a, int x, int y, int z, int w) {
     asm volatile("st.shared.v4.s32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(x), "r"(y), "r"(z), "r"(w) : "memory");
 }
+// The same updates taken by the leading lane only, for scalar code that every
+// lane of the warp runs on the same values.
+__device__ __forceinline__ void red_add_if(bool p, uint32_t a, int v) {
+    asm volatile("{\n\t.reg .pred q;\n\tsetp.ne.u32 q, %0, 0;\n\t@q red.shared.add.s32 [%1], %2;\n\t}"
+                 ::"r"((unsigned)p), "r"(a), "r"(v) : "memory");
+}
+__device__ __forceinline__ void red_or_if(bool p, uint32_t a, uint32_t v) {
+    asm volatile("{\n\t.reg .pred q;\n\tsetp.ne.u32 q, %0, 0;\n\t@q red.shared.or.b32 [%1], %2;\n\t}"
+                 ::"r"((unsigned)p), "r"(a), "r"(v) : "memory");
+}
+__device__ __forceinline__ void sts4_if(bool p, uint32_t a, int x, int y, int z, int w) {
+    asm volatile("{\n\t.reg .pred q;\n\tsetp.ne.u32 q, %0, 0;\n\t@q st.shared.v4.s32 [%1], {%2, %3, %4, %5};\n\t}"
+                 ::"r"((unsigned)p), "r"(a), "r"(x), "r"(y), "r"(z), "r"(w) : "memory");
+}
 
-// Scalar view of one instance's trajectory state, used by a single lane: the
-// step loop is a chain of dependent decisions, so it runs as plain scalar
-// code over shared memory without warp-wide round trips.
+// Scalar view of one instance's trajectory state.  The step loop is a chain of
+// dependent decisions: every lane runs it as the same scalar code over shared
+// memory (loads broadcast), and only the leading lane stores.
 struct Track {
     uint32_t cal, bm, dl;       // shared addresses of the calendar, its bitmap and the decoder list
     int nlist;                  // decoders in the list
     unsigned long long words;   // bit w set: calendar word w has a non-empty batch
+    int lane;                   // lane 0 stores
+    bool lead;
 
     // Smallest last-decode batch >= L of any decoder; ends beyond the calendar
     // (always later than every calendar end) are found in the list.
     __device__ int next_end(int L) const {
+        __syncwarp();  // the leading lane's appends are visible to every lane
         if (L < kCalendar) {
             const int w = L >> 5;
             const uint32_t word = (uint32_t)lds(bm + 4u * w) & (~0u << (L & 31));
@@ -121,31 +177,32 @@ struct Track {
                 return (w2 << 5) + __ffs(lds(bm + 4u * w2)) - 1;
             }
         }
-        int mn = kBig;
-        for (int i = 0; i < nlist; ++i) {
+        int mn = kBig;  // the lanes split the list
+        for (int i = lane; i < nlist; i += 32) {
             const int f = lds(dl + 16u * i + 4u);
             if (f >= L && f < mn) mn = f;
         }
-        return mn;
+        return __reduce_min_sync(kFull, mn);
     }
 
     // Number of decoders whose last decode batch is fc.
     __device__ int ends_at(int fc) const {
+        __syncwarp();
         if (fc < kCalendar) return lds(cal + 4u * fc);
         int eq = 0;
-        for (int i = 0; i < nlist; ++i) eq += (lds(dl + 16u * i + 4u) == fc) ? 1 : 0;
-        return eq;
+        for (int i = lane; i < nlist; i += 32) eq += (lds(dl + 16u * i + 4u) == fc) ? 1 : 0;
+        return __reduce_add_sync(kFull, eq);
     }
 
     // A new decoder with first decode batch s and last decode batch f.  The
     // calendar updates are reductions whose results are not returned, so the
     // loop does not wait for a load-modify-store round trip.
     __device__ void append(int s, int f, int cb) {
-        sts4(dl + 16u * nlist, s, f, cb, 0);
+        sts4_if(lead, dl + 16u * nlist, s, f, cb, 0);
         ++nlist;
         if (f < kCalendar) {
-            red_add(cal + 4u * f, 1);
-            red_or(bm + 4u * (f >> 5), 1u << (f & 31));
+            red_add_if(lead, cal + 4u * f, 1);
+            red_or_if(lead, bm + 4u * (f >> 5), 1u << (f & 31));
             words |= 1ull << (f >> 5);
         }
     }
@@ -285,29 +342,126 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         (unsigned long long)__ballot_sync(kFull, m.bm[lane] != 0u) |
         ((unsigned long long)__ballot_sync(kFull, m.bm[lane + 32] != 0u) << 32);
 
-    // Step the scheduler on lane 0 until a query appended now would be admitted.
-    if (lane == 0) {
+    // Step the scheduler until a query appended now would be admitted.  Every
+    // lane runs the loop on the same values; the whole warp joins in for runs of
+    // end batches in which only seats limit admission.
+    {
         Track tr;
         tr.cal = saddr(m.cal);
         tr.bm = saddr(m.bm);
         tr.dl = saddr(m.dl);
         tr.nlist = n0;
         tr.words = words0;
-        const uint32_t sP = saddr(m.P), sW = saddr(m.wdec);
+        tr.lane = lane;
+        tr.lead = lane == 0;
+        const uint32_t sP = saddr(m.P), sW = saddr(m.wdec), sE = saddr(m.scr);
         bool pf = pfR > 0;
         int n = n0;  // decoders alive at the start of batch l
         int l = 1, head = 0, iters = 0;
         int ph = 0;  // prompt prefix sum at the waiting head
         int fnext = tr.next_end(1);
         int la = 0, r0 = 0;
-        int pn_head = lds(sP + 4u);
-        int d_head = lds(sW);
+
+        // A seat-limited run.  Precondition: after batch e0 every seat is held by
+        // a decoder, no prompt is part-way, and decoders end in batch
+        // e0 < kCalendar.  Let e0 = e_0 < e_1 < ... be the next batches in which
+        // decoders end, c_k how many.  Batch e_k + 1 then runs S - c_k decoders
+        // and admits exactly the next c_k waiting requests, as long as (a) the
+        // queue holds them, (b) their prompts fit the budget B - (S - c_k) whole
+        // and (c) no request admitted after e_j (j < k) ends by batch e_k (in the
+        // first-token-on-prefill mode a one-token request ends in its prefill
+        // batch, so (c) excludes those too).  Lane k takes e_k (up to 32 end
+        // batches), lane i the i-th request admitted in the run (up to 32).  The
+        // run keeps the longest valid prefix: the admissions after e_0 .. e_{K-1}
+        // are appended in FCFS order, and the state moves to batch e_K + 1, whose
+        // admissions the scalar step takes.  Returns false if K = 0.
+        auto seat_run = [&](int e0) -> bool {
+            __syncwarp();
+            const unsigned lt = (1u << lane) - 1u;
+            // waiting request head + lane: its decode length and the prompt sum through it
+            const int rq = head + lane;
+            const int dq = rq < nw ? lds(sW + 4u * rq) : 0;
+            const int pq = rq < nw ? lds(sP + 4u * (rq + 1)) : 0;
+            // e_k: set bit k of the calendar bitmap from e0 on (32 words ahead at most)
+            const int w0 = e0 >> 5;
+            uint32_t bits = w0 + lane < kCalendar / 32 ? (uint32_t)lds(tr.bm + 4u * (w0 + lane)) : 0u;
+            bits &= lane == 0 ? ~0u << (e0 & 31) : ~0u;
+            const int nb = __popc(bits);
+            const int nbx = warp_excl_sum6(nb, lt);
+            const int ne = min(__shfl_sync(kFull, nbx + nb, 31), 32);
+            int e = kBig;
+            {
+                const int j = warp_rank(nbx + nb, lane);  // the word holding bit number lane
+                const uint32_t x = __shfl_sync(kFull, bits, j);
+                const int r = lane - __shfl_sync(kFull, nbx, j);
+                if (lane < ne) e = ((w0 + j) << 5) + select_bit(x, r);
+            }
+            const int ck = lane < ne ? lds(tr.cal + 4u * e) : 0;
+            const int cc = min(ck, 33);                 // more than 32 never fit the lanes
+            const int x0 = warp_excl_sum6(cc, lt);      // requests admitted before batch e_k + 1
+            const int x1 = x0 + cc;
+            const int phi = __shfl_sync(kFull, pq, (x1 - 1) & 31);  // prompt sums at the ends
+            const int plo = __shfl_sync(kFull, pq, (x0 - 1) & 31);
+            const bool ok = lane < ne && x1 <= 32 && head + x1 <= nw &&
+                            (x1 > 0 ? phi : ph) - (x0 > 0 ? plo : ph) <= B - (S - ck);
+            const unsigned bad = __ballot_sync(kFull, !ok);
+            const int A = bad ? __ffs(bad) - 1 : 32;  // (a) and (b) hold before e_A
+            const int kmax = min(A, ne - 1);
+            if (kmax <= 0) return false;
+            // request lane i: its end batch index and last decode batch
+            const int nreq = __shfl_sync(kFull, x0, kmax);
+            const int kq = warp_rank(x1, lane);
+            const int ei = __shfl_sync(kFull, e, kq & 31);
+            const int fi = lane < nreq ? ei + 1 + dq - MODE : kBig;
+            // (c): a request ending in batch f cuts the run before the first e_K >= f after its own
+            int K = kmax;
+            const int emax = __shfl_sync(kFull, e, kmax);
+            for (unsigned sh = __ballot_sync(kFull, fi <= emax); sh != 0u; sh &= sh - 1u) {
+                const int i = __ffs(sh) - 1;
+                const int f = __shfl_sync(kFull, fi, i);
+                const int first = __popc(__ballot_sync(kFull, e < f));
+                K = min(K, max(__shfl_sync(kFull, kq, i) + 1, first) - 1);
+            }
+            if (K <= 0) return false;
+            // every request admitted in the run decodes: (c) excludes the one-token ones
+            const int taken = __shfl_sync(kFull, x0, K);  // >= c_0 >= 1
+            int pprev = __shfl_up_sync(kFull, pq, 1);
+            if (lane == 0) pprev = ph;
+            unsigned wlo = 0u, whi = 0u;
+            int fmin = kBig;
+            if (lane < taken) {
+                fmin = fi;
+                sts4(tr.dl + 16u * (tr.nlist + lane), ei + 2, fi, pq - pprev - (ei + 2), 0);
+                if (fi < kCalendar) {
+                    red_add(tr.cal + 4u * fi, 1);
+                    red_or(tr.bm + 4u * (fi >> 5), 1u << (fi & 31));
+                    if (fi < kCalendar / 2) wlo |= 1u << (fi >> 5);
+                    else whi |= 1u << ((fi >> 5) - 32);
+                }
+            }
+            tr.words |= ((unsigned long long)__reduce_or_sync(kFull, whi) << 32) | __reduce_or_sync(kFull, wlo);
+            const int fK = __reduce_min_sync(kFull, fmin);       // > e_K
+            const int eK = __shfl_sync(kFull, e, K);
+            const int cK = __shfl_sync(kFull, ck, K);
+            const int eN = __shfl_sync(kFull, e, (K + 1) & 31);  // the next end batch if K + 1 < ne
+            const int pK = __shfl_sync(kFull, pq, taken - 1);
+            __syncwarp();  // the appended decoders are visible to every lane
+            tr.nlist += taken;
+            head += taken;
+            ph = pK;
+            n = S - cK;
+            l = eK + 1;
+            fnext = K + 1 < ne ? min(eN, fK) : tr.next_end(l);
+            return true;
+        };
+
         while (iters < c.max_iters && l < (1 << 30)) {
             ++iters;
             int cnt = n + (pf ? 1 : 0);  // requests running in batch l
             if (!pf && cnt >= S) {
                 // Every sequence slot is taken: nothing but decoding until one frees.
                 if (fnext == kBig) break;  // excluded: a decoder is running
+                if (fnext < kCalendar && seat_run(fnext)) continue;
                 n -= tr.ends_at(fnext);
                 l = fnext + 1;
                 fnext = tr.next_end(l);
@@ -339,33 +493,50 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                     fnext = min(fnext, f);
                 }
             }
-            // FCFS admission while budget and a sequence slot remain.
-            // requests this batch can admit at most: the queue and the free seats
-            const int lim = min(nw, head + (S - cnt));
+            // FCFS admission while budget and a sequence slot remain, up to 32
+            // requests at a time: the prompt prefix sums increase, so the requests
+            // that fit whole are a prefix of the queue (lane i tests head + i).
+            const int lim = min(nw, head + (S - cnt));  // the queue and the free seats
             const int head0 = head;
             while (budget > 0 && head < lim) {
-                const int pn = pn_head;
-                const int d = d_head;
-                const int p = pn - ph;
-                ++head;
-                ph = pn;
-                // the next head's prompt sum and length, loaded ahead of their use
-                // (head <= nw <= capW here: both reads are in bounds, the pads included)
-                pn_head = lds(sP + 4u * (head + 1));
-                d_head = lds(sW + 4u * head);
-                if (p <= budget) {
-                    budget -= p;
-                    int f, cb;
-                    if (decoder_of<MODE>(l, p, d, &f, &cb)) {
-                        tr.append(l + 1, f, cb);
-                        fnext = min(fnext, f);
+                const int r = head + lane;
+                const int pe = r < lim ? lds(sP + 4u * (r + 1)) : 0;  // prompt sum through request r
+                const bool whole = r < lim && pe - ph <= budget;
+                const int k = __popc(__ballot_sync(kFull, whole));
+                if (k > 0) {
+                    int before = __shfl_up_sync(kFull, pe, 1);
+                    if (lane == 0) before = ph;
+                    int f = kBig, cb = 0;
+                    const bool dec = whole && decoder_of<MODE>(l, pe - before, lds(sW + 4u * r), &f, &cb);
+                    const unsigned dm = __ballot_sync(kFull, dec);
+                    unsigned wlo = 0u, whi = 0u;
+                    if (dec) {
+                        sts4(tr.dl + 16u * (tr.nlist + __popc(dm & lanemask_lt())), l + 1, f, cb, 0);
+                        if (f < kCalendar) {
+                            red_add(tr.cal + 4u * f, 1);
+                            red_or(tr.bm + 4u * (f >> 5), 1u << (f & 31));
+                            if (f < kCalendar / 2) wlo |= 1u << (f >> 5);
+                            else whi |= 1u << ((f >> 5) - 32);
+                        }
                     }
-                } else {  // the prompt continues in later batches
+                    tr.words |= ((unsigned long long)__reduce_or_sync(kFull, whi) << 32) | __reduce_or_sync(kFull, wlo);
+                    fnext = min(fnext, __reduce_min_sync(kFull, f));
+                    tr.nlist += __popc(dm);
+                    const int pk = __shfl_sync(kFull, pe, k - 1);
+                    budget -= pk - ph;
+                    ph = pk;
+                    head += k;
+                }
+                if (k < 32 && budget > 0 && head < lim) {
+                    // the next prompt does not fit whole: it continues in later batches
+                    const int pn = lds(sP + 4u * (head + 1));
                     pf = true;
-                    pfR = p - budget;
+                    pfR = pn - ph - budget;
                     pfC = budget;
-                    pfD = d;
+                    pfD = lds(sW + 4u * head);
                     budget = 0;
+                    ++head;
+                    ph = pn;
                 }
             }
             cnt += head - head0;  // every request taken from the queue holds a seat
@@ -376,15 +547,20 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             }
             n += tr.nlist - nl0;
             if (l == fnext) {
+                // all seats held by decoders after this batch: a seat-limited run may follow
+                if (!pf && n == S && fnext < kCalendar && seat_run(l)) continue;
                 n -= tr.ends_at(l);
                 fnext = tr.next_end(l + 1);
             }
             ++l;
         }
-        m.scr[0] = la;
-        m.scr[1] = r0;
-        m.scr[2] = tr.nlist;
-        m.scr[3] = iters;
+        __syncwarp();  // the run's scratch is read before it is overwritten
+        if (lane == 0) {
+            m.scr[0] = la;
+            m.scr[1] = r0;
+            m.scr[2] = tr.nlist;
+            m.scr[3] = iters;
+        }
     }
     __syncwarp();
     const int la = m.scr[0];

@@ -89,6 +89,23 @@ def test_random_small_pools(mode):
         rt.close()
 
 
+@pytest.mark.parametrize("mode", [0, 1])
+def test_seat_limited_pools(mode):
+    # long queues behind nearly full seat caps: most admissions refill the seats freed
+    # in the batch before, which the trajectory kernel takes many end batches at a
+    # time; prompts close to the budget, short responses and queues that run out in
+    # the middle of such a run cut it short
+    for seed in range(8):
+        wl = W.small_workload(seed, num_instances=32, num_models=3, num_queries=29, cap_running=64,
+                              cap_waiting=128, first_token_mode=mode, budget_range=(300, 1200), min_gap=8)
+        rt = make_router(wl)
+        F, t, fb = full_estimate(rt, wl)
+        Q, I = wl.num_queries, wl.num_instances
+        qq, jj = np.meshgrid(np.arange(Q), np.arange(I), indexing="ij")
+        check_candidates(wl, F.reshape(-1, 5), t.ravel(), fb.ravel(), qq.ravel(), jj.ravel())
+        rt.close()
+
+
 def test_instance_tiles_beyond_one_cta():
     # 300 instances: the estimate kernel splits instances over several CTAs
     wl = W.small_workload(101, num_instances=300, num_models=5, num_queries=37, budget_range=(16, 128), min_gap=16)
