@@ -77,7 +77,7 @@ typedef struct {
     const int32_t *max_seqs;           /* [I] sequence cap S_j, 1 <= S_j <= B_j */
     int32_t cap_running;               /* row stride of the running arrays (>= 1) */
     int32_t cap_waiting;               /* row stride of the waiting arrays (>= 1) */
-    int32_t max_queries;               /* largest Q of any call */
+    int32_t max_queries;               /* largest Q of any call, 1 .. 2^30 */
     int32_t max_pairs;                 /* largest P of lr_route, 1..64 */
     int32_t max_prompt_len;            /* largest prompt length of any query, 1..2^20 */
     int32_t first_token_mode;          /* enum lr_first_token_mode */

@@ -22,6 +22,7 @@ struct lr_ctx {
     int max_seqs = 0;
     size_t k3_smem = 0;
     float *scratch_tch = nullptr;
+    uint32_t *k2_work = nullptr;  // the candidate kernel's row counters
     // average-case TTFT sources
     lr::QueueRaw *qraw = nullptr;
     lr::QueueDev *qd = nullptr;
@@ -118,6 +119,18 @@ lr_ctx::Shape make_shape(const lr::DevConfig &d, bool route, int max_pairs) {
     return s;
 }
 
+// Row split of a candidate-kernel launch of `ctas` CTAs per tile.  The CTAs that fit
+// beside a snapshot load's K1 CTAs (one candidate-kernel slot each) start with a
+// static range of 90% of their share of the rows; the other rows are claimed as
+// they run out, by the remaining CTAs and by whichever finish early, so that every
+// CTA ends on small claimed chunks.
+void set_row_split(lr::K2Launch &a, const lr_ctx *c, int ctas, int tiles, int occ) {
+    const int k1 = (c->cfg.I + lr::kK1Warps - 1) / lr::kK1Warps;
+    a.first_ctas = tiles == 1 ? std::max(0, std::min(ctas, c->sms * occ - k1)) : 0;
+    const int f = (int)((long long)a.Q * 9 / (10LL * std::max(1, ctas)));
+    a.first_rows = std::max(a.QS, f - f % a.QS);
+}
+
 lr::K2Launch k2_base(const lr_ctx *c) {
     lr::K2Launch a;
     std::memset(&a, 0, sizeof(a));
@@ -127,6 +140,7 @@ lr::K2Launch k2_base(const lr_ctx *c) {
     a.ctl = c->ctl;
     a.src = c->source;
     a.qd = c->qd;
+    a.work = c->k2_work;
     return a;
 }
 
@@ -152,7 +166,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
         return bail(LR_EINVAL, "null configuration array");
     if (cfg->cap_running < 1 || cfg->cap_waiting < 1 || cfg->cap_running > 4096 || cfg->cap_waiting > 4096)
         return bail(LR_EINVAL, "cap_running / cap_waiting out of range");
-    if (cfg->max_queries < 1 || cfg->max_pairs < 1 || cfg->max_pairs > lr::kMaxPairs)
+    if (cfg->max_queries < 1 || cfg->max_queries > (1 << 30) || cfg->max_pairs < 1 || cfg->max_pairs > lr::kMaxPairs)
         return bail(LR_EINVAL, "max_queries / max_pairs out of range");
     if (cfg->max_prompt_len < 1 || cfg->max_prompt_len > (1 << 20)) return bail(LR_EINVAL, "max_prompt_len out of range");
     if (cfg->first_token_mode != LR_FIRST_TOKEN_SEPARATE_DECODE && cfg->first_token_mode != LR_FIRST_TOKEN_WITH_LAST_CHUNK)
@@ -249,6 +263,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     }
     LR_ALLOC(c->ctl, 1);
     LR_ALLOC(c->scratch_tch, (size_t)cfg->max_pairs * cfg->max_queries);
+    LR_ALLOC(c->k2_work, lr::k2_work_words(I));
     LR_ALLOC(c->qraw, I);
     LR_ALLOC(c->qd, I);
     LR_ALLOC(c->cal_acc, (size_t)M * lr::kCalAcc * 2);
@@ -263,6 +278,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     if (e == cudaSuccess) e = cudaMemcpy(pout, cfg->price_out, M * 4, cudaMemcpyHostToDevice);
     lr::DevCtl ctl0{-1, 0, 0, 0u};
     if (e == cudaSuccess) e = cudaMemcpy(c->ctl, &ctl0, sizeof(ctl0), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemset(c->k2_work, 0, sizeof(uint32_t) * lr::k2_work_words(I));
     if (e != cudaSuccess) return bail(LR_ECUDA, cudaGetErrorString(e));
     d.moi = moi;
     d.B = B;
@@ -350,6 +366,7 @@ static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, 
     a.QT = c->est.QT;
     a.vec_ok = (c->cfg.I % 4 == 0) && ((uintptr_t)ttft % 16 == 0);
     dim3 grid(std::min(c->sms * c->est.occ, (Q + a.QS - 1) / a.QS), c->est.tiles);
+    set_row_split(a, c, (int)grid.x, (int)grid.y, c->est.occ);
     e = lr::launch_cand(a, lr::cand_out_flags(true, iters != nullptr, false, false, 1), grid, lr::kK2Block,
                         c->est.smem, (cudaStream_t)stream);
     return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "estimate launch");
@@ -404,6 +421,7 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
     a.QT = c->rt.QT;
     a.vec_ok = (c->cfg.I % 4 == 0) && ((uintptr_t)ttft_matrix_out % 16 == 0);
     dim3 grid(std::min(c->sms * c->rt.occ, (Q + a.QS - 1) / a.QS), 1);
+    set_row_split(a, c, (int)grid.x, 1, c->rt.occ);
     cudaError_t e = lr::launch_cand(a, lr::cand_out_flags(ttft_matrix_out != nullptr, false, true, tau != nullptr, P),
                                     grid, lr::kK2Block, c->rt.smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(c, e, "route launch");

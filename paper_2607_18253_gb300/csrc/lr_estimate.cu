@@ -223,6 +223,51 @@ struct Flag {
     static constexpr bool value = B;
 };
 
+// The rows of a launch, per tile, as ranges (x, end) that a CTA works through QT rows
+// at a time.  CTA b < first_ctas starts with the static range [b F, (b + 1) F)
+// (F = first_rows, most of its share of the rows): those CTAs fit beside a snapshot
+// load's CTAs running on another stream and start at once.  The remaining rows are
+// claimed from the tile's counter, which counts the rows past the static ones: QT
+// rows while many are left, down to 4 QS at the end (a claim's atomic still returns
+// well within the chunk before it).  So CTAs that start late (their SM busy with the
+// load) or run slower take less, and all finish at about the same time.  `seen` is
+// a row index recently reached.
+__device__ __forceinline__ int claim_size(const K2Launch &a, int seen) {
+    const int n = (a.Q - seen) / (int)gridDim.x;
+    return min(a.QT, max(4 * a.QS, n - n % a.QS));
+}
+__device__ __forceinline__ int static_rows(const K2Launch &a) { return min(a.Q, a.first_ctas * a.first_rows); }
+__device__ __forceinline__ int claim_rows(const K2Launch &a, int seen) {
+    return static_rows(a) + (int)atomicAdd(a.work + 1 + blockIdx.y, (unsigned)claim_size(a, seen));
+}
+__device__ __forceinline__ int2 first_range(const K2Launch &a) {
+    if ((int)blockIdx.x < a.first_ctas)
+        return make_int2((int)blockIdx.x * a.first_rows, ((int)blockIdx.x + 1) * a.first_rows);
+    const int seen = static_rows(a) + (int)*(volatile uint32_t *)(a.work + 1 + blockIdx.y);
+    const int x = claim_rows(a, seen);
+    return make_int2(x, x + claim_size(a, seen));
+}
+// The range left after the chunk at the head of r, if any: no claim needed.
+__device__ __forceinline__ bool has_rest(const K2Launch &a, int2 r) { return r.x + a.QT < min(r.y, a.Q); }
+// The range that follows the chunk at the head of r (the claim x was made for it).
+__device__ __forceinline__ int2 range_after(const K2Launch &a, int2 r, int x) {
+    return has_rest(a, r) ? make_int2(r.x + a.QT, r.y) : make_int2(x, x + claim_size(a, r.x));
+}
+
+// End of a candidate-kernel CTA: the last of `ctas` to finish clears the row
+// counters of the `tiles` tiles and the completion count for the next launch.
+__device__ __forceinline__ void k2_finish(uint32_t *work, unsigned ctas, unsigned tiles) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        if (atomicAdd(work, 1u) == ctas - 1) {
+            for (unsigned y = 0; y < tiles; ++y) atomicExch(work + 1 + y, 0u);
+            atomicExch(work, 0u);
+            __threadfence();
+        }
+    }
+}
+
 // MODE 0 / 1: SFS with the first output token in its own batch / with the last
 // prompt chunk.  MODE 2: an average-case source (Sec. 4, App. E), affine in p:
 // t = fma(p, g_j, C_j) with g_j = fp32(1/theta_j) and C_j = fp32(W_j + Tdec_j).
@@ -242,33 +287,44 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     const int j0 = blockIdx.y * Gp * 4;
     const int jb = j0 + 4 * g;                         // first instance of this thread
     const int nv = max(0, min(4, I - jb));             // instances this thread owns
-    const int rows_per = (a.Q + gridDim.x - 1) / gridDim.x;
-    const int rb = blockIdx.x * rows_per;
-    const int re = min(a.Q, rb + rows_per);
-    if (rb >= re) return;
+    // Query rows come in ranges (first_range, range_after): a static one, then claims
+    // from this tile's counter, in the no-snapshot path as in the main one.
     // one read of the live-buffer index per CTA (every thread reading the same word
     // would queue them all on one L2 line)
     __shared__ int s_active;
+    __shared__ int2 s_claim[2];
     if (threadIdx.x == 0) s_active = load_acquire(&a.ctl->active);
     __syncthreads();
     const int active = s_active;
     // the LPS source needs no live snapshot; every other source does
     if (active < 0 && !(AFF && a.src == kSrcLps)) {
         if (threadIdx.x == 0) record_status(a.ctl, kENoState);
-        for (int rr = rb + qs; rr < re; rr += QS) {
-            for (int u = 0; u < nv; ++u) {
-                if (OUT & kOutMatrix) a.ttft[(size_t)rr * I + jb + u] = kNaN;
-                if (OUT & kOutIters) a.first_batch[(size_t)rr * I + jb + u] = -1;
+        for (int k = 0;; ++k) {
+            __syncthreads();  // the previous range has been read
+            if (threadIdx.x == 0) {
+                const int2 r = s_claim[0];
+                s_claim[0] = k == 0 ? first_range(a) : range_after(a, r, has_rest(a, r) ? 0 : claim_rows(a, r.x));
             }
-            if (ROUTE && g == 0)
-                for (int pp = 0; pp < a.P; ++pp) {
-                    a.assign[(size_t)pp * a.Q + rr] = -1;
-                    a.util[(size_t)pp * a.Q + rr] = kNaN;
-                    if (a.ttft_chosen) a.ttft_chosen[(size_t)pp * a.Q + rr] = kNaN;
+            __syncthreads();
+            const int rb = s_claim[0].x, re = min(min(a.Q, s_claim[0].y), rb + QT);
+            if (rb >= a.Q) break;
+            for (int rr = rb + qs; rr < re; rr += QS) {
+                for (int u = 0; u < nv; ++u) {
+                    if (OUT & kOutMatrix) a.ttft[(size_t)rr * I + jb + u] = kNaN;
+                    if (OUT & kOutIters) a.first_batch[(size_t)rr * I + jb + u] = -1;
                 }
+                if (ROUTE && g == 0)
+                    for (int pp = 0; pp < a.P; ++pp) {
+                        a.assign[(size_t)pp * a.Q + rr] = -1;
+                        a.util[(size_t)pp * a.Q + rr] = kNaN;
+                        if (a.ttft_chosen) a.ttft_chosen[(size_t)pp * a.Q + rr] = kNaN;
+                    }
+            }
         }
+        k2_finish(a.work, gridDim.x * gridDim.y, gridDim.y);
         return;
     }
+    {
     const StateBuf sb = active ? a.buf1 : a.buf0;
     // Shared memory: the tile block (tables and per-instance scalars, exactly as K1
     // laid it out for this tile), query records, row partials, utility inputs,
@@ -295,13 +351,10 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     // cheaper than thousands of scattered loads of the same lines.
     __shared__ __align__(8) unsigned long long s_mbar;
     const uint32_t mbar = (uint32_t)__cvta_generic_to_shared(&s_mbar);
-    if (!AFF) {
-        if (threadIdx.x == 0) {
+    if (threadIdx.x == 0) {
+        if (!AFF) {
             asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar) : "memory");
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        }
-        __syncthreads();
-        if (threadIdx.x == 0) {
             const uint32_t bytes = (uint32_t)tile_bytes(c);
             const unsigned char *src = sb.tile + (size_t)blockIdx.y * tile_bytes(c);
             // the block was written by generic stores (possibly of a load on another
@@ -314,7 +367,13 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                 "l"(src), "r"(bytes), "r"(mbar)
                 : "memory");
         }
+        s_claim[0] = first_range(a);
     }
+    __syncthreads();
+    const int2 first = s_claim[0];
+    // what follows the first chunk: found now, published once the tile block has landed
+    int2 second = make_int2(a.Q, a.Q);
+    if (threadIdx.x == 0 && first.x < a.Q) second = range_after(a, first, has_rest(a, first) ? 0 : claim_rows(a, first.x));
     // copies of query rows [q0, q0 + nrows) into raw buffer b
     auto issue = [&](int q0, int nrows, int b) {
         for (int t = threadIdx.x; t < nrows; t += blockDim.x) {
@@ -330,7 +389,8 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
         }
         cp_async_commit();
     };
-    issue(rb, min(QT, re - rb), 0);  // the first chunk travels while the tile block lands
+    // the first chunk travels while the tile block lands
+    if (first.x < a.Q) issue(first.x, min(QT, min(first.y, a.Q) - first.x), 0);
     if (!AFF) {
         // bounded wait for the tile block; a copy that never lands is reported, not waited out
         bool landed = false;
@@ -340,7 +400,7 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
             for (int it = 0; it < (1 << 22) && !mbar_test(mbar); ++it) {
             }
             cp_async_wait<0>();
-            return;
+            goto finish;
         }
     }
     Inst4 r;
@@ -374,20 +434,18 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
         la[u] = s_scal[kScLa * fs + col];
         if (u < nv) fast_mine = fast_mine && s_scal[kScFast * fs + col] != 0;
     }
+    if (threadIdx.x == 0) s_claim[1] = second;
     const bool fast = __syncthreads_and(fast_mine);
     const bool vec = a.vec_ok && nv == 4;
     const unsigned gmask = group_mask(Gp, lane);
     const int grp_lane0 = lane & ~(min(Gp, 32) - 1);  // first lane of this row group in the warp
     const int wrow = g / 32;                          // warp index within a wide row
-    // shared addresses of this thread's table columns: entry (k, u) at ecol[u] + k * erow,
-    // bucket (b, u) at bcol[u] + b * brow
-    uint32_t ecol[4], bcol[4];
-    const uint32_t e0 = (uint32_t)__cvta_generic_to_shared(s_ent), b0 = (uint32_t)__cvta_generic_to_shared(s_bkt);
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-        ecol[u] = e0 + 16u * (uint32_t)(u * Gp + g);
-        bcol[u] = b0 + 8u * (uint32_t)(u * Gp + g);
-    }
+    // shared addresses of this thread's table columns: entry (k, u) at
+    // ecol + u * ecst + k * erow, bucket (b, u) at bcol + u * bcst + b * brow (formed
+    // at each use: the kernel is at its register limit)
+    const uint32_t ecol = (uint32_t)__cvta_generic_to_shared(s_ent) + 16u * (uint32_t)g;
+    const uint32_t bcol = (uint32_t)__cvta_generic_to_shared(s_bkt) + 8u * (uint32_t)g;
+    const uint32_t ecst = 16u * (uint32_t)Gp, bcst = 8u * (uint32_t)Gp;
     const uint32_t erow = 16u * 4u * (uint32_t)Gp, brow = 8u * 4u * (uint32_t)Gp;
     bool same_model = true;
 #pragma unroll
@@ -395,16 +453,26 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
 
     auto run = [&](auto fast_tag) {
         constexpr bool FAST = decltype(fast_tag)::value;
-        int buf = 0;
-        for (int q0 = rb; q0 < re; q0 += QT, buf ^= 1) {
-            const int nrows = min(QT, re - q0);
-            if (q0 + QT < re) {
-                issue(q0 + QT, min(QT, re - q0 - QT), buf ^ 1);
-                cp_async_wait<1>();
-            } else {
-                cp_async_wait<0>();
+        // chunk k: the first QT rows of the range in s_claim[k & 1], staged in raw buffer k & 1
+        for (int buf = 0;; buf ^= 1) {
+            int q0, nrows;
+            {
+                const int2 cur = s_claim[buf], nxt = s_claim[buf ^ 1];
+                if (cur.x >= a.Q) break;
+                q0 = cur.x;
+                nrows = min(QT, min(cur.y, a.Q) - q0);
+                if (nxt.x < a.Q) {
+                    issue(nxt.x, min(QT, min(nxt.y, a.Q) - nxt.x), buf ^ 1);
+                    cp_async_wait<1>();
+                } else {
+                    cp_async_wait<0>();
+                }
             }
             __syncthreads();  // every thread's copies of this chunk have landed
+            // the range after the next chunk: claimed now if needed, published when this chunk is done
+            int ahead = a.Q;
+            if (threadIdx.x == 0 && s_claim[buf ^ 1].x < a.Q && !has_rest(a, s_claim[buf ^ 1]))
+                ahead = claim_rows(a, s_claim[buf ^ 1].x);
             const int32_t *bp = r_p + buf * QT;
             for (int t = threadIdx.x; t < nrows; t += blockDim.x) {
                 bool ok;
@@ -438,9 +506,9 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                         kk[u] = 0;
                         continue;
                     }
-                    const int2 bk = lds_int2(bcol[u] + (uint32_t)(q.p >> r.shift[u]) * brow);
+                    const int2 bk = lds_int2(bcol + u * bcst + (uint32_t)(q.p >> r.shift[u]) * brow);
                     kk[u] = bk.y + (q.p > bk.x ? 1 : 0);
-                    const float4 e = lds_float4(ecol[u] + (uint32_t)kk[u] * erow);
+                    const float4 e = lds_float4(ecol + u * ecst + (uint32_t)kk[u] * erow);
                     if (FAST) t[u] = ttft_fast<MODE>(q, r, u, e);
                     else t[u] = (u < nv) ? ttft_exact64<MODE>(c, sb, q, jb + u, kk[u], e) : 0.f;
                 }
@@ -541,12 +609,19 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                     write_pick(a, (size_t)pp * a.Q + q0 + r2, (CON && c1.key == 0u) ? c2 : c1);
                 }
             }
+            if (threadIdx.x == 0) {  // into the slot this chunk was read from
+                const int2 nxt = s_claim[buf ^ 1];
+                s_claim[buf] = nxt.x < a.Q ? range_after(a, nxt, ahead) : make_int2(a.Q, a.Q);
+            }
             __syncthreads();
         }
     };
     if (fast) run(Flag<true>{});
     else run(Flag<false>{});
     (void)grp_lane0;
+    }
+finish:
+    k2_finish(a.work, gridDim.x * gridDim.y, gridDim.y);
 }
 
 // Per-pair means of (accuracy, cost, TTFT) of the chosen instances, fp64, fixed

@@ -203,7 +203,14 @@ struct K2Launch {
     // TTFT source (kSrc*) and, for the average-case ones, the instance constants
     int32_t src;
     const QueueDev *qd;
+    // [0]: CTAs finished; [1 + tile]: query rows of the tile claimed past the static
+    // ones.  Zero before a launch; the last CTA to finish clears them for the next.
+    uint32_t *work;
+    // CTAs (per tile) that start with a static chunk of first_rows query rows
+    int32_t first_ctas, first_rows;
 };
+// Entries of the candidate kernel's work counters for I instances.
+inline int k2_work_words(int I) { return (I + 1023) / 1024 + 2; }
 int cand_out_flags(bool matrix, bool iters, bool route, bool constrained, int P);
 cudaError_t launch_cand(const K2Launch &a, int out, dim3 grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_features(const K2Launch &a, int sms, cudaStream_t st);

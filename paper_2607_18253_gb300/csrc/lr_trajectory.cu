@@ -91,18 +91,6 @@ __device__ __forceinline__ int warp_excl_sum6(int v, unsigned lt) {
     return r;
 }
 
-// Number of lanes whose key is <= x, for keys that do not decrease over the
-// lanes and a last key above x: a binary search by shuffles.
-__device__ __forceinline__ int warp_rank(int key, int x) {
-    int j = 0;
-#pragma unroll
-    for (int step = 16; step >= 1; step >>= 1) {
-        const int v = __shfl_sync(kFull, key, j + step - 1);
-        if (v <= x) j += step;
-    }
-    return j;
-}
-
 // Position of set bit number r (from 0) of x, which has more than r set bits.
 __device__ __forceinline__ int select_bit(uint32_t x, int r) {
     int pos = 0;
@@ -364,17 +352,18 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
 
         // A seat-limited run.  Precondition: after batch e0 every seat is held by
         // a decoder, no prompt is part-way, and decoders end in batch
-        // e0 < kCalendar.  Let e0 = e_0 < e_1 < ... be the next batches in which
-        // decoders end, c_k how many.  Batch e_k + 1 then runs S - c_k decoders
-        // and admits exactly the next c_k waiting requests, as long as (a) the
-        // queue holds them, (b) their prompts fit the budget B - (S - c_k) whole
-        // and (c) no request admitted after e_j (j < k) ends by batch e_k (in the
-        // first-token-on-prefill mode a one-token request ends in its prefill
-        // batch, so (c) excludes those too).  Lane k takes e_k (up to 32 end
-        // batches), lane i the i-th request admitted in the run (up to 32).  The
-        // run keeps the longest valid prefix: the admissions after e_0 .. e_{K-1}
-        // are appended in FCFS order, and the state moves to batch e_K + 1, whose
-        // admissions the scalar step takes.  Returns false if K = 0.
+        // e0 < kCalendar.  If c_b decoders end in batch b, batch b + 1 then runs
+        // S - c_b decoders and admits exactly the next c_b waiting requests, as
+        // long as (a) the queue holds them, (b) their prompts fit the budget
+        // B - (S - c_b) whole and (c) no request admitted after an earlier batch
+        // of the run ends by batch b (in the first-token-on-prefill mode a
+        // one-token request ends in its prefill batch, so (c) excludes those
+        // too); batches in which no decoder ends admit nobody.  Lane k takes
+        // batch e0 + k, lane i the i-th request admitted in the run (32 at most).
+        // The run moves to the last batch e0 + K with ends before the first that
+        // breaks (a)-(c): the admissions after batches e0 .. e0 + K - 1 are
+        // appended in FCFS order, and the scalar step takes those of batch
+        // e0 + K + 1.  Returns false if there is no such K > 0.
         auto seat_run = [&](int e0) -> bool {
             __syncwarp();
             const unsigned lt = (1u << lane) - 1u;
@@ -382,56 +371,45 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             const int rq = head + lane;
             const int dq = rq < nw ? lds(sW + 4u * rq) : 0;
             const int pq = rq < nw ? lds(sP + 4u * (rq + 1)) : 0;
-            // e_k: set bit k of the calendar bitmap from e0 on (32 words ahead at most)
-            const int w0 = e0 >> 5;
-            uint32_t bits = w0 + lane < kCalendar / 32 ? (uint32_t)lds(tr.bm + 4u * (w0 + lane)) : 0u;
-            bits &= lane == 0 ? ~0u << (e0 & 31) : ~0u;
-            const int nb = __popc(bits);
-            const int nbx = warp_excl_sum6(nb, lt);
-            const int ne = min(__shfl_sync(kFull, nbx + nb, 31), 32);
-            int e = kBig;
-            {
-                const int j = warp_rank(nbx + nb, lane);  // the word holding bit number lane
-                const uint32_t x = __shfl_sync(kFull, bits, j);
-                const int r = lane - __shfl_sync(kFull, nbx, j);
-                if (lane < ne) e = ((w0 + j) << 5) + select_bit(x, r);
-            }
-            const int ck = lane < ne ? lds(tr.cal + 4u * e) : 0;
+            const bool incal = e0 + lane < kCalendar;
+            const int ck = incal ? lds(tr.cal + 4u * (e0 + lane)) : 0;
             const int cc = min(ck, 33);                 // more than 32 never fit the lanes
-            const int x0 = warp_excl_sum6(cc, lt);      // requests admitted before batch e_k + 1
+            const int x0 = warp_excl_sum6(cc, lt);      // requests admitted before batch e0 + k + 1
             const int x1 = x0 + cc;
             const int phi = __shfl_sync(kFull, pq, (x1 - 1) & 31);  // prompt sums at the ends
             const int plo = __shfl_sync(kFull, pq, (x0 - 1) & 31);
-            const bool ok = lane < ne && x1 <= 32 && head + x1 <= nw &&
-                            (x1 > 0 ? phi : ph) - (x0 > 0 ? plo : ph) <= B - (S - ck);
+            const bool ok = incal && (ck == 0 || (x1 <= 32 && head + x1 <= nw &&
+                                                  (x1 > 0 ? phi : ph) - (x0 > 0 ? plo : ph) <= B - (S - ck)));
             const unsigned bad = __ballot_sync(kFull, !ok);
-            const int A = bad ? __ffs(bad) - 1 : 32;  // (a) and (b) hold before e_A
-            const int kmax = min(A, ne - 1);
-            if (kmax <= 0) return false;
-            // request lane i: its end batch index and last decode batch
+            const unsigned em = __ballot_sync(kFull, ck > 0);  // batches with ends (lane 0 among them)
+            const int kmax = min(bad ? __ffs(bad) - 1 : 32, 31);  // (a) and (b) hold below it
+            if (kmax <= 0 || (em & ((2u << kmax) - 1u) & ~1u) == 0u) return false;
+            // request lane i: the lane of its batch (the run's request starts, by rank) and its last batch
             const int nreq = __shfl_sync(kFull, x0, kmax);
-            const int kq = warp_rank(x1, lane);
-            const int ei = __shfl_sync(kFull, e, kq & 31);
-            const int fi = lane < nreq ? ei + 1 + dq - MODE : kBig;
-            // (c): a request ending in batch f cuts the run before the first e_K >= f after its own
+            const unsigned starts = __reduce_or_sync(kFull, ck > 0 && x0 < 32 ? 1u << x0 : 0u);
+            const int kq = select_bit(em, (__popc(starts & ((2u << lane) - 1u)) - 1) & 31);
+            const int fi = lane < nreq ? e0 + kq + 1 + dq - MODE : kBig;
+            // (c): a request of lane kq ending in batch f rules out every K > kq with e0 + K >= f
             int K = kmax;
-            const int emax = __shfl_sync(kFull, e, kmax);
-            for (unsigned sh = __ballot_sync(kFull, fi <= emax); sh != 0u; sh &= sh - 1u) {
+            for (unsigned sh = __ballot_sync(kFull, fi <= e0 + kmax); sh != 0u; sh &= sh - 1u) {
                 const int i = __ffs(sh) - 1;
                 const int f = __shfl_sync(kFull, fi, i);
-                const int first = __popc(__ballot_sync(kFull, e < f));
-                K = min(K, max(__shfl_sync(kFull, kq, i) + 1, first) - 1);
+                K = min(K, max(__shfl_sync(kFull, kq, i) + 1, f - e0) - 1);
             }
             if (K <= 0) return false;
+            const unsigned cand = em & ((2u << K) - 1u) & ~1u;
+            if (cand == 0u) return false;
+            K = 31 - __clz(cand);
             // every request admitted in the run decodes: (c) excludes the one-token ones
-            const int taken = __shfl_sync(kFull, x0, K);  // >= c_0 >= 1
+            const int taken = __shfl_sync(kFull, x0, K);  // >= c_e0 >= 1
             int pprev = __shfl_up_sync(kFull, pq, 1);
             if (lane == 0) pprev = ph;
             unsigned wlo = 0u, whi = 0u;
             int fmin = kBig;
             if (lane < taken) {
+                const int e = e0 + kq;  // the admission batch is e + 1
                 fmin = fi;
-                sts4(tr.dl + 16u * (tr.nlist + lane), ei + 2, fi, pq - pprev - (ei + 2), 0);
+                sts4(tr.dl + 16u * (tr.nlist + lane), e + 2, fi, pq - pprev - (e + 2), 0);
                 if (fi < kCalendar) {
                     red_add(tr.cal + 4u * fi, 1);
                     red_or(tr.bm + 4u * (fi >> 5), 1u << (fi & 31));
@@ -440,18 +418,17 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                 }
             }
             tr.words |= ((unsigned long long)__reduce_or_sync(kFull, whi) << 32) | __reduce_or_sync(kFull, wlo);
-            const int fK = __reduce_min_sync(kFull, fmin);       // > e_K
-            const int eK = __shfl_sync(kFull, e, K);
+            const int fK = __reduce_min_sync(kFull, fmin);  // > e0 + K
             const int cK = __shfl_sync(kFull, ck, K);
-            const int eN = __shfl_sync(kFull, e, (K + 1) & 31);  // the next end batch if K + 1 < ne
             const int pK = __shfl_sync(kFull, pq, taken - 1);
+            const unsigned later = em & ~((2u << K) - 1u);  // end batches after e0 + K in the window
             __syncwarp();  // the appended decoders are visible to every lane
             tr.nlist += taken;
             head += taken;
             ph = pK;
             n = S - cK;
-            l = eK + 1;
-            fnext = K + 1 < ne ? min(eN, fK) : tr.next_end(l);
+            l = e0 + K + 1;
+            fnext = later ? min(e0 + __ffs(later) - 1, fK) : tr.next_end(l);
             return true;
         };
 

@@ -115,6 +115,19 @@ def test_instance_tiles_beyond_one_cta():
     check_candidates(wl, F.reshape(-1, 5), t.ravel(), fb.ravel(), qq.ravel(), jj.ravel())
 
 
+def test_two_instance_tiles():
+    # 1100 instances: two instance tiles, whose CTAs claim every query row dynamically
+    wl = W.small_workload(7, num_instances=1100, num_models=4, num_queries=53, budget_range=(64, 160), min_gap=64)
+    rt = make_router(wl)
+    F, t, fb = full_estimate(rt, wl)
+    qq, jj = np.meshgrid(np.arange(53), np.arange(1100), indexing="ij")
+    check_candidates(wl, F.reshape(-1, 5), t.ravel(), fb.ravel(), qq.ravel(), jj.ravel())
+    # a second call starts from counters the first one cleared
+    F2, t2, fb2 = full_estimate(rt, wl)
+    np.testing.assert_array_equal(bits(t2), bits(t))
+    rt.close()
+
+
 @pytest.mark.parametrize("name,ns", [("pool64", 40000), ("pool256", 60000)])
 def test_full_size_sampled(name, ns):
     # full query count, the launch shape the benchmark times; sampled candidates
