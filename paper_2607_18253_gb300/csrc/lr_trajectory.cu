@@ -612,38 +612,52 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         };
         // Window decoders are few but scattered, so they are first gathered into a
         // list (stable ballot compaction) and then taken 32 at a time: a warp would
-        // otherwise run the per-row path in almost every step over the list.
+        // otherwise run the per-row path in almost every step over the list.  Each
+        // lane classifies two decoders per step, loaded together.
+        // Branch-free: a decoder alive over the whole window contributes its tokens up to
+        // L0, one finished before it all of its tokens; both are the same closed form
+        // (u tokens at contexts cb + s .. cb + e: u cb + (s + e) u / 2, where (s + e) u
+        // is twice a sum of consecutive integers, so the halving is exact).
+        auto classify = [&](const int4 dd) -> bool {
+            const int s = dd.x;
+            const bool reg = s <= lk0 && dd.y >= Lend;
+            const bool fin = dd.y < lk0;
+            const int e = reg ? L0 : dd.y;
+            const int u = (reg || fin) ? e - s + 1 : 0;
+            nreg += reg ? 1 : 0;
+            A2 += u;
+            A3 += (long long)u * dd.z + (((long long)s + e) * u >> 1);
+            CB += reg ? dd.z : 0;
+            return !(reg || fin);
+        };
+        const unsigned lt = lanemask_lt();
         int nwin = 0;
-        for (int base = 0; base < nl; base += 32) {
-            const int i = base + lane;
-            bool win = false;
-            if (i < nl) {
-                const int4 dd = m.dl[i];
-                const int s = dd.x;
-                // u tokens at contexts cb + s .. cb + e: u cb + (s + e) u / 2, where
-                // (s + e) u is twice a sum of consecutive integers, so the halving is exact
-                if (s <= lk0 && dd.y >= Lend) {
-                    const int u = L0 - s + 1;
-                    ++nreg;
-                    A2 += u;
-                    A3 += (long long)u * dd.z + (((long long)s + L0) * u >> 1);
-                    CB += dd.z;
-                } else if (dd.y < lk0) {
-                    // finished before the window: all of its tokens, in every row
-                    const int u = dd.y - s + 1;
-                    A2 += u;
-                    A3 += (long long)u * dd.z + (((long long)s + dd.y) * u >> 1);
-                } else {
-                    win = true;
+        for (int base = 0; base < nl; base += 64) {
+            const int i0 = base + lane, i1 = i0 + 32;
+            const int4 d0 = m.dl[min(i0, nl - 1)], d1 = m.dl[min(i1, nl - 1)];
+            const bool w0 = i0 < nl && classify(d0);
+            const bool w1 = i1 < nl && classify(d1);
+            const unsigned b0 = __ballot_sync(kFull, w0), b1 = __ballot_sync(kFull, w1);
+            const int s0 = nwin + __popc(b0 & lt), s1 = nwin + __popc(b0) + __popc(b1 & lt);
+            if (w0 && s0 < kWinList) wlist[s0] = i0;
+            if (w1 && s1 < kWinList) wlist[s1] = i1;
+            nwin += __popc(b0) + __popc(b1);
+        }
+        if (nwin > kWinList) {
+            // the list is full: the window decoders beyond it take the per-row path here
+            // (the same compaction finds them again, without accumulating anything)
+            int seen = 0;
+            for (int base = 0; base < nl; base += 32) {
+                const int i = base + lane;
+                bool win = false;
+                if (i < nl) {
+                    const int4 dd = m.dl[i];
+                    win = !(dd.x <= lk0 && dd.y >= Lend) && !(dd.y < lk0);
                 }
+                const unsigned bal = __ballot_sync(kFull, win);
+                if (win && seen + __popc(bal & lt) >= kWinList) rows(m.dl[i]);
+                seen += __popc(bal);
             }
-            const unsigned bal = __ballot_sync(kFull, win);
-            if (win) {
-                const int slot = nwin + __popc(bal & lanemask_lt());
-                if (slot < kWinList) wlist[slot] = i;
-                else rows(m.dl[i]);  // list full: on the spot
-            }
-            nwin += __popc(bal);
         }
         __syncwarp();
         for (int t = lane; t < min(nwin, kWinList); t += 32) rows(m.dl[wlist[t]]);

@@ -115,6 +115,29 @@ def test_instance_tiles_beyond_one_cta():
     check_candidates(wl, F.reshape(-1, 5), t.ravel(), fb.ravel(), qq.ravel(), jj.ravel())
 
 
+@pytest.mark.parametrize("mode", [0, 1])
+def test_window_list_overflow(mode):
+    # 450 running decoders that all end within the first table rows' batches: more
+    # window decoders than the trajectory kernel's compacted list holds
+    wl = W.small_workload(11, num_instances=5, num_models=2, num_queries=31, cap_running=512, cap_waiting=32,
+                          first_token_mode=mode, budget_range=(2048, 4096), min_gap=1024)
+    rng = np.random.default_rng(5)
+    I = wl.num_instances
+    n_run = np.full(I, 450, np.int32)
+    run_ctx = np.zeros((I, 512), np.int32)
+    run_dec = np.zeros((I, 512), np.int32)
+    run_ctx[:, :450] = rng.integers(1, 400, (I, 450))
+    run_dec[:, :450] = rng.integers(1, 12, (I, 450))
+    S = np.maximum(wl.max_seqs, 480).astype(np.int32)
+    wl = dataclasses.replace(wl, n_run=n_run, run_ctx=run_ctx, run_pre=np.zeros((I, 512), np.int32),
+                             run_dec=run_dec, max_seqs=np.minimum(S, wl.max_batched_tokens).astype(np.int32))
+    rt = make_router(wl)
+    F, t, fb = full_estimate(rt, wl)
+    qq, jj = np.meshgrid(np.arange(wl.num_queries), np.arange(I), indexing="ij")
+    check_candidates(wl, F.reshape(-1, 5), t.ravel(), fb.ravel(), qq.ravel(), jj.ravel())
+    rt.close()
+
+
 def test_two_instance_tiles():
     # 1100 instances: two instance tiles, whose CTAs claim every query row dynamically
     wl = W.small_workload(7, num_instances=1100, num_models=4, num_queries=53, budget_range=(64, 160), min_gap=64)
