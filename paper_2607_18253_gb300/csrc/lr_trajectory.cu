@@ -210,6 +210,30 @@ __device__ __forceinline__ bool decoder_of(int e, int ce, int d, int *f, int *cb
 template <int MODE>
 __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j, int lane, int32_t *wbase) {
     const DevConfig &c = a.cfg;
+    const size_t rrow = (size_t)j * c.capR;
+    const size_t wrow = (size_t)j * c.capW;
+    const int32_t *__restrict__ ic = a.in.run_ctx + rrow;
+    const int32_t *__restrict__ ip = a.in.run_pre + rrow;
+    const int32_t *__restrict__ id = a.in.run_dec + rrow;
+    const int32_t *__restrict__ iwp = a.in.wait_pre + wrow;
+    const int32_t *__restrict__ iwd = a.in.wait_dec + wrow;
+    // The snapshot rows are read in blocks of 256 entries, all loads of a block issued
+    // before any of them is used; the first block's loads go out before anything
+    // waits on the counts, so that one memory round trip covers both.
+    constexpr int kBlk = 8;  // entries per lane and block
+    int xc[kBlk], xp[kBlk], xd[kBlk], yp[kBlk], yd[kBlk];
+    auto load_block = [&](int base) {
+#pragma unroll
+        for (int k = 0; k < kBlk; ++k) {
+            const int t = base + lane + 32 * k;
+            xc[k] = t < c.capR ? __ldg(ic + t) : 0;
+            xp[k] = t < c.capR ? __ldg(ip + t) : 0;
+            xd[k] = t < c.capR ? __ldg(id + t) : 0;
+            yp[k] = t < c.capW ? __ldg(iwp + t) : 0;
+            yd[k] = t < c.capW ? __ldg(iwd + t) : 0;
+        }
+    };
+    load_block(0);
     const int B = c.B[j];
     const int S = c.S[j];
     const int nr = a.in.n_run[j];
@@ -219,41 +243,37 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         out.n_wait[j] = nw;
         out.clock[j] = a.in.clock ? a.in.clock[j] : 0.0;
     }
+    WarpSmem m = carve(wbase, c);
+    // Clear the calendar.
+    for (int i = lane; i < kCalendar / 4; i += 32) reinterpret_cast<int4 *>(m.cal)[i] = make_int4(0, 0, 0, 0);
+    for (int i = lane; i < kCalendar / 32; i += 32) m.bm[i] = 0u;
     if (!(nr >= 0 && nr <= c.capR && nr <= S && nw >= 0 && nw <= c.capW)) {
         fail(a.ctl, kEState, lane);
         return;
     }
-    WarpSmem m = carve(wbase, c);
-    const size_t rrow = (size_t)j * c.capR;
-    const size_t wrow = (size_t)j * c.capW;
-
-    // Clear the calendar.
-    for (int i = lane; i < kCalendar / 4; i += 32) reinterpret_cast<int4 *>(m.cal)[i] = make_int4(0, 0, 0, 0);
-    for (int i = lane; i < kCalendar / 32; i += 32) m.bm[i] = 0u;
     __syncwarp();
 
     // Copy the snapshot into library memory, validate it, total the prefill work
-    // and list the running decoders (decoding from batch 1).  Loads and stores
-    // go through non-aliasing row pointers so that loads of later elements can
-    // be issued ahead of earlier stores.
+    // and list the running decoders (decoding from batch 1).
     bool bad = false;
     long long f1 = 0, f4 = 0, wsum = 0;
     int pf_pre = 0, pf_ctx = 0, pf_dec = 0;
-    {
-        const int32_t *__restrict__ ic = a.in.run_ctx + rrow;
-        const int32_t *__restrict__ ip = a.in.run_pre + rrow;
-        const int32_t *__restrict__ id = a.in.run_dec + rrow;
-        int32_t *__restrict__ oc = out.run_ctx + rrow;
-        int32_t *__restrict__ op = out.run_pre + rrow;
-        int32_t *__restrict__ od = out.run_dec + rrow;
-#pragma unroll 4
-        for (int t = lane; t < c.capR; t += 32) {
-            const int ctx = __ldg(ic + t);
-            const int pre = __ldg(ip + t);
-            const int dec = __ldg(id + t);
-            oc[t] = ctx;
-            op[t] = pre;
-            od[t] = dec;
+    int32_t *__restrict__ oc = out.run_ctx + rrow;
+    int32_t *__restrict__ op = out.run_pre + rrow;
+    int32_t *__restrict__ od = out.run_dec + rrow;
+    int32_t *__restrict__ owp = out.wait_pre + wrow;
+    int32_t *__restrict__ owd = out.wait_dec + wrow;
+    for (int base = 0; base < max(c.capR, c.capW); base += 32 * kBlk) {
+        if (base > 0) load_block(base);
+#pragma unroll
+        for (int k = 0; k < kBlk; ++k) {
+            const int t = base + lane + 32 * k;
+            const int ctx = xc[k], pre = xp[k], dec = xd[k];
+            if (t < c.capR) {
+                oc[t] = ctx;
+                op[t] = pre;
+                od[t] = dec;
+            }
             if (t < nr) {
                 bad |= ctx < 0 || ctx > (1 << 28) || pre < 0 || pre > (1 << 24) || dec < 1 || dec > (1 << 24);
                 bad |= pre > 0 && t != nr - 1;
@@ -273,14 +293,11 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
                 }
             }
         }
-        const int32_t *__restrict__ iwp = a.in.wait_pre + wrow;
-        const int32_t *__restrict__ iwd = a.in.wait_dec + wrow;
-        int32_t *__restrict__ owp = out.wait_pre + wrow;
-        int32_t *__restrict__ owd = out.wait_dec + wrow;
-#pragma unroll 4
-        for (int t = lane; t < c.capW; t += 32) {
-            const int pre = __ldg(iwp + t);
-            const int dec = __ldg(iwd + t);
+#pragma unroll
+        for (int k = 0; k < kBlk; ++k) {
+            const int t = base + lane + 32 * k;
+            if (t >= c.capW) continue;
+            const int pre = yp[k], dec = yd[k];
             owp[t] = pre;
             owd[t] = dec;
             m.wdec[t] = dec;
@@ -295,24 +312,28 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         }
     }
     __syncwarp();
-    // exclusive prefix sums of the prompts, in place (valid while the total stays below 2^30)
+    // exclusive prefix sums of the prompts, in place (valid while the total stays below
+    // 2^30): each lane sums the consecutive entries it owns, the lane totals are scanned
+    // once, and each lane then writes its entries' sums
     {
-        int carry = 0;
-        for (int base = 0; base < c.capW; base += 32) {
-            const int t = base + lane;
-            const int incl = carry + warp_incl_sum(t < c.capW ? m.P[t + 1] : 0, lane);
-            if (t < c.capW) m.P[t + 1] = incl;
-            carry = __shfl_sync(kFull, incl, 31);
+        const int seg = (c.capW + 31) >> 5;
+        const int t0 = lane * seg, t1 = min(t0 + seg, c.capW);
+        int own = 0;
+        for (int t = t0; t < t1; ++t) own += m.P[t + 1];
+        int run = warp_incl_sum(own, lane) - own;
+        for (int t = t0; t < t1; ++t) {
+            run += m.P[t + 1];
+            m.P[t + 1] = run;
         }
         if (lane == 0) m.P[0] = 0;
     }
     wsum = warp_sum64(wsum);
+    f1 = warp_sum64(f1);
+    f4 = warp_sum64(f4);
     if (__any_sync(kFull, bad) || wsum > (1LL << 30)) {
         fail(a.ctl, kEState, lane);
         return;
     }
-    f1 = warp_sum64(f1);
-    f4 = warp_sum64(f4);
     __syncwarp();
 
     // the request still in prefill, if any, is the last running one
@@ -478,13 +499,14 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             while (budget > 0 && head < lim) {
                 const int r = head + lane;
                 const int pe = r < lim ? lds(sP + 4u * (r + 1)) : 0;  // prompt sum through request r
+                const int dr = r < lim ? lds(sW + 4u * r) : 0;        // and its decode length
                 const bool whole = r < lim && pe - ph <= budget;
                 const int k = __popc(__ballot_sync(kFull, whole));
                 if (k > 0) {
                     int before = __shfl_up_sync(kFull, pe, 1);
                     if (lane == 0) before = ph;
                     int f = kBig, cb = 0;
-                    const bool dec = whole && decoder_of<MODE>(l, pe - before, lds(sW + 4u * r), &f, &cb);
+                    const bool dec = whole && decoder_of<MODE>(l, pe - before, dr, &f, &cb);
                     const unsigned dm = __ballot_sync(kFull, dec);
                     unsigned wlo = 0u, whi = 0u;
                     if (dec) {
