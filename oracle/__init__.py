@@ -75,6 +75,12 @@ def _load():
         lib.orc_throughput_wait.restype = ctypes.c_double
         lib.orc_avgcase_ttft.argtypes = [i32, i32, P, P, P, P, P, P]
         lib.orc_avgcase_ttft.restype = ctypes.c_int
+        lib.orc_round_robin.argtypes = [i32, i32, i64, P]
+        lib.orc_round_robin.restype = ctypes.c_int
+        lib.orc_shortest_queue.argtypes = [i32, i32, P, P]
+        lib.orc_shortest_queue.restype = ctypes.c_int
+        lib.orc_on_time_utility.argtypes = [i32, P, P, P, P, P]
+        lib.orc_on_time_utility.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -285,3 +291,74 @@ def calibrate(features, model, time, num_models: int, shared_beta1: bool = True)
             continue
         out[m] = [beta[0], beta[1], beta[1], beta[2], beta[3]] if shared_beta1 else beta
     return out
+
+
+# ---- Baseline routing policies and stream metrics (Sec. 6 baselines; Eq. 4) ----
+
+POLICY_ROUND_ROBIN, POLICY_SHORTEST_QUEUE, POLICY_LATENCY_AGNOSTIC = 0, 1, 2
+
+
+def round_robin(Q: int, I: int, start: int = 0) -> np.ndarray:
+    """Round Robin: query q to instance (start + q) mod I."""
+    a = np.zeros(Q, np.int32)
+    if _load().orc_round_robin(Q, I, int(start), _p(a)) != 0:
+        raise RuntimeError("oracle round robin failed")
+    return a
+
+
+def shortest_queue(counts, Q: int) -> np.ndarray:
+    """Shortest Queue: each query in turn to the instance with the fewest resident
+    requests, the queries routed before it included (ties to the lowest index)."""
+    c = _c(counts, np.int32)
+    a = np.zeros(Q, np.int32)
+    if _load().orc_shortest_queue(Q, c.shape[0], _p(c), _p(a)) != 0:
+        raise RuntimeError("oracle shortest queue failed")
+    return a
+
+
+def baseline_route(wl, policy: int, lam: float, rr_start: int = 0, ttft32: Optional[np.ndarray] = None):
+    """A baseline policy's assignment, the chosen instance's utility (Eq. 2) and its
+    canonical fp32 SFS TTFT: assign/util/ttft [Q].  Latency-Agnostic is the argmax of
+    U over the instances (ties to the lowest index); rows whose prompt is out of range
+    get -1 / NaN / NaN."""
+    Q, I = wl.num_queries, wl.num_instances
+    lam32 = np.float32(lam)
+    if policy == POLICY_ROUND_ROBIN:
+        assign = round_robin(Q, I, rr_start)
+    elif policy == POLICY_SHORTEST_QUEUE:
+        assign = shortest_queue(np.asarray(wl.n_run) + np.asarray(wl.n_wait), Q)
+    elif policy == POLICY_LATENCY_AGNOSTIC:
+        assign = np.zeros(Q, np.int32)
+        for i in range(Q):
+            us = [utility(wl.acc[i, wl.model_of_instance[j]], lam32, wl.prompt_len[i],
+                          wl.dec_hat[i, wl.model_of_instance[j]], wl.price_in[wl.model_of_instance[j]],
+                          wl.price_out[wl.model_of_instance[j]]) for j in range(I)]
+            assign[i] = int(np.argmax(np.asarray(us, np.float32)))  # first maximum
+    else:
+        raise ValueError(policy)
+    valid = (np.asarray(wl.prompt_len) >= 1) & (np.asarray(wl.prompt_len) <= wl.max_prompt_len)
+    util = np.full(Q, np.nan, np.float32)
+    ttft = np.full(Q, np.nan, np.float32)
+    qs = np.nonzero(valid)[0]
+    if qs.size:
+        if ttft32 is None:
+            _, _, t32, _ = estimate_candidates(wl, qs, assign[qs])
+        else:
+            t32 = np.asarray(ttft32, np.float32)[qs, assign[qs]]
+        ttft[qs] = t32
+        for i in qs:
+            m = wl.model_of_instance[assign[i]]
+            util[i] = utility(wl.acc[i, m], lam32, wl.prompt_len[i], wl.dec_hat[i, m], wl.price_in[m],
+                              wl.price_out[m])
+    assign = np.where(valid, assign, -1).astype(np.int32)
+    return assign, util, ttft
+
+
+def on_time_utility(util, ttft, tau, delay=None):
+    """(OnTimeUtility of Eq. 4, SLO attainment): realized TTFT = fp32 delay + ttft."""
+    u, t, ta = (_c(x, np.float32) for x in (util, ttft, tau))
+    d = None if delay is None else _c(delay, np.float32)
+    out = np.zeros(2, np.float64)
+    if _load().orc_on_time_utility(u.shape[0], _p(u), _p(t), _p(ta), _p(d), _p(out)) != 0:
+        raise RuntimeError("oracle on-time utility failed")
+    return float(out[0]), float(out[1])

@@ -460,3 +460,46 @@ int orc_avgcase_ttft(int32_t I, int32_t Q, const double *W, const double *theta,
     }
     return ORC_OK;
 }
+
+/* ---- Baseline routing policies and stream metrics (Sec. 6 baselines; Eq. 4) ---- */
+
+int orc_round_robin(int32_t Q, int32_t I, int64_t start, int32_t *assign)
+{
+    if (Q < 0 || I < 1 || start < 0) return ORC_EINVAL;
+    for (int32_t q = 0; q < Q; ++q) assign[q] = (int32_t)((start + q) % I);
+    return ORC_OK;
+}
+
+int orc_shortest_queue(int32_t Q, int32_t I, const int32_t *counts, int32_t *assign)
+{
+    if (Q < 0 || I < 1) return ORC_EINVAL;
+    int64_t *n = (int64_t *)malloc(sizeof(int64_t) * (size_t)I);
+    if (!n) return ORC_EINVAL;
+    for (int32_t j = 0; j < I; ++j) n[j] = counts[j];
+    for (int32_t q = 0; q < Q; ++q) {
+        int32_t best = 0;
+        for (int32_t j = 1; j < I; ++j)
+            if (n[j] < n[best]) best = j;
+        assign[q] = best;
+        n[best] += 1;  /* the routed query joins that queue */
+    }
+    free(n);
+    return ORC_OK;
+}
+
+int orc_on_time_utility(int32_t Q, const float *util, const float *ttft, const float *tau,
+                        const float *delay, double *out)
+{
+    if (Q < 1) return ORC_EINVAL;
+    double su = 0.0, sn = 0.0;
+    for (int32_t i = 0; i < Q; ++i) {
+        const float realized = delay ? delay[i] + ttft[i] : ttft[i];
+        if (realized <= tau[i]) {  /* false for NaN */
+            su += (double)util[i];
+            sn += 1.0;
+        }
+    }
+    out[0] = su / Q;
+    out[1] = sn / Q;
+    return ORC_OK;
+}

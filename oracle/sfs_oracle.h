@@ -109,6 +109,24 @@ double orc_throughput_wait(const orc_instance *inst, double theta);
 int orc_avgcase_ttft(int32_t I, int32_t Q, const double *W, const double *theta, const double *tdec,
                      const int32_t *prompt_len, float *t32, double *t64);
 
+/* ---- Baseline routing policies and stream metrics (Sec. 6 baselines; Eq. 4) ---- */
+
+/* Round Robin: query q goes to instance (start + q) mod I, whatever the load,
+ * utility or latency. */
+int orc_round_robin(int32_t Q, int32_t I, int64_t start, int32_t *assign);
+
+/* Shortest Queue: the queries in order each go to the instance with the fewest
+ * resident requests, counting the queries routed before them (ties to the lowest
+ * index).  counts[I] are the resident requests (running + waiting) at the start. */
+int orc_shortest_queue(int32_t Q, int32_t I, const int32_t *counts, int32_t *assign);
+
+/* OnTimeUtility (Eq. 4) and SLO attainment over Q routed queries.  The realized TTFT
+ * of query i is the fp32 sum delay_i + ttft_i (delay NULL: 0); it is on time if that
+ * is <= tau_i (NaN never is).  out[0] = (1/Q) sum of util_i over on-time queries,
+ * out[1] = (on-time count) / Q; fp64 sums in index order. */
+int orc_on_time_utility(int32_t Q, const float *util, const float *ttft, const float *tau,
+                        const float *delay, double *out);
+
 #ifdef __cplusplus
 }
 #endif
