@@ -273,6 +273,43 @@ LR_API const char *lr_strerror(int code);
  * validation that failed); empty if none.  Valid until the next call on ctx. */
 LR_API const char *lr_last_error(const lr_ctx *ctx);
 
+/* ---- Baseline routing policies and stream metrics (Sec. 6 "Baselines"; Eq. 4) ---- */
+
+enum lr_policy {
+    LR_POLICY_ROUND_ROBIN = 0,      /* query i -> instance (rr_start + i) mod I */
+    LR_POLICY_SHORTEST_QUEUE = 1,   /* fewest resident requests (running + waiting) */
+    LR_POLICY_LATENCY_AGNOSTIC = 2  /* largest utility U (Eq. 2), latency ignored */
+};
+
+/* The paper's baseline routers (Sec. 6 "Baselines"), for comparison with lr_route.
+ * Round Robin assigns cyclically; Shortest Queue lets the Q queries, in order, each
+ * join the instance with the fewest resident requests of the live snapshot, counting
+ * the queries routed before it in this call (ties: lowest index); Latency-Agnostic
+ * picks the largest utility (ties: lowest index), i.e. Eq. 5 with mu = 0.  For each
+ * query the chosen instance, its utility U (Eq. 2, cost as in lr_route, one lambda)
+ * and its SFS TTFT estimate (the value lr_estimate_ttft gives for that candidate,
+ * whatever TTFT source is selected) are written.
+ * prompt_len [Q], dec_hat [Q][M], acc [Q][M]: device, as in lr_route.  lambda: host
+ * value, finite and >= 0.  rr_start >= 0: Round Robin's first index.
+ * assign_out [Q] int32, util_out [Q] fp32, ttft_chosen_out [Q] fp32 or NULL: device.
+ * Needs a live snapshot (else the rows are -1 / NaN and the status word records
+ * LR_ENOSTATE); a prompt out of range gives that row -1 / NaN (LR_EINVAL recorded).
+ * LR_ECAPACITY if the per-CTA sort of the instances' queue counts does not fit in
+ * shared memory (about 10,000 instances or more). */
+LR_API int lr_route_baseline(lr_ctx *ctx, int32_t policy, int32_t Q, const int32_t *prompt_len,
+                             const int32_t *dec_hat, const float *acc, float lambda, int64_t rr_start,
+                             int32_t *assign_out, float *util_out, float *ttft_chosen_out, void *cuda_stream);
+
+/* OnTimeUtility (Eq. 4) and SLO attainment over Q >= 1 routed queries.  The
+ * realized TTFT of query i is the fp32 sum delay[i] + ttft[i] (delay NULL: 0), e.g.
+ * the time the query waited for its routing decision plus the chosen instance's
+ * TTFT; it is on time if it is <= tau[i] (NaN never is).
+ * out[0] = (1/Q) * sum of util[i] over on-time queries, out[1] = on-time count / Q.
+ * util, ttft, tau, delay: [Q] device fp32; out: [2] device fp64.  The sums are fp64
+ * in a fixed order (the same result on every run). */
+LR_API int lr_on_time_utility(lr_ctx *ctx, int32_t Q, const float *util, const float *ttft, const float *tau,
+                              const float *delay, double *out, void *cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

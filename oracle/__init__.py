@@ -79,6 +79,8 @@ def _load():
         lib.orc_round_robin.restype = ctypes.c_int
         lib.orc_shortest_queue.argtypes = [i32, i32, P, P]
         lib.orc_shortest_queue.restype = ctypes.c_int
+        lib.orc_latency_agnostic.argtypes = [i32, i32, i32, P, P, P, P, P, P, ctypes.c_float, P]
+        lib.orc_latency_agnostic.restype = ctypes.c_int
         lib.orc_on_time_utility.argtypes = [i32, P, P, P, P, P]
         lib.orc_on_time_utility.restype = ctypes.c_int
         _lib = lib
@@ -329,11 +331,11 @@ def baseline_route(wl, policy: int, lam: float, rr_start: int = 0, ttft32: Optio
         assign = shortest_queue(np.asarray(wl.n_run) + np.asarray(wl.n_wait), Q)
     elif policy == POLICY_LATENCY_AGNOSTIC:
         assign = np.zeros(Q, np.int32)
-        for i in range(Q):
-            us = [utility(wl.acc[i, wl.model_of_instance[j]], lam32, wl.prompt_len[i],
-                          wl.dec_hat[i, wl.model_of_instance[j]], wl.price_in[wl.model_of_instance[j]],
-                          wl.price_out[wl.model_of_instance[j]]) for j in range(I)]
-            assign[i] = int(np.argmax(np.asarray(us, np.float32)))  # first maximum
+        moi, p, dh = (_c(a, np.int32) for a in (wl.model_of_instance, wl.prompt_len, wl.dec_hat))
+        acc, pin, pout = (_c(a, np.float32) for a in (wl.acc, wl.price_in, wl.price_out))
+        if _load().orc_latency_agnostic(Q, I, wl.num_models, _p(moi), _p(pin), _p(pout), _p(p), _p(dh), _p(acc),
+                                        float(lam32), _p(assign)) != 0:
+            raise RuntimeError("oracle latency-agnostic failed")
     else:
         raise ValueError(policy)
     valid = (np.asarray(wl.prompt_len) >= 1) & (np.asarray(wl.prompt_len) <= wl.max_prompt_len)

@@ -487,6 +487,25 @@ int orc_shortest_queue(int32_t Q, int32_t I, const int32_t *counts, int32_t *ass
     return ORC_OK;
 }
 
+int orc_latency_agnostic(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instance,
+                         const float *price_in, const float *price_out, const int32_t *prompt_len,
+                         const int32_t *dec_hat, const float *acc, float lambda, int32_t *assign)
+{
+    if (Q < 0 || I < 1 || M < 1) return ORC_EINVAL;
+    for (int32_t i = 0; i < Q; ++i) {
+        int32_t best_j = 0;
+        float best = 0.0f;
+        for (int32_t j = 0; j < I; ++j) {
+            const int32_t m = model_of_instance[j];
+            const float u = orc_utility(acc[(int64_t)i * M + m], lambda, prompt_len[i],
+                                        dec_hat[(int64_t)i * M + m], price_in[m], price_out[m]);
+            if (j == 0 || u > best) { best = u; best_j = j; }
+        }
+        assign[i] = best_j;
+    }
+    return ORC_OK;
+}
+
 int orc_on_time_utility(int32_t Q, const float *util, const float *ttft, const float *tau,
                         const float *delay, double *out)
 {

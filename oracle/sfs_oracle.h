@@ -120,6 +120,12 @@ int orc_round_robin(int32_t Q, int32_t I, int64_t start, int32_t *assign);
  * index).  counts[I] are the resident requests (running + waiting) at the start. */
 int orc_shortest_queue(int32_t Q, int32_t I, const int32_t *counts, int32_t *assign);
 
+/* Latency-Agnostic: argmax over instances of the utility of Eq. 2 (ties to the lowest
+ * index), i.e. Eq. 5 with mu = 0. */
+int orc_latency_agnostic(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instance,
+                         const float *price_in, const float *price_out, const int32_t *prompt_len,
+                         const int32_t *dec_hat, const float *acc, float lambda, int32_t *assign);
+
 /* OnTimeUtility (Eq. 4) and SLO attainment over Q routed queries.  The realized TTFT
  * of query i is the fp32 sum delay_i + ttft_i (delay NULL: 0); it is on time if that
  * is <= tau_i (NaN never is).  out[0] = (1/Q) sum of util_i over on-time queries,

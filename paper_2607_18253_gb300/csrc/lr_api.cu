@@ -23,6 +23,8 @@ struct lr_ctx {
     size_t k3_smem = 0;
     float *scratch_tch = nullptr;
     uint32_t *k2_work = nullptr;  // the candidate kernel's row counters
+    double *ontime_part = nullptr;  // per-CTA partial sums of lr_on_time_utility
+    bool bl_ok = false;             // the baseline policies' shared memory fits
     // average-case TTFT sources
     lr::QueueRaw *qraw = nullptr;
     lr::QueueDev *qd = nullptr;
@@ -264,6 +266,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     LR_ALLOC(c->ctl, 1);
     LR_ALLOC(c->scratch_tch, (size_t)cfg->max_pairs * cfg->max_queries);
     LR_ALLOC(c->k2_work, lr::k2_work_words(I));
+    LR_ALLOC(c->ontime_part, 2 * (size_t)lr::kOnTimeParts);
     LR_ALLOC(c->qraw, I);
     LR_ALLOC(c->qd, I);
     LR_ALLOC(c->cal_acc, (size_t)M * lr::kCalAcc * 2);
@@ -306,6 +309,8 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     if (e == cudaSuccess && c->k3_smem <= 200 * 1024) e = lr::set_k3_smem(c->k3_smem);
     if (e == cudaSuccess && M <= lr::kCalMaxModels) e = lr::set_calib_smem(M);
     if (e == cudaSuccess) e = lr::set_k2_smem(std::max(c->est.smem, c->rt.ok ? c->rt.smem : 0));
+    c->bl_ok = lr::baseline_smem(d) <= 200 * 1024;
+    if (e == cudaSuccess && c->bl_ok) e = lr::set_baseline_smem(lr::baseline_smem(d));
     if (e == cudaSuccess) e = lr::cand_occupancy(d.mode, false, lr::kK2Block, c->est.smem, &c->est.occ);
     if (e == cudaSuccess && c->rt.ok) e = lr::cand_occupancy(d.mode, true, lr::kK2Block, c->rt.smem, &c->rt.occ);
     if (e != cudaSuccess) return bail(LR_ECUDA, cudaGetErrorString(e));
@@ -430,6 +435,42 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
         if (e != cudaSuccess) return cuda_fail(c, e, "frontier launch");
     }
     return LR_OK;
+}
+
+int lr_route_baseline(lr_ctx *c, int32_t policy, int32_t Q, const int32_t *prompt_len, const int32_t *dec_hat,
+                      const float *acc, float lambda, int64_t rr_start, int32_t *assign_out, float *util_out,
+                      float *ttft_chosen_out, void *stream) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    if (policy < LR_POLICY_ROUND_ROBIN || policy > LR_POLICY_LATENCY_AGNOSTIC) return fail(c, LR_EINVAL, "policy");
+    if (Q < 0) return fail(c, LR_EINVAL, "Q < 0");
+    if (Q > c->max_queries) return fail(c, LR_ECAPACITY, "Q exceeds max_queries");
+    if (!finite_nonneg(lambda)) return fail(c, LR_EINVAL, "lambda must be finite and >= 0");
+    if (rr_start < 0) return fail(c, LR_EINVAL, "rr_start < 0");
+    if (!c->bl_ok) return fail(c, LR_ECAPACITY, "num_instances too large for the baseline policies");
+    if (Q == 0) return LR_OK;
+    if (!prompt_len || !dec_hat || !acc || !assign_out || !util_out) return fail(c, LR_EINVAL, "null array");
+    lr::K2Launch a = k2_base(c);
+    a.Q = Q;
+    a.prompt = prompt_len;
+    a.dec_hat = dec_hat;
+    a.acc = acc;
+    a.assign = assign_out;
+    a.util = util_out;
+    a.ttft_chosen = ttft_chosen_out;
+    const cudaError_t e = lr::launch_baseline(a, policy, (long long)rr_start, lambda, c->sms, (cudaStream_t)stream);
+    return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "baseline launch");
+}
+
+int lr_on_time_utility(lr_ctx *c, int32_t Q, const float *util, const float *ttft, const float *tau,
+                       const float *delay, double *out, void *stream) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    if (Q < 1) return fail(c, LR_EINVAL, "Q < 1");
+    if (!util || !ttft || !tau || !out) return fail(c, LR_EINVAL, "null array");
+    const cudaError_t e = lr::launch_on_time(Q, util, ttft, tau, delay, c->ontime_part, lr::kOnTimeParts, out,
+                                             (cudaStream_t)stream);
+    return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "on-time utility launch");
 }
 
 // Chosen-TTFT intermediate of lr_route_frontier_static: [P][Q] fp32 in static

@@ -743,6 +743,181 @@ __global__ void k_queue_params(int I, const QueueRaw *raw, QueueDev *qd) {
     qd[j] = o;
 }
 
+// ---------------------------------------------------------------------------
+// Baseline routing policies (Sec. 6 "Baselines"): the instance is chosen without the
+// latency estimates, and the chosen candidate's utility (Eq. 2) and SFS TTFT estimate
+// are reported beside it (the TTFT through the same exact path as the candidate
+// kernel's, so the two agree bit for bit).  One thread per query.
+//   Round Robin: (start + i) mod I.
+//   Shortest Queue: the queries in order each join the instance with the fewest
+//     resident requests, counting those routed before them, ties to the lowest index.
+//     Query k therefore takes the k-th smallest slot (level, j) over the slots
+//     instance j offers at levels c_j, c_j + 1, ...: the level L is the largest with
+//     N(L) = sum_j max(0, L - c_j) <= k (N from the sorted counts and their prefix
+//     sums), and the instance is the (k - N(L))-th, by index, of those with c_j <= L.
+//   Latency-Agnostic: the largest utility, ties to the lowest index (utility depends
+//     on the instance's model only, so the models are compared at their first instance).
+template <int MODE>
+__global__ void __launch_bounds__(256) k_baseline(const K2Launch a, int policy, long long rr_start, float lam) {
+    extern __shared__ __align__(16) unsigned char bsm[];
+    const DevConfig &c = a.cfg;
+    const int I = c.I, M = c.M;
+    __shared__ int s_active;
+    if (threadIdx.x == 0) s_active = load_acquire(&a.ctl->active);
+    __syncthreads();
+    const int active = s_active;
+    const StateBuf sb = active > 0 ? a.buf1 : a.buf0;
+    int P2 = 1;
+    while (P2 < I) P2 <<= 1;
+    int *cnt = reinterpret_cast<int *>(bsm);                              // [I] resident requests
+    int *srt = cnt + I;                                                   // [P2] the counts, sorted
+    long long *pre = reinterpret_cast<long long *>(bsm + 8 * ((I + P2 + 1) / 2));  // [I + 1] prefix sums
+    int *firstj = reinterpret_cast<int *>(pre + I + 1);                   // [M] first instance of each model
+    if (active >= 0 && policy == 1) {
+        for (int j = threadIdx.x; j < P2; j += blockDim.x) {
+            const int v = j < I ? sb.n_run[j] + sb.n_wait[j] : 0x7fffffff;
+            if (j < I) cnt[j] = v;
+            srt[j] = v;
+        }
+        __syncthreads();
+        // bitonic sort of srt, ascending
+        for (int k = 2; k <= P2; k <<= 1) {
+            for (int h = k >> 1; h > 0; h >>= 1) {
+                for (int t = threadIdx.x; t < P2; t += blockDim.x) {
+                    const int u = t ^ h;
+                    if (u > t) {
+                        const int x = srt[t], y = srt[u];
+                        if (((t & k) == 0) == (x > y)) {
+                            srt[t] = y;
+                            srt[u] = x;
+                        }
+                    }
+                }
+                __syncthreads();
+            }
+        }
+        if (threadIdx.x == 0) {
+            long long run = 0;
+            for (int t = 0; t < I; ++t) {
+                pre[t] = run;
+                run += srt[t];
+            }
+            pre[I] = run;
+        }
+    }
+    if (policy == 2) {
+        for (int m = threadIdx.x; m < M; m += blockDim.x) firstj[m] = -1;
+        __syncthreads();
+        for (int j = threadIdx.x; j < I; j += blockDim.x) atomicMin(reinterpret_cast<unsigned *>(firstj) + c.moi[j], (unsigned)j);
+    }
+    __syncthreads();
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < a.Q; i += gridDim.x * blockDim.x) {
+        const int p = a.prompt[i];
+        bool ok;
+        const QRec q = make_qrec(p, c.pmax, &ok);
+        if (!ok || active < 0) {
+            record_status(a.ctl, active < 0 ? kENoState : kEInval);
+            a.assign[i] = -1;
+            a.util[i] = kNaN;
+            if (a.ttft_chosen) a.ttft_chosen[i] = kNaN;
+            continue;
+        }
+        int j = 0;
+        if (policy == 0) {
+            j = (int)((rr_start + i) % I);
+        } else if (policy == 1) {
+            // N(L): slots below level L = (#counts below L) * L - (their sum)
+            auto slots_below = [&](long long L) -> long long {
+                int lo = 0, hi = I;  // first sorted count >= L
+                while (lo < hi) {
+                    const int mid = (lo + hi) >> 1;
+                    if ((long long)srt[mid] < L) lo = mid + 1;
+                    else hi = mid;
+                }
+                return (long long)lo * L - pre[lo];
+            };
+            long long lo = srt[0], hi = (long long)srt[0] + i + 1;  // N(lo) <= i < N(hi)
+            while (hi - lo > 1) {
+                const long long mid = (lo + hi) >> 1;
+                if (slots_below(mid) <= i) lo = mid;
+                else hi = mid;
+            }
+            long long r = i - slots_below(lo);  // < #{j : c_j <= lo}, so the scan finds it
+            for (j = 0; j < I; ++j)
+                if ((long long)cnt[j] <= lo && r-- == 0) break;
+            j = min(j, I - 1);
+        } else {
+            float best = 0.f;
+            int bj = -1;
+            for (int m = 0; m < M; ++m) {
+                const int fj = firstj[m];
+                if (fj < 0) continue;
+                const float cost = __fmaf_rn((float)a.dec_hat[(size_t)i * M + m], c.pout[m], __fmul_rn((float)p, c.pin[m]));
+                const float U = __fmaf_rn(-lam, cost, a.acc[(size_t)i * M + m]);
+                if (bj < 0 || U > best || (U == best && fj < bj)) {
+                    best = U;
+                    bj = fj;
+                }
+            }
+            j = bj;
+        }
+        const int m = c.moi[j];
+        const float cost = __fmaf_rn((float)a.dec_hat[(size_t)i * M + m], c.pout[m], __fmul_rn((float)p, c.pin[m]));
+        const float U = __fmaf_rn(-lam, cost, a.acc[(size_t)i * M + m]);
+        const InstParams ip = sb.inst[j];
+        const int2 bk = sb.bkt[(size_t)(q.p >> ip.shift) * I + j];
+        const int k = bk.y + (q.p > bk.x ? 1 : 0);
+        const float4 e = reinterpret_cast<const float4 *>(sb.tile + tile_base(c, j))[(size_t)k * 4 * c.tgp + tile_col(c, j)];
+        a.assign[i] = j;
+        a.util[i] = U;
+        if (a.ttft_chosen) a.ttft_chosen[i] = ttft_exact64<MODE>(c, sb, q, j, k, e);
+    }
+}
+
+// OnTimeUtility (Eq. 4) and SLO attainment: CTA b sums the fixed row range
+// [b R, (b + 1) R) in a fixed tree order into part[2 b .. 2 b + 1]; k_on_time_final
+// adds the parts in index order.  The realized TTFT is the fp32 sum delay + ttft.
+__global__ void __launch_bounds__(256) k_on_time_part(int Q, const float *util, const float *ttft, const float *tau,
+                                                      const float *delay, double *part) {
+    __shared__ double su[256], sn[256];
+    const int R = (Q + gridDim.x - 1) / gridDim.x;
+    const int lo = blockIdx.x * R, hi = min(Q, lo + R);
+    double u = 0.0, n = 0.0;
+    for (int i = lo + threadIdx.x; i < hi; i += blockDim.x) {
+        const float realized = delay ? __fadd_rn(delay[i], ttft[i]) : ttft[i];
+        if (realized <= tau[i]) {
+            u += (double)util[i];
+            n += 1.0;
+        }
+    }
+    su[threadIdx.x] = u;
+    sn[threadIdx.x] = n;
+    __syncthreads();
+    for (int h = 128; h > 0; h >>= 1) {
+        if (threadIdx.x < h) {
+            su[threadIdx.x] += su[threadIdx.x + h];
+            sn[threadIdx.x] += sn[threadIdx.x + h];
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        part[2 * blockIdx.x] = su[0];
+        part[2 * blockIdx.x + 1] = sn[0];
+    }
+}
+
+__global__ void k_on_time_final(int Q, int parts, const double *part, double *out) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) {
+        double u = 0.0, n = 0.0;
+        for (int b = 0; b < parts; ++b) {
+            u += part[2 * b];
+            n += part[2 * b + 1];
+        }
+        out[0] = u / Q;
+        out[1] = n / Q;
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_queue_params(int I, const QueueRaw *raw, QueueDev *qd, cudaStream_t st) {
@@ -760,6 +935,36 @@ cudaError_t launch_features(const K2Launch &a, int sms, cudaStream_t st) {
 cudaError_t launch_frontier(const K2Launch &a, double *out, cudaStream_t st) {
     k_frontier<<<a.P, 256, 0, st>>>(a, out);
     return cudaGetLastError();
+}
+
+size_t baseline_smem(const DevConfig &c) {
+    int P2 = 1;
+    while (P2 < c.I) P2 <<= 1;
+    return 8 * (size_t)((c.I + P2 + 1) / 2) + 8 * (size_t)(c.I + 1) + 4 * (size_t)c.M;
+}
+
+cudaError_t launch_baseline(const K2Launch &a, int policy, long long rr_start, float lam, int sms, cudaStream_t st) {
+    const size_t smem = baseline_smem(a.cfg);
+    const int grid = std::max(1, std::min((a.Q + 255) / 256, sms * 4));
+    if (a.cfg.mode == 0) k_baseline<0><<<grid, 256, smem, st>>>(a, policy, rr_start, lam);
+    else k_baseline<1><<<grid, 256, smem, st>>>(a, policy, rr_start, lam);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_on_time(int Q, const float *util, const float *ttft, const float *tau, const float *delay,
+                           double *part, int max_parts, double *out, cudaStream_t st) {
+    const int parts = std::max(1, std::min(max_parts, (Q + 2047) / 2048));
+    k_on_time_part<<<parts, 256, 0, st>>>(Q, util, ttft, tau, delay, part);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    k_on_time_final<<<1, 32, 0, st>>>(Q, parts, part, out);
+    return cudaGetLastError();
+}
+
+cudaError_t set_baseline_smem(size_t bytes) {
+    cudaError_t e = cudaFuncSetAttribute(k_baseline<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_baseline<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    return e;
 }
 
 cudaError_t set_k2_smem(size_t bytes) {

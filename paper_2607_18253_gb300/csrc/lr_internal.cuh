@@ -215,6 +215,14 @@ int cand_out_flags(bool matrix, bool iters, bool route, bool constrained, int P)
 cudaError_t launch_cand(const K2Launch &a, int out, dim3 grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_features(const K2Launch &a, int sms, cudaStream_t st);
 cudaError_t launch_frontier(const K2Launch &a, double *out, cudaStream_t st);
+// Baseline routing policies (0 Round Robin, 1 Shortest Queue, 2 Latency-Agnostic) and
+// the stream metrics (OnTimeUtility, SLO attainment) over routed queries.
+size_t baseline_smem(const DevConfig &c);
+cudaError_t set_baseline_smem(size_t bytes);
+cudaError_t launch_baseline(const K2Launch &a, int policy, long long rr_start, float lam, int sms, cudaStream_t st);
+constexpr int kOnTimeParts = 1024;
+cudaError_t launch_on_time(int Q, const float *util, const float *ttft, const float *tau, const float *delay,
+                           double *part, int max_parts, double *out, cudaStream_t st);
 cudaError_t cand_occupancy(int mode, bool route, int block, size_t smem, int *blocks_per_sm);
 cudaError_t set_k2_smem(size_t bytes);
 constexpr int kK2Block = 256;

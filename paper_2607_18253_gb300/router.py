@@ -21,10 +21,12 @@ LR_OK, LR_EINVAL, LR_ENOMEM, LR_ECUDA, LR_ECAPACITY, LR_ETRAJ, LR_ESTATE, LR_ENO
 FIRST_TOKEN_SEPARATE_DECODE = 0
 FIRST_TOKEN_WITH_LAST_CHUNK = 1
 LR_TTFT_SFS, LR_TTFT_THROUGHPUT, LR_TTFT_LPS = 0, 1, 2
+LR_POLICY_ROUND_ROBIN, LR_POLICY_SHORTEST_QUEUE, LR_POLICY_LATENCY_AGNOSTIC = 0, 1, 2
 
 EXPORTED_SYMBOLS = ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
                     "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
-                    "lr_set_queue_params", "lr_set_ttft_source", "lr_calibrate", "lr_strerror", "lr_last_error")
+                    "lr_set_queue_params", "lr_set_ttft_source", "lr_calibrate", "lr_route_baseline",
+                    "lr_on_time_utility", "lr_strerror", "lr_last_error")
 
 _P = ctypes.c_void_p
 _I32 = ctypes.c_int32
@@ -69,6 +71,8 @@ def load_library(path: str = LIB_PATH):
     lib.lr_set_queue_params.argtypes = [_P, ctypes.POINTER(_QueueParams), _P]
     lib.lr_set_ttft_source.argtypes = [_P, _I32]
     lib.lr_calibrate.argtypes = [_P, ctypes.c_int64, _P, _P, _P, _I32, _P, _P]
+    lib.lr_route_baseline.argtypes = [_P, _I32, _I32, _P, _P, _P, ctypes.c_float, ctypes.c_int64, _P, _P, _P, _P]
+    lib.lr_on_time_utility.argtypes = [_P, _I32, _P, _P, _P, _P, _P, _P]
     lib.lr_read_state.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.lr_status.argtypes = [_P, _P]
     lib.lr_strerror.argtypes = [ctypes.c_int]
@@ -77,7 +81,8 @@ def load_library(path: str = LIB_PATH):
     lib.lr_last_error.restype = ctypes.c_char_p
     for name in ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
                  "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
-                 "lr_set_queue_params", "lr_set_ttft_source", "lr_calibrate"):
+                 "lr_set_queue_params", "lr_set_ttft_source", "lr_calibrate", "lr_route_baseline",
+                 "lr_on_time_utility"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -249,6 +254,37 @@ class LatencyRouter:
             _dev(o["assign"], torch.int32, "assign_out", P * Q), _dev(o["util"], torch.float32, "util_out", P * Q),
             _dev(o["frontier"], torch.float64, "frontier_out", P * 3), _stream(stream))
         self._check(rc, "lr_route_frontier_static")
+        return o
+
+    def route_baseline(self, policy: int, prompt_len: torch.Tensor, dec_hat: torch.Tensor, acc: torch.Tensor,
+                       lam: float, rr_start: int = 0, out: Optional[dict] = None, stream=None) -> dict:
+        """A baseline router (LR_POLICY_*): {"assign", "util", "ttft_chosen"} [Q] on the device."""
+        Q, M = int(prompt_len.numel()), self.num_models
+        dev = prompt_len.device
+        o = {} if out is None else out
+        if "assign" not in o:
+            o["assign"] = torch.empty(Q, dtype=torch.int32, device=dev)
+            o["util"] = torch.empty(Q, dtype=torch.float32, device=dev)
+            o["ttft_chosen"] = torch.empty(Q, dtype=torch.float32, device=dev)
+        rc = self._lib.lr_route_baseline(
+            self._h, int(policy), Q, _dev(prompt_len, torch.int32, "prompt_len"),
+            _dev(dec_hat, torch.int32, "dec_hat", Q * M), _dev(acc, torch.float32, "acc", Q * M), float(lam),
+            int(rr_start), _dev(o["assign"], torch.int32, "assign_out", Q), _dev(o["util"], torch.float32, "util_out", Q),
+            _dev(o.get("ttft_chosen"), torch.float32, "ttft_chosen_out", Q), _stream(stream))
+        self._check(rc, "lr_route_baseline")
+        return o
+
+    def on_time_utility(self, util: torch.Tensor, ttft: torch.Tensor, tau: torch.Tensor,
+                        delay: Optional[torch.Tensor] = None, out: Optional[torch.Tensor] = None,
+                        stream=None) -> torch.Tensor:
+        """[OnTimeUtility (Eq. 4), SLO attainment] as a float64 device tensor of 2."""
+        Q = int(util.numel())
+        o = torch.empty(2, dtype=torch.float64, device=util.device) if out is None else out
+        rc = self._lib.lr_on_time_utility(
+            self._h, Q, _dev(util, torch.float32, "util", Q), _dev(ttft, torch.float32, "ttft", Q),
+            _dev(tau, torch.float32, "tau", Q), _dev(delay, torch.float32, "delay", Q),
+            _dev(o, torch.float64, "out", 2), _stream(stream))
+        self._check(rc, "lr_on_time_utility")
         return o
 
     def set_queue_params(self, prefill_tput, decode_batch_time, arrival_rate=None, service_rate=None,
