@@ -340,6 +340,7 @@ def run_gpu(args):
     avgcase = run_avgcase(args, dev, wl, flush)
     calibration = run_calibration(args, dev, flush)
     stream = None if args.no_stream else run_stream(args, dev)
+    policy_eval = None if args.no_stream else run_policy_eval(args, dev)
 
     if rank == 0:
         cpu = cpu_baseline(wl, args.cpu_seconds) if (world == 1 and not args.no_cpu) else None
@@ -362,6 +363,7 @@ def run_gpu(args):
             "avgcase": avgcase,
             "calibration": calibration,
             "stream": stream,
+            "policy_eval": policy_eval,
         }
         print(json.dumps(line), flush=True)
     rt.close()
@@ -603,6 +605,128 @@ def run_stream(args, dev):
     out["gpu_launches"] = launches
     rt.close()
     return out
+
+
+POLICY_WORKLOAD = "paper3"
+POLICY_LOADS = (0.2, 0.4, 0.6, 0.8)
+POLICY_QUERIES = 4096
+POLICY_BATCH = 1  # every query is routed on arrival, as in the paper
+POLICIES = (("sfs_constrained", None), ("round_robin", 0), ("shortest_queue", 1), ("latency_agnostic", 2))
+
+
+def run_policy_eval(args, dev):
+    """Routing quality of the SFS router and the baselines on synthetic streams (Sec. 6, Eq. 4).
+
+    A pool of one instance per model, as in the paper (the Latency-Agnostic baseline sends
+    every query of a model to one instance, so replicas would only stand idle), starting
+    empty, fed Poisson arrivals at 0.2 .. 0.8 x its capacity (the paper's OnTimeUtility
+    against arrival rate) and MMPP-2 arrivals at 0.6 x.  "auc" is the mean OnTimeUtility
+    over the Poisson rates (trapezoids on the evenly spaced grid)."""
+    import dataclasses
+
+    from paper_2607_18253_gb300 import router as R
+    from paper_2607_18253_gb300 import workloads as W
+
+    wl = W.make_workload(POLICY_WORKLOAD, num_queries=POLICY_QUERIES, cap_waiting=1024)
+    cap = pool_capacity(R, W, wl, dev)
+    I = wl.num_instances
+    wl = dataclasses.replace(wl, n_run=np.zeros(I, np.int32), n_wait=np.zeros(I, np.int32))
+    rt = R.LatencyRouter.from_workload(wl, max_queries=POLICY_BATCH)
+    p, dh, acc, _ = R.query_tensors(wl, dev)
+    out = {"workload": f"{POLICY_WORKLOAD}: 3 models, one instance each, starting empty; {POLICY_QUERIES} arrivals "
+                       f"per trace, TTFT targets of App. B.2", "capacity_qps": float(cap.sum()), "poisson": {}}
+    launches = 0
+    for f in POLICY_LOADS:
+        rate = f * float(cap.sum())
+        r = _policy_eval(rt, wl, W.poisson_arrivals(POLICY_QUERIES, rate, wl.seed), dev, p, dh, acc)
+        out["poisson"][f"{f:.1f}"] = r
+        launches += r["gpu_launches"]
+    rate = 0.6 * float(cap.sum())
+    out["mmpp2_r6_0.6"] = _policy_eval(rt, wl, W.mmpp2_arrivals(POLICY_QUERIES, rate, 6.0, wl.seed), dev, p, dh, acc)
+    launches += out["mmpp2_r6_0.6"]["gpu_launches"]
+    auc = {}
+    for name, _ in POLICIES:
+        y = [out["poisson"][f"{f:.1f}"]["policies"][name]["on_time_utility"] for f in POLICY_LOADS]
+        auc[name] = float(np.mean([(a + b) / 2 for a, b in zip(y[:-1], y[1:])]))
+    out["auc"] = auc
+    best = max(v for k, v in auc.items() if k != "sfs_constrained")
+    out["sfs_auc_over_best_baseline"] = auc["sfs_constrained"] / best if best > 0 else None
+    out["gpu_launches"] = launches
+    rt.close()
+    return out
+
+
+def _policy_eval(rt, wl, arr, dev, p, dh, acc):
+    """One trace: every policy routes the same arrivals from the same initial state.
+
+    The first POLICY_QUERIES arrivals are routed in micro-batches of POLICY_BATCH at the
+    arrival of each batch's last query, by the constrained objective (Eq. 3) on SFS
+    estimates or by a baseline policy; every batch joins its chosen instances before the
+    next is routed.  A query's realized TTFT is the time it waited for the decision
+    plus the chosen instance's SFS estimate (the synthetic engine runs the same batch
+    model), on time if within its target; OnTimeUtility and SLO attainment come from
+    lr_on_time_utility.  Also reported: mean utility, mean realized TTFT, and the device
+    time per micro-batch (advance + route)."""
+    import ctypes
+
+    import torch
+    from paper_2607_18253_gb300 import router as R
+
+    m, n = POLICY_BATCH, POLICY_QUERIES
+    nb = n // m
+    M = wl.num_models
+    lib, h = rt._lib, rt._h
+    sp = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    V = ctypes.c_void_p
+    td = np.repeat(arr[m - 1:nb * m:m], m)  # decision time of each query's batch
+    delay = torch.from_numpy((td - arr[:nb * m]).astype(np.float32)).to(dev)
+    tau = torch.from_numpy(np.ascontiguousarray(wl.tau[:nb * m], np.float32)).to(dev)
+    util = torch.empty(nb * m, dtype=torch.float32, device=dev)
+    ttft = torch.empty(nb * m, dtype=torch.float32, device=dev)
+    assign = torch.full((2, m), -1, dtype=torch.int32, device=dev)
+    lam = np.ascontiguousarray(wl.lam[:1], np.float32)
+    lamp = lam.ctypes.data_as(V)
+    pp, dhp, accp, taup = p.data_ptr(), dh.data_ptr(), acc.data_ptr(), tau.data_ptr()
+    up, tp = util.data_ptr(), ttft.data_ptr()
+    ap = [assign[0].data_ptr(), assign[1].data_ptr()]
+    state = R.state_tensors(wl, dev)
+    res = {}
+    for name, pol in POLICIES:
+        rt.load_state(*state)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record()
+        for b in range(nb):
+            lo = b * m
+            cur, prev = ap[b & 1], ap[(b - 1) & 1]
+            pm = m if b > 0 else 0
+            plo = max((b - 1) * m, 0)
+            rc = lib.lr_advance(h, pm, V(prev), V(pp + 4 * plo), V(dhp + 4 * M * plo), M,
+                                ctypes.c_double(float(td[lo])), sp)
+            if pol is None:
+                rc |= lib.lr_route(h, m, V(pp + 4 * lo), V(dhp + 4 * M * lo), V(accp + 4 * M * lo), V(taup + 4 * lo),
+                                   1, lamp, None, V(cur), V(up + 4 * lo), V(tp + 4 * lo), None, None, sp)
+            else:
+                rc |= lib.lr_route_baseline(h, pol, m, V(pp + 4 * lo), V(dhp + 4 * M * lo), V(accp + 4 * M * lo),
+                                            ctypes.c_float(float(lam[0])), ctypes.c_int64(lo), V(cur),
+                                            V(up + 4 * lo), V(tp + 4 * lo), sp)
+            if rc:
+                raise RuntimeError(f"policy run {name} failed: {lib.lr_last_error(h).decode()}")
+        e1.record()
+        torch.cuda.synchronize()
+        st = rt.status()
+        if st != R.LR_OK:
+            raise RuntimeError(f"policy run {name} ended with device status {st}")
+        otu, slo = (float(x) for x in rt.on_time_utility(util, ttft, tau, delay).cpu().numpy())
+        realized = (delay + ttft).cpu().numpy()
+        fin = rt.read_state(device=dev)
+        res[name] = {"on_time_utility": otu, "slo_attainment": slo, "mean_utility": float(util.mean().item()),
+                     "mean_realized_ttft_s": float(realized.mean()), "us_per_batch": e0.elapsed_time(e1) * 1e3 / nb,
+                     "final_max_waiting": int(fin["n_wait"].max().item())}
+    return {"queries": nb * m, "micro_batch": m, "lambda": float(lam[0]),
+            "objective": "SFS router: Eq. 3 (max utility within the TTFT target, else least TTFT)",
+            "realized_ttft": "decision delay + SFS estimate of the chosen instance",
+            "policies": res, "gpu_launches": len(POLICIES) * (3 * nb + 3)}
 
 
 def _oracle_rows(wl, nq, seed):

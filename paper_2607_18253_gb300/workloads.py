@@ -152,6 +152,9 @@ RECIPES: Dict[str, dict] = {
                    p_median=1024, p_cap=8192, budget=4096, seqs=64, acc="uniform"),
     "pool256": dict(models=8, replicas=32, queries=65536, seed=2, run_max=256, wait_max=256,
                     p_median=1024, p_cap=32768, budget=8192, seqs=256, acc="beta22"),
+    # one instance per model, as in the paper's pool of three models (Sec. 6)
+    "paper3": dict(models=3, replicas=1, queries=4096, seed=4, run_max=64, wait_max=64,
+                   p_median=1024, p_cap=8192, budget=4096, seqs=64, acc="uniform"),
 }
 
 
@@ -163,7 +166,7 @@ def make_workload(name: str, num_queries: Optional[int] = None, seed: Optional[i
                   lam: Optional[np.ndarray] = None, mu: Optional[np.ndarray] = None,
                   first_token_mode: int = FIRST_TOKEN_SEPARATE_DECODE, cap_running: Optional[int] = None,
                   cap_waiting: Optional[int] = None) -> Workload:
-    """Build one of the named workloads ("tiny", "pool64", "pool256").
+    """Build one of the named workloads ("tiny", "pool64", "pool256", "paper3").
 
     The instance state and the queries come from independent child streams of
     the seed, so changing the query count leaves the state unchanged and keeps
