@@ -33,6 +33,10 @@ sys.path.insert(0, ROOT)
 METRIC = "TTFT estimates/sec (query×instance) on 1 GB300; p50 per-batch route latency"
 UNIT = "estimates/s"
 WORKLOAD = "pool256"
+# DRAM bytes (read + write) per launch of the step's kernels on this workload, from one
+# ncu capture of the kernels as they are built now (summaries under profiles/); they
+# are retaken whenever one of the kernels changes.
+NCU_TRAFFIC = {"k_route": 4_569_856 + 6_927_872, "k_trajectory": 1_392_896}
 
 
 def _peaks():
@@ -330,12 +334,13 @@ def run_gpu(args):
         ach = route_bytes / (route_avg * 1e-3) / 1e9
         roof = {"kernel": "k_route", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                 "frac": ach / hbm, "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs, copy)",
-                "traffic": args.traffic}
+                "traffic": args.traffic if args.traffic is not None else NCU_TRAFFIC["k_route"]}
     else:
         ach = load_bytes / (load_avg * 1e-3) / 1e9
         roof = {"kernel": "k_trajectory", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                 "frac": ach / hbm, "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs, copy)",
-                "traffic": None, "note": "latency-bound event loop; bytes fraction shown for reference"}
+                "traffic": args.traffic if args.traffic is not None else NCU_TRAFFIC["k_trajectory"],
+                "note": "latency-bound event loop; bytes fraction shown for reference"}
 
     avgcase = run_avgcase(args, dev, wl, flush)
     calibration = run_calibration(args, dev, flush)
