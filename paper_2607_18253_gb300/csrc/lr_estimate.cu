@@ -451,8 +451,13 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
 #pragma unroll
     for (int u = 1; u < 4; ++u) same_model = same_model && model[u] == model[0];
 
-    auto run = [&](auto fast_tag) {
+    // SPEC: every thread of the CTA has four instances of one model, the fp32 split path
+    // and aligned vector stores, so none of the per-thread checks below is needed (an
+    // invalid prompt still gives NaN times, which no comparison selects)
+    const bool spec = __syncthreads_and(fast && nv == 4 && same_model && a.vec_ok);
+    auto run = [&](auto fast_tag, auto spec_tag) {
         constexpr bool FAST = decltype(fast_tag)::value;
+        constexpr bool SPEC = decltype(spec_tag)::value;
         // chunk k: the first QT rows of the range in s_claim[k & 1], staged in raw buffer k & 1
         for (int buf = 0;; buf ^= 1) {
             int q0, nrows;
@@ -510,10 +515,10 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                     kk[u] = bk.y + (q.p > bk.x ? 1 : 0);
                     const float4 e = lds_float4(ecol + u * ecst + (uint32_t)kk[u] * erow);
                     if (FAST) t[u] = ttft_fast<MODE>(q, r, u, e);
-                    else t[u] = (u < nv) ? ttft_exact64<MODE>(c, sb, q, jb + u, kk[u], e) : 0.f;
+                    else t[u] = (SPEC || u < nv) ? ttft_exact64<MODE>(c, sb, q, jb + u, kk[u], e) : 0.f;
                 }
                 if (OUT & kOutMatrix) {
-                    if (vec) {
+                    if (SPEC || vec) {
                         __stcs(reinterpret_cast<float4 *>(orow), make_float4(t[0], t[1], t[2], t[3]));
                     } else {
                         for (int u = 0; u < nv; ++u) __stcs(orow + u, t[u]);
@@ -526,7 +531,7 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                     for (int u = 0; u < nv; ++u) a.first_batch[o + u] = bad ? -1 : la[u] + kk[u] + off;
                 }
                 if (ROUTE) {
-                    const bool row_ok = q.fp == q.fp;
+                    const bool row_ok = SPEC || q.fp == q.fp;
                     const float2 *carow = s_ca + rr * M;
                     const float tau = CON ? s_tau[rr] : 0.f;
 #pragma unroll 1
@@ -534,7 +539,7 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                         const float lam = SWEEP ? a.lam[pp] : 0.f;
                         const float mu = a.mu[pp];
                         float U[4];
-                        if (same_model) {
+                        if (SPEC || same_model) {
                             const float2 ca = carow[model[0]];
                             U[0] = U[1] = U[2] = U[3] = SWEEP ? __fmaf_rn(-lam, ca.x, ca.y) : ca.x;
                         } else {
@@ -549,19 +554,19 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                         float best1, best2 = 0.f;
                         int u1 = 0, u2 = 0;
                         if (CON) {
-                            best1 = (0 < nv && row_ok && t[0] <= tau) ? U[0] : kNaN;
-                            best2 = (0 < nv && row_ok) ? t[0] : kNaN;
+                            best1 = ((SPEC || 0 < nv) && row_ok && t[0] <= tau) ? U[0] : kNaN;
+                            best2 = ((SPEC || 0 < nv) && row_ok) ? t[0] : kNaN;
 #pragma unroll
                             for (int u = 1; u < 4; ++u) {
-                                if (u < nv && t[u] <= tau && (U[u] > best1 || best1 != best1)) { best1 = U[u]; u1 = u; }
-                                if (u < nv && t[u] < best2) { best2 = t[u]; u2 = u; }
+                                if ((SPEC || u < nv) && t[u] <= tau && (U[u] > best1 || best1 != best1)) { best1 = U[u]; u1 = u; }
+                                if ((SPEC || u < nv) && t[u] < best2) { best2 = t[u]; u2 = u; }
                             }
                         } else {
-                            best1 = (0 < nv && row_ok) ? __fmaf_rn(-mu, t[0], U[0]) : kNaN;
+                            best1 = ((SPEC || 0 < nv) && row_ok) ? __fmaf_rn(-mu, t[0], U[0]) : kNaN;
 #pragma unroll
                             for (int u = 1; u < 4; ++u) {
                                 const float J = __fmaf_rn(-mu, t[u], U[u]);
-                                if (u < nv && J > best1) { best1 = J; u1 = u; }
+                                if ((SPEC || u < nv) && J > best1) { best1 = J; u1 = u; }
                             }
                         }
                         const unsigned k1 = (best1 == best1) ? order_key(best1) : 0u;
@@ -616,8 +621,9 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
             __syncthreads();
         }
     };
-    if (fast) run(Flag<true>{});
-    else run(Flag<false>{});
+    if (spec) run(Flag<true>{}, Flag<true>{});
+    else if (fast) run(Flag<true>{}, Flag<false>{});
+    else run(Flag<false>{}, Flag<false>{});
     (void)grp_lane0;
     }
 finish:
