@@ -325,10 +325,13 @@ def run_gpu(args):
     route_bytes = cands * 4 + Q * (4 + 8 * M) + Q * 12
     load_bytes = 2 * 4 * (I * (3 * wl.cap_running + 2 * wl.cap_waiting) + 2 * I)
     kernels = {
-        "k_route (TTFT matrix + utility + argmax)": {"ms": route_avg, "share": route_avg / seq_ms,
-                                                      "algorithmic_bytes": route_bytes},
-        "k_trajectory (snapshot copy + summary)": {"ms": load_avg, "share": load_avg / seq_ms,
-                                                    "algorithmic_bytes": load_bytes},
+        "k_route (TTFT matrix + utility + argmax)": {
+            "ms": route_avg, "share": route_avg / seq_ms, "algorithmic_bytes": route_bytes,
+            "hbm_frac": route_bytes / (route_avg * 1e-3) / 1e9 / hbm, "dram_bytes_ncu": NCU_TRAFFIC["k_route"]},
+        "k_trajectory (snapshot copy + summary)": {
+            "ms": load_avg, "share": load_avg / seq_ms, "algorithmic_bytes": load_bytes,
+            "hbm_frac": load_bytes / (load_avg * 1e-3) / 1e9 / hbm, "dram_bytes_ncu": NCU_TRAFFIC["k_trajectory"],
+            "bound": "dependency-latency chain of the slowest instance"},
     }
     if route_avg >= load_avg:
         ach = route_bytes / (route_avg * 1e-3) / 1e9
@@ -342,6 +345,7 @@ def run_gpu(args):
                 "traffic": args.traffic if args.traffic is not None else NCU_TRAFFIC["k_trajectory"],
                 "note": "latency-bound event loop; bytes fraction shown for reference"}
 
+    estimate = run_estimate(args, dev, wl, flush)
     avgcase = run_avgcase(args, dev, wl, flush)
     calibration = run_calibration(args, dev, flush)
     stream = None if args.no_stream else run_stream(args, dev)
@@ -365,6 +369,7 @@ def run_gpu(args):
             "gpu_launches": 2 * K, "clocks": clk.summary(), "wall_s_timed_region": t_wall,
             "sequential": {"ms_per_step": seq_ms, "value": cands * world / (seq_ms * 1e-3), "unit": UNIT,
                            "note": "K1 then K2 on one stream, same steps (kernel shares are of this time)"},
+            "estimate": estimate,
             "avgcase": avgcase,
             "calibration": calibration,
             "stream": stream,
@@ -416,6 +421,57 @@ def run_calibration(args, dev, flush):
             "value": N / (ms_avg * 1e-3), "unit": "batches/s", "max_rel_error_vs_generating_coef": rel,
             "gpu_launches": 2 * K,
             "roofline": {"kernel": "k_calib_accum", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+                         "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
+                         "algorithmic_bytes": nbytes}}
+
+
+def run_estimate(args, dev, wl, flush):
+    """The SFS estimate alone (Eq. 8-9, lr_estimate_ttft) on the same workload: the full
+    TTFT matrix from the live snapshot, timed against HBM (4 B per candidate, 4 B per
+    query and the ~64 KiB summary).  The snapshot is loaded on the capture stream, so
+    the call runs alone with a static row split."""
+    import torch
+    from paper_2607_18253_gb300 import router as R
+
+    Q, I = wl.num_queries, wl.num_instances
+    rt = R.LatencyRouter.from_workload(wl)
+    state = R.state_tensors(wl, dev)
+    p = torch.from_numpy(np.ascontiguousarray(wl.prompt_len)).to(dev)
+    mat = torch.empty((Q, I), dtype=torch.float32, device=dev)
+    cap = torch.cuda.Stream(device=dev)
+    cap.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(cap):
+        rt.load_state(*state)
+        for _ in range(3):
+            rt.estimate_ttft(p, out=mat)
+    cap.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=cap):
+        rt.estimate_ttft(p, out=mat)
+    for _ in range(args.warmup):
+        flush.fill_(1.0)
+        g.replay()
+    torch.cuda.synchronize()
+    K = max(3, min(args.steps, 500))
+    ms = []
+    for k in range(K):
+        flush.fill_(float(k))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        g.replay()
+        e1.record()
+        e1.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    if rt.status() != R.LR_OK:
+        raise RuntimeError("SFS estimate failed")
+    rt.close()
+    ms_avg = sum(ms) / K
+    hbm, src = _peaks()
+    nbytes = Q * I * 4 + Q * 4 + 64 * 1024
+    ach = nbytes / (ms_avg * 1e-3) / 1e9
+    return {"call": "lr_estimate_ttft (SFS), full Q x I matrix", "ms": ms_avg, "value": Q * I / (ms_avg * 1e-3),
+            "unit": UNIT, "steps": K, "gpu_launches": K,
+            "roofline": {"kernel": "k_cand<0, 1>", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                          "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
                          "algorithmic_bytes": nbytes}}
 

@@ -25,6 +25,10 @@ struct lr_ctx {
     uint32_t *k2_work = nullptr;  // the candidate kernel's row counters
     double *ontime_part = nullptr;  // per-CTA partial sums of lr_on_time_utility
     bool bl_ok = false;             // the baseline policies' shared memory fits
+    // stream of the last snapshot load (lr_load_state or lr_advance): a candidate-kernel
+    // call on another stream may run beside it
+    void *load_stream = nullptr;
+    bool loaded_any = false;
     // average-case TTFT sources
     lr::QueueRaw *qraw = nullptr;
     lr::QueueDev *qd = nullptr;
@@ -121,12 +125,19 @@ lr_ctx::Shape make_shape(const lr::DevConfig &d, bool route, int max_pairs) {
     return s;
 }
 
-// Row split of a candidate-kernel launch of `ctas` CTAs per tile.  The CTAs that fit
-// beside a snapshot load's K1 CTAs (one candidate-kernel slot each) start with a
-// static range of 90% of their share of the rows; the other rows are claimed as
-// they run out, by the remaining CTAs and by whichever finish early, so that every
-// CTA ends on small claimed chunks.
-void set_row_split(lr::K2Launch &a, const lr_ctx *c, int ctas, int tiles, int occ) {
+// Row split of a candidate-kernel launch of `ctas` CTAs per tile.  Calls on one
+// context are ordered except a snapshot load beside an estimate or route on another
+// stream, so a call on the last load's stream runs alone: every CTA takes an equal
+// static range.  Otherwise the CTAs that fit beside the load's K1 CTAs (one
+// candidate-kernel slot each) start with a static range of 90% of their share, and
+// the other rows are claimed as they run out, by the remaining CTAs and by whichever
+// finish early, so that every CTA ends on small claimed chunks.
+void set_row_split(lr::K2Launch &a, const lr_ctx *c, int ctas, int tiles, int occ, void *stream) {
+    if (!c->loaded_any || stream == c->load_stream) {
+        a.first_ctas = ctas;
+        a.first_rows = std::max(1, (a.Q + ctas - 1) / std::max(1, ctas));
+        return;
+    }
     const int k1 = (c->cfg.I + lr::kK1Warps - 1) / lr::kK1Warps;
     a.first_ctas = tiles == 1 ? std::max(0, std::min(ctas, c->sms * occ - k1)) : 0;
     const int f = (int)((long long)a.Q * 9 / (10LL * std::max(1, ctas)));
@@ -342,7 +353,10 @@ int lr_load_state(lr_ctx *c, const lr_state_view *v, void *stream) {
     a.in = lr::StateIn{v->n_run, v->run_ctx, v->run_pre, v->run_dec, v->n_wait, v->wait_pre, v->wait_dec, nullptr};
     const int grid = (c->cfg.I + lr::kK1Warps - 1) / lr::kK1Warps;
     cudaError_t e = lr::launch_trajectory(a, grid, lr::kK1Warps * 32, c->k1_smem, (cudaStream_t)stream);
-    return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "trajectory launch");
+    if (e != cudaSuccess) return cuda_fail(c, e, "trajectory launch");
+    c->load_stream = stream;
+    c->loaded_any = true;
+    return LR_OK;
 }
 
 static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, int32_t *iters, int64_t *feat,
@@ -371,7 +385,7 @@ static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, 
     a.QT = c->est.QT;
     a.vec_ok = (c->cfg.I % 4 == 0) && ((uintptr_t)ttft % 16 == 0);
     dim3 grid(std::min(c->sms * c->est.occ, (Q + a.QS - 1) / a.QS), c->est.tiles);
-    set_row_split(a, c, (int)grid.x, (int)grid.y, c->est.occ);
+    set_row_split(a, c, (int)grid.x, (int)grid.y, c->est.occ, stream);
     e = lr::launch_cand(a, lr::cand_out_flags(true, iters != nullptr, false, false, 1), grid, lr::kK2Block,
                         c->est.smem, (cudaStream_t)stream);
     return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "estimate launch");
@@ -426,7 +440,7 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
     a.QT = c->rt.QT;
     a.vec_ok = (c->cfg.I % 4 == 0) && ((uintptr_t)ttft_matrix_out % 16 == 0);
     dim3 grid(std::min(c->sms * c->rt.occ, (Q + a.QS - 1) / a.QS), 1);
-    set_row_split(a, c, (int)grid.x, 1, c->rt.occ);
+    set_row_split(a, c, (int)grid.x, 1, c->rt.occ, stream);
     cudaError_t e = lr::launch_cand(a, lr::cand_out_flags(ttft_matrix_out != nullptr, false, true, tau != nullptr, P),
                                     grid, lr::kK2Block, c->rt.smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(c, e, "route launch");
@@ -624,7 +638,10 @@ int lr_advance(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_t *promp
     a.in = lr::StateIn{sc.n_run, sc.run_ctx, sc.run_pre, sc.run_dec, sc.n_wait, sc.wait_pre, sc.wait_dec, sc.clock};
     const int grid = (c->cfg.I + lr::kK1Warps - 1) / lr::kK1Warps;
     e = lr::launch_trajectory(a, grid, lr::kK1Warps * 32, c->k1_smem, st);
-    return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "trajectory launch");
+    if (e != cudaSuccess) return cuda_fail(c, e, "trajectory launch");
+    c->load_stream = stream;
+    c->loaded_any = true;
+    return LR_OK;
 }
 
 int lr_read_state(const lr_ctx *c, int32_t *n_run, int32_t *run_ctx, int32_t *run_pre, int32_t *run_dec,
