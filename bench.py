@@ -36,7 +36,7 @@ WORKLOAD = "pool256"
 # DRAM bytes (read + write) per launch of the step's kernels on this workload, from one
 # ncu capture of the kernels as they are built now (summaries under profiles/); they
 # are retaken whenever one of the kernels changes.
-NCU_TRAFFIC = {"k_route": 4_569_856 + 6_927_872, "k_trajectory": 1_392_896}
+NCU_TRAFFIC = {"k_route": 4_585_216 + 8_863_744, "k_trajectory": 1_392_896, "k_estimate": 357_632 + 7_219_456}
 
 
 def _peaks():
@@ -473,7 +473,7 @@ def run_estimate(args, dev, wl, flush):
             "unit": UNIT, "steps": K, "gpu_launches": K,
             "roofline": {"kernel": "k_cand<0, 1>", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                          "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
-                         "algorithmic_bytes": nbytes}}
+                         "algorithmic_bytes": nbytes, "traffic": NCU_TRAFFIC["k_estimate"]}}
 
 
 def run_avgcase(args, dev, wl, flush):
