@@ -51,7 +51,7 @@ struct WarpSmem {
     int32_t *P;      // [capW + 2] exclusive prefix sums of waiting prompts (+1 unread pad)
     int32_t *wdec;   // [capW + 1] waiting decode lengths (+1 unread pad)
     int32_t *rcum;   // [kph] cumulative budgets
-    int32_t *scr;    // [32] results of the step loop
+    int32_t *scr;    // [32] a seat run's request-to-batch map, then the step loop's results
 };
 
 __device__ __forceinline__ WarpSmem carve(int32_t *base, const DevConfig &c) {
@@ -91,24 +91,9 @@ __device__ __forceinline__ int warp_excl_sum6(int v, unsigned lt) {
     return r;
 }
 
-// Position of set bit number r (from 0) of x, which has more than r set bits.
-__device__ __forceinline__ int select_bit(uint32_t x, int r) {
-    int pos = 0;
-#pragma unroll
-    for (int half = 16; half >= 1; half >>= 1) {
-        const int c = __popc(x & ((1u << half) - 1u));
-        if (r >= c) {
-            r -= c;
-            x >>= half;
-            pos += half;
-        }
-    }
-    return pos;
-}
-
 // Shared-memory accesses of the step loop by 32-bit shared address: the loop is
-// a chain of dependent decisions on one lane, so every address computation and
-// every generic-to-shared translation sits on its critical path.  The volatile
+// a chain of dependent decisions, so every address computation and every
+// generic-to-shared translation sits on its critical path.  The volatile
 // statements keep their program order, which the loop relies on.
 __device__ __forceinline__ uint32_t saddr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 __device__ __forceinline__ int lds(uint32_t a) {
@@ -123,6 +108,9 @@ __device__ __forceinline__ void red_or(uint32_t a, uint32_t v) {
     asm volatile("red.shared.or.b32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
 }
 
+__device__ __forceinline__ void sts(uint32_t a, int v) {
+    asm volatile("st.shared.s32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
 __device__ __forceinline__ void sts4(uint32_t a, int x, int y, int z, int w) {
     asm volatile("st.shared.v4.s32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(x), "r"(y), "r"(z), "r"(w) : "memory");
 }
@@ -407,8 +395,12 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             if (kmax <= 0 || (em & ((2u << kmax) - 1u) & ~1u) == 0u) return false;
             // request lane i: the lane of its batch (the run's request starts, by rank) and its last batch
             const int nreq = __shfl_sync(kFull, x0, kmax);
-            const unsigned starts = __reduce_or_sync(kFull, ck > 0 && x0 < 32 ? 1u << x0 : 0u);
-            const int kq = select_bit(em, (__popc(starts & ((2u << lane) - 1u)) - 1) & 31);
+            // each batch lane below kmax writes its index into its requests' slots (those
+            // requests fit the 32 lanes: x1 <= 32), and request lane i reads slot i
+            if (lane < kmax)
+                for (int t = x0; t < x1; ++t) sts(sE + 4u * t, lane);
+            __syncwarp();
+            const int kq = lane < nreq ? lds(sE + 4u * lane) : 0;
             const int fi = lane < nreq ? e0 + kq + 1 + dq - MODE : kBig;
             // (c): a request of lane kq ending in batch f rules out every K > kq with e0 + K >= f
             int K = kmax;
