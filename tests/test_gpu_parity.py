@@ -236,6 +236,38 @@ def test_route_full_size_against_gpu_matrix():
     np.testing.assert_array_equal(bits(o["ttft_matrix"][cq, cj]), bits(t32))
 
 
+def test_route_on_a_second_stream_full_size():
+    # the bench's step configuration: pool256 routed on a stream other than the
+    # load's, so that its rows are claimed dynamically, first alone and then beside a
+    # concurrent reload of the same snapshot; 256 sampled queries against the
+    # oracle's route over their full oracle rows
+    wl = W.make_workload("pool256")
+    rt = make_router(wl)
+    state = R().state_tensors(wl)
+    p, dh, acc, _ = R().query_tensors(wl)
+    main = torch.cuda.current_stream()
+    side = torch.cuda.Stream()
+    results = []
+    for reload in (False, True):
+        side.wait_stream(main)
+        if reload:
+            rt.load_state(*state)  # on the main stream, while the side stream routes
+        with torch.cuda.stream(side):
+            o = rt.route(p, dh, acc, wl.lam, wl.mu, stream=side)
+        torch.cuda.synchronize()
+        assert rt.status() == R().LR_OK
+        results.append({k: o[k].cpu().numpy() for k in ("assign", "util", "ttft_chosen")})
+    for k in ("assign", "util", "ttft_chosen"):
+        np.testing.assert_array_equal(results[0][k].view(np.uint32), results[1][k].view(np.uint32))
+    qs = np.sort(np.random.default_rng(11).choice(wl.num_queries, 256, replace=False))
+    sub = wl.with_queries(qs)
+    _, _, t32, _ = oracle.estimate_matrix(sub)
+    ea, eu, et = oracle.route(sub, t32, lam=wl.lam, mu=wl.mu)
+    np.testing.assert_array_equal(results[0]["assign"][0][qs], ea[0])
+    np.testing.assert_array_equal(bits(results[0]["util"][0][qs]), bits(eu[0]))
+    np.testing.assert_array_equal(bits(results[0]["ttft_chosen"][0][qs]), bits(et[0]))
+
+
 def test_edge_prompts_and_ragged_rows():
     wl = W.make_workload("pool64", num_queries=1001)
     wl.prompt_len[:6] = [1, 2, wl.max_prompt_len, wl.max_prompt_len - 1, 4095, 4097]
