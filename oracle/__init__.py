@@ -83,6 +83,10 @@ def _load():
         lib.orc_latency_agnostic.restype = ctypes.c_int
         lib.orc_on_time_utility.argtypes = [i32, P, P, P, P, P]
         lib.orc_on_time_utility.restype = ctypes.c_int
+        lib.orc_sfs_candidate_kv.argtypes = [P, i32, i32, i32, P, i32, i32, i64, P, P, P, P, P]
+        lib.orc_sfs_candidate_kv.restype = ctypes.c_int
+        lib.orc_kv_residents.argtypes = [P, i32, i32, i32, P, i64, P]
+        lib.orc_kv_residents.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -364,3 +368,50 @@ def on_time_utility(util, ttft, tau, delay=None):
     if _load().orc_on_time_utility(u.shape[0], _p(u), _p(t), _p(ta), _p(d), _p(out)) != 0:
         raise RuntimeError("oracle on-time utility failed")
     return float(out[0]), float(out[1])
+
+
+# ---- KV-cache limits, context limit and preemption (App. F; rule in sfs_oracle.c) ----
+
+class _KV(ctypes.Structure):
+    _fields_ = [("block_size", ctypes.c_int32), ("num_blocks", ctypes.c_int64), ("max_ctx", ctypes.c_int64)]
+
+
+ORC_ELIMIT = 2
+
+
+def simulate_kv(running, waiting, B: int, S: int, p: int, d: int, block_size: int, num_blocks: int, max_ctx: int,
+                mode: int = FIRST_TOKEN_SEPARATE_DECODE, max_batches: int = 1 << 20):
+    """One candidate under KV limits.  running: list of (ctx, pre, dec); waiting: list of (pre, dec).
+
+    Returns (F[5], admit batch, first-token batch, residents' per-batch features [l][5],
+    most blocks in use)."""
+    run = np.asarray(running, dtype=np.int32).reshape(-1, 3)
+    wt = np.asarray(waiting, dtype=np.int32).reshape(-1, 2)
+    rc_, rp_, rd_ = (_c(run[:, k], np.int32) for k in range(3))
+    wp_, wd_ = (_c(wt[:, k], np.int32) for k in range(2))
+    inst = _Instance(run.shape[0], _p(rc_), _p(rp_), _p(rd_), wt.shape[0], _p(wp_), _p(wd_))
+    kv = _KV(block_size, num_blocks, max_ctx)
+    F = np.zeros(5, np.int64)
+    res = np.zeros((max_batches, 5), np.int64)
+    la, lt, mu = ctypes.c_int64(0), ctypes.c_int64(0), ctypes.c_int64(0)
+    rc = _load().orc_sfs_candidate_kv(ctypes.byref(inst), B, S, mode, ctypes.byref(kv), p, d, max_batches, _p(F),
+                                      ctypes.byref(la), ctypes.byref(lt), _p(res), ctypes.byref(mu))
+    if rc != 0:
+        raise RuntimeError(f"oracle KV simulation failed with code {rc}")
+    return F, la.value, lt.value, res[:lt.value].copy(), mu.value
+
+
+def kv_residents(running, waiting, B: int, S: int, L: int, block_size: int, num_blocks: int, max_ctx: int,
+                 mode: int = FIRST_TOKEN_SEPARATE_DECODE):
+    """The residents alone for L batches under KV limits: per-batch features [L][5]."""
+    run = np.asarray(running, dtype=np.int32).reshape(-1, 3)
+    wt = np.asarray(waiting, dtype=np.int32).reshape(-1, 2)
+    rc_, rp_, rd_ = (_c(run[:, k], np.int32) for k in range(3))
+    wp_, wd_ = (_c(wt[:, k], np.int32) for k in range(2))
+    inst = _Instance(run.shape[0], _p(rc_), _p(rp_), _p(rd_), wt.shape[0], _p(wp_), _p(wd_))
+    kv = _KV(block_size, num_blocks, max_ctx)
+    res = np.zeros((L, 5), np.int64)
+    rc = _load().orc_kv_residents(ctypes.byref(inst), B, S, mode, ctypes.byref(kv), L, _p(res))
+    if rc != 0:
+        raise RuntimeError(f"oracle KV residents failed with code {rc}")
+    return res

@@ -522,3 +522,176 @@ int orc_on_time_utility(int32_t Q, const float *util, const float *ttft, const f
     out[1] = sn / Q;
     return ORC_OK;
 }
+
+/* ---- KV-cache limits, context limit and preemption (App. F) ----
+ *
+ * The paper lists "context limits, KV-cache allocation state, and preemption
+ * behavior" among what the simulation accounts for, without a rule.  Reading
+ * (a paged KV cache as in vLLM, whose engine the paper uses):
+ *  - an instance has num_blocks blocks of block_size tokens; a request with ctx
+ *    tokens in the cache holds ceil(ctx / block_size) blocks;
+ *  - the running list is served in order as before; a request whose tokens of
+ *    this batch need blocks that are not free makes room by preempting the last
+ *    running request (recompute: its blocks are freed, its whole context becomes
+ *    prefill again, and it goes to the front of the waiting queue), repeatedly,
+ *    and preempts itself if it is the last;
+ *  - the waiting head is admitted only if the blocks of its first chunk are free
+ *    (FCFS, no skipping, no preemption for admission);
+ *  - a request whose context reaches max_ctx stops (its response ends there);
+ *  - a request whose whole context (capped at max_ctx) needs more blocks than the
+ *    instance has can never finish and is rejected with the input (an engine
+ *    refuses it).  Then the oldest running request can always proceed by
+ *    preempting later ones, so every simulation ends.
+ */
+static int64_t kv_blocks(int64_t ctx, int64_t bs) { return (ctx + bs - 1) / bs; }
+
+static int kv_sim(const orc_instance *inst, int32_t B, int32_t S, int32_t mode, const orc_kv *kv,
+                  int with_query, int32_t p, int32_t d, int64_t max_batches,
+                  int64_t F[5], int64_t *l_admit, int64_t *l_ttft, int64_t *res_F, int64_t *max_used)
+{
+    if (!inst || !kv || B < 1 || S < 1 || inst->n_run < 0 || inst->n_wait < 0) return ORC_EINVAL;
+    if (kv->block_size < 1 || kv->num_blocks < 0 || kv->max_ctx < 2) return ORC_EINVAL;
+    if (mode != ORC_FIRST_TOKEN_SEPARATE_DECODE && mode != ORC_FIRST_TOKEN_WITH_LAST_CHUNK) return ORC_EINVAL;
+    if (with_query && (p < 1 || d < 1 || p >= kv->max_ctx)) return ORC_EINVAL;
+    const int64_t bs = kv->block_size;
+    const int64_t total = (int64_t)inst->n_run + inst->n_wait + 1;
+    orc_req *run = (orc_req *)calloc((size_t)total, sizeof(orc_req));
+    orc_req *wait = (orc_req *)calloc((size_t)(2 * total + 1), sizeof(orc_req)); /* room at the front */
+    int64_t *alloc = (int64_t *)calloc((size_t)total, sizeof(int64_t));
+    int *kind = (int *)calloc((size_t)total, sizeof(int));
+    if (!run || !wait || !alloc || !kind) {
+        free(run); free(wait); free(alloc); free(kind);
+        return ORC_ENOMEM;
+    }
+    int rc = ORC_EINVAL;
+    int64_t nr = 0, wh = total, we = total;  /* waiting queue: wait[wh .. we) */
+    int64_t free_blocks = kv->num_blocks;
+    for (int32_t r = 0; r < inst->n_run; ++r) {
+        orc_req q = {inst->run_ctx[r], inst->run_pre[r], inst->run_dec[r], 0};
+        if (q.ctx < 0 || q.pre < 0 || q.dec < 1 || q.ctx + q.pre >= kv->max_ctx) goto done;
+        if (kv_blocks(min64(q.ctx + q.pre + q.dec, kv->max_ctx), bs) > kv->num_blocks) goto done;
+        free_blocks -= kv_blocks(q.ctx, bs);
+        run[nr++] = q;
+    }
+    if (free_blocks < 0) goto done;
+    for (int32_t w = 0; w < inst->n_wait; ++w) {
+        orc_req q = {0, inst->wait_pre[w], inst->wait_dec[w], 0};
+        if (q.pre < 1 || q.dec < 1 || q.pre >= kv->max_ctx) goto done;
+        if (kv_blocks(min64(q.pre + q.dec, kv->max_ctx), bs) > kv->num_blocks) goto done;
+        wait[we++] = q;
+    }
+    if (with_query) {
+        orc_req q = {0, p, d, 1};
+        if (kv_blocks(min64((int64_t)p + d, kv->max_ctx), bs) > kv->num_blocks) goto done;
+        wait[we++] = q;
+    }
+    if (F) for (int k = 0; k < 5; ++k) F[k] = 0;
+    if (max_used) *max_used = kv->num_blocks - free_blocks;
+    int64_t admitted_at = 0;
+    rc = ORC_ELIMIT;
+    for (int64_t l = 1; l <= max_batches; ++l) {
+        int64_t *rf = res_F ? res_F + (l - 1) * 5 : NULL;
+        if (rf) for (int k = 0; k < 5; ++k) rf[k] = 0;
+        /* 1. the running list in order, each request's blocks found or made */
+        int64_t budget = B;
+        for (int64_t r = 0; r < nr; ++r) { kind[r] = SCHED_NONE; alloc[r] = 0; }
+        int64_t r = 0;
+        while (r < nr && budget > 0) {
+            const int64_t x = run[r].pre > 0 ? min64(run[r].pre, budget) : 1;
+            const int64_t need = kv_blocks(run[r].ctx + x, bs) - kv_blocks(run[r].ctx, bs);
+            while (free_blocks < need && nr - 1 >= r) {
+                /* preempt the last running request (possibly r itself) */
+                orc_req v = run[nr - 1];
+                free_blocks += kv_blocks(v.ctx, bs);
+                v.pre += v.ctx;
+                v.ctx = 0;
+                wait[--wh] = v;
+                --nr;
+            }
+            if (r >= nr) break;  /* r preempted itself */
+            free_blocks -= need;
+            alloc[r] = x;
+            kind[r] = run[r].pre > 0 ? SCHED_PREFILL : SCHED_DECODE;
+            budget -= x;
+            ++r;
+        }
+        /* 2. admission from the waiting head while budget, a slot and its blocks allow */
+        while (budget > 0 && wh < we && nr < S) {
+            const int64_t x = min64(wait[wh].pre, budget);
+            const int64_t need = kv_blocks(x, bs);
+            if (free_blocks < need) break;
+            free_blocks -= need;
+            run[nr] = wait[wh++];
+            alloc[nr] = x;
+            kind[nr] = SCHED_PREFILL;
+            budget -= x;
+            if (run[nr].is_query) admitted_at = l;
+            ++nr;
+        }
+        if (max_used && kv->num_blocks - free_blocks > *max_used) *max_used = kv->num_blocks - free_blocks;
+        /* 3. account the batch */
+        int done_q = 0;
+        if (F) F[0] += 1;
+        if (rf) rf[0] = 1;
+        for (int64_t t = 0; t < nr; ++t) {
+            int64_t f[5] = {0, 0, 0, 0, 0};
+            if (kind[t] == SCHED_PREFILL) {
+                const int64_t x = alloc[t];
+                f[1] = x;
+                f[4] = x * run[t].ctx + x * (x + 1) / 2;
+                run[t].ctx += x;
+                run[t].pre -= x;
+                if (run[t].pre == 0 && mode == ORC_FIRST_TOKEN_WITH_LAST_CHUNK) {
+                    run[t].dec -= 1;
+                    if (run[t].is_query) done_q = 1;
+                }
+            } else if (kind[t] == SCHED_DECODE) {
+                f[2] = 1;
+                f[3] = run[t].ctx;
+                run[t].ctx += 1;
+                run[t].dec -= 1;
+                if (run[t].is_query) done_q = 1;
+            }
+            if (run[t].pre == 0 && run[t].ctx >= kv->max_ctx) run[t].dec = 0;  /* context limit */
+            for (int k = 1; k < 5; ++k) {
+                if (F) F[k] += f[k];
+                if (rf && !run[t].is_query) rf[k] += f[k];
+            }
+        }
+        if (with_query && done_q) {
+            if (l_admit) *l_admit = admitted_at;
+            if (l_ttft) *l_ttft = l;
+            rc = ORC_OK;
+            break;
+        }
+        if (!with_query && l == max_batches) {
+            rc = ORC_OK;
+            break;
+        }
+        /* 4. finished requests leave and free their blocks */
+        int64_t keep = 0;
+        for (int64_t t = 0; t < nr; ++t) {
+            if (run[t].dec > 0) run[keep++] = run[t];
+            else free_blocks += kv_blocks(run[t].ctx, bs);
+        }
+        nr = keep;
+    }
+done:
+    free(run); free(wait); free(alloc); free(kind);
+    return rc;
+}
+
+int orc_sfs_candidate_kv(const orc_instance *inst, int32_t B, int32_t S, int32_t mode, const orc_kv *kv,
+                         int32_t p, int32_t d, int64_t max_batches,
+                         int64_t F[5], int64_t *l_admit, int64_t *l_ttft, int64_t *res_F, int64_t *max_used)
+{
+    if (!F) return ORC_EINVAL;
+    return kv_sim(inst, B, S, mode, kv, 1, p, d, max_batches, F, l_admit, l_ttft, res_F, max_used);
+}
+
+int orc_kv_residents(const orc_instance *inst, int32_t B, int32_t S, int32_t mode, const orc_kv *kv,
+                     int64_t L, int64_t *res_F)
+{
+    if (L < 1 || !res_F) return ORC_EINVAL;
+    return kv_sim(inst, B, S, mode, kv, 0, 1, 1, L, NULL, NULL, NULL, res_F, NULL);
+}

@@ -40,6 +40,31 @@ int orc_sfs_candidate(const orc_instance *inst, int32_t B, int32_t S, int32_t mo
                       int32_t p, int32_t d, int64_t max_batches,
                       int64_t F[5], int64_t *l_admit, int64_t *l_ttft);
 
+/* KV-cache limits of one instance (App. F: "context limits, KV-cache allocation
+ * state, and preemption behavior"): block_size tokens per block, num_blocks blocks,
+ * and max_ctx, the longest context a request may reach. */
+typedef struct {
+    int32_t block_size;
+    int64_t num_blocks;
+    int64_t max_ctx;
+} orc_kv;
+
+/* orc_sfs_candidate with the KV-cache limits of `kv` (the step rule in sfs_oracle.c).
+ * If res_F is not NULL it receives, for each batch 1..l_ttft, the features of the
+ * batch without the query's own tokens ([l_ttft][5], room for max_batches rows);
+ * *max_used (may be NULL) receives the most blocks in use at the end of any batch's
+ * scheduling.  Returns ORC_EINVAL if the residents hold more blocks than the
+ * instance has, a context reaches max_ctx in the input, p >= max_ctx, or a request's
+ * whole context (capped at max_ctx) needs more blocks than the instance has. */
+int orc_sfs_candidate_kv(const orc_instance *inst, int32_t B, int32_t S, int32_t mode, const orc_kv *kv,
+                         int32_t p, int32_t d, int64_t max_batches,
+                         int64_t F[5], int64_t *l_admit, int64_t *l_ttft, int64_t *res_F, int64_t *max_used);
+
+/* The residents alone (no query) for exactly L batches under the same rule:
+ * res_F[L][5] per-batch features. */
+int orc_kv_residents(const orc_instance *inst, int32_t B, int32_t S, int32_t mode, const orc_kv *kv,
+                     int64_t L, int64_t *res_F);
+
 /* Canonical single-precision batch-time sum (Eq. 9 summed per Eq. 8) and its fp64 value. */
 float orc_ttft_f32(const float coef[5], const int64_t F[5]);
 double orc_ttft_f64(const float coef[5], const int64_t F[5]);

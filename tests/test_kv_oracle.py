@@ -1,0 +1,99 @@
+"""Pins of the oracle's KV-cache step rule (App. F: context limits, KV-cache
+allocation, preemption; the reading is stated in oracle/sfs_oracle.c).
+
+The rule is pinned against: the plain step rule when the limits cannot bind (an
+independent code path), a hand-worked trace with a preemption of the query
+(tests/golden/kv_hand_trace.json), a context limit that reduces to a shorter
+response, and the property the GPU design rests on: the residents' batches do not
+depend on the appended query, preemptions included.
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "kv_hand_trace.json")
+
+
+def random_pool(rng, max_run=12, max_wait=10):
+    S = int(rng.integers(2, 16))
+    B = int(rng.integers(S + 4, 200))
+    nr = int(rng.integers(0, min(S, max_run) + 1))
+    running = [(int(rng.integers(0, 300)), 0, int(rng.integers(1, 40))) for _ in range(nr)]
+    if nr and rng.random() < 0.3:  # the last running request still in prefill
+        c, _, d = running[-1]
+        running[-1] = (c, int(rng.integers(1, 150)), d)
+    waiting = [(int(rng.integers(1, 200)), int(rng.integers(1, 40))) for _ in range(int(rng.integers(0, max_wait + 1)))]
+    return B, S, running, waiting
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_unbounded_limits_reduce_to_the_plain_rule(mode):
+    rng = np.random.default_rng(100 + mode)
+    for _ in range(300):
+        B, S, running, waiting = random_pool(rng)
+        p, d = int(rng.integers(1, 300)), int(rng.integers(1, 30))
+        F0, la0, lt0 = oracle.simulate(running, waiting, B, S, p, d, mode=mode)
+        F, la, lt, _, _ = oracle.simulate_kv(running, waiting, B, S, p, d, block_size=16, num_blocks=1 << 40,
+                                             max_ctx=1 << 40, mode=mode)
+        np.testing.assert_array_equal(F, F0)
+        assert (la, lt) == (la0, lt0)
+
+
+def test_hand_trace_with_a_preemption_of_the_query():
+    g = json.load(open(GOLDEN))
+    F, la, lt, _, used = oracle.simulate_kv(g["running"], g["waiting"], g["B"], g["S"], *g["query"],
+                                            block_size=g["block_size"], num_blocks=g["num_blocks"],
+                                            max_ctx=g["max_ctx"], mode=g["mode"])
+    np.testing.assert_array_equal(F, g["F"])
+    assert la == g["admit_batch"] and lt == g["first_token_batch"] and used == g["most_blocks_in_use"]
+
+
+def test_context_limit_is_a_shorter_response():
+    # a decoder at context 60 under a limit of 62 decodes twice, exactly like one
+    # with two tokens left and no limit
+    for mode in (0, 1):
+        F, la, lt, _, _ = oracle.simulate_kv([(60, 0, 100), (5, 0, 9)], [(20, 4)], 16, 4, 30, 3, block_size=8,
+                                             num_blocks=1 << 20, max_ctx=62, mode=mode)
+        F0, la0, lt0 = oracle.simulate([(60, 0, 2), (5, 0, 9)], [(20, 4)], 16, 4, 30, 3, mode=mode)
+        np.testing.assert_array_equal(F, F0)
+        assert (la, lt) == (la0, lt0)
+
+
+def test_invalid_inputs():
+    with pytest.raises(RuntimeError):  # the query's prompt reaches the context limit
+        oracle.simulate_kv([], [], 16, 4, 64, 2, block_size=8, num_blocks=100, max_ctx=64)
+    with pytest.raises(RuntimeError):  # the query could never hold its whole context
+        oracle.simulate_kv([], [], 16, 4, 30, 20, block_size=8, num_blocks=6, max_ctx=1000)
+    with pytest.raises(RuntimeError):  # the residents hold more blocks than there are
+        oracle.simulate_kv([(40, 0, 3)], [], 16, 4, 5, 2, block_size=8, num_blocks=4, max_ctx=1000)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_residents_do_not_depend_on_the_query(mode):
+    # the residents' batches up to the query's first token are those of the residents
+    # alone, also when blocks run out and requests (the query included) are preempted
+    rng = np.random.default_rng(7 + mode)
+    binding = 0
+    n = 400
+    for _ in range(n):
+        B, S, running, waiting = random_pool(rng)
+        bs = int(rng.integers(1, 9))
+        p, d = int(rng.integers(1, 250)), int(rng.integers(1, 30))
+        held = sum((c + bs - 1) // bs for c, _, _ in running)
+        # enough blocks for any one request's whole context, few enough to bind
+        whole = [c + pr + dd for c, pr, dd in running] + [pr + dd for pr, dd in waiting] + [p + d]
+        nb = max(held + int(rng.integers(1, 40)), max((w + bs - 1) // bs for w in whole))
+        max_ctx = 1 << 20
+        F, la, lt, res, used = oracle.simulate_kv(running, waiting, B, S, p, d, block_size=bs, num_blocks=nb,
+                                                  max_ctx=max_ctx, mode=mode)
+        alone = oracle.kv_residents(running, waiting, B, S, lt, block_size=bs, num_blocks=nb, max_ctx=max_ctx,
+                                    mode=mode)
+        np.testing.assert_array_equal(res, alone)
+        assert used <= nb
+        F0, _, lt0 = oracle.simulate(running, waiting, B, S, p, d, mode=mode)
+        binding += int(lt != lt0 or not np.array_equal(F, F0))
+    assert binding >= n // 4  # the limits bind in a good share of the cases
