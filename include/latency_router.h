@@ -224,6 +224,35 @@ LR_API int lr_set_queue_params(lr_ctx *ctx, const lr_queue_params *params, void 
  * (LR_ENOSTATE before one is loaded); the LPS source reads none. */
 LR_API int lr_set_ttft_source(lr_ctx *ctx, int32_t source);
 
+/* KV-cache limits in the simulated step rule (App. F: the simulation accounts for
+ * "context limits, KV-cache allocation state, and preemption behavior").  Reading:
+ * instance j has num_blocks[j] blocks of block_size[j] tokens, a request with c
+ * tokens in the cache holds ceil(c / block_size) of them; a running request whose
+ * tokens of a batch need blocks that are not free preempts the last running request
+ * (its blocks return, its whole context becomes prefill again and it goes to the
+ * front of the waiting queue), preempting itself if it is the last; the waiting
+ * head is admitted only if its first chunk's blocks are free; a request whose
+ * context reaches max_ctx[j] ends there.  The query appended at the waiting tail
+ * never changes the residents' batches, so every later lr_load_state simulates
+ * each instance's residents once, recording up to `horizon` batches from the first
+ * one in which a query could be admitted, and lr_estimate_ttft /
+ * lr_estimate_features follow each query through those records.
+ * block_size [I] int32 in [1, 2^20], num_blocks [I] int64 in [1, 2^40], max_ctx [I]
+ * int64 in [2, 2^40]: host arrays, copied.  horizon in [1, 2^16].  All three arrays
+ * NULL turns the limits off (the default).  The call synchronizes the device and drops
+ * the live snapshot: estimates return LR_ENOSTATE until the next lr_load_state.
+ * With limits on, lr_route, lr_route_frontier_static, the average-case sources and
+ * lr_advance return LR_EINVAL (lr_route_baseline reads only queue lengths and stays
+ * open).  Device errors: a snapshot in which a running request other than the last is
+ * in prefill, a context has reached max_ctx, the residents hold more blocks than the
+ * instance has, or a request's whole context (capped at max_ctx) needs more blocks than
+ * the instance has, is LR_ESTATE; a query whose prompt is not below max_ctx, or whose
+ * prompt and first token need more blocks than the instance has, gets NaN (features -1)
+ * and LR_EINVAL; one that needs batches past the recorded horizon gets NaN and
+ * LR_ETRAJ. */
+LR_API int lr_set_kv_limits(lr_ctx *ctx, const int32_t *block_size, const int64_t *num_blocks,
+                            const int64_t *max_ctx, int32_t horizon);
+
 /* Least-squares calibration of the Eq. 9 coefficients per model from a log of executed
  * token batches (Sec. 4.1: calibrated from observed token-batch processing times).
  * features: [N][5] int64 device, each batch's (F0 = 1, prefill tokens, decode tokens, sum of

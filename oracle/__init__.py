@@ -87,6 +87,9 @@ def _load():
         lib.orc_sfs_candidate_kv.restype = ctypes.c_int
         lib.orc_kv_residents.argtypes = [P, i32, i32, i32, P, i64, P]
         lib.orc_kv_residents.restype = ctypes.c_int
+        lib.orc_estimate_candidates_kv.argtypes = [i32, P, P, P, P, i32, i32, P, P, P, P, P, P, P, P, P, P, P,
+                                                   i32, i64, i64, P, P, P, P, P, P, P]
+        lib.orc_estimate_candidates_kv.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -415,3 +418,40 @@ def kv_residents(running, waiting, B: int, S: int, L: int, block_size: int, num_
     if rc != 0:
         raise RuntimeError(f"oracle KV residents failed with code {rc}")
     return res
+
+
+def estimate_matrix_kv(wl, block_size, num_blocks, max_ctx, max_batches: int = DEFAULT_MAX_BATCHES,
+                       cand_q=None, cand_j=None):
+    """Every candidate (or the listed ones) under per-instance KV limits, the query taken
+    up to its first token.  Returns status, F[...,5], first-token batch, fp32, fp64
+    ([Q,I] shapes for the full matrix, [C] for a list); failed candidates carry F = -1,
+    batch -1 and NaN times."""
+    Q, I = wl.num_queries, wl.num_instances
+    full = cand_q is None
+    if full:
+        qq, jj = np.meshgrid(np.arange(Q), np.arange(I), indexing="ij")
+        cand_q, cand_j = qq.ravel(), jj.ravel()
+    cq, cj = _c(cand_q, np.int32), _c(cand_j, np.int32)
+    C = cq.shape[0]
+    st = np.zeros(C, np.int32)
+    F = np.zeros((C, 5), np.int64)
+    lt = np.zeros(C, np.int64)
+    t32 = np.zeros(C, np.float32)
+    t64 = np.zeros(C, np.float64)
+    arrs = [_c(a, np.int32) for a in (wl.model_of_instance, wl.max_batched_tokens, wl.max_seqs, wl.n_run,
+                                      wl.run_ctx, wl.run_pre, wl.run_dec, wl.n_wait, wl.wait_pre,
+                                      wl.wait_dec, wl.prompt_len)]
+    moi, B, S, n_run, run_ctx, run_pre, run_dec, n_wait, wait_pre, wait_dec, p = arrs
+    bs = _c(np.broadcast_to(np.asarray(block_size, np.int32), (I,)), np.int32)
+    nb = _c(np.broadcast_to(np.asarray(num_blocks, np.int64), (I,)), np.int64)
+    mc = _c(np.broadcast_to(np.asarray(max_ctx, np.int64), (I,)), np.int64)
+    coef = _c(wl.coef, np.float32)
+    rc = _load().orc_estimate_candidates_kv(
+        I, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running, wl.cap_waiting, _p(n_run), _p(run_ctx), _p(run_pre),
+        _p(run_dec), _p(n_wait), _p(wait_pre), _p(wait_dec), _p(p), _p(bs), _p(nb), _p(mc), wl.first_token_mode,
+        max_batches, C, _p(cq), _p(cj), _p(st), _p(F), _p(lt), _p(t32), _p(t64))
+    if rc != 0:
+        raise RuntimeError(f"oracle KV estimate failed with code {rc}")
+    if full:
+        return st.reshape(Q, I), F.reshape(Q, I, 5), lt.reshape(Q, I), t32.reshape(Q, I), t64.reshape(Q, I)
+    return st, F, lt, t32, t64

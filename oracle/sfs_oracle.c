@@ -168,6 +168,48 @@ float orc_ttft_f32(const float coef[5], const int64_t F[5])
     return t;
 }
 
+int orc_estimate_candidates_kv(int32_t num_instances, const int32_t *model_of_instance,
+                               const float *coef, const int32_t *B, const int32_t *S,
+                               int32_t cap_running, int32_t cap_waiting,
+                               const int32_t *n_run, const int32_t *run_ctx, const int32_t *run_pre,
+                               const int32_t *run_dec, const int32_t *n_wait, const int32_t *wait_pre,
+                               const int32_t *wait_dec, const int32_t *prompt_len,
+                               const int32_t *block_size, const int64_t *num_blocks, const int64_t *max_ctx,
+                               int32_t mode, int64_t max_batches,
+                               int64_t num_cand, const int32_t *cand_q, const int32_t *cand_j,
+                               int32_t *status, int64_t *F, int64_t *l_ttft, float *ttft32, double *ttft64)
+{
+    for (int64_t c = 0; c < num_cand; ++c) {
+        const int32_t i = cand_q[c], j = cand_j[c];
+        if (j < 0 || j >= num_instances) return ORC_EINVAL;
+        orc_instance inst;
+        inst.n_run = n_run[j];
+        inst.run_ctx = run_ctx + (int64_t)j * cap_running;
+        inst.run_pre = run_pre + (int64_t)j * cap_running;
+        inst.run_dec = run_dec + (int64_t)j * cap_running;
+        inst.n_wait = n_wait[j];
+        inst.wait_pre = wait_pre + (int64_t)j * cap_waiting;
+        inst.wait_dec = wait_dec + (int64_t)j * cap_waiting;
+        if (inst.n_run > cap_running || inst.n_wait > cap_waiting) return ORC_EINVAL;
+        const orc_kv kv = {block_size[j], num_blocks[j], max_ctx[j]};
+        int64_t Fc[5] = {-1, -1, -1, -1, -1}, la = 0, lt = -1;
+        /* the query up to its first token: one output token */
+        const int rc = orc_sfs_candidate_kv(&inst, B[j], S[j], mode, &kv, prompt_len[i], 1, max_batches, Fc, &la,
+                                            &lt, NULL, NULL);
+        status[c] = rc;
+        if (rc != ORC_OK) {
+            for (int k = 0; k < 5; ++k) Fc[k] = -1;
+            lt = -1;
+        }
+        for (int k = 0; k < 5; ++k) F[c * 5 + k] = Fc[k];
+        if (l_ttft) l_ttft[c] = lt;
+        const float *cf = coef + 5 * model_of_instance[j];
+        if (ttft32) ttft32[c] = rc == ORC_OK ? orc_ttft_f32(cf, Fc) : NAN;
+        if (ttft64) ttft64[c] = rc == ORC_OK ? orc_ttft_f64(cf, Fc) : NAN;
+    }
+    return ORC_OK;
+}
+
 double orc_ttft_f64(const float coef[5], const int64_t F[5])
 {
     return (double)coef[0] * (double)F[0] + (double)coef[1] * (double)F[1] +

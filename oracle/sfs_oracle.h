@@ -65,6 +65,22 @@ int orc_sfs_candidate_kv(const orc_instance *inst, int32_t B, int32_t S, int32_t
 int orc_kv_residents(const orc_instance *inst, int32_t B, int32_t S, int32_t mode, const orc_kv *kv,
                      int64_t L, int64_t *res_F);
 
+/* Every candidate of a list under per-instance KV limits, the query taken up to its
+ * first token (one output token).  status[c] receives the candidate's return code
+ * (ORC_OK, ORC_EINVAL for an invalid snapshot or query, ORC_ELIMIT past max_batches);
+ * a failed candidate gets F = -1, l_ttft = -1 and NaN times.  Returns ORC_EINVAL only
+ * for a bad candidate index or row count. */
+int orc_estimate_candidates_kv(int32_t num_instances, const int32_t *model_of_instance,
+                               const float *coef, const int32_t *B, const int32_t *S,
+                               int32_t cap_running, int32_t cap_waiting,
+                               const int32_t *n_run, const int32_t *run_ctx, const int32_t *run_pre,
+                               const int32_t *run_dec, const int32_t *n_wait, const int32_t *wait_pre,
+                               const int32_t *wait_dec, const int32_t *prompt_len,
+                               const int32_t *block_size, const int64_t *num_blocks, const int64_t *max_ctx,
+                               int32_t mode, int64_t max_batches,
+                               int64_t num_cand, const int32_t *cand_q, const int32_t *cand_j,
+                               int32_t *status, int64_t *F, int64_t *l_ttft, float *ttft32, double *ttft64);
+
 /* Canonical single-precision batch-time sum (Eq. 9 summed per Eq. 8) and its fp64 value. */
 float orc_ttft_f32(const float coef[5], const int64_t F[5]);
 double orc_ttft_f64(const float coef[5], const int64_t F[5]);

@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "liblr.so")
-SOURCES = ["lr_api.cu", "lr_trajectory.cu", "lr_estimate.cu", "lr_advance.cu", "lr_calibrate.cu"]
+SOURCES = ["lr_api.cu", "lr_trajectory.cu", "lr_estimate.cu", "lr_advance.cu", "lr_calibrate.cu", "lr_kv.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-std=c++17", "-O3", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
               "--expt-relaxed-constexpr"]

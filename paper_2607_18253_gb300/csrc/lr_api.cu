@@ -35,6 +35,13 @@ struct lr_ctx {
     unsigned long long *cal_acc = nullptr;  // calibration sums [M][kCalAcc][2] (128-bit)
     int source = lr::kSrcSfs;
     bool have_qp = false, have_lps = false;
+    // KV-cache limits (lr_set_kv_limits): per-instance arrays, the records of both
+    // buffers, and the load's launch shape
+    bool kv_on = false;
+    lr::KvLimits kv{};
+    int kv_warps = 0;
+    size_t kv_smem = 0;
+    std::vector<void *> kv_allocs;
     std::vector<void *> allocs;
     std::string err;
     int max_queries = 0, max_pairs = 0;
@@ -83,7 +90,19 @@ int round_up(int x, int m) { return ((x + m - 1) / m) * m; }
 
 bool finite_nonneg(float v) { return std::isfinite(v) && v >= 0.0f; }
 
+void free_kv(lr_ctx *c) {
+    for (void *p : c->kv_allocs) cudaFree(p);
+    c->kv_allocs.clear();
+    c->kv = lr::KvLimits{};
+    c->kv_on = false;
+    for (int b = 0; b < 2; ++b) {
+        c->buf[b].kvi = nullptr;
+        c->buf[b].kvr = nullptr;
+    }
+}
+
 void free_all(lr_ctx *c) {
+    free_kv(c);
     for (void *p : c->allocs) cudaFree(p);
     c->allocs.clear();
 }
@@ -344,6 +363,22 @@ int lr_load_state(lr_ctx *c, const lr_state_view *v, void *stream) {
     c->err.clear();
     if (!v || !v->n_run || !v->run_ctx || !v->run_pre || !v->run_dec || !v->n_wait || !v->wait_pre || !v->wait_dec)
         return fail(c, LR_EINVAL, "null snapshot array");
+    if (c->kv_on) {
+        lr::KvLoad k;
+        std::memset(&k, 0, sizeof(k));
+        k.cfg = c->cfg;
+        k.kv = c->kv;
+        k.buf0 = c->buf[0];
+        k.buf1 = c->buf[1];
+        k.ctl = c->ctl;
+        k.in = lr::StateIn{v->n_run, v->run_ctx, v->run_pre, v->run_dec, v->n_wait, v->wait_pre, v->wait_dec, nullptr};
+        const int grid = (c->cfg.I + c->kv_warps - 1) / c->kv_warps;
+        cudaError_t e = lr::launch_kv_load(k, grid, c->kv_warps, c->kv_smem, (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(c, e, "KV load launch");
+        c->load_stream = stream;
+        c->loaded_any = true;
+        return LR_OK;
+    }
     lr::K1Launch a;
     std::memset(&a, 0, sizeof(a));
     a.cfg = c->cfg;
@@ -369,6 +404,22 @@ static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, 
     if (!p || (!ttft && !feat)) return fail(c, LR_EINVAL, "null array");
     if (iters && c->source != lr::kSrcSfs)
         return fail(c, LR_EINVAL, "first_batch_out exists only for the SFS source");
+    if (c->kv_on) {
+        lr::KvEst k;
+        std::memset(&k, 0, sizeof(k));
+        k.cfg = c->cfg;
+        k.kv = c->kv;
+        k.buf0 = c->buf[0];
+        k.buf1 = c->buf[1];
+        k.ctl = c->ctl;
+        k.Q = Q;
+        k.prompt = p;
+        k.ttft = ttft;
+        k.first_batch = iters;
+        k.features = reinterpret_cast<long long *>(feat);
+        cudaError_t e = lr::launch_kv_estimate(k, c->sms, (cudaStream_t)stream);
+        return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "KV estimate launch");
+    }
     lr::K2Launch a = k2_base(c);
     a.Q = Q;
     a.prompt = p;
@@ -411,6 +462,7 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
     if (Q > c->max_queries) return fail(c, LR_ECAPACITY, "Q exceeds max_queries");
     if (P < 1) return fail(c, LR_EINVAL, "P < 1");
     if (P > c->max_pairs) return fail(c, LR_ECAPACITY, "P exceeds max_pairs");
+    if (c->kv_on) return fail(c, LR_EINVAL, "routing with KV-cache limits is not supported");
     if (!c->rt.ok) return fail(c, LR_ECAPACITY, "routing needs num_instances <= 1024 and its tiles in shared memory");
     if (!lambda || (!tau && !mu)) return fail(c, LR_EINVAL, "null lambda / mu");
     if (tau && P != 1) return fail(c, LR_EINVAL, "the constrained objective takes one lambda (P == 1)");
@@ -582,9 +634,79 @@ int lr_set_ttft_source(lr_ctx *c, int32_t source) {
     c->err.clear();
     if (source != LR_TTFT_SFS && source != LR_TTFT_THROUGHPUT && source != LR_TTFT_LPS)
         return fail(c, LR_EINVAL, "unknown TTFT source");
+    if (source != LR_TTFT_SFS && c->kv_on) return fail(c, LR_EINVAL, "KV-cache limits apply to the SFS source only");
     if (source != LR_TTFT_SFS && !c->have_qp) return fail(c, LR_EINVAL, "set the queue parameters first");
     if (source == LR_TTFT_LPS && !c->have_lps) return fail(c, LR_EINVAL, "the LPS source needs arrival and service rates");
     c->source = source;
+    return LR_OK;
+}
+
+int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_blocks, const int64_t *max_ctx,
+                     int32_t horizon) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    const bool on = block_size || num_blocks || max_ctx;
+    if (on && !(block_size && num_blocks && max_ctx)) return fail(c, LR_EINVAL, "pass all three arrays or none");
+    const int I = c->cfg.I;
+    if (on) {
+        if (horizon < 1 || horizon > (1 << 16)) return fail(c, LR_EINVAL, "horizon must be in [1, 2^16]");
+        if (c->source != lr::kSrcSfs) return fail(c, LR_EINVAL, "KV-cache limits apply to the SFS source only");
+        for (int j = 0; j < I; ++j) {
+            if (block_size[j] < 1 || block_size[j] > (1 << 20)) return fail(c, LR_EINVAL, "block_size out of range");
+            if (num_blocks[j] < 1 || num_blocks[j] > (1LL << 40)) return fail(c, LR_EINVAL, "num_blocks out of range");
+            if (max_ctx[j] < 2 || max_ctx[j] > (1LL << 40)) return fail(c, LR_EINVAL, "max_ctx out of range");
+        }
+    }
+    const size_t per_warp = lr::kv_smem_per_warp(c->cfg);
+    if (on && per_warp > 200 * 1024) return fail(c, LR_ECAPACITY, "snapshot capacities too large for one KV-load warp");
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(c, e, "synchronize");
+    free_kv(c);
+    // the live snapshot was summarized for the previous rule
+    const int32_t none = -1;
+    e = cudaMemcpy(&c->ctl->active, &none, sizeof(none), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(c, e, "snapshot reset");
+    if (!on) return LR_OK;
+    int warps = lr::kKvWarps;
+    while (warps > 1 && warps * per_warp > 200 * 1024) --warps;
+    e = lr::set_kv_smem(warps * per_warp);
+    if (e != cudaSuccess) return cuda_fail(c, e, "KV load shared memory");
+    auto alloc = [&](size_t bytes, void **p) {
+        cudaError_t ee = cudaMalloc(p, bytes > 0 ? bytes : 16);
+        if (ee == cudaSuccess) c->kv_allocs.push_back(*p);
+        return ee;
+    };
+    void *bs = nullptr, *nb = nullptr, *mc = nullptr, *kvi[2] = {nullptr, nullptr}, *kvr[2] = {nullptr, nullptr};
+    e = alloc(sizeof(int32_t) * I, &bs);
+    if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &nb);
+    if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &mc);
+    for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+        e = alloc(sizeof(lr::KvInst) * I, &kvi[b]);
+        if (e == cudaSuccess) e = alloc(sizeof(lr::KvRec) * (size_t)I * horizon, &kvr[b]);
+    }
+    if (e != cudaSuccess) {
+        free_kv(c);
+        return fail(c, LR_ENOMEM, cudaGetErrorString(e));
+    }
+    e = cudaMemcpy(bs, block_size, sizeof(int32_t) * I, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(nb, num_blocks, sizeof(long long) * I, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(mc, max_ctx, sizeof(long long) * I, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) {
+        free_kv(c);
+        return cuda_fail(c, e, "KV limits upload");
+    }
+    c->kv.bs = static_cast<const int32_t *>(bs);
+    c->kv.nb = static_cast<const long long *>(nb);
+    c->kv.mctx = static_cast<const long long *>(mc);
+    c->kv.horizon = horizon;
+    c->kv.on = 1;
+    for (int b = 0; b < 2; ++b) {
+        c->buf[b].kvi = static_cast<lr::KvInst *>(kvi[b]);
+        c->buf[b].kvr = static_cast<lr::KvRec *>(kvr[b]);
+    }
+    c->kv_warps = warps;
+    c->kv_smem = warps * per_warp;
+    c->kv_on = true;
     return LR_OK;
 }
 
@@ -609,6 +731,7 @@ int lr_advance(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_t *promp
     if (Q > 0 && (!assign || !prompt_len || !dec)) return fail(c, LR_EINVAL, "null array");
     if (dec_cols != 1 && dec_cols != c->cfg.M) return fail(c, LR_EINVAL, "dec_cols must be 1 or num_models");
     if (!std::isfinite(t_now)) return fail(c, LR_EINVAL, "t_now must be finite");
+    if (c->kv_on) return fail(c, LR_EINVAL, "advancing with KV-cache limits is not supported");
     if (c->cfg.capR < c->max_seqs) return fail(c, LR_ECAPACITY, "advancing needs cap_running >= every max_seqs");
     if (c->k3_smem > 200 * 1024) return fail(c, LR_ECAPACITY, "queue capacities too large for one advance warp");
     lr::K3Launch k;

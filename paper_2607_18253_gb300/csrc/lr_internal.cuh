@@ -51,6 +51,33 @@ struct DevConfig {
     const float *coef, *pin, *pout;
 };
 
+// KV-limited simulation (App. F): one batch of an instance's residents alone, from
+// the first batch in which a query could be admitted (the waiting queue empty after
+// admissions, budget and a seat left).  64 bytes.
+struct __align__(16) KvRec {
+    long long f3, f4;       // residents' decode contexts and prefill attention pairs
+    int32_t f1, f2;         // residents' prefill and decode tokens
+    int32_t bar, bl;        // budget left after the running scan, after admissions
+    int32_t seats, flags;   // free seats after admissions; bit 0: waiting queue empty
+    long long slack;        // least (free blocks - blocks needed) over the running scan
+    long long far, fa;      // free blocks after the running scan, after admissions
+};
+// Per instance: the residents' features before the first record, and the records' extent.
+struct __align__(16) KvInst {
+    long long fcum[5];
+    int32_t la0;   // batch of record 0
+    int32_t nrec;  // records written
+    int32_t done;  // 1: no resident is left after the last record (later batches are empty)
+    int32_t pad;
+};
+struct KvLimits {
+    const int32_t *bs;     // [I] block size (tokens)
+    const long long *nb;   // [I] blocks
+    const long long *mctx; // [I] context limit
+    int32_t horizon;       // records per instance
+    int32_t on;
+};
+
 struct StateBuf {
     int32_t *n_run, *run_ctx, *run_pre, *run_dec, *n_wait, *wait_pre, *wait_dec;
     double *clock;  // [I] end time of the instance's last completed batch (s)
@@ -59,6 +86,8 @@ struct StateBuf {
     unsigned char *tile;  // candidate-kernel tile blocks
     long long *f2, *f3;
     int32_t *rcum;
+    KvInst *kvi;  // [I], with KV limits
+    KvRec *kvr;   // [I][horizon], with KV limits
 };
 
 struct DevCtl {
@@ -147,6 +176,36 @@ struct K1Launch {
 cudaError_t launch_trajectory(const K1Launch &a, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t set_k1_smem(size_t bytes);
 constexpr int kK1Warps = 4;
+
+// KV-limited load (residents alone, records) and estimate (per-candidate walk).
+struct KvLoad {
+    DevConfig cfg;
+    KvLimits kv;
+    StateBuf buf0, buf1;
+    DevCtl *ctl;
+    StateIn in;
+};
+constexpr int kKvWarps = 4;
+// shared memory per warp of the KV load: running (ctx, pre, dec, chunk) and the waiting
+// ring (pre, dec) over capR + capW requests
+__host__ __device__ inline size_t kv_smem_per_warp(const DevConfig &c) {
+    return sizeof(int32_t) * 6 * (size_t)(c.capR + c.capW) + 64;
+}
+// warps: instances per CTA, 1 .. kKvWarps
+cudaError_t launch_kv_load(const KvLoad &a, int grid, int warps, size_t smem, cudaStream_t st);
+cudaError_t set_kv_smem(size_t bytes);
+struct KvEst {
+    DevConfig cfg;
+    KvLimits kv;
+    StateBuf buf0, buf1;
+    DevCtl *ctl;
+    int32_t Q;
+    const int32_t *prompt;
+    float *ttft;
+    int32_t *first_batch;
+    long long *features;
+};
+cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st);
 
 // Batches covered by K1's completion calendar; decoders ending later are
 // tracked by scanning the decoder list.

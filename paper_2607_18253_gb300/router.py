@@ -26,7 +26,7 @@ LR_POLICY_ROUND_ROBIN, LR_POLICY_SHORTEST_QUEUE, LR_POLICY_LATENCY_AGNOSTIC = 0,
 EXPORTED_SYMBOLS = ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
                     "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
                     "lr_set_queue_params", "lr_set_ttft_source", "lr_calibrate", "lr_route_baseline",
-                    "lr_on_time_utility", "lr_strerror", "lr_last_error")
+                    "lr_on_time_utility", "lr_set_kv_limits", "lr_strerror", "lr_last_error")
 
 _P = ctypes.c_void_p
 _I32 = ctypes.c_int32
@@ -73,6 +73,7 @@ def load_library(path: str = LIB_PATH):
     lib.lr_calibrate.argtypes = [_P, ctypes.c_int64, _P, _P, _P, _I32, _P, _P]
     lib.lr_route_baseline.argtypes = [_P, _I32, _I32, _P, _P, _P, ctypes.c_float, ctypes.c_int64, _P, _P, _P, _P]
     lib.lr_on_time_utility.argtypes = [_P, _I32, _P, _P, _P, _P, _P, _P]
+    lib.lr_set_kv_limits.argtypes = [_P, _P, _P, _P, _I32]
     lib.lr_read_state.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.lr_status.argtypes = [_P, _P]
     lib.lr_strerror.argtypes = [ctypes.c_int]
@@ -82,7 +83,7 @@ def load_library(path: str = LIB_PATH):
     for name in ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
                  "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
                  "lr_set_queue_params", "lr_set_ttft_source", "lr_calibrate", "lr_route_baseline",
-                 "lr_on_time_utility"):
+                 "lr_on_time_utility", "lr_set_kv_limits"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -304,6 +305,19 @@ class LatencyRouter:
     def set_ttft_source(self, source: int):
         """LR_TTFT_SFS (default), LR_TTFT_THROUGHPUT or LR_TTFT_LPS."""
         self._check(self._lib.lr_set_ttft_source(self._h, int(source)), "lr_set_ttft_source")
+
+    def set_kv_limits(self, block_size=None, num_blocks=None, max_ctx=None, horizon: int = 4096):
+        """KV-cache block limits, context limits and preemption in the simulated step rule
+        (host arrays of length I, or scalars for every instance); all None turns them off.
+        Drops the live snapshot: load one again before estimating."""
+        I = self.num_instances
+        if block_size is None and num_blocks is None and max_ctx is None:
+            self._check(self._lib.lr_set_kv_limits(self._h, None, None, None, 0), "lr_set_kv_limits")
+            return
+        keep = [np.ascontiguousarray(np.broadcast_to(np.asarray(x, dt), (I,)))
+                for x, dt in ((block_size, np.int32), (num_blocks, np.int64), (max_ctx, np.int64))]
+        self._check(self._lib.lr_set_kv_limits(self._h, *(k.ctypes.data_as(_P) for k in keep), int(horizon)),
+                    "lr_set_kv_limits")
 
     def calibrate(self, features: torch.Tensor, model: torch.Tensor, time: torch.Tensor, shared_beta1: bool = True,
                   out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:

@@ -299,6 +299,44 @@ def batch_log(num_batches: int, num_models: int, seed: int, coef: np.ndarray, no
     return F, mdl.astype(np.int32), t
 
 
+def kv_limits(wl: Workload, seed: int, block_sizes=(16,), tightness=(0.3, 1.0), ctx_limited: float = 0.5,
+              ctx_slack=(1, 64), unlimited: int = 1 << 40):
+    """Seeded per-instance KV-cache limits for a workload's snapshot: block sizes drawn
+    from `block_sizes`; a context limit on a `ctx_limited` share of the instances, just
+    above the longest context any request or query already needs (so that decoding runs
+    into it), else `unlimited`; and a block count that a `tightness` draw places between
+    the most any single request (or the first token of the longest query) can need and
+    the residents' whole demand, never below the blocks the running requests hold.
+    Returns (block_size [I] int32, num_blocks [I] int64, max_ctx [I] int64).  Token
+    counts are turned into blocks by the bound tokens // bs + 1 >= ceil(tokens / bs)."""
+    rng = np.random.default_rng(seed)
+    I = wl.num_instances
+    bs = rng.choice(np.asarray(block_sizes, np.int64), I).astype(np.int32)
+    nb = np.zeros(I, np.int64)
+    mctx = np.zeros(I, np.int64)
+    for j in range(I):
+        b = int(bs[j])
+        nr, nw = int(wl.n_run[j]), int(wl.n_wait[j])
+        ctx = wl.run_ctx[j, :nr].astype(np.int64)
+        pre = wl.run_pre[j, :nr].astype(np.int64)
+        dec = wl.run_dec[j, :nr].astype(np.int64)
+        wpre = wl.wait_pre[j, :nw].astype(np.int64)
+        wdec = wl.wait_dec[j, :nw].astype(np.int64)
+        lo = max([wl.max_prompt_len] + list(ctx + pre) + list(wpre)) + 1
+        if rng.random() < ctx_limited:
+            mctx[j] = lo + int(rng.integers(ctx_slack[0], ctx_slack[1] + 1))
+        else:
+            mctx[j] = unlimited
+        whole = np.concatenate([np.minimum(ctx + pre + dec, mctx[j]), np.minimum(wpre + wdec, mctx[j]),
+                                [min(wl.max_prompt_len + 1, int(mctx[j]))]])
+        one = int((whole // b + 1).max())
+        held = int((ctx // b + 1).sum())
+        demand = int((whole // b + 1).sum())
+        u = rng.uniform(*tightness)
+        nb[j] = max(one, held, int(one + u * (demand - one)))
+    return bs, nb, mctx
+
+
 def sweep_pairs():
     """The trade-off grid: 4 lambda values (log 0.1..10) x 8 mu values (log 0.01..1 /s), lambda-major."""
     lam = np.logspace(-1, 1, 4)

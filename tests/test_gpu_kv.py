@@ -1,0 +1,224 @@
+"""KV-cache block limits, context limits and preemption in the SFS estimate (App. F):
+CUDA path vs the CPU oracle, through the C ABI.
+
+Features and first-token batches match exactly and times bit for bit (both sides
+take the canonical fp32 sum of the same integer features).  Candidates the oracle
+rejects (a prompt at the context limit, a first token that cannot fit) are NaN with
+features -1 and the status word reads LR_EINVAL; queries that need more batches than
+the recorded horizon are NaN with LR_ETRAJ.
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import oracle  # noqa: E402
+from paper_2607_18253_gb300 import workloads as W  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+def R():
+    from paper_2607_18253_gb300 import router
+    return router
+
+
+def bits(a):
+    return np.ascontiguousarray(a, np.float32).view(np.uint32)
+
+
+def make(wl, limits, horizon=4096, load=True, **kw):
+    rt = R().LatencyRouter.from_workload(wl, **kw)
+    rt.set_kv_limits(*limits, horizon=horizon)
+    if load:
+        rt.load_state(*R().state_tensors(wl))
+    return rt
+
+
+def gpu_estimate(rt, wl):
+    p = torch.from_numpy(np.ascontiguousarray(wl.prompt_len, np.int32)).cuda()
+    fb = torch.empty((wl.num_queries, wl.num_instances), dtype=torch.int32, device="cuda")
+    t = rt.estimate_ttft(p, first_batch=fb)
+    F = rt.estimate_features(p)
+    torch.cuda.synchronize()
+    return t.cpu().numpy(), fb.cpu().numpy(), F.cpu().numpy()
+
+
+def compare(got, want, ok):
+    t, fb, F = got
+    eF, elt, et = want
+    np.testing.assert_array_equal(F[ok], eF[ok])
+    np.testing.assert_array_equal(fb[ok], elt[ok])
+    np.testing.assert_array_equal(bits(t[ok]), bits(et[ok]))
+
+
+def check(wl, limits, horizon=4096):
+    rt = make(wl, limits, horizon)
+    got = gpu_estimate(rt, wl)
+    st, eF, elt, et, _ = oracle.estimate_matrix_kv(wl, *limits)
+    ok = st == 0
+    compare(got, (eF, elt, et), ok)
+    t, fb, F = got
+    assert np.isnan(t[~ok]).all() and (fb[~ok] == -1).all() and (F[~ok] == -1).all()
+    assert rt.status() == (R().LR_OK if ok.all() else R().LR_EINVAL)
+    rt.close()
+    return st, eF
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_small_pools(mode):
+    binding = 0
+    for seed in range(8):
+        I = (1, 3, 6, 17, 33, 64, 5, 100)[seed]
+        wl = W.small_workload(seed, num_instances=I, num_models=3, num_queries=45, first_token_mode=mode,
+                              budget_range=(8, 96), min_gap=8)
+        limits = W.kv_limits(wl, 100 + seed, block_sizes=(1, 4, 16))
+        st, eF = check(wl, limits)
+        F0 = oracle.estimate_matrix(wl)[0]
+        binding += int((eF != F0).any(axis=-1).sum())
+    assert binding > 0
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_tight_blocks_and_context_limits(mode):
+    # every instance near its least block count, most with a context limit that
+    # decoding runs into: preemptions and limit-ended responses throughout
+    for seed in range(4):
+        wl = W.small_workload(20 + seed, num_instances=24, num_models=2, num_queries=40, first_token_mode=mode,
+                              cap_running=16, cap_waiting=24, budget_range=(16, 128), min_gap=8)
+        limits = W.kv_limits(wl, 200 + seed, block_sizes=(1, 2, 8), tightness=(0.0, 0.2), ctx_limited=0.8,
+                             ctx_slack=(1, 12))
+        check(wl, limits)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_unbounded_limits_give_the_plain_estimate(mode):
+    wl = W.small_workload(31 + mode, num_instances=40, num_models=3, num_queries=64, first_token_mode=mode,
+                          budget_range=(8, 96), min_gap=8)
+    I = wl.num_instances
+    limits = (np.full(I, 16, np.int32), np.full(I, 1 << 40, np.int64), np.full(I, 1 << 40, np.int64))
+    rt = make(wl, limits)
+    got = gpu_estimate(rt, wl)
+    assert rt.status() == R().LR_OK
+    rt.close()
+    plain = R().LatencyRouter.from_workload(wl)
+    plain.load_state(*R().state_tensors(wl))
+    ref = gpu_estimate(plain, wl)
+    plain.close()
+    for a, b in zip(got, ref):
+        np.testing.assert_array_equal(np.asarray(a).view(np.uint8), np.asarray(b).view(np.uint8))
+    F0, lt0, t0, _ = oracle.estimate_matrix(wl)
+    compare(got, (F0, lt0, t0), np.ones(lt0.shape, bool))
+
+
+def test_invalid_queries_are_nan():
+    # an idle instance whose context limit some prompts reach, and one whose blocks
+    # cannot hold some prompts' first token
+    wl = W.small_workload(61, num_instances=5, num_models=2, num_queries=50, budget_range=(8, 96), min_gap=8)
+    bs, nb, mc = W.kv_limits(wl, 7, block_sizes=(4,))
+    for j in (0, 1):
+        wl.n_run[j] = 0
+        wl.n_wait[j] = 0
+    med = int(np.median(wl.prompt_len))
+    mc[0] = med
+    nb[1] = med // 4
+    st, _ = check(wl, (bs, nb, mc))
+    assert (st[:, 0] != 0).any() and (st[:, 1] != 0).any() and (st[:, 2:] == 0).all()
+
+
+def test_horizon_exceeded():
+    wl = W.small_workload(62, num_instances=12, num_models=2, num_queries=30, budget_range=(8, 48), min_gap=8)
+    limits = W.kv_limits(wl, 8, block_sizes=(4,))
+    rt = make(wl, limits, horizon=2)
+    t, fb, F = gpu_estimate(rt, wl)
+    st, eF, elt, et, _ = oracle.estimate_matrix_kv(wl, *limits)
+    assert (st == 0).all()
+    cut = np.isnan(t)
+    assert cut.any() and (~cut).any()
+    compare((t, fb, F), (eF, elt, et), ~cut)
+    assert (fb[cut] == -1).all() and (F[cut] == -1).all()
+    assert rt.status() == R().LR_ETRAJ
+    rt.close()
+
+
+def test_invalid_snapshot_keeps_the_live_one():
+    wl = W.small_workload(63, num_instances=9, num_models=2, num_queries=20, budget_range=(8, 96), min_gap=8)
+    bs, nb, mc = W.kv_limits(wl, 9, block_sizes=(4,))
+    j = int(np.argmax(wl.n_run))
+    assert wl.n_run[j] > 0 and wl.run_ctx[j, :wl.n_run[j]].sum() > 8
+    # before any load: no snapshot
+    rt = make(wl, (bs, nb, mc), load=False)
+    t, _, _ = gpu_estimate(rt, wl)
+    assert np.isnan(t).all() and rt.status() == R().LR_ENOSTATE
+    rt.load_state(*R().state_tensors(wl))
+    good = gpu_estimate(rt, wl)
+    assert rt.status() == R().LR_OK
+    # the same snapshot with one request's context past the instance's blocks
+    bad = [a.clone() for a in R().state_tensors(wl)]
+    bad[1][j, 0] = int(nb[j] * bs[j] + 1)
+    rt.load_state(*bad)
+    again = gpu_estimate(rt, wl)
+    assert rt.status() == R().LR_ESTATE
+    for a, b in zip(good, again):
+        np.testing.assert_array_equal(np.asarray(a).view(np.uint8), np.asarray(b).view(np.uint8))
+    rt.close()
+
+
+def test_calls_closed_with_limits_and_turning_them_off():
+    wl = W.small_workload(64, num_instances=8, num_models=2, num_queries=16, budget_range=(8, 96), min_gap=8)
+    limits = W.kv_limits(wl, 10)
+    rt = make(wl, limits)
+    p, dh, acc, tau = R().query_tensors(wl)
+    with pytest.raises(R().LRError) as e:
+        rt.route(p, dh, acc, [1.0], [0.1])
+    assert e.value.code == R().LR_EINVAL
+    with pytest.raises(R().LRError) as e:
+        rt.set_ttft_source(R().LR_TTFT_THROUGHPUT)
+    assert e.value.code == R().LR_EINVAL
+    with pytest.raises(R().LRError) as e:
+        rt.advance(torch.zeros(16, dtype=torch.int32, device="cuda"), p, dh, 0.0)
+    assert e.value.code == R().LR_EINVAL
+    # the queue-length baselines stay open
+    o = rt.route_baseline(R().LR_POLICY_SHORTEST_QUEUE, p, dh, acc, 1.0, 0)
+    torch.cuda.synchronize()
+    ea, _, _ = oracle.baseline_route(wl, R().LR_POLICY_SHORTEST_QUEUE, 1.0, 0)
+    np.testing.assert_array_equal(o["assign"].cpu().numpy(), ea)
+    # turning the limits off drops the snapshot; a new load gives the plain estimate
+    rt.set_kv_limits()
+    t, _, _ = gpu_estimate(rt, wl)
+    assert np.isnan(t).all() and rt.status() == R().LR_ENOSTATE
+    rt.load_state(*R().state_tensors(wl))
+    got = gpu_estimate(rt, wl)
+    F0, lt0, t0, _ = oracle.estimate_matrix(wl)
+    compare(got, (F0, lt0, t0), np.ones(lt0.shape, bool))
+    assert rt.status() == R().LR_OK
+    rt.close()
+
+
+@pytest.mark.parametrize("name", ["pool64", "pool256"])
+def test_full_size_sampled(name):
+    # the full query set and pool in one call; the oracle checks sampled candidates
+    wl = W.make_workload(name)
+    limits = W.kv_limits(wl, 11, block_sizes=(16,))
+    rt = make(wl, limits)
+    t, fb, F = gpu_estimate(rt, wl)
+    assert rt.status() == R().LR_OK
+    rt.close()
+    rng = np.random.default_rng(5)
+    n = 4000
+    cq = rng.integers(0, wl.num_queries, n)
+    cj = rng.integers(0, wl.num_instances, n)
+    st, eF, elt, et, _ = oracle.estimate_matrix_kv(wl, *limits, cand_q=cq, cand_j=cj)
+    assert (st == 0).all()
+    np.testing.assert_array_equal(F[cq, cj], eF)
+    np.testing.assert_array_equal(fb[cq, cj], elt)
+    np.testing.assert_array_equal(bits(t[cq, cj]), bits(et))
+    assert not np.isnan(t).any()

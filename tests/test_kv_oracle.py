@@ -97,3 +97,56 @@ def test_residents_do_not_depend_on_the_query(mode):
         F0, _, lt0 = oracle.simulate(running, waiting, B, S, p, d, mode=mode)
         binding += int(lt != lt0 or not np.array_equal(F, F0))
     assert binding >= n // 4  # the limits bind in a good share of the cases
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_candidate_matrix_reduces_to_the_plain_matrix(mode):
+    # the batch entry point with limits that cannot bind gives the plain SFS matrix
+    # (an independent code path): features, first-token batches and times
+    from paper_2607_18253_gb300 import workloads as W
+    wl = W.small_workload(40 + mode, num_instances=7, num_queries=20, first_token_mode=mode)
+    st, F, lt, t32, t64 = oracle.estimate_matrix_kv(wl, 16, 1 << 40, 1 << 40)
+    F0, lt0, t320, t640 = oracle.estimate_matrix(wl)
+    assert (st == 0).all()
+    np.testing.assert_array_equal(F, F0)
+    np.testing.assert_array_equal(lt, lt0)
+    np.testing.assert_array_equal(t32.view(np.uint32), t320.view(np.uint32))
+    np.testing.assert_array_equal(t64, t640)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_candidate_matrix_matches_single_candidates(mode):
+    # the batch entry point under binding limits: each candidate as the single-candidate
+    # simulation gives it with one output token; invalid queries are flagged, not fatal
+    from paper_2607_18253_gb300 import workloads as W
+    wl = W.small_workload(50 + mode, num_instances=6, num_queries=12, first_token_mode=mode)
+    bs, nb, mc = W.kv_limits(wl, 3, block_sizes=(1, 4, 16))
+    mc = mc.copy()
+    wl.n_run[0] = 0  # an idle instance whose context limit some queries' prompts reach
+    wl.n_wait[0] = 0
+    mc[0] = int(np.median(wl.prompt_len))
+    nb[0] = max(nb[0], int(wl.run_ctx[0].max() + wl.run_pre[0].max() + wl.run_dec[0].max()) + 64)
+    st, F, lt, t32, _ = oracle.estimate_matrix_kv(wl, bs, nb, mc)
+    changed = 0
+    F0, lt0, _, _ = oracle.estimate_matrix(wl)
+    for i in range(wl.num_queries):
+        for j in range(wl.num_instances):
+            n, w = int(wl.n_run[j]), int(wl.n_wait[j])
+            running = list(zip(wl.run_ctx[j, :n], wl.run_pre[j, :n], wl.run_dec[j, :n]))
+            waiting = list(zip(wl.wait_pre[j, :w], wl.wait_dec[j, :w]))
+            p = int(wl.prompt_len[i])
+            try:
+                Fs, _, lts, _, _ = oracle.simulate_kv(running, waiting, int(wl.max_batched_tokens[j]),
+                                                      int(wl.max_seqs[j]), p, 1, block_size=int(bs[j]),
+                                                      num_blocks=int(nb[j]), max_ctx=int(mc[j]), mode=mode,
+                                                      max_batches=1 << 16)
+            except RuntimeError:
+                assert st[i, j] != 0 and (F[i, j] == -1).all() and lt[i, j] == -1 and np.isnan(t32[i, j])
+                assert j == 0 and p >= mc[0]
+                continue
+            assert st[i, j] == 0
+            np.testing.assert_array_equal(F[i, j], Fs)
+            assert lt[i, j] == lts
+            changed += int(lts != lt0[i, j] or not np.array_equal(Fs, F0[i, j]))
+    assert (st[:, 0] != 0).any() and (st[:, 0] == 0).any()
+    assert changed > 0  # the generated limits bind somewhere
