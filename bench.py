@@ -346,6 +346,7 @@ def run_gpu(args):
                 "note": "latency-bound event loop; bytes fraction shown for reference"}
 
     estimate = run_estimate(args, dev, wl, flush)
+    kv = run_kv(args, dev, wl, flush)
     avgcase = run_avgcase(args, dev, wl, flush)
     calibration = run_calibration(args, dev, flush)
     stream = None if args.no_stream else run_stream(args, dev)
@@ -370,6 +371,7 @@ def run_gpu(args):
             "sequential": {"ms_per_step": seq_ms, "value": cands * world / (seq_ms * 1e-3), "unit": UNIT,
                            "note": "K1 then K2 on one stream, same steps (kernel shares are of this time)"},
             "estimate": estimate,
+            "kv": kv,
             "avgcase": avgcase,
             "calibration": calibration,
             "stream": stream,
@@ -474,6 +476,86 @@ def run_estimate(args, dev, wl, flush):
             "roofline": {"kernel": "k_cand<0, 1>", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                          "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
                          "algorithmic_bytes": nbytes, "traffic": NCU_TRAFFIC["k_estimate"]}}
+
+
+KV_SEED = 11
+KV_BLOCK = 16
+KV_HORIZON = 1024
+
+
+def run_kv(args, dev, wl, flush):
+    """The SFS estimate under KV-cache block limits, context limits and preemption
+    (App. F) on the same workload: seeded limits (16-token blocks, each instance's
+    block count between its largest request and its residents' whole demand, half the
+    instances with a context limit).  A step is the snapshot load (residents alone
+    with per-batch records, k_kv_load) then the full Q x I TTFT matrix (per-candidate
+    walk over the records, k_kv_estimate), on one stream; each kernel is also timed
+    alone.  The estimate is timed against HBM: 4 B per candidate, 4 B per query, the
+    instance headers and the records up to each instance's last first-token batch."""
+    import torch
+    from paper_2607_18253_gb300 import router as R
+    from paper_2607_18253_gb300 import workloads as W
+
+    Q, I = wl.num_queries, wl.num_instances
+    limits = W.kv_limits(wl, KV_SEED, block_sizes=(KV_BLOCK,))
+    rt = R.LatencyRouter.from_workload(wl)
+    rt.set_kv_limits(*limits, horizon=KV_HORIZON)
+    state = R.state_tensors(wl, dev)
+    p = torch.from_numpy(np.ascontiguousarray(wl.prompt_len)).to(dev)
+    mat = torch.empty((Q, I), dtype=torch.float32, device=dev)
+    fb = torch.empty((Q, I), dtype=torch.int32, device=dev)
+    cap = torch.cuda.Stream(device=dev)
+    cap.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(cap):
+        for _ in range(3):
+            rt.load_state(*state)
+            rt.estimate_ttft(p, out=mat, first_batch=fb)
+    cap.synchronize()
+    if rt.status() != R.LR_OK:
+        raise RuntimeError("KV estimate failed")
+    last = fb.amax(dim=0).to(torch.int64).sum().item()  # records up to each instance's last first token
+    graphs = {}
+    for name in ("load", "estimate", "step"):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cap):
+            if name != "estimate":
+                rt.load_state(*state)
+            if name != "load":
+                rt.estimate_ttft(p, out=mat)
+        graphs[name] = g
+    K = max(3, min(args.steps, 300))
+    out = {}
+    for name, g in graphs.items():
+        for _ in range(args.warmup):
+            flush.fill_(1.0)
+            g.replay()
+        torch.cuda.synchronize()
+        ms = []
+        for k in range(K):
+            flush.fill_(float(k))
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            g.replay()
+            e1.record()
+            e1.synchronize()
+            ms.append(e0.elapsed_time(e1))
+        out[name] = sum(ms) / K
+    if rt.status() != R.LR_OK:
+        raise RuntimeError("KV estimate failed")
+    rt.close()
+    hbm, src = _peaks()
+    nbytes = Q * I * 4 + Q * 4 + I * 64 + last * 64
+    ach = nbytes / (out["estimate"] * 1e-3) / 1e9
+    return {"call": "lr_set_kv_limits, then per step lr_load_state + lr_estimate_ttft (SFS with KV limits)",
+            "limits": {"block_size": KV_BLOCK, "seed": KV_SEED, "horizon": KV_HORIZON,
+                       "ctx_limited_instances": int((limits[2] < (1 << 40)).sum()),
+                       "blocks_median": int(np.median(limits[1]))},
+            "ms_per_step": out["step"], "value": Q * I / (out["step"] * 1e-3), "unit": UNIT, "steps": K,
+            "gpu_launches": 2 * K, "load_ms": out["load"], "estimate_ms": out["estimate"],
+            "estimate_value": Q * I / (out["estimate"] * 1e-3),
+            "roofline": {"kernel": "k_kv_estimate", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+                         "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
+                         "algorithmic_bytes": nbytes, "traffic": NCU_TRAFFIC.get("k_kv_estimate")}}
 
 
 def run_avgcase(args, dev, wl, flush):

@@ -98,6 +98,7 @@ void free_kv(lr_ctx *c) {
     for (int b = 0; b < 2; ++b) {
         c->buf[b].kvi = nullptr;
         c->buf[b].kvr = nullptr;
+        c->buf[b].kvp = nullptr;
     }
 }
 
@@ -676,13 +677,15 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
         if (ee == cudaSuccess) c->kv_allocs.push_back(*p);
         return ee;
     };
-    void *bs = nullptr, *nb = nullptr, *mc = nullptr, *kvi[2] = {nullptr, nullptr}, *kvr[2] = {nullptr, nullptr};
+    void *bs = nullptr, *nb = nullptr, *mc = nullptr, *kvi[2] = {nullptr, nullptr}, *kvr[2] = {nullptr, nullptr},
+         *kvp[2] = {nullptr, nullptr};
     e = alloc(sizeof(int32_t) * I, &bs);
     if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &nb);
     if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &mc);
     for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
         e = alloc(sizeof(lr::KvInst) * I, &kvi[b]);
         if (e == cudaSuccess) e = alloc(sizeof(lr::KvRec) * (size_t)I * horizon, &kvr[b]);
+        if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (size_t)I * horizon, &kvp[b]);
     }
     if (e != cudaSuccess) {
         free_kv(c);
@@ -703,6 +706,7 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
     for (int b = 0; b < 2; ++b) {
         c->buf[b].kvi = static_cast<lr::KvInst *>(kvi[b]);
         c->buf[b].kvr = static_cast<lr::KvRec *>(kvr[b]);
+        c->buf[b].kvp = static_cast<int32_t *>(kvp[b]);
     }
     c->kv_warps = warps;
     c->kv_smem = warps * per_warp;

@@ -55,12 +55,11 @@ struct DevConfig {
 // the first batch in which a query could be admitted (the waiting queue empty after
 // admissions, budget and a seat left).  64 bytes.
 struct __align__(16) KvRec {
-    long long f3, f4;       // residents' decode contexts and prefill attention pairs
-    int32_t f1, f2;         // residents' prefill and decode tokens
-    int32_t bar, bl;        // budget left after the running scan, after admissions
-    int32_t seats, flags;   // free seats after admissions; bit 0: waiting queue empty
-    long long slack;        // least (free blocks - blocks needed) over the running scan
-    long long far, fa;      // free blocks after the running scan, after admissions
+    long long cf[4];   // residents' features 1..4 summed from the first record through this one
+    long long slack;   // least (free blocks - blocks needed) over the running scan; < 0: a preemption
+    long long far;     // free blocks after the running scan
+    long long thr;     // a waiting query with prompt p is admitted in this batch iff p <= thr
+    int32_t bar, bl;   // budget left after the running scan, after admissions
 };
 // Per instance: the residents' features before the first record, and the records' extent.
 struct __align__(16) KvInst {
@@ -86,8 +85,9 @@ struct StateBuf {
     unsigned char *tile;  // candidate-kernel tile blocks
     long long *f2, *f3;
     int32_t *rcum;
-    KvInst *kvi;  // [I], with KV limits
-    KvRec *kvr;   // [I][horizon], with KV limits
+    KvInst *kvi;   // [I], with KV limits
+    KvRec *kvr;    // [I][horizon], with KV limits
+    int32_t *kvp;  // [I][horizon] running maximum of the records' thr (clamped to int32), with KV limits
 };
 
 struct DevCtl {
@@ -186,10 +186,11 @@ struct KvLoad {
     StateIn in;
 };
 constexpr int kKvWarps = 4;
-// shared memory per warp of the KV load: running (ctx, pre, dec, chunk) and the waiting
-// ring (pre, dec) over capR + capW requests
+// shared memory per warp of the KV load: the running list (context, prefill, decode,
+// blocks) and the waiting ring (prefill, decode) over capR + capW requests, 16-byte
+// aligned
 __host__ __device__ inline size_t kv_smem_per_warp(const DevConfig &c) {
-    return sizeof(int32_t) * 6 * (size_t)(c.capR + c.capW) + 64;
+    return (sizeof(int32_t) * 6 * (size_t)(c.capR + c.capW) + 64 + 15) & ~(size_t)15;
 }
 // warps: instances per CTA, 1 .. kKvWarps
 cudaError_t launch_kv_load(const KvLoad &a, int grid, int warps, size_t smem, cudaStream_t st);

@@ -1,5 +1,5 @@
-// KV-limited Serving Framework Simulation (Sec. 4.1 with App. F's "context limits,
-// KV-cache allocation state, and preemption behavior").
+// KV-limited Serving Framework Simulation (Sec. 4.1; App. F names context limits,
+// the KV-cache allocation state and preemption among what the simulation models).
 //
 // Reading of the step rule: instance j has nb_j blocks of bs_j tokens and a request
 // with c tokens in the cache holds ceil(c / bs_j) of them.  The running list is
@@ -14,12 +14,14 @@
 // running request, so it is the first preemption victim and no resident ever waits
 // for its blocks.  So the load (k_kv_load) simulates each instance's residents
 // alone, once, and records for every batch from the first in which q could be
-// admitted what q's fate depends on: the budget, seats and free blocks left to it,
-// the least block slack of the residents' scan (q, holding h blocks, is preempted in
-// a batch whose slack is below h) and the residents' Eq. 9 features.  The estimate
-// (k_kv_estimate) then follows each (query, instance) candidate through those
-// records: waiting, admitted, prefilling chunk by chunk, preempted and readmitted,
-// until its first token.
+// admitted what q's fate depends on: the budget left to it, the largest prompt it
+// could be admitted with, the free blocks and the least block slack of the
+// residents' scan (q, holding h blocks, is preempted in a batch whose slack is
+// below h), and the residents' Eq. 9 features summed so far.  The estimate
+// (k_kv_estimate) then finds each (query, instance) candidate's admission batch by
+// a binary search over the running maximum of the admission bounds and follows it
+// from there, record by record, through prefill chunks, preemptions and
+// readmissions, to its first token.
 #include "lr_internal.cuh"
 
 namespace lr {
@@ -30,6 +32,10 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr long long kHuge = 1LL << 62;
 
 __device__ __forceinline__ long long kv_blocks(long long c, long long bs) { return (c + bs - 1) / bs; }
+// ceil(c / bs) for 0 <= c < 2^31 (32-bit division)
+__device__ __forceinline__ int kv_blocks32(int c, int bs) {
+    return (int)(((unsigned)c + (unsigned)bs - 1u) / (unsigned)bs);
+}
 
 __device__ void kv_fail(DevCtl *ctl, int code, int lane) {
     if (lane == 0) {
@@ -46,19 +52,44 @@ __device__ __forceinline__ long long warp_incl_sum64(long long x, int lane) {
     }
     return x;
 }
+__device__ __forceinline__ int warp_incl_sum32(int x, int lane) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(kFull, x, o);
+        if (lane >= o) x += y;
+    }
+    return x;
+}
+__device__ __forceinline__ long long warp_sum64(long long x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(kFull, x, o);
+    return x;
+}
+__device__ __forceinline__ int warp_sum32(int x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(kFull, x, o);
+    return x;
+}
 
 // One instance's residents alone, batch by batch, from the snapshot.  Every lane
 // holds the same scalar state; lane r of a chunk handles running request base + r.
+//
+// Running request r: rq[r] = (context, remaining prefill, remaining decode, blocks
+// held = ceil(context / bs)).  Only the last running request may be in prefill; it
+// holds its values as they are.  The others decode one token a batch, so they hold
+// context - G and decode + G, G being the number of batches done: a decode step
+// then writes nothing but a new block, and the decoders' context sum (Eq. 9's F3
+// term) is their stored sum plus G per decoder.
 template <int MODE>
 __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lane, int32_t *wb) {
     const DevConfig &c = a.cfg;
     const int B = c.B[j];
     const int S = c.S[j];
-    const long long bs = a.kv.bs[j], nbk = a.kv.nb[j], mctx = a.kv.mctx[j];
+    const long long nbk = a.kv.nb[j], mctx = a.kv.mctx[j];
+    const int bs = a.kv.bs[j];
     const int C = c.capR + c.capW;  // at most this many residents
-    int32_t *rctx = wb, *rpre = rctx + C, *rdec = rpre + C, *rx = rdec + C;  // running list, chunk of the batch
-    int32_t *wpre = rx + C, *wdec = wpre + C;                                  // waiting ring
-    long long *scr = reinterpret_cast<long long *>(wdec + C);                  // [8] lane 0 -> warp
+    int4 *rq = reinterpret_cast<int4 *>(wb);                    // running list
+    int2 *wq = reinterpret_cast<int2 *>(rq + C);                // waiting ring (prefill, decode)
     const int nr0 = a.in.n_run[j];
     const int nw0 = a.in.n_wait[j];
     if (lane == 0) {
@@ -75,21 +106,23 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
     // instance's blocks, and the running requests' blocks fit together.
     const size_t rrow = (size_t)j * c.capR, wrow = (size_t)j * c.capW;
     bool bad = false;
-    long long held = 0;
+    long long held = 0, wsum = 0, src = 0;
     for (int t = lane; t < c.capR; t += 32) {
         const int ctx = a.in.run_ctx[rrow + t], pre = a.in.run_pre[rrow + t], dec = a.in.run_dec[rrow + t];
         out.run_ctx[rrow + t] = ctx;
         out.run_pre[rrow + t] = pre;
         out.run_dec[rrow + t] = dec;
         if (t < nr0) {
-            bad |= ctx < 0 || ctx > (1 << 28) || pre < 0 || pre > (1 << 24) || dec < 1 || dec > (1 << 24);
+            const bool ok = ctx >= 0 && ctx <= (1 << 28) && pre >= 0 && pre <= (1 << 24) && dec >= 1 &&
+                            dec <= (1 << 24);
+            bad |= !ok;
             bad |= pre > 0 && t != nr0 - 1;
             bad |= (long long)ctx + pre >= mctx;
-            bad |= kv_blocks(min((long long)ctx + pre + dec, mctx), bs) > nbk;
-            held += kv_blocks(max(ctx, 0), bs);
-            rctx[t] = ctx;
-            rpre[t] = pre;
-            rdec[t] = dec;
+            bad |= ok && kv_blocks(min((long long)ctx + pre + dec, mctx), bs) > nbk;
+            const int h = ok ? kv_blocks32(ctx, bs) : 0;
+            held += h;
+            if (pre == 0) src += ctx;
+            rq[t] = make_int4(ctx, pre, dec, h);
         }
     }
     for (int t = lane; t < c.capW; t += 32) {
@@ -100,13 +133,14 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             bad |= pre < 1 || pre > (1 << 24) || dec < 1 || dec > (1 << 24);
             bad |= (long long)pre >= mctx;
             bad |= kv_blocks(min((long long)pre + dec, mctx), bs) > nbk;
-            wpre[t] = pre;
-            wdec[t] = dec;
+            wsum += pre;
+            wq[t] = make_int2(pre, dec);
         }
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) held += __shfl_xor_sync(kFull, held, o);
-    if (__any_sync(kFull, bad) || held > nbk) {
+    held = warp_sum64(held);
+    wsum = warp_sum64(wsum);
+    src = warp_sum64(src);
+    if (__any_sync(kFull, bad) || held > nbk || wsum > (1LL << 30)) {
         kv_fail(a.ctl, kEState, lane);
         return;
     }
@@ -114,123 +148,173 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
 
     long long freeb = nbk - held;
     int nr = nr0, wh = 0, wc = nw0;  // running count; waiting ring head and count
+    int G = 0;                       // batches done
     long long fcum[5] = {0, 0, 0, 0, 0};
-    int la0 = 0, nrec = 0, done = 0;
+    long long cf1 = 0, cf2 = 0, cf3 = 0, cf4 = 0;  // features summed over the records
+    int la0 = 0, nrec = 0, done = 0, pmx = 0;
     KvRec *rec = out.kvr + (size_t)j * a.kv.horizon;
+    int32_t *pmxo = out.kvp + (size_t)j * a.kv.horizon;
     for (int l = 1;; ++l) {
         if (l > c.max_iters) {
             kv_fail(a.ctl, kETraj, lane);
             return;
         }
         // 1. The running scan.  n_run <= S <= B and only the last request may be in
-        //    prefill, so every request gets its tokens: one per decoder, and the last
-        //    one's chunk from what the decoders leave.
-        long long need_all = 0;
-        for (int base = 0; base < nr; base += 32) {
+        //    prefill, so every request gets its tokens if the blocks suffice: one per
+        //    decoder, and the last one's chunk from what the decoders leave.  Each
+        //    decoder's new block is taken here; the first request to finish is noted.
+        const int4 plast = nr > 0 ? rq[nr - 1] : make_int4(0, 0, 0, 0);
+        const bool pf = plast.y > 0;
+        const int nd = nr - (pf ? 1 : 0);
+        int need = 0, fd = nr;
+        for (int base = 0; base < nd; base += 32) {
             const int r = base + lane;
-            long long need = 0;
-            if (r < nr) {
-                const int x = rpre[r] > 0 ? min(rpre[r], B - (nr - 1)) : 1;
-                rx[r] = x;
-                need = kv_blocks((long long)rctx[r] + x, bs) - kv_blocks(rctx[r], bs);
+            bool ends = false;
+            if (r < nd) {
+                const int4 q = rq[r];
+                const int cx = q.x + G;
+                const bool nw = (long long)q.w * bs < (long long)cx + 1;
+                if (nw) reinterpret_cast<int *>(rq + r)[3] = q.w + 1;
+                need += nw ? 1 : 0;
+                ends = q.z - G <= 1 || (long long)cx + 1 >= mctx;
             }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) need += __shfl_xor_sync(kFull, need, o);
-            need_all += need;
+            const unsigned m = __ballot_sync(kFull, ends);
+            if (m && fd == nr) fd = base + __ffs(m) - 1;
         }
-        __syncwarp();
-        long long slack;
+        int px = 0, pneed = 0;
+        if (pf) {
+            px = min(plast.y, B - nd);
+            pneed = kv_blocks32(plast.x + px, bs) - plast.w;
+        }
+        const int need_all = warp_sum32(need) + pneed;
+        long long slack, f1, f2, f3, f4;
         int budget;
+        bool pf_run = pf;  // the prefill request still runs after the scan
         if (need_all <= freeb) {
-            // nobody runs out: the least slack is at the last request
             slack = nr > 0 ? freeb - need_all : kHuge;
             freeb -= need_all;
-            budget = nr > 0 ? B - (nr - 1) - rx[nr - 1] : B;
+            budget = B - nd - px;
+            f1 = px;
+            f2 = nd;
+            f3 = src + (long long)nd * G;
+            f4 = (long long)px * plast.x + (long long)px * (px + 1) / 2;
         } else {
-            // a request runs out of blocks: the scan as the rule states it, with tail
-            // preemptions, on one lane (rare)
-            if (lane == 0) {
-                long long fb = freeb, sl = kHuge;
-                int n = nr, bud = B, r = 0, h = wh, cnt = wc;
-                while (r < n && bud > 0) {
-                    const int x = rpre[r] > 0 ? min(rpre[r], bud) : 1;
-                    const long long need = kv_blocks((long long)rctx[r] + x, bs) - kv_blocks(rctx[r], bs);
-                    sl = min(sl, fb - need);
-                    while (fb < need && n - 1 >= r) {
-                        const int v = n - 1;  // recompute: the whole context becomes prefill
-                        fb += kv_blocks(rctx[v], bs);
-                        h = (h - 1 + C) % C;
-                        wpre[h] = rpre[v] + rctx[v];
-                        wdec[h] = rdec[v];
-                        ++cnt;
-                        --n;
-                    }
-                    if (r >= n) break;
-                    fb -= need;
-                    rx[r] = x;
-                    bud -= x;
-                    ++r;
+            // a request runs out of blocks.  Preempting the tail until each request, in
+            // order, has its blocks leaves the longest prefix of the list whose blocks
+            // after the batch fit in the instance (what the rest held is what was free
+            // to them): those run, the rest go, in order, to the front of the waiting
+            // queue.  The prefill request, last, goes first, so the survivors are
+            // decoders, and the new blocks taken above stay theirs.
+            long long acc = 0, fitb = -1;  // blocks after the batch: before the chunk; of the survivors
+            int n = nr;
+            for (int base = 0; base < nr; base += 32) {
+                const int r = base + lane;
+                long long wv = 0;
+                if (r < nd) wv = rq[r].w;
+                else if (r < nr) wv = plast.w + pneed;
+                const long long cum = acc + warp_incl_sum64(wv, lane);
+                const int k = __popc(__ballot_sync(kFull, r < nr && cum <= nbk));
+                if (k < 32) {
+                    n = base + k;
+                    fitb = k > 0 ? __shfl_sync(kFull, cum, k - 1) : acc;
+                    break;
                 }
-                scr[0] = n;
-                scr[1] = bud;
-                scr[2] = fb;
-                scr[3] = sl;
-                scr[4] = h;
-                scr[5] = cnt;
+                acc = __shfl_sync(kFull, cum, 31);
             }
-            __syncwarp();
-            nr = (int)scr[0];
-            budget = (int)scr[1];
-            freeb = scr[2];
-            slack = scr[3];
-            wh = (int)scr[4];
-            wc = (int)scr[5];
-            __syncwarp();
+            if (fitb < 0) fitb = acc;
+            const int m = nr - n;
+            const int wh2 = (wh - m + C) % C;
+            long long gone = 0;
+            for (int base = 0; base < m; base += 32) {
+                const int k = base + lane;
+                if (k < m) {
+                    const int r = n + k;
+                    int slot = wh2 + k;
+                    if (slot >= C) slot -= C;
+                    if (r < nd) {
+                        const int4 q = rq[r];
+                        wq[slot] = make_int2(q.x + G, q.z - G);
+                        gone += q.x;
+                    } else {
+                        wq[slot] = make_int2(plast.x + plast.y, plast.z);
+                    }
+                }
+            }
+            src -= warp_sum64(gone);
+            wh = wh2;
+            wc += m;
+            nr = n;
+            freeb = nbk - fitb;
+            budget = B - n;
+            fd = min(fd, n);
+            f3 = src + (long long)n * G;
+            slack = -1;
+            f1 = 0;
+            f2 = n;
+            f4 = 0;
+            pf_run = false;
         }
+        __syncwarp();
+        if (pf_run) {
+            // the prefill request's chunk; at its last chunk it turns decoder
+            const int r = nr - 1;
+            const int cx = plast.x + px, pre = plast.y - px;
+            int dec = plast.z;
+            if (pre == 0 && MODE == 1) dec -= 1;
+            const bool ends = pre == 0 && (dec <= 0 || (long long)cx >= mctx);
+            if (pre == 0) src += cx - (G + 1);
+            if (lane == 0)
+                rq[r] = pre > 0 ? make_int4(cx, pre, dec, plast.w + pneed)
+                                : make_int4(cx - (G + 1), 0, dec + (G + 1), plast.w + pneed);
+            if (ends) fd = min(fd, r);
+        }
+        __syncwarp();
         const int bar = budget;
         const long long far = freeb;
         // 2. Admission from the waiting front while budget, a seat and the first chunk's
         //    blocks allow: the prompts that fit whole are a prefix (lane i tests the
-        //    i-th waiting request), then possibly one partial chunk.
+        //    i-th waiting request), then possibly one partial chunk.  An admitted
+        //    request's chunk is applied at once.
         while (budget > 0 && wc > 0 && nr < S) {
             const bool in = lane < wc && lane < S - nr;
-            const int slot = (wh + lane) % C;
-            const int pre_i = in ? wpre[slot] : 0;
-            const long long cp = warp_incl_sum64(pre_i, lane);
-            const long long cb = warp_incl_sum64(in ? kv_blocks(pre_i, bs) : 0, lane);
-            const bool whole = in && cp <= budget && cb <= freeb;
+            int slot = wh + lane;
+            if (slot >= C) slot -= C;
+            const int2 wv = in ? wq[slot] : make_int2(0, 0);
+            const int hb_i = in ? kv_blocks32(wv.x, bs) : 0;
+            const int cp = warp_incl_sum32(wv.x, lane);  // 32 prompts of at most 2^24 tokens
+            const int cb = warp_incl_sum32(hb_i, lane);
+            const bool whole = in && cp <= budget && (long long)cb <= freeb;
             const int k = __popc(__ballot_sync(kFull, whole));
-            if (whole) {
-                rctx[nr + lane] = 0;
-                rpre[nr + lane] = pre_i;
-                rdec[nr + lane] = wdec[slot];
-                rx[nr + lane] = pre_i;
-            }
+            const int dec_a = wv.y - (MODE == 1 ? 1 : 0);
+            if (whole) rq[nr + lane] = make_int4(wv.x - (G + 1), 0, dec_a + (G + 1), hb_i);
+            const unsigned em = __ballot_sync(kFull, whole && (dec_a <= 0 || (long long)wv.x >= mctx));
+            if (em) fd = min(fd, nr + __ffs(em) - 1);
             if (k > 0) {
-                budget -= (int)__shfl_sync(kFull, cp, k - 1);
-                freeb -= __shfl_sync(kFull, cb, k - 1);
+                const int sp = __shfl_sync(kFull, cp, k - 1), sb = __shfl_sync(kFull, cb, k - 1);
+                f1 += sp;
+                f4 += warp_sum64(whole ? (long long)wv.x * (wv.x + 1) / 2 : 0);
+                src += sp - (long long)k * (G + 1);
+                budget -= sp;
+                freeb -= sb;
                 nr += k;
-                wh = (wh + k) % C;
+                wh = wh + k >= C ? wh + k - C : wh + k;
                 wc -= k;
             }
             __syncwarp();
             if (k < 32) {
                 if (budget > 0 && wc > 0 && nr < S) {
-                    const int pre_h = wpre[wh];
-                    const int x = min(pre_h, budget);
-                    const long long need = kv_blocks(x, bs);
-                    if (x < pre_h && need <= freeb) {
-                        if (lane == 0) {
-                            rctx[nr] = 0;
-                            rpre[nr] = pre_h;
-                            rdec[nr] = wdec[wh];
-                            rx[nr] = x;
-                        }
+                    const int2 hv = wq[wh];
+                    const int x = min(hv.x, budget);
+                    const int nb1 = kv_blocks32(x, bs);
+                    if (x < hv.x && nb1 <= freeb) {
+                        if (lane == 0) rq[nr] = make_int4(x, hv.x - x, hv.y, nb1);
+                        f1 += x;
+                        f4 += (long long)x * (x + 1) / 2;
                         ++nr;
-                        wh = (wh + 1) % C;
+                        wh = wh + 1 >= C ? wh + 1 - C : wh + 1;
                         --wc;
                         budget -= x;
-                        freeb -= need;
+                        freeb -= nb1;
                     }
                 }
                 break;
@@ -239,54 +323,29 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
         __syncwarp();
         const bool qcan = wc == 0;
         if (la0 == 0 && qcan && budget > 0 && nr < S) la0 = l;
-        // 3. The batch's features, and each request's progress.
-        long long f1 = 0, f2 = 0, f3 = 0, f4 = 0;
-        for (int base = 0; base < nr; base += 32) {
-            const int r = base + lane;
-            if (r < nr) {
-                long long ctx = rctx[r];
-                int pre = rpre[r], dec = rdec[r];
-                if (pre > 0) {
-                    const long long x = rx[r];
-                    f1 += x;
-                    f4 += x * ctx + x * (x + 1) / 2;
-                    ctx += x;
-                    pre -= (int)x;
-                    if (pre == 0 && MODE == 1) dec -= 1;
-                } else {
-                    f2 += 1;
-                    f3 += ctx;
-                    ctx += 1;
-                    dec -= 1;
-                }
-                if (pre == 0 && ctx >= mctx) dec = 0;  // the context limit ends the response
-                rctx[r] = (int)ctx;
-                rpre[r] = pre;
-                rdec[r] = dec;
-            }
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            f1 += __shfl_xor_sync(kFull, f1, o);
-            f2 += __shfl_xor_sync(kFull, f2, o);
-            f3 += __shfl_xor_sync(kFull, f3, o);
-            f4 += __shfl_xor_sync(kFull, f4, o);
-        }
+        // 3. The batch's record, or the features before the first record.
         if (la0 != 0) {
+            cf1 += f1;
+            cf2 += f2;
+            cf3 += f3;
+            cf4 += f4;
+            // the largest prompt p admitted now: min(p, bl) tokens need at most fa blocks
+            long long thr = 0;
+            if (qcan && budget > 0 && nr < S) thr = ((long long)budget <= freeb * bs) ? kHuge : freeb * bs;
+            pmx = (int)max((long long)pmx, min(thr, (long long)INT32_MAX));
             if (lane == 0) {
                 KvRec R;
-                R.f3 = f3;
-                R.f4 = f4;
-                R.f1 = (int)f1;
-                R.f2 = (int)f2;
-                R.bar = bar;
-                R.bl = budget;
-                R.seats = S - nr;
-                R.flags = qcan ? 1 : 0;
+                R.cf[0] = cf1;
+                R.cf[1] = cf2;
+                R.cf[2] = cf3;
+                R.cf[3] = cf4;
                 R.slack = slack;
                 R.far = far;
-                R.fa = freeb;
+                R.thr = thr;
+                R.bar = bar;
+                R.bl = budget;
                 rec[nrec] = R;
+                pmxo[nrec] = pmx;
             }
             ++nrec;
         } else {
@@ -296,30 +355,35 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             fcum[3] += f3;
             fcum[4] += f4;
         }
-        __syncwarp();
-        // 4. Finished requests leave in order and return their blocks.
-        int kept = 0;
-        long long back = 0;
-        for (int base = 0; base < nr; base += 32) {
-            const int r = base + lane;
-            const bool live = r < nr && rdec[r] > 0;
-            const int v0 = r < nr ? rctx[r] : 0, v1 = r < nr ? rpre[r] : 0, v2 = r < nr ? rdec[r] : 0;
-            if (r < nr && !live) back += kv_blocks(v0, bs);
-            const unsigned m = __ballot_sync(kFull, live);
-            __syncwarp();
-            if (live) {
-                const int dst = kept + __popc(m & ((1u << lane) - 1u));
-                rctx[dst] = v0;
-                rpre[dst] = v1;
-                rdec[dst] = v2;
+        // 4. Finished requests leave in order and return their blocks (from the first
+        //    that finished: the list before it does not move).
+        const int G1 = G + 1;
+        if (fd < nr) {
+            int kept = fd;
+            long long back = 0, gone = 0;
+            for (int base = fd; base < nr; base += 32) {
+                const int r = base + lane;
+                int4 q = make_int4(0, 0, 0, 0);
+                bool live = false;
+                if (r < nr) {
+                    q = rq[r];
+                    live = q.y > 0 || (q.z - G1 > 0 && (long long)q.x + G1 < mctx);
+                    if (!live) {
+                        back += q.w;
+                        gone += q.x;
+                    }
+                }
+                const unsigned m = __ballot_sync(kFull, live);
+                __syncwarp();
+                if (live) rq[kept + __popc(m & ((1u << lane) - 1u))] = q;
+                kept += __popc(m);
+                __syncwarp();
             }
-            kept += __popc(m);
-            __syncwarp();
+            nr = kept;
+            freeb += warp_sum64(back);
+            src -= warp_sum64(gone);
         }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) back += __shfl_xor_sync(kFull, back, o);
-        nr = kept;
-        freeb += back;
+        G = G1;
         if (nr == 0 && wc == 0) {  // no resident left: every later batch is empty
             if (la0 == 0) la0 = l + 1;
             done = 1;
@@ -367,146 +431,240 @@ __global__ void __launch_bounds__(kKvWarps * 32) k_kv_load(const KvLoad a) {
 }
 
 constexpr float kNaN = __builtin_nanf("");
+constexpr int kEstGroup = 8;   // instances per CTA: one 32-byte sector of a query row
+constexpr int kEstWarps = 8;   // warps per CTA, each taking 32 queries against the whole group
+constexpr int kEstStage = 64;  // leading records of each instance staged in shared memory
 
-// One (query, instance) candidate through the instance's records (one thread each).
-// The query's state: waiting, or running with ctx tokens in the cache (h blocks) and
-// pre still to prefill.  In a batch it is preempted if the residents' scan leaves a
-// slack below h, or if its own tokens need more blocks than are free to it (it is
-// the last running request: it preempts itself); a preempted query recomputes its
-// whole context and may be readmitted in the same batch.  Admission needs the
-// residents' queue empty, budget, a seat and the first chunk's blocks.
-template <int MODE>
-__global__ void __launch_bounds__(256) k_kv_estimate(const KvEst a) {
-    const DevConfig &c = a.cfg;
-    const int active = load_acquire(&a.ctl->active);
-    const long long total = (long long)a.Q * c.I;
-    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
-         idx += (long long)gridDim.x * blockDim.x) {
-        const int i = (int)(idx / c.I);
-        const int j = (int)(idx - (long long)i * c.I);
-        const int p = a.prompt[i];
-        const long long bs = a.kv.bs[j], nbk = a.kv.nb[j], mctx = a.kv.mctx[j];
-        // a query with one output token: its prompt below the context limit and its
-        // whole context within the instance's blocks
-        const bool valid = p >= 1 && p <= c.pmax && (long long)p < mctx && kv_blocks(min((long long)p + 1, mctx), bs) <= nbk;
-        long long F[5] = {-1, -1, -1, -1, -1};
-        int lt = -1;
-        int err = 0;
-        if (active < 0) {
-            err = kENoState;
-        } else if (!valid) {
-            err = kEInval;
+// One instance as the estimate reads it: the first `ns` records (with their admission
+// maxima) from shared memory, the rest from global memory.
+struct KvView {
+    const KvRec *rec;
+    const int32_t *pmx;
+    long long fcum[5];
+    long long nb, mctx;
+    float b[5];
+    int la0, nrec, ns, done, B, bs;
+};
+
+// Record t of the view; past the records of a finished instance, an empty batch.
+__device__ __forceinline__ void kv_record(const KvView &v, const KvRec *srec, int t, long long &slack,
+                                          long long &far, long long &thr, int &bar, int &bl) {
+    if (t < v.ns) {
+        const KvRec &r = srec[t];
+        slack = r.slack;
+        far = r.far;
+        thr = r.thr;
+        bar = r.bar;
+        bl = r.bl;
+    } else if (t < v.nrec) {
+        const KvRec *r = v.rec + t;
+        slack = __ldg(&r->slack);
+        far = __ldg(&r->far);
+        thr = __ldg(&r->thr);
+        bar = __ldg(&r->bar);
+        bl = __ldg(&r->bl);
+    } else {
+        slack = kHuge;
+        far = v.nb;
+        thr = kHuge;
+        bar = v.B;
+        bl = v.B;
+    }
+}
+
+// first index in [lo, lo + n) whose value is >= p, in a nondecreasing array
+__device__ __forceinline__ int kv_lower_bound(const int32_t *a, int lo, int n, int p) {
+    while (n > 0) {
+        const int half = n >> 1;
+        if (a[lo + half] < p) {
+            lo += half + 1;
+            n -= half + 1;
         } else {
+            n = half;
+        }
+    }
+    return lo;
+}
+
+// One (query, instance) candidate: its features and first-token record, or an error.
+// The query waits (pre = p) until the first record whose admission bound reaches p,
+// found by binary search over the bounds' running maximum; from there it holds ctx
+// tokens in `held` blocks and pre still to prefill.  In a batch it is preempted if
+// the residents' scan leaves a slack below its blocks, or if its own tokens need more
+// blocks than are free to it (it is the last running request: it preempts itself);
+// a preempted query recomputes its whole context and may be readmitted in the same
+// batch.  Token counts stay below p + 2 <= 2^31.
+template <int MODE>
+__device__ int kv_candidate(const KvView &v, const KvRec *srec, const int32_t *spmx, int p, long long F[5],
+                            int &lt) {
+    int lo;
+    if (v.ns > 0 && spmx[v.ns - 1] >= p) lo = kv_lower_bound(spmx, 0, v.ns, p);
+    else lo = kv_lower_bound(v.pmx, v.ns, v.nrec - v.ns, p);
+    if (lo == v.nrec && !v.done) return kETraj;
+    // after the records the instance is empty; the query then needs at most
+    // ceil(p / B) + 2 batches
+    const int limit = v.nrec + (v.done ? (p / v.B + 3) : 0);
+    bool run = false;
+    int pre = p, ctx = 0, held = 0;
+    long long o1 = 0, o2 = 0, o3 = 0, o4 = 0;
+    int t = lo;
+    for (;; ++t) {
+        if (t >= limit) return kETraj;
+        long long slack, far, thr;
+        int bar, bl;
+        kv_record(v, srec, t, slack, far, thr, bar, bl);
+        if (run) {
+            if (slack < held) {  // a resident needs the query's blocks
+                pre += ctx;
+                ctx = 0;
+                held = 0;
+                run = false;
+            } else if (bar > 0) {
+                const int x = pre > 0 ? min(pre, bar) : 1;
+                const int nh = kv_blocks32(ctx + x, v.bs);
+                if (nh > far) {  // its own tokens do not fit: it preempts itself
+                    pre += ctx;
+                    ctx = 0;
+                    held = 0;
+                    run = false;
+                } else {
+                    held = nh;
+                    if (pre > 0) {
+                        o1 += x;
+                        o4 += (long long)x * ctx + (long long)x * (x + 1) / 2;
+                        ctx += x;
+                        pre -= x;
+                        if (pre == 0 && MODE == 1) break;
+                    } else {
+                        o2 += 1;
+                        o3 += ctx;
+                        break;
+                    }
+                    continue;
+                }
+            } else {
+                continue;  // no budget reached the query this batch
+            }
+        }
+        if (pre <= thr) {  // admission (pre == p while waiting)
+            const int x = min(pre, bl);
+            held = kv_blocks32(x, v.bs);
+            o1 += x;
+            o4 += (long long)x * (x + 1) / 2;
+            ctx = x;
+            pre -= x;
+            run = true;
+            if (pre == 0 && MODE == 1) break;
+        }
+    }
+    lt = t;
+    const int tc = min(t, v.nrec - 1);
+    long long cf[4] = {0, 0, 0, 0};
+    if (tc >= 0 && tc < v.ns) {
+        for (int k = 0; k < 4; ++k) cf[k] = srec[tc].cf[k];
+    } else if (tc >= 0) {
+        const KvRec *r = v.rec + tc;
+        for (int k = 0; k < 4; ++k) cf[k] = __ldg(&r->cf[k]);
+    }
+    F[0] = v.fcum[0] + t + 1;
+    F[1] = v.fcum[1] + cf[0] + o1;
+    F[2] = v.fcum[2] + cf[1] + o2;
+    F[3] = v.fcum[3] + cf[2] + o3;
+    F[4] = v.fcum[4] + cf[3] + o4;
+    return 0;
+}
+
+// CTA: kEstGroup instances, their leading records staged in shared memory.  Each
+// warp takes 32 queries at a time (lane -> query) against every instance of the
+// group, so a query row's kEstGroup estimates leave as one 32-byte sector, and no
+// warp waits for another.
+template <int MODE>
+__global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a) {
+    __shared__ KvView sv[kEstGroup];
+    __shared__ KvRec srec[kEstGroup][kEstStage];
+    __shared__ int32_t spmx[kEstGroup][kEstStage];
+    __shared__ float rows[kEstWarps][32][kEstGroup + 1];
+    const DevConfig &c = a.cfg;
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int j0 = blockIdx.y * kEstGroup;
+    const int ng = min(kEstGroup, c.I - j0);
+    const int active = load_acquire(&a.ctl->active);
+    if (w < ng) {
+        const int j = j0 + w;
+        KvView v;
+        v.nb = a.kv.nb[j];
+        v.mctx = a.kv.mctx[j];
+        v.bs = a.kv.bs[j];
+        v.B = c.B[j];
+        const float *cf = c.coef + 5 * c.moi[j];
+        for (int k = 0; k < 5; ++k) v.b[k] = cf[k];
+        v.ns = 0;
+        v.nrec = 0;
+        if (active >= 0) {
             const StateBuf sb = active ? a.buf1 : a.buf0;
             const KvInst hd = sb.kvi[j];
-            const KvRec *rec = sb.kvr + (size_t)j * a.kv.horizon;
-            for (int k = 0; k < 5; ++k) F[k] = hd.fcum[k];
-            const int B = c.B[j], S = c.S[j];
-            bool run = false;
-            long long pre = p, ctx = 0, held = 0;
-            // after the records the instance is empty; the query then needs at most
-            // ceil(p / B) + 2 batches
-            const int limit = hd.nrec + (hd.done ? (p / B + 3) : 0);
-            for (int t = 0;; ++t) {
-                if (t >= limit) {
-                    err = kETraj;
-                    break;
-                }
-                KvRec R;
-                if (t < hd.nrec) {
-                    R = rec[t];
+            for (int k = 0; k < 5; ++k) v.fcum[k] = hd.fcum[k];
+            v.la0 = hd.la0;
+            v.nrec = hd.nrec;
+            v.done = hd.done;
+            v.rec = sb.kvr + (size_t)j * a.kv.horizon;
+            v.pmx = sb.kvp + (size_t)j * a.kv.horizon;
+            v.ns = min(v.nrec, kEstStage);
+            const int4 *src = reinterpret_cast<const int4 *>(v.rec);
+            int4 *dst = reinterpret_cast<int4 *>(srec[w]);
+            constexpr int kWords = (int)(sizeof(KvRec) / sizeof(int4));
+            for (int e = lane; e < v.ns * kWords; e += 32) dst[e] = __ldg(src + e);
+            for (int e = lane; e < v.ns; e += 32) spmx[w][e] = __ldg(v.pmx + e);
+        }
+        if (lane == 0) sv[w] = v;
+    }
+    __syncthreads();
+    const bool vec = ng == kEstGroup && c.I % 4 == 0 && (reinterpret_cast<uintptr_t>(a.ttft) & 15) == 0;
+    const int nblk = (a.Q + 31) / 32;
+    for (int qb = blockIdx.x * kEstWarps + w; qb < nblk; qb += gridDim.x * kEstWarps) {
+        const int i = qb * 32 + lane;
+        const bool qv = i < a.Q;
+        const int p = qv ? a.prompt[i] : 1;
+        for (int g = 0; g < ng; ++g) {
+            const KvView &v = sv[g];
+            float tt = kNaN;
+            if (qv) {
+                long long F[5] = {-1, -1, -1, -1, -1};
+                int lt = -1;
+                int err;
+                // a query with one output token: its prompt below the context limit and
+                // its first token within the instance's blocks
+                if (active < 0) err = kENoState;
+                else if (!(p >= 1 && p <= c.pmax && (long long)p < v.mctx && kv_blocks32(p + 1, v.bs) <= v.nb))
+                    err = kEInval;
+                else err = kv_candidate<MODE>(v, srec[g], spmx[g], p, F, lt);
+                if (err) {
+                    record_status(a.ctl, err);
+                    for (int k = 0; k < 5; ++k) F[k] = -1;
                 } else {
-                    R.f3 = 0;
-                    R.f4 = 0;
-                    R.f1 = 0;
-                    R.f2 = 0;
-                    R.bar = B;
-                    R.bl = B;
-                    R.seats = S;
-                    R.flags = 1;
-                    R.slack = kHuge;
-                    R.far = nbk;
-                    R.fa = nbk;
+                    tt = __fmul_rn(v.b[0], __ll2float_rn(F[0]));
+                    tt = __fmaf_rn(v.b[2], __ll2float_rn(F[2]), tt);
+                    tt = __fmaf_rn(v.b[1], __ll2float_rn(F[1]), tt);
+                    tt = __fmaf_rn(v.b[3], __ll2float_rn(F[3]), tt);
+                    tt = __fmaf_rn(v.b[4], __ll2float_rn(F[4]), tt);
                 }
-                const int l = hd.la0 + t;
-                F[0] += 1;
-                F[1] += R.f1;
-                F[2] += R.f2;
-                F[3] += R.f3;
-                F[4] += R.f4;
-                bool first = false;
-                if (run) {
-                    if (R.slack < held) {  // a resident needs the query's blocks
-                        pre += ctx;
-                        ctx = 0;
-                        held = 0;
-                        run = false;
-                    } else if (R.bar > 0) {
-                        const long long x = pre > 0 ? min(pre, (long long)R.bar) : 1;
-                        const long long need = kv_blocks(ctx + x, bs) - held;
-                        if (need > R.far - held) {  // its own tokens do not fit: it preempts itself
-                            pre += ctx;
-                            ctx = 0;
-                            held = 0;
-                            run = false;
-                        } else {
-                            held += need;
-                            if (pre > 0) {
-                                F[1] += x;
-                                F[4] += x * ctx + x * (x + 1) / 2;
-                                ctx += x;
-                                pre -= x;
-                                first = (pre == 0 && MODE == 1);
-                            } else {
-                                F[2] += 1;
-                                F[3] += ctx;
-                                first = true;
-                            }
-                            if (first) {
-                                lt = l;
-                                break;
-                            }
-                            continue;
-                        }
-                    } else {
-                        continue;  // no budget reached the query this batch
-                    }
-                }
-                if ((R.flags & 1) && R.bl > 0 && R.seats > 0) {
-                    const long long x = min(pre, (long long)R.bl);
-                    const long long need = kv_blocks(x, bs);
-                    if (R.fa >= need) {
-                        held = need;
-                        F[1] += x;
-                        F[4] += x * (x + 1) / 2;
-                        ctx = x;
-                        pre -= x;
-                        run = true;
-                        if (pre == 0 && MODE == 1) {
-                            lt = l;
-                            break;
-                        }
-                    }
-                }
+                const size_t idx = (size_t)i * c.I + j0 + g;
+                if (a.first_batch) a.first_batch[idx] = err ? -1 : v.la0 + lt;
+                if (a.features)
+                    for (int k = 0; k < 5; ++k) a.features[idx * 5 + k] = F[k];
+            }
+            rows[w][lane][g] = tt;
+        }
+        if (qv && a.ttft) {
+            float *row = a.ttft + (size_t)i * c.I + j0;
+            const float *r = rows[w][lane];
+            if (vec) {
+                reinterpret_cast<float4 *>(row)[0] = make_float4(r[0], r[1], r[2], r[3]);
+                reinterpret_cast<float4 *>(row)[1] = make_float4(r[4], r[5], r[6], r[7]);
+            } else {
+                for (int g = 0; g < ng; ++g) row[g] = r[g];
             }
         }
-        if (err) record_status(a.ctl, err);
-        if (a.ttft) {
-            float t = kNaN;
-            if (!err) {
-                const int m = c.moi[j];
-                const float *b = c.coef + 5 * m;
-                t = __fmul_rn(b[0], __ll2float_rn(F[0]));
-                t = __fmaf_rn(b[2], __ll2float_rn(F[2]), t);
-                t = __fmaf_rn(b[1], __ll2float_rn(F[1]), t);
-                t = __fmaf_rn(b[3], __ll2float_rn(F[3]), t);
-                t = __fmaf_rn(b[4], __ll2float_rn(F[4]), t);
-            }
-            a.ttft[idx] = t;
-        }
-        if (a.first_batch) a.first_batch[idx] = err ? -1 : lt;
-        if (a.features)
-            for (int k = 0; k < 5; ++k) a.features[idx * 5 + k] = err ? -1 : F[k];
     }
 }
 
@@ -525,10 +683,12 @@ cudaError_t set_kv_smem(size_t bytes) {
 }
 
 cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st) {
-    const long long total = (long long)a.Q * a.cfg.I;
-    const int grid = (int)std::max<long long>(1, std::min<long long>((total + 255) / 256, (long long)sms * 8));
-    if (a.cfg.mode == 0) k_kv_estimate<0><<<grid, 256, 0, st>>>(a);
-    else k_kv_estimate<1><<<grid, 256, 0, st>>>(a);
+    const int gy = (a.cfg.I + kEstGroup - 1) / kEstGroup;
+    const int blocks = (a.Q + 32 * kEstWarps - 1) / (32 * kEstWarps);
+    const int gx = std::max(1, std::min(blocks, (sms * 4 + gy - 1) / gy));
+    const dim3 grid(gx, gy);
+    if (a.cfg.mode == 0) k_kv_estimate<0><<<grid, kEstWarps * 32, 0, st>>>(a);
+    else k_kv_estimate<1><<<grid, kEstWarps * 32, 0, st>>>(a);
     return cudaGetLastError();
 }
 
