@@ -551,7 +551,7 @@ def run_kv(args, dev, wl, flush):
                        "ctx_limited_instances": int((limits[2] < (1 << 40)).sum()),
                        "blocks_median": int(np.median(limits[1]))},
             "ms_per_step": out["step"], "value": Q * I / (out["step"] * 1e-3), "unit": UNIT, "steps": K,
-            "gpu_launches": 2 * K, "load_ms": out["load"], "estimate_ms": out["estimate"],
+            "gpu_launches": 3 * K, "load_ms": out["load"], "estimate_ms": out["estimate"],
             "estimate_value": Q * I / (out["estimate"] * 1e-3),
             "roofline": {"kernel": "k_kv_estimate", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                          "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",

@@ -41,6 +41,7 @@ struct lr_ctx {
     lr::KvLimits kv{};
     int kv_warps = 0;
     size_t kv_smem = 0;
+    int32_t *kv_order = nullptr;  // [max_queries] the estimate's query order
     std::vector<void *> kv_allocs;
     std::vector<void *> allocs;
     std::string err;
@@ -95,6 +96,7 @@ void free_kv(lr_ctx *c) {
     c->kv_allocs.clear();
     c->kv = lr::KvLimits{};
     c->kv_on = false;
+    c->kv_order = nullptr;
     for (int b = 0; b < 2; ++b) {
         c->buf[b].kvi = nullptr;
         c->buf[b].kvr = nullptr;
@@ -418,6 +420,7 @@ static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, 
         k.ttft = ttft;
         k.first_batch = iters;
         k.features = reinterpret_cast<long long *>(feat);
+        k.order = c->kv_order;
         cudaError_t e = lr::launch_kv_estimate(k, c->sms, (cudaStream_t)stream);
         return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "KV estimate launch");
     }
@@ -678,8 +681,9 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
         return ee;
     };
     void *bs = nullptr, *nb = nullptr, *mc = nullptr, *kvi[2] = {nullptr, nullptr}, *kvr[2] = {nullptr, nullptr},
-         *kvp[2] = {nullptr, nullptr};
+         *kvp[2] = {nullptr, nullptr}, *ord = nullptr;
     e = alloc(sizeof(int32_t) * I, &bs);
+    if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (size_t)c->max_queries, &ord);
     if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &nb);
     if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &mc);
     for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
@@ -703,6 +707,7 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
     c->kv.mctx = static_cast<const long long *>(mc);
     c->kv.horizon = horizon;
     c->kv.on = 1;
+    c->kv_order = static_cast<int32_t *>(ord);
     for (int b = 0; b < 2; ++b) {
         c->buf[b].kvi = static_cast<lr::KvInst *>(kvi[b]);
         c->buf[b].kvr = static_cast<lr::KvRec *>(kvr[b]);

@@ -205,6 +205,7 @@ struct KvEst {
     float *ttft;
     int32_t *first_batch;
     long long *features;
+    int32_t *order;  // [Q] scratch: the queries bucketed by prompt length
 };
 cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st);
 

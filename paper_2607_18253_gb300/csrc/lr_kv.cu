@@ -166,21 +166,27 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
         const int4 plast = nr > 0 ? rq[nr - 1] : make_int4(0, 0, 0, 0);
         const bool pf = plast.y > 0;
         const int nd = nr - (pf ? 1 : 0);
-        int need = 0, fd = nr;
-        for (int base = 0; base < nd; base += 32) {
-            const int r = base + lane;
-            bool ends = false;
-            if (r < nd) {
-                const int4 q = rq[r];
-                const int cx = q.x + G;
-                const bool nw = (long long)q.w * bs < (long long)cx + 1;
-                if (nw) reinterpret_cast<int *>(rq + r)[3] = q.w + 1;
-                need += nw ? 1 : 0;
-                ends = q.z - G <= 1 || (long long)cx + 1 >= mctx;
+        int need = 0, fdl = nr;  // this lane's blocks taken; its first request to finish
+        for (int base = 0; base < nd; base += 4 * 32) {
+            int4 q[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int r = base + u * 32 + lane;
+                q[u] = r < nd ? rq[r] : make_int4(0, 0, 1 << 30, 1 << 30);
             }
-            const unsigned m = __ballot_sync(kFull, ends);
-            if (m && fd == nr) fd = base + __ffs(m) - 1;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int r = base + u * 32 + lane;
+                const int cx = q[u].x + G;
+                const bool nw = (long long)q[u].w * bs < (long long)cx + 1;
+                if (nw) reinterpret_cast<int *>(rq + r)[3] = q[u].w + 1;  // never for r >= nd
+                need += nw ? 1 : 0;
+                if (r < nd && (q[u].z - G <= 1 || (long long)cx + 1 >= mctx) && r < fdl) fdl = r;
+            }
         }
+        int fd = fdl;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) fd = min(fd, __shfl_xor_sync(kFull, fd, o));
         int px = 0, pneed = 0;
         if (pf) {
             px = min(plast.y, B - nd);
@@ -574,6 +580,49 @@ __device__ int kv_candidate(const KvView &v, const KvRec *srec, const int32_t *s
     return 0;
 }
 
+// The queries in an order bucketed by prompt length (a counting sort over
+// kOrderBuckets ranges of [0, pmax]).  A candidate's walk through the records
+// depends on the instance and, mostly, on p, so lanes with near-equal p take
+// near-equal walks.  One CTA.
+constexpr int kOrderBuckets = 4096;
+constexpr int kOrderThreads = 1024;
+
+__global__ void __launch_bounds__(kOrderThreads) k_kv_order(const int32_t *prompt, int Q, int pmax, int32_t *order) {
+    __shared__ int cnt[kOrderBuckets];
+    __shared__ int wsum[kOrderThreads / 32];
+    const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+    for (int b = tid; b < kOrderBuckets; b += kOrderThreads) cnt[b] = 0;
+    __syncthreads();
+    auto bucket = [&](int p) {
+        const long long q = min(max(p, 0), pmax);
+        return (int)(q * kOrderBuckets / ((long long)pmax + 1));
+    };
+    for (int i = tid; i < Q; i += kOrderThreads) atomicAdd(&cnt[bucket(prompt[i])], 1);
+    __syncthreads();
+    // exclusive prefix sum: four buckets per thread, then warps, then the block
+    constexpr int kPer = kOrderBuckets / kOrderThreads;
+    int v[kPer], s = 0;
+    for (int k = 0; k < kPer; ++k) {
+        v[k] = cnt[tid * kPer + k];
+        s += v[k];
+    }
+    int incl = warp_incl_sum32(s, lane);
+    if (lane == 31) wsum[w] = incl;
+    __syncthreads();
+    if (w == 0) {
+        const int x = wsum[lane];
+        wsum[lane] = warp_incl_sum32(x, lane) - x;
+    }
+    __syncthreads();
+    int off = wsum[w] + incl - s;
+    for (int k = 0; k < kPer; ++k) {
+        cnt[tid * kPer + k] = off;
+        off += v[k];
+    }
+    __syncthreads();
+    for (int i = tid; i < Q; i += kOrderThreads) order[atomicAdd(&cnt[bucket(prompt[i])], 1)] = i;
+}
+
 // CTA: kEstGroup instances, their leading records staged in shared memory.  Each
 // warp takes 32 queries at a time (lane -> query) against every instance of the
 // group, so a query row's kEstGroup estimates leave as one 32-byte sector, and no
@@ -622,8 +671,8 @@ __global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a) {
     const bool vec = ng == kEstGroup && c.I % 4 == 0 && (reinterpret_cast<uintptr_t>(a.ttft) & 15) == 0;
     const int nblk = (a.Q + 31) / 32;
     for (int qb = blockIdx.x * kEstWarps + w; qb < nblk; qb += gridDim.x * kEstWarps) {
-        const int i = qb * 32 + lane;
-        const bool qv = i < a.Q;
+        const bool qv = qb * 32 + lane < a.Q;
+        const int i = qv ? a.order[qb * 32 + lane] : 0;
         const int p = qv ? a.prompt[i] : 1;
         for (int g = 0; g < ng; ++g) {
             const KvView &v = sv[g];
@@ -687,6 +736,7 @@ cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st) {
     const int blocks = (a.Q + 32 * kEstWarps - 1) / (32 * kEstWarps);
     const int gx = std::max(1, std::min(blocks, (sms * 4 + gy - 1) / gy));
     const dim3 grid(gx, gy);
+    k_kv_order<<<1, kOrderThreads, 0, st>>>(a.prompt, a.Q, a.cfg.pmax, a.order);
     if (a.cfg.mode == 0) k_kv_estimate<0><<<grid, kEstWarps * 32, 0, st>>>(a);
     else k_kv_estimate<1><<<grid, kEstWarps * 32, 0, st>>>(a);
     return cudaGetLastError();
