@@ -224,8 +224,9 @@ LR_API int lr_set_queue_params(lr_ctx *ctx, const lr_queue_params *params, void 
  * (LR_ENOSTATE before one is loaded); the LPS source reads none. */
 LR_API int lr_set_ttft_source(lr_ctx *ctx, int32_t source);
 
-/* KV-cache limits in the simulated step rule (App. F: the simulation accounts for
- * "context limits, KV-cache allocation state, and preemption behavior").  Reading:
+/* KV-cache limits in the simulated step rule (App. F counts context limits, the
+ * state of KV-cache allocation and preemption among what the simulation models,
+ * without a rule).  Reading:
  * instance j has num_blocks[j] blocks of block_size[j] tokens, a request with c
  * tokens in the cache holds ceil(c / block_size) of them; a running request whose
  * tokens of a batch need blocks that are not free preempts the last running request

@@ -567,8 +567,8 @@ int orc_on_time_utility(int32_t Q, const float *util, const float *ttft, const f
 
 /* ---- KV-cache limits, context limit and preemption (App. F) ----
  *
- * The paper lists "context limits, KV-cache allocation state, and preemption
- * behavior" among what the simulation accounts for, without a rule.  Reading
+ * App. F names context limits, the KV-cache allocation state and preemption
+ * among what the simulation models, without a rule.  Reading
  * (a paged KV cache as in vLLM, whose engine the paper uses):
  *  - an instance has num_blocks blocks of block_size tokens; a request with ctx
  *    tokens in the cache holds ceil(ctx / block_size) blocks;

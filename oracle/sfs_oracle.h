@@ -40,9 +40,10 @@ int orc_sfs_candidate(const orc_instance *inst, int32_t B, int32_t S, int32_t mo
                       int32_t p, int32_t d, int64_t max_batches,
                       int64_t F[5], int64_t *l_admit, int64_t *l_ttft);
 
-/* KV-cache limits of one instance (App. F: "context limits, KV-cache allocation
- * state, and preemption behavior"): block_size tokens per block, num_blocks blocks,
- * and max_ctx, the longest context a request may reach. */
+/* KV-cache limits of one instance (App. F names context limits, KV-cache
+ * allocation and preemption among what the simulation models): block_size tokens
+ * per block, num_blocks blocks, and max_ctx, the longest context a request may
+ * reach. */
 typedef struct {
     int32_t block_size;
     int64_t num_blocks;
