@@ -9,8 +9,8 @@
  * fmaf() calls of the canonical expressions below.
  *
  * Readings of points the paper leaves open (each is a stated convention):
- *  - Scheduler step (Sec. 2 "chunked prefills", App. F "queue order, admission
- *    limits, token-budget constraints"): a batch starts with budget B; the
+ *  - Scheduler step (Sec. 2 on chunked prefill; App. F on queue order, admission
+ *    limits and the token budget): a batch starts with budget B; the
  *    running list is served in order, a request with remaining prefill taking
  *    min(remaining, budget) tokens and a decoding request one token, until the
  *    budget is spent; then, while budget remains, the waiting list is non-empty
