@@ -42,6 +42,7 @@ struct lr_ctx {
     int kv_warps = 0;
     size_t kv_smem = 0;
     int32_t *kv_order = nullptr;  // [max_queries] the estimate's query order
+    int32_t *kv_leaders = nullptr, *kv_sort = nullptr;  // [max_queries]; [4][kKvBuckets] + 1
     std::vector<void *> kv_allocs;
     std::vector<void *> allocs;
     std::string err;
@@ -97,6 +98,8 @@ void free_kv(lr_ctx *c) {
     c->kv = lr::KvLimits{};
     c->kv_on = false;
     c->kv_order = nullptr;
+    c->kv_leaders = nullptr;
+    c->kv_sort = nullptr;
     for (int b = 0; b < 2; ++b) {
         c->buf[b].kvi = nullptr;
         c->buf[b].kvr = nullptr;
@@ -421,6 +424,12 @@ static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, 
         k.first_batch = iters;
         k.features = reinterpret_cast<long long *>(feat);
         k.order = c->kv_order;
+        k.leaders = c->kv_leaders;
+        k.cnt = c->kv_sort;
+        k.start = k.cnt + lr::kKvBuckets;
+        k.run = k.start + lr::kKvBuckets;
+        k.uid = k.run + lr::kKvBuckets;
+        k.nu = k.uid + lr::kKvBuckets;
         cudaError_t e = lr::launch_kv_estimate(k, c->sms, (cudaStream_t)stream);
         return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "KV estimate launch");
     }
@@ -681,9 +690,12 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
         return ee;
     };
     void *bs = nullptr, *nb = nullptr, *mc = nullptr, *kvi[2] = {nullptr, nullptr}, *kvr[2] = {nullptr, nullptr},
-         *kvp[2] = {nullptr, nullptr}, *ord = nullptr;
+         *kvp[2] = {nullptr, nullptr}, *ord = nullptr, *lead = nullptr, *srt = nullptr;
     e = alloc(sizeof(int32_t) * I, &bs);
     if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (size_t)c->max_queries, &ord);
+    if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (size_t)c->max_queries, &lead);
+    if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (4 * (size_t)lr::kKvBuckets + 1), &srt);
+    if (e == cudaSuccess) e = cudaMemset(srt, 0, sizeof(int32_t) * (4 * (size_t)lr::kKvBuckets + 1));
     if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &nb);
     if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &mc);
     for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
@@ -708,6 +720,8 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
     c->kv.horizon = horizon;
     c->kv.on = 1;
     c->kv_order = static_cast<int32_t *>(ord);
+    c->kv_leaders = static_cast<int32_t *>(lead);
+    c->kv_sort = static_cast<int32_t *>(srt);
     for (int b = 0; b < 2; ++b) {
         c->buf[b].kvi = static_cast<lr::KvInst *>(kvi[b]);
         c->buf[b].kvr = static_cast<lr::KvRec *>(kvr[b]);

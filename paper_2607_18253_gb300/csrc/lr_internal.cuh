@@ -205,8 +205,14 @@ struct KvEst {
     float *ttft;
     int32_t *first_batch;
     long long *features;
-    int32_t *order;  // [Q] scratch: the queries bucketed by prompt length
+    // the call's queries sorted by prompt length (counting sort over kKvBuckets
+    // buckets: invalid lengths, then valid ones >> shift); with shift 0 one
+    // query per length is estimated and the others copy its rows
+    int32_t *cnt, *start, *run, *uid;  // [kKvBuckets]
+    int32_t *nu;                       // [1] distinct lengths
+    int32_t *order, *leaders;          // [max_queries]
 };
+constexpr int kKvBuckets = 1 << 16;
 cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st);
 
 // Batches covered by K1's completion calendar; decoders ending later are

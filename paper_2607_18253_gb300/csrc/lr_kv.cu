@@ -580,47 +580,116 @@ __device__ int kv_candidate(const KvView &v, const KvRec *srec, const int32_t *s
     return 0;
 }
 
-// The queries in an order bucketed by prompt length (a counting sort over
-// kOrderBuckets ranges of [0, pmax]).  A candidate's walk through the records
-// depends on the instance and, mostly, on p, so lanes with near-equal p take
-// near-equal walks.  One CTA.
-constexpr int kOrderBuckets = 4096;
-constexpr int kOrderThreads = 1024;
+// The call's queries sorted by prompt length, by a counting sort over buckets:
+// bucket 0 holds the invalid lengths, bucket 1 + ((p - 1) >> shift) the valid ones.
+// A candidate depends on the instance and p alone, so with shift 0 (one bucket per
+// length) the estimate runs once per distinct length, on the bucket's first query
+// (its leader), and k_kv_expand copies the leader's rows to the bucket's other
+// queries; with a coarser shift every query is estimated, in sorted order, which
+// keeps the lanes of a warp on near-equal walks through the records.
+__device__ __forceinline__ int kv_bucket(int p, int pmax, int shift) {
+    return (p >= 1 && p <= pmax) ? 1 + ((p - 1) >> shift) : 0;
+}
 
-__global__ void __launch_bounds__(kOrderThreads) k_kv_order(const int32_t *prompt, int Q, int pmax, int32_t *order) {
-    __shared__ int cnt[kOrderBuckets];
-    __shared__ int wsum[kOrderThreads / 32];
-    const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-    for (int b = tid; b < kOrderBuckets; b += kOrderThreads) cnt[b] = 0;
-    __syncthreads();
-    auto bucket = [&](int p) {
-        const long long q = min(max(p, 0), pmax);
-        return (int)(q * kOrderBuckets / ((long long)pmax + 1));
-    };
-    for (int i = tid; i < Q; i += kOrderThreads) atomicAdd(&cnt[bucket(prompt[i])], 1);
-    __syncthreads();
-    // exclusive prefix sum: four buckets per thread, then warps, then the block
-    constexpr int kPer = kOrderBuckets / kOrderThreads;
-    int v[kPer], s = 0;
-    for (int k = 0; k < kPer; ++k) {
-        v[k] = cnt[tid * kPer + k];
-        s += v[k];
+__global__ void __launch_bounds__(256) k_kv_count(const int32_t *prompt, int Q, int pmax, int shift, int32_t *cnt) {
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < Q; i += gridDim.x * blockDim.x) {
+        const int b = kv_bucket(prompt[i], pmax, shift);
+        const unsigned m = __match_any_sync(__activemask(), b);
+        if ((threadIdx.x & 31) == __ffs(m) - 1) atomicAdd(&cnt[b], __popc(m));
     }
-    int incl = warp_incl_sum32(s, lane);
-    if (lane == 31) wsum[w] = incl;
+}
+
+// One CTA: start = run = exclusive prefix sums of the counts, uid = the number of
+// non-empty buckets before each one, nu = their total; the counts are cleared for
+// the next call.
+constexpr int kScanThreads = 1024;
+__global__ void __launch_bounds__(kScanThreads) k_kv_scan(int32_t *cnt, int32_t *start, int32_t *run, int32_t *uid,
+                                                          int32_t *nu, int nbk) {
+    __shared__ int ws[2][kScanThreads / 32];
+    const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+    const int per = (nbk + kScanThreads - 1) / kScanThreads;
+    const int b0 = min(nbk, tid * per), b1 = min(nbk, b0 + per);
+    int sc = 0, su = 0;
+    for (int b = b0; b < b1; ++b) {
+        const int v = cnt[b];
+        sc += v;
+        su += v > 0 ? 1 : 0;
+    }
+    const int ic = warp_incl_sum32(sc, lane), iu = warp_incl_sum32(su, lane);
+    if (lane == 31) {
+        ws[0][w] = ic;
+        ws[1][w] = iu;
+    }
     __syncthreads();
     if (w == 0) {
-        const int x = wsum[lane];
-        wsum[lane] = warp_incl_sum32(x, lane) - x;
+        const int xc = ws[0][lane], xu = ws[1][lane];
+        ws[0][lane] = warp_incl_sum32(xc, lane) - xc;
+        ws[1][lane] = warp_incl_sum32(xu, lane) - xu;
     }
     __syncthreads();
-    int off = wsum[w] + incl - s;
-    for (int k = 0; k < kPer; ++k) {
-        cnt[tid * kPer + k] = off;
-        off += v[k];
+    int oc = ws[0][w] + ic - sc, ou = ws[1][w] + iu - su;
+    for (int b = b0; b < b1; ++b) {
+        const int v = cnt[b];
+        start[b] = oc;
+        run[b] = oc;
+        uid[b] = ou;
+        cnt[b] = 0;
+        oc += v;
+        ou += v > 0 ? 1 : 0;
     }
-    __syncthreads();
-    for (int i = tid; i < Q; i += kOrderThreads) order[atomicAdd(&cnt[bucket(prompt[i])], 1)] = i;
+    if (tid == kScanThreads - 1) *nu = ou;
+}
+
+__global__ void __launch_bounds__(256) k_kv_scatter(const int32_t *prompt, int Q, int pmax, int shift, int32_t *run,
+                                                    const int32_t *start, const int32_t *uid, int32_t *order,
+                                                    int32_t *leaders) {
+    const int lane = threadIdx.x & 31;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < Q; i += gridDim.x * blockDim.x) {
+        const int b = kv_bucket(prompt[i], pmax, shift);
+        const unsigned act = __activemask();
+        const unsigned m = __match_any_sync(act, b);
+        const int lead = __ffs(m) - 1;
+        int base = 0;
+        if (lane == lead) base = atomicAdd(&run[b], __popc(m));
+        base = __shfl_sync(m, base, lead);
+        const int pos = base + __popc(m & ((1u << lane) - 1u));
+        order[pos] = i;
+        if (pos == start[b]) leaders[uid[b]] = i;
+    }
+}
+
+// One warp per query row: a query that is not its bucket's leader copies the
+// leader's rows (times, and first batches and features if asked for).
+__global__ void __launch_bounds__(256) k_kv_expand(const KvEst a) {
+    const int I = a.cfg.I, lane = threadIdx.x & 31;
+    const int warps = gridDim.x * (blockDim.x >> 5);
+    const bool v4 = I % 4 == 0 && (reinterpret_cast<uintptr_t>(a.ttft) & 15) == 0;
+    const bool f2 = I % 2 == 0 && (reinterpret_cast<uintptr_t>(a.features) & 15) == 0;
+    for (int i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); i < a.Q; i += warps) {
+        const int L = a.order[a.start[kv_bucket(a.prompt[i], a.cfg.pmax, 0)]];
+        if (L == i) continue;
+        const size_t ri = (size_t)i * I, rl = (size_t)L * I;
+        if (a.ttft) {
+            if (v4) {
+                const float4 *src = reinterpret_cast<const float4 *>(a.ttft + rl);
+                float4 *dst = reinterpret_cast<float4 *>(a.ttft + ri);
+                for (int c = lane; c < I / 4; c += 32) dst[c] = src[c];
+            } else {
+                for (int c = lane; c < I; c += 32) a.ttft[ri + c] = a.ttft[rl + c];
+            }
+        }
+        if (a.first_batch)
+            for (int c = lane; c < I; c += 32) a.first_batch[ri + c] = a.first_batch[rl + c];
+        if (a.features) {
+            if (f2) {
+                const int4 *src = reinterpret_cast<const int4 *>(a.features + rl * 5);
+                int4 *dst = reinterpret_cast<int4 *>(a.features + ri * 5);
+                for (int c = lane; c < I * 5 / 2; c += 32) dst[c] = src[c];
+            } else {
+                for (int c = lane; c < I * 5; c += 32) a.features[ri * 5 + c] = a.features[rl * 5 + c];
+            }
+        }
+    }
 }
 
 // CTA: kEstGroup instances, their leading records staged in shared memory.  Each
@@ -628,7 +697,7 @@ __global__ void __launch_bounds__(kOrderThreads) k_kv_order(const int32_t *promp
 // group, so a query row's kEstGroup estimates leave as one 32-byte sector, and no
 // warp waits for another.
 template <int MODE>
-__global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a) {
+__global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a, bool exact) {
     __shared__ KvView sv[kEstGroup];
     __shared__ KvRec srec[kEstGroup][kEstStage];
     __shared__ int32_t spmx[kEstGroup][kEstStage];
@@ -669,10 +738,13 @@ __global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a) {
     }
     __syncthreads();
     const bool vec = ng == kEstGroup && c.I % 4 == 0 && (reinterpret_cast<uintptr_t>(a.ttft) & 15) == 0;
-    const int nblk = (a.Q + 31) / 32;
+    // the work: one query per distinct prompt length, or every query, by length
+    const int nwork = exact ? *a.nu : a.Q;
+    const int32_t *work = exact ? a.leaders : a.order;
+    const int nblk = (nwork + 31) / 32;
     for (int qb = blockIdx.x * kEstWarps + w; qb < nblk; qb += gridDim.x * kEstWarps) {
-        const bool qv = qb * 32 + lane < a.Q;
-        const int i = qv ? a.order[qb * 32 + lane] : 0;
+        const bool qv = qb * 32 + lane < nwork;
+        const int i = qv ? work[qb * 32 + lane] : 0;
         const int p = qv ? a.prompt[i] : 1;
         for (int g = 0; g < ng; ++g) {
             const KvView &v = sv[g];
@@ -736,9 +808,17 @@ cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st) {
     const int blocks = (a.Q + 32 * kEstWarps - 1) / (32 * kEstWarps);
     const int gx = std::max(1, std::min(blocks, (sms * 4 + gy - 1) / gy));
     const dim3 grid(gx, gy);
-    k_kv_order<<<1, kOrderThreads, 0, st>>>(a.prompt, a.Q, a.cfg.pmax, a.order);
-    if (a.cfg.mode == 0) k_kv_estimate<0><<<grid, kEstWarps * 32, 0, st>>>(a);
-    else k_kv_estimate<1><<<grid, kEstWarps * 32, 0, st>>>(a);
+    int shift = 0;
+    while (2 + ((a.cfg.pmax - 1) >> shift) > kKvBuckets) ++shift;
+    const int nbk = 2 + ((a.cfg.pmax - 1) >> shift);
+    const bool exact = shift == 0;
+    const int g1 = std::max(1, std::min((a.Q + 255) / 256, sms * 4));
+    k_kv_count<<<g1, 256, 0, st>>>(a.prompt, a.Q, a.cfg.pmax, shift, a.cnt);
+    k_kv_scan<<<1, kScanThreads, 0, st>>>(a.cnt, a.start, a.run, a.uid, a.nu, nbk);
+    k_kv_scatter<<<g1, 256, 0, st>>>(a.prompt, a.Q, a.cfg.pmax, shift, a.run, a.start, a.uid, a.order, a.leaders);
+    if (a.cfg.mode == 0) k_kv_estimate<0><<<grid, kEstWarps * 32, 0, st>>>(a, exact);
+    else k_kv_estimate<1><<<grid, kEstWarps * 32, 0, st>>>(a, exact);
+    if (exact) k_kv_expand<<<std::max(1, std::min((a.Q + 7) / 8, sms * 8)), 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 

@@ -222,3 +222,33 @@ def test_full_size_sampled(name):
     np.testing.assert_array_equal(fb[cq, cj], elt)
     np.testing.assert_array_equal(bits(t[cq, cj]), bits(et))
     assert not np.isnan(t).any()
+
+
+def test_prompt_bound_beyond_exact_buckets():
+    # a prompt bound above 2^16 - 2: the sort buckets group several lengths, so
+    # every query is estimated (in sorted order) instead of one per length
+    wl = W.small_workload(65, num_instances=10, num_models=2, num_queries=60, max_prompt_len=150_000,
+                          budget_range=(6000, 8192), min_gap=4096)
+    p = wl.prompt_len.copy()
+    p[:6] = (1, 1, 150_000, 150_000, 65_535, 65_536)  # duplicates and bucket edges
+    wl.prompt_len = p
+    limits = W.kv_limits(wl, 12, block_sizes=(16, 64))
+    check(wl, limits)
+
+
+def test_many_duplicate_lengths():
+    # 2,000 queries over 40 distinct prompt lengths: most rows are copies of the
+    # row of the first query with the same length
+    wl = W.small_workload(66, num_instances=12, num_models=2, num_queries=2000, budget_range=(8, 96), min_gap=8)
+    rng = np.random.default_rng(0)
+    wl.prompt_len = rng.choice(np.arange(1, 161, 4, dtype=np.int32), 2000)
+    limits = W.kv_limits(wl, 13, block_sizes=(4,))
+    rt = make(wl, limits)
+    p = torch.from_numpy(np.ascontiguousarray(wl.prompt_len, np.int32)).cuda()
+    t_only = rt.estimate_ttft(p).cpu().numpy()  # times alone, then with first batches
+    got = gpu_estimate(rt, wl)
+    assert rt.status() == R().LR_OK
+    rt.close()
+    np.testing.assert_array_equal(bits(t_only), bits(got[0]))
+    st, eF, elt, et, _ = oracle.estimate_matrix_kv(wl, *limits)
+    compare(got, (eF, elt, et), st == 0)
