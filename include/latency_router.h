@@ -238,7 +238,7 @@ LR_API int lr_set_ttft_source(lr_ctx *ctx, int32_t source);
  * each instance's residents once, recording up to `horizon` batches from the first
  * one in which a query could be admitted, and lr_estimate_ttft /
  * lr_estimate_features follow each query through those records.
- * block_size [I] int32 in [1, 2^20], num_blocks [I] int64 in [1, 2^40], max_ctx [I]
+ * block_size [I] int32 in [1, 4096], num_blocks [I] int64 in [1, 2^40], max_ctx [I]
  * int64 in [2, 2^40]: host arrays, copied.  horizon in [1, 2^16].  All three arrays
  * NULL turns the limits off (the default).  The call synchronizes the device and drops
  * the live snapshot: estimates return LR_ENOSTATE until the next lr_load_state.

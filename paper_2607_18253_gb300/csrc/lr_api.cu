@@ -665,12 +665,14 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
         if (horizon < 1 || horizon > (1 << 16)) return fail(c, LR_EINVAL, "horizon must be in [1, 2^16]");
         if (c->source != lr::kSrcSfs) return fail(c, LR_EINVAL, "KV-cache limits apply to the SFS source only");
         for (int j = 0; j < I; ++j) {
-            if (block_size[j] < 1 || block_size[j] > (1 << 20)) return fail(c, LR_EINVAL, "block_size out of range");
+            if (block_size[j] < 1 || block_size[j] > lr::kKvMaxBlock) return fail(c, LR_EINVAL, "block_size out of range");
             if (num_blocks[j] < 1 || num_blocks[j] > (1LL << 40)) return fail(c, LR_EINVAL, "num_blocks out of range");
             if (max_ctx[j] < 2 || max_ctx[j] > (1LL << 40)) return fail(c, LR_EINVAL, "max_ctx out of range");
         }
     }
-    const size_t per_warp = lr::kv_smem_per_warp(c->cfg);
+    int hist = 1;
+    for (int j = 0; on && j < I; ++j) hist = std::max(hist, (int)block_size[j]);
+    const size_t per_warp = lr::kv_smem_per_warp(c->cfg, hist);
     if (on && per_warp > 200 * 1024) return fail(c, LR_ECAPACITY, "snapshot capacities too large for one KV-load warp");
     cudaError_t e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return cuda_fail(c, e, "synchronize");
@@ -718,7 +720,7 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
     c->kv.nb = static_cast<const long long *>(nb);
     c->kv.mctx = static_cast<const long long *>(mc);
     c->kv.horizon = horizon;
-    c->kv.on = 1;
+    c->kv.hist = hist;
     c->kv_order = static_cast<int32_t *>(ord);
     c->kv_leaders = static_cast<int32_t *>(lead);
     c->kv_sort = static_cast<int32_t *>(srt);

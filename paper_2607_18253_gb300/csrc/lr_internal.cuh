@@ -70,12 +70,14 @@ struct __align__(16) KvInst {
     int32_t pad;
 };
 struct KvLimits {
-    const int32_t *bs;     // [I] block size (tokens)
+    const int32_t *bs;     // [I] block size (tokens), at most kKvMaxBlock
     const long long *nb;   // [I] blocks
     const long long *mctx; // [I] context limit
     int32_t horizon;       // records per instance
-    int32_t on;
+    int32_t hist;          // the largest block size: entries of the load's residue histogram
 };
+constexpr int kKvMaxBlock = 4096;
+constexpr int kKvCal = 1024;  // batches covered by the load's end calendar
 
 struct StateBuf {
     int32_t *n_run, *run_ctx, *run_pre, *run_dec, *n_wait, *wait_pre, *wait_dec;
@@ -187,10 +189,11 @@ struct KvLoad {
 };
 constexpr int kKvWarps = 4;
 // shared memory per warp of the KV load: the running list (context, prefill, decode,
-// blocks) and the waiting ring (prefill, decode) over capR + capW requests, 16-byte
-// aligned
-__host__ __device__ inline size_t kv_smem_per_warp(const DevConfig &c) {
-    return (sizeof(int32_t) * 6 * (size_t)(c.capR + c.capW) + 64 + 15) & ~(size_t)15;
+// blocks) and the waiting ring (prefill, decode) over capR + capW requests, the end
+// calendar (links and blocks at the end per request, kKvCal heads) and the residue
+// histogram, 16-byte aligned
+__host__ __device__ inline size_t kv_smem_per_warp(const DevConfig &c, int hist) {
+    return (sizeof(int32_t) * (8 * (size_t)(c.capR + c.capW) + kKvCal + hist + 16) + 15) & ~(size_t)15;
 }
 // warps: instances per CTA, 1 .. kKvWarps
 cudaError_t launch_kv_load(const KvLoad &a, int grid, int warps, size_t smem, cudaStream_t st);

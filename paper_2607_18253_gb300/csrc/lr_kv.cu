@@ -71,15 +71,37 @@ __device__ __forceinline__ int warp_sum32(int x) {
     return x;
 }
 
+// End calendar of the KV load: a decoder that ends in batch E (>= the current
+// batch G) waits in list E mod kKvCal if E < G + kKvCal, else in the overflow list,
+// whose nodes are re-filed at every multiple of kKvCal.  Pushes from several lanes
+// at once are safe.
+__device__ __forceinline__ void kv_cal_push(int32_t *head, int32_t *nxt, int32_t *ovf, int s, long long E, int G) {
+    int32_t *h = E < (long long)G + kKvCal ? &head[E & (kKvCal - 1)] : ovf;
+    nxt[s] = atomicExch(h, s);
+}
+// the batch (as a value of G) in which a decoder held as (context - G, decode + G) ends
+__device__ __forceinline__ long long kv_end(const int4 &q, long long mctx) {
+    return min((long long)q.z - 1, mctx - 1 - q.x);
+}
+__device__ __forceinline__ int kv_res(int x, int bs) {
+    const int r = x % bs;
+    return r < 0 ? r + bs : r;
+}
+
 // One instance's residents alone, batch by batch, from the snapshot.  Every lane
-// holds the same scalar state; lane r of a chunk handles running request base + r.
+// holds the same scalar state.
 //
-// Running request r: rq[r] = (context, remaining prefill, remaining decode, blocks
-// held = ceil(context / bs)).  Only the last running request may be in prefill; it
-// holds its values as they are.  The others decode one token a batch, so they hold
-// context - G and decode + G, G being the number of batches done: a decode step
-// then writes nothing but a new block, and the decoders' context sum (Eq. 9's F3
-// term) is their stored sum plus G per decoder.
+// Running request in slot s: rq[s] = (context, prefill, decode, blocks held) for
+// the prefill request, (context - G, 0, decode + G, context residue mod bs) for a
+// decoder, whose blocks at its end wait in eb[s].  Slots keep the list's order; a
+// request that leaves becomes a hole (prefill -1) until a compaction.  Only the last running request may be in prefill (slot pfs); it holds
+// its values as they are.  The others decode one token a batch, so they hold
+// context - G and decode + G (G = batches done) and no word of theirs changes until
+// they end.  The decoders crossing into a new block in batch G are those whose
+// context is a multiple of bs, counted by a histogram of stored contexts mod bs;
+// their context sum (Eq. 9's F3 term) is a running total; the batch each one ends in
+// (decode count or context limit) waits in the end calendar.  A request that ends
+// frees ceil(context / bs) blocks after its last batch.
 template <int MODE>
 __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lane, int32_t *wb) {
     const DevConfig &c = a.cfg;
@@ -88,8 +110,13 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
     const long long nbk = a.kv.nb[j], mctx = a.kv.mctx[j];
     const int bs = a.kv.bs[j];
     const int C = c.capR + c.capW;  // at most this many residents
-    int4 *rq = reinterpret_cast<int4 *>(wb);                    // running list
-    int2 *wq = reinterpret_cast<int2 *>(rq + C);                // waiting ring (prefill, decode)
+    int4 *rq = reinterpret_cast<int4 *>(wb);               // running list slots
+    int2 *wq = reinterpret_cast<int2 *>(rq + C);           // waiting ring (prefill, decode)
+    int32_t *nxt = reinterpret_cast<int32_t *>(wq + C);    // [C] calendar links
+    int32_t *eb = nxt + C;                                 // [C] a decoder's blocks at its end
+    int32_t *head = eb + C;                                // [kKvCal] calendar lists
+    int32_t *hist = head + kKvCal;                         // [bs] residue histogram
+    int32_t *ovf = hist + a.kv.hist;                       // overflow list head
     const int nr0 = a.in.n_run[j];
     const int nw0 = a.in.n_wait[j];
     if (lane == 0) {
@@ -101,12 +128,22 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
         kv_fail(a.ctl, kEState, lane);
         return;
     }
+    for (int b = lane; b < kKvCal; b += 32) head[b] = -1;
+    for (int b = lane; b < bs; b += 32) hist[b] = 0;
+    if (lane == 0) *ovf = -1;
+    // file decoder slot s, held as q (fourth word: residue) at batch G
+    auto file = [&](int s, const int4 &q, int G_) {
+        const long long E = kv_end(q, mctx);
+        eb[s] = kv_blocks32((int)(q.x + E + 1), bs);
+        kv_cal_push(head, nxt, ovf, s, E, G_);
+    };
     // Copy and validate the snapshot: only the last running request may still be in
     // prefill, no context reaches the limit, every request's whole context fits the
     // instance's blocks, and the running requests' blocks fit together.
     const size_t rrow = (size_t)j * c.capR, wrow = (size_t)j * c.capW;
     bool bad = false;
     long long held = 0, wsum = 0, src = 0;
+    int nd = 0;
     for (int t = lane; t < c.capR; t += 32) {
         const int ctx = a.in.run_ctx[rrow + t], pre = a.in.run_pre[rrow + t], dec = a.in.run_dec[rrow + t];
         out.run_ctx[rrow + t] = ctx;
@@ -121,8 +158,11 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             bad |= ok && kv_blocks(min((long long)ctx + pre + dec, mctx), bs) > nbk;
             const int h = ok ? kv_blocks32(ctx, bs) : 0;
             held += h;
-            if (pre == 0) src += ctx;
-            rq[t] = make_int4(ctx, pre, dec, h);
+            if (pre == 0) {
+                src += ctx;
+                ++nd;
+            }
+            rq[t] = pre > 0 ? make_int4(ctx, pre, dec, h) : make_int4(ctx, 0, dec, ctx % bs);
         }
     }
     for (int t = lane; t < c.capW; t += 32) {
@@ -140,62 +180,104 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
     held = warp_sum64(held);
     wsum = warp_sum64(wsum);
     src = warp_sum64(src);
+    nd = warp_sum32(nd);
     if (__any_sync(kFull, bad) || held > nbk || wsum > (1LL << 30)) {
         kv_fail(a.ctl, kEState, lane);
         return;
     }
     __syncwarp();
+    // the decoders into the histogram and the calendar (G = 0)
+    for (int t = lane; t < nr0; t += 32) {
+        const int4 q = rq[t];
+        if (q.y == 0) {
+            atomicAdd(&hist[q.w], 1);
+            file(t, q, 0);
+        }
+    }
+    __syncwarp();
 
     long long freeb = nbk - held;
-    int nr = nr0, wh = 0, wc = nw0;  // running count; waiting ring head and count
-    int G = 0;                       // batches done
+    int nr = nr0, ne = nr0;                             // running requests; slots in use
+    int pfs = (nr0 > 0 && rq[nr0 - 1].y > 0) ? nr0 - 1 : -1;  // the prefill request's slot
+    int wh = 0, wc = nw0;                               // waiting ring head and count
+    int G = 0, gr = 0;                                  // batches done; G mod bs
+    long long f4c = 0;                                  // this lane's part of F4 before the first record
     long long fcum[5] = {0, 0, 0, 0, 0};
     long long cf1 = 0, cf2 = 0, cf3 = 0, cf4 = 0;  // features summed over the records
     int la0 = 0, nrec = 0, done = 0, pmx = 0;
     KvRec *rec = out.kvr + (size_t)j * a.kv.horizon;
     int32_t *pmxo = out.kvp + (size_t)j * a.kv.horizon;
+
+    // live slots to [0, nr) in order, and the calendar rebuilt
+    auto compact = [&]() {
+        int kept = 0;
+        for (int base = 0; base < ne; base += 32) {
+            const int s = base + lane;
+            const int4 q = s < ne ? rq[s] : make_int4(0, -1, 0, 0);
+            const int e = s < ne ? eb[s] : 0;
+            const bool live = q.y >= 0;
+            const unsigned m = __ballot_sync(kFull, live);
+            __syncwarp();
+            if (live) {
+                const int d = kept + __popc(m & ((1u << lane) - 1u));
+                rq[d] = q;
+                eb[d] = e;
+            }
+            kept += __popc(m);
+            __syncwarp();
+        }
+        ne = kept;
+        for (int b = lane; b < kKvCal; b += 32) head[b] = -1;
+        if (lane == 0) *ovf = -1;
+        __syncwarp();
+        for (int s = lane; s < ne; s += 32) {
+            const int4 q = rq[s];
+            if (q.y == 0) kv_cal_push(head, nxt, ovf, s, kv_end(q, mctx), G);
+        }
+        pfs = (ne > 0 && rq[ne - 1].y > 0) ? ne - 1 : -1;
+        __syncwarp();
+    };
+
     for (int l = 1;; ++l) {
         if (l > c.max_iters) {
             kv_fail(a.ctl, kETraj, lane);
             return;
         }
+        if (G > 0 && (G & (kKvCal - 1)) == 0) {
+            // re-file the overflow list
+            if (lane == 0) {
+                int s = *ovf, keep = -1;
+                while (s >= 0) {
+                    const int ns = nxt[s];
+                    const int4 q = rq[s];
+                    if (q.y == 0) {
+                        const long long E = kv_end(q, mctx);
+                        int32_t *h = E < (long long)G + kKvCal ? &head[E & (kKvCal - 1)] : &keep;
+                        nxt[s] = *h;
+                        *h = s;
+                    }
+                    s = ns;
+                }
+                *ovf = keep;
+            }
+            __syncwarp();
+        }
         // 1. The running scan.  n_run <= S <= B and only the last request may be in
         //    prefill, so every request gets its tokens if the blocks suffice: one per
-        //    decoder, and the last one's chunk from what the decoders leave.  Each
-        //    decoder's new block is taken here; the first request to finish is noted.
-        const int4 plast = nr > 0 ? rq[nr - 1] : make_int4(0, 0, 0, 0);
-        const bool pf = plast.y > 0;
-        const int nd = nr - (pf ? 1 : 0);
-        int need = 0, fdl = nr;  // this lane's blocks taken; its first request to finish
-        for (int base = 0; base < nd; base += 4 * 32) {
-            int4 q[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int r = base + u * 32 + lane;
-                q[u] = r < nd ? rq[r] : make_int4(0, 0, 1 << 30, 1 << 30);
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int r = base + u * 32 + lane;
-                const int cx = q[u].x + G;
-                const bool nw = (long long)q[u].w * bs < (long long)cx + 1;
-                if (nw) reinterpret_cast<int *>(rq + r)[3] = q[u].w + 1;  // never for r >= nd
-                need += nw ? 1 : 0;
-                if (r < nd && (q[u].z - G <= 1 || (long long)cx + 1 >= mctx) && r < fdl) fdl = r;
-            }
-        }
-        int fd = fdl;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) fd = min(fd, __shfl_xor_sync(kFull, fd, o));
+        //    decoder, and the last one's chunk from what the decoders leave.
+        const int4 pq = pfs >= 0 ? rq[pfs] : make_int4(0, 0, 0, 0);
+        const int need_d = nd > 0 ? hist[gr == 0 ? 0 : bs - gr] : 0;  // decoders at a block boundary
         int px = 0, pneed = 0;
-        if (pf) {
-            px = min(plast.y, B - nd);
-            pneed = kv_blocks32(plast.x + px, bs) - plast.w;
+        if (pfs >= 0) {
+            px = min(pq.y, B - nd);
+            pneed = kv_blocks32(pq.x + px, bs) - pq.w;
         }
-        const int need_all = warp_sum32(need) + pneed;
+        const int need_all = need_d + pneed;
         long long slack, f1, f2, f3, f4;
         int budget;
-        bool pf_run = pf;  // the prefill request still runs after the scan
+        bool pf_run = pfs >= 0;  // the prefill request still runs after the scan
+        int dying = 0;           // requests leaving after this batch
+        long long back = 0;      // and their blocks
         if (need_all <= freeb) {
             slack = nr > 0 ? freeb - need_all : kHuge;
             freeb -= need_all;
@@ -203,85 +285,115 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             f1 = px;
             f2 = nd;
             f3 = src + (long long)nd * G;
-            f4 = (long long)px * plast.x + (long long)px * (px + 1) / 2;
+            f4 = (long long)px * pq.x + (long long)px * (px + 1) / 2;
         } else {
             // a request runs out of blocks.  Preempting the tail until each request, in
             // order, has its blocks leaves the longest prefix of the list whose blocks
             // after the batch fit in the instance (what the rest held is what was free
             // to them): those run, the rest go, in order, to the front of the waiting
             // queue.  The prefill request, last, goes first, so the survivors are
-            // decoders, and the new blocks taken above stay theirs.
+            // decoders.
             long long acc = 0, fitb = -1;  // blocks after the batch: before the chunk; of the survivors
-            int n = nr;
-            for (int base = 0; base < nr; base += 32) {
-                const int r = base + lane;
+            int cut = ne;
+            for (int base = 0; base < ne; base += 32) {
+                const int s = base + lane;
                 long long wv = 0;
-                if (r < nd) wv = rq[r].w;
-                else if (r < nr) wv = plast.w + pneed;
+                if (s < ne) {
+                    const int4 q = rq[s];
+                    if (q.y == 0) wv = kv_blocks32(q.x + G + 1, bs);
+                    else if (q.y > 0) wv = kv_blocks32(q.x + px, bs);
+                }
                 const long long cum = acc + warp_incl_sum64(wv, lane);
-                const int k = __popc(__ballot_sync(kFull, r < nr && cum <= nbk));
+                const int k = __popc(__ballot_sync(kFull, s < ne && cum <= nbk));
                 if (k < 32) {
-                    n = base + k;
+                    cut = base + k;
                     fitb = k > 0 ? __shfl_sync(kFull, cum, k - 1) : acc;
                     break;
                 }
                 acc = __shfl_sync(kFull, cum, 31);
             }
             if (fitb < 0) fitb = acc;
-            const int m = nr - n;
+            int m = 0;
+            for (int base = cut; base < ne; base += 32) {
+                const int s = base + lane;
+                m += __popc(__ballot_sync(kFull, s < ne && rq[s].y >= 0));
+            }
             const int wh2 = (wh - m + C) % C;
+            int k0 = 0, gd = 0;
             long long gone = 0;
-            for (int base = 0; base < m; base += 32) {
-                const int k = base + lane;
-                if (k < m) {
-                    const int r = n + k;
-                    int slot = wh2 + k;
+            for (int base = cut; base < ne; base += 32) {
+                const int s = base + lane;
+                const int4 q = s < ne ? rq[s] : make_int4(0, -1, 0, 0);
+                const bool live = q.y >= 0;
+                const unsigned bl = __ballot_sync(kFull, live);
+                if (live) {
+                    int slot = wh2 + k0 + __popc(bl & ((1u << lane) - 1u));
                     if (slot >= C) slot -= C;
-                    if (r < nd) {
-                        const int4 q = rq[r];
+                    if (q.y == 0) {
                         wq[slot] = make_int2(q.x + G, q.z - G);
+                        atomicSub(&hist[q.w], 1);
                         gone += q.x;
+                        ++gd;
                     } else {
-                        wq[slot] = make_int2(plast.x + plast.y, plast.z);
+                        wq[slot] = make_int2(q.x + q.y, q.z);
                     }
+                    reinterpret_cast<int *>(rq + s)[1] = -1;
                 }
+                k0 += __popc(bl);
             }
             src -= warp_sum64(gone);
+            nd -= warp_sum32(gd);
+            if (pfs >= cut) pfs = -1;
             wh = wh2;
             wc += m;
-            nr = n;
+            nr -= m;
             freeb = nbk - fitb;
-            budget = B - n;
-            fd = min(fd, n);
-            f3 = src + (long long)n * G;
-            slack = -1;
+            budget = B - nr;
             f1 = 0;
-            f2 = n;
+            f2 = nd;
+            f3 = src + (long long)nd * G;
             f4 = 0;
+            slack = -1;
             pf_run = false;
         }
         __syncwarp();
         if (pf_run) {
             // the prefill request's chunk; at its last chunk it turns decoder
-            const int r = nr - 1;
-            const int cx = plast.x + px, pre = plast.y - px;
-            int dec = plast.z;
+            const int r = pfs;
+            const int cx = pq.x + px, pre = pq.y - px;
+            int dec = pq.z;
             if (pre == 0 && MODE == 1) dec -= 1;
-            const bool ends = pre == 0 && (dec <= 0 || (long long)cx >= mctx);
-            if (pre == 0) src += cx - (G + 1);
-            if (lane == 0)
-                rq[r] = pre > 0 ? make_int4(cx, pre, dec, plast.w + pneed)
-                                : make_int4(cx - (G + 1), 0, dec + (G + 1), plast.w + pneed);
-            if (ends) fd = min(fd, r);
+            if (pre > 0) {
+                if (lane == 0) rq[r] = make_int4(cx, pre, dec, pq.w + pneed);
+            } else if (dec <= 0 || (long long)cx >= mctx) {
+                if (lane == 0) reinterpret_cast<int *>(rq + r)[1] = -1;
+                back += pq.w + pneed;
+                ++dying;
+                pfs = -1;
+            } else {
+                const int4 q = make_int4(cx - (G + 1), 0, dec + (G + 1), kv_res(cx - (G + 1), bs));
+                if (lane == 0) {
+                    rq[r] = q;
+                    hist[q.w] += 1;
+                    file(r, q, G);
+                }
+                src += q.x;
+                ++nd;
+                pfs = -1;
+            }
         }
         __syncwarp();
         const int bar = budget;
         const long long far = freeb;
+        long long f4l = 0;      // this lane's whole admissions' F4 terms
+        bool admitted = false;  // any whole admission this batch
         // 2. Admission from the waiting front while budget, a seat and the first chunk's
         //    blocks allow: the prompts that fit whole are a prefix (lane i tests the
         //    i-th waiting request), then possibly one partial chunk.  An admitted
-        //    request's chunk is applied at once.
+        //    request's chunk is applied at once; one that prefills whole decodes from
+        //    the next batch.
         while (budget > 0 && wc > 0 && nr < S) {
+            if (ne + 32 > C) compact();
             const bool in = lane < wc && lane < S - nr;
             int slot = wh + lane;
             if (slot >= C) slot -= C;
@@ -292,17 +404,34 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             const bool whole = in && cp <= budget && (long long)cb <= freeb;
             const int k = __popc(__ballot_sync(kFull, whole));
             const int dec_a = wv.y - (MODE == 1 ? 1 : 0);
-            if (whole) rq[nr + lane] = make_int4(wv.x - (G + 1), 0, dec_a + (G + 1), hb_i);
-            const unsigned em = __ballot_sync(kFull, whole && (dec_a <= 0 || (long long)wv.x >= mctx));
-            if (em) fd = min(fd, nr + __ffs(em) - 1);
+            const bool ends = whole && (dec_a <= 0 || (long long)wv.x >= mctx);
+            if (whole) {
+                const int s = ne + lane;
+                const int4 q = make_int4(wv.x - (G + 1), ends ? -1 : 0, dec_a + (G + 1), kv_res(wv.x - (G + 1), bs));
+                rq[s] = q;
+                if (!ends) {
+                    atomicAdd(&hist[q.w], 1);
+                    file(s, q, G);
+                }
+                f4l += (long long)wv.x * (wv.x + 1) / 2;
+            }
+            const unsigned em = __ballot_sync(kFull, ends);
             if (k > 0) {
                 const int sp = __shfl_sync(kFull, cp, k - 1), sb = __shfl_sync(kFull, cb, k - 1);
                 f1 += sp;
-                f4 += warp_sum64(whole ? (long long)wv.x * (wv.x + 1) / 2 : 0);
+                admitted = true;
                 src += sp - (long long)k * (G + 1);
+                nd += k;
+                if (em) {
+                    src -= warp_sum64(ends ? (long long)wv.x - (G + 1) : 0);
+                    back += warp_sum64(ends ? (long long)hb_i : 0);
+                    dying += __popc(em);
+                    nd -= __popc(em);
+                }
                 budget -= sp;
                 freeb -= sb;
                 nr += k;
+                ne += k;
                 wh = wh + k >= C ? wh + k - C : wh + k;
                 wc -= k;
             }
@@ -313,10 +442,12 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
                     const int x = min(hv.x, budget);
                     const int nb1 = kv_blocks32(x, bs);
                     if (x < hv.x && nb1 <= freeb) {
-                        if (lane == 0) rq[nr] = make_int4(x, hv.x - x, hv.y, nb1);
+                        if (lane == 0) rq[ne] = make_int4(x, hv.x - x, hv.y, nb1);
+                        pfs = ne;
                         f1 += x;
                         f4 += (long long)x * (x + 1) / 2;
                         ++nr;
+                        ++ne;
                         wh = wh + 1 >= C ? wh + 1 - C : wh + 1;
                         --wc;
                         budget -= x;
@@ -330,6 +461,7 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
         const bool qcan = wc == 0;
         if (la0 == 0 && qcan && budget > 0 && nr < S) la0 = l;
         // 3. The batch's record, or the features before the first record.
+        if (la0 != 0 && admitted) f4 += warp_sum64(f4l);
         if (la0 != 0) {
             cf1 += f1;
             cf2 += f2;
@@ -360,43 +492,43 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             fcum[2] += f2;
             fcum[3] += f3;
             fcum[4] += f4;
+            f4c += f4l;  // summed over the warp at the end
         }
-        // 4. Finished requests leave in order and return their blocks (from the first
-        //    that finished: the list before it does not move).
-        const int G1 = G + 1;
-        if (fd < nr) {
-            int kept = fd;
-            long long back = 0, gone = 0;
-            for (int base = fd; base < nr; base += 32) {
-                const int r = base + lane;
-                int4 q = make_int4(0, 0, 0, 0);
-                bool live = false;
-                if (r < nr) {
-                    q = rq[r];
-                    live = q.y > 0 || (q.z - G1 > 0 && (long long)q.x + G1 < mctx);
-                    if (!live) {
-                        back += q.w;
-                        gone += q.x;
+        // 4. The decoders whose last batch this is leave and return their blocks.
+        {
+            int s = head[G & (kKvCal - 1)];
+            while (s >= 0) {
+                const int ns = nxt[s];
+                const int4 q = rq[s];
+                if (q.y == 0) {  // a hole is a request preempted after it was filed
+                    back += eb[s];
+                    ++dying;
+                    src -= q.x;
+                    --nd;
+                    if (lane == 0) {
+                        hist[q.w] -= 1;
+                        reinterpret_cast<int *>(rq + s)[1] = -1;
                     }
                 }
-                const unsigned m = __ballot_sync(kFull, live);
-                __syncwarp();
-                if (live) rq[kept + __popc(m & ((1u << lane) - 1u))] = q;
-                kept += __popc(m);
-                __syncwarp();
+                s = ns;
             }
-            nr = kept;
-            freeb += warp_sum64(back);
-            src -= warp_sum64(gone);
+            __syncwarp();
+            if (lane == 0) head[G & (kKvCal - 1)] = -1;
         }
-        G = G1;
+        nr -= dying;
+        freeb += back;
+        G = G + 1;
+        gr = gr + 1 == bs ? 0 : gr + 1;
+        __syncwarp();
         if (nr == 0 && wc == 0) {  // no resident left: every later batch is empty
             if (la0 == 0) la0 = l + 1;
             done = 1;
             break;
         }
         if (nrec == a.kv.horizon) break;
+        if (ne - nr >= max(32, nr)) compact();
     }
+    fcum[4] += warp_sum64(f4c);
     if (lane == 0) {
         KvInst hd;
         for (int k = 0; k < 5; ++k) hd.fcum[k] = fcum[k];
@@ -419,7 +551,7 @@ __global__ void __launch_bounds__(kKvWarps * 32) k_kv_load(const KvLoad a) {
     __syncthreads();
     const int dst = (s_active == 0) ? 1 : 0;
     const StateBuf out = dst ? a.buf1 : a.buf0;
-    const size_t per_warp = kv_smem_per_warp(a.cfg) / sizeof(int32_t);
+    const size_t per_warp = kv_smem_per_warp(a.cfg, a.kv.hist) / sizeof(int32_t);
     if (j < a.cfg.I) kv_instance<MODE>(a, out, j, lane, kv_smem + wid * per_warp);
     // the last CTA to finish publishes the new snapshot if every instance succeeded
     __syncthreads();
