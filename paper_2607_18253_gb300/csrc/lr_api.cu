@@ -42,7 +42,7 @@ struct lr_ctx {
     int kv_warps = 0;
     size_t kv_smem = 0;
     int32_t *kv_order = nullptr;  // [max_queries] the estimate's query order
-    int32_t *kv_leaders = nullptr, *kv_sort = nullptr;  // [max_queries]; [4][kKvBuckets] + 1
+    int32_t *kv_leaders = nullptr, *kv_sort = nullptr;  // [max_queries]; [4][kKvBuckets] + 4 + [ceil(I/8)]
     std::vector<void *> kv_allocs;
     std::vector<void *> allocs;
     std::string err;
@@ -430,6 +430,7 @@ static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, 
         k.run = k.start + lr::kKvBuckets;
         k.uid = k.run + lr::kKvBuckets;
         k.nu = k.uid + lr::kKvBuckets;
+        k.claim = k.nu + 4;
         cudaError_t e = lr::launch_kv_estimate(k, c->sms, (cudaStream_t)stream);
         return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "KV estimate launch");
     }
@@ -696,8 +697,9 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
     e = alloc(sizeof(int32_t) * I, &bs);
     if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (size_t)c->max_queries, &ord);
     if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (size_t)c->max_queries, &lead);
-    if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (4 * (size_t)lr::kKvBuckets + 1), &srt);
-    if (e == cudaSuccess) e = cudaMemset(srt, 0, sizeof(int32_t) * (4 * (size_t)lr::kKvBuckets + 1));
+    const size_t srt_words = 4 * (size_t)lr::kKvBuckets + 4 + (size_t)(I + 7) / 8;
+    if (e == cudaSuccess) e = alloc(sizeof(int32_t) * srt_words, &srt);
+    if (e == cudaSuccess) e = cudaMemset(srt, 0, sizeof(int32_t) * srt_words);
     if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &nb);
     if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &mc);
     for (int b = 0; b < 2 && e == cudaSuccess; ++b) {

@@ -214,6 +214,7 @@ struct KvEst {
     int32_t *cnt, *start, *run, *uid;  // [kKvBuckets]
     int32_t *nu;                       // [1] distinct lengths
     int32_t *order, *leaders;          // [max_queries]
+    int32_t *claim;                    // [ceil(I / 8)] the estimate's block counters per instance group
 };
 constexpr int kKvBuckets = 1 << 16;
 cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st);

@@ -733,43 +733,65 @@ __global__ void __launch_bounds__(256) k_kv_count(const int32_t *prompt, int Q, 
 
 // One CTA: start = run = exclusive prefix sums of the counts, uid = the number of
 // non-empty buckets before each one, nu = their total; the counts are cleared for
-// the next call.
+// the next call, and the estimate's block counters too.  Tiles of 4096 buckets,
+// four per thread as one 16-byte word.
 constexpr int kScanThreads = 1024;
+static_assert(kKvBuckets % (4 * kScanThreads) == 0, "scan tiles cover the buckets");
 __global__ void __launch_bounds__(kScanThreads) k_kv_scan(int32_t *cnt, int32_t *start, int32_t *run, int32_t *uid,
-                                                          int32_t *nu, int nbk) {
+                                                          int32_t *nu, int nbk, int32_t *claim, int groups) {
     __shared__ int ws[2][kScanThreads / 32];
+    __shared__ int tot[2];
     const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-    const int per = (nbk + kScanThreads - 1) / kScanThreads;
-    const int b0 = min(nbk, tid * per), b1 = min(nbk, b0 + per);
-    int sc = 0, su = 0;
-    for (int b = b0; b < b1; ++b) {
-        const int v = cnt[b];
-        sc += v;
-        su += v > 0 ? 1 : 0;
+    for (int g = tid; g < groups; g += kScanThreads) claim[g] = 0;
+    int carry_c = 0, carry_u = 0;
+    constexpr int kTile = 4 * kScanThreads;
+    for (int t0 = 0; t0 < nbk; t0 += kTile) {  // nbk <= kKvBuckets, a multiple of kTile
+        const int b = t0 + 4 * tid;
+        const int4 v = reinterpret_cast<const int4 *>(cnt)[b / 4];
+        const int sc = v.x + v.y + v.z + v.w;
+        const int su = (v.x > 0) + (v.y > 0) + (v.z > 0) + (v.w > 0);
+        const int ic = warp_incl_sum32(sc, lane), iu = warp_incl_sum32(su, lane);
+        if (lane == 31) {
+            ws[0][w] = ic;
+            ws[1][w] = iu;
+        }
+        __syncthreads();
+        if (w == 0) {
+            const int xc = ws[0][lane], xu = ws[1][lane];
+            const int yc = warp_incl_sum32(xc, lane), yu = warp_incl_sum32(xu, lane);
+            ws[0][lane] = yc - xc;
+            ws[1][lane] = yu - xu;
+            if (lane == 31) {
+                tot[0] = yc;
+                tot[1] = yu;
+            }
+        }
+        __syncthreads();
+        int oc = carry_c + ws[0][w] + ic - sc, ou = carry_u + ws[1][w] + iu - su;
+        int4 so, uo;
+        so.x = oc;
+        uo.x = ou;
+        oc += v.x;
+        ou += v.x > 0;
+        so.y = oc;
+        uo.y = ou;
+        oc += v.y;
+        ou += v.y > 0;
+        so.z = oc;
+        uo.z = ou;
+        oc += v.z;
+        ou += v.z > 0;
+        so.w = oc;
+        uo.w = ou;
+        reinterpret_cast<int4 *>(start)[b / 4] = so;
+        reinterpret_cast<int4 *>(run)[b / 4] = so;
+        reinterpret_cast<int4 *>(uid)[b / 4] = uo;
+        reinterpret_cast<int4 *>(cnt)[b / 4] = make_int4(0, 0, 0, 0);
+        carry_c += tot[0];
+        carry_u += tot[1];
+        __syncthreads();
     }
-    const int ic = warp_incl_sum32(sc, lane), iu = warp_incl_sum32(su, lane);
-    if (lane == 31) {
-        ws[0][w] = ic;
-        ws[1][w] = iu;
-    }
-    __syncthreads();
-    if (w == 0) {
-        const int xc = ws[0][lane], xu = ws[1][lane];
-        ws[0][lane] = warp_incl_sum32(xc, lane) - xc;
-        ws[1][lane] = warp_incl_sum32(xu, lane) - xu;
-    }
-    __syncthreads();
-    int oc = ws[0][w] + ic - sc, ou = ws[1][w] + iu - su;
-    for (int b = b0; b < b1; ++b) {
-        const int v = cnt[b];
-        start[b] = oc;
-        run[b] = oc;
-        uid[b] = ou;
-        cnt[b] = 0;
-        oc += v;
-        ou += v > 0 ? 1 : 0;
-    }
-    if (tid == kScanThreads - 1) *nu = ou;
+    if (tid == 0) *nu = carry_u;
 }
 
 __global__ void __launch_bounds__(256) k_kv_scatter(const int32_t *prompt, int Q, int pmax, int shift, int32_t *run,
@@ -874,9 +896,15 @@ __global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a, b
     const int nwork = exact ? *a.nu : a.Q;
     const int32_t *work = exact ? a.leaders : a.order;
     const int nblk = (nwork + 31) / 32;
-    for (int qb = blockIdx.x * kEstWarps + w; qb < nblk; qb += gridDim.x * kEstWarps) {
-        const bool qv = qb * 32 + lane < nwork;
-        const int i = qv ? work[qb * 32 + lane] : 0;
+    for (;;) {
+        // the group's warps claim blocks of 32 queries, the longest prompts first
+        int qb = 0;
+        if (lane == 0) qb = atomicAdd(&a.claim[blockIdx.y], 1);
+        qb = __shfl_sync(kFull, qb, 0);
+        if (qb >= nblk) break;
+        const int pos = nwork - 1 - (qb * 32 + lane);
+        const bool qv = pos >= 0;
+        const int i = qv ? work[pos] : 0;
         const int p = qv ? a.prompt[i] : 1;
         for (int g = 0; g < ng; ++g) {
             const KvView &v = sv[g];
@@ -946,7 +974,7 @@ cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st) {
     const bool exact = shift == 0;
     const int g1 = std::max(1, std::min((a.Q + 255) / 256, sms * 4));
     k_kv_count<<<g1, 256, 0, st>>>(a.prompt, a.Q, a.cfg.pmax, shift, a.cnt);
-    k_kv_scan<<<1, kScanThreads, 0, st>>>(a.cnt, a.start, a.run, a.uid, a.nu, nbk);
+    k_kv_scan<<<1, kScanThreads, 0, st>>>(a.cnt, a.start, a.run, a.uid, a.nu, (nbk + 4095) / 4096 * 4096, a.claim, gy);
     k_kv_scatter<<<g1, 256, 0, st>>>(a.prompt, a.Q, a.cfg.pmax, shift, a.run, a.start, a.uid, a.order, a.leaders);
     if (a.cfg.mode == 0) k_kv_estimate<0><<<grid, kEstWarps * 32, 0, st>>>(a, exact);
     else k_kv_estimate<1><<<grid, kEstWarps * 32, 0, st>>>(a, exact);
