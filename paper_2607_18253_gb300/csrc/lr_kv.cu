@@ -569,9 +569,30 @@ __global__ void __launch_bounds__(kKvWarps * 32) k_kv_load(const KvLoad a) {
 }
 
 constexpr float kNaN = __builtin_nanf("");
-constexpr int kEstGroup = 8;   // instances per CTA: one 32-byte sector of a query row
-constexpr int kEstWarps = 8;   // warps per CTA, each taking 32 queries against the whole group
-constexpr int kEstStage = 64;  // leading records of each instance staged in shared memory
+constexpr int kEstGroup = 8;    // instances per CTA
+constexpr int kEstWarps = 8;    // warps per CTA
+constexpr int kEstStage = 256;  // leading records of each instance staged in shared memory
+// the staged fields of the walk: slack, far, thr (8 bytes), bar, bl, admission maximum (4)
+constexpr size_t kEstSmem = (size_t)kEstGroup * kEstStage * (3 * 8 + 3 * 4);
+
+// The walk's fields of an instance's leading records, in shared memory.
+struct KvStage {
+    long long *slack, *far, *thr;
+    int32_t *bar, *bl, *pmx;
+};
+__device__ __forceinline__ KvStage kv_stage(unsigned char *smem, int g) {
+    KvStage st;
+    long long *b64 = reinterpret_cast<long long *>(smem) + (size_t)g * 3 * kEstStage;
+    st.slack = b64;
+    st.far = b64 + kEstStage;
+    st.thr = b64 + 2 * kEstStage;
+    int32_t *b32 = reinterpret_cast<int32_t *>(reinterpret_cast<long long *>(smem) + (size_t)kEstGroup * 3 * kEstStage) +
+                   (size_t)g * 3 * kEstStage;
+    st.bar = b32;
+    st.bl = b32 + kEstStage;
+    st.pmx = b32 + 2 * kEstStage;
+    return st;
+}
 
 // One instance as the estimate reads it: the first `ns` records (with their admission
 // maxima) from shared memory, the rest from global memory.
@@ -585,15 +606,14 @@ struct KvView {
 };
 
 // Record t of the view; past the records of a finished instance, an empty batch.
-__device__ __forceinline__ void kv_record(const KvView &v, const KvRec *srec, int t, long long &slack,
+__device__ __forceinline__ void kv_record(const KvView &v, const KvStage &st, int t, long long &slack,
                                           long long &far, long long &thr, int &bar, int &bl) {
     if (t < v.ns) {
-        const KvRec &r = srec[t];
-        slack = r.slack;
-        far = r.far;
-        thr = r.thr;
-        bar = r.bar;
-        bl = r.bl;
+        slack = st.slack[t];
+        far = st.far[t];
+        thr = st.thr[t];
+        bar = st.bar[t];
+        bl = st.bl[t];
     } else if (t < v.nrec) {
         const KvRec *r = v.rec + t;
         slack = __ldg(&r->slack);
@@ -633,10 +653,9 @@ __device__ __forceinline__ int kv_lower_bound(const int32_t *a, int lo, int n, i
 // a preempted query recomputes its whole context and may be readmitted in the same
 // batch.  Token counts stay below p + 2 <= 2^31.
 template <int MODE>
-__device__ int kv_candidate(const KvView &v, const KvRec *srec, const int32_t *spmx, int p, long long F[5],
-                            int &lt) {
+__device__ int kv_candidate(const KvView &v, const KvStage &st, int p, long long F[5], int &lt) {
     int lo;
-    if (v.ns > 0 && spmx[v.ns - 1] >= p) lo = kv_lower_bound(spmx, 0, v.ns, p);
+    if (v.ns > 0 && st.pmx[v.ns - 1] >= p) lo = kv_lower_bound(st.pmx, 0, v.ns, p);
     else lo = kv_lower_bound(v.pmx, v.ns, v.nrec - v.ns, p);
     if (lo == v.nrec && !v.done) return kETraj;
     // after the records the instance is empty; the query then needs at most
@@ -650,7 +669,7 @@ __device__ int kv_candidate(const KvView &v, const KvRec *srec, const int32_t *s
         if (t >= limit) return kETraj;
         long long slack, far, thr;
         int bar, bl;
-        kv_record(v, srec, t, slack, far, thr, bar, bl);
+        kv_record(v, st, t, slack, far, thr, bar, bl);
         if (run) {
             if (slack < held) {  // a resident needs the query's blocks
                 pre += ctx;
@@ -698,9 +717,7 @@ __device__ int kv_candidate(const KvView &v, const KvRec *srec, const int32_t *s
     lt = t;
     const int tc = min(t, v.nrec - 1);
     long long cf[4] = {0, 0, 0, 0};
-    if (tc >= 0 && tc < v.ns) {
-        for (int k = 0; k < 4; ++k) cf[k] = srec[tc].cf[k];
-    } else if (tc >= 0) {
+    if (tc >= 0) {
         const KvRec *r = v.rec + tc;
         for (int k = 0; k < 4; ++k) cf[k] = __ldg(&r->cf[k]);
     }
@@ -846,16 +863,14 @@ __global__ void __launch_bounds__(256) k_kv_expand(const KvEst a) {
     }
 }
 
-// CTA: kEstGroup instances, their leading records staged in shared memory.  Each
-// warp takes 32 queries at a time (lane -> query) against every instance of the
-// group, so a query row's kEstGroup estimates leave as one 32-byte sector, and no
-// warp waits for another.
+// CTA: kEstGroup instances, the walk's fields of their leading records staged in
+// shared memory.  The CTAs of a group claim units of (32 queries, one instance),
+// the longest prompts first, so the longest walks start first and no warp holds
+// more than one instance's walks of one block.
 template <int MODE>
 __global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a, bool exact) {
+    extern __shared__ __align__(16) unsigned char est_smem[];
     __shared__ KvView sv[kEstGroup];
-    __shared__ KvRec srec[kEstGroup][kEstStage];
-    __shared__ int32_t spmx[kEstGroup][kEstStage];
-    __shared__ float rows[kEstWarps][32][kEstGroup + 1];
     const DevConfig &c = a.cfg;
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     const int j0 = blockIdx.y * kEstGroup;
@@ -882,69 +897,60 @@ __global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a, b
             v.rec = sb.kvr + (size_t)j * a.kv.horizon;
             v.pmx = sb.kvp + (size_t)j * a.kv.horizon;
             v.ns = min(v.nrec, kEstStage);
-            const int4 *src = reinterpret_cast<const int4 *>(v.rec);
-            int4 *dst = reinterpret_cast<int4 *>(srec[w]);
-            constexpr int kWords = (int)(sizeof(KvRec) / sizeof(int4));
-            for (int e = lane; e < v.ns * kWords; e += 32) dst[e] = __ldg(src + e);
-            for (int e = lane; e < v.ns; e += 32) spmx[w][e] = __ldg(v.pmx + e);
+            const KvStage st = kv_stage(est_smem, w);
+            for (int t = lane; t < v.ns; t += 32) {
+                const KvRec *r = v.rec + t;
+                st.slack[t] = __ldg(&r->slack);
+                st.far[t] = __ldg(&r->far);
+                st.thr[t] = __ldg(&r->thr);
+                st.bar[t] = __ldg(&r->bar);
+                st.bl[t] = __ldg(&r->bl);
+                st.pmx[t] = __ldg(v.pmx + t);
+            }
         }
         if (lane == 0) sv[w] = v;
     }
     __syncthreads();
-    const bool vec = ng == kEstGroup && c.I % 4 == 0 && (reinterpret_cast<uintptr_t>(a.ttft) & 15) == 0;
     // the work: one query per distinct prompt length, or every query, by length
     const int nwork = exact ? *a.nu : a.Q;
     const int32_t *work = exact ? a.leaders : a.order;
-    const int nblk = (nwork + 31) / 32;
+    const int nitems = (nwork + 31) / 32 * ng;
     for (;;) {
-        // the group's warps claim blocks of 32 queries, the longest prompts first
-        int qb = 0;
-        if (lane == 0) qb = atomicAdd(&a.claim[blockIdx.y], 1);
-        qb = __shfl_sync(kFull, qb, 0);
-        if (qb >= nblk) break;
+        int it = 0;
+        if (lane == 0) it = atomicAdd(&a.claim[blockIdx.y], 1);
+        it = __shfl_sync(kFull, it, 0);
+        if (it >= nitems) break;
+        const int qb = it / ng, g = it - qb * ng;
         const int pos = nwork - 1 - (qb * 32 + lane);
-        const bool qv = pos >= 0;
-        const int i = qv ? work[pos] : 0;
-        const int p = qv ? a.prompt[i] : 1;
-        for (int g = 0; g < ng; ++g) {
+        if (pos >= 0) {
+            const int i = work[pos];
+            const int p = a.prompt[i];
             const KvView &v = sv[g];
+            long long F[5] = {-1, -1, -1, -1, -1};
+            int lt = -1;
+            int err;
+            // a query with one output token: its prompt below the context limit and
+            // its first token within the instance's blocks
+            if (active < 0) err = kENoState;
+            else if (!(p >= 1 && p <= c.pmax && (long long)p < v.mctx && kv_blocks32(p + 1, v.bs) <= v.nb))
+                err = kEInval;
+            else err = kv_candidate<MODE>(v, kv_stage(est_smem, g), p, F, lt);
             float tt = kNaN;
-            if (qv) {
-                long long F[5] = {-1, -1, -1, -1, -1};
-                int lt = -1;
-                int err;
-                // a query with one output token: its prompt below the context limit and
-                // its first token within the instance's blocks
-                if (active < 0) err = kENoState;
-                else if (!(p >= 1 && p <= c.pmax && (long long)p < v.mctx && kv_blocks32(p + 1, v.bs) <= v.nb))
-                    err = kEInval;
-                else err = kv_candidate<MODE>(v, srec[g], spmx[g], p, F, lt);
-                if (err) {
-                    record_status(a.ctl, err);
-                    for (int k = 0; k < 5; ++k) F[k] = -1;
-                } else {
-                    tt = __fmul_rn(v.b[0], __ll2float_rn(F[0]));
-                    tt = __fmaf_rn(v.b[2], __ll2float_rn(F[2]), tt);
-                    tt = __fmaf_rn(v.b[1], __ll2float_rn(F[1]), tt);
-                    tt = __fmaf_rn(v.b[3], __ll2float_rn(F[3]), tt);
-                    tt = __fmaf_rn(v.b[4], __ll2float_rn(F[4]), tt);
-                }
-                const size_t idx = (size_t)i * c.I + j0 + g;
-                if (a.first_batch) a.first_batch[idx] = err ? -1 : v.la0 + lt;
-                if (a.features)
-                    for (int k = 0; k < 5; ++k) a.features[idx * 5 + k] = F[k];
-            }
-            rows[w][lane][g] = tt;
-        }
-        if (qv && a.ttft) {
-            float *row = a.ttft + (size_t)i * c.I + j0;
-            const float *r = rows[w][lane];
-            if (vec) {
-                reinterpret_cast<float4 *>(row)[0] = make_float4(r[0], r[1], r[2], r[3]);
-                reinterpret_cast<float4 *>(row)[1] = make_float4(r[4], r[5], r[6], r[7]);
+            if (err) {
+                record_status(a.ctl, err);
+                for (int k = 0; k < 5; ++k) F[k] = -1;
             } else {
-                for (int g = 0; g < ng; ++g) row[g] = r[g];
+                tt = __fmul_rn(v.b[0], __ll2float_rn(F[0]));
+                tt = __fmaf_rn(v.b[2], __ll2float_rn(F[2]), tt);
+                tt = __fmaf_rn(v.b[1], __ll2float_rn(F[1]), tt);
+                tt = __fmaf_rn(v.b[3], __ll2float_rn(F[3]), tt);
+                tt = __fmaf_rn(v.b[4], __ll2float_rn(F[4]), tt);
             }
+            const size_t idx = (size_t)i * c.I + j0 + g;
+            if (a.ttft) a.ttft[idx] = tt;
+            if (a.first_batch) a.first_batch[idx] = err ? -1 : v.la0 + lt;
+            if (a.features)
+                for (int k = 0; k < 5; ++k) a.features[idx * 5 + k] = F[k];
         }
     }
 }
@@ -960,13 +966,17 @@ cudaError_t launch_kv_load(const KvLoad &a, int grid, int warps, size_t smem, cu
 cudaError_t set_kv_smem(size_t bytes) {
     cudaError_t e = cudaFuncSetAttribute(k_kv_load<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_kv_load<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_kv_estimate<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kEstSmem);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_kv_estimate<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kEstSmem);
     return e;
 }
 
 cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st) {
     const int gy = (a.cfg.I + kEstGroup - 1) / kEstGroup;
     const int blocks = (a.Q + 32 * kEstWarps - 1) / (32 * kEstWarps);
-    const int gx = std::max(1, std::min(blocks, (sms * 4 + gy - 1) / gy));
+    const int gx = std::max(1, std::min(blocks, (sms * 3 + gy - 1) / gy));  // three CTAs fit an SM
     const dim3 grid(gx, gy);
     int shift = 0;
     while (2 + ((a.cfg.pmax - 1) >> shift) > kKvBuckets) ++shift;
@@ -976,8 +986,8 @@ cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st) {
     k_kv_count<<<g1, 256, 0, st>>>(a.prompt, a.Q, a.cfg.pmax, shift, a.cnt);
     k_kv_scan<<<1, kScanThreads, 0, st>>>(a.cnt, a.start, a.run, a.uid, a.nu, (nbk + 4095) / 4096 * 4096, a.claim, gy);
     k_kv_scatter<<<g1, 256, 0, st>>>(a.prompt, a.Q, a.cfg.pmax, shift, a.run, a.start, a.uid, a.order, a.leaders);
-    if (a.cfg.mode == 0) k_kv_estimate<0><<<grid, kEstWarps * 32, 0, st>>>(a, exact);
-    else k_kv_estimate<1><<<grid, kEstWarps * 32, 0, st>>>(a, exact);
+    if (a.cfg.mode == 0) k_kv_estimate<0><<<grid, kEstWarps * 32, kEstSmem, st>>>(a, exact);
+    else k_kv_estimate<1><<<grid, kEstWarps * 32, kEstSmem, st>>>(a, exact);
     if (exact) k_kv_expand<<<std::max(1, std::min((a.Q + 7) / 8, sms * 8)), 256, 0, st>>>(a);
     return cudaGetLastError();
 }
