@@ -551,11 +551,14 @@ def run_kv(args, dev, wl, flush):
                        "ctx_limited_instances": int((limits[2] < (1 << 40)).sum()),
                        "blocks_median": int(np.median(limits[1]))},
             "ms_per_step": out["step"], "value": Q * I / (out["step"] * 1e-3), "unit": UNIT, "steps": K,
-            "gpu_launches": 3 * K, "load_ms": out["load"], "estimate_ms": out["estimate"],
+            "gpu_launches": 12 * K, "load_ms": out["load"], "estimate_ms": out["estimate"],
             "estimate_value": Q * I / (out["estimate"] * 1e-3),
-            "roofline": {"kernel": "k_kv_estimate", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+            "roofline": {"kernel": "lr_estimate_ttft with KV limits (count, scan, scatter, k_kv_estimate, "
+                                   "k_kv_expand)", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                          "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
-                         "algorithmic_bytes": nbytes, "traffic": NCU_TRAFFIC.get("k_kv_estimate")}}
+                         "algorithmic_bytes": nbytes, "traffic": None,
+                         "note": "the call's five kernels together; k_kv_estimate alone read 4.92 MB and wrote "
+                                 "0.19 MB per launch (ncu); the load is one dependency chain per instance"}}
 
 
 def run_avgcase(args, dev, wl, flush):
