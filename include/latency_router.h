@@ -155,7 +155,10 @@ LR_API int lr_estimate_features(lr_ctx *ctx, int32_t Q, const int32_t *prompt_le
  *  tau != NULL ([Q] device, seconds): constrained objective (Eq. 3), argmax U over
  *  {j : TTFT <= tau_i}, or the least TTFT when that set is empty; it takes one
  *  lambda (P == 1, else LR_EINVAL), and mu is then unused and may be NULL.
- *  Ties go to the lowest instance index.
+ *  Ties go to the lowest instance index.  A candidate whose TTFT is NaN (no
+ *  estimate: an invalid prompt, or an instance that cannot take the query under
+ *  KV limits) is never chosen; a query with no eligible instance gets assign -1
+ *  and NaN utility and TTFT.
  *  lambda, mu: [P] HOST arrays, finite and >= 0, 1 <= P <= max_pairs.
  *  Outputs, device: assign_out [P][Q] int32, util_out [P][Q] fp32 U of the chosen
  *  instance, ttft_chosen_out [P][Q] fp32 or NULL, frontier_out [P][3] fp64 means of
@@ -242,9 +245,12 @@ LR_API int lr_set_ttft_source(lr_ctx *ctx, int32_t source);
  * int64 in [2, 2^40]: host arrays, copied.  horizon in [1, 2^16].  All three arrays
  * NULL turns the limits off (the default).  The call synchronizes the device and drops
  * the live snapshot: estimates return LR_ENOSTATE until the next lr_load_state.
- * With limits on, lr_route, lr_route_frontier_static, the average-case sources and
- * lr_advance return LR_EINVAL (lr_route_baseline reads only queue lengths and stays
- * open).  Device errors: a snapshot in which a running request other than the last is
+ * With limits on, lr_route and lr_route_frontier_static first write the KV-limited
+ * estimate matrix (to ttft_matrix_out if given, else to library memory) and score
+ * and pick over it; lr_route_baseline reports the chosen instance's KV-limited time;
+ * the average-case sources and lr_advance return LR_EINVAL.  Each estimate call
+ * runs one walk per distinct prompt length (the queries are counting-sorted by
+ * length in library memory sized by max_queries).  Device errors: a snapshot in which a running request other than the last is
  * in prefill, a context has reached max_ctx, the residents hold more blocks than the
  * instance has, or a request's whole context (capped at max_ctx) needs more blocks than
  * the instance has, is LR_ESTATE; a query whose prompt is not below max_ctx, or whose

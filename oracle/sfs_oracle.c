@@ -278,6 +278,7 @@ int orc_route(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instance,
                 const float u = orc_utility(acc[(int64_t)i * M + m], lambda[pp], prompt_len[i],
                                             dec_hat[(int64_t)i * M + m], price_in[m], price_out[m]);
                 const float t = row[j];
+                if (t != t) continue;  /* no estimate (an invalid candidate): not eligible */
                 if (tau == NULL) {
                     /* Eq. 5: argmax_j U - mu * L, ties to the lowest index */
                     const float J = fmaf(-mu[pp], t, u);
@@ -290,6 +291,12 @@ int orc_route(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instance,
             }
             int32_t pick = best_j;
             if (tau != NULL && best_j < 0) pick = fast_j;
+            if (pick < 0) {  /* no eligible instance */
+                assign[(int64_t)pp * Q + i] = -1;
+                util[(int64_t)pp * Q + i] = NAN;
+                if (ttft_chosen) ttft_chosen[(int64_t)pp * Q + i] = NAN;
+                continue;
+            }
             const int32_t m = model_of_instance[pick];
             assign[(int64_t)pp * Q + i] = pick;
             util[(int64_t)pp * Q + i] = orc_utility(acc[(int64_t)i * M + m], lambda[pp], prompt_len[i],

@@ -102,6 +102,9 @@ int orc_estimate_candidates(int32_t num_instances, const int32_t *model_of_insta
 /* Brute-force routing of Q queries given their full TTFT rows ttft[Q][I] (canonical fp32).
  * tau == NULL: Lagrangian objective (Eq. 5) for each of the P (lambda, mu) pairs.
  * tau != NULL: constrained objective (Eq. 3) for each lambda; mu is ignored.
+ * A candidate whose TTFT is NaN (no estimate: an invalid prompt, or an instance that
+ * cannot take the query under KV limits) is not eligible; a query with no eligible
+ * instance gets assign -1 and NaN utility and TTFT.
  * Outputs [P][Q]: assign, util (U of the chosen instance), ttft_chosen. */
 int orc_route(int32_t Q, int32_t I, int32_t M, const int32_t *model_of_instance,
               const float *price_in, const float *price_out, const int32_t *prompt_len,

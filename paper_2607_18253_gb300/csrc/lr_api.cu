@@ -43,6 +43,7 @@ struct lr_ctx {
     size_t kv_smem = 0;
     int32_t *kv_order = nullptr;  // [max_queries] the estimate's query order
     int32_t *kv_leaders = nullptr, *kv_sort = nullptr;  // [max_queries]; [4][kKvBuckets] + 4 + [ceil(I/8)]
+    float *kv_mat = nullptr;  // [max_queries][I] the KV estimate matrix a route scores
     std::vector<void *> kv_allocs;
     std::vector<void *> allocs;
     std::string err;
@@ -100,6 +101,7 @@ void free_kv(lr_ctx *c) {
     c->kv_order = nullptr;
     c->kv_leaders = nullptr;
     c->kv_sort = nullptr;
+    c->kv_mat = nullptr;
     for (int b = 0; b < 2; ++b) {
         c->buf[b].kvi = nullptr;
         c->buf[b].kvr = nullptr;
@@ -476,7 +478,6 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
     if (Q > c->max_queries) return fail(c, LR_ECAPACITY, "Q exceeds max_queries");
     if (P < 1) return fail(c, LR_EINVAL, "P < 1");
     if (P > c->max_pairs) return fail(c, LR_ECAPACITY, "P exceeds max_pairs");
-    if (c->kv_on) return fail(c, LR_EINVAL, "routing with KV-cache limits is not supported");
     if (!c->rt.ok) return fail(c, LR_ECAPACITY, "routing needs num_instances <= 1024 and its tiles in shared memory");
     if (!lambda || (!tau && !mu)) return fail(c, LR_EINVAL, "null lambda / mu");
     if (tau && P != 1) return fail(c, LR_EINVAL, "the constrained objective takes one lambda (P == 1)");
@@ -486,6 +487,14 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
     }
     if (Q == 0) return LR_OK;
     if (!prompt_len || !dec_hat || !acc || !assign_out || !util_out) return fail(c, LR_EINVAL, "null array");
+    float *kv_matrix = nullptr;
+    if (c->kv_on) {
+        // KV limits: the estimate matrix first (into the caller's matrix if asked
+        // for, else library memory), then utility and argmax over it
+        kv_matrix = ttft_matrix_out ? ttft_matrix_out : c->kv_mat;
+        const int rc = estimate_common(c, Q, prompt_len, kv_matrix, nullptr, nullptr, stream);
+        if (rc != LR_OK) return rc;
+    }
     lr::K2Launch a = k2_base(c);
     a.Q = Q;
     a.prompt = prompt_len;
@@ -500,15 +509,19 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
     a.assign = assign_out;
     a.util = util_out;
     a.ttft_chosen = ttft_chosen_out ? ttft_chosen_out : (frontier_out ? c->scratch_tch : nullptr);
-    a.ttft = ttft_matrix_out;
+    a.ttft = kv_matrix ? nullptr : ttft_matrix_out;
+    if (kv_matrix) {
+        a.src = lr::kSrcMatrix;
+        a.ttft_in = kv_matrix;
+    }
     a.Gp = c->rt.Gp;
     a.QS = c->rt.QS;
     a.QT = c->rt.QT;
-    a.vec_ok = (c->cfg.I % 4 == 0) && ((uintptr_t)ttft_matrix_out % 16 == 0);
+    a.vec_ok = (c->cfg.I % 4 == 0) && ((uintptr_t)a.ttft % 16 == 0);
     dim3 grid(std::min(c->sms * c->rt.occ, (Q + a.QS - 1) / a.QS), 1);
     set_row_split(a, c, (int)grid.x, 1, c->rt.occ, stream);
-    cudaError_t e = lr::launch_cand(a, lr::cand_out_flags(ttft_matrix_out != nullptr, false, true, tau != nullptr, P),
-                                    grid, lr::kK2Block, c->rt.smem, (cudaStream_t)stream);
+    cudaError_t e = lr::launch_cand(a, lr::cand_out_flags(a.ttft != nullptr, false, true, tau != nullptr, P), grid,
+                                    lr::kK2Block, c->rt.smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(c, e, "route launch");
     if (frontier_out) {
         e = lr::launch_frontier(a, frontier_out, (cudaStream_t)stream);
@@ -530,6 +543,11 @@ int lr_route_baseline(lr_ctx *c, int32_t policy, int32_t Q, const int32_t *promp
     if (!c->bl_ok) return fail(c, LR_ECAPACITY, "num_instances too large for the baseline policies");
     if (Q == 0) return LR_OK;
     if (!prompt_len || !dec_hat || !acc || !assign_out || !util_out) return fail(c, LR_EINVAL, "null array");
+    if (c->kv_on && ttft_chosen_out) {
+        // the chosen instance's time is read from the KV-limited estimate matrix
+        const int rc = estimate_common(c, Q, prompt_len, c->kv_mat, nullptr, nullptr, stream);
+        if (rc != LR_OK) return rc;
+    }
     lr::K2Launch a = k2_base(c);
     a.Q = Q;
     a.prompt = prompt_len;
@@ -537,6 +555,7 @@ int lr_route_baseline(lr_ctx *c, int32_t policy, int32_t Q, const int32_t *promp
     a.acc = acc;
     a.assign = assign_out;
     a.util = util_out;
+    if (c->kv_on) a.ttft_in = c->kv_mat;
     a.ttft_chosen = ttft_chosen_out;
     const cudaError_t e = lr::launch_baseline(a, policy, (long long)rr_start, lambda, c->sms, (cudaStream_t)stream);
     return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "baseline launch");
@@ -693,10 +712,11 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
         return ee;
     };
     void *bs = nullptr, *nb = nullptr, *mc = nullptr, *kvi[2] = {nullptr, nullptr}, *kvr[2] = {nullptr, nullptr},
-         *kvp[2] = {nullptr, nullptr}, *ord = nullptr, *lead = nullptr, *srt = nullptr;
+         *kvp[2] = {nullptr, nullptr}, *ord = nullptr, *lead = nullptr, *srt = nullptr, *mat = nullptr;
     e = alloc(sizeof(int32_t) * I, &bs);
     if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (size_t)c->max_queries, &ord);
     if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (size_t)c->max_queries, &lead);
+    if (e == cudaSuccess) e = alloc(sizeof(float) * (size_t)c->max_queries * I, &mat);
     const size_t srt_words = 4 * (size_t)lr::kKvBuckets + 4 + (size_t)(I + 7) / 8;
     if (e == cudaSuccess) e = alloc(sizeof(int32_t) * srt_words, &srt);
     if (e == cudaSuccess) e = cudaMemset(srt, 0, sizeof(int32_t) * srt_words);
@@ -726,6 +746,7 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
     c->kv_order = static_cast<int32_t *>(ord);
     c->kv_leaders = static_cast<int32_t *>(lead);
     c->kv_sort = static_cast<int32_t *>(srt);
+    c->kv_mat = static_cast<float *>(mat);
     for (int b = 0; b < 2; ++b) {
         c->buf[b].kvi = static_cast<lr::KvInst *>(kvi[b]);
         c->buf[b].kvr = static_cast<lr::KvRec *>(kvr[b]);

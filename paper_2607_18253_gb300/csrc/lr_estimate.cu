@@ -296,8 +296,8 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     if (threadIdx.x == 0) s_active = load_acquire(&a.ctl->active);
     __syncthreads();
     const int active = s_active;
-    // the LPS source needs no live snapshot; every other source does
-    if (active < 0 && !(AFF && a.src == kSrcLps)) {
+    // the LPS source and a given matrix need no live snapshot; every other source does
+    if (active < 0 && !(AFF && (a.src == kSrcLps || a.src == kSrcMatrix))) {
         if (threadIdx.x == 0) record_status(a.ctl, kENoState);
         for (int k = 0;; ++k) {
             __syncthreads();  // the previous range has been read
@@ -416,9 +416,9 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
             const QueueDev qd = a.qd[j];
             ag[u] = qd.g;
             // throughput source: residents' remaining prefill tokens / theta + Tdec
-            ac[u] = (a.src == kSrcLps)
-                        ? qd.clps
-                        : __double2float_rn(__dadd_rn(__ddiv_rn((double)sb.inst[j].f1tot, qd.theta), qd.tdec));
+            ac[u] = (a.src == kSrcLps)      ? qd.clps
+                    : (a.src == kSrcMatrix) ? 0.f
+                                            : __double2float_rn(__dadd_rn(__ddiv_rn((double)sb.inst[j].f1tot, qd.theta), qd.tdec));
             continue;
         }
         const int col = u * Gp + g;
@@ -507,7 +507,9 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     if (AFF) {
-                        t[u] = __fmaf_rn(q.fp, ag[u], ac[u]);
+                        if (a.src == kSrcMatrix)
+                            t[u] = u < nv ? __ldcs(a.ttft_in + (size_t)(q0 + rr) * I + jb + u) : kNaN;
+                        else t[u] = __fmaf_rn(q.fp, ag[u], ac[u]);
                         kk[u] = 0;
                         continue;
                     }
@@ -559,14 +561,16 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
 #pragma unroll
                             for (int u = 1; u < 4; ++u) {
                                 if ((SPEC || u < nv) && t[u] <= tau && (U[u] > best1 || best1 != best1)) { best1 = U[u]; u1 = u; }
-                                if ((SPEC || u < nv) && t[u] < best2) { best2 = t[u]; u2 = u; }
+                                // a NaN time (no estimate) is never the least
+                                if ((SPEC || u < nv) && t[u] == t[u] && (t[u] < best2 || best2 != best2)) { best2 = t[u]; u2 = u; }
                             }
                         } else {
                             best1 = ((SPEC || 0 < nv) && row_ok) ? __fmaf_rn(-mu, t[0], U[0]) : kNaN;
 #pragma unroll
                             for (int u = 1; u < 4; ++u) {
+                                // J is NaN exactly when the time is (no estimate): never chosen
                                 const float J = __fmaf_rn(-mu, t[u], U[u]);
-                                if ((SPEC || u < nv) && J > best1) { best1 = J; u1 = u; }
+                                if ((SPEC || u < nv) && J == J && (J > best1 || best1 != best1)) { best1 = J; u1 = u; }
                             }
                         }
                         const unsigned k1 = (best1 == best1) ? order_key(best1) : 0u;
@@ -870,13 +874,18 @@ __global__ void __launch_bounds__(256) k_baseline(const K2Launch a, int policy, 
         const int m = c.moi[j];
         const float cost = __fmaf_rn((float)a.dec_hat[(size_t)i * M + m], c.pout[m], __fmul_rn((float)p, c.pin[m]));
         const float U = __fmaf_rn(-lam, cost, a.acc[(size_t)i * M + m]);
-        const InstParams ip = sb.inst[j];
-        const int2 bk = sb.bkt[(size_t)(q.p >> ip.shift) * I + j];
-        const int k = bk.y + (q.p > bk.x ? 1 : 0);
-        const float4 e = reinterpret_cast<const float4 *>(sb.tile + tile_base(c, j))[(size_t)k * 4 * c.tgp + tile_col(c, j)];
         a.assign[i] = j;
         a.util[i] = U;
-        if (a.ttft_chosen) a.ttft_chosen[i] = ttft_exact64<MODE>(c, sb, q, j, k, e);
+        if (a.ttft_chosen && a.ttft_in) {
+            a.ttft_chosen[i] = a.ttft_in[(size_t)i * I + j];  // the KV-limited estimate
+        } else if (a.ttft_chosen) {
+            const InstParams ip = sb.inst[j];
+            const int2 bk = sb.bkt[(size_t)(q.p >> ip.shift) * I + j];
+            const int k = bk.y + (q.p > bk.x ? 1 : 0);
+            const float4 e =
+                reinterpret_cast<const float4 *>(sb.tile + tile_base(c, j))[(size_t)k * 4 * c.tgp + tile_col(c, j)];
+            a.ttft_chosen[i] = ttft_exact64<MODE>(c, sb, q, j, k, e);
+        }
     }
 }
 

@@ -234,7 +234,9 @@ __host__ __device__ inline size_t trajectory_smem_per_warp(const DevConfig &c) {
 
 // Average-case TTFT sources (Sec. 4, App. E): per-instance parameters as given
 // and the derived constants of t = fma(p, g, C).
-enum : int { kSrcSfs = 0, kSrcThroughput = 1, kSrcLps = 2 };
+// kSrcMatrix (internal): the times come from a [Q][I] matrix already computed (the
+// KV-limited estimate), read by the candidate kernel's affine mode
+enum : int { kSrcSfs = 0, kSrcThroughput = 1, kSrcLps = 2, kSrcMatrix = 3 };
 struct QueueRaw {      // 64 bytes, copied from the caller's arrays
     double theta, tdec, alpha, mu, ca2, cs2;
     int32_t k, has_lps;
@@ -274,6 +276,7 @@ struct K2Launch {
     // TTFT source (kSrc*) and, for the average-case ones, the instance constants
     int32_t src;
     const QueueDev *qd;
+    const float *ttft_in;  // kSrcMatrix: [Q][I]
     // [0]: CTAs finished; [1 + tile]: query rows of the tile claimed past the static
     // ones.  Zero before a launch; the last CTA to finish clears them for the next.
     uint32_t *work;

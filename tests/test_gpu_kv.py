@@ -172,25 +172,99 @@ def test_invalid_snapshot_keeps_the_live_one():
     rt.close()
 
 
+def _route_pool(seed, mode, nq=200):
+    wl = W.small_workload(seed, num_instances=24, num_models=3, num_queries=nq, first_token_mode=mode,
+                          budget_range=(8, 96), min_gap=8)
+    bs, nb, mc = W.kv_limits(wl, seed, block_sizes=(1, 4, 16))
+    # an idle instance whose context limit a third of the prompts reach: rows mixing
+    # candidates with and without an estimate
+    wl.n_run[0] = 0
+    wl.n_wait[0] = 0
+    mc[0] = int(np.percentile(wl.prompt_len, 66))
+    return wl, (bs, nb, mc)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_route_under_limits(mode):
+    # Eq. 5 and Eq. 3 over the KV estimate matrix: assignments exact, utility and
+    # chosen time bit for bit against the oracle's argmax over its own KV matrix, a
+    # candidate without an estimate never chosen
+    wl, limits = _route_pool(70 + mode, mode)
+    rt = make(wl, limits, max_pairs=32)
+    p, dh, acc, tau = R().query_tensors(wl)
+    st, _, _, et, _ = oracle.estimate_matrix_kv(wl, *limits)
+    assert (st[:, 0] != 0).any() and (st[:, 0] == 0).any()
+    mat = torch.empty((wl.num_queries, wl.num_instances), dtype=torch.float32, device="cuda")
+    lam, mu = [float(wl.lam[0])], [float(wl.mu[0])]
+    o = rt.route(p, dh, acc, lam, mu, ttft_matrix=mat)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(bits(mat.cpu().numpy()), bits(et))
+    a, u, tc = oracle.route(wl, et, lam=np.array(lam, np.float32), mu=np.array(mu, np.float32))
+    np.testing.assert_array_equal(o["assign"].cpu().numpy(), a)
+    np.testing.assert_array_equal(bits(o["util"].cpu().numpy()), bits(u))
+    np.testing.assert_array_equal(bits(o["ttft_chosen"].cpu().numpy()), bits(tc))
+    assert (a[0] != 0).all() or np.isfinite(et[a[0] == 0, 0]).all()
+    # the constrained objective, without a matrix output (library memory)
+    oc = rt.route(p, dh, acc, lam, None, tau=tau)
+    torch.cuda.synchronize()
+    ac, uc, tcc = oracle.route(wl, et, lam=np.array(lam, np.float32), tau=wl.tau)
+    np.testing.assert_array_equal(oc["assign"].cpu().numpy(), ac)
+    np.testing.assert_array_equal(bits(oc["util"].cpu().numpy()), bits(uc))
+    np.testing.assert_array_equal(bits(oc["ttft_chosen"].cpu().numpy()), bits(tcc))
+    # a 32-pair sweep
+    lam_s, mu_s = W.sweep_pairs()
+    os_ = rt.route(p, dh, acc, lam_s, mu_s)
+    torch.cuda.synchronize()
+    asw, usw, _ = oracle.route(wl, et, lam=lam_s, mu=mu_s)
+    np.testing.assert_array_equal(os_["assign"].cpu().numpy(), asw)
+    np.testing.assert_array_equal(bits(os_["util"].cpu().numpy()), bits(usw))
+    assert rt.status() == R().LR_EINVAL  # the candidates without an estimate
+    rt.close()
+
+
+def test_route_under_limits_no_eligible_instance():
+    # a row whose every candidate lacks an estimate gets -1 and NaN
+    wl = W.small_workload(72, num_instances=4, num_models=2, num_queries=30, budget_range=(8, 96), min_gap=8)
+    bs, nb, mc = W.kv_limits(wl, 15, block_sizes=(4,))
+    wl.n_run[:] = 0
+    wl.n_wait[:] = 0
+    mc[:] = int(np.median(wl.prompt_len))
+    rt = make(wl, (bs, nb, mc))
+    p, dh, acc, tau = R().query_tensors(wl)
+    o = rt.route(p, dh, acc, [1.0], [0.1])
+    torch.cuda.synchronize()
+    st, _, _, et, _ = oracle.estimate_matrix_kv(wl, bs, nb, mc)
+    a, u, tc = oracle.route(wl, et, lam=np.array([1.0], np.float32), mu=np.array([0.1], np.float32))
+    none = (st != 0).all(axis=1)
+    assert none.any() and (~none).any()
+    np.testing.assert_array_equal(o["assign"].cpu().numpy(), a)
+    assert (a[0, none] == -1).all() and np.isnan(u[0, none]).all()
+    np.testing.assert_array_equal(bits(o["util"].cpu().numpy()), bits(u))
+    np.testing.assert_array_equal(bits(o["ttft_chosen"].cpu().numpy()), bits(tc))
+    rt.close()
+
+
 def test_calls_closed_with_limits_and_turning_them_off():
     wl = W.small_workload(64, num_instances=8, num_models=2, num_queries=16, budget_range=(8, 96), min_gap=8)
     limits = W.kv_limits(wl, 10)
     rt = make(wl, limits)
     p, dh, acc, tau = R().query_tensors(wl)
     with pytest.raises(R().LRError) as e:
-        rt.route(p, dh, acc, [1.0], [0.1])
-    assert e.value.code == R().LR_EINVAL
-    with pytest.raises(R().LRError) as e:
         rt.set_ttft_source(R().LR_TTFT_THROUGHPUT)
     assert e.value.code == R().LR_EINVAL
     with pytest.raises(R().LRError) as e:
         rt.advance(torch.zeros(16, dtype=torch.int32, device="cuda"), p, dh, 0.0)
     assert e.value.code == R().LR_EINVAL
-    # the queue-length baselines stay open
-    o = rt.route_baseline(R().LR_POLICY_SHORTEST_QUEUE, p, dh, acc, 1.0, 0)
-    torch.cuda.synchronize()
-    ea, _, _ = oracle.baseline_route(wl, R().LR_POLICY_SHORTEST_QUEUE, 1.0, 0)
-    np.testing.assert_array_equal(o["assign"].cpu().numpy(), ea)
+    # the baselines: their choices, with the chosen instance's KV-limited time
+    _, _, _, et, _ = oracle.estimate_matrix_kv(wl, *limits)
+    for pol in (R().LR_POLICY_ROUND_ROBIN, R().LR_POLICY_SHORTEST_QUEUE, R().LR_POLICY_LATENCY_AGNOSTIC):
+        o = rt.route_baseline(pol, p, dh, acc, 1.0, 3)
+        torch.cuda.synchronize()
+        ea, eu, _ = oracle.baseline_route(wl, pol, 1.0, 3)
+        got = o["assign"].cpu().numpy()
+        np.testing.assert_array_equal(got, ea)
+        np.testing.assert_array_equal(bits(o["util"].cpu().numpy()), bits(eu))
+        np.testing.assert_array_equal(bits(o["ttft_chosen"].cpu().numpy()), bits(et[np.arange(len(got)), got]))
     # turning the limits off drops the snapshot; a new load gives the plain estimate
     rt.set_kv_limits()
     t, _, _ = gpu_estimate(rt, wl)

@@ -150,3 +150,33 @@ def test_candidate_matrix_matches_single_candidates(mode):
             changed += int(lts != lt0[i, j] or not np.array_equal(Fs, F0[i, j]))
     assert (st[:, 0] != 0).any() and (st[:, 0] == 0).any()
     assert changed > 0  # the generated limits bind somewhere
+
+
+def test_route_skips_candidates_without_an_estimate():
+    # a NaN time (no estimate) is not eligible: on rows with a finite time the choice
+    # equals the choice with NaN read as an infinite time (never preferred under
+    # Eq. 5 with mu > 0, never within a target under Eq. 3, never the least); a row
+    # with no finite time gets -1 and NaN
+    from paper_2607_18253_gb300 import workloads as W
+    wl = W.small_workload(80, num_instances=9, num_queries=40)
+    rng = np.random.default_rng(2)
+    t = rng.uniform(0.05, 2.0, (40, 9)).astype(np.float32)
+    t[rng.random(t.shape) < 0.3] = np.nan
+    t[:, 0] = np.nan       # the lowest index never has a time
+    t[5, :] = np.nan       # nor does any instance of row 5
+    inf = np.where(np.isnan(t), np.float32(np.inf), t)
+    lam = np.array([0.5], np.float32)
+    for mu in (np.array([0.2], np.float32), np.array([3.0], np.float32)):
+        a, u, tc = oracle.route(wl, t, lam=lam, mu=mu)
+        ai, ui, tci = oracle.route(wl, inf, lam=lam, mu=mu)
+        ok = ~np.isnan(t).all(axis=1)
+        np.testing.assert_array_equal(a[0, ok], ai[0, ok])
+        np.testing.assert_array_equal(u[0, ok], ui[0, ok])
+        assert (a[0, ~ok] == -1).all() and np.isnan(u[0, ~ok]).all() and np.isnan(tc[0, ~ok]).all()
+        assert not (a[0] == 0).any()
+    tau = np.full(40, 0.6, np.float32)
+    a, u, tc = oracle.route(wl, t, lam=lam, tau=tau)
+    ai, _, _ = oracle.route(wl, inf, lam=lam, tau=tau)
+    ok = ~np.isnan(t).all(axis=1)
+    np.testing.assert_array_equal(a[0, ok], ai[0, ok])
+    assert (a[0, ~ok] == -1).all() and not (a[0] == 0).any()
