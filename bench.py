@@ -36,7 +36,7 @@ WORKLOAD = "pool256"
 # DRAM bytes (read + write) per launch of the step's kernels on this workload, from one
 # ncu capture of the kernels as they are built now (summaries under profiles/); they
 # are retaken whenever one of the kernels changes.
-NCU_TRAFFIC = {"k_route": 4_585_216 + 8_863_744, "k_trajectory": 1_392_896, "k_estimate": 357_632 + 7_219_456}
+NCU_TRAFFIC = {"k_route": 4_579_328 + 8_607_488, "k_trajectory": 1_392_896, "k_estimate": 357_376 + 7_084_800}
 
 
 def _peaks():

@@ -561,16 +561,24 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
 #pragma unroll
                             for (int u = 1; u < 4; ++u) {
                                 if ((SPEC || u < nv) && t[u] <= tau && (U[u] > best1 || best1 != best1)) { best1 = U[u]; u1 = u; }
-                                // a NaN time (no estimate) is never the least
-                                if ((SPEC || u < nv) && t[u] == t[u] && (t[u] < best2 || best2 != best2)) { best2 = t[u]; u2 = u; }
+                                // a NaN time (no estimate, per candidate only from a matrix
+                                // source) is never the least
+                                if ((SPEC || u < nv) && (!AFF || t[u] == t[u]) && (t[u] < best2 || (AFF && best2 != best2))) {
+                                    best2 = t[u];
+                                    u2 = u;
+                                }
                             }
                         } else {
                             best1 = ((SPEC || 0 < nv) && row_ok) ? __fmaf_rn(-mu, t[0], U[0]) : kNaN;
 #pragma unroll
                             for (int u = 1; u < 4; ++u) {
-                                // J is NaN exactly when the time is (no estimate): never chosen
+                                // J is NaN exactly when the time is (no estimate): never chosen.
+                                // Only a matrix source mixes NaN and finite times in a row.
                                 const float J = __fmaf_rn(-mu, t[u], U[u]);
-                                if ((SPEC || u < nv) && J == J && (J > best1 || best1 != best1)) { best1 = J; u1 = u; }
+                                if ((SPEC || u < nv) && (!AFF || J == J) && (J > best1 || (AFF && best1 != best1))) {
+                                    best1 = J;
+                                    u1 = u;
+                                }
                             }
                         }
                         const unsigned k1 = (best1 == best1) ? order_key(best1) : 0u;
