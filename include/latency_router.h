@@ -250,7 +250,10 @@ LR_API int lr_set_ttft_source(lr_ctx *ctx, int32_t source);
  * and pick over it; lr_route_baseline reports the chosen instance's KV-limited time;
  * the average-case sources and lr_advance return LR_EINVAL.  Each estimate call
  * runs one walk per distinct prompt length (the queries are counting-sorted by
- * length in library memory sized by max_queries).  Device errors: a snapshot in which a running request other than the last is
+ * length in library memory sized by max_queries).  Memory taken here: per buffer
+ * 68 B x I x horizon of records, and max_queries x (8 B + 4 B x I) for the sort
+ * and the routed matrix (LR_ENOMEM if it cannot be had; nothing is allocated
+ * later, so routing stays allocation-free).  Device errors: a snapshot in which a running request other than the last is
  * in prefill, a context has reached max_ctx, the residents hold more blocks than the
  * instance has, or a request's whole context (capped at max_ctx) needs more blocks than
  * the instance has, is LR_ESTATE; a query whose prompt is not below max_ctx, or whose
