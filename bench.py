@@ -480,7 +480,7 @@ def run_estimate(args, dev, wl, flush):
 
 KV_SEED = 11
 KV_BLOCK = 16
-KV_HORIZON = 1024
+KV_HORIZON = 4096
 
 
 def run_kv(args, dev, wl, flush):

@@ -238,6 +238,135 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
         __syncwarp();
     };
 
+    // Up to 32 batches at once, lane k taking batch G + k, while no resident waits
+    // (after the first record): then a batch admits nobody, and all it depends on is
+    // known at the window's start -- the decoders ending in it (the calendar), those
+    // crossing into a new block (the histogram, less the earlier ends of the
+    // window), the prefill request's chunk (the budget the decoders leave, summed)
+    // and the free blocks (needs and returns, summed).  The window stops before a
+    // batch that preempts or in which the prefill request finishes (both taken by
+    // the batch step), at a re-file boundary, at the horizon, and after the batch
+    // that empties the instance.  The window's ends are listed in the idle waiting
+    // ring.  Returns the batches done (0: none).
+    int32_t *evn = ovf + 1;  // the window's ends
+    auto window = [&]() -> int {
+        const int W = min(min(32, a.kv.horizon - nrec), kKvCal - (G & (kKvCal - 1)));
+        if (lane == 0) *evn = 0;
+        __syncwarp();
+        const int k = lane;
+        int cntk = 0;
+        long long rck = 0, ebk = 0;
+        if (k < W) {
+            for (int s = head[(G + k) & (kKvCal - 1)]; s >= 0;) {
+                const int ns = nxt[s];
+                const int4 q = rq[s];
+                if (q.y == 0) {
+                    ++cntk;
+                    rck += q.x;
+                    ebk += eb[s];
+                    wq[atomicAdd(evn, 1)] = make_int2(k, s);
+                }
+                s = ns;
+            }
+        }
+        __syncwarp();
+        const int nev = *evn;
+        const int endsb = warp_incl_sum32(cntk, lane) - cntk;  // ends before batch k
+        const long long rcb = warp_incl_sum64(rck, lane) - rck;
+        const int ndk = nd - endsb, nrk = nr - endsb;
+        const long long srck = src - rcb;
+        // decoders at a block boundary in batch G + k, the window's earlier ends removed
+        const int gk = (gr + k) % bs;
+        const int rk = gk == 0 ? 0 : bs - gk;
+        int sub = 0;
+        for (int e = 0; e < nev; ++e) {
+            const int2 ev = wq[e];
+            if (ev.x < k && rq[ev.y].w == rk) ++sub;
+        }
+        const int need_d = ndk > 0 ? hist[rk] - sub : 0;
+        // the prefill request's chunk: what the decoders leave, until it finishes
+        int x = 0, pneed = 0, ctxp = 0, remk = 0;
+        bool pf_ends = false;
+        const int4 pq = pfs >= 0 ? rq[pfs] : make_int4(0, 0, 0, 0);
+        if (pfs >= 0) {
+            const int avail = B - ndk;
+            const int before = warp_incl_sum32(k < W ? avail : 0, lane) - (k < W ? avail : 0);
+            remk = max(0, pq.y - before);
+            x = min(remk, avail);
+            pf_ends = remk - x == 0;
+            ctxp = pq.x + (pq.y - remk);
+            pneed = kv_blocks32(ctxp + x, bs) - kv_blocks32(ctxp, bs);
+        }
+        const int need_all = need_d + pneed;
+        const long long dl = k < W ? ebk - need_all : 0;       // free blocks gained over batch k
+        const long long fb = freeb + warp_incl_sum64(dl, lane) - dl;  // free blocks before batch k
+        const unsigned okm = __ballot_sync(kFull, k < W && !pf_ends && need_all <= fb);
+        int n = okm == kFull ? 32 : __ffs(~okm) - 1;
+        const unsigned em = __ballot_sync(kFull, k < n && nrk - cntk == 0);  // the instance empties
+        if (em) n = __ffs(em);
+        if (n == 0) return 0;
+        const bool in = k < n;
+        const long long fa = fb - need_all;
+        const int bar = B - ndk - x;
+        const long long c1 = cf1 + warp_incl_sum64(in ? x : 0, lane);
+        const long long c2 = cf2 + warp_incl_sum64(in ? ndk : 0, lane);
+        const long long c3 = cf3 + warp_incl_sum64(in ? srck + (long long)ndk * (G + k) : 0, lane);
+        const long long c4 = cf4 + warp_incl_sum64(in ? (long long)x * ctxp + (long long)x * (x + 1) / 2 : 0, lane);
+        long long thr = 0;
+        if (in && bar > 0 && nrk < S) thr = ((long long)bar <= fa * bs) ? kHuge : fa * bs;
+        int pm = max(pmx, (int)min(thr, (long long)INT32_MAX));
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(kFull, pm, o);
+            if (lane >= o) pm = max(pm, y);
+        }
+        if (in) {
+            KvRec R;
+            R.cf[0] = c1;
+            R.cf[1] = c2;
+            R.cf[2] = c3;
+            R.cf[3] = c4;
+            R.slack = fa;  // nrk > 0: the window never starts on an empty instance
+            R.far = fa;
+            R.thr = thr;
+            R.bar = bar;
+            R.bl = bar;
+            rec[nrec + k] = R;
+            pmxo[nrec + k] = pm;
+        }
+        // the state after batch n - 1
+        const int L = n - 1;
+        const int ndL = __shfl_sync(kFull, ndk, L), nrL = __shfl_sync(kFull, nrk, L), cntL = __shfl_sync(kFull, cntk, L);
+        const long long srcL = __shfl_sync(kFull, srck, L), rckL = __shfl_sync(kFull, rck, L);
+        const long long fbL = __shfl_sync(kFull, fb, L), dlL = __shfl_sync(kFull, dl, L);
+        const int xL = __shfl_sync(kFull, x, L), ctxpL = __shfl_sync(kFull, ctxp, L), remL = __shfl_sync(kFull, remk, L);
+        cf1 = __shfl_sync(kFull, c1, L);
+        cf2 = __shfl_sync(kFull, c2, L);
+        cf3 = __shfl_sync(kFull, c3, L);
+        cf4 = __shfl_sync(kFull, c4, L);
+        pmx = __shfl_sync(kFull, pm, L);
+        __syncwarp();
+        for (int e = lane; e < nev; e += 32) {  // the window's ends leave
+            const int2 ev = wq[e];
+            if (ev.x < n) {
+                atomicSub(&hist[rq[ev.y].w], 1);
+                reinterpret_cast<int *>(rq + ev.y)[1] = -1;
+            }
+        }
+        if (in) head[(G + k) & (kKvCal - 1)] = -1;
+        if (pfs >= 0 && lane == 0) rq[pfs] = make_int4(ctxpL + xL, remL - xL, pq.z, kv_blocks32(ctxpL + xL, bs));
+        nd = ndL - cntL;
+        nr = nrL - cntL;
+        src = srcL - rckL;
+        freeb = fbL + dlL;
+        nrec += n;
+        G += n;
+        gr = G % bs;
+        if (nr == 0) done = 1;
+        __syncwarp();
+        return n;
+    };
+
     for (int l = 1;; ++l) {
         if (l > c.max_iters) {
             kv_fail(a.ctl, kETraj, lane);
@@ -261,6 +390,15 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
                 *ovf = keep;
             }
             __syncwarp();
+        }
+        if (la0 != 0 && wc == 0) {
+            const int n = window();
+            if (n > 0) {
+                l += n - 1;
+                if (done || nrec == a.kv.horizon) break;
+                if (ne - nr >= max(32, nr)) compact();
+                continue;
+            }
         }
         // 1. The running scan.  n_run <= S <= B and only the last request may be in
         //    prefill, so every request gets its tokens if the blocks suffice: one per
