@@ -326,3 +326,38 @@ def test_many_duplicate_lengths():
     np.testing.assert_array_equal(bits(t_only), bits(got[0]))
     st, eF, elt, et, _ = oracle.estimate_matrix_kv(wl, *limits)
     compare(got, (eF, elt, et), st == 0)
+
+
+def test_hand_trace_with_residents_preempting_each_other():
+    # the worked trace of tests/golden/kv_hand_trace_residents.json on the GPU: one
+    # instance, the query of the trace twice (one walk, a copied row) and a longer one
+    import json
+    import os
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "kv_hand_trace_residents.json")))
+    wl = W.small_workload(90, num_instances=1, num_models=1, num_queries=3, cap_running=8, cap_waiting=8,
+                          first_token_mode=g["mode"])
+    wl.max_batched_tokens[:] = g["B"]
+    wl.max_seqs[:] = g["S"]
+    wl.n_run[:] = len(g["running"])
+    wl.run_ctx[:] = 0
+    wl.run_pre[:] = 0
+    wl.run_dec[:] = 0
+    for r, (c_, p_, d_) in enumerate(g["running"]):
+        wl.run_ctx[0, r], wl.run_pre[0, r], wl.run_dec[0, r] = c_, p_, d_
+    wl.n_wait[:] = len(g["waiting"])
+    wl.wait_pre[:] = 0
+    wl.wait_dec[:] = 0
+    for r, (p_, d_) in enumerate(g["waiting"]):
+        wl.wait_pre[0, r], wl.wait_dec[0, r] = p_, d_
+    wl.prompt_len = np.array([g["query"][0], g["query"][0], 3], np.int32)
+    limits = (np.array([g["block_size"]], np.int32), np.array([g["num_blocks"]], np.int64),
+              np.array([g["max_ctx"]], np.int64))
+    rt = make(wl, limits)
+    t, fb, F = gpu_estimate(rt, wl)
+    assert rt.status() == R().LR_OK
+    rt.close()
+    for row in (0, 1):
+        assert F[row, 0].tolist() == g["F"] and fb[row, 0] == g["first_token_batch"]
+    st, eF, elt, et, _ = oracle.estimate_matrix_kv(wl, *limits)
+    assert (st == 0).all()
+    compare((t, fb, F), (eF, elt, et), np.ones(st.shape, bool))

@@ -52,6 +52,22 @@ def test_hand_trace_with_a_preemption_of_the_query():
     assert la == g["admit_batch"] and lt == g["first_token_batch"] and used == g["most_blocks_in_use"]
 
 
+def test_hand_trace_with_residents_preempting_each_other():
+    # a resident preempting itself and readmitted in the same batch, one preempted
+    # by an older one, a partial chunk, and the query admitted once the instance
+    # drains (tests/golden/kv_hand_trace_residents.json); the residents' own
+    # batches are also those of the residents alone
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "kv_hand_trace_residents.json")))
+    args = (g["running"], g["waiting"], g["B"], g["S"])
+    kw = dict(block_size=g["block_size"], num_blocks=g["num_blocks"], max_ctx=g["max_ctx"], mode=g["mode"])
+    F, la, lt, res, used = oracle.simulate_kv(*args, *g["query"], **kw)
+    np.testing.assert_array_equal(F, g["F"])
+    assert la == g["admit_batch"] and lt == g["first_token_batch"] and used == g["most_blocks_in_use"]
+    np.testing.assert_array_equal(res, g["residents_per_batch"])
+    alone = oracle.kv_residents(*args, lt, **kw)
+    np.testing.assert_array_equal(alone, g["residents_per_batch"])
+
+
 def test_context_limit_is_a_shorter_response():
     # a decoder at context 60 under a limit of 62 decodes twice, exactly like one
     # with two tokens left and no limit
