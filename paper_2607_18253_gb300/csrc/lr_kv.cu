@@ -21,7 +21,10 @@
 // (k_kv_estimate) then finds each (query, instance) candidate's admission batch by
 // a binary search over the running maximum of the admission bounds and follows it
 // from there, record by record, through prefill chunks, preemptions and
-// readmissions, to its first token.
+// readmissions, to its first token.  A candidate depends only on the instance and
+// the prompt length, so each call first counting-sorts its queries by length
+// (k_kv_count, k_kv_scan, k_kv_scatter), walks once per distinct length, and
+// copies those rows to the other queries of the same length (k_kv_expand).
 #include "lr_internal.cuh"
 
 namespace lr {
@@ -94,14 +97,14 @@ __device__ __forceinline__ int kv_res(int x, int bs) {
 // Running request in slot s: rq[s] = (context, prefill, decode, blocks held) for
 // the prefill request, (context - G, 0, decode + G, context residue mod bs) for a
 // decoder, whose blocks at its end wait in eb[s].  Slots keep the list's order; a
-// request that leaves becomes a hole (prefill -1) until a compaction.  Only the last running request may be in prefill (slot pfs); it holds
-// its values as they are.  The others decode one token a batch, so they hold
-// context - G and decode + G (G = batches done) and no word of theirs changes until
-// they end.  The decoders crossing into a new block in batch G are those whose
-// context is a multiple of bs, counted by a histogram of stored contexts mod bs;
-// their context sum (Eq. 9's F3 term) is a running total; the batch each one ends in
-// (decode count or context limit) waits in the end calendar.  A request that ends
-// frees ceil(context / bs) blocks after its last batch.
+// request that leaves becomes a hole (prefill -1) until a compaction.  Only the
+// last running request may be in prefill (slot pfs).  The others decode one token
+// a batch (G = batches done), so no word of theirs changes until they end.  The
+// decoders crossing into a new block in batch G are those whose context is a
+// multiple of bs, counted by a histogram of stored contexts mod bs; their context
+// sum (Eq. 9's F3 term) is a running total; the batch each one ends in (decode
+// count or context limit) waits in the end calendar.  A request that ends frees
+// ceil(context / bs) blocks after its last batch.
 template <int MODE>
 __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lane, int32_t *wb) {
     const DevConfig &c = a.cfg;
