@@ -53,14 +53,14 @@ enum lr_code {
     LR_ENOSTATE = 7     /* no snapshot has been loaded successfully yet (device) */
 };
 
-/* When the first output token is produced (Sec. 4.1: the decode stage begins only
- * after all prefill tokens have been processed). */
+/* When the first output token is produced (Sec. 4.1: decoding starts once every
+ * prompt token has been processed). */
 enum lr_first_token_mode {
     LR_FIRST_TOKEN_SEPARATE_DECODE = 0,  /* its own decode batch after the last prefill chunk (default) */
     LR_FIRST_TOKEN_WITH_LAST_CHUNK = 1   /* sampled in the batch that completes the prompt */
 };
 
-/* Pool description (Sec. 3 "System model"; Eq. 9 coefficients; App. B.4 prices). */
+/* Pool description (Sec. 3, the system model; Eq. 9 coefficients; App. B.4 prices). */
 typedef struct {
     int32_t num_instances;             /* I >= 1 model instances j */
     int32_t num_models;                /* M >= 1 distinct models */
@@ -84,8 +84,8 @@ typedef struct {
     int32_t max_iters;                 /* bound on simulation steps per instance and load */
 } lr_config;
 
-/* One snapshot of every instance (Sec. 4 "Setup": resident set R_j = Q_j u A_j with
- * remaining prefill and predicted decode tokens; App. F "Query workload snapshots").
+/* One snapshot of every instance (Sec. 4 setup: resident set R_j = Q_j u A_j with
+ * remaining prefill and predicted decode tokens; App. F on workload snapshots).
  * DEVICE pointers.  Per-instance arrays are [I]; per-request arrays are
  * [I][cap] with row stride cap_running / cap_waiting; entries beyond a row's
  * count are ignored.
@@ -312,7 +312,7 @@ LR_API const char *lr_strerror(int code);
  * validation that failed); empty if none.  Valid until the next call on ctx. */
 LR_API const char *lr_last_error(const lr_ctx *ctx);
 
-/* ---- Baseline routing policies and stream metrics (Sec. 6 "Baselines"; Eq. 4) ---- */
+/* ---- Baseline routing policies and stream metrics (Sec. 6 baselines; Eq. 4) ---- */
 
 enum lr_policy {
     LR_POLICY_ROUND_ROBIN = 0,      /* query i -> instance (rr_start + i) mod I */
@@ -320,7 +320,7 @@ enum lr_policy {
     LR_POLICY_LATENCY_AGNOSTIC = 2  /* largest utility U (Eq. 2), latency ignored */
 };
 
-/* The paper's baseline routers (Sec. 6 "Baselines"), for comparison with lr_route.
+/* The paper's baseline routers (Sec. 6), for comparison with lr_route.
  * Round Robin assigns cyclically; Shortest Queue lets the Q queries, in order, each
  * join the instance with the fewest resident requests of the live snapshot, counting
  * the queries routed before it in this call (ties: lowest index); Latency-Agnostic

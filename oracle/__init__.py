@@ -234,7 +234,7 @@ def advance(wl, clock, assign, prompt_len, dec, t_now: float, max_batches: int =
 
 
 # ---------------------------------------------------------------------------
-# Average-case estimators (Sec. 4 "Average-case TTFT estimation"; App. E)
+# Average-case estimators (Sec. 4, average-case TTFT estimation; App. E)
 
 def pow_int(x: float, k: int) -> float:
     """x**k by binary exponentiation in fp64 (the order both sides use)."""

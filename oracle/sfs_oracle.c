@@ -18,10 +18,12 @@
  *    prefill chunk of min(prompt, budget).  Requests whose decode count reaches
  *    zero leave after the batch.
  *  - First output token: by default a separate decode batch after the last
- *    prefill chunk (Sec. 4.1 "the decode stage ... begins only after all
- *    prefill tokens"); optionally sampled in the batch of the last chunk.
+ *    prefill chunk (Sec. 4.1: decoding starts once every prompt token has been
+ *    processed); optionally sampled in the batch of the last chunk.
  *  - Context of a decode token = tokens in the KV cache before the batch.
- *  - KV capacity is unbounded and nothing is preempted.
+ *  - orc_sfs_candidate: KV capacity is unbounded and nothing is preempted;
+ *    orc_sfs_candidate_kv adds block and context limits with preemption (the
+ *    reading stated before kv_sim below).
  *  - Canonical fp32 order for Eq. 9 summed over batches: intercept, decode
  *    tokens, prefill tokens, decode context, prefill attention.
  *
@@ -458,7 +460,7 @@ int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, 
 }
 
 /* ------------------------------------------------------------------------- */
-/* Average-case estimators (Sec. 4 "Average-case TTFT estimation"; App. E).   */
+/* Average-case estimators (Sec. 4, average-case TTFT estimation; App. E).   */
 
 double orc_pow_int(double x, int32_t k)
 {

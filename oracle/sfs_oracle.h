@@ -134,7 +134,7 @@ int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, 
 /* Utility of Eq. 2 with the cost of App. B.4 in canonical fp32. */
 float orc_utility(float acc, float lambda, int32_t p, int32_t dec_hat, float price_in, float price_out);
 
-/* ---- Average-case TTFT estimators (Sec. 4 "Average-case TTFT estimation"; App. E) ---- */
+/* ---- Average-case TTFT estimators (Sec. 4, average-case TTFT estimation; App. E) ---- */
 
 /* x^k for an integer k >= 0 by binary exponentiation (bits of k from the least
  * significant; a fixed sequence of IEEE products). */

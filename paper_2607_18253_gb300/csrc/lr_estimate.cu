@@ -762,7 +762,7 @@ __global__ void k_queue_params(int I, const QueueRaw *raw, QueueDev *qd) {
 }
 
 // ---------------------------------------------------------------------------
-// Baseline routing policies (Sec. 6 "Baselines"): the instance is chosen without the
+// Baseline routing policies (Sec. 6, the baselines): the instance is chosen without the
 // latency estimates, and the chosen candidate's utility (Eq. 2) and SFS TTFT estimate
 // are reported beside it (the TTFT through the same exact path as the candidate
 // kernel's, so the two agree bit for bit).  One thread per query.
