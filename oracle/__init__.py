@@ -273,8 +273,8 @@ def avgcase_matrix(wl, W, theta, tdec):
 
 
 # ---------------------------------------------------------------------------
-# Calibration of the batch-time model (Sec. 4.1, "Token-batch processing time
-# estimator": the coefficients are calibrated from observed batch times)
+# Calibration of the batch-time model (Sec. 4.1, the token-batch time estimator:
+# the coefficients are calibrated from observed batch times)
 
 def calibrate(features, model, time, num_models: int, shared_beta1: bool = True) -> np.ndarray:
     """Least-squares Eq. 9 coefficients per model from per-batch (F, observed time) rows.

@@ -6,7 +6,7 @@ CUDA path and the CPU oracle consume the arrays it returns, so they always see
 identical bytes.
 
 Shapes follow the paper's setting: model instances with a running set and an
-FCFS waiting queue (Sec. 4, "Setup"), prompts of roughly 10 to 1e4 tokens and
+FCFS waiting queue (Sec. 4 setup), prompts of roughly 10 to 1e4 tokens and
 responses of roughly 1e2 to 1e3 tokens (App. B.3), per-token prices
 (App. B.1/B.4) and TTFT targets drawn with the recipe of App. B.2.  The paper's
 datasets (Alpaca, HotpotQA, GovReport, WritingPrompts) are not available; these
