@@ -533,7 +533,11 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
         //    i-th waiting request), then possibly one partial chunk.  An admitted
         //    request's chunk is applied at once; one that prefills whole decodes from
         //    the next batch.
-        while (budget > 0 && wc > 0 && nr < S) {
+        // FCFS: a head whose first chunk's blocks are not free admits nobody (the
+        // usual case while a queue waits on a full cache)
+        bool adm = budget > 0 && wc > 0 && nr < S;
+        if (adm) adm = kv_blocks32(min(wq[wh].x, budget), bs) <= freeb;
+        while (adm && budget > 0 && wc > 0 && nr < S) {
             if (ne + 32 > C) compact();
             const bool in = lane < wc && lane < S - nr;
             int slot = wh + lane;
