@@ -72,3 +72,34 @@ def test_workload_generator_is_deterministic():
     assert np.array_equal(a.prompt_len, b.prompt_len[:50])
     assert np.all(a.n_run <= a.max_seqs)
     assert a.run_ctx.shape == (64, a.cap_running)
+
+
+def _prototypes():
+    protos = {}
+    for h in HEADERS:
+        text = open(h).read()
+        for m in re.finditer(r"^LR_API\s+[\w\s\*]+?\b(lr_\w+)\s*\((.*?)\);", text, flags=re.M | re.S):
+            args = m.group(2).strip()
+            protos[m.group(1)] = [" ".join(a.split()) for a in args.split(",")] if args not in ("", "void") else []
+    return protos
+
+
+def test_binding_argtypes_match_the_header(lib):
+    # every parameter of every prototype against the binding's ctypes declaration:
+    # a pointer for a pointer, the same width and kind for a scalar
+    from paper_2607_18253_gb300 import router
+    bound = router.load_library()
+    scalar = {"int32_t": ctypes.c_int32, "int64_t": ctypes.c_int64, "float": ctypes.c_float,
+              "double": ctypes.c_double, "int": ctypes.c_int}
+    protos = _prototypes()
+    assert set(protos) == set(_declared())
+    for name, params in protos.items():
+        at = getattr(bound, name).argtypes
+        assert at is not None and len(at) == len(params), (name, params, at)
+        for p, t in zip(params, at):
+            if "*" in p:
+                assert t in (ctypes.c_void_p, ctypes.c_char_p) or issubclass(t, ctypes._Pointer), (name, p, t)
+            else:
+                ctype = p.replace("const ", "").split()[0]
+                assert ctypes.sizeof(t) == ctypes.sizeof(scalar[ctype]), (name, p, t)
+                assert (t in (ctypes.c_float, ctypes.c_double)) == (ctype in ("float", "double")), (name, p, t)
