@@ -52,12 +52,13 @@ def test_hand_trace_with_a_preemption_of_the_query():
     assert la == g["admit_batch"] and lt == g["first_token_batch"] and used == g["most_blocks_in_use"]
 
 
-def test_hand_trace_with_residents_preempting_each_other():
+@pytest.mark.parametrize("fixture", ["kv_hand_trace_residents.json", "kv_hand_trace_residents_mode1.json"])
+def test_hand_trace_with_residents_preempting_each_other(fixture):
     # a resident preempting itself and readmitted in the same batch, one preempted
     # by an older one, a partial chunk, and the query admitted once the instance
-    # drains (tests/golden/kv_hand_trace_residents.json); the residents' own
-    # batches are also those of the residents alone
-    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "kv_hand_trace_residents.json")))
+    # drains (tests/golden/kv_hand_trace_residents*.json, both first-token modes);
+    # the residents' own batches are also those of the residents alone
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", fixture)))
     args = (g["running"], g["waiting"], g["B"], g["S"])
     kw = dict(block_size=g["block_size"], num_blocks=g["num_blocks"], max_ctx=g["max_ctx"], mode=g["mode"])
     F, la, lt, res, used = oracle.simulate_kv(*args, *g["query"], **kw)
