@@ -23,6 +23,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 import numpy as np
@@ -76,7 +77,8 @@ class Clocks:
     def __init__(self, index: int):
         self.index = index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+        # the raw samples (one CSV per rank) go to LR_CLOCK_DIR, else the system temp dir
+        self.path = os.path.join(os.environ.get("LR_CLOCK_DIR", tempfile.gettempdir()), f"lr_clocks_rank{index}.csv")
 
     def __enter__(self):
         try:
@@ -358,7 +360,7 @@ def run_gpu(args):
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
             "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "f32+i64", "data": "synthetic (seeded lognormal/uniform stand-ins, see DESIGN.md)",
+            "dtype": "f32+i64", "data": "synthetic (seeded lognormal/uniform stand-ins for the paper's workloads)",
             "config": _config_desc(wl),
             "p50_step_ms": srt[len(srt) // 2], "p99_step_ms": srt[min(len(srt) - 1, int(0.99 * len(srt)))],
             "kernels": kernels, "roofline": roof, "cpu_baseline": cpu,
