@@ -197,3 +197,25 @@ def test_route_skips_candidates_without_an_estimate():
     ok = ~np.isnan(t).all(axis=1)
     np.testing.assert_array_equal(a[0, ok], ai[0, ok])
     assert (a[0, ~ok] == -1).all() and not (a[0] == 0).any()
+
+
+@pytest.mark.parametrize("name", ["tiny", "pool64", "pool256"])
+def test_generated_limits_are_valid_inputs(name):
+    # the seeded limits keep every snapshot valid under the KV rule: the running
+    # requests' blocks fit, every request's whole context (capped) fits, no context
+    # reaches the limit, and the longest prompt's first token fits
+    from paper_2607_18253_gb300 import workloads as W
+    wl = W.make_workload(name)
+    bs, nb, mc = W.kv_limits(wl, 11, block_sizes=(16,))
+    ceil = lambda c, b: -(-c // b)  # noqa: E731
+    for j in range(wl.num_instances):
+        n, w = int(wl.n_run[j]), int(wl.n_wait[j])
+        ctx, pre, dec = (a[j, :n].astype(np.int64) for a in (wl.run_ctx, wl.run_pre, wl.run_dec))
+        wp, wd = (a[j, :w].astype(np.int64) for a in (wl.wait_pre, wl.wait_dec))
+        b = int(bs[j])
+        assert ceil(ctx, b).sum() <= nb[j]
+        assert ((ctx + pre) < mc[j]).all() and (wp < mc[j]).all() and wl.max_prompt_len < mc[j]
+        assert (ceil(np.minimum(ctx + pre + dec, mc[j]), b) <= nb[j]).all()
+        assert (ceil(np.minimum(wp + wd, mc[j]), b) <= nb[j]).all()
+        assert ceil(wl.max_prompt_len + 1, b) <= nb[j]
+    assert (mc < (1 << 40)).any() and (mc == (1 << 40)).any()  # both kinds of instance
