@@ -56,6 +56,22 @@ def _dist():
     return rank, world, local
 
 
+def _max_over_ranks(x: float, world: int) -> float:
+    """The largest of the ranks' values (the slowest rank's time); x itself on one rank."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _job_rate(units_per_rank: float, world: int, ms: float) -> float:
+    """Whole-job throughput: the units every rank processed over the slowest rank's time."""
+    return units_per_rank * world / (ms * 1e-3)
+
+
 def _config_desc(wl, extra=None):
     d = {"workload": f"{WORKLOAD}: {wl.num_instances} instances ({wl.num_models} models x "
                      f"{wl.num_instances // wl.num_models} replicas) x {wl.num_queries} queries, "
@@ -216,11 +232,7 @@ def run_gpu(args):
         dist.barrier()
     assert rt.status() == R.LR_OK
     step_ms = [e0.elapsed_time(e1) for e0, e1 in evp]
-    total_ms = sum(step_ms)
-    if world > 1:
-        tt = torch.tensor([total_ms], dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = _max_over_ranks(sum(step_ms), world)
     ms_per_step = total_ms / K
 
     # The same steps with K1 and K2 in sequence: each kernel's own duration (roofline,
@@ -239,7 +251,7 @@ def run_gpu(args):
     route_ms = [ev[k][1].elapsed_time(ev[k][2]) for k in range(K)]
     seq_ms = sum(a + b for a, b in zip(load_ms, route_ms)) / K
     cands = Q * I
-    value = cands * world / (ms_per_step * 1e-3)
+    value = _job_rate(cands, world, ms_per_step)
 
     # End to end, as a serving loop runs it: every step copies its snapshot and queries
     # from pinned host memory, ingests and routes them (K1 || K2 as above) and copies
@@ -308,11 +320,7 @@ def run_gpu(args):
     run_e2e(max(3, args.warmup), False)
     KE = max(3, min(K, 200))
     e2e_ms = run_e2e(KE, True)
-    e2e_mean = sum(e2e_ms) / KE
-    if world > 1:
-        tt = torch.tensor([e2e_mean], dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_mean = float(tt.item())
+    e2e_mean = _max_over_ranks(sum(e2e_ms) / KE, world)
     host_out = host_outs[(KE - 1) & 1]
     out = outs[(KE - 1) & 1]
     assert rt.status() == R.LR_OK
@@ -364,13 +372,13 @@ def run_gpu(args):
             "config": _config_desc(wl),
             "p50_step_ms": srt[len(srt) // 2], "p99_step_ms": srt[min(len(srt) - 1, int(0.99 * len(srt)))],
             "kernels": kernels, "roofline": roof, "cpu_baseline": cpu,
-            "e2e": {"value": cands * world / (e2e_mean * 1e-3), "unit": UNIT, "ms_per_step": e2e_mean,
+            "e2e": {"value": _job_rate(cands, world, e2e_mean), "unit": UNIT, "ms_per_step": e2e_mean,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "note": "per step: pinned-host snapshot + queries -> device (copy stream, overlapping the "
                             "previous step), K1 || K2, result -> pinned host read by the host one step later; "
                             "L2 flushed before each step's compute"},
             "gpu_launches": 2 * K, "clocks": clk.summary(), "wall_s_timed_region": t_wall,
-            "sequential": {"ms_per_step": seq_ms, "value": cands * world / (seq_ms * 1e-3), "unit": UNIT,
+            "sequential": {"ms_per_step": seq_ms, "value": _job_rate(cands, world, seq_ms), "unit": UNIT,
                            "note": "K1 then K2 on one stream, same steps (kernel shares are of this time)"},
             "estimate": estimate,
             "kv": kv,
