@@ -10,6 +10,11 @@
  * time model of Eq. 9.  It then scores each candidate with the accuracy-cost
  * utility of Eq. 2 and picks one instance per query by the Lagrangian
  * objective of Eq. 5 or the latency-constrained objective of Eq. 3.
+ * Also: the online stream (lr_advance), the average-case TTFT sources of Sec. 4 /
+ * App. E (lr_set_queue_params, lr_set_ttft_source), KV-cache block and context
+ * limits with preemption (lr_set_kv_limits), least-squares calibration of the
+ * batch-time coefficients (lr_calibrate), and the baseline routers with
+ * OnTimeUtility (lr_route_baseline, lr_on_time_utility).
  *
  * Conventions for every call:
  *  - All integers are int32 unless stated; all arrays are dense, row-major.
