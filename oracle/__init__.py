@@ -27,6 +27,33 @@ FIRST_TOKEN_WITH_LAST_CHUNK = 1
 DEFAULT_MAX_BATCHES = 1 << 40
 
 
+def host_threads() -> int:
+    """Host threads the candidate loops use by default: every core this process may run on."""
+    try:
+        return max(1, len(os.sched_getaffinity(0)))
+    except (AttributeError, OSError):
+        return max(1, os.cpu_count() or 1)
+
+
+def _in_slices(C: int, threads: Optional[int], call) -> None:
+    """Run call(lo, hi) over [0, C) split into contiguous slices, one per thread.
+
+    Every candidate is independent (its own copy of its instance's state), and the
+    C loop holds no shared state, so slices may run concurrently; ctypes releases
+    the interpreter lock for the duration of each foreign call.  The result does
+    not depend on the thread count."""
+    n = host_threads() if threads is None else max(1, int(threads))
+    n = min(n, max(1, C // 64))
+    if n <= 1:
+        call(0, C)
+        return
+    from concurrent.futures import ThreadPoolExecutor
+    bounds = [C * k // n for k in range(n + 1)]
+    with ThreadPoolExecutor(max_workers=n) as ex:
+        for f in [ex.submit(call, bounds[k], bounds[k + 1]) for k in range(n)]:
+            f.result()
+
+
 def build(force: bool = False) -> str:
     """Compile the oracle with gcc (no fp contraction, no fast-math)."""
     os.makedirs(_LIBDIR, exist_ok=True)
@@ -145,8 +172,11 @@ def utility(acc, lam, p, dec_hat, price_in, price_out) -> np.float32:
                                           float(np.float32(price_in)), float(np.float32(price_out))))
 
 
-def estimate_candidates(wl, cand_q, cand_j, max_batches: int = DEFAULT_MAX_BATCHES):
-    """F[C,5], first-token batch [C], canonical fp32 TTFT [C], fp64 TTFT [C]."""
+def estimate_candidates(wl, cand_q, cand_j, max_batches: int = DEFAULT_MAX_BATCHES,
+                        threads: Optional[int] = None):
+    """F[C,5], first-token batch [C], canonical fp32 TTFT [C], fp64 TTFT [C].
+
+    The candidates are split over `threads` host threads (default: every core)."""
     cq = _c(cand_q, np.int32)
     cj = _c(cand_j, np.int32)
     C = cq.shape[0]
@@ -159,20 +189,29 @@ def estimate_candidates(wl, cand_q, cand_j, max_batches: int = DEFAULT_MAX_BATCH
                                       wl.wait_dec, wl.prompt_len, wl.dec_hat)]
     coef = _c(wl.coef, np.float32)
     moi, B, S, n_run, run_ctx, run_pre, run_dec, n_wait, wait_pre, wait_dec, p, dh = arrs
-    rc = _load().orc_estimate_candidates(
-        wl.num_instances, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running, wl.cap_waiting, _p(n_run),
-        _p(run_ctx), _p(run_pre), _p(run_dec), _p(n_wait), _p(wait_pre), _p(wait_dec), wl.num_models, _p(p),
-        _p(dh), wl.first_token_mode, max_batches, C, _p(cq), _p(cj), _p(F), _p(lt), _p(t32), _p(t64))
+    lib = _load()
+    codes = []
+
+    def run(lo, hi):
+        rc = lib.orc_estimate_candidates(
+            wl.num_instances, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running, wl.cap_waiting, _p(n_run),
+            _p(run_ctx), _p(run_pre), _p(run_dec), _p(n_wait), _p(wait_pre), _p(wait_dec), wl.num_models, _p(p),
+            _p(dh), wl.first_token_mode, max_batches, hi - lo, _p(cq[lo:]), _p(cj[lo:]), _p(F[lo:]), _p(lt[lo:]),
+            _p(t32[lo:]), _p(t64[lo:]))
+        codes.append(rc)
+
+    _in_slices(C, threads, run)
+    rc = next((r for r in codes if r != 0), 0)
     if rc != 0:
         raise RuntimeError(f"oracle estimate failed with code {rc}")
     return F, lt, t32, t64
 
 
-def estimate_matrix(wl, max_batches: int = DEFAULT_MAX_BATCHES):
+def estimate_matrix(wl, max_batches: int = DEFAULT_MAX_BATCHES, threads: Optional[int] = None):
     """Every candidate: F[Q,I,5], first-token batch [Q,I], fp32 [Q,I], fp64 [Q,I]."""
     Q, I = wl.num_queries, wl.num_instances
     qq, jj = np.meshgrid(np.arange(Q), np.arange(I), indexing="ij")
-    F, lt, t32, t64 = estimate_candidates(wl, qq.ravel(), jj.ravel(), max_batches)
+    F, lt, t32, t64 = estimate_candidates(wl, qq.ravel(), jj.ravel(), max_batches, threads)
     return F.reshape(Q, I, 5), lt.reshape(Q, I), t32.reshape(Q, I), t64.reshape(Q, I)
 
 
@@ -231,6 +270,43 @@ def advance(wl, clock, assign, prompt_len, dec, t_now: float, max_batches: int =
     if rc != 0:
         raise RuntimeError(f"oracle advance failed with code {rc}")
     return dataclasses.replace(wl, **st), clk
+
+
+def pool_capacity(wl, horizon: float = 300.0, warm: float = 30.0, dt: float = 2.0, depth: int = 256) -> np.ndarray:
+    """Completions/s of every instance fed a saturating FCFS stream of the workload's queries.
+
+    The reading of pool capacity for the online stream (App. E defines an
+    instance's capacity from its peak throughput): each instance starts empty;
+    before every advance of dt seconds (the oracle's stream step) its waiting
+    queue is topped up to `depth` with the workload's next queries, each with the
+    predicted output length of the instance's model, so the scheduler never runs
+    dry; completions are counted from t = warm to t = horizon."""
+    import dataclasses
+    I = wl.num_instances
+    z = np.zeros(I, np.int32)
+    st = dataclasses.replace(wl, n_run=z, n_wait=z.copy(), cap_waiting=depth,
+                             run_ctx=np.zeros((I, wl.cap_running), np.int32),
+                             run_pre=np.zeros((I, wl.cap_running), np.int32),
+                             run_dec=np.zeros((I, wl.cap_running), np.int32),
+                             wait_pre=np.zeros((I, depth), np.int32), wait_dec=np.zeros((I, depth), np.int32))
+    clk = np.zeros(I)
+    appended = np.zeros(I, np.int64)
+    nxt, t, c_warm = 0, 0.0, None
+    while True:
+        completed = appended - st.n_run - st.n_wait
+        if c_warm is None and t >= warm:
+            c_warm = completed.copy()
+        if t >= horizon:
+            break
+        need = depth - st.n_wait
+        a = np.repeat(np.arange(I, dtype=np.int32), need)
+        idx = (nxt + np.arange(a.shape[0])) % wl.num_queries
+        nxt += a.shape[0]
+        appended += need
+        t += dt
+        dec = np.ascontiguousarray(wl.dec_hat[idx, wl.model_of_instance[a]])
+        st, clk = advance(st, clk, a, wl.prompt_len[idx], dec, t)
+    return (completed - c_warm) / (horizon - warm)
 
 
 # ---------------------------------------------------------------------------
@@ -421,7 +497,7 @@ def kv_residents(running, waiting, B: int, S: int, L: int, block_size: int, num_
 
 
 def estimate_matrix_kv(wl, block_size, num_blocks, max_ctx, max_batches: int = DEFAULT_MAX_BATCHES,
-                       cand_q=None, cand_j=None):
+                       cand_q=None, cand_j=None, threads: Optional[int] = None):
     """Every candidate (or the listed ones) under per-instance KV limits, the query taken
     up to its first token.  Returns status, F[...,5], first-token batch, fp32, fp64
     ([Q,I] shapes for the full matrix, [C] for a list); failed candidates carry F = -1,
@@ -446,10 +522,18 @@ def estimate_matrix_kv(wl, block_size, num_blocks, max_ctx, max_batches: int = D
     nb = _c(np.broadcast_to(np.asarray(num_blocks, np.int64), (I,)), np.int64)
     mc = _c(np.broadcast_to(np.asarray(max_ctx, np.int64), (I,)), np.int64)
     coef = _c(wl.coef, np.float32)
-    rc = _load().orc_estimate_candidates_kv(
-        I, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running, wl.cap_waiting, _p(n_run), _p(run_ctx), _p(run_pre),
-        _p(run_dec), _p(n_wait), _p(wait_pre), _p(wait_dec), _p(p), _p(bs), _p(nb), _p(mc), wl.first_token_mode,
-        max_batches, C, _p(cq), _p(cj), _p(st), _p(F), _p(lt), _p(t32), _p(t64))
+    lib = _load()
+    codes = []
+
+    def run(lo, hi):
+        codes.append(lib.orc_estimate_candidates_kv(
+            I, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running, wl.cap_waiting, _p(n_run), _p(run_ctx),
+            _p(run_pre), _p(run_dec), _p(n_wait), _p(wait_pre), _p(wait_dec), _p(p), _p(bs), _p(nb), _p(mc),
+            wl.first_token_mode, max_batches, hi - lo, _p(cq[lo:]), _p(cj[lo:]), _p(st[lo:]), _p(F[lo:]),
+            _p(lt[lo:]), _p(t32[lo:]), _p(t64[lo:])))
+
+    _in_slices(C, threads, run)
+    rc = next((r for r in codes if r != 0), 0)
     if rc != 0:
         raise RuntimeError(f"oracle KV estimate failed with code {rc}")
     if full:

@@ -257,3 +257,49 @@ def test_ttft_target_generator_mean():
         expect = min(1120.0, max(150.0, 158.0 + 3.5e-3 * p))
         assert abs(t.mean() - expect) < 0.01 * expect
         assert t.min() >= 150.0 - 1e-3 and t.max() <= 1120.0 + 1e-3
+
+
+def test_coefficient_row_follows_the_instance_model():
+    # Each instance's estimate uses its own model's Eq. 9 coefficients.  Two idle
+    # instances, instance 0 serving
+    # model 1 and instance 1 serving model 0; power-of-two coefficients make every
+    # product and partial sum exact in fp32, so the expected times are exact rationals.
+    import dataclasses
+    from fractions import Fraction as Fr
+    base = W.small_workload(0, num_instances=2, num_models=2, num_queries=3)
+    z = np.zeros(2, np.int32)
+    coef = np.array([[2.0 ** -8, 2.0 ** -12, 2.0 ** -10, 2.0 ** -16, 2.0 ** -20],
+                     [2.0 ** -6, 2.0 ** -11, 2.0 ** -9, 2.0 ** -15, 2.0 ** -19]], np.float32)
+    wl = dataclasses.replace(base, model_of_instance=np.array([1, 0], np.int32), coef=coef,
+                             max_batched_tokens=np.array([2048, 2048], np.int32), max_seqs=np.array([8, 8], np.int32),
+                             n_run=z, n_wait=z.copy(), prompt_len=np.array([100, 3000, 1], np.int32),
+                             dec_hat=np.array([[5, 7], [1, 2], [3, 4]], np.int32), first_token_mode=0)
+    F, lt, t32, t64 = oracle.estimate_matrix(wl)
+    for i, p in enumerate((100, 3000, 1)):
+        # idle instance, paper mode: ceil(p/B) prefill batches then one decode batch at context p
+        Fx = [-(-p // 2048) + 1, p, 1, p, p * (p + 1) // 2]
+        for j in range(2):
+            assert F[i, j].tolist() == Fx
+            m = 1 - j
+            exact = sum(Fr(float(coef[m, k])) * Fx[k] for k in range(5))
+            assert Fr(float(t32[i, j])) == exact, (i, j)
+            assert Fr(t64[i, j]) == exact, (i, j)
+    # the two instances differ (a shared or swapped row would make them equal or exchange them)
+    assert t32[0, 0] == np.float32(2.0 ** -6 * 2 + 100 * 2.0 ** -11 + 2.0 ** -9 + 100 * 2.0 ** -15 + 5050 * 2.0 ** -19)
+    assert t32[0, 1] == np.float32(2.0 ** -8 * 2 + 100 * 2.0 ** -12 + 2.0 ** -10 + 100 * 2.0 ** -16 + 5050 * 2.0 ** -20)
+
+
+def test_candidate_slices_on_several_threads_change_nothing():
+    # the candidate loop split over host threads gives the single-thread result bit for bit
+    wl = W.make_workload("pool64", num_queries=70)
+    Q, I = wl.num_queries, wl.num_instances
+    qq, jj = np.meshgrid(np.arange(Q), np.arange(I), indexing="ij")
+    one = oracle.estimate_candidates(wl, qq.ravel(), jj.ravel(), threads=1)
+    many = oracle.estimate_candidates(wl, qq.ravel(), jj.ravel(), threads=5)
+    for a, b in zip(one, many):
+        np.testing.assert_array_equal(a.view(np.uint8), b.view(np.uint8))
+    lim = W.kv_limits(wl, 3)
+    one = oracle.estimate_matrix_kv(wl, *lim, threads=1)
+    many = oracle.estimate_matrix_kv(wl, *lim, threads=3)
+    for a, b in zip(one, many):
+        np.testing.assert_array_equal(np.ascontiguousarray(a).view(np.uint8), np.ascontiguousarray(b).view(np.uint8))
