@@ -185,8 +185,9 @@ LR_API int lr_route(lr_ctx *ctx, int32_t Q, const int32_t *prompt_len, const int
  * of memory taken from the context.  Arguments and outputs are those of lr_route with
  * ttft_chosen_out and ttft_matrix_out absent; frontier_out is required.
  *  - Requires P * Q <= LR_STATIC_ROUTE_CAP, else LR_ECAPACITY before any launch.
- *  - Set-up: the first call on each device (which must be current, and the context's
- *    device) looks the array up once; make that first call before any stream capture.
+ *  - Set-up: lr_create (the context's device current) looks up the array's device
+ *    address once and keeps it in the context; this call itself makes no runtime
+ *    query of it, so a capture may begin at any point after lr_create.
  *  - Nothing in the array needs to start at zero: every entry the frontier reads is
  *    written earlier in the same call, in stream order.
  *  - The array is shared by every context on a device: two of these calls in flight at

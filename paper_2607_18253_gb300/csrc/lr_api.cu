@@ -4,7 +4,6 @@
 #include <cstdint>
 #include <cstdio>
 #include <cstring>
-#include <mutex>
 #include <new>
 #include <string>
 #include <vector>
@@ -12,9 +11,17 @@
 #include "latency_router.h"
 #include "lr_internal.cuh"
 
+// Chosen-TTFT intermediate of lr_route_frontier_static: [P][Q] fp32 in static
+// device memory, so that the call itself allocates nothing.  In host code this
+// name is a host-side stand-in, not a device address: lr_create looks the
+// device address up (cudaGetSymbolAddress, the context's device current) and
+// keeps it in the context.
+static __device__ __align__(256) float g_static_route_tch[LR_STATIC_ROUTE_CAP];
+
 struct lr_ctx {
     int device = 0;
     int sms = 0;
+    float *static_tch = nullptr;  // device address of g_static_route_tch on this context's device
     lr::DevConfig cfg{};
     lr::StateBuf buf[2]{};
     lr::StateBuf scratch{};  // advanced snapshot before it is summarized
@@ -238,6 +245,14 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     cudaError_t e = cudaGetDevice(&c->device);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, c->device);
     if (e != cudaSuccess) return bail(LR_ECUDA, std::string("cuda device: ") + cudaGetErrorString(e));
+    {
+        // the static array of lr_route_frontier_static on this device (the device is
+        // current here, and lr_create runs before any capture of the context's calls)
+        void *sp = nullptr;
+        e = cudaGetSymbolAddress(&sp, g_static_route_tch);
+        if (e != cudaSuccess) return bail(LR_ECUDA, std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e));
+        c->static_tch = static_cast<float *>(sp);
+    }
 
     lr::DevConfig &d = c->cfg;
     d.I = I;
@@ -572,36 +587,6 @@ int lr_on_time_utility(lr_ctx *c, int32_t Q, const float *util, const float *ttf
     return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "on-time utility launch");
 }
 
-// Chosen-TTFT intermediate of lr_route_frontier_static: [P][Q] fp32 in static
-// device memory, so that the call itself allocates nothing.
-static __device__ __align__(256) float g_static_route_tch[LR_STATIC_ROUTE_CAP];
-
-namespace {
-
-constexpr int kMaxDevices = 64;
-std::mutex g_static_mu;
-float *g_static_tch[kMaxDevices] = {};
-
-// Address of the static array on the current device, looked up once per device.
-int static_route_tch(lr_ctx *c, float **out) {
-    int dev = -1;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return cuda_fail(c, e, "cudaGetDevice");
-    if (dev != c->device) return fail(c, LR_EINVAL, "the context's device must be current");
-    if (dev < 0 || dev >= kMaxDevices) return fail(c, LR_ECAPACITY, "device index beyond the static table");
-    std::lock_guard<std::mutex> lock(g_static_mu);
-    if (!g_static_tch[dev]) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_static_route_tch);
-        if (e != cudaSuccess) return cuda_fail(c, e, "cudaGetSymbolAddress");
-        g_static_tch[dev] = static_cast<float *>(p);
-    }
-    *out = g_static_tch[dev];
-    return LR_OK;
-}
-
-}  // namespace
-
 int lr_route_frontier_static(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec_hat,
                              const float *acc, const float *tau, int32_t P, const float *lambda, const float *mu,
                              int32_t *assign_out, float *util_out, double *frontier_out, void *stream) {
@@ -610,9 +595,8 @@ int lr_route_frontier_static(lr_ctx *c, int32_t Q, const int32_t *prompt_len, co
     if (!frontier_out) return fail(c, LR_EINVAL, "null frontier_out");
     if (Q > 0 && P > 0 && (int64_t)P * Q > LR_STATIC_ROUTE_CAP)
         return fail(c, LR_ECAPACITY, "P * Q exceeds LR_STATIC_ROUTE_CAP (the static chosen-TTFT array)");
-    float *tch = nullptr;
-    const int rc = static_route_tch(c, &tch);
-    if (rc != LR_OK) return rc;
+    float *tch = c->static_tch;
+    if (!tch) return fail(c, LR_ECUDA, "no device address of the static chosen-TTFT array");
     // the same kernels as lr_route with a frontier and no chosen-TTFT output; only
     // the intermediate's storage differs
     return lr_route(c, Q, prompt_len, dec_hat, acc, tau, P, lambda, mu, assign_out, util_out, tch, frontier_out,

@@ -4,7 +4,8 @@ lr_route_frontier_static runs the same kernels as lr_route with a frontier,
 keeping the chosen-TTFT intermediate in the library's static device memory;
 its outputs must equal lr_route's (assignments and utilities bit for bit, the
 fp64 frontier within 1e-12 relative) on every call, including back-to-back
-calls that reuse the static array.
+calls that reuse the static array, with and without KV-cache limits; and the
+device's free memory must not change across the calls (nothing is allocated).
 """
 import numpy as np
 import pytest
@@ -58,11 +59,14 @@ def test_static_route_matches_lr_route(mode):
     out = {"assign": torch.empty((P, Q), dtype=torch.int32, device="cuda"),
            "util": torch.empty((P, Q), dtype=torch.float32, device="cuda"),
            "frontier": torch.empty((P, 3), dtype=torch.float64, device="cuda")}
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
     for _ in range(2):  # two calls in a row reuse the static array
         o = rt.route_frontier_static(p, dh, acc, lam, mu, out=out)
         torch.cuda.synchronize()
         assert rt.status() == R().LR_OK
         check_same(o, ref)
+    assert torch.cuda.mem_get_info()[0] == free0
     # constrained objective (Eq. 3, one lambda) with the per-query targets
     refc = rt.route(p, dh, acc, lam[:1], None, tau=tau, ttft_chosen=False, frontier=True)
     for _ in range(2):
@@ -89,3 +93,29 @@ def test_static_route_capacity_is_checked_before_launch():
     torch.cuda.synchronize()
     assert rt.status() == R().LR_OK
     check_same(o, ref)
+
+
+def test_static_route_under_kv_limits():
+    # with KV-cache limits the route scores the KV-limited estimate matrix, which the
+    # library keeps in memory taken by lr_set_kv_limits: still nothing allocated per call
+    wl = W.make_workload("tiny")
+    rt = make_router(wl, max_pairs=32)
+    rt.set_kv_limits(*W.kv_limits(wl, 1, block_sizes=(16,)), horizon=1024)
+    rt.load_state(*R().state_tensors(wl))
+    p, dh, acc, _ = R().query_tensors(wl)
+    lam, mu = W.sweep_pairs()
+    ref = rt.route(p, dh, acc, lam, mu, ttft_chosen=False, frontier=True)
+    P, Q = len(lam), wl.num_queries
+    out = {"assign": torch.empty((P, Q), dtype=torch.int32, device="cuda"),
+           "util": torch.empty((P, Q), dtype=torch.float32, device="cuda"),
+           "frontier": torch.empty((P, 3), dtype=torch.float64, device="cuda")}
+    torch.cuda.synchronize()
+    assert rt.status() == R().LR_OK
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(2):
+        o = rt.route_frontier_static(p, dh, acc, lam, mu, out=out)
+        torch.cuda.synchronize()
+        assert rt.status() == R().LR_OK
+        check_same(o, ref)
+    assert torch.cuda.mem_get_info()[0] == free0
+    rt.close()
