@@ -13,8 +13,12 @@ value      = candidates (query x instance) per second, device time, inputs resid
 e2e        = same metric through the public API from pinned host buffers, with the
              host->device copy of the snapshot and queries and the device->host copy
              of the routing result inside each timed step
-roofline   = the dominant kernel against measured HBM bandwidth
-cpu_baseline / --impl reference = the CPU oracle (literal per-candidate simulation)
+roofline   = the SFS estimate call (lr_estimate_ttft, the full Q x I matrix) on the same
+             workload against measured HBM bandwidth; per-kernel figures of the step
+             (route, K1) under "kernels"
+configs    = the other single-GPU configurations (tiny, pool64, the 32-pair sweep)
+cpu_baseline / --impl reference = the CPU oracle (literal per-candidate simulation) on
+             every host core (and one core), with the host's core count and CPU model
 """
 import argparse
 import json
@@ -220,6 +224,20 @@ def run_gpu(args):
         dist.barrier()
     torch.cuda.synchronize()
     with Clocks(local) as clk:
+        # the same step replayed back to back for args.sustain_seconds first, so that the
+        # clock sampler (one sample per 100 ms) sees the GPU under this load; then the K
+        # timed steps
+        t_s0 = time.perf_counter()
+        ev_s = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+        ev_s[0].record(stream)
+        sustained = 0
+        while time.perf_counter() - t_s0 < args.sustain_seconds:
+            for _ in range(256):
+                flush.fill_(1.0)
+                g_pipe.replay()
+            sustained += 256
+            torch.cuda.synchronize()
+        ev_s[1].record(stream)
         t_wall0 = time.perf_counter()
         for k in range(K):
             flush.fill_(float(k))
@@ -228,6 +246,7 @@ def run_gpu(args):
             evp[k][1].record(stream)
         torch.cuda.synchronize()
         t_wall = time.perf_counter() - t_wall0
+    sustained_ms = ev_s[0].elapsed_time(ev_s[1])
     if world > 1:
         dist.barrier()
     assert rt.status() == R.LR_OK
@@ -296,31 +315,34 @@ def run_gpu(args):
         g_up.append(gu)
         g_step.append(gs)
 
-    def run_e2e(steps, timed):
-        ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    def run_e2e(steps):
+        # `steps` pipelined steps with no L2 flush inside the loop (each step's inputs
+        # arrive by their own host->device copy).  Returns the span from the first
+        # upload's issue to the last result's arrival, and each step's latency from
+        # its upload's issue to its result's arrival.
+        ev_up0 = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
         ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
         up = [torch.cuda.Event() for _ in range(steps)]
         for k in range(steps):
             b = k & 1
             if k >= 2:
                 copy_stream.wait_event(ev1[k - 2])  # buffer set b is free again
+            ev_up0[k].record(copy_stream)
             with torch.cuda.stream(copy_stream):
                 g_up[b].replay()
             up[k].record(copy_stream)
-            flush.fill_(float(k))
-            ev0[k].record(stream)
             stream.wait_event(up[k])
             g_step[b].replay()
             ev1[k].record(stream)
             if k >= 1:
                 ev1[k - 1].synchronize()  # the host has the previous step's result
         torch.cuda.synchronize()
-        return [ev0[k].elapsed_time(ev1[k]) for k in range(steps)] if timed else None
+        return ev_up0[0].elapsed_time(ev1[-1]), [ev_up0[k].elapsed_time(ev1[k]) for k in range(steps)]
 
-    run_e2e(max(3, args.warmup), False)
-    KE = max(3, min(K, 200))
-    e2e_ms = run_e2e(KE, True)
-    e2e_mean = _max_over_ranks(sum(e2e_ms) / KE, world)
+    run_e2e(max(3, args.warmup))
+    KE = max(3, min(K, 2000))
+    e2e_span, e2e_lat = run_e2e(KE)
+    e2e_mean = _max_over_ranks(e2e_span / KE, world)
     host_out = host_outs[(KE - 1) & 1]
     out = outs[(KE - 1) & 1]
     assert rt.status() == R.LR_OK
@@ -343,19 +365,14 @@ def run_gpu(args):
             "hbm_frac": load_bytes / (load_avg * 1e-3) / 1e9 / hbm, "dram_bytes_ncu": NCU_TRAFFIC["k_trajectory"],
             "bound": "dependency-latency chain of the slowest instance"},
     }
-    if route_avg >= load_avg:
-        ach = route_bytes / (route_avg * 1e-3) / 1e9
-        roof = {"kernel": "k_route", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
-                "frac": ach / hbm, "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs, copy)",
-                "traffic": args.traffic if args.traffic is not None else NCU_TRAFFIC["k_route"]}
-    else:
-        ach = load_bytes / (load_avg * 1e-3) / 1e9
-        roof = {"kernel": "k_trajectory", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
-                "frac": ach / hbm, "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs, copy)",
-                "traffic": args.traffic if args.traffic is not None else NCU_TRAFFIC["k_trajectory"],
-                "note": "latency-bound event loop; bytes fraction shown for reference"}
-
+    # the line's roofline: the SFS estimate call (lr_estimate_ttft) on this workload,
+    # HBM-bound (the full Q x I fp32 matrix written, the prompts and the summary read)
     estimate = run_estimate(args, dev, wl, flush)
+    roof = dict(estimate["roofline"])
+    roof["call"] = estimate["call"]
+    roof["target"] = "frac >= 0.5 (the 256-instance x 65,536-query configuration)"
+    roof["target_met"] = bool(roof["frac"] >= 0.5)
+    configs = run_configs(args, dev, flush)
     kv = run_kv(args, dev, wl, flush)
     avgcase = run_avgcase(args, dev, wl, flush)
     calibration = run_calibration(args, dev, flush)
@@ -365,22 +382,35 @@ def run_gpu(args):
     if rank == 0:
         cpu = cpu_baseline(wl, args.cpu_seconds) if (world == 1 and not args.no_cpu) else None
         srt = sorted(step_ms)
+        elat = sorted(e2e_lat)
+        clocks = clk.summary()
+        if clocks.get("sm_mhz"):
+            clocks["ms_x_mhz_per_step"] = ms_per_step * clocks["sm_mhz"]
+        clocks["sampled_region"] = (f"{sustained} back-to-back steps ({sustained_ms / 1e3:.2f} s) then the "
+                                    f"{K} timed steps")
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
             "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f32+i64", "data": "synthetic (seeded lognormal/uniform stand-ins for the paper's workloads)",
             "config": _config_desc(wl),
             "p50_step_ms": srt[len(srt) // 2], "p99_step_ms": srt[min(len(srt) - 1, int(0.99 * len(srt)))],
-            "kernels": kernels, "roofline": roof, "cpu_baseline": cpu,
+            "roofline": roof, "kernels": kernels, "cpu_baseline": cpu,
             "e2e": {"value": _job_rate(cands, world, e2e_mean), "unit": UNIT, "ms_per_step": e2e_mean,
-                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "note": "per step: pinned-host snapshot + queries -> device (copy stream, overlapping the "
-                            "previous step), K1 || K2, result -> pinned host read by the host one step later; "
-                            "L2 flushed before each step's compute"},
-            "gpu_launches": 2 * K, "clocks": clk.summary(), "wall_s_timed_region": t_wall,
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": KE,
+                    "p50_latency_ms": elat[len(elat) // 2],
+                    "p99_latency_ms": elat[min(len(elat) - 1, int(0.99 * len(elat)))],
+                    "note": "through the public API (lr_load_state + lr_route): per step the snapshot and "
+                            "queries are copied from pinned host memory on a copy stream, ingested and routed "
+                            "(K1 || K2), and the result copied back to pinned host memory, which the host "
+                            "reads one step later; two device buffer sets alternate, so a step's upload "
+                            "overlaps the previous step's compute.  ms_per_step = span from the first upload's "
+                            "issue to the last result's arrival / steps (no L2 flush inside the loop: every "
+                            "step's inputs arrive by copy); latency = a step's upload issue to its result"},
+            "gpu_launches": 2 * K, "clocks": clocks, "wall_s_timed_region": t_wall,
             "sequential": {"ms_per_step": seq_ms, "value": _job_rate(cands, world, seq_ms), "unit": UNIT,
                            "note": "K1 then K2 on one stream, same steps (kernel shares are of this time)"},
             "estimate": estimate,
+            "configs": configs,
             "kv": kv,
             "avgcase": avgcase,
             "calibration": calibration,
@@ -486,6 +516,86 @@ def run_estimate(args, dev, wl, flush):
             "roofline": {"kernel": "k_cand<0, 1>", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                          "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
                          "algorithmic_bytes": nbytes, "traffic": NCU_TRAFFIC["k_estimate"]}}
+
+
+def run_configs(args, dev, flush):
+    """The other single-GPU configurations, one router each, every call captured in a
+    CUDA graph and timed with CUDA events after an L2 flush:
+      tiny   -- 8 instances (2 models x 4 replicas) x 16 queries, B = 2048, S = 64;
+      pool64 -- 64 instances (4 models x 16) x 4,096 queries, B = 4096, S = 64;
+      sweep  -- the pool64 state and queries routed for 32 (lambda, mu) pairs (4 x 8 on a log
+                grid) with the per-pair frontier.
+    For each: the route call alone (lr_route: the full TTFT matrix, utility, argmax) and the
+    step (lr_load_state + lr_route on one stream); estimates/s counts query x instance TTFT
+    estimates (the sweep's 32 pairs reuse one matrix; pair evaluations are given beside)."""
+    import torch
+    from paper_2607_18253_gb300 import router as R
+    from paper_2607_18253_gb300 import workloads as W
+
+    lam5, mu5 = W.sweep_pairs()
+    cases = (("tiny", W.make_workload("tiny"), False),
+             ("pool64", W.make_workload("pool64"), False),
+             ("sweep_pool64_32pairs", W.make_workload("pool64", lam=lam5, mu=mu5), True))
+    K = max(3, min(args.steps, 200))
+    out = {}
+    for label, wl, frontier in cases:
+        Q, I, P = wl.num_queries, wl.num_instances, wl.num_pairs
+        rt = R.LatencyRouter.from_workload(wl)
+        state = R.state_tensors(wl, dev)
+        p, dh, acc, _ = R.query_tensors(wl, dev)
+        mat = torch.empty((Q, I), dtype=torch.float32, device=dev)
+        res = {"assign": torch.empty((P, Q), dtype=torch.int32, device=dev),
+               "util": torch.empty((P, Q), dtype=torch.float32, device=dev),
+               "ttft_chosen": torch.empty((P, Q), dtype=torch.float32, device=dev)}
+        if frontier:
+            res["frontier"] = torch.empty((P, 3), dtype=torch.float64, device=dev)
+        cap = torch.cuda.Stream(device=dev)
+        cap.wait_stream(torch.cuda.current_stream())
+
+        def route():
+            rt.route(p, dh, acc, wl.lam, wl.mu, ttft_matrix=mat, frontier=frontier, out=res)
+
+        with torch.cuda.stream(cap):
+            for _ in range(3):
+                rt.load_state(*state)
+                route()
+        cap.synchronize()
+        graphs = {}
+        for name in ("route", "step"):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=cap):
+                if name == "step":
+                    rt.load_state(*state)
+                route()
+            graphs[name] = g
+        ms = {}
+        for name, g in graphs.items():
+            for _ in range(args.warmup):
+                flush.fill_(1.0)
+                g.replay()
+            torch.cuda.synchronize()
+            t = []
+            for k in range(K):
+                flush.fill_(float(k))
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                g.replay()
+                e1.record()
+                e1.synchronize()
+                t.append(e0.elapsed_time(e1))
+            ms[name] = sorted(t)
+        if rt.status() != R.LR_OK:
+            raise RuntimeError(f"{label}: device status after the timed calls")
+        rt.close()
+        mean = {k: sum(v) / len(v) for k, v in ms.items()}
+        out[label] = {"queries": Q, "instances": I, "pairs": P, "steps": K,
+                      "route_us": mean["route"] * 1e3, "route_p50_us": ms["route"][K // 2] * 1e3,
+                      "step_us": mean["step"] * 1e3, "step_p50_us": ms["step"][K // 2] * 1e3,
+                      "value": Q * I / (mean["route"] * 1e-3), "step_value": Q * I / (mean["step"] * 1e-3),
+                      "unit": UNIT, "pair_evaluations_per_s": Q * I * P / (mean["route"] * 1e-3),
+                      # route: the candidate kernel (+ the frontier kernel); step: K1 and the route
+                      "gpu_launches": K * (2 * (1 + int(frontier)) + 1)}
+    return out
 
 
 KV_SEED = 11
@@ -721,7 +831,7 @@ def run_stream(args, dev):
     launches = 0
     for label, arr, sizes in traces:
         for m in sizes:
-            nq = STREAM_QUERIES if (m > 1 or args.stream_full) else min(STREAM_QUERIES, args.stream_queries_b1)
+            nq = STREAM_QUERIES if m > 1 else min(STREAM_QUERIES, args.stream_queries_b1)
             nb = nq // m
             rt.load_state(*state)
             chunk = 4096
@@ -885,27 +995,133 @@ def _policy_eval(rt, wl, arr, dev, p, dh, acc):
             "policies": res, "gpu_launches": len(POLICIES) * (3 * nb + 3)}
 
 
-def _oracle_rows(wl, nq, seed):
+def _host_cpu():
+    """Core count and CPU model of this host (lscpu, else /proc/cpuinfo)."""
+    import platform
+    model = None
+    try:
+        txt = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        names = [ln.split(":", 1)[1].strip() for ln in txt.splitlines() if ln.startswith("Model name:")]
+        model = " / ".join(dict.fromkeys(names)) or None
+    except Exception:
+        pass
+    if not model:
+        try:
+            for ln in open("/proc/cpuinfo"):
+                if ln.lower().startswith("model name"):
+                    model = ln.split(":", 1)[1].strip()
+                    break
+        except OSError:
+            pass
+    try:
+        usable = len(os.sched_getaffinity(0))
+    except (AttributeError, OSError):
+        usable = os.cpu_count()
+    return {"nproc": os.cpu_count(), "usable_cores": usable, "cpu_model": model or platform.machine(),
+            "arch": platform.machine()}
+
+
+def _oracle_rows(wl, nq, seed, threads):
     """Full TTFT rows for nq sampled queries, then the oracle's argmax over them."""
     import oracle
     rng = np.random.default_rng(seed)
     qs = np.sort(rng.choice(wl.num_queries, nq, replace=False))
     sub = wl.with_queries(qs)
     t0 = time.perf_counter()
-    _, _, t32, _ = oracle.estimate_matrix(sub)
+    _, _, t32, _ = oracle.estimate_matrix(sub, threads=threads)
     oracle.route(sub, t32)
     return nq * wl.num_instances, time.perf_counter() - t0
 
 
+def _sized_rows(wl, seconds, seed, threads):
+    """About `seconds` of oracle work on whole rows: (candidates, seconds, queries)."""
+    probe = 8 if threads == 1 else 64
+    cands, dt = _oracle_rows(wl, probe, seed, threads)
+    per_row = dt / probe
+    nq = max(probe, min(wl.num_queries, int(seconds / per_row)))
+    cands, dt = _oracle_rows(wl, nq, seed + 1, threads)
+    return cands, dt, nq
+
+
+def _repeat_for(fn, seconds):
+    """Run fn() (which returns units of work) until `seconds` have passed: (units, seconds)."""
+    units, t0 = 0, time.perf_counter()
+    while True:
+        units += fn()
+        dt = time.perf_counter() - t0
+        if dt >= seconds:
+            return units, dt
+
+
+def _oracle_configs(threads, seconds):
+    """The oracle on the other configurations, on `threads` host threads."""
+    import dataclasses
+
+    import oracle
+    from paper_2607_18253_gb300 import workloads as W
+    out = {}
+    lam5, mu5 = W.sweep_pairs()
+    for label, wl in (("tiny", W.make_workload("tiny")), ("pool64", W.make_workload("pool64")),
+                      ("sweep_pool64_32pairs", W.make_workload("pool64", lam=lam5, mu=mu5))):
+        def one(wl=wl, label=label):
+            _, _, t32, _ = oracle.estimate_matrix(wl, threads=threads)
+            a, _, tc = oracle.route(wl, t32)
+            if label.startswith("sweep"):
+                oracle.frontier(wl, a, tc)
+            return wl.num_queries * wl.num_instances
+        units, dt = _repeat_for(one, min(seconds, 2.0))
+        out[label] = {"value": units / dt, "unit": UNIT, "seconds": dt,
+                      "sample": f"the whole configuration ({wl.num_queries} x {wl.num_instances}"
+                                f"{', 32 pairs + frontier' if label.startswith('sweep') else ''}), repeated"}
+    # the online stream: decisions of the Poisson trace at micro-batch 256, each the
+    # oracle's advance to the decision time, then the batch's rows and argmax
+    wl = W.make_workload(STREAM_WORKLOAD, num_queries=STREAM_QUERIES, seed=STREAM_SEED, cap_waiting=512)
+    rate = 0.8 * float(oracle.pool_capacity(wl).sum())
+    arr = W.poisson_arrivals(STREAM_QUERIES, rate, STREAM_SEED)
+    m, st, clk, prev = 256, wl, np.zeros(wl.num_instances), None
+    none = np.zeros(0, np.int32)
+    t0, b = time.perf_counter(), 0
+    while time.perf_counter() - t0 < seconds and (b + 1) * m <= STREAM_QUERIES:
+        lo = b * m
+        t_now = float(arr[lo + m - 1])
+        if prev is None:
+            st, clk = oracle.advance(st, clk, none, none, none, t_now)
+        else:
+            pa, pq = prev
+            d = np.ascontiguousarray(pq.dec_hat[np.arange(m), wl.model_of_instance[pa]])
+            st, clk = oracle.advance(st, clk, pa, pq.prompt_len, d, t_now)
+        q = dataclasses.replace(st, prompt_len=wl.prompt_len[lo:lo + m], dec_hat=wl.dec_hat[lo:lo + m],
+                                acc=wl.acc[lo:lo + m], tau=wl.tau[lo:lo + m])
+        _, _, t32, _ = oracle.estimate_matrix(q, threads=threads)
+        a, _, _ = oracle.route(q, t32, lam=wl.lam[:1], mu=wl.mu[:1])
+        prev = (a[0], q)
+        b += 1
+    dt = time.perf_counter() - t0
+    out["stream_pool64_b256"] = {"value": b * m * wl.num_instances / dt, "unit": UNIT, "seconds": dt,
+                                 "decisions_per_s": b / dt,
+                                 "sample": f"the first {b} decisions of the Poisson trace at micro-batch {m} "
+                                           f"(advance + rows + argmax)"}
+    return out
+
+
 def cpu_baseline(wl, seconds: float):
-    """The oracle as it stands, one host core, on a bounded sample of the workload."""
-    cands, dt = _oracle_rows(wl, 8, 1)
-    per = dt / cands
-    nq = max(8, min(wl.num_queries, int(seconds / (per * wl.num_instances))))
-    cands, dt = _oracle_rows(wl, nq, 2)
-    return {"value": cands / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{nq} random queries of {WORKLOAD} x all {wl.num_instances} instances "
-                      f"({cands} candidates, {dt:.1f} s): literal per-candidate simulation + brute-force argmax"}
+    """The oracle as it stands on this host's cores, on bounded samples of each workload.
+
+    value: the headline workload on every core (one thread per core, candidates split
+    into contiguous slices); one_core: the same on one thread; configs: the other
+    configurations on every core."""
+    import oracle
+    n = oracle.host_threads()
+    c1, d1, q1 = _sized_rows(wl, seconds, 2, 1)
+    cn, dn, qn = _sized_rows(wl, seconds, 4, n)
+    sample = (f"{qn} random queries of {WORKLOAD} x all {wl.num_instances} instances ({cn} candidates, "
+              f"{dn:.1f} s): literal per-candidate simulation + brute-force argmax, {n} threads; estimates/s "
+              f"extrapolate to the whole {wl.num_queries}-query batch")
+    return {"value": cn / dn, "unit": UNIT, "cores": n, "kind": "oracle", "sample": sample,
+            "host": _host_cpu(),
+            "one_core": {"value": c1 / d1, "unit": UNIT, "cores": 1,
+                         "sample": f"{q1} random queries x all instances ({c1} candidates, {d1:.1f} s)"},
+            "configs": _oracle_configs(n, min(seconds, 5.0))}
 
 
 def run_reference(args):
@@ -915,26 +1131,29 @@ def run_reference(args):
     import oracle
     from paper_2607_18253_gb300 import workloads as W
     oracle.build()
+    n = oracle.host_threads()
     wl = W.make_workload(WORKLOAD)
-    cands, dt = _oracle_rows(wl, 4, 0)
-    per_row = dt / 4
+    probe = 64
+    _, dt = _oracle_rows(wl, probe, 0, n)
+    per_row = dt / probe
     # about two minutes in total, whatever K and W are
     step_s = min(args.ref_step_seconds, 120.0 / max(1, args.steps + args.warmup))
     nq = max(2, min(wl.num_queries, int(step_s / per_row)))
     for w in range(args.warmup):
-        _oracle_rows(wl, nq, 100 + w)
+        _oracle_rows(wl, nq, 100 + w, n)
     times = []
     for k in range(args.steps):
-        c, t = _oracle_rows(wl, nq, 1000 + k)
+        c, t = _oracle_rows(wl, nq, 1000 + k, n)
         times.append(t)
     ms = 1e3 * sum(times) / len(times)
     v = nq * wl.num_instances / (ms * 1e-3)
     sample = (f"each step: {nq} random queries of {WORKLOAD} x all {wl.num_instances} instances, literal "
-              f"per-candidate simulation + brute-force argmax, 1 host core")
+              f"per-candidate simulation + brute-force argmax, {n} host threads (one per core)")
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32+i64", "data": "synthetic", "config": _config_desc(wl),
-            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": n, "kind": "oracle", "sample": sample,
+                             "host": _host_cpu()},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -947,12 +1166,12 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--ref-step-seconds", type=float, default=2.0)
+    ap.add_argument("--sustain-seconds", type=float, default=1.5,
+                    help="back-to-back steps before the timed ones, while the clocks are sampled")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-stream", action="store_true", help="skip the online-stream latency run")
-    ap.add_argument("--stream-full", action="store_true",
-                    help="route the whole 10^6-query trace at micro-batch 1 too (about a minute)")
-    ap.add_argument("--stream-queries-b1", type=int, default=50_000,
-                    help="queries of the trace routed one at a time (default: the first 50,000)")
+    ap.add_argument("--stream-queries-b1", type=int, default=STREAM_QUERIES,
+                    help="queries of the trace routed one at a time (default: the whole trace)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="dram bytes per launch of the dominant kernel from an ncu capture of this build")
     args = ap.parse_args()
