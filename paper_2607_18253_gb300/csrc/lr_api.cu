@@ -60,7 +60,7 @@ struct lr_ctx {
     // candidate kernel shapes: estimate (instances may span several tiles) and
     // route (all instances of a row in one CTA)
     struct Shape {
-        int Gp = 0, QS = 0, QT = 0, tiles = 1, occ = 1;
+        int Gp = 0, QS = 0, QT = 0, tiles = 1, occ = 1, block = 0;
         size_t smem = 0;
         bool ok = false;
     } est, rt;
@@ -131,9 +131,12 @@ int pow2_ceil(int x) {
 // Launch shape of the candidate kernel: threads own four consecutive instances;
 // Gp groups per row (power of two up to 32, else a multiple of 32); the
 // summary tables of the tile and QT staged query rows fit the shared-memory
-// target so that four CTAs share an SM.
+// target.  Routing runs three 256-thread CTAs per SM (one of them fits beside a
+// snapshot load's CTA); the estimate alone runs one 768-thread CTA per SM, so
+// that each SM copies its tile block once.
 lr_ctx::Shape make_shape(const lr::DevConfig &d, bool route, int max_pairs) {
     lr_ctx::Shape s;
+    s.block = route ? lr::kK2Block : lr::kK2EstBlock;
     const int G = (d.I + 3) / 4;
     s.Gp = G <= 32 ? pow2_ceil(G) : round_up(G, 32);
     if (s.Gp > lr::kK2Block) {
@@ -141,16 +144,19 @@ lr_ctx::Shape make_shape(const lr::DevConfig &d, bool route, int max_pairs) {
         s.Gp = lr::kK2Block;
     }
     s.tiles = (d.I + 4 * s.Gp - 1) / (4 * s.Gp);
-    s.QS = lr::kK2Block / s.Gp;
+    s.QS = s.block / s.Gp;
     const int wpr = s.Gp > 32 ? s.Gp / 32 : 1;
     // the tile block (tables and per-instance scalars), brought in by one bulk copy
-    const size_t tables = (size_t)d.kph * 4 * s.Gp * 16 + (size_t)d.nbh * 4 * s.Gp * 8 + (size_t)lr::kScal * 4 * s.Gp * 4;
+    lr::DevConfig dt = d;
+    dt.tgp = s.Gp;
+    const size_t tables = lr::tile_bytes(dt);
     const size_t part = s.Gp > 32 ? 2 * (size_t)wpr * 16 * max_pairs : 0;  // wide-row partials per pair
     // staged row (16 B) and two raw copies of its prompt; routing adds the wide-row
     // partials, (cost, acc) per model, tau, and two raw copies of tau, dec_hat and acc
     const size_t per_row = 16 + 8 + (route ? part + (size_t)d.M * 8 + 4 + 8 + (size_t)d.M * 16 : 0);
-    const size_t room = lr::kK2SmemTarget > tables ? lr::kK2SmemTarget - tables : 0;
-    int qt = (int)std::min<size_t>(256, room / per_row);
+    const size_t target = route ? lr::kK2SmemTarget : lr::kK2EstSmemTarget;
+    const size_t room = target > tables ? target - tables : 0;
+    int qt = (int)std::min<size_t>(route ? 256 : 1024, room / per_row);
     if (route && (size_t)qt * per_row + tables > 200 * 1024) qt = 0;
     qt = std::max(s.QS, (qt / s.QS) * s.QS);
     s.QT = qt;
@@ -364,8 +370,8 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     if (e == cudaSuccess) e = lr::set_k2_smem(std::max(c->est.smem, c->rt.ok ? c->rt.smem : 0));
     c->bl_ok = lr::baseline_smem(d) <= 200 * 1024;
     if (e == cudaSuccess && c->bl_ok) e = lr::set_baseline_smem(lr::baseline_smem(d));
-    if (e == cudaSuccess) e = lr::cand_occupancy(d.mode, false, lr::kK2Block, c->est.smem, &c->est.occ);
-    if (e == cudaSuccess && c->rt.ok) e = lr::cand_occupancy(d.mode, true, lr::kK2Block, c->rt.smem, &c->rt.occ);
+    if (e == cudaSuccess) e = lr::cand_occupancy(d.mode, false, c->est.block, c->est.smem, &c->est.occ);
+    if (e == cudaSuccess && c->rt.ok) e = lr::cand_occupancy(d.mode, true, c->rt.block, c->rt.smem, &c->rt.occ);
     if (e != cudaSuccess) return bail(LR_ECUDA, cudaGetErrorString(e));
     c->est.occ = std::max(1, c->est.occ);
     c->rt.occ = std::max(1, c->rt.occ);
@@ -468,7 +474,7 @@ static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, 
     a.vec_ok = (c->cfg.I % 4 == 0) && ((uintptr_t)ttft % 16 == 0);
     dim3 grid(std::min(c->sms * c->est.occ, (Q + a.QS - 1) / a.QS), c->est.tiles);
     set_row_split(a, c, (int)grid.x, (int)grid.y, c->est.occ, stream);
-    e = lr::launch_cand(a, lr::cand_out_flags(true, iters != nullptr, false, false, 1), grid, lr::kK2Block,
+    e = lr::launch_cand(a, lr::cand_out_flags(true, iters != nullptr, false, false, 1), grid, c->est.block,
                         c->est.smem, (cudaStream_t)stream);
     return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "estimate launch");
 }
@@ -536,7 +542,7 @@ int lr_route(lr_ctx *c, int32_t Q, const int32_t *prompt_len, const int32_t *dec
     dim3 grid(std::min(c->sms * c->rt.occ, (Q + a.QS - 1) / a.QS), 1);
     set_row_split(a, c, (int)grid.x, 1, c->rt.occ, stream);
     cudaError_t e = lr::launch_cand(a, lr::cand_out_flags(a.ttft != nullptr, false, true, tau != nullptr, P), grid,
-                                    lr::kK2Block, c->rt.smem, (cudaStream_t)stream);
+                                    c->rt.block, c->rt.smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(c, e, "route launch");
     if (frontier_out) {
         e = lr::launch_frontier(a, frontier_out, (cudaStream_t)stream);

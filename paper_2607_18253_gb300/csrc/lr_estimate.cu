@@ -109,12 +109,11 @@ struct Inst4 {
     float h1[4], l1[4], h4[4], l4[4], b1p[4], b2[4], b3[4];
 };
 
-template <int MODE>
-__device__ __forceinline__ float ttft_fast(const QRec &q, const Inst4 &r, int u, const float4 e) {
+// T = T_k (the first two terms, which depend on k* only), f3 = fp32(F3 of the candidate).
+__device__ __forceinline__ float ttft_fast(const QRec &q, const Inst4 &r, int u, float T, float f3) {
     const float f1 = __fadd_rn(r.h1[u], __fadd_rn(r.l1[u], q.fp));
-    const float f3 = (MODE == 0) ? __fadd_rn(e.y, __fadd_rn(e.z, q.fp)) : e.w;
     const float f4 = __fadd_rn(__fadd_rn(r.h4[u], q.ph), __fadd_rn(r.l4[u], q.pl));
-    float t = __fmaf_rn(r.b1p[u], f1, e.x);
+    float t = __fmaf_rn(r.b1p[u], f1, T);
     t = __fmaf_rn(r.b2[u], f3, t);
     t = __fmaf_rn(r.b3[u], f4, t);
     return t;
@@ -122,7 +121,7 @@ __device__ __forceinline__ float ttft_fast(const QRec &q, const Inst4 &r, int u,
 
 // Exact int64 path for instances whose totals do not split into fp32.
 template <int MODE>
-__device__ float ttft_exact64(const DevConfig &c, const StateBuf &sb, const QRec &q, int j, int k, const float4 e) {
+__device__ float ttft_exact64(const DevConfig &c, const StateBuf &sb, const QRec &q, int j, int k, const float T) {
     if (q.fp != q.fp) return q.fp;
     const InstParams ip = sb.inst[j];
     const int m = c.moi[j];
@@ -130,7 +129,7 @@ __device__ float ttft_exact64(const DevConfig &c, const StateBuf &sb, const QRec
     const float f1 = __ll2float_rn(ip.f1tot + p);
     const float f3 = __ll2float_rn(sb.f3[(size_t)k * c.I + j] + (MODE == 0 ? p : 0));
     const float f4 = __ll2float_rn(ip.f4tot + (p * (p + 1)) / 2);
-    float t = __fmaf_rn(c.coef[m * 5 + 1], f1, e.x);
+    float t = __fmaf_rn(c.coef[m * 5 + 1], f1, T);
     t = __fmaf_rn(c.coef[m * 5 + 3], f3, t);
     t = __fmaf_rn(c.coef[m * 5 + 4], f4, t);
     return t;
@@ -174,15 +173,21 @@ __device__ __forceinline__ void write_pick(const K2Launch &a, size_t o, const Ca
 
 // Table loads by 32-bit shared-memory address.  The tables are written once
 // before the first barrier and only read afterwards.
-__device__ __forceinline__ int2 lds_int2(uint32_t addr) {
-    int2 v;
-    asm("ld.shared.v2.s32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+__device__ __forceinline__ float2 lds_float2(uint32_t addr) {
+    float2 v;
+    asm("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr));
     return v;
 }
 
-__device__ __forceinline__ float4 lds_float4(uint32_t addr) {
-    float4 v;
-    asm("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+__device__ __forceinline__ uint32_t lds_u32(uint32_t addr) {
+    uint32_t v;
+    asm("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint4 lds_u32x4(uint32_t addr) {
+    uint4 v;
+    asm("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
     return v;
 }
 
@@ -237,7 +242,11 @@ __device__ __forceinline__ int claim_size(const K2Launch &a, int seen) {
     return min(a.QT, max(4 * a.QS, n - n % a.QS));
 }
 __device__ __forceinline__ int static_rows(const K2Launch &a) { return min(a.Q, a.first_ctas * a.first_rows); }
+// Every row of the launch lies in a static range: no CTA claims, and the counters stay
+// untouched (and zero) -- a call that runs alone takes no atomic round trip at all.
+__device__ __forceinline__ bool all_static(const K2Launch &a) { return (long long)a.first_ctas * a.first_rows >= a.Q; }
 __device__ __forceinline__ int claim_rows(const K2Launch &a, int seen) {
+    if (all_static(a)) return a.Q;
     return static_rows(a) + (int)atomicAdd(a.work + 1 + blockIdx.y, (unsigned)claim_size(a, seen));
 }
 __device__ __forceinline__ int2 first_range(const K2Launch &a) {
@@ -256,7 +265,8 @@ __device__ __forceinline__ int2 range_after(const K2Launch &a, int2 r, int x) {
 
 // End of a candidate-kernel CTA: the last of `ctas` to finish clears the row
 // counters of the `tiles` tiles and the completion count for the next launch.
-__device__ __forceinline__ void k2_finish(uint32_t *work, unsigned ctas, unsigned tiles) {
+__device__ __forceinline__ void k2_finish(const K2Launch &a, uint32_t *work, unsigned ctas, unsigned tiles) {
+    if (all_static(a)) return;  // no counter was touched
     __syncthreads();
     if (threadIdx.x == 0) {
         __threadfence();
@@ -271,8 +281,11 @@ __device__ __forceinline__ void k2_finish(uint32_t *work, unsigned ctas, unsigne
 // MODE 0 / 1: SFS with the first output token in its own batch / with the last
 // prompt chunk.  MODE 2: an average-case source (Sec. 4, App. E), affine in p:
 // t = fma(p, g_j, C_j) with g_j = fp32(1/theta_j) and C_j = fp32(W_j + Tdec_j).
+// Routing launches three 256-thread CTAs per SM, the estimate alone one 768-thread CTA
+// (the same registers per thread either way).
 template <int MODE, int OUT>
-__global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
+__global__ void __launch_bounds__((OUT & (kOutLag | kOutCon | kOutSweep)) ? kK2Block : kK2EstBlock,
+                                  (OUT & (kOutLag | kOutCon | kOutSweep)) ? 3 : 1) k_cand(const K2Launch a) {
     extern __shared__ __align__(16) unsigned char smem[];
     constexpr bool AFF = MODE == 2;
     constexpr bool ROUTE = (OUT & (kOutLag | kOutCon | kOutSweep)) != 0;
@@ -289,21 +302,83 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     const int nv = max(0, min(4, I - jb));             // instances this thread owns
     // Query rows come in ranges (first_range, range_after): a static one, then claims
     // from this tile's counter, in the no-snapshot path as in the main one.
-    // one read of the live-buffer index per CTA (every thread reading the same word
-    // would queue them all on one L2 line)
     __shared__ int s_active;
     __shared__ int2 s_claim[2];
+    __shared__ __align__(8) unsigned long long s_mbar;
+    const uint32_t mbar = (uint32_t)__cvta_generic_to_shared(&s_mbar);
+    const size_t tb = tile_bytes(c);
+    // Shared memory: the tile block (tables and per-instance scalars, exactly as K1
+    // laid it out for this tile), query records, row partials, utility inputs,
+    // targets and the raw query rows (route with one pair stages (U, cost) per row
+    // and model, sweeps (cost, acc)).
+    const int WPR = Gp > 32 ? Gp / 32 : 1;  // warps per row
+    const int NP = SWEEP ? a.P : 1;
+    QRec *s_q = reinterpret_cast<QRec *>(smem + tb);                                   // [QT]
+    int4 *s_part = reinterpret_cast<int4 *>(s_q + QT);                                 // [NP][QT][WPR][2]
+    float2 *s_ca = reinterpret_cast<float2 *>(s_part + (ROUTE && Gp > 32 ? 2 * NP * QT * WPR : 0));  // [QT][M]
+    float *s_tau = reinterpret_cast<float *>(s_ca + (ROUTE ? QT * M : 0));             // [QT]
+    // raw query rows as copied from global memory, two chunks in flight:
+    // prompt [2][QT], and for routing tau [2][QT], dec_hat [2][QT][M], acc [2][QT][M]
+    int32_t *r_p = reinterpret_cast<int32_t *>(s_tau + (ROUTE ? QT : 0));
+    float *r_t = reinterpret_cast<float *>(r_p + 2 * QT);
+    int32_t *r_d = reinterpret_cast<int32_t *>(r_t + (ROUTE ? 2 * QT : 0));
+    float *r_a = reinterpret_cast<float *>(r_d + (ROUTE ? 2 * QT * M : 0));
+    // copies of query rows [q0, q0 + nrows) into raw buffer b
+    auto issue = [&](int q0, int nrows, int b) {
+        for (int t = threadIdx.x; t < nrows; t += blockDim.x) {
+            cp_async4(r_p + b * QT + t, a.prompt + q0 + t);
+            if (CON) cp_async4(r_t + b * QT + t, a.tau + q0 + t);
+        }
+        if (ROUTE) {
+            const size_t g0 = (size_t)q0 * M;
+            for (int idx = threadIdx.x; idx < nrows * M; idx += blockDim.x) {
+                cp_async4(r_d + b * QT * M + idx, a.dec_hat + g0 + idx);
+                cp_async4(r_a + b * QT * M + idx, a.acc + g0 + idx);
+            }
+        }
+        cp_async_commit();
+    };
+    // The tile block arrives with one bulk copy (TMA) completing on an mbarrier:
+    // every CTA reads the same few tens of KB, and one large request per CTA is far
+    // cheaper than thousands of scattered loads of the same lines.
+    auto tile_copy = [&](const unsigned char *src, uint32_t dst_off) {
+        asm volatile(
+            "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                (uint32_t)__cvta_generic_to_shared(smem) + dst_off),
+            "l"(src), "r"((uint32_t)tb), "r"(mbar)
+            : "memory");
+    };
+    // bounded wait for the tile block: a copy that never lands is reported, not waited out
+    auto tile_wait = [&]() -> bool {
+        bool landed = false;
+        for (int it = 0; it < (1 << 22) && !landed; ++it) landed = mbar_test(mbar);
+        return landed;
+    };
+    if (threadIdx.x == 0) {
+        if (!AFF) {
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar) : "memory");
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        }
+        s_claim[0] = first_range(a);
+    }
+    __syncthreads();
+    const int2 first = s_claim[0];
+    // the first chunk of query rows travels while the live index is read and the tile
+    // block lands; one read of the live-buffer index per CTA (every thread reading the
+    // same word would queue them all on one L2 line)
+    if (first.x < a.Q) issue(first.x, min(QT, min(first.y, a.Q) - first.x), 0);
     if (threadIdx.x == 0) s_active = load_acquire(&a.ctl->active);
     __syncthreads();
     const int active = s_active;
     // the LPS source and a given matrix need no live snapshot; every other source does
     if (active < 0 && !(AFF && (a.src == kSrcLps || a.src == kSrcMatrix))) {
         if (threadIdx.x == 0) record_status(a.ctl, kENoState);
+        cp_async_wait<0>();  // nothing may still be landing when the CTA leaves
         for (int k = 0;; ++k) {
             __syncthreads();  // the previous range has been read
-            if (threadIdx.x == 0) {
+            if (threadIdx.x == 0 && k > 0) {
                 const int2 r = s_claim[0];
-                s_claim[0] = k == 0 ? first_range(a) : range_after(a, r, has_rest(a, r) ? 0 : claim_rows(a, r.x));
+                s_claim[0] = range_after(a, r, has_rest(a, r) ? 0 : claim_rows(a, r.x));
             }
             __syncthreads();
             const int rb = s_claim[0].x, re = min(min(a.Q, s_claim[0].y), rb + QT);
@@ -321,81 +396,28 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                     }
             }
         }
-        k2_finish(a.work, gridDim.x * gridDim.y, gridDim.y);
+        k2_finish(a, a.work, gridDim.x * gridDim.y, gridDim.y);
         return;
     }
     {
     const StateBuf sb = active ? a.buf1 : a.buf0;
-    // Shared memory: the tile block (tables and per-instance scalars, exactly as K1
-    // laid it out for this tile), query records, row partials, utility inputs,
-    // targets and the raw query rows (route with one pair stages (U, cost) per row
-    // and model, sweeps (cost, acc)).
-    const int WPR = Gp > 32 ? Gp / 32 : 1;  // warps per row
-    const int NP = SWEEP ? a.P : 1;
-    float4 *s_ent = reinterpret_cast<float4 *>(smem);                                  // [kph][4][Gp]
-    int2 *s_bkt = reinterpret_cast<int2 *>(s_ent + c.kph * 4 * Gp);                    // [nbh][4][Gp]
-    const int32_t *s_scal = reinterpret_cast<const int32_t *>(s_bkt + c.nbh * 4 * Gp);  // [kScal][4][Gp]
-    QRec *s_q = reinterpret_cast<QRec *>(smem + tile_bytes(c));                        // [QT]
-    int4 *s_part = reinterpret_cast<int4 *>(s_q + QT);                                 // [NP][QT][WPR][2]
-    float2 *s_ca = reinterpret_cast<float2 *>(s_part + (ROUTE && Gp > 32 ? 2 * NP * QT * WPR : 0));  // [QT][M]
-    float *s_tau = reinterpret_cast<float *>(s_ca + (ROUTE ? QT * M : 0));             // [QT]
-    // raw query rows as copied from global memory, two chunks in flight:
-    // prompt [2][QT], and for routing tau [2][QT], dec_hat [2][QT][M], acc [2][QT][M]
-    int32_t *r_p = reinterpret_cast<int32_t *>(s_tau + (ROUTE ? QT : 0));
-    float *r_t = reinterpret_cast<float *>(r_p + 2 * QT);
-    int32_t *r_d = reinterpret_cast<int32_t *>(r_t + (ROUTE ? 2 * QT : 0));
-    float *r_a = reinterpret_cast<float *>(r_d + (ROUTE ? 2 * QT * M : 0));
-
-    // The tile block arrives with one bulk copy (TMA) completing on an mbarrier:
-    // every CTA reads the same few tens of KB, and one large request per CTA is far
-    // cheaper than thousands of scattered loads of the same lines.
-    __shared__ __align__(8) unsigned long long s_mbar;
-    const uint32_t mbar = (uint32_t)__cvta_generic_to_shared(&s_mbar);
-    if (threadIdx.x == 0) {
-        if (!AFF) {
-            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar) : "memory");
-            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-            const uint32_t bytes = (uint32_t)tile_bytes(c);
-            const unsigned char *src = sb.tile + (size_t)blockIdx.y * tile_bytes(c);
-            // the block was written by generic stores (possibly of a load on another
-            // stream, acquired above); order them before the bulk copy's reads
-            asm volatile("fence.proxy.async.global;" ::: "memory");
-            asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(mbar), "r"(bytes) : "memory");
-            asm volatile(
-                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                    (uint32_t)__cvta_generic_to_shared(smem)),
-                "l"(src), "r"(bytes), "r"(mbar)
-                : "memory");
-        }
-        s_claim[0] = first_range(a);
+    // (Gp == c.tgp: the tile block's sections at the offsets K1 wrote them)
+    const unsigned char *tile = smem;
+    const unsigned char *s_ent = tile;                                                         // entA, entB
+    const unsigned char *s_bkt = tile + tile_ent_bytes(c);                                     // [nbh][4][Gp]
+    const int32_t *s_scal = reinterpret_cast<const int32_t *>(s_bkt + tile_bkt_bytes(c));    // [kScal][4][Gp]
+    if (threadIdx.x == 0 && !AFF) {
+        // the block was written by generic stores (possibly of a load on another
+        // stream, acquired above); order them before the bulk copy's reads
+        asm volatile("fence.proxy.async.global;" ::: "memory");
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(mbar), "r"((uint32_t)tb) : "memory");
+        tile_copy(sb.tile + (size_t)blockIdx.y * tb, 0u);
     }
-    __syncthreads();
-    const int2 first = s_claim[0];
     // what follows the first chunk: found now, published once the tile block has landed
     int2 second = make_int2(a.Q, a.Q);
     if (threadIdx.x == 0 && first.x < a.Q) second = range_after(a, first, has_rest(a, first) ? 0 : claim_rows(a, first.x));
-    // copies of query rows [q0, q0 + nrows) into raw buffer b
-    auto issue = [&](int q0, int nrows, int b) {
-        for (int t = threadIdx.x; t < nrows; t += blockDim.x) {
-            cp_async4(r_p + b * QT + t, a.prompt + q0 + t);
-            if (CON) cp_async4(r_t + b * QT + t, a.tau + q0 + t);
-        }
-        if (ROUTE) {
-            const size_t g0 = (size_t)q0 * M;
-            for (int idx = threadIdx.x; idx < nrows * M; idx += blockDim.x) {
-                cp_async4(r_d + b * QT * M + idx, a.dec_hat + g0 + idx);
-                cp_async4(r_a + b * QT * M + idx, a.acc + g0 + idx);
-            }
-        }
-        cp_async_commit();
-    };
-    // the first chunk travels while the tile block lands
-    if (first.x < a.Q) issue(first.x, min(QT, min(first.y, a.Q) - first.x), 0);
     if (!AFF) {
-        // bounded wait for the tile block; a copy that never lands is reported, not waited out
-        bool landed = false;
-        for (int it = 0; it < (1 << 22) && !landed; ++it) landed = mbar_test(mbar);
-        if (__syncthreads_or(!landed)) {
+        if (__syncthreads_or(!tile_wait())) {
             if (threadIdx.x == 0) record_status(a.ctl, kECuda);
             for (int it = 0; it < (1 << 22) && !mbar_test(mbar); ++it) {
             }
@@ -406,7 +428,7 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     Inst4 r;
     int model[4], la[4];
     float ag[4], ac[4];  // average-case sources: t = fma(p, ag, ac)
-    bool fast_mine = true;
+    bool fast_mine = true, compact_mine = true;
     const int fs = 4 * Gp;  // scalar field stride
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
@@ -433,28 +455,37 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
         model[u] = s_scal[kScModel * fs + col];
         la[u] = s_scal[kScLa * fs + col];
         if (u < nv) fast_mine = fast_mine && s_scal[kScFast * fs + col] != 0;
+        if (u < nv) compact_mine = compact_mine && s_scal[kScCompact * fs + col] != 0;
     }
+    // the bucket width of the tile's first instance (SPEC needs one width per CTA)
+    const int shift0 = AFF ? 0 : s_scal[kScShift * fs];
     if (threadIdx.x == 0) s_claim[1] = second;
     const bool fast = __syncthreads_and(fast_mine);
     const bool vec = a.vec_ok && nv == 4;
     const unsigned gmask = group_mask(Gp, lane);
     const int grp_lane0 = lane & ~(min(Gp, 32) - 1);  // first lane of this row group in the warp
     const int wrow = g / 32;                          // warp index within a wide row
-    // shared addresses of this thread's table columns: entry (k, u) at
-    // ecol + u * ecst + k * erow, bucket (b, u) at bcol + u * bcst + b * brow (formed
-    // at each use: the kernel is at its register limit)
-    const uint32_t ecol = (uint32_t)__cvta_generic_to_shared(s_ent) + 16u * (uint32_t)g;
-    const uint32_t bcol = (uint32_t)__cvta_generic_to_shared(s_bkt) + 8u * (uint32_t)g;
-    const uint32_t ecst = 16u * (uint32_t)Gp, bcst = 8u * (uint32_t)Gp;
-    const uint32_t erow = 16u * 4u * (uint32_t)Gp, brow = 8u * 4u * (uint32_t)Gp;
+    // shared addresses of this thread's table columns: entA (k, u) at
+    // ecol + u * ecst + k * erow (entB ebofs further), bucket (b, u) at
+    // bcol + 4 u + b * brow (formed at each use: the kernel is at its register limit)
+    const uint32_t ecol = (uint32_t)__cvta_generic_to_shared(s_ent) + 8u * (uint32_t)g;
+    const uint32_t bcol = (uint32_t)__cvta_generic_to_shared(s_bkt) + 16u * (uint32_t)g;
+    const uint32_t ecst = 8u * (uint32_t)Gp;
+    const uint32_t erow = 8u * 4u * (uint32_t)Gp, brow = 4u * 4u * (uint32_t)Gp;
+    const uint32_t ebofs = (uint32_t)tile_enta_bytes(c);
     bool same_model = true;
 #pragma unroll
     for (int u = 1; u < 4; ++u) same_model = same_model && model[u] == model[0];
 
-    // SPEC: every thread of the CTA has four instances of one model, the fp32 split path
-    // and aligned vector stores, so none of the per-thread checks below is needed (an
-    // invalid prompt still gives NaN times, which no comparison selects)
-    const bool spec = __syncthreads_and(fast && nv == 4 && same_model && a.vec_ok);
+    bool same_shift = true;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) same_shift = same_shift && (AFF || r.shift[u] == shift0);
+    // SPEC: every thread of the CTA has four compact instances of one model (the fp32
+    // split path, F3 read from entA alone), every instance of the CTA the same bucket
+    // width (a thread's four buckets are one 16-byte load) and aligned vector stores, so
+    // none of the per-thread checks below is needed (an invalid prompt still gives NaN
+    // times, which no comparison selects)
+    const bool spec = __syncthreads_and(fast && compact_mine && nv == 4 && same_model && same_shift && a.vec_ok);
     auto run = [&](auto fast_tag, auto spec_tag) {
         constexpr bool FAST = decltype(fast_tag)::value;
         constexpr bool SPEC = decltype(spec_tag)::value;
@@ -502,8 +533,11 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
             const size_t ostep = (size_t)QS * I;
             for (int rr = qs; rr < nrows; rr += QS) {
                 const QRec q = s_q[rr];
+                const uint32_t p7 = (uint32_t)q.p << 7;
                 float t[4];
                 int kk[4];
+                uint4 bw4 = make_uint4(0u, 0u, 0u, 0u);
+                if (SPEC && !AFF) bw4 = lds_u32x4(bcol + (uint32_t)(q.p >> shift0) * brow);
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     if (AFF) {
@@ -513,11 +547,26 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
                         kk[u] = 0;
                         continue;
                     }
-                    const int2 bk = lds_int2(bcol + u * bcst + (uint32_t)(q.p >> r.shift[u]) * brow);
-                    kk[u] = bk.y + (q.p > bk.x ? 1 : 0);
-                    const float4 e = lds_float4(ecol + u * ecst + (uint32_t)kk[u] * erow);
-                    if (FAST) t[u] = ttft_fast<MODE>(q, r, u, e);
-                    else t[u] = (SPEC || u < nv) ? ttft_exact64<MODE>(c, sb, q, jb + u, kk[u], e) : 0.f;
+                    // bucket word (boundary << 7) | below: p > boundary iff (p << 7) > word
+                    const uint32_t bw = SPEC ? (u == 0 ? bw4.x : u == 1 ? bw4.y : u == 2 ? bw4.z : bw4.w)
+                                             : lds_u32(bcol + 4u * u + (uint32_t)(q.p >> r.shift[u]) * brow);
+                    kk[u] = (int)(bw & 127u) + (p7 > bw ? 1 : 0);
+                    const uint32_t ea = ecol + u * ecst + (uint32_t)kk[u] * erow;
+                    const float2 e = lds_float2(ea);
+                    if (SPEC) {
+                        // compact: F3 + p below 2^31, one exact int -> fp32 rounding
+                        const float f3 = MODE == 0 ? __int2float_rn(__float_as_int(e.y) + q.p) : e.y;
+                        t[u] = ttft_fast(q, r, u, e.x, f3);
+                    } else if (FAST) {
+                        float f3 = e.y;
+                        if (MODE == 0) {
+                            const float2 hl = lds_float2(ea + ebofs);
+                            f3 = __fadd_rn(hl.x, __fadd_rn(hl.y, q.fp));
+                        }
+                        t[u] = ttft_fast(q, r, u, e.x, f3);
+                    } else {
+                        t[u] = (u < nv) ? ttft_exact64<MODE>(c, sb, q, jb + u, kk[u], e.x) : 0.f;
+                    }
                 }
                 if (OUT & kOutMatrix) {
                     if (SPEC || vec) {
@@ -639,7 +688,7 @@ __global__ void __launch_bounds__(256, 3) k_cand(const K2Launch a) {
     (void)grp_lane0;
     }
 finish:
-    k2_finish(a.work, gridDim.x * gridDim.y, gridDim.y);
+    k2_finish(a, a.work, gridDim.x * gridDim.y, gridDim.y);
 }
 
 // Per-pair means of (accuracy, cost, TTFT) of the chosen instances, fp64, fixed
@@ -890,9 +939,9 @@ __global__ void __launch_bounds__(256) k_baseline(const K2Launch a, int policy, 
             const InstParams ip = sb.inst[j];
             const int2 bk = sb.bkt[(size_t)(q.p >> ip.shift) * I + j];
             const int k = bk.y + (q.p > bk.x ? 1 : 0);
-            const float4 e =
-                reinterpret_cast<const float4 *>(sb.tile + tile_base(c, j))[(size_t)k * 4 * c.tgp + tile_col(c, j)];
-            a.ttft_chosen[i] = ttft_exact64<MODE>(c, sb, q, j, k, e);
+            const float T =
+                reinterpret_cast<const float2 *>(sb.tile + tile_base(c, j))[(size_t)k * 4 * c.tgp + tile_col(c, j)].x;
+            a.ttft_chosen[i] = ttft_exact64<MODE>(c, sb, q, j, k, T);
         }
     }
 }

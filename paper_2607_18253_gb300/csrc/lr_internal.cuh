@@ -131,13 +131,25 @@ __device__ __forceinline__ long long warp_sum64(long long v) {
 // Candidate-kernel tile block: everything one CTA of the candidate kernel needs about
 // its tile of 4 * tgp instances, laid out as that CTA's shared memory so that a single
 // bulk copy brings it in.  Instance j0 + 4g + u of the tile sits in column u * tgp + g:
-//   ent  [kph][4][tgp]    float4 (T_k, H3_k, L3_k, f3_k)
-//   bkt  [nbh][4][tgp]    int2 (in-bucket boundary, boundaries below)
+//   entA [kph][4][tgp]    8 bytes: T_k (fp32) and X_k, which is f3_k (fp32) when the
+//                         first token comes with the last chunk, else F3_k as an int32
+//                         (valid when the instance is compact: F3_k + pmax < 2^31)
+//   entB [kph][4][tgp]    8 bytes: H3_k, L3_k, the exact fp32 split of F3_k
+//   bkt  [nbh][tgp][4]    uint32: (in-bucket boundary << 7) | boundaries below, the
+//                         boundary 2^24 - 1 when the bucket holds none; a thread's four
+//                         instances are adjacent (one 16-byte load when they share the
+//                         bucket width)
 //   scal [kScal][4][tgp]  32-bit scalars, fields kSc*
+// A warp reads a table as one dense 4- or 8-byte word per lane (1 or 2 shared-memory
+// wavefronts); a compact CTA reads only entA.
 constexpr int kScal = 12;
-enum : int { kScShift = 0, kScH1, kScL1, kScH4, kScL4, kScB1p, kScB2, kScB3, kScModel, kScLa, kScFast };
-__host__ __device__ inline size_t tile_ent_bytes(const DevConfig &c) { return (size_t)c.kph * 4 * c.tgp * 16; }
-__host__ __device__ inline size_t tile_bkt_bytes(const DevConfig &c) { return (size_t)c.nbh * 4 * c.tgp * 8; }
+enum : int { kScShift = 0, kScH1, kScL1, kScH4, kScL4, kScB1p, kScB2, kScB3, kScModel, kScLa, kScFast, kScCompact };
+constexpr uint32_t kBktNone = (1u << 24) - 1;  // bucket boundary field of a bucket without one
+__host__ __device__ inline size_t tile_enta_bytes(const DevConfig &c) { return (size_t)c.kph * 4 * c.tgp * 8; }
+__host__ __device__ inline size_t tile_ent_bytes(const DevConfig &c) { return 2 * tile_enta_bytes(c); }
+__host__ __device__ inline size_t tile_bkt_bytes(const DevConfig &c) {
+    return ((size_t)c.nbh * 4 * c.tgp * 4 + 15) & ~(size_t)15;
+}
 __host__ __device__ inline size_t tile_bytes(const DevConfig &c) {
     return tile_ent_bytes(c) + tile_bkt_bytes(c) + (size_t)kScal * 4 * c.tgp * 4;
 }
@@ -299,8 +311,10 @@ cudaError_t launch_on_time(int Q, const float *util, const float *ttft, const fl
                            double *part, int max_parts, double *out, cudaStream_t st);
 cudaError_t cand_occupancy(int mode, bool route, int block, size_t smem, int *blocks_per_sm);
 cudaError_t set_k2_smem(size_t bytes);
-constexpr int kK2Block = 256;
+constexpr int kK2Block = 256;                // route: three CTAs per SM, one fits beside a load's CTA
 constexpr size_t kK2SmemTarget = 72 * 1024;  // three CTAs per SM
+constexpr int kK2EstBlock = 768;             // estimate alone: one CTA per SM, one tile copy per SM
+constexpr size_t kK2EstSmemTarget = 120 * 1024;
 
 // K3: append routed queries and advance every instance to t_now (online stream).
 struct K3Launch {

@@ -589,6 +589,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
     const float b1d = c.coef[m_j * 5 + 2];
     const long long ppmax = ((long long)c.pmax * (c.pmax + 1)) / 2;
     bool fast = (f1 + c.pmax < kFastLimit) && (f4 + ppmax < kFastLimit);
+    bool compact = true;  // every F3_k + pmax below 2^31 (first token in its own batch)
     const long long lowmask = (1LL << kSplitBits) - 1;
     int kp = 0;          // table rows kept
     long long rc = r0;   // cumulative budget R_k
@@ -712,16 +713,19 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             const long long F3 = A3w + q * CBw + Nw * ((long long)q * L0 + (long long)q * (q + 1) / 2) +
                                  red[(2 * kRows + q) * 32];
             fast = fast && (F3 + c.pmax < kFastLimit);
+            compact = compact && (MODE == 1 || F3 + c.pmax < (1LL << 31));
             if (lane == (k & 31)) {
                 const float t = __fmaf_rn(b1d, __ll2float_rn(F2), __fmul_rn(b0, __int2float_rn(L)));
                 const long long lo = F3 & lowmask;
-                float4 e;
-                e.x = t;
-                e.y = __ll2float_rn(F3 - lo);
-                e.z = __ll2float_rn(lo);
-                e.w = __ll2float_rn(F3);
+                // entA: (T_k, X_k); entB: (H3_k, L3_k)
+                const int x = MODE == 1 ? __float_as_int(__ll2float_rn(F3))
+                                        : (F3 + c.pmax < (1LL << 31) ? (int)F3 : 0);
+                const size_t slot = (size_t)k * 4 * c.tgp + tile_col(c, j);
+                unsigned char *tb = out.tile + tile_base(c, j);
+                reinterpret_cast<float2 *>(tb)[slot] = make_float2(t, __int_as_float(x));
+                reinterpret_cast<float2 *>(tb + tile_enta_bytes(c))[slot] =
+                    make_float2(__ll2float_rn(F3 - lo), __ll2float_rn(lo));
                 const size_t o = (size_t)k * c.I + j;
-                reinterpret_cast<float4 *>(out.tile + tile_base(c, j))[(size_t)k * 4 * c.tgp + tile_col(c, j)] = e;
                 out.f2[o] = F2;
                 out.f3[o] = F3;
                 out.rcum[o] = rk;
@@ -748,8 +752,11 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             else if (rk <= hi) bnd = (int)rk;
         }
         out.bkt[(size_t)b * c.I + j] = make_int2(bnd, below);
-        reinterpret_cast<int2 *>(out.tile + tile_base(c, j) + tile_ent_bytes(c))[(size_t)b * 4 * c.tgp + tile_col(c, j)] =
-            make_int2(bnd, below);
+        // packed word: a boundary at or above kBktNone (> every allowed prompt, 2^20) reads
+        // as none; below is at most kKMax < 128
+        reinterpret_cast<uint32_t *>(out.tile + tile_base(c, j) + tile_ent_bytes(c))[(size_t)b * 4 * c.tgp +
+                                                                                   j % (4 * c.tgp)] =
+            (min((uint32_t)bnd, kBktNone) << 7) | (uint32_t)below;
     }
     if (lane == 0) {
         InstParams ip;
@@ -782,6 +789,7 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         sc[kScModel * fs] = m_j;
         sc[kScLa * fs] = la;
         sc[kScFast * fs] = ip.fast;
+        sc[kScCompact * fs] = (fast && compact) ? 1 : 0;
     }
 }
 
@@ -822,7 +830,7 @@ __global__ void __launch_bounds__(kK1Warps * 32) k_trajectory(const K1Launch a) 
 namespace {
 
 // Padding columns of the last tile: no boundary in any bucket, zero tables, an
-// exact ("fast") instance of model 0, and a bucket shift of 30 so that every
+// exact ("fast", compact) instance of model 0, and a bucket shift of 30 so that every
 // allowed prompt (at most 2^20 tokens) looks up bucket 0 and entry 0.
 __global__ void k_tile_pad(const DevConfig c, unsigned char *tile) {
     const int first = c.I;
@@ -830,12 +838,16 @@ __global__ void k_tile_pad(const DevConfig c, unsigned char *tile) {
     for (int j = first + blockIdx.x * blockDim.x + threadIdx.x; j < last; j += gridDim.x * blockDim.x) {
         unsigned char *base = tile + tile_base(c, j);
         const int col = tile_col(c, j);
-        for (int k = 0; k < c.kph; ++k)
-            reinterpret_cast<float4 *>(base)[(size_t)k * 4 * c.tgp + col] = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int k = 0; k < c.kph; ++k) {
+            reinterpret_cast<float2 *>(base)[(size_t)k * 4 * c.tgp + col] = make_float2(0.f, 0.f);
+            reinterpret_cast<float2 *>(base + tile_enta_bytes(c))[(size_t)k * 4 * c.tgp + col] = make_float2(0.f, 0.f);
+        }
         for (int b = 0; b < c.nbh; ++b)
-            reinterpret_cast<int2 *>(base + tile_ent_bytes(c))[(size_t)b * 4 * c.tgp + col] = make_int2(kBig, 0);
+            reinterpret_cast<uint32_t *>(base + tile_ent_bytes(c))[(size_t)b * 4 * c.tgp + j % (4 * c.tgp)] =
+                kBktNone << 7;
         int32_t *sc = reinterpret_cast<int32_t *>(base + tile_ent_bytes(c) + tile_bkt_bytes(c)) + col;
-        for (int f = 0; f < kScal; ++f) sc[(size_t)f * 4 * c.tgp] = (f == kScFast) ? 1 : (f == kScShift) ? 30 : 0;
+        for (int f = 0; f < kScal; ++f)
+            sc[(size_t)f * 4 * c.tgp] = (f == kScFast || f == kScCompact) ? 1 : (f == kScShift) ? 30 : 0;
     }
 }
 
