@@ -100,6 +100,19 @@ int round_up(int x, int m) { return ((x + m - 1) / m) * m; }
 
 bool finite_nonneg(float v) { return std::isfinite(v) && v >= 0.0f; }
 
+// The live-buffer index and its copies, from the host (no kernel of the context may
+// be running); the other control words start at zero.
+cudaError_t set_live_host(lr_ctx *c, int32_t v) {
+    lr::DevCtl h;
+    std::memset(&h, 0, sizeof(h));
+    h.active = v;
+    for (int r = 0; r < lr::kLiveReps; ++r) h.live[r][0] = v;
+    // only the index and its copies change: the status words stay as they are
+    cudaError_t e = cudaMemcpy(&c->ctl->active, &h.active, sizeof(int32_t), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(&c->ctl->live[0][0], &h.live[0][0], sizeof(h.live), cudaMemcpyHostToDevice);
+    return e;
+}
+
 void free_kv(lr_ctx *c) {
     for (void *p : c->kv_allocs) cudaFree(p);
     c->kv_allocs.clear();
@@ -338,8 +351,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     if (e == cudaSuccess) e = cudaMemcpy(coef, cfg->coef, (size_t)M * 20, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(pin, cfg->price_in, M * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(pout, cfg->price_out, M * 4, cudaMemcpyHostToDevice);
-    lr::DevCtl ctl0{-1, 0, 0, 0u};
-    if (e == cudaSuccess) e = cudaMemcpy(c->ctl, &ctl0, sizeof(ctl0), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = set_live_host(c, -1);
     if (e == cudaSuccess) e = cudaMemset(c->k2_work, 0, sizeof(uint32_t) * lr::k2_work_words(I));
     if (e != cudaSuccess) return bail(LR_ECUDA, cudaGetErrorString(e));
     d.moi = moi;
@@ -688,8 +700,7 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
     if (e != cudaSuccess) return cuda_fail(c, e, "synchronize");
     free_kv(c);
     // the live snapshot was summarized for the previous rule
-    const int32_t none = -1;
-    e = cudaMemcpy(&c->ctl->active, &none, sizeof(none), cudaMemcpyHostToDevice);
+    e = set_live_host(c, -1);
     if (e != cudaSuccess) return cuda_fail(c, e, "snapshot reset");
     if (!on) return LR_OK;
     int warps = lr::kKvWarps;

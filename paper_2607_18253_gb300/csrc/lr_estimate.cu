@@ -367,7 +367,7 @@ __global__ void __launch_bounds__((OUT & (kOutLag | kOutCon | kOutSweep)) ? kK2B
     // block lands; one read of the live-buffer index per CTA (every thread reading the
     // same word would queue them all on one L2 line)
     if (first.x < a.Q) issue(first.x, min(QT, min(first.y, a.Q) - first.x), 0);
-    if (threadIdx.x == 0) s_active = load_acquire(&a.ctl->active);
+    if (threadIdx.x == 0) s_active = load_live(a.ctl);
     __syncthreads();
     const int active = s_active;
     // the LPS source and a given matrix need no live snapshot; every other source does
@@ -830,7 +830,7 @@ __global__ void __launch_bounds__(256) k_baseline(const K2Launch a, int policy, 
     const DevConfig &c = a.cfg;
     const int I = c.I, M = c.M;
     __shared__ int s_active;
-    if (threadIdx.x == 0) s_active = load_acquire(&a.ctl->active);
+    if (threadIdx.x == 0) s_active = load_live(a.ctl);
     __syncthreads();
     const int active = s_active;
     const StateBuf sb = active > 0 ? a.buf1 : a.buf0;

@@ -92,11 +92,17 @@ struct StateBuf {
     int32_t *kvp;  // [I][horizon] running maximum of the records' thr (clamped to int32), with KV limits
 };
 
-struct DevCtl {
+// Copies of the live-buffer index, each in its own 128-byte line: the CTAs of a
+// candidate-kernel launch (hundreds, all starting at once) read different copies
+// instead of queueing on one line.
+constexpr int kLiveReps = 64;
+struct __align__(128) DevCtl {
     int32_t active;      // live buffer, -1 before the first successful load
     int32_t status;      // first error since the last lr_status
     int32_t load_err;    // error of the load in progress
     uint32_t done_ctas;  // K1 completion counter
+    int32_t pad[28];
+    int32_t live[kLiveReps][32];  // live[r][0]: copies of active
 };
 
 struct StateIn {
@@ -110,6 +116,19 @@ __device__ __forceinline__ int32_t load_acquire(const int32_t *p) {
     int32_t v;
     asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
+}
+
+// Publish a new live buffer (after a __threadfence of the writes that made it): the
+// index and its copies, which readers take with acquire loads.
+__device__ __forceinline__ void publish_live(DevCtl *ctl, int32_t v) {
+    atomicExch(&ctl->active, v);
+    for (int r = 0; r < kLiveReps; ++r)
+        asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(&ctl->live[r][0]), "r"(v) : "memory");
+}
+
+// The live-buffer index from this CTA's copy, with acquire ordering.
+__device__ __forceinline__ int32_t load_live(const DevCtl *ctl) {
+    return load_acquire(&ctl->live[blockIdx.x % kLiveReps][0]);
 }
 
 __device__ __forceinline__ void record_status(DevCtl *ctl, int code) {

@@ -818,7 +818,7 @@ __global__ void __launch_bounds__(kK1Warps * 32) k_trajectory(const K1Launch a) 
         if (prev == gridDim.x - 1) {
             __threadfence();
             const int err = atomicExch(&a.ctl->load_err, 0);
-            if (err == 0) atomicExch(&a.ctl->active, dst);
+            if (err == 0) publish_live(a.ctl, dst);
             atomicExch(&a.ctl->done_ctas, 0u);
             __threadfence();
         }
