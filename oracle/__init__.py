@@ -92,6 +92,9 @@ def _load():
         lib.orc_advance.argtypes = [i32, P, P, P, P, i32, i32, P, P, P, P, P, P, P, P, i32, P, P, P, i32,
                                     ctypes.c_double, i64]
         lib.orc_advance.restype = ctypes.c_int
+        lib.orc_advance_ids.argtypes = [i32, P, P, P, P, i32, i32, P, P, P, P, P, P, P, P, i32, P, P, P, i32,
+                                        ctypes.c_double, i64, P, P, i64, P]
+        lib.orc_advance_ids.restype = ctypes.c_int
         lib.orc_utility.argtypes = [ctypes.c_float, ctypes.c_float, i32, i32, ctypes.c_float, ctypes.c_float]
         lib.orc_utility.restype = ctypes.c_float
         lib.orc_pow_int.argtypes = [ctypes.c_double, i32]
@@ -250,10 +253,15 @@ def frontier(wl, assign: np.ndarray, ttft_chosen: np.ndarray) -> np.ndarray:
     return out
 
 
-def advance(wl, clock, assign, prompt_len, dec, t_now: float, max_batches: int = 1 << 30):
+def advance(wl, clock, assign, prompt_len, dec, t_now: float, max_batches: int = 1 << 30, track=None,
+            id_base: int = -1):
     """Online stream step on a copy of the workload's state.
 
-    Returns (new workload with the advanced state, new clocks)."""
+    Returns (new workload with the advanced state, new clocks).  With `track` -- a dict of
+    run_id [I, cap_running] int64, wait_id [I, cap_waiting] int64 and first_token_time [N]
+    float64 -- the routed query i joins as id id_base + i (id_base >= 0) and every tracked
+    request that emits its first output token in an executed batch gets that batch's end
+    time; the call then returns (workload, clocks, new track dict)."""
     import dataclasses
     st = {k: np.array(getattr(wl, k), dtype=np.int32, copy=True)
           for k in ("n_run", "run_ctx", "run_pre", "run_dec", "n_wait", "wait_pre", "wait_dec")}
@@ -263,13 +271,29 @@ def advance(wl, clock, assign, prompt_len, dec, t_now: float, max_batches: int =
     d = _c(dec, np.int32)
     moi, B, S = (_c(x, np.int32) for x in (wl.model_of_instance, wl.max_batched_tokens, wl.max_seqs))
     coef = _c(wl.coef, np.float32)
-    rc = _load().orc_advance(wl.num_instances, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running, wl.cap_waiting,
-                             _p(st["n_run"]), _p(st["run_ctx"]), _p(st["run_pre"]), _p(st["run_dec"]),
-                             _p(st["n_wait"]), _p(st["wait_pre"]), _p(st["wait_dec"]), _p(clk), int(a.shape[0]),
-                             _p(a), _p(p), _p(d), wl.first_token_mode, float(t_now), int(max_batches))
+    tr = None
+    if track is not None:
+        tr = {k: np.array(track[k], dtype=(np.float64 if k == "first_token_time" else np.int64), copy=True)
+              for k in ("run_id", "wait_id", "first_token_time")}
+    rc = _load().orc_advance_ids(wl.num_instances, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running,
+                                 wl.cap_waiting, _p(st["n_run"]), _p(st["run_ctx"]), _p(st["run_pre"]),
+                                 _p(st["run_dec"]), _p(st["n_wait"]), _p(st["wait_pre"]), _p(st["wait_dec"]),
+                                 _p(clk), int(a.shape[0]), _p(a), _p(p), _p(d), wl.first_token_mode, float(t_now),
+                                 int(max_batches), _p(None if tr is None else tr["run_id"]),
+                                 _p(None if tr is None else tr["wait_id"]), int(id_base),
+                                 _p(None if tr is None else tr["first_token_time"]))
     if rc != 0:
         raise RuntimeError(f"oracle advance failed with code {rc}")
-    return dataclasses.replace(wl, **st), clk
+    if tr is None:
+        return dataclasses.replace(wl, **st), clk
+    return dataclasses.replace(wl, **st), clk, tr
+
+
+def new_track(wl, num_ids: int):
+    """Empty first-token tracking state for `advance`: every resident untracked, times NaN."""
+    return {"run_id": np.full((wl.num_instances, wl.cap_running), -1, np.int64),
+            "wait_id": np.full((wl.num_instances, wl.cap_waiting), -1, np.int64),
+            "first_token_time": np.full(num_ids, np.nan)}
 
 
 def pool_capacity(wl, horizon: float = 300.0, warm: float = 30.0, dt: float = 2.0, depth: int = 256) -> np.ndarray:

@@ -40,6 +40,7 @@ typedef struct {
     int64_t pre;  /* remaining prefill tokens */
     int64_t dec;  /* remaining decode tokens */
     int is_query; /* the new query q_i */
+    int64_t id;   /* stream step: tracked query id until its first output token, else -1 */
 } orc_req;
 
 enum { SCHED_NONE = 0, SCHED_PREFILL = 1, SCHED_DECODE = 2 };
@@ -347,6 +348,33 @@ int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, 
                 const int32_t *prompt_len, const int32_t *dec, int32_t mode, double t_now,
                 int64_t max_batches)
 {
+    return orc_advance_ids(I, model_of_instance, coef, B, S, cap_running, cap_waiting, n_run, run_ctx, run_pre,
+                           run_dec, n_wait, wait_pre, wait_dec, clock, Q, assign, prompt_len, dec, mode, t_now,
+                           max_batches, NULL, NULL, -1, NULL);
+}
+
+/* The realized first output token (Sec. 4.1: the TTFT ends with the first output
+ * token; Eq. 4 scores each query by its realized TTFT).  A tracked request emits it
+ * in the first executed batch that gives it a decode token, or, when the first token
+ * comes with the last prompt chunk, in the batch that completes its prompt; the time
+ * is that batch's end on the instance's clock. */
+static void first_token(orc_req *q, int emitted, double t_end, double *first_token_time)
+{
+    if (emitted && q->id >= 0) {
+        first_token_time[q->id] = t_end;
+        q->id = -1;
+    }
+}
+
+int orc_advance_ids(int32_t I, const int32_t *model_of_instance, const float *coef, const int32_t *B,
+                    const int32_t *S, int32_t cap_running, int32_t cap_waiting, int32_t *n_run,
+                    int32_t *run_ctx, int32_t *run_pre, int32_t *run_dec, int32_t *n_wait, int32_t *wait_pre,
+                    int32_t *wait_dec, double *clock, int32_t Q, const int32_t *assign,
+                    const int32_t *prompt_len, const int32_t *dec, int32_t mode, double t_now,
+                    int64_t max_batches, int64_t *run_id, int64_t *wait_id, int64_t id_base,
+                    double *first_token_time)
+{
+    const int track = run_id != NULL && wait_id != NULL && first_token_time != NULL;
     int rc_all = ORC_OK;
     for (int32_t j = 0; j < I; ++j) {
         const int64_t total = (int64_t)cap_running + cap_waiting + Q + 1;
@@ -362,17 +390,21 @@ int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, 
         for (int32_t r = 0; r < n_run[j]; ++r) {
             const int64_t o = (int64_t)j * cap_running + r;
             run[nr].ctx = run_ctx[o]; run[nr].pre = run_pre[o]; run[nr].dec = run_dec[o]; run[nr].is_query = 0;
+            run[nr].id = track ? run_id[o] : -1;
             ++nr;
         }
         for (int32_t w = 0; w < n_wait[j]; ++w) {
             const int64_t o = (int64_t)j * cap_waiting + w;
             wait[nw].ctx = 0; wait[nw].pre = wait_pre[o]; wait[nw].dec = wait_dec[o]; wait[nw].is_query = 0;
+            wait[nw].id = track ? wait_id[o] : -1;
             ++nw;
         }
-        /* 1. the routed queries join the waiting tail in query order */
+        /* 1. the routed queries join the waiting tail in query order (query i tracked
+         *    as id_base + i when id_base >= 0) */
         for (int32_t i = 0; i < Q; ++i) {
             if (assign[i] != j) continue;
             wait[nw].ctx = 0; wait[nw].pre = prompt_len[i]; wait[nw].dec = dec[i]; wait[nw].is_query = 0;
+            wait[nw].id = (track && id_base >= 0) ? id_base + i : -1;
             ++nw;
         }
         int rc = (nw > cap_waiting) ? ORC_ELIMIT : ORC_OK;
@@ -424,10 +456,15 @@ int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, 
                 if (kind[r] == SCHED_PREFILL) {
                     run[r].ctx += alloc[r];
                     run[r].pre -= alloc[r];
-                    if (run[r].pre == 0 && mode == ORC_FIRST_TOKEN_WITH_LAST_CHUNK) run[r].dec -= 1;
+                    if (run[r].pre == 0 && mode == ORC_FIRST_TOKEN_WITH_LAST_CHUNK) {
+                        run[r].dec -= 1;
+                        if (track) first_token(&run[r], 1, t + (double)T, first_token_time);
+                    }
                 } else if (kind[r] == SCHED_DECODE) {
                     run[r].ctx += 1;
                     run[r].dec -= 1;
+                    if (track) first_token(&run[r], mode == ORC_FIRST_TOKEN_SEPARATE_DECODE, t + (double)T,
+                                           first_token_time);
                 }
             }
             int64_t keep = 0;
@@ -443,12 +480,14 @@ int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, 
                 run_ctx[o] = r < nr ? (int32_t)run[r].ctx : 0;
                 run_pre[o] = r < nr ? (int32_t)run[r].pre : 0;
                 run_dec[o] = r < nr ? (int32_t)run[r].dec : 0;
+                if (track) run_id[o] = r < nr ? run[r].id : -1;
             }
             n_wait[j] = (int32_t)(nw - wh);
             for (int64_t w = 0; w < cap_waiting; ++w) {
                 const int64_t o = (int64_t)j * cap_waiting + w;
                 wait_pre[o] = w < nw - wh ? (int32_t)wait[wh + w].pre : 0;
                 wait_dec[o] = w < nw - wh ? (int32_t)wait[wh + w].dec : 0;
+                if (track) wait_id[o] = w < nw - wh ? wait[wh + w].id : -1;
             }
             clock[j] = t;
         } else {

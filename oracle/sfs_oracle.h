@@ -131,6 +131,21 @@ int orc_advance(int32_t I, const int32_t *model_of_instance, const float *coef, 
                 const int32_t *prompt_len, const int32_t *dec, int32_t mode, double t_now,
                 int64_t max_batches);
 
+/* orc_advance that also follows tracked queries to their first output token (Sec. 4.1;
+ * Eq. 4 scores the realized TTFT).  run_id / wait_id ([I][cap], in/out) hold each
+ * request's tracking id or -1; routed query i joins as id_base + i (id_base < 0: -1).
+ * When a tracked request emits its first output token in an executed batch -- its first
+ * decode token, or the last prompt chunk's token when the first token comes with it --
+ * first_token_time[id] receives that batch's end time and the request's id becomes -1.
+ * NULL id arrays: nothing is tracked (exactly orc_advance). */
+int orc_advance_ids(int32_t I, const int32_t *model_of_instance, const float *coef, const int32_t *B,
+                    const int32_t *S, int32_t cap_running, int32_t cap_waiting, int32_t *n_run,
+                    int32_t *run_ctx, int32_t *run_pre, int32_t *run_dec, int32_t *n_wait, int32_t *wait_pre,
+                    int32_t *wait_dec, double *clock, int32_t Q, const int32_t *assign,
+                    const int32_t *prompt_len, const int32_t *dec, int32_t mode, double t_now,
+                    int64_t max_batches, int64_t *run_id, int64_t *wait_id, int64_t id_base,
+                    double *first_token_time);
+
 /* Utility of Eq. 2 with the cost of App. B.4 in canonical fp32. */
 float orc_utility(float acc, float lambda, int32_t p, int32_t dec_hat, float price_in, float price_out);
 
