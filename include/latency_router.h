@@ -301,6 +301,30 @@ LR_API int lr_calibrate(lr_ctx *ctx, int64_t N, const int64_t *features, const i
 LR_API int lr_advance(lr_ctx *ctx, int32_t Q, const int32_t *assign, const int32_t *prompt_len,
                       const int32_t *dec, int32_t dec_cols, double t_now, void *cuda_stream);
 
+/* Record when tracked queries emit their first output token in the executed stream
+ * (Sec. 4.1: the TTFT ends with the first output token; Eq. 4 scores each query by its
+ * realized TTFT).  first_token_time: [capacity] fp64 device array owned by the caller,
+ * 1 <= capacity < 2^31; NULL turns tracking off.  Queries appended by
+ * lr_advance_tracked with ids become tracked; when a tracked request's first output token
+ * comes out of a batch that a stream step executes -- its first decode token, or, with
+ * LR_FIRST_TOKEN_WITH_LAST_CHUNK, the token of the batch that completes its prompt --
+ * first_token_time[id] receives that batch's end time (the instance's fp64 clock after
+ * it) and the request stops being tracked.  Entries of ids that have not produced their
+ * first token yet are left as they are (e.g. NaN set by the caller).  Requests of a
+ * snapshot given to lr_load_state are untracked.  Synchronizes the device and makes every
+ * resident request untracked.  An advance whose snapshot is then rejected (LR_ETRAJ) may
+ * already have written entries for the batches it executed. */
+LR_API int lr_track_first_tokens(lr_ctx *ctx, double *first_token_time, int64_t capacity);
+
+/* lr_advance that tracks the appended queries: query i of this call (if assign[i] is an
+ * instance) gets id id_base + i.  id_base >= 0 needs tracking on (LR_EINVAL otherwise) and
+ * id_base + Q <= capacity (LR_ECAPACITY); id_base < 0 appends untracked queries, exactly
+ * like lr_advance.  Either call records the first tokens of tracked requests already
+ * queued. */
+LR_API int lr_advance_tracked(lr_ctx *ctx, int32_t Q, const int32_t *assign, const int32_t *prompt_len,
+                              const int32_t *dec, int32_t dec_cols, int64_t id_base, double t_now,
+                              void *cuda_stream);
+
 /* Copy the live snapshot (as advanced so far) into caller arrays: device pointers with the
  * shapes of lr_state_view plus clock [I] fp64; any pointer may be NULL to skip it. */
 LR_API int lr_read_state(const lr_ctx *ctx, int32_t *n_run, int32_t *run_ctx, int32_t *run_pre,

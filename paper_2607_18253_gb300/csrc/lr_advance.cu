@@ -38,7 +38,21 @@ __device__ void fail3(DevCtl *ctl, int code, int lane) {
     }
 }
 
-__device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, int lane, int32_t *wbase) {
+// First-token tracking (Sec. 4.1: the TTFT ends with the first output token; Eq. 4
+// scores the realized TTFT): a tracked request (id >= 0) that emits its first output
+// token in an executed batch -- its first decode token, or the token sampled with its
+// last prompt chunk in that mode -- records the batch's end time and drops its id.
+__device__ __forceinline__ int emit_first(const K3Launch &a, int id, bool emitted, double t_end) {
+    if (emitted && id >= 0) {
+        a.ftt[id] = t_end;
+        return -1;
+    }
+    return id;
+}
+
+// src: the live snapshot; idst: the buffer K1 publishes next (it receives the ids)
+__device__ void advance_instance(const K3Launch &a, const StateBuf &src, const StateBuf &idst, int j, int lane,
+                                 int32_t *wbase) {
     const DevConfig &c = a.cfg;
     const StateBuf &dst = a.scratch;
     const int B = c.B[j];
@@ -47,6 +61,8 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
     int32_t *rc0 = wbase, *rp0 = rc0 + capR, *rd0 = rp0 + capR;
     int32_t *rc1 = rd0 + capR, *rp1 = rc1 + capR, *rd1 = rp1 + capR;
     int32_t *wp = rd1 + capR, *wd = wp + capW;
+    int32_t *ri0 = wd + capW, *ri1 = ri0 + capR, *wi = ri1 + capR;  // ids (tracking only)
+    const bool track = a.track != 0;
     const size_t rrow = (size_t)j * capR, wrow = (size_t)j * capW;
     int nr = src.n_run[j];
     int nw = src.n_wait[j];
@@ -54,10 +70,12 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
         rc0[t] = src.run_ctx[rrow + t];
         rp0[t] = src.run_pre[rrow + t];
         rd0[t] = src.run_dec[rrow + t];
+        if (track) ri0[t] = src.run_id[rrow + t];
     }
     for (int t = lane; t < nw; t += 32) {
         wp[t] = src.wait_pre[wrow + t];
         wd[t] = src.wait_dec[wrow + t];
+        if (track) wi[t] = src.wait_id[wrow + t];
     }
     // routed queries join the waiting tail in query order
     for (int base = 0; base < a.Q; base += 32) {
@@ -69,6 +87,7 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
             if (pos < capW) {
                 wp[pos] = a.prompt[i];
                 wd[pos] = a.dec[(size_t)i * a.dec_cols + (a.dec_cols == 1 ? 0 : c.moi[j])];
+                if (track) wi[pos] = a.id_base >= 0 ? (int)(a.id_base + i) : -1;
             }
         }
         nw += __popc(bal);
@@ -92,7 +111,7 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
     double t = src.clock[j];
     int wh = 0, iters = 0;
     bool ok = true;
-    int32_t *rc = rc0, *rp = rp0, *rd = rd0, *nc = rc1, *np = rp1, *nd = rd1;
+    int32_t *rc = rc0, *rp = rp0, *rd = rd0, *nc = rc1, *np = rp1, *nd = rd1, *ri = ri0, *ni = ri1;
     while (true) {
         if (nr == 0 && wh == nw) {  // nothing to run: idle until t_now (never backwards)
             t = fmax(t, a.t_now);
@@ -119,6 +138,7 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
                 const int run = (int)min((long long)dmin, (long long)c.max_iters - iters);
                 const float f1 = 0.0f, f2 = __int2float_rn(nr), f4 = 0.0f;
                 int done = 0;
+                double t_first = t;  // end of the run's first batch, where every request decodes
                 for (; done < run; ++done) {
                     float T = __fmul_rn(b0, 1.0f);
                     T = __fmaf_rn(b1d, f2, T);
@@ -127,6 +147,7 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
                     T = __fmaf_rn(b3, f4, T);
                     if (t + (double)T > a.t_now) break;
                     t += (double)T;
+                    if (done == 0) t_first = t;
                 }
                 iters += done;
                 if (done > 0) {
@@ -135,6 +156,9 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
                         const int r = base + lane;
                         const bool live = r < nr;
                         const int dec = live ? rd[r] - done : 0;
+                        // every request decodes in the run's first batch: that is the first
+                        // token of a tracked one when the first token has its own batch
+                        const int id = (track && live) ? emit_first(a, ri[r], c.mode == 0, t_first) : -1;
                         const bool keep = live && dec > 0;
                         const unsigned bal = __ballot_sync(kFull, keep);
                         if (keep) {
@@ -142,17 +166,20 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
                             nc[pos] = rc[r] + done;
                             np[pos] = 0;
                             nd[pos] = dec;
+                            if (track) ni[pos] = id;
                         }
                         kept += __popc(bal);
                     }
                     __syncwarp();
-                    int32_t *x0 = rc, *x1 = rp, *x2 = rd;
+                    int32_t *x0 = rc, *x1 = rp, *x2 = rd, *x3 = ri;
                     rc = nc;
                     rp = np;
                     rd = nd;
+                    ri = ni;
                     nc = x0;
                     np = x1;
                     nd = x2;
+                    ni = x3;
                     nr = kept;
                 }
                 if (done < run) break;  // the next batch would end after t_now
@@ -229,7 +256,7 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
         long long wst = 0;
         for (int base = 0; base < total; base += 32) {
             const int r = base + lane;
-            int ctx = 0, pre = 0, dec = 0;
+            int ctx = 0, pre = 0, dec = 0, id = -1;
             long long need = 0;
             const bool live = r < total;
             if (live) {
@@ -238,10 +265,12 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
                     pre = rp[r];
                     dec = rd[r];
                     need = pre > 0 ? pre : 1;
+                    if (track) id = ri[r];
                 } else {
                     pre = wp[wh + r - nr];
                     dec = wd[wh + r - nr];
                     need = pre;
+                    if (track) id = wi[wh + r - nr];
                 }
             }
             const long long inr = (live && r < nr) ? need : 0;
@@ -255,10 +284,14 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
                 if (pre > 0) {
                     ctx += (int)x;
                     pre -= (int)x;
-                    if (pre == 0 && c.mode == 1) dec -= 1;  // first token with the last chunk
+                    if (pre == 0 && c.mode == 1) {
+                        dec -= 1;  // first token with the last chunk
+                        if (track) id = emit_first(a, id, true, t + (double)T);
+                    }
                 } else {
                     ctx += 1;
                     dec -= 1;
+                    if (track) id = emit_first(a, id, c.mode == 0, t + (double)T);
                 }
             }
             const bool keep = live && dec > 0;
@@ -268,19 +301,22 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
                 nc[pos] = ctx;
                 np[pos] = pre;
                 nd[pos] = dec;
+                if (track) ni[pos] = id;
             }
             kept += __popc(bal);
             used = __shfl_sync(kFull, incl_r, 31);
             wst = __shfl_sync(kFull, incl_w, 31);
         }
         __syncwarp();
-        int32_t *x0 = rc, *x1 = rp, *x2 = rd;
+        int32_t *x0 = rc, *x1 = rp, *x2 = rd, *x3 = ri;
         rc = nc;
         rp = np;
         rd = nd;
+        ri = ni;
         nc = x0;
         np = x1;
         nd = x2;
+        ni = x3;
         nr = kept;
         wh += na;
         t += (double)T;
@@ -298,6 +334,10 @@ __device__ void advance_instance(const K3Launch &a, const StateBuf &src, int j, 
     for (int q = lane; q < capW; q += 32) {
         dst.wait_pre[wrow + q] = q < nw2 ? wp[wh + q] : 0;
         dst.wait_dec[wrow + q] = q < nw2 ? wd[wh + q] : 0;
+    }
+    if (track) {
+        for (int q = lane; q < capR; q += 32) idst.run_id[rrow + q] = q < nr ? ri[q] : -1;
+        for (int q = lane; q < capW; q += 32) idst.wait_id[wrow + q] = q < nw2 ? wi[wh + q] : -1;
     }
     if (lane == 0) {
         dst.n_run[j] = nr;
@@ -318,8 +358,10 @@ __global__ void __launch_bounds__(kK3Warps * 32) k_advance(const K3Launch a) {
         return;
     }
     const StateBuf src = active ? a.buf1 : a.buf0;
+    // the buffer the summary (K1) publishes next, as K1 chooses it from the same index
+    const StateBuf idst = active ? a.buf0 : a.buf1;
     const size_t per_warp = advance_smem_per_warp(a.cfg) / sizeof(int32_t);
-    advance_instance(a, src, j, lane, k3_smem + wid * per_warp);
+    advance_instance(a, src, idst, j, lane, k3_smem + wid * per_warp);
 }
 
 // Copy of the live snapshot into caller arrays (the live buffer is known only on

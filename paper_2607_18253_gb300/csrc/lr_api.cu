@@ -22,6 +22,8 @@ struct lr_ctx {
     int device = 0;
     int sms = 0;
     float *static_tch = nullptr;  // device address of g_static_route_tch on this context's device
+    double *ftt = nullptr;        // first-token times of tracked queries (caller's array), or none
+    int64_t ftt_cap = 0;
     lr::DevConfig cfg{};
     lr::StateBuf buf[2]{};
     lr::StateBuf scratch{};  // advanced snapshot before it is summarized
@@ -99,6 +101,18 @@ int floor_log2(long long x) {
 int round_up(int x, int m) { return ((x + m - 1) / m) * m; }
 
 bool finite_nonneg(float v) { return std::isfinite(v) && v >= 0.0f; }
+
+// Every request of both snapshot buffers untracked (-1), on `stream` (nullptr: the
+// legacy stream).
+cudaError_t reset_ids(lr_ctx *c, void *stream) {
+    const size_t R = (size_t)c->cfg.I * c->cfg.capR, W = (size_t)c->cfg.I * c->cfg.capW;
+    cudaError_t e = cudaSuccess;
+    for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+        e = cudaMemsetAsync(c->buf[b].run_id, 0xff, R * sizeof(int32_t), (cudaStream_t)stream);
+        if (e == cudaSuccess) e = cudaMemsetAsync(c->buf[b].wait_id, 0xff, W * sizeof(int32_t), (cudaStream_t)stream);
+    }
+    return e;
+}
 
 // The live-buffer index and its copies, from the host (no kernel of the context may
 // be running); the other control words start at zero.
@@ -323,6 +337,8 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
         LR_ALLOC(s.f2, (size_t)kph * I);
         LR_ALLOC(s.f3, (size_t)kph * I);
         LR_ALLOC(s.rcum, (size_t)kph * I);
+        LR_ALLOC(s.run_id, R);
+        LR_ALLOC(s.wait_id, W);
     }
     {
         lr::StateBuf &s = c->scratch;
@@ -428,7 +444,10 @@ int lr_load_state(lr_ctx *c, const lr_state_view *v, void *stream) {
     a.ctl = c->ctl;
     a.in = lr::StateIn{v->n_run, v->run_ctx, v->run_pre, v->run_dec, v->n_wait, v->wait_pre, v->wait_dec, nullptr};
     const int grid = (c->cfg.I + lr::kK1Warps - 1) / lr::kK1Warps;
-    cudaError_t e = lr::launch_trajectory(a, grid, lr::kK1Warps * 32, c->k1_smem, (cudaStream_t)stream);
+    // a loaded snapshot's requests are untracked (only the stream step assigns ids)
+    cudaError_t e = c->ftt ? reset_ids(c, stream) : cudaSuccess;
+    if (e != cudaSuccess) return cuda_fail(c, e, "tracking reset");
+    e = lr::launch_trajectory(a, grid, lr::kK1Warps * 32, c->k1_smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(c, e, "trajectory launch");
     c->load_stream = stream;
     c->loaded_any = true;
@@ -774,8 +793,34 @@ int lr_calibrate(lr_ctx *c, int64_t N, const int64_t *features, const int32_t *m
 
 int lr_advance(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_t *prompt_len, const int32_t *dec,
                int32_t dec_cols, double t_now, void *stream) {
+    return lr_advance_tracked(c, Q, assign, prompt_len, dec, dec_cols, -1, t_now, stream);
+}
+
+int lr_track_first_tokens(lr_ctx *c, double *first_token_time, int64_t capacity) {
     if (!c) return LR_EINVAL;
     c->err.clear();
+    if (!first_token_time) {
+        c->ftt = nullptr;
+        c->ftt_cap = 0;
+        return LR_OK;
+    }
+    if (capacity < 1 || capacity > (1LL << 31) - 1) return fail(c, LR_EINVAL, "capacity must be in [1, 2^31 - 1]");
+    cudaError_t e = cudaDeviceSynchronize();
+    e = e == cudaSuccess ? reset_ids(c, nullptr) : e;
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(c, e, "tracking reset");
+    c->ftt = first_token_time;
+    c->ftt_cap = capacity;
+    return LR_OK;
+}
+
+int lr_advance_tracked(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_t *prompt_len, const int32_t *dec,
+                       int32_t dec_cols, int64_t id_base, double t_now, void *stream) {
+    if (!c) return LR_EINVAL;
+    c->err.clear();
+    if (id_base >= 0 && !c->ftt) return fail(c, LR_EINVAL, "first-token tracking is off (lr_track_first_tokens)");
+    if (id_base >= 0 && (Q > c->ftt_cap || id_base > c->ftt_cap - Q))
+        return fail(c, LR_ECAPACITY, "ids id_base .. id_base + Q - 1 exceed the tracking capacity");
     if (Q < 0) return fail(c, LR_EINVAL, "Q < 0");
     if (Q > 0 && (!assign || !prompt_len || !dec)) return fail(c, LR_EINVAL, "null array");
     if (dec_cols != 1 && dec_cols != c->cfg.M) return fail(c, LR_EINVAL, "dec_cols must be 1 or num_models");
@@ -796,6 +841,9 @@ int lr_advance(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_t *promp
     k.dec = dec;
     k.dec_cols = dec_cols;
     k.t_now = t_now;
+    k.track = c->ftt != nullptr;
+    k.id_base = id_base;
+    k.ftt = c->ftt;
     cudaStream_t st = (cudaStream_t)stream;
     cudaError_t e = lr::launch_advance(k, (c->cfg.I + lr::kK3Warps - 1) / lr::kK3Warps, c->k3_smem, st);
     if (e != cudaSuccess) return cuda_fail(c, e, "advance launch");

@@ -90,6 +90,9 @@ struct StateBuf {
     KvInst *kvi;   // [I], with KV limits
     KvRec *kvr;    // [I][horizon], with KV limits
     int32_t *kvp;  // [I][horizon] running maximum of the records' thr (clamped to int32), with KV limits
+    // first-token tracking (lr_track_first_tokens): each request's id until its first output
+    // token, else -1; written by the stream step only (a snapshot load makes every request -1)
+    int32_t *run_id, *wait_id;  // [I][capR], [I][capW]
 };
 
 // Copies of the live-buffer index, each in its own 128-byte line: the CTAs of a
@@ -345,12 +348,18 @@ struct K3Launch {
     int32_t dec_cols;  // 1: dec[i]; M: dec[i][model of the chosen instance]
     const int32_t *assign, *prompt, *dec;
     double t_now;
+    // first-token tracking: the appended query i gets id id_base + i (id_base < 0: -1);
+    // ftt[id] receives the end time of the batch with its first output token
+    int32_t track;
+    long long id_base;
+    double *ftt;
 };
 constexpr int kK3Warps = 4;
-// Shared memory of one K3 warp: the running list twice (ctx, pre, dec; the
-// batch's survivors are compacted into the other copy) and the waiting queue.
+// Shared memory of one K3 warp: the running list twice (ctx, pre, dec, id; the
+// batch's survivors are compacted into the other copy) and the waiting queue (pre,
+// dec, id).
 __host__ __device__ inline size_t advance_smem_per_warp(const DevConfig &c) {
-    return sizeof(int32_t) * ((size_t)6 * c.capR + (size_t)2 * c.capW + 32);
+    return sizeof(int32_t) * ((size_t)8 * c.capR + (size_t)3 * c.capW + 32);
 }
 cudaError_t launch_advance(const K3Launch &a, int grid, size_t smem, cudaStream_t st);
 cudaError_t set_k3_smem(size_t bytes);

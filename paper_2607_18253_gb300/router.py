@@ -26,7 +26,8 @@ LR_POLICY_ROUND_ROBIN, LR_POLICY_SHORTEST_QUEUE, LR_POLICY_LATENCY_AGNOSTIC = 0,
 EXPORTED_SYMBOLS = ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
                     "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
                     "lr_set_queue_params", "lr_set_ttft_source", "lr_calibrate", "lr_route_baseline",
-                    "lr_on_time_utility", "lr_set_kv_limits", "lr_strerror", "lr_last_error")
+                    "lr_on_time_utility", "lr_set_kv_limits", "lr_strerror", "lr_last_error",
+                    "lr_track_first_tokens", "lr_advance_tracked")
 
 _P = ctypes.c_void_p
 _I32 = ctypes.c_int32
@@ -68,6 +69,8 @@ def load_library(path: str = LIB_PATH):
     lib.lr_route.argtypes = [_P, _I32, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.lr_route_frontier_static.argtypes = [_P, _I32, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P]
     lib.lr_advance.argtypes = [_P, _I32, _P, _P, _P, _I32, ctypes.c_double, _P]
+    lib.lr_advance_tracked.argtypes = [_P, _I32, _P, _P, _P, _I32, ctypes.c_int64, ctypes.c_double, _P]
+    lib.lr_track_first_tokens.argtypes = [_P, _P, ctypes.c_int64]
     lib.lr_set_queue_params.argtypes = [_P, ctypes.POINTER(_QueueParams), _P]
     lib.lr_set_ttft_source.argtypes = [_P, _I32]
     lib.lr_calibrate.argtypes = [_P, ctypes.c_int64, _P, _P, _P, _I32, _P, _P]
@@ -83,7 +86,7 @@ def load_library(path: str = LIB_PATH):
     for name in ("lr_create", "lr_destroy", "lr_load_state", "lr_estimate_ttft", "lr_estimate_features",
                  "lr_route", "lr_route_frontier_static", "lr_advance", "lr_read_state", "lr_status",
                  "lr_set_queue_params", "lr_set_ttft_source", "lr_calibrate", "lr_route_baseline",
-                 "lr_on_time_utility", "lr_set_kv_limits"):
+                 "lr_on_time_utility", "lr_set_kv_limits", "lr_advance_tracked", "lr_track_first_tokens"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -332,17 +335,30 @@ class LatencyRouter:
         return out
 
     def advance(self, assign: torch.Tensor, prompt_len: torch.Tensor, dec: torch.Tensor, t_now: float,
-                stream=None):
+                stream=None, id_base: Optional[int] = None):
         """Append routed queries (assign[i] >= 0) and advance every instance to t_now.
 
-        dec is [Q] (one output length per query) or [Q, M] (the chosen model's column is used)."""
+        dec is [Q] (one output length per query) or [Q, M] (the chosen model's column is used).
+        id_base: track query i of this call as id id_base + i (lr_advance_tracked)."""
         Q = int(assign.numel())
         cols = 1 if dec.dim() == 1 else int(dec.shape[1])
-        self._check(self._lib.lr_advance(self._h, Q, _dev(assign, torch.int32, "assign"),
-                                         _dev(prompt_len, torch.int32, "prompt_len", Q),
-                                         _dev(dec, torch.int32, "dec", Q * cols), cols, float(t_now),
-                                         _stream(stream)),
-                    "lr_advance")
+        args = (_dev(assign, torch.int32, "assign"), _dev(prompt_len, torch.int32, "prompt_len", Q),
+                _dev(dec, torch.int32, "dec", Q * cols), cols)
+        if id_base is None:
+            rc = self._lib.lr_advance(self._h, Q, *args, float(t_now), _stream(stream))
+        else:
+            rc = self._lib.lr_advance_tracked(self._h, Q, *args, int(id_base), float(t_now), _stream(stream))
+        self._check(rc, "lr_advance")
+
+    def track_first_tokens(self, first_token_time: Optional[torch.Tensor]):
+        """Record tracked queries' first-token times into first_token_time [N] fp64 (None: off)."""
+        if first_token_time is None:
+            self._check(self._lib.lr_track_first_tokens(self._h, None, 0), "lr_track_first_tokens")
+            return
+        self._check(self._lib.lr_track_first_tokens(self._h, _dev(first_token_time, torch.float64,
+                                                                  "first_token_time"),
+                                                    int(first_token_time.numel())),
+                    "lr_track_first_tokens")
 
     def read_state(self, device="cuda", stream=None) -> dict:
         """The live snapshot as device tensors (n_run, run_ctx, ..., wait_dec, clock)."""

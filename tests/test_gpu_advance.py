@@ -216,3 +216,66 @@ def test_advance_beyond_max_iters_keeps_previous_snapshot():
     assert rt.status() == R().LR_OK
     w2, c2 = oracle.advance(wl, np.zeros(wl.num_instances), [], [], [], 0.05)
     check_state(read(rt), w2, c2)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_first_token_times_match_the_oracle(mode):
+    # random small pools, four successive advances with tracked appends (one of them
+    # untracked), the last one draining everything: every first-token time equal to the
+    # oracle's, bit for bit, and the same queries without one until then
+    for seed in range(8):
+        rng = np.random.default_rng(2000 + seed)
+        wl = W.small_workload(seed, num_instances=int(3 + seed % 29), num_models=3, num_queries=48,
+                              cap_running=64, cap_waiting=200, first_token_mode=mode, wait_max=24,
+                              budget_range=(8, 64), min_gap=8)
+        rt = make_router(wl)
+        N = 4 * 40
+        ftt = torch.full((N,), float("nan"), dtype=torch.float64, device="cuda")
+        rt.track_first_tokens(ftt)
+        tr = oracle.new_track(wl, N)
+        clk = np.zeros(wl.num_instances)
+        for step, t_now in enumerate((4.0, 9.0, 15.0, 1e7)):
+            Q = 40
+            a = rng.integers(-1, wl.num_instances, Q).astype(np.int32)
+            p = rng.integers(1, 160, Q).astype(np.int32)
+            d = rng.integers(1, 30, Q).astype(np.int32)
+            base = None if step == 2 else 40 * step
+            rt.advance(dev(a), dev(p), dev(d), t_now, id_base=base)
+            torch.cuda.synchronize()
+            assert rt.status() == R().LR_OK, (seed, step)
+            wl, clk, tr = oracle.advance(wl, clk, a, p, d, t_now, track=tr, id_base=-1 if base is None else base)
+            check_state(read(rt), wl, clk)
+            got, exp = ftt.cpu().numpy(), tr["first_token_time"]
+            np.testing.assert_array_equal(np.isnan(got), np.isnan(exp), err_msg=f"seed {seed} step {step}")
+            np.testing.assert_array_equal(got[~np.isnan(exp)].view(np.uint64), exp[~np.isnan(exp)].view(np.uint64))
+        # everything drained; the untracked step's ids were never given out
+        assert np.isnan(got[80:120]).all()
+        assert np.isfinite(got[:80]).sum() > 0
+        rt.close()
+
+
+def test_tracking_errors_and_reload():
+    wl = W.make_workload("tiny", cap_running=64)
+    rt = make_router(wl)
+    a = dev(np.zeros(4, np.int32))
+    p = dev(np.full(4, 10, np.int32))
+    d = dev(np.full(4, 3, np.int32))
+    with pytest.raises(R().LRError) as e:  # ids without tracking
+        rt.advance(a, p, d, 1.0, id_base=0)
+    assert e.value.code == R().LR_EINVAL
+    ftt = torch.full((6,), float("nan"), dtype=torch.float64, device="cuda")
+    rt.track_first_tokens(ftt)
+    with pytest.raises(R().LRError) as e:  # ids 3 .. 6 beyond the capacity of 6
+        rt.advance(a, p, d, 1.0, id_base=3)
+    assert e.value.code == R().LR_ECAPACITY
+    rt.advance(a, p, d, 1.0, id_base=2)
+    # a reload makes every request untracked: draining it records nothing more
+    rt.load_state(*R().state_tensors(wl))
+    before = ftt.cpu().numpy().copy()
+    rt.advance(a[:0], p[:0], d[:0], 1e7)
+    torch.cuda.synchronize()
+    assert rt.status() == R().LR_OK
+    after = ftt.cpu().numpy()
+    np.testing.assert_array_equal(np.isnan(after), np.isnan(before))
+    rt.track_first_tokens(None)
+    rt.close()

@@ -194,6 +194,9 @@ def test_stream_micro_batches(stream_trace, m):
     assign = torch.empty((nb, m), dtype=torch.int32, device="cuda")
     util = torch.empty((nb, m), dtype=torch.float32, device="cuda")
     tch = torch.empty((nb, m), dtype=torch.float32, device="cuda")
+    # every routed query is tracked to its first output token (its id = its trace index)
+    ftt = torch.full((n,), float("nan"), dtype=torch.float64, device="cuda")
+    rt.track_first_tokens(ftt)
     import ctypes
     V = ctypes.c_void_p
     sp = V(torch.cuda.current_stream().cuda_stream)
@@ -203,7 +206,7 @@ def test_stream_micro_batches(stream_trace, m):
         if b == 0:
             rt.advance(assign[0, :0], p[:0], dh[:0], t_now)
         else:
-            rt.advance(assign[b - 1], p[lo - m:lo], dh[lo - m:lo], t_now)
+            rt.advance(assign[b - 1], p[lo - m:lo], dh[lo - m:lo], t_now, id_base=lo - m)
         rc = lib.lr_read_state(h, *(V(snaps[k][b].data_ptr()) for k in STATE + ("clock",)), sp)
         assert rc == 0
         rt.route(p[lo:lo + m], dh[lo:lo + m], acc[lo:lo + m], wl.lam, wl.mu,
@@ -212,20 +215,22 @@ def test_stream_micro_batches(stream_trace, m):
     assert rt.status() == R().LR_OK
     snaps = {k: v.cpu().numpy() for k, v in snaps.items()}
     assign, util, tch = assign.cpu().numpy(), util.cpu().numpy(), tch.cpu().numpy()
+    ftt = ftt.cpu().numpy()
     rt.close()
 
     st, clk = wl, np.zeros(I)
+    tr = oracle.new_track(wl, n)
     none = np.zeros(0, np.int32)
     prev = None
     for b in range(nb):
         lo = b * m
         t_now = float(arr[lo + m - 1])
         if prev is None:
-            st, clk = oracle.advance(st, clk, none, none, none, t_now)
+            st, clk, tr = oracle.advance(st, clk, none, none, none, t_now, track=tr)
         else:
             pa, pq = prev
             d = np.ascontiguousarray(pq.dec_hat[np.arange(m), wl.model_of_instance[np.maximum(pa, 0)]])
-            st, clk = oracle.advance(st, clk, pa, pq.prompt_len, d, t_now)
+            st, clk, tr = oracle.advance(st, clk, pa, pq.prompt_len, d, t_now, track=tr, id_base=lo - m)
         np.testing.assert_array_equal(snaps["n_run"][b], st.n_run, err_msg=f"decision {b}")
         np.testing.assert_array_equal(snaps["n_wait"][b], st.n_wait, err_msg=f"decision {b}")
         np.testing.assert_array_equal(snaps["clock"][b].view(np.uint64), clk.view(np.uint64),
@@ -247,3 +252,9 @@ def test_stream_micro_batches(stream_trace, m):
         prev = (a[0], q)
     # the trace kept the pool busy: work arrived and queues formed somewhere
     assert st.n_run.sum() > 0
+    # the realized first-token times (Eq. 4's realized TTFT): the same queries have one, at
+    # the same fp64 times
+    ot = tr["first_token_time"]
+    np.testing.assert_array_equal(np.isnan(ftt), np.isnan(ot))
+    np.testing.assert_array_equal(ftt[~np.isnan(ot)].view(np.uint64), ot[~np.isnan(ot)].view(np.uint64))
+    assert (~np.isnan(ot)).sum() > n // 2
