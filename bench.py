@@ -41,7 +41,7 @@ WORKLOAD = "pool256"
 # DRAM bytes (read + write) per launch of the step's kernels on this workload, from one
 # ncu capture of the kernels as they are built now (summaries under profiles/); they
 # are retaken whenever one of the kernels changes.
-NCU_TRAFFIC = {"k_route": 4_579_328 + 8_607_488, "k_trajectory": 1_392_896, "k_estimate": 357_376 + 7_084_800}
+NCU_TRAFFIC = {"k_route": 4_577_792 + 8_019_712, "k_trajectory": 1_393_408, "k_estimate": 357_888 + 7_386_624}
 
 
 def _peaks():
@@ -928,11 +928,14 @@ def _policy_eval(rt, wl, arr, dev, p, dh, acc):
     The first POLICY_QUERIES arrivals are routed in micro-batches of POLICY_BATCH at the
     arrival of each batch's last query, by the constrained objective (Eq. 3) on SFS
     estimates or by a baseline policy; every batch joins its chosen instances before the
-    next is routed.  A query's realized TTFT is the time it waited for the decision
-    plus the chosen instance's SFS estimate (the synthetic engine runs the same batch
-    model), on time if within its target; OnTimeUtility and SLO attainment come from
-    lr_on_time_utility.  Also reported: mean utility, mean realized TTFT, and the device
-    time per micro-batch (advance + route)."""
+    next is routed, tracked to its first output token (lr_advance_tracked), and the
+    pool is finally run until every query has one.  A query's realized TTFT is its
+    first-token time in that executed stream minus its arrival: it includes the wait for
+    the decision and the batches that later queries lengthened, which no estimate made
+    at the decision can see.  On time if within its target; OnTimeUtility and SLO
+    attainment come from lr_on_time_utility.  Also reported: the same two metrics with
+    the decision-time view (decision delay + the chosen instance's SFS estimate), mean
+    utility, mean realized TTFT, and the device time per micro-batch (advance + route)."""
     import ctypes
 
     import torch
@@ -956,8 +959,12 @@ def _policy_eval(rt, wl, arr, dev, p, dh, acc):
     up, tp = util.data_ptr(), ttft.data_ptr()
     ap = [assign[0].data_ptr(), assign[1].data_ptr()]
     state = R.state_tensors(wl, dev)
+    ftt = torch.empty(nb * m, dtype=torch.float64, device=dev)
+    arr_d = torch.from_numpy(np.ascontiguousarray(arr[:nb * m], np.float64)).to(dev)
     res = {}
     for name, pol in POLICIES:
+        ftt.fill_(float("nan"))
+        rt.track_first_tokens(ftt)
         rt.load_state(*state)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         torch.cuda.synchronize()
@@ -967,8 +974,8 @@ def _policy_eval(rt, wl, arr, dev, p, dh, acc):
             cur, prev = ap[b & 1], ap[(b - 1) & 1]
             pm = m if b > 0 else 0
             plo = max((b - 1) * m, 0)
-            rc = lib.lr_advance(h, pm, V(prev), V(pp + 4 * plo), V(dhp + 4 * M * plo), M,
-                                ctypes.c_double(float(td[lo])), sp)
+            rc = lib.lr_advance_tracked(h, pm, V(prev), V(pp + 4 * plo), V(dhp + 4 * M * plo), M,
+                                        ctypes.c_int64(plo), ctypes.c_double(float(td[lo])), sp)
             if pol is None:
                 rc |= lib.lr_route(h, m, V(pp + 4 * lo), V(dhp + 4 * M * lo), V(accp + 4 * M * lo), V(taup + 4 * lo),
                                    1, lamp, None, V(cur), V(up + 4 * lo), V(tp + 4 * lo), None, None, sp)
@@ -979,20 +986,38 @@ def _policy_eval(rt, wl, arr, dev, p, dh, acc):
             if rc:
                 raise RuntimeError(f"policy run {name} failed: {lib.lr_last_error(h).decode()}")
         e1.record()
+        fin = rt.read_state(device=dev)
+        # the last batch joins, then the pool runs until every routed query has its first token
+        plo = (nb - 1) * m
+        rc = lib.lr_advance_tracked(h, m, V(ap[(nb - 1) & 1]), V(pp + 4 * plo), V(dhp + 4 * M * plo), M,
+                                    ctypes.c_int64(plo), ctypes.c_double(1e9), sp)
+        if rc:
+            raise RuntimeError(f"policy run {name} failed: {lib.lr_last_error(h).decode()}")
         torch.cuda.synchronize()
         st = rt.status()
         if st != R.LR_OK:
             raise RuntimeError(f"policy run {name} ended with device status {st}")
-        otu, slo = (float(x) for x in rt.on_time_utility(util, ttft, tau, delay).cpu().numpy())
-        realized = (delay + ttft).cpu().numpy()
-        fin = rt.read_state(device=dev)
+        if torch.isnan(ftt).any():
+            raise RuntimeError(f"policy run {name}: a query never produced its first token")
+        realized = (ftt - arr_d).to(torch.float32)
+        otu, slo = (float(x) for x in rt.on_time_utility(util, realized, tau).cpu().numpy())
+        otu_e, slo_e = (float(x) for x in rt.on_time_utility(util, ttft, tau, delay).cpu().numpy())
+        gap = (realized - (delay + ttft)).double()
         res[name] = {"on_time_utility": otu, "slo_attainment": slo, "mean_utility": float(util.mean().item()),
-                     "mean_realized_ttft_s": float(realized.mean()), "us_per_batch": e0.elapsed_time(e1) * 1e3 / nb,
+                     "mean_realized_ttft_s": float(realized.double().mean().item()),
+                     "decision_view": {"on_time_utility": otu_e, "slo_attainment": slo_e,
+                                       "mean_ttft_s": float((delay + ttft).double().mean().item())},
+                     "realized_minus_decision_view_s": {"mean": float(gap.mean().item()),
+                                                        "max": float(gap.max().item()),
+                                                        "min": float(gap.min().item())},
+                     "us_per_batch": e0.elapsed_time(e1) * 1e3 / nb,
                      "final_max_waiting": int(fin["n_wait"].max().item())}
+    rt.track_first_tokens(None)
     return {"queries": nb * m, "micro_batch": m, "lambda": float(lam[0]),
             "objective": "SFS router: Eq. 3 (max utility within the TTFT target, else least TTFT)",
-            "realized_ttft": "decision delay + SFS estimate of the chosen instance",
-            "policies": res, "gpu_launches": len(POLICIES) * (3 * nb + 3)}
+            "realized_ttft": "first-token time in the executed stream (lr_advance_tracked) - arrival; "
+                             "decision_view: decision delay + SFS estimate of the chosen instance",
+            "policies": res, "gpu_launches": len(POLICIES) * (3 * nb + 3 + 2)}
 
 
 def _host_cpu():
