@@ -445,9 +445,139 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
             return true;
         };
 
+        // A window of up to 32 batches l .. l + 31 stepped without touching shared memory
+        // per batch, while only the token budget and free sequence slots limit admission.
+        // In FCFS order the prefill tokens form one stream: the carried prefill, then the
+        // waiting prompts.  Batch b serves its decoders one token each and gives the stream
+        // min(B - n_b, the end of the last prompt a free sequence slot lets start); the
+        // prompts completed in batch b become decoders from b + 1; n_{b+1} = n_b + (new
+        // decoders) - (decoders ending in batch b: the calendar's and those created in
+        // this window).  Lane k holds stream entry k (start, end, context at completion,
+        // decode length, completion batch) and lane w the calendar count of batch l + w;
+        // each batch is a few ballots and shuffles, one shuffle and one ballot on the
+        // chain from n_b to n_{b+1}.  The window stops before a batch with every slot taken
+        // by decoders (the seat-limited path takes those), one that would need an entry
+        // beyond the lanes, one at or past the calendar's end, one in which the queue could
+        // run out (the admission batch is the scalar step's), or after 32 batches.
+        // Returns the batches taken (0: none).
+        auto window = [&]() -> int {
+            __syncwarp();  // the leading lane's appends are visible to every lane
+            const int pfo = pf ? 1 : 0;
+            const int base = pf ? pfR : 0;
+            const int q = head + lane - pfo;  // waiting request of this lane's entry
+            bool valid;
+            int st0, en, ce, d;
+            if (pf && lane == 0) {
+                valid = true;
+                st0 = -1;
+                en = pfR;
+                ce = pfC + pfR;
+                d = pfD;
+            } else {
+                valid = q < nw;
+                const int a0 = valid ? lds(sP + 4u * q) : 0;
+                const int a1 = valid ? lds(sP + 4u * (q + 1)) : 0;
+                st0 = base + a0 - ph;
+                en = valid ? base + a1 - ph : kBig;
+                ce = a1 - a0;
+                d = valid ? lds(sW + 4u * q) : 0;
+            }
+            const bool dc = valid && (MODE == 0 || d >= 2);  // becomes a decoder when it completes
+            const int fl0 = d - MODE;                        // last decode batch - completion batch
+            const unsigned dcm = __ballot_sync(kFull, dc);
+            const int nent = __popc(__ballot_sync(kFull, valid));
+            const int last_end = __shfl_sync(kFull, en, max(nent - 1, 0));
+            const int total_left = base + lds(sP + 4u * nw) - ph;
+            const int lb = l + lane;
+            const int calw = lb < kCalendar ? lds(tr.cal + 4u * lb) : -1;
+            const unsigned calok = __ballot_sync(kFull, calw >= 0);
+            int T = 0, nn = n, w = 0, ndone = 0;
+            bool ip = pf;            // a prompt is part-way at the start of the batch
+            int dn = -1, fl = kBig;  // this lane's completion batch and last decode batch
+            while (w < 32 && ((calok >> w) & 1u)) {
+                const int lw = l + w;
+                // decoders ending in batch lw: the calendar's and this window's (off the chain)
+                const int ecal = __shfl_sync(kFull, calw, w);
+                const int ewin = __popc(__ballot_sync(kFull, dn >= 0 && fl == lw) & dcm);
+                const int freeseats = S - nn - (ip ? 1 : 0);
+                if (freeseats <= 0 && !ip) break;  // every slot holds a decoder
+                const int budget = B - nn;
+                if (budget <= 0) break;
+                int T2 = T + budget;
+                if (T2 >= total_left) break;  // the queue could run out in this batch
+                if (freeseats > 0) {
+                    const int kl = ndone + (ip ? 1 : 0) + freeseats - 1;  // last entry a free slot lets start
+                    const int lim = __shfl_sync(kFull, en, min(kl, 31));
+                    if (kl < nent) T2 = min(T2, lim);
+                    else if (T2 > last_end) break;  // beyond the lanes
+                } else {
+                    T2 = min(T2, __shfl_sync(kFull, en, ndone & 31));  // only the prefill in progress advances
+                }
+                const bool nd = valid && dn < 0 && en <= T2;
+                if (nd) {
+                    dn = lw;
+                    fl = lw + fl0;
+                }
+                const unsigned ndm = __ballot_sync(kFull, nd);
+                ip = __ballot_sync(kFull, valid && st0 < T2 && T2 < en) != 0u;
+                ndone += __popc(ndm);
+                nn += __popc(ndm & dcm) - ecal - ewin;
+                T = T2;
+                ++w;
+            }
+            if (w == 0) return 0;
+            // the window's new decoders, in completion (stream) order
+            const bool ap = dn >= 0 && dc;
+            const unsigned apm = __ballot_sync(kFull, ap);
+            unsigned wlo = 0u, whi = 0u;
+            if (ap) {
+                sts4(tr.dl + 16u * (tr.nlist + __popc(apm & lanemask_lt())), dn + 1, fl, ce - (dn + 1), 0);
+                if (fl < kCalendar) {
+                    red_add(tr.cal + 4u * fl, 1);
+                    red_or(tr.bm + 4u * (fl >> 5), 1u << (fl & 31));
+                    if (fl < kCalendar / 2) wlo |= 1u << (fl >> 5);
+                    else whi |= 1u << ((fl >> 5) - 32);
+                }
+            }
+            tr.words |= ((unsigned long long)__reduce_or_sync(kFull, whi) << 32) | __reduce_or_sync(kFull, wlo);
+            tr.nlist += __popc(apm);
+            // the new stream position: started prompts leave the queue; the entry in progress
+            // at T, if any, is the prefill carried into batch l + w
+            head += __popc(__ballot_sync(kFull, valid && lane >= pfo && st0 < T));
+            ph = lds(sP + 4u * head);
+            const int snd = __shfl_sync(kFull, st0, ndone & 31);
+            const int end_nd = __shfl_sync(kFull, en, ndone & 31);
+            const int ce_nd = __shfl_sync(kFull, ce, ndone & 31);
+            const int d_nd = __shfl_sync(kFull, d, ndone & 31);
+            if (ndone < nent && snd < T) {
+                pf = true;
+                pfR = end_nd - T;
+                pfC = ce_nd - pfR;
+                pfD = d_nd;
+            } else {
+                pf = false;
+            }
+            n = nn;
+            // the next end: the calendar's within the lanes' batches, or one of the window's
+            // new decoders, else a search
+            const unsigned cm = __ballot_sync(kFull, calw > 0) & (w < 32 ? (~0u << w) : 0u);
+            const int fc = cm ? l + __ffs(cm) - 1 : kBig;
+            const int fm = __reduce_min_sync(kFull, (ap && fl >= l + w) ? fl : kBig);
+            l += w;
+            fnext = (fc < kBig) ? min(fc, fm) : tr.next_end(l);
+            return w;
+        };
+
         while (iters < c.max_iters && l < (1 << 30)) {
             ++iters;
             int cnt = n + (pf ? 1 : 0);  // requests running in batch l
+            if (pf || cnt < S) {
+                const int wt = window();  // every batch of a window counts against max_iters
+                if (wt > 0) {
+                    iters += wt - 1;
+                    continue;
+                }
+            }
             if (!pf && cnt >= S) {
                 // Every sequence slot is taken: nothing but decoding until one frees.
                 if (fnext == kBig) break;  // excluded: a decoder is running
