@@ -95,6 +95,9 @@ def _load():
         lib.orc_advance_ids.argtypes = [i32, P, P, P, P, i32, i32, P, P, P, P, P, P, P, P, i32, P, P, P, i32,
                                         ctypes.c_double, i64, P, P, i64, P]
         lib.orc_advance_ids.restype = ctypes.c_int
+        lib.orc_advance_kv.argtypes = [i32, P, P, P, P, i32, i32, P, P, P, P, P, P, P, P, i32, P, P, P, i32,
+                                       ctypes.c_double, i64, P, P, P, P, P, i64, P]
+        lib.orc_advance_kv.restype = ctypes.c_int
         lib.orc_utility.argtypes = [ctypes.c_float, ctypes.c_float, i32, i32, ctypes.c_float, ctypes.c_float]
         lib.orc_utility.restype = ctypes.c_float
         lib.orc_pow_int.argtypes = [ctypes.c_double, i32]
@@ -254,14 +257,16 @@ def frontier(wl, assign: np.ndarray, ttft_chosen: np.ndarray) -> np.ndarray:
 
 
 def advance(wl, clock, assign, prompt_len, dec, t_now: float, max_batches: int = 1 << 30, track=None,
-            id_base: int = -1):
+            id_base: int = -1, kv=None):
     """Online stream step on a copy of the workload's state.
 
     Returns (new workload with the advanced state, new clocks).  With `track` -- a dict of
     run_id [I, cap_running] int64, wait_id [I, cap_waiting] int64 and first_token_time [N]
     float64 -- the routed query i joins as id id_base + i (id_base >= 0) and every tracked
     request that emits its first output token in an executed batch gets that batch's end
-    time; the call then returns (workload, clocks, new track dict)."""
+    time; the call then returns (workload, clocks, new track dict).  With `kv` =
+    (block_size, num_blocks, max_ctx), scalars or per-instance arrays, every executed
+    batch follows the KV step rule (orc_advance_kv)."""
     import dataclasses
     st = {k: np.array(getattr(wl, k), dtype=np.int32, copy=True)
           for k in ("n_run", "run_ctx", "run_pre", "run_dec", "n_wait", "wait_pre", "wait_dec")}
@@ -275,13 +280,20 @@ def advance(wl, clock, assign, prompt_len, dec, t_now: float, max_batches: int =
     if track is not None:
         tr = {k: np.array(track[k], dtype=(np.float64 if k == "first_token_time" else np.int64), copy=True)
               for k in ("run_id", "wait_id", "first_token_time")}
-    rc = _load().orc_advance_ids(wl.num_instances, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running,
-                                 wl.cap_waiting, _p(st["n_run"]), _p(st["run_ctx"]), _p(st["run_pre"]),
-                                 _p(st["run_dec"]), _p(st["n_wait"]), _p(st["wait_pre"]), _p(st["wait_dec"]),
-                                 _p(clk), int(a.shape[0]), _p(a), _p(p), _p(d), wl.first_token_mode, float(t_now),
-                                 int(max_batches), _p(None if tr is None else tr["run_id"]),
-                                 _p(None if tr is None else tr["wait_id"]), int(id_base),
-                                 _p(None if tr is None else tr["first_token_time"]))
+    head = (wl.num_instances, _p(moi), _p(coef), _p(B), _p(S), wl.cap_running, wl.cap_waiting, _p(st["n_run"]),
+            _p(st["run_ctx"]), _p(st["run_pre"]), _p(st["run_dec"]), _p(st["n_wait"]), _p(st["wait_pre"]),
+            _p(st["wait_dec"]), _p(clk), int(a.shape[0]), _p(a), _p(p), _p(d), wl.first_token_mode,
+            float(t_now), int(max_batches))
+    ids = (_p(None if tr is None else tr["run_id"]), _p(None if tr is None else tr["wait_id"]), int(id_base),
+           _p(None if tr is None else tr["first_token_time"]))
+    if kv is None:
+        rc = _load().orc_advance_ids(*head, *ids)
+    else:
+        I = wl.num_instances
+        bs = _c(np.broadcast_to(np.asarray(kv[0], np.int32), (I,)), np.int32)
+        nb = _c(np.broadcast_to(np.asarray(kv[1], np.int64), (I,)), np.int64)
+        mc = _c(np.broadcast_to(np.asarray(kv[2], np.int64), (I,)), np.int64)
+        rc = _load().orc_advance_kv(*head, _p(bs), _p(nb), _p(mc), *ids)
     if rc != 0:
         raise RuntimeError(f"oracle advance failed with code {rc}")
     if tr is None:

@@ -785,3 +785,179 @@ int orc_kv_residents(const orc_instance *inst, int32_t B, int32_t S, int32_t mod
     if (L < 1 || !res_F) return ORC_EINVAL;
     return kv_sim(inst, B, S, mode, kv, 0, 1, 1, L, NULL, NULL, NULL, res_F, NULL);
 }
+
+
+/* Online stream step under KV-cache limits: orc_advance with the KV step rule of kv_sim
+ * above (App. F names KV-cache allocation, context limits and preemption among what
+ * the serving simulation models; the same reading).  Each executed batch: the running
+ * list in order, each request's new blocks found, preempting the last running request
+ * (possibly itself) while they are not free; then FCFS admission while budget, a slot
+ * and the first chunk's blocks allow; a request whose context reaches max_ctx ends and
+ * frees its blocks.  The batch takes the Eq. 9 time of its own composition (canonical
+ * fp32, accumulated into the fp64 clock) and runs only if it ends by t_now.  Limits per
+ * instance: block_size[I], num_blocks[I], max_ctx[I].  First-token tracking as in
+ * orc_advance_ids (run_id, wait_id, first_token_time may be NULL).  Returns ORC_EINVAL
+ * when a routed query could never run (its prompt reaches max_ctx, or its whole
+ * context capped at max_ctx needs more blocks than the instance has), ORC_ELIMIT when
+ * a queue outgrows its capacity or an instance needs more than max_batches batches;
+ * an instance that fails keeps its state. */
+int orc_advance_kv(int32_t I, const int32_t *model_of_instance, const float *coef, const int32_t *B,
+                   const int32_t *S, int32_t cap_running, int32_t cap_waiting, int32_t *n_run,
+                   int32_t *run_ctx, int32_t *run_pre, int32_t *run_dec, int32_t *n_wait, int32_t *wait_pre,
+                   int32_t *wait_dec, double *clock, int32_t Q, const int32_t *assign,
+                   const int32_t *prompt_len, const int32_t *dec, int32_t mode, double t_now,
+                   int64_t max_batches, const int32_t *block_size, const int64_t *num_blocks,
+                   const int64_t *max_ctx, int64_t *run_id, int64_t *wait_id, int64_t id_base,
+                   double *first_token_time)
+{
+    const int track = run_id != NULL && wait_id != NULL && first_token_time != NULL;
+    int rc_all = ORC_OK;
+    for (int32_t j = 0; j < I; ++j) {
+        const int64_t bs = block_size[j], nb = num_blocks[j], mc = max_ctx[j];
+        const int64_t total = (int64_t)cap_running + cap_waiting + Q + 1;
+        orc_req *run = (orc_req *)calloc((size_t)total, sizeof(orc_req));
+        orc_req *next = (orc_req *)calloc((size_t)total, sizeof(orc_req));  /* the planned running list */
+        orc_req *wait = (orc_req *)calloc((size_t)(2 * total + 1), sizeof(orc_req)); /* room at the front */
+        int64_t *alloc = (int64_t *)calloc((size_t)total, sizeof(int64_t));
+        int *kind = (int *)calloc((size_t)total, sizeof(int));
+        if (!run || !next || !wait || !alloc || !kind) {
+            free(run); free(next); free(wait); free(alloc); free(kind);
+            return ORC_ENOMEM;
+        }
+        int64_t nr = 0, wh = total, we = total;  /* waiting queue: wait[wh .. we) */
+        int64_t free_blocks = nb;
+        for (int32_t r = 0; r < n_run[j]; ++r) {
+            const int64_t o = (int64_t)j * cap_running + r;
+            run[nr].ctx = run_ctx[o]; run[nr].pre = run_pre[o]; run[nr].dec = run_dec[o]; run[nr].is_query = 0;
+            run[nr].id = track ? run_id[o] : -1;
+            free_blocks -= kv_blocks(run[nr].ctx, bs);
+            ++nr;
+        }
+        for (int32_t w = 0; w < n_wait[j]; ++w) {
+            const int64_t o = (int64_t)j * cap_waiting + w;
+            wait[we].ctx = 0; wait[we].pre = wait_pre[o]; wait[we].dec = wait_dec[o]; wait[we].is_query = 0;
+            wait[we].id = track ? wait_id[o] : -1;
+            ++we;
+        }
+        int rc = ORC_OK;
+        /* 1. the routed queries join the waiting tail in query order */
+        for (int32_t i = 0; i < Q; ++i) {
+            if (assign[i] != j) continue;
+            if ((int64_t)prompt_len[i] >= mc || kv_blocks(min64((int64_t)prompt_len[i] + dec[i], mc), bs) > nb)
+                rc = ORC_EINVAL;
+            wait[we].ctx = 0; wait[we].pre = prompt_len[i]; wait[we].dec = dec[i]; wait[we].is_query = 0;
+            wait[we].id = (track && id_base >= 0) ? id_base + i : -1;
+            ++we;
+        }
+        if (rc == ORC_OK && we - wh > cap_waiting) rc = ORC_ELIMIT;
+        const float *cf = coef + 5 * model_of_instance[j];
+        double t = clock[j];
+        /* 2. execute whole batches that end by t_now */
+        for (int64_t step = 0; rc == ORC_OK; ++step) {
+            if (nr == 0 && wh == we) {                        /* idle: nothing to run */
+                if (t < t_now) t = t_now;
+                break;
+            }
+            if (step >= max_batches) { rc = ORC_ELIMIT; break; }
+            /* plan the batch on a copy of the running list; a preempted request is written
+             * below the waiting head, which moves only if the batch runs */
+            memcpy(next, run, sizeof(orc_req) * (size_t)nr);
+            int64_t pnr = nr, pwh = wh, pfree = free_blocks;
+            int64_t budget = B[j];
+            for (int64_t r = 0; r < nr; ++r) { kind[r] = SCHED_NONE; alloc[r] = 0; }
+            int64_t r = 0;
+            while (r < pnr && budget > 0) {
+                const int64_t x = next[r].pre > 0 ? min64(next[r].pre, budget) : 1;
+                const int64_t need = kv_blocks(next[r].ctx + x, bs) - kv_blocks(next[r].ctx, bs);
+                while (pfree < need && pnr - 1 >= r) {          /* preempt the last running request */
+                    orc_req v = next[pnr - 1];
+                    pfree += kv_blocks(v.ctx, bs);
+                    v.pre += v.ctx;
+                    v.ctx = 0;
+                    wait[--pwh] = v;
+                    --pnr;
+                }
+                if (r >= pnr) break;                             /* r preempted itself */
+                pfree -= need;
+                alloc[r] = x;
+                kind[r] = next[r].pre > 0 ? SCHED_PREFILL : SCHED_DECODE;
+                budget -= x;
+                ++r;
+            }
+            while (budget > 0 && pwh < we && pnr < S[j]) {      /* admission */
+                const int64_t x = min64(wait[pwh].pre, budget);
+                const int64_t need = kv_blocks(x, bs);
+                if (pfree < need) break;
+                pfree -= need;
+                next[pnr] = wait[pwh++];
+                alloc[pnr] = x;
+                kind[pnr] = SCHED_PREFILL;
+                budget -= x;
+                ++pnr;
+            }
+            int64_t F[5] = {1, 0, 0, 0, 0};
+            for (int64_t q = 0; q < pnr; ++q) {
+                if (kind[q] == SCHED_PREFILL) {
+                    const int64_t x = alloc[q];
+                    F[1] += x;
+                    F[4] += x * next[q].ctx + x * (x + 1) / 2;
+                } else if (kind[q] == SCHED_DECODE) {
+                    F[2] += 1;
+                    F[3] += next[q].ctx;
+                }
+            }
+            const float T = orc_ttft_f32(cf, F);   /* Eq. 9 for this one batch */
+            if (t + (double)T > t_now) break;       /* still running at t_now */
+            if (pnr > cap_running) { rc = ORC_ELIMIT; break; }
+            /* apply the batch */
+            for (int64_t q = 0; q < pnr; ++q) {
+                if (kind[q] == SCHED_PREFILL) {
+                    next[q].ctx += alloc[q];
+                    next[q].pre -= alloc[q];
+                    if (next[q].pre == 0 && mode == ORC_FIRST_TOKEN_WITH_LAST_CHUNK) {
+                        next[q].dec -= 1;
+                        if (track) first_token(&next[q], 1, t + (double)T, first_token_time);
+                    }
+                } else if (kind[q] == SCHED_DECODE) {
+                    next[q].ctx += 1;
+                    next[q].dec -= 1;
+                    if (track) first_token(&next[q], mode == ORC_FIRST_TOKEN_SEPARATE_DECODE, t + (double)T,
+                                           first_token_time);
+                }
+                if (next[q].pre == 0 && next[q].ctx >= mc) next[q].dec = 0;  /* context limit */
+            }
+            int64_t keep = 0;
+            for (int64_t q = 0; q < pnr; ++q) {
+                if (next[q].dec > 0) run[keep++] = next[q];
+                else pfree += kv_blocks(next[q].ctx, bs);      /* finished: its blocks return */
+            }
+            nr = keep;
+            wh = pwh;
+            free_blocks = pfree;
+            t += (double)T;
+            if (we - wh > cap_waiting) { rc = ORC_ELIMIT; break; }
+        }
+        if (rc == ORC_OK) {
+            n_run[j] = (int32_t)nr;
+            for (int64_t q = 0; q < cap_running; ++q) {
+                const int64_t o = (int64_t)j * cap_running + q;
+                run_ctx[o] = q < nr ? (int32_t)run[q].ctx : 0;
+                run_pre[o] = q < nr ? (int32_t)run[q].pre : 0;
+                run_dec[o] = q < nr ? (int32_t)run[q].dec : 0;
+                if (track) run_id[o] = q < nr ? run[q].id : -1;
+            }
+            n_wait[j] = (int32_t)(we - wh);
+            for (int64_t w = 0; w < cap_waiting; ++w) {
+                const int64_t o = (int64_t)j * cap_waiting + w;
+                wait_pre[o] = w < we - wh ? (int32_t)wait[wh + w].pre : 0;
+                wait_dec[o] = w < we - wh ? (int32_t)wait[wh + w].dec : 0;
+                if (track) wait_id[o] = w < we - wh ? wait[wh + w].id : -1;
+            }
+            clock[j] = t;
+        } else {
+            rc_all = rc;
+        }
+        free(run); free(next); free(wait); free(alloc); free(kind);
+    }
+    return rc_all;
+}

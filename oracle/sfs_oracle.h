@@ -146,6 +146,21 @@ int orc_advance_ids(int32_t I, const int32_t *model_of_instance, const float *co
                     int64_t max_batches, int64_t *run_id, int64_t *wait_id, int64_t id_base,
                     double *first_token_time);
 
+/* orc_advance_ids under per-instance KV-cache limits (block_size, num_blocks, max_ctx
+ * [I]): each executed batch follows the KV step rule of orc_sfs_candidate_kv (blocks
+ * found in running order with preemption of the last running request, admission only
+ * with the first chunk's blocks, the context limit ending a request).  ORC_EINVAL for a
+ * routed query that could never run (prompt at max_ctx, or its capped whole context
+ * needing more blocks than the instance has). */
+int orc_advance_kv(int32_t I, const int32_t *model_of_instance, const float *coef, const int32_t *B,
+                   const int32_t *S, int32_t cap_running, int32_t cap_waiting, int32_t *n_run,
+                   int32_t *run_ctx, int32_t *run_pre, int32_t *run_dec, int32_t *n_wait, int32_t *wait_pre,
+                   int32_t *wait_dec, double *clock, int32_t Q, const int32_t *assign,
+                   const int32_t *prompt_len, const int32_t *dec, int32_t mode, double t_now,
+                   int64_t max_batches, const int32_t *block_size, const int64_t *num_blocks,
+                   const int64_t *max_ctx, int64_t *run_id, int64_t *wait_id, int64_t id_base,
+                   double *first_token_time);
+
 /* Utility of Eq. 2 with the cost of App. B.4 in canonical fp32. */
 float orc_utility(float acc, float lambda, int32_t p, int32_t dec_hat, float price_in, float price_out);
 

@@ -300,13 +300,15 @@ def batch_log(num_batches: int, num_models: int, seed: int, coef: np.ndarray, no
 
 
 def kv_limits(wl: Workload, seed: int, block_sizes=(16,), tightness=(0.3, 1.0), ctx_limited: float = 0.5,
-              ctx_slack=(1, 64), unlimited: int = 1 << 40):
+              ctx_slack=(1, 64), unlimited: int = 1 << 40, max_new: int = 1):
     """Seeded per-instance KV-cache limits for a workload's snapshot: block sizes drawn
     from `block_sizes`; a context limit on a `ctx_limited` share of the instances, just
     above the longest context any request or query already needs (so that decoding runs
     into it), else `unlimited`; and a block count that a `tightness` draw places between
-    the most any single request (or the first token of the longest query) can need and
-    the residents' whole demand, never below the blocks the running requests hold.
+    the most any single request (or the longest query with `max_new` output tokens: 1
+    for an estimate up to the first token, the longest response for a stream that runs
+    queries to their end) can need and the residents' whole demand, never below the
+    blocks the running requests hold.
     Returns (block_size [I] int32, num_blocks [I] int64, max_ctx [I] int64).  Token
     counts are turned into blocks by the bound tokens // bs + 1 >= ceil(tokens / bs)."""
     rng = np.random.default_rng(seed)
@@ -328,7 +330,7 @@ def kv_limits(wl: Workload, seed: int, block_sizes=(16,), tightness=(0.3, 1.0), 
         else:
             mctx[j] = unlimited
         whole = np.concatenate([np.minimum(ctx + pre + dec, mctx[j]), np.minimum(wpre + wdec, mctx[j]),
-                                [min(wl.max_prompt_len + 1, int(mctx[j]))]])
+                                [min(wl.max_prompt_len + max_new, int(mctx[j]))]])
         one = int((whole // b + 1).max())
         held = int((ctx // b + 1).sum())
         demand = int((whole // b + 1).sum())
