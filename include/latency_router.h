@@ -254,7 +254,7 @@ LR_API int lr_set_ttft_source(lr_ctx *ctx, int32_t source);
  * With limits on, lr_route and lr_route_frontier_static first write the KV-limited
  * estimate matrix (to ttft_matrix_out if given, else to library memory) and score
  * and pick over it; lr_route_baseline reports the chosen instance's KV-limited time;
- * the average-case sources and lr_advance return LR_EINVAL.  Each estimate call
+ * lr_advance executes the same rule; the average-case sources return LR_EINVAL.  Each estimate call
  * runs one walk per distinct prompt length (the queries are counting-sorted by
  * length in library memory sized by max_queries).  Memory taken here: per buffer
  * 68 B x I x horizon of records, and max_queries x (8 B + 4 B x I) for the sort
@@ -297,7 +297,16 @@ LR_API int lr_calibrate(lr_ctx *ctx, int64_t N, const int64_t *features, const i
  * or num_models (the column of the chosen instance's model is used, e.g. the dec_hat
  * matrix given to lr_route).  Requires cap_running >= every max_seqs (LR_ECAPACITY
  * otherwise).  A waiting queue that would exceed cap_waiting records LR_ECAPACITY, an
- * out-of-range length LR_EINVAL; either leaves the previous snapshot live. */
+ * out-of-range length LR_EINVAL; either leaves the previous snapshot live.
+ * With KV-cache limits on (lr_set_kv_limits) every executed batch follows the KV step
+ * rule described there (blocks found in running order with preemption of the last running
+ * request, admission only with the first chunk's blocks, the context limit ending a
+ * request), and the advanced snapshot is summarized and published as a loaded one under
+ * those limits.  There a query whose prompt is not below max_ctx, or whose whole context
+ * (capped at max_ctx) needs more blocks than the instance has, records LR_EINVAL; a
+ * waiting queue that preemptions grow past cap_waiting records LR_ECAPACITY; either keeps
+ * the previous snapshot live.  The KV step needs 4 x (11 cap_running + 3 cap_waiting + 32)
+ * bytes of shared memory per instance, at most 200 KB for 4 (LR_ECAPACITY otherwise). */
 LR_API int lr_advance(lr_ctx *ctx, int32_t Q, const int32_t *assign, const int32_t *prompt_len,
                       const int32_t *dec, int32_t dec_cols, double t_now, void *cuda_stream);
 

@@ -50,6 +50,7 @@ struct lr_ctx {
     lr::KvLimits kv{};
     int kv_warps = 0;
     size_t kv_smem = 0;
+    size_t k3_kv_smem = 0;  // the KV stream step's shared memory (all warps of a CTA)
     int32_t *kv_order = nullptr;  // [max_queries] the estimate's query order
     int32_t *kv_leaders = nullptr, *kv_sort = nullptr;  // [max_queries]; [4][kKvBuckets] + 4 + [ceil(I/8)]
     float *kv_mat = nullptr;  // [max_queries][I] the KV estimate matrix a route scores
@@ -430,7 +431,10 @@ int lr_load_state(lr_ctx *c, const lr_state_view *v, void *stream) {
         k.ctl = c->ctl;
         k.in = lr::StateIn{v->n_run, v->run_ctx, v->run_pre, v->run_dec, v->n_wait, v->wait_pre, v->wait_dec, nullptr};
         const int grid = (c->cfg.I + c->kv_warps - 1) / c->kv_warps;
-        cudaError_t e = lr::launch_kv_load(k, grid, c->kv_warps, c->kv_smem, (cudaStream_t)stream);
+        // a loaded snapshot's requests are untracked (only the stream step assigns ids)
+        cudaError_t e = c->ftt ? reset_ids(c, stream) : cudaSuccess;
+        if (e != cudaSuccess) return cuda_fail(c, e, "tracking reset");
+        e = lr::launch_kv_load(k, grid, c->kv_warps, c->kv_smem, (cudaStream_t)stream);
         if (e != cudaSuccess) return cuda_fail(c, e, "KV load launch");
         c->load_stream = stream;
         c->loaded_any = true;
@@ -774,6 +778,14 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
     }
     c->kv_warps = warps;
     c->kv_smem = warps * per_warp;
+    c->k3_kv_smem = lr::kK3Warps * lr::advance_kv_smem_per_warp(c->cfg);
+    if (c->k3_kv_smem <= 200 * 1024) {
+        e = lr::set_k3_kv_smem(c->k3_kv_smem);
+        if (e != cudaSuccess) {
+            free_kv(c);
+            return cuda_fail(c, e, "KV advance shared memory");
+        }
+    }
     c->kv_on = true;
     return LR_OK;
 }
@@ -825,9 +837,9 @@ int lr_advance_tracked(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_
     if (Q > 0 && (!assign || !prompt_len || !dec)) return fail(c, LR_EINVAL, "null array");
     if (dec_cols != 1 && dec_cols != c->cfg.M) return fail(c, LR_EINVAL, "dec_cols must be 1 or num_models");
     if (!std::isfinite(t_now)) return fail(c, LR_EINVAL, "t_now must be finite");
-    if (c->kv_on) return fail(c, LR_EINVAL, "advancing with KV-cache limits is not supported");
     if (c->cfg.capR < c->max_seqs) return fail(c, LR_ECAPACITY, "advancing needs cap_running >= every max_seqs");
-    if (c->k3_smem > 200 * 1024) return fail(c, LR_ECAPACITY, "queue capacities too large for one advance warp");
+    if ((c->kv_on ? c->k3_kv_smem : c->k3_smem) > 200 * 1024)
+        return fail(c, LR_ECAPACITY, "queue capacities too large for one advance warp");
     lr::K3Launch k;
     std::memset(&k, 0, sizeof(k));
     k.cfg = c->cfg;
@@ -845,7 +857,28 @@ int lr_advance_tracked(lr_ctx *c, int32_t Q, const int32_t *assign, const int32_
     k.id_base = id_base;
     k.ftt = c->ftt;
     cudaStream_t st = (cudaStream_t)stream;
-    cudaError_t e = lr::launch_advance(k, (c->cfg.I + lr::kK3Warps - 1) / lr::kK3Warps, c->k3_smem, st);
+    const int k3_grid = (c->cfg.I + lr::kK3Warps - 1) / lr::kK3Warps;
+    if (c->kv_on) {
+        // the KV step rule, then the KV load summarizes and publishes the snapshot
+        k.kv = c->kv;
+        cudaError_t e = lr::launch_advance_kv(k, k3_grid, c->k3_kv_smem, st);
+        if (e != cudaSuccess) return cuda_fail(c, e, "KV advance launch");
+        lr::KvLoad kl;
+        std::memset(&kl, 0, sizeof(kl));
+        kl.cfg = c->cfg;
+        kl.kv = c->kv;
+        kl.buf0 = c->buf[0];
+        kl.buf1 = c->buf[1];
+        kl.ctl = c->ctl;
+        const lr::StateBuf &sc = c->scratch;
+        kl.in = lr::StateIn{sc.n_run, sc.run_ctx, sc.run_pre, sc.run_dec, sc.n_wait, sc.wait_pre, sc.wait_dec, sc.clock};
+        e = lr::launch_kv_load(kl, (c->cfg.I + c->kv_warps - 1) / c->kv_warps, c->kv_warps, c->kv_smem, st);
+        if (e != cudaSuccess) return cuda_fail(c, e, "KV load launch");
+        c->load_stream = stream;
+        c->loaded_any = true;
+        return LR_OK;
+    }
+    cudaError_t e = lr::launch_advance(k, k3_grid, c->k3_smem, st);
     if (e != cudaSuccess) return cuda_fail(c, e, "advance launch");
     // summarize and publish the advanced snapshot exactly as a loaded one
     lr::K1Launch a;

@@ -353,6 +353,7 @@ struct K3Launch {
     int32_t track;
     long long id_base;
     double *ftt;
+    KvLimits kv;  // the KV stream step (launch_advance_kv) only
 };
 constexpr int kK3Warps = 4;
 // Shared memory of one K3 warp: the running list twice (ctx, pre, dec, id; the
@@ -361,7 +362,14 @@ constexpr int kK3Warps = 4;
 __host__ __device__ inline size_t advance_smem_per_warp(const DevConfig &c) {
     return sizeof(int32_t) * ((size_t)8 * c.capR + (size_t)3 * c.capW + 32);
 }
+// The KV stream step's waiting queue is a ring of capW + capR entries: preempted
+// requests return to its front.
+__host__ __device__ inline size_t advance_kv_smem_per_warp(const DevConfig &c) {
+    return sizeof(int32_t) * ((size_t)8 * c.capR + (size_t)3 * ((size_t)c.capW + c.capR) + 32);
+}
 cudaError_t launch_advance(const K3Launch &a, int grid, size_t smem, cudaStream_t st);
+cudaError_t launch_advance_kv(const K3Launch &a, int grid, size_t smem, cudaStream_t st);
+cudaError_t set_k3_kv_smem(size_t bytes);
 cudaError_t set_k3_smem(size_t bytes);
 struct StateOut {
     int32_t *n_run, *run_ctx, *run_pre, *run_dec, *n_wait, *wait_pre, *wait_dec;

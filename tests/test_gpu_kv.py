@@ -252,9 +252,6 @@ def test_calls_closed_with_limits_and_turning_them_off():
     with pytest.raises(R().LRError) as e:
         rt.set_ttft_source(R().LR_TTFT_THROUGHPUT)
     assert e.value.code == R().LR_EINVAL
-    with pytest.raises(R().LRError) as e:
-        rt.advance(torch.zeros(16, dtype=torch.int32, device="cuda"), p, dh, 0.0)
-    assert e.value.code == R().LR_EINVAL
     # the baselines: their choices, with the chosen instance's KV-limited time
     _, _, _, et, _ = oracle.estimate_matrix_kv(wl, *limits)
     for pol in (R().LR_POLICY_ROUND_ROBIN, R().LR_POLICY_SHORTEST_QUEUE, R().LR_POLICY_LATENCY_AGNOSTIC):
