@@ -477,8 +477,8 @@ def run_calibration(args, dev, flush):
     ach = nbytes / (ms_avg * 1e-3) / 1e9
     return {"log": f"{N} batches of {M} models, grouped by model, 4% noise", "ms": ms_avg,
             "value": N / (ms_avg * 1e-3), "unit": "batches/s", "max_rel_error_vs_generating_coef": rel,
-            "gpu_launches": 2 * K,
-            "roofline": {"kernel": "k_calib_accum", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+            "gpu_launches": K,
+            "roofline": {"kernel": "k_calibrate (one pass over the log, then the last CTA's solve)", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                          "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
                          "algorithmic_bytes": nbytes}}
 

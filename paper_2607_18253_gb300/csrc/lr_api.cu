@@ -41,7 +41,7 @@ struct lr_ctx {
     // average-case TTFT sources
     lr::QueueRaw *qraw = nullptr;
     lr::QueueDev *qd = nullptr;
-    unsigned long long *cal_acc = nullptr;  // calibration sums [M][kCalAcc][2] (128-bit)
+    unsigned long long *cal_acc = nullptr;  // calibration sums [M][kCalAcc][2] (128-bit) and counter
     int source = lr::kSrcSfs;
     bool have_qp = false, have_lps = false;
     // KV-cache limits (lr_set_kv_limits): per-instance arrays, the records of both
@@ -358,7 +358,7 @@ int lr_create(const lr_config *cfg, lr_ctx **out) {
     LR_ALLOC(c->ontime_part, 2 * (size_t)lr::kOnTimeParts);
     LR_ALLOC(c->qraw, I);
     LR_ALLOC(c->qd, I);
-    LR_ALLOC(c->cal_acc, (size_t)M * lr::kCalAcc * 2);
+    LR_ALLOC(c->cal_acc, lr::cal_acc_words(M));
 #undef LR_ALLOC
     e = cudaMemcpy(moi, cfg->model_of_instance, I * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(B, cfg->max_batched_tokens, I * 4, cudaMemcpyHostToDevice);

@@ -191,12 +191,18 @@ constexpr int kCalAcc = 21;        // per model: 15 sums of the upper triangle o
 constexpr int kCalMaxModels = 128;  // shared-memory sums of one CTA (128-bit each)
 constexpr double kCalTimeScale = 17592186044416.0;  // 2^44: times in 2^-44 s fixed point
 constexpr double kCalTimeMax = 524288.0;            // 2^19 s
-constexpr int kCalTile = 512;                       // rows per staged tile
-constexpr int kCalStages = 4;                       // tiles in flight per CTA
+constexpr int kCalThreads = 512;                    // one CTA per SM
+constexpr int kCalConsumerWarps = kCalThreads / 32 - 1;  // the last warp issues the copies
+constexpr int kCalTile = 2 * 32 * kCalConsumerWarps;     // rows per staged tile, two a consumer lane (16-byte copies)
+constexpr int kCalStagesMax = 3;                    // tiles in flight per CTA
+constexpr int kCalFlushRows = 128;                  // rows a lane sums in 64 bits between flushes
+constexpr size_t kCalSmemMax = 227 * 1024;
 constexpr size_t kCalStageBytes = (size_t)kCalTile * (kCalCols * 8 + 8 + 4);
-// copies of the shared 128-bit sums: one per warp of the 256-thread CTA up to 16 models
-__host__ __device__ inline int cal_copies(int M) { return M <= 16 ? 8 : 1; }
-__host__ __device__ inline size_t cal_sums_bytes(int M) { return (size_t)cal_copies(M) * M * kCalAcc * 16; }
+// the CTA's shared 128-bit sums [M][kCalAcc]
+__host__ __device__ inline size_t cal_sums_bytes(int M) { return (size_t)M * kCalAcc * 16; }
+// the calibration's device words: the sums [M][kCalAcc][2] and the CTA counter of the
+// last-CTA solve (zero between calls)
+__host__ __device__ inline size_t cal_acc_words(int M) { return (size_t)M * kCalAcc * 2 + 2; }
 cudaError_t launch_calibrate(long long N, const long long *F, const int32_t *model, const double *time, int M,
                              int shared_beta1, unsigned long long *acc, double *coef, DevCtl *ctl, int grid,
                              cudaStream_t st);
