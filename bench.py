@@ -41,7 +41,8 @@ WORKLOAD = "pool256"
 # DRAM bytes (read + write) per launch of the step's kernels on this workload, from one
 # ncu capture of the kernels as they are built now (summaries under profiles/); they
 # are retaken whenever one of the kernels changes.
-NCU_TRAFFIC = {"k_route": 4_577_792 + 8_019_712, "k_trajectory": 1_393_408, "k_estimate": 357_888 + 7_386_624}
+NCU_TRAFFIC = {"k_route": 4_577_792 + 8_019_712, "k_trajectory": 1_399_040, "k_estimate": 357_888 + 7_386_624,
+               "k_calibrate": 208_430_848 + 3_465_728}
 
 
 def _peaks():
@@ -480,7 +481,7 @@ def run_calibration(args, dev, flush):
             "gpu_launches": K,
             "roofline": {"kernel": "k_calibrate (one pass over the log, then the last CTA's solve)", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                          "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
-                         "algorithmic_bytes": nbytes}}
+                         "algorithmic_bytes": nbytes, "traffic": NCU_TRAFFIC["k_calibrate"]}}
 
 
 def run_estimate(args, dev, wl, flush):
@@ -884,11 +885,58 @@ def run_stream(args, dev):
                    "mean_us": float(np.mean(lat) * 1e3), "wall_s": wall, "simulated_s": float(arr[nb * m - 1]),
                    "final_mean_waiting": float(fin["n_wait"].float().mean().item())}
             out["sizes" if label == "poisson" else label][str(m)] = res
+    # A Poisson stream under KV-cache limits (App. F; the stream step executes the KV
+    # rule and the KV load summarizes each snapshot): STREAM_KV_QUERIES arrivals at 0.5 x
+    # the plain pool's capacity (the limits lower it), micro-batches of 16.  Limits:
+    # 16-token blocks, each instance's block count between its largest request (a
+    # query's whole response included) and its residents' demand, a context limit on
+    # half the instances.
+    limits = W.kv_limits(wl, KV_SEED, block_sizes=(KV_BLOCK,), max_new=int(wl.dec_hat.max()))
+    rt.set_kv_limits(*limits, horizon=KV_HORIZON)
+    rt.load_state(*state)
+    arr = W.poisson_arrivals(STREAM_KV_QUERIES, 0.5 * float(cap.sum()), STREAM_SEED)
+    m = 16
+    nb = STREAM_KV_QUERIES // m
+    lat = []
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(nb)]
+    torch.cuda.synchronize()
+    w0 = time.perf_counter()
+    for b in range(nb):
+        lo = b * m
+        cur, prev = ap[b & 1], ap[(b - 1) & 1]
+        ev[b][0].record()
+        pm = m if b > 0 else 0
+        plo = (b - 1) * m
+        rc = lib.lr_advance(h, pm, V(prev), V(pp + 4 * max(plo, 0)), V(dhp + 4 * M * max(plo, 0)), M,
+                            ctypes.c_double(float(arr[lo + m - 1])), sp)
+        rc |= lib.lr_route(h, m, V(pp + 4 * lo), V(dhp + 4 * M * lo), V(accp + 4 * M * lo), None, 1, lamp,
+                           mup, V(cur), V(util.data_ptr()), None, None, None, sp)
+        ev[b][1].record()
+        if rc:
+            raise RuntimeError(f"KV stream call failed: {lib.lr_last_error(h).decode()}")
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - w0
+    st = rt.status()
+    if st != R.LR_OK:
+        raise RuntimeError(f"KV stream run ended with device status {st}")
+    lat = [e0.elapsed_time(e1) for e0, e1 in ev]
+    q = np.percentile(np.asarray(lat) * 1e3, [50, 99])
+    fin = rt.read_state(device=dev)
+    # launches per decision: advance (K3 KV, KV load) + route (count, scan, scatter, walk,
+    # expand, route)
+    launches += 8 * nb
+    out["kv_poisson_16"] = {"arrival_qps": 0.5 * float(cap.sum()), "batches": nb, "queries": nb * m, "p50_us": float(q[0]), "p99_us": float(q[1]),
+                            "mean_us": float(np.mean(lat) * 1e3), "wall_s": wall,
+                            "simulated_s": float(arr[nb * m - 1]),
+                            "final_mean_waiting": float(fin["n_wait"].float().mean().item()),
+                            "limits": {"block_size": KV_BLOCK, "seed": KV_SEED, "horizon": KV_HORIZON,
+                                       "ctx_limited_instances": int((limits[2] < (1 << 40)).sum())}}
     out["gpu_launches"] = launches
     rt.close()
     return out
 
 
+STREAM_KV_QUERIES = 32_768
 POLICY_WORKLOAD = "paper3"
 POLICY_LOADS = (0.2, 0.4, 0.6, 0.8)
 POLICY_QUERIES = 4096
