@@ -100,14 +100,6 @@ __device__ __forceinline__ double u128_to_double(const U128 &v, int e2) {
     return __longlong_as_double((long long)(((unsigned long long)(e + e2 + 1023) << 52) | (q & ((1ull << 52) - 1))));
 }
 
-// 1/x for x in [2^-120, 2^120]: one Newton-Raphson step r <- r (2 - x r) from the fp32
-// reciprocal squares its relative error, 2^-24 -> 2^-48 (the pivots need no more: the
-// solve's error is set by the conditioning, far above 2^-48).
-__device__ __forceinline__ double recip(double x) {
-    const double r = (double)__frcp_rn((float)x);
-    return __fma_rn(r, __fma_rn(-x, r, 1.0), r);
-}
-
 // The solve of every model's system, on the last CTA: regressors, power-of-two Jacobi
 // scaling, LDL^T, unscaling.  D regressors: 4 (the paper's form, F1 + F2 as one token
 // count) or 5; with four, a unit fifth regressor uncoupled from the others keeps one
@@ -152,7 +144,7 @@ __device__ __forceinline__ int half_lead(const U128 &g) {
 }
 
 // entry e of model m: e < 15 the packed lower triangle of A (row p, column q <= p), else b
-__device__ __noinline__ void calib_entry(int m, int e, bool four, const unsigned long long *S, double *W) {
+__device__ void calib_entry(int m, int e, bool four, const unsigned long long *S, double *W) {
     const unsigned long long *Sm = S + (size_t)m * kCalAcc * 2;
     double *Wm = W + (size_t)m * kCalSolveWords;
     int p = e - 15, q = -1;
@@ -166,12 +158,37 @@ __device__ __noinline__ void calib_entry(int m, int e, bool four, const unsigned
 }
 
 // the scale exponent h_p of regressor p of model m (before the entries)
-__device__ __noinline__ void calib_scale(int m, int p, bool four, const unsigned long long *S, double *W) {
+__device__ void calib_scale(int m, int p, bool four, const unsigned long long *S, double *W) {
     reinterpret_cast<int *>(W + (size_t)m * kCalSolveWords + 20)[p] =
         half_lead(calib_gsum(S + (size_t)m * kCalAcc * 2, four, p, p));
 }
 
-__device__ __noinline__ void calib_factor(int m, int D, const unsigned long long *S, const double *W, double *coef) {
+// On this part the SM's fp64 unit is narrow: each fp64 instruction of a warp costs
+// tens of cycles whatever the active lanes, so the solve keeps its fp64 instructions
+// few and does comparisons, clamps and power-of-two scalings on the bits.
+
+// 1/x for a positive normal double: the fp32 reciprocal of its significand truncated to
+// 24 bits (built from the bits, relative error below 2^-23), rescaled by the exponent,
+// then one Newton-Raphson step r <- r (2 - x r), which squares the error (2^-46).
+__device__ __forceinline__ double recip_pos(double x) {
+    const unsigned long long bx = (unsigned long long)__double_as_longlong(x);
+    const long long e = (long long)((bx >> 52) & 0x7ff) - 1023;
+    const float m = __int_as_float((int)((127u << 23) | (unsigned)((bx >> 29) & 0x7fffffu)));  // [1, 2)
+    const unsigned rb = (unsigned)__float_as_int(__frcp_rn(m));                                  // (1/2, 1]
+    const long long re = (long long)((rb >> 23) & 0xff) - 127 - e;
+    const double r = __longlong_as_double((long long)(((unsigned long long)(re + 1023) << 52) |
+                                                      ((unsigned long long)(rb & 0x7fffffu) << 29)));
+    return __fma_rn(r, __fma_rn(-x, r, 1.0), r);
+}
+
+// v * 2^-h for a finite v (0 stays 0; the results here stay normal): the exponent field
+__device__ __forceinline__ double scale_pow2(double v, int h) {
+    const long long bv = __double_as_longlong(v);
+    return (bv & 0x7ff0000000000000LL) ? __longlong_as_double(bv - ((long long)h << 52)) : v;
+}
+
+// The scaled 5x5 system of model m by LDL^T, with straight-line code in registers.
+__device__ void calib_factor(int m, int D, const unsigned long long *S, const double *W, double *coef) {
     const double *Wm = W + (size_t)m * kCalSolveWords;
     const int *h = reinterpret_cast<const int *>(Wm + 20);
     const unsigned long long *cnt = S + ((size_t)m * kCalAcc + 20) * 2;
@@ -183,6 +200,7 @@ __device__ __noinline__ void calib_factor(int m, int D, const unsigned long long
 #pragma unroll
         for (int q = 0; q <= p; ++q) A[p][q] = Wm[p * (p + 1) / 2 + q];
     }
+    constexpr long long kMinPivot = 0x3d3c25c268497682LL;  // the bits of 1e-13
 #pragma unroll
     for (int p = 0; p < 5; ++p) {
 #pragma unroll
@@ -196,8 +214,11 @@ __device__ __noinline__ void calib_factor(int m, int D, const unsigned long long
         double v = A[p][p];
 #pragma unroll
         for (int k = 0; k < p; ++k) v = __fma_rn(-LD[p][k], L[p][k], v);
-        ok = ok && v > 1e-13;  // rank-deficient design (or a zero G_pp)
-        inv[p] = recip(fmin(fmax(v, 1e-13), 1e30));
+        // v > 1e-13 on the bits (a positive double orders as its bits; NaN fails)
+        const long long bv = __double_as_longlong(v);
+        const bool piv = bv > kMinPivot && bv < 0x7ff0000000000000LL;
+        ok = ok && piv;  // rank-deficient design (or a zero G_pp)
+        inv[p] = piv ? recip_pos(v) : 0.0;
     }
 #pragma unroll
     for (int p = 0; p < 5; ++p) {
@@ -213,17 +234,16 @@ __device__ __noinline__ void calib_factor(int m, int D, const unsigned long long
         for (int k = p + 1; k < 5; ++k) v = __fma_rn(-L[k][p], w[k], v);
         w[p] = v;
     }
-#pragma unroll
-    for (int p = 0; p < 5; ++p) w[p] *= __longlong_as_double((long long)(1023 - h[p]) << 52);  // unscaled: 2^-h_p
-    // the five coefficients: with four regressors the token slope serves prefill and decode
+    // the five coefficients, unscaled by 2^-h_p: with four regressors the token slope
+    // serves prefill and decode
     const double nan = __longlong_as_double(0x7ff8000000000000LL);
     const bool four = D == 4;
     double out[5];
-    out[0] = w[0];
-    out[1] = w[1];
-    out[2] = four ? w[1] : w[2];
-    out[3] = four ? w[2] : w[3];
-    out[4] = four ? w[3] : w[4];
+    out[0] = scale_pow2(w[0], h[0]);
+    out[1] = scale_pow2(w[1], h[1]);
+    out[2] = four ? out[1] : scale_pow2(w[2], h[2]);
+    out[3] = four ? scale_pow2(w[2], h[2]) : scale_pow2(w[3], h[3]);
+    out[4] = four ? scale_pow2(w[3], h[3]) : scale_pow2(w[4], h[4]);
 #pragma unroll
     for (int k = 0; k < 5; ++k) coef[(size_t)m * 5 + k] = ok ? out[k] : nan;
 }
@@ -253,12 +273,16 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(long long N, const
                                                               unsigned long long *acc, double *coef, DevCtl *ctl) {
     extern __shared__ __align__(16) unsigned char cal_smem[];
     unsigned long long *sacc = reinterpret_cast<unsigned long long *>(cal_smem);  // [M][kCalAcc][2] (lo, hi)
+    // the flushes' totals in carry-save form: [M][26][2], sum k = w0 + 2^32 w1, each flush
+    // adding the low and the high 32 bits of its (below 2^64) total with a reduction that
+    // returns nothing (no carry to wait for)
+    unsigned long long *scs = sacc + (size_t)M * kCalAcc * 2;
     const int lane = threadIdx.x & 31;
     unsigned char *stages = cal_smem + cal_sums_bytes(M);
     __shared__ __align__(8) unsigned long long s_mbar[kCalStagesMax];
     __shared__ int s_last;
     unsigned int *done = reinterpret_cast<unsigned int *>(acc + 2 * (size_t)M * kCalAcc);
-    for (int i = threadIdx.x; i < M * kCalAcc * 2; i += blockDim.x) sacc[i] = 0ull;
+    for (int i = threadIdx.x; i < M * (kCalAcc + kCalFlushSums) * 2; i += blockDim.x) sacc[i] = 0ull;
     unsigned long long g[15], bl[5], bh[5];  // 64-bit sums since the last flush
     int nfast = 0, cur = -1;
     bool bad = false;
@@ -294,10 +318,10 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(long long N, const
                     a[j] = (up ? a[j + w] : a[j]) + __shfl_xor_sync(kFull, give, w);
                 }
             }
-            if (lane < 26) {  // a[0]: the warp's total of sum `lane`
-                const int slot = lane < 20 ? lane : (lane < 25 ? lane - 5 : 20);
-                const int sh = (lane >= 20 && lane < 25) ? 26 : 0;
-                atomic_add128(sacc + ((size_t)mk * kCalAcc + slot) * 2, a[0] << sh, sh ? a[0] >> (64 - sh) : 0ull);
+            if (lane < kCalFlushSums) {  // a[0]: the warp's total of sum `lane`
+                const uint32_t sa = (uint32_t)__cvta_generic_to_shared(scs + ((size_t)mk * kCalFlushSums + lane) * 2);
+                asm volatile("red.shared.add.u64 [%0], %1;" ::"r"(sa), "l"(a[0] & 0xffffffffull) : "memory");
+                asm volatile("red.shared.add.u64 [%0], %1;" ::"r"(sa + 8u), "l"(a[0] >> 32) : "memory");
             }
             pend &= ~__ballot_sync(kFull, mine);
         }
@@ -391,19 +415,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(long long N, const
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    __shared__ double s_warm[kCalSolveWords + 8];
-    __shared__ unsigned long long s_zero[kCalAcc * 2];
-    if (threadIdx.x < kCalAcc * 2) s_zero[threadIdx.x] = 0ull;
     __syncthreads();  // the sums are zero and the barriers ready
-    // The solve runs once, at the end, on whichever CTA finishes last: every CTA's first
-    // warp runs its code once on zero sums while the first tiles are in flight, so that
-    // the code is cached there (the results are dropped).
-    if (threadIdx.x < 5) calib_scale(0, threadIdx.x, D == 4, s_zero, s_warm);
-    __syncwarp();
-    if (threadIdx.x < 20) calib_entry(0, threadIdx.x, D == 4, s_zero, s_warm);
-    __syncwarp();
-    if (threadIdx.x == 0) calib_factor(0, D, s_zero, s_warm, s_warm + kCalSolveWords);
-    __syncwarp();
     if (TMA && c0 < c1) {
         // The last warp produces (its lane 0 issues each tile once the consumers have
         // released the stage), the others consume at their own pace: no CTA barrier in
@@ -490,7 +502,25 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(long long N, const
     if (__any_sync(kFull, bad) && lane == 0) record_status(ctl, kEInval);
     if (!ok && threadIdx.x == 0) record_status(ctl, kECuda);
     __syncthreads();
-    for (int i = threadIdx.x; i < M * kCalAcc; i += blockDim.x) atomic_add128(acc + 2 * i, sacc[2 * i], sacc[2 * i + 1]);
+    // each sum: the direct adds plus the flushes' carry-save words (the x t_hi halves of b
+    // weigh 2^26)
+    for (int i = threadIdx.x; i < M * kCalAcc; i += blockDim.x) {
+        const int mm = i / kCalAcc, k = i - mm * kCalAcc;
+        U128 v{sacc[2 * i], sacc[2 * i + 1]};
+        auto add_cs = [&](int f, int sh) {
+            const unsigned long long *w = scs + ((size_t)mm * kCalFlushSums + f) * 2;
+            // w0 + 2^32 w1, then shifted left by sh (< 32): below 2^128
+            U128 c{w[0], 0ull};
+            add128(c, w[1] << 32, w[1] >> 32);
+            add128(v, c.lo << sh, sh ? (c.hi << sh) | (c.lo >> (64 - sh)) : c.hi);
+        };
+        if (k < 15) add_cs(k, 0);
+        else if (k < 20) {
+            add_cs(k, 0);
+            add_cs(k + 5, 26);
+        } else add_cs(25, 0);
+        atomic_add128(acc + 2 * i, v.lo, v.hi);
+    }
     // the last CTA to finish solves every model and clears the sums for the next call
     __threadfence();
     __syncthreads();
@@ -519,9 +549,10 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(long long N, const
 
 }  // namespace
 
-static_assert(kCalMaxModels * kCalAcc * 16 + 3 * kCalStageBytes <= kCalSmemMax, "three stages at most models");
+static_assert(kCalMaxModels * (kCalAcc + kCalFlushSums) * 16 + 2 * kCalStageBytes <= kCalSmemMax,
+              "two stages at most models");
 
-static_assert((size_t)kCalMaxModels * kCalSolveWords * 8 <= 3 * kCalStageBytes, "the solve's entries fit the ring");
+static_assert((size_t)kCalMaxModels * kCalSolveWords * 8 <= 2 * kCalStageBytes, "the solve's entries fit the ring");
 static size_t solve_bytes(int M) { return (size_t)M * kCalSolveWords * 8; }
 
 static int calib_stages(int M) {

@@ -198,8 +198,9 @@ constexpr int kCalStagesMax = 3;                    // tiles in flight per CTA
 constexpr int kCalFlushRows = 128;                  // rows a lane sums in 64 bits between flushes
 constexpr size_t kCalSmemMax = 227 * 1024;
 constexpr size_t kCalStageBytes = (size_t)kCalTile * (kCalCols * 8 + 8 + 4);
-// the CTA's shared 128-bit sums [M][kCalAcc]
-__host__ __device__ inline size_t cal_sums_bytes(int M) { return (size_t)M * kCalAcc * 16; }
+constexpr int kCalFlushSums = 26;  // a warp flush's sums: 15 of G, 5 + 5 halves of b, the row count
+// the CTA's shared sums: 128-bit [M][kCalAcc] and the flushes' carry-save words [M][kCalFlushSums]
+__host__ __device__ inline size_t cal_sums_bytes(int M) { return (size_t)M * (kCalAcc + kCalFlushSums) * 16; }
 // the calibration's device words: the sums [M][kCalAcc][2] and the CTA counter of the
 // last-CTA solve (zero between calls)
 __host__ __device__ inline size_t cal_acc_words(int M) { return (size_t)M * kCalAcc * 2 + 2; }
