@@ -107,3 +107,46 @@ def test_unaligned_inputs_take_the_direct_path():
     np.testing.assert_allclose(got, oracle.calibrate(F[1:], m[1:], t[1:], M, shared_beta1=False), rtol=RTOL)
     aligned = rt.calibrate(Fd, md, td, shared_beta1=False).cpu().numpy()
     np.testing.assert_allclose(aligned, oracle.calibrate(F, m, t, M, shared_beta1=False), rtol=RTOL)
+
+
+def test_large_values_take_the_exact_128_bit_path():
+    # features at or above 2^26 (up to just below 2^32) and times at or above 2^8 s skip
+    # the 64-bit register sums and add to the 128-bit sums directly; rows of both kinds
+    # interleave within warps
+    M = 3
+    coef = coef_of(M, 9)
+    F, m, t = W.batch_log(40_000, M, seed=10, coef=coef, noise=0.03)
+    F = F.copy()
+    t = t.copy()
+    big = np.arange(len(t)) % 3 == 0
+    F[big, 3] *= 64      # up to ~6.7e7 > 2^26
+    F[big, 4] = np.minimum(F[big, 4] * 64, (1 << 32) - 1)
+    slow = np.arange(len(t)) % 7 == 0
+    t[slow] += 300.0     # beyond 2^8 s
+    assert (F[big] >> 26).any() and (t[slow] >= 256.0).all() and (F < (1 << 32)).all()
+    rt = router_for(M)
+    for shared in (True, False):
+        got = rt.calibrate(dev(F), dev(m), dev(t), shared_beta1=shared).cpu().numpy()
+        assert rt.status() == R().LR_OK
+        np.testing.assert_allclose(got, oracle.calibrate(F, m, t, M, shared_beta1=shared), rtol=RTOL)
+
+
+def test_many_models():
+    # 128 models, the most the kernel takes: its shared sums leave room for two stages
+    M = 128
+    coef = coef_of(M, 11)
+    F, m, t = W.batch_log(400_000, M, seed=12, coef=coef, noise=0.04, grouped=True)
+    got = router_for(M).calibrate(dev(F), dev(m), dev(t), shared_beta1=False).cpu().numpy()
+    np.testing.assert_allclose(got, oracle.calibrate(F, m, t, M, shared_beta1=False), rtol=RTOL)
+
+
+def test_long_slices_flush_within_128_rows():
+    # more than 128 rows a consumer lane (10M rows over one CTA per SM): the warps flush
+    # their 64-bit sums before they could overflow, mid-model
+    M = 2
+    coef = coef_of(M, 13)
+    F, m, t = W.batch_log(10_000_000, M, seed=14, coef=coef, noise=0.02)
+    rt = router_for(M)
+    got = rt.calibrate(dev(F), dev(m), dev(t), shared_beta1=True).cpu().numpy()
+    assert rt.status() == R().LR_OK
+    np.testing.assert_allclose(got, oracle.calibrate(F, m, t, M, shared_beta1=True), rtol=RTOL)
