@@ -434,26 +434,32 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             // to them): those run, the rest go, in order, to the front of the waiting
             // queue.  The prefill request, last, goes first, so the survivors are
             // decoders.
-            long long acc = 0, fitb = -1;  // blocks after the batch: before the chunk; of the survivors
-            int cut = ne;
-            for (int base = 0; base < ne; base += 32) {
-                const int s = base + lane;
+            // Every request's blocks after the batch sum to what is held plus what the
+            // batch needs, so the cut is found from the tail: the first slot cut (from the
+            // end) whose suffix of post-batch blocks reaches the excess over nb_j.  Usually
+            // few requests go, and the walk stops in the first 32 slots.
+            const long long total = (nbk - freeb) + need_all, excess = total - nbk;
+            long long acc = 0, fitb = -1;  // post-batch blocks: of the suffix so far; of the survivors
+            int cut = 0;
+            for (int top = ne - 1; top >= 0; top -= 32) {
+                const int s = top - lane;
                 long long wv = 0;
-                if (s < ne) {
+                if (s >= 0) {
                     const int4 q = rq[s];
                     if (q.y == 0) wv = kv_blocks32(q.x + G + 1, bs);
                     else if (q.y > 0) wv = kv_blocks32(q.x + px, bs);
                 }
-                const long long cum = acc + warp_incl_sum64(wv, lane);
-                const int k = __popc(__ballot_sync(kFull, s < ne && cum <= nbk));
-                if (k < 32) {
-                    cut = base + k;
-                    fitb = k > 0 ? __shfl_sync(kFull, cum, k - 1) : acc;
+                const long long suf = acc + warp_incl_sum64(wv, lane);
+                const unsigned hit = __ballot_sync(kFull, s >= 0 && suf >= excess);
+                if (hit) {
+                    const int l0 = __ffs(hit) - 1;
+                    cut = top - l0;
+                    fitb = total - __shfl_sync(kFull, suf, l0);
                     break;
                 }
-                acc = __shfl_sync(kFull, cum, 31);
+                acc = __shfl_sync(kFull, suf, 31);
             }
-            if (fitb < 0) fitb = acc;
+            if (fitb < 0) fitb = total - acc;  // (unreachable: the whole list reaches the excess)
             int m = 0;
             for (int base = cut; base < ne; base += 32) {
                 const int s = base + lane;
