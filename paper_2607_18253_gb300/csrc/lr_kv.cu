@@ -86,9 +86,37 @@ __device__ __forceinline__ void kv_cal_push(int32_t *head, int32_t *nxt, int32_t
 __device__ __forceinline__ long long kv_end(const int4 &q, long long mctx) {
     return min((long long)q.z - 1, mctx - 1 - q.x);
 }
-__device__ __forceinline__ int kv_res(int x, int bs) {
-    const int r = x % bs;
-    return r < 0 ? r + bs : r;
+// Division by an instance's block size, which the load repeats many times a batch:
+// unsigned n / d for any 32-bit n as a multiply-high and shifts (Granlund and
+// Montgomery's method for invariant divisors: l = ceil(log2 d), m = floor(2^32 (2^l - d)
+// / d) + 1, q = (t + ((n - t) >> 1)) >> (l - 1) with t = mulhi(m, n); d = 1 takes
+// shifts of 0).
+struct Div32 {
+    unsigned d, m;
+    int s1, s2;
+};
+__device__ __forceinline__ Div32 make_div32(int d) {
+    const unsigned ud = (unsigned)d;
+    const int l = ud <= 1u ? 0 : 32 - __clz((int)(ud - 1u));
+    Div32 v;
+    v.d = ud;
+    v.m = (unsigned)((((1ull << 32) * ((1ull << l) - ud)) / ud) + 1ull);
+    v.s1 = min(l, 1);
+    v.s2 = max(l - 1, 0);
+    return v;
+}
+__device__ __forceinline__ unsigned udiv32(const Div32 &v, unsigned n) {
+    const unsigned t = __umulhi(v.m, n);
+    return (t + ((n - t) >> v.s1)) >> v.s2;
+}
+// ceil(c / d) for 0 <= c < 2^31
+__device__ __forceinline__ int dblk(const Div32 &v, int c) { return (int)udiv32(v, (unsigned)c + v.d - 1u); }
+// x mod d in [0, d) for any int x
+__device__ __forceinline__ int dres(const Div32 &v, int x) {
+    if (x >= 0) return (int)((unsigned)x - udiv32(v, (unsigned)x) * v.d);
+    const unsigned ax = (unsigned)(-(long long)x);
+    const unsigned r = ax - udiv32(v, ax) * v.d;
+    return r == 0u ? 0 : (int)(v.d - r);
 }
 
 // One instance's residents alone, batch by batch, from the snapshot.  Every lane
@@ -112,6 +140,7 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
     const int S = c.S[j];
     const long long nbk = a.kv.nb[j], mctx = a.kv.mctx[j];
     const int bs = a.kv.bs[j];
+    const Div32 dv = make_div32(bs);
     const int C = c.capR + c.capW;  // at most this many residents
     int4 *rq = reinterpret_cast<int4 *>(wb);               // running list slots
     int2 *wq = reinterpret_cast<int2 *>(rq + C);           // waiting ring (prefill, decode)
@@ -137,7 +166,7 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
     // file decoder slot s, held as q (fourth word: residue) at batch G
     auto file = [&](int s, const int4 &q, int G_) {
         const long long E = kv_end(q, mctx);
-        eb[s] = kv_blocks32((int)(q.x + E + 1), bs);
+        eb[s] = dblk(dv, (int)(q.x + E + 1));
         kv_cal_push(head, nxt, ovf, s, E, G_);
     };
     // Copy and validate the snapshot: only the last running request may still be in
@@ -159,13 +188,13 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             bad |= pre > 0 && t != nr0 - 1;
             bad |= (long long)ctx + pre >= mctx;
             bad |= ok && kv_blocks(min((long long)ctx + pre + dec, mctx), bs) > nbk;
-            const int h = ok ? kv_blocks32(ctx, bs) : 0;
+            const int h = ok ? dblk(dv, ctx) : 0;
             held += h;
             if (pre == 0) {
                 src += ctx;
                 ++nd;
             }
-            rq[t] = pre > 0 ? make_int4(ctx, pre, dec, h) : make_int4(ctx, 0, dec, ctx % bs);
+            rq[t] = pre > 0 ? make_int4(ctx, pre, dec, h) : make_int4(ctx, 0, dec, dres(dv, ctx));
         }
     }
     for (int t = lane; t < c.capW; t += 32) {
@@ -279,7 +308,7 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
         const int ndk = nd - endsb, nrk = nr - endsb;
         const long long srck = src - rcb;
         // decoders at a block boundary in batch G + k, the window's earlier ends removed
-        const int gk = (gr + k) % bs;
+        const int gk = dres(dv, gr + k);
         const int rk = gk == 0 ? 0 : bs - gk;
         int sub = 0;
         for (int e = 0; e < nev; ++e) {
@@ -298,7 +327,7 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             x = min(remk, avail);
             pf_ends = remk - x == 0;
             ctxp = pq.x + (pq.y - remk);
-            pneed = kv_blocks32(ctxp + x, bs) - kv_blocks32(ctxp, bs);
+            pneed = dblk(dv, ctxp + x) - dblk(dv, ctxp);
         }
         const int need_all = need_d + pneed;
         const long long dl = k < W ? ebk - need_all : 0;       // free blocks gained over batch k
@@ -357,14 +386,14 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             }
         }
         if (in) head[(G + k) & (kKvCal - 1)] = -1;
-        if (pfs >= 0 && lane == 0) rq[pfs] = make_int4(ctxpL + xL, remL - xL, pq.z, kv_blocks32(ctxpL + xL, bs));
+        if (pfs >= 0 && lane == 0) rq[pfs] = make_int4(ctxpL + xL, remL - xL, pq.z, dblk(dv, ctxpL + xL));
         nd = ndL - cntL;
         nr = nrL - cntL;
         src = srcL - rckL;
         freeb = fbL + dlL;
         nrec += n;
         G += n;
-        gr = G % bs;
+        gr = dres(dv, G);
         if (nr == 0) done = 1;
         __syncwarp();
         return n;
@@ -411,7 +440,7 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
         int px = 0, pneed = 0;
         if (pfs >= 0) {
             px = min(pq.y, B - nd);
-            pneed = kv_blocks32(pq.x + px, bs) - pq.w;
+            pneed = dblk(dv, pq.x + px) - pq.w;
         }
         const int need_all = need_d + pneed;
         long long slack, f1, f2, f3, f4;
@@ -446,8 +475,8 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
                 long long wv = 0;
                 if (s >= 0) {
                     const int4 q = rq[s];
-                    if (q.y == 0) wv = kv_blocks32(q.x + G + 1, bs);
-                    else if (q.y > 0) wv = kv_blocks32(q.x + px, bs);
+                    if (q.y == 0) wv = dblk(dv, q.x + G + 1);
+                    else if (q.y > 0) wv = dblk(dv, q.x + px);
                 }
                 const long long suf = acc + warp_incl_sum64(wv, lane);
                 const unsigned hit = __ballot_sync(kFull, s >= 0 && suf >= excess);
@@ -518,7 +547,7 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
                 ++dying;
                 pfs = -1;
             } else {
-                const int4 q = make_int4(cx - (G + 1), 0, dec + (G + 1), kv_res(cx - (G + 1), bs));
+                const int4 q = make_int4(cx - (G + 1), 0, dec + (G + 1), dres(dv, cx - (G + 1)));
                 if (lane == 0) {
                     rq[r] = q;
                     hist[q.w] += 1;
@@ -542,14 +571,14 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
         // FCFS: a head whose first chunk's blocks are not free admits nobody (the
         // usual case while a queue waits on a full cache)
         bool adm = budget > 0 && wc > 0 && nr < S;
-        if (adm) adm = kv_blocks32(min(wq[wh].x, budget), bs) <= freeb;
+        if (adm) adm = dblk(dv, min(wq[wh].x, budget)) <= freeb;
         while (adm && budget > 0 && wc > 0 && nr < S) {
             if (ne + 32 > C) compact();
             const bool in = lane < wc && lane < S - nr;
             int slot = wh + lane;
             if (slot >= C) slot -= C;
             const int2 wv = in ? wq[slot] : make_int2(0, 0);
-            const int hb_i = in ? kv_blocks32(wv.x, bs) : 0;
+            const int hb_i = in ? dblk(dv, wv.x) : 0;
             const int cp = warp_incl_sum32(wv.x, lane);  // 32 prompts of at most 2^24 tokens
             const int cb = warp_incl_sum32(hb_i, lane);
             const bool whole = in && cp <= budget && (long long)cb <= freeb;
@@ -558,7 +587,7 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
             const bool ends = whole && (dec_a <= 0 || (long long)wv.x >= mctx);
             if (whole) {
                 const int s = ne + lane;
-                const int4 q = make_int4(wv.x - (G + 1), ends ? -1 : 0, dec_a + (G + 1), kv_res(wv.x - (G + 1), bs));
+                const int4 q = make_int4(wv.x - (G + 1), ends ? -1 : 0, dec_a + (G + 1), dres(dv, wv.x - (G + 1)));
                 rq[s] = q;
                 if (!ends) {
                     atomicAdd(&hist[q.w], 1);
@@ -591,7 +620,7 @@ __device__ void kv_instance(const KvLoad &a, const StateBuf &out, int j, int lan
                 if (budget > 0 && wc > 0 && nr < S) {
                     const int2 hv = wq[wh];
                     const int x = min(hv.x, budget);
-                    const int nb1 = kv_blocks32(x, bs);
+                    const int nb1 = dblk(dv, x);
                     if (x < hv.x && nb1 <= freeb) {
                         if (lane == 0) rq[ne] = make_int4(x, hv.x - x, hv.y, nb1);
                         pfs = ne;
