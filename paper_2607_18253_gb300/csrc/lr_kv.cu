@@ -783,6 +783,7 @@ struct KvView {
     long long nb, mctx;
     float b[5];
     int la0, nrec, ns, done, B, bs;
+    Div32 dv;  // division by bs
 };
 
 // Record t of the view; past the records of a finished instance, an empty batch.
@@ -858,7 +859,7 @@ __device__ int kv_candidate(const KvView &v, const KvStage &st, int p, long long
                 run = false;
             } else if (bar > 0) {
                 const int x = pre > 0 ? min(pre, bar) : 1;
-                const int nh = kv_blocks32(ctx + x, v.bs);
+                const int nh = dblk(v.dv, ctx + x);
                 if (nh > far) {  // its own tokens do not fit: it preempts itself
                     pre += ctx;
                     ctx = 0;
@@ -885,7 +886,7 @@ __device__ int kv_candidate(const KvView &v, const KvStage &st, int p, long long
         }
         if (pre <= thr) {  // admission (pre == p while waiting)
             const int x = min(pre, bl);
-            held = kv_blocks32(x, v.bs);
+            held = dblk(v.dv, x);
             o1 += x;
             o4 += (long long)x * (x + 1) / 2;
             ctx = x;
@@ -1062,6 +1063,7 @@ __global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a, b
         v.nb = a.kv.nb[j];
         v.mctx = a.kv.mctx[j];
         v.bs = a.kv.bs[j];
+        v.dv = make_div32(v.bs);
         v.B = c.B[j];
         const float *cf = c.coef + 5 * c.moi[j];
         for (int k = 0; k < 5; ++k) v.b[k] = cf[k];
