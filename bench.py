@@ -688,13 +688,13 @@ def run_kv(args, dev, wl, flush):
                        "ctx_limited_instances": int((limits[2] < (1 << 40)).sum()),
                        "blocks_median": int(np.median(limits[1]))},
             "ms_per_step": out["step"], "value": Q * I / (out["step"] * 1e-3), "unit": UNIT, "steps": K,
-            "gpu_launches": 12 * K, "load_ms": out["load"], "estimate_ms": out["estimate"],
+            "gpu_launches": 14 * K, "load_ms": out["load"], "estimate_ms": out["estimate"],
             "estimate_value": Q * I / (out["estimate"] * 1e-3),
-            "roofline": {"kernel": "lr_estimate_ttft with KV limits (count, scan, scatter, k_kv_estimate, "
-                                   "k_kv_expand)", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+            "roofline": {"kernel": "lr_estimate_ttft with KV limits (count, tile sums, scan, scatter, "
+                                   "k_kv_estimate, k_kv_expand)", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                          "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
                          "algorithmic_bytes": nbytes, "traffic": None,
-                         "note": "the call's five kernels together; k_kv_estimate alone read 4.92 MB and wrote "
+                         "note": "the call's six kernels together; k_kv_estimate alone read 4.92 MB and wrote "
                                  "0.19 MB per launch (ncu); the load is one dependency chain per instance"}}
 
 
@@ -922,9 +922,9 @@ def run_stream(args, dev):
     lat = [e0.elapsed_time(e1) for e0, e1 in ev]
     q = np.percentile(np.asarray(lat) * 1e3, [50, 99])
     fin = rt.read_state(device=dev)
-    # launches per decision: advance (K3 KV, KV load) + route (count, scan, scatter, walk,
-    # expand, route)
-    launches += 8 * nb
+    # launches per decision: advance (K3 KV, KV load) + route (count, tile sums, scan,
+    # scatter, walk, expand, route)
+    launches += 9 * nb
     out["kv_poisson_16"] = {"arrival_qps": 0.5 * float(cap.sum()), "batches": nb, "queries": nb * m, "p50_us": float(q[0]), "p99_us": float(q[1]),
                             "mean_us": float(np.mean(lat) * 1e3), "wall_s": wall,
                             "simulated_s": float(arr[nb * m - 1]),

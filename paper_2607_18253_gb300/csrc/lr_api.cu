@@ -52,7 +52,7 @@ struct lr_ctx {
     size_t kv_smem = 0;
     size_t k3_kv_smem = 0;  // the KV stream step's shared memory (all warps of a CTA)
     int32_t *kv_order = nullptr;  // [max_queries] the estimate's query order
-    int32_t *kv_leaders = nullptr, *kv_sort = nullptr;  // [max_queries]; [4][kKvBuckets] + 4 + [ceil(I/8)]
+    int32_t *kv_leaders = nullptr, *kv_sort = nullptr;  // [max_queries]; [4][kKvBuckets] + 4 + [2][tiles] + [ceil(I/8)]
     float *kv_mat = nullptr;  // [max_queries][I] the KV estimate matrix a route scores
     std::vector<void *> kv_allocs;
     std::vector<void *> allocs;
@@ -488,7 +488,8 @@ static int estimate_common(lr_ctx *c, int32_t Q, const int32_t *p, float *ttft, 
         k.run = k.start + lr::kKvBuckets;
         k.uid = k.run + lr::kKvBuckets;
         k.nu = k.uid + lr::kKvBuckets;
-        k.claim = k.nu + 4;
+        k.tsum = k.nu + 4;
+        k.claim = k.tsum + 2 * lr::kKvScanTiles;
         cudaError_t e = lr::launch_kv_estimate(k, c->sms, (cudaStream_t)stream);
         return e == cudaSuccess ? LR_OK : cuda_fail(c, e, "KV estimate launch");
     }
@@ -741,7 +742,7 @@ int lr_set_kv_limits(lr_ctx *c, const int32_t *block_size, const int64_t *num_bl
     if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (size_t)c->max_queries, &ord);
     if (e == cudaSuccess) e = alloc(sizeof(int32_t) * (size_t)c->max_queries, &lead);
     if (e == cudaSuccess) e = alloc(sizeof(float) * (size_t)c->max_queries * I, &mat);
-    const size_t srt_words = 4 * (size_t)lr::kKvBuckets + 4 + (size_t)(I + 7) / 8;
+    const size_t srt_words = 4 * (size_t)lr::kKvBuckets + 4 + 2 * (size_t)lr::kKvScanTiles + (size_t)(I + 7) / 8;
     if (e == cudaSuccess) e = alloc(sizeof(int32_t) * srt_words, &srt);
     if (e == cudaSuccess) e = cudaMemset(srt, 0, sizeof(int32_t) * srt_words);
     if (e == cudaSuccess) e = alloc(sizeof(long long) * I, &nb);

@@ -254,10 +254,12 @@ struct KvEst {
     // query per length is estimated and the others copy its rows
     int32_t *cnt, *start, *run, *uid;  // [kKvBuckets]
     int32_t *nu;                       // [1] distinct lengths
+    int32_t *tsum;                     // [2][kKvScanTiles] per-tile bucket sums of the scan
     int32_t *order, *leaders;          // [max_queries]
     int32_t *claim;                    // [ceil(I / 8)] the estimate's block counters per instance group
 };
 constexpr int kKvBuckets = 1 << 16;
+constexpr int kKvScanTiles = kKvBuckets / 4096;  // the bucket scan's tiles, one CTA each
 cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st);
 
 // Batches covered by K1's completion calendar; decoders ending later are

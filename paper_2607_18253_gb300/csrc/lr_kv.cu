@@ -934,62 +934,87 @@ __global__ void __launch_bounds__(256) k_kv_count(const int32_t *prompt, int Q, 
 // the next call, and the estimate's block counters too.  Tiles of 4096 buckets,
 // four per thread as one 16-byte word.
 constexpr int kScanThreads = 1024;
-static_assert(kKvBuckets % (4 * kScanThreads) == 0, "scan tiles cover the buckets");
-__global__ void __launch_bounds__(kScanThreads) k_kv_scan(int32_t *cnt, int32_t *start, int32_t *run, int32_t *uid,
-                                                          int32_t *nu, int nbk, int32_t *claim, int groups) {
+static_assert(kKvBuckets == kKvScanTiles * 4 * kScanThreads, "scan tiles cover the buckets");
+// The bucket scan in two launches, one CTA per tile of 4,096 buckets: the tiles'
+// sums (count and non-empty buckets), then each tile's exclusive scan from the sums of
+// the tiles before it.  (One CTA over every bucket was bound by one SM's bandwidth.)
+__global__ void __launch_bounds__(kScanThreads) k_kv_tile_sums(const int32_t *cnt, int32_t *tsum, int32_t *claim,
+                                                               int groups) {
     __shared__ int ws[2][kScanThreads / 32];
-    __shared__ int tot[2];
     const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-    for (int g = tid; g < groups; g += kScanThreads) claim[g] = 0;
-    int carry_c = 0, carry_u = 0;
-    constexpr int kTile = 4 * kScanThreads;
-    for (int t0 = 0; t0 < nbk; t0 += kTile) {  // nbk <= kKvBuckets, a multiple of kTile
-        const int b = t0 + 4 * tid;
-        const int4 v = reinterpret_cast<const int4 *>(cnt)[b / 4];
-        const int sc = v.x + v.y + v.z + v.w;
-        const int su = (v.x > 0) + (v.y > 0) + (v.z > 0) + (v.w > 0);
-        const int ic = warp_incl_sum32(sc, lane), iu = warp_incl_sum32(su, lane);
-        if (lane == 31) {
-            ws[0][w] = ic;
-            ws[1][w] = iu;
-        }
-        __syncthreads();
-        if (w == 0) {
-            const int xc = ws[0][lane], xu = ws[1][lane];
-            const int yc = warp_incl_sum32(xc, lane), yu = warp_incl_sum32(xu, lane);
-            ws[0][lane] = yc - xc;
-            ws[1][lane] = yu - xu;
-            if (lane == 31) {
-                tot[0] = yc;
-                tot[1] = yu;
-            }
-        }
-        __syncthreads();
-        int oc = carry_c + ws[0][w] + ic - sc, ou = carry_u + ws[1][w] + iu - su;
-        int4 so, uo;
-        so.x = oc;
-        uo.x = ou;
-        oc += v.x;
-        ou += v.x > 0;
-        so.y = oc;
-        uo.y = ou;
-        oc += v.y;
-        ou += v.y > 0;
-        so.z = oc;
-        uo.z = ou;
-        oc += v.z;
-        ou += v.z > 0;
-        so.w = oc;
-        uo.w = ou;
-        reinterpret_cast<int4 *>(start)[b / 4] = so;
-        reinterpret_cast<int4 *>(run)[b / 4] = so;
-        reinterpret_cast<int4 *>(uid)[b / 4] = uo;
-        reinterpret_cast<int4 *>(cnt)[b / 4] = make_int4(0, 0, 0, 0);
-        carry_c += tot[0];
-        carry_u += tot[1];
-        __syncthreads();
+    if (blockIdx.x == 0)
+        for (int g = tid; g < groups; g += kScanThreads) claim[g] = 0;
+    const int4 v = reinterpret_cast<const int4 *>(cnt)[blockIdx.x * kScanThreads + tid];
+    int sc = v.x + v.y + v.z + v.w;
+    int su = (v.x > 0) + (v.y > 0) + (v.z > 0) + (v.w > 0);
+    sc = warp_sum32(sc);
+    su = warp_sum32(su);
+    if (lane == 0) {
+        ws[0][w] = sc;
+        ws[1][w] = su;
     }
-    if (tid == 0) *nu = carry_u;
+    __syncthreads();
+    if (w == 0) {
+        const int xc = warp_sum32(ws[0][lane]), xu = warp_sum32(ws[1][lane]);
+        if (lane == 0) {
+            tsum[2 * blockIdx.x] = xc;
+            tsum[2 * blockIdx.x + 1] = xu;
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kScanThreads) k_kv_scan(int32_t *cnt, int32_t *start, int32_t *run, int32_t *uid,
+                                                          int32_t *nu, const int32_t *tsum) {
+    __shared__ int ws[2][kScanThreads / 32];
+    __shared__ int base[2];
+    const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+    if (tid == 0) {  // the tiles before this one
+        int c = 0, u = 0;
+        for (int t = 0; t < (int)blockIdx.x; ++t) {
+            c += tsum[2 * t];
+            u += tsum[2 * t + 1];
+        }
+        base[0] = c;
+        base[1] = u;
+        if (blockIdx.x == gridDim.x - 1) *nu = u + tsum[2 * blockIdx.x + 1];
+    }
+    const int b = (blockIdx.x * kScanThreads + tid) * 4;
+    const int4 v = reinterpret_cast<const int4 *>(cnt)[b / 4];
+    const int sc = v.x + v.y + v.z + v.w;
+    const int su = (v.x > 0) + (v.y > 0) + (v.z > 0) + (v.w > 0);
+    const int ic = warp_incl_sum32(sc, lane), iu = warp_incl_sum32(su, lane);
+    if (lane == 31) {
+        ws[0][w] = ic;
+        ws[1][w] = iu;
+    }
+    __syncthreads();
+    if (w == 0) {
+        const int xc = ws[0][lane], xu = ws[1][lane];
+        const int yc = warp_incl_sum32(xc, lane), yu = warp_incl_sum32(xu, lane);
+        ws[0][lane] = yc - xc;
+        ws[1][lane] = yu - xu;
+    }
+    __syncthreads();
+    int oc = base[0] + ws[0][w] + ic - sc, ou = base[1] + ws[1][w] + iu - su;
+    int4 so, uo;
+    so.x = oc;
+    uo.x = ou;
+    oc += v.x;
+    ou += v.x > 0;
+    so.y = oc;
+    uo.y = ou;
+    oc += v.y;
+    ou += v.y > 0;
+    so.z = oc;
+    uo.z = ou;
+    oc += v.z;
+    ou += v.z > 0;
+    so.w = oc;
+    uo.w = ou;
+    reinterpret_cast<int4 *>(start)[b / 4] = so;
+    reinterpret_cast<int4 *>(run)[b / 4] = so;
+    reinterpret_cast<int4 *>(uid)[b / 4] = uo;
+    reinterpret_cast<int4 *>(cnt)[b / 4] = make_int4(0, 0, 0, 0);
 }
 
 __global__ void __launch_bounds__(256) k_kv_scatter(const int32_t *prompt, int Q, int pmax, int shift, int32_t *run,
@@ -1166,7 +1191,9 @@ cudaError_t launch_kv_estimate(const KvEst &a, int sms, cudaStream_t st) {
     const bool exact = shift == 0;
     const int g1 = std::max(1, std::min((a.Q + 255) / 256, sms * 4));
     k_kv_count<<<g1, 256, 0, st>>>(a.prompt, a.Q, a.cfg.pmax, shift, a.cnt);
-    k_kv_scan<<<1, kScanThreads, 0, st>>>(a.cnt, a.start, a.run, a.uid, a.nu, (nbk + 4095) / 4096 * 4096, a.claim, gy);
+    const int tiles = (nbk + 4095) / 4096;
+    k_kv_tile_sums<<<tiles, kScanThreads, 0, st>>>(a.cnt, a.tsum, a.claim, gy);
+    k_kv_scan<<<tiles, kScanThreads, 0, st>>>(a.cnt, a.start, a.run, a.uid, a.nu, a.tsum);
     k_kv_scatter<<<g1, 256, 0, st>>>(a.prompt, a.Q, a.cfg.pmax, shift, a.run, a.start, a.uid, a.order, a.leaders);
     if (a.cfg.mode == 0) k_kv_estimate<0><<<grid, kEstWarps * 32, kEstSmem, st>>>(a, exact);
     else k_kv_estimate<1><<<grid, kEstWarps * 32, kEstSmem, st>>>(a, exact);
