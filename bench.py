@@ -319,10 +319,10 @@ def run_gpu(args):
             with torch.cuda.stream(side):
                 rt.route(dqq[0], dqq[1], dqq[2], wl.lam, wl.mu, ttft_matrix=mat, out=outs[b], stream=side)
             main.wait_stream(side)
-            host_out_flat[b].copy_(dev_out[b], non_blocking=True)
 
         upload()
         step()
+        host_out_flat[b].copy_(dev_out[b], non_blocking=True)
         torch.cuda.synchronize()
         gu, gs = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
         with torch.cuda.graph(gu):
@@ -332,29 +332,40 @@ def run_gpu(args):
         g_up.append(gu)
         g_step.append(gs)
 
+    d2h_stream = torch.cuda.Stream(device=dev)
+
     def run_e2e(steps):
         # `steps` pipelined steps with no L2 flush inside the loop (each step's inputs
-        # arrive by their own host->device copy).  Returns the span from the first
-        # upload's issue to the last result's arrival, and each step's latency from
-        # its upload's issue to its result's arrival.
+        # arrive by their own host->device copy).  Three streams: uploads, compute and
+        # read-backs, so that step k's read-back and step k+1's upload overlap step
+        # k+1's compute.  Returns the span from the first upload's issue to the last
+        # result's arrival in host memory, and each step's latency from its upload's
+        # issue to its result's arrival.
         ev_up0 = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
-        ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+        ev1 = [torch.cuda.Event() for _ in range(steps)]          # compute done
+        ev2 = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]  # result in host memory
         up = [torch.cuda.Event() for _ in range(steps)]
         for k in range(steps):
             b = k & 1
             if k >= 2:
-                copy_stream.wait_event(ev1[k - 2])  # buffer set b is free again
+                copy_stream.wait_event(ev1[k - 2])  # step k-2 has read buffer set b's inputs
             ev_up0[k].record(copy_stream)
             with torch.cuda.stream(copy_stream):
                 g_up[b].replay()
             up[k].record(copy_stream)
             stream.wait_event(up[k])
+            if k >= 2:
+                stream.wait_event(ev2[k - 2])  # step k-2's results have left buffer set b
             g_step[b].replay()
             ev1[k].record(stream)
+            d2h_stream.wait_event(ev1[k])
+            with torch.cuda.stream(d2h_stream):
+                host_out_flat[b].copy_(dev_out[b], non_blocking=True)
+            ev2[k].record(d2h_stream)
             if k >= 1:
-                ev1[k - 1].synchronize()  # the host has the previous step's result
+                ev2[k - 1].synchronize()  # the host has the previous step's result
         torch.cuda.synchronize()
-        return ev_up0[0].elapsed_time(ev1[-1]), [ev_up0[k].elapsed_time(ev1[k]) for k in range(steps)]
+        return ev_up0[0].elapsed_time(ev2[-1]), [ev_up0[k].elapsed_time(ev2[k]) for k in range(steps)]
 
     run_e2e(max(3, args.warmup))
     KE = max(3, min(K, 2000))
@@ -417,12 +428,13 @@ def run_gpu(args):
                     "p50_latency_ms": elat[len(elat) // 2],
                     "p99_latency_ms": elat[min(len(elat) - 1, int(0.99 * len(elat)))],
                     "note": "through the public API (lr_load_state + lr_route): per step the snapshot and "
-                            "queries are copied from pinned host memory on a copy stream (one packed copy), "
+                            "queries are copied from pinned host memory on an upload stream (one packed copy), "
                             "ingested and routed (K1 || K2), and the result copied back to pinned host memory "
-                            "(one copy), which the host reads one step later; two device buffer sets "
-                            "alternate, so a step's upload overlaps the previous step's compute.  ms_per_step = span from the first upload's "
-                            "issue to the last result's arrival / steps (no L2 flush inside the loop: every "
-                            "step's inputs arrive by copy); latency = a step's upload issue to its result"},
+                            "on a read-back stream (one copy), which the host reads one step later; two device "
+                            "buffer sets alternate, so a step's upload and the previous step's read-back overlap "
+                            "its compute.  ms_per_step = span from the first upload's issue to the last result's "
+                            "arrival / steps (no L2 flush inside the loop: every step's inputs arrive by copy); "
+                            "latency = a step's upload issue to its result's arrival"},
             "gpu_launches": 2 * K, "clocks": clocks, "wall_s_timed_region": t_wall,
             "sequential": {"ms_per_step": seq_ms, "value": _job_rate(cands, world, seq_ms), "unit": UNIT,
                            "note": "K1 then K2 on one stream, same steps (kernel shares are of this time)"},
