@@ -1074,7 +1074,7 @@ __global__ void __launch_bounds__(256) k_kv_expand(const KvEst a) {
 // the longest prompts first, so the longest walks start first and no warp holds
 // more than one instance's walks of one block.
 template <int MODE>
-__global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a, bool exact) {
+__global__ void __launch_bounds__(kEstWarps * 32, 3) k_kv_estimate(const KvEst a, bool exact) {
     extern __shared__ __align__(16) unsigned char est_smem[];
     __shared__ KvView sv[kEstGroup];
     const DevConfig &c = a.cfg;
@@ -1105,14 +1105,38 @@ __global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a, b
             v.pmx = sb.kvp + (size_t)j * a.kv.horizon;
             v.ns = min(v.nrec, kEstStage);
             const KvStage st = kv_stage(est_smem, w);
-            for (int t = lane; t < v.ns; t += 32) {
-                const KvRec *r = v.rec + t;
-                st.slack[t] = __ldg(&r->slack);
-                st.far[t] = __ldg(&r->far);
-                st.thr[t] = __ldg(&r->thr);
-                st.bar[t] = __ldg(&r->bar);
-                st.bl[t] = __ldg(&r->bl);
-                st.pmx[t] = __ldg(v.pmx + t);
+            // the loads of a half of the staged fields issued before its stores (two
+            // memory round trips, within the register budget of three CTAs an SM)
+            constexpr int kPer = kEstStage / 64;
+#pragma unroll 1
+            for (int h = 0; h < 2; ++h) {
+                long long f_sl[kPer], f_fa[kPer], f_th[kPer];
+                int f_ba[kPer], f_bl[kPer], f_pm[kPer];
+#pragma unroll
+                for (int k = 0; k < kPer; ++k) {
+                    const int t = lane + 32 * (k + h * kPer);
+                    if (t < v.ns) {
+                        const KvRec *r = v.rec + t;
+                        f_sl[k] = __ldg(&r->slack);
+                        f_fa[k] = __ldg(&r->far);
+                        f_th[k] = __ldg(&r->thr);
+                        f_ba[k] = __ldg(&r->bar);
+                        f_bl[k] = __ldg(&r->bl);
+                        f_pm[k] = __ldg(v.pmx + t);
+                    }
+                }
+#pragma unroll
+                for (int k = 0; k < kPer; ++k) {
+                    const int t = lane + 32 * (k + h * kPer);
+                    if (t < v.ns) {
+                        st.slack[t] = f_sl[k];
+                        st.far[t] = f_fa[k];
+                        st.thr[t] = f_th[k];
+                        st.bar[t] = f_ba[k];
+                        st.bl[t] = f_bl[k];
+                        st.pmx[t] = f_pm[k];
+                    }
+                }
             }
         }
         if (lane == 0) sv[w] = v;
@@ -1122,16 +1146,35 @@ __global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a, b
     const int nwork = exact ? *a.nu : a.Q;
     const int32_t *work = exact ? a.leaders : a.order;
     const int nitems = (nwork + 31) / 32 * ng;
+    // Software-pipelined: the claim of the next item and its query's prompt are in
+    // flight while the current item is walked.
+    auto claim = [&]() {
+        int v = 0;
+        if (lane == 0) v = atomicAdd(&a.claim[blockIdx.y], 1);
+        return __shfl_sync(kFull, v, 0);
+    };
+    auto fetch = [&](int it_, int &i_, int &p_) {  // this lane's query of item it_ (i_ < 0: none)
+        i_ = -1;
+        p_ = 0;
+        if (it_ < nitems) {
+            const int pos_ = nwork - 1 - ((it_ / ng) * 32 + lane);
+            if (pos_ >= 0) {
+                i_ = work[pos_];
+                p_ = a.prompt[i_];
+            }
+        }
+    };
+    int it = claim();
+    int i_cur, p_cur;
+    fetch(it, i_cur, p_cur);
     for (;;) {
-        int it = 0;
-        if (lane == 0) it = atomicAdd(&a.claim[blockIdx.y], 1);
-        it = __shfl_sync(kFull, it, 0);
         if (it >= nitems) break;
+        const int it_next = claim();
         const int qb = it / ng, g = it - qb * ng;
-        const int pos = nwork - 1 - (qb * 32 + lane);
-        if (pos >= 0) {
-            const int i = work[pos];
-            const int p = a.prompt[i];
+        const int i = i_cur, p = p_cur;
+        int i_nx, p_nx;
+        fetch(it_next, i_nx, p_nx);
+        if (i >= 0) {
             const KvView &v = sv[g];
             long long F[5] = {-1, -1, -1, -1, -1};
             int lt = -1;
@@ -1159,6 +1202,9 @@ __global__ void __launch_bounds__(kEstWarps * 32) k_kv_estimate(const KvEst a, b
             if (a.features)
                 for (int k = 0; k < 5; ++k) a.features[idx * 5 + k] = F[k];
         }
+        it = it_next;
+        i_cur = i_nx;
+        p_cur = p_nx;
     }
 }
 
