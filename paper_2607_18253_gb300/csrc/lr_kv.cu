@@ -749,9 +749,11 @@ __global__ void __launch_bounds__(kKvWarps * 32) k_kv_load(const KvLoad a) {
 }
 
 constexpr float kNaN = __builtin_nanf("");
-constexpr int kEstGroup = 8;    // instances per CTA
+constexpr int kEstGroup = 32;   // instances per CTA
 constexpr int kEstWarps = 8;    // warps per CTA
-constexpr int kEstStage = 256;  // leading records of each instance staged in shared memory
+// leading records of each instance staged in shared memory: on pool256, 99.3% of the
+// candidates reach their first token within 64 records (88% within 16)
+constexpr int kEstStage = 60;  // (60, not 64: three CTAs with their views fit an SM)
 // the staged fields of the walk: slack, far, thr (8 bytes), bar, bl, admission maximum (4)
 constexpr size_t kEstSmem = (size_t)kEstGroup * kEstStage * (3 * 8 + 3 * 4);
 
@@ -1069,8 +1071,8 @@ __global__ void __launch_bounds__(256) k_kv_expand(const KvEst a) {
     }
 }
 
-// CTA: kEstGroup instances, the walk's fields of their leading records staged in
-// shared memory.  The CTAs of a group claim units of (32 queries, one instance),
+// CTA: kEstGroup instances (strided over the pool), the walk's fields of their
+// leading records staged in shared memory.  The CTAs of a group claim units of (32 queries, one instance),
 // the longest prompts first, so the longest walks start first and no warp holds
 // more than one instance's walks of one block.
 template <int MODE>
@@ -1079,11 +1081,13 @@ __global__ void __launch_bounds__(kEstWarps * 32, 3) k_kv_estimate(const KvEst a
     __shared__ KvView sv[kEstGroup];
     const DevConfig &c = a.cfg;
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    const int j0 = blockIdx.y * kEstGroup;
-    const int ng = min(kEstGroup, c.I - j0);
+    // group y holds instances y, y + gy, y + 2 gy, ... (gy groups): every group mixes the
+    // pool's models, whose walks differ in length, so the groups' work is alike
+    const int gy = gridDim.y;
+    const int ng = min(kEstGroup, (c.I - (int)blockIdx.y + gy - 1) / gy);
     const int active = load_acquire(&a.ctl->active);
-    if (w < ng) {
-        const int j = j0 + w;
+    for (int gw = w; gw < ng; gw += kEstWarps) {  // warp w stages instances w, w + 8, ...
+        const int j = gw * gy + blockIdx.y;
         KvView v;
         v.nb = a.kv.nb[j];
         v.mctx = a.kv.mctx[j];
@@ -1104,12 +1108,12 @@ __global__ void __launch_bounds__(kEstWarps * 32, 3) k_kv_estimate(const KvEst a
             v.rec = sb.kvr + (size_t)j * a.kv.horizon;
             v.pmx = sb.kvp + (size_t)j * a.kv.horizon;
             v.ns = min(v.nrec, kEstStage);
-            const KvStage st = kv_stage(est_smem, w);
-            // the loads of a half of the staged fields issued before its stores (two
-            // memory round trips, within the register budget of three CTAs an SM)
-            constexpr int kPer = kEstStage / 64;
-#pragma unroll 1
-            for (int h = 0; h < 2; ++h) {
+            const KvStage st = kv_stage(est_smem, gw);
+            // the loads of the staged fields issued before their stores (one memory
+            // round trip)
+            constexpr int kPer = (kEstStage + 31) / 32;
+            {
+                constexpr int h = 0;
                 long long f_sl[kPer], f_fa[kPer], f_th[kPer];
                 int f_ba[kPer], f_bl[kPer], f_pm[kPer];
 #pragma unroll
@@ -1139,7 +1143,7 @@ __global__ void __launch_bounds__(kEstWarps * 32, 3) k_kv_estimate(const KvEst a
                 }
             }
         }
-        if (lane == 0) sv[w] = v;
+        if (lane == 0) sv[gw] = v;
     }
     __syncthreads();
     // the work: one query per distinct prompt length, or every query, by length
@@ -1196,7 +1200,7 @@ __global__ void __launch_bounds__(kEstWarps * 32, 3) k_kv_estimate(const KvEst a
                 tt = __fmaf_rn(v.b[3], __ll2float_rn(F[3]), tt);
                 tt = __fmaf_rn(v.b[4], __ll2float_rn(F[4]), tt);
             }
-            const size_t idx = (size_t)i * c.I + j0 + g;
+            const size_t idx = (size_t)i * c.I + g * gy + blockIdx.y;
             if (a.ttft) a.ttft[idx] = tt;
             if (a.first_batch) a.first_batch[idx] = err ? -1 : v.la0 + lt;
             if (a.features)
