@@ -818,9 +818,16 @@ __device__ void summarize_instance(const K1Launch &a, const StateBuf &out, int j
         red[(3 * kRows + 2) * 32 + lane] = A3;
         red[(3 * kRows + 3) * 32 + lane] = CB;
         __syncwarp();
+        // lane c sums column c, starting at its own offset so that the 28 lanes read
+        // different banks (a column's 32 partials share one bank group), with four
+        // independent partial sums
         long long tot = 0;
-        if (lane < kCols)
-            for (int l = 0; l < 32; ++l) tot += red[lane * 32 + l];
+        if (lane < kCols) {
+            long long t4[4] = {0, 0, 0, 0};
+#pragma unroll
+            for (int l = 0; l < 32; ++l) t4[l & 3] += red[lane * 32 + ((l + lane) & 31)];
+            tot = (t4[0] + t4[1]) + (t4[2] + t4[3]);
+        }
         __syncwarp();
         if (lane < kCols) red[lane * 32] = tot;  // each column's head holds its sum
         __syncwarp();
