@@ -753,9 +753,13 @@ constexpr int kEstGroup = 32;   // instances per CTA
 constexpr int kEstWarps = 8;    // warps per CTA
 // leading records of each instance staged in shared memory: on pool256, 99.3% of the
 // candidates reach their first token within 64 records (88% within 16)
-constexpr int kEstStage = 60;  // (60, not 64: three CTAs with their views fit an SM)
+constexpr int kEstStage = 52;
 // the staged fields of the walk: slack, far, thr (8 bytes), bar, bl, admission maximum (4)
-constexpr size_t kEstSmem = (size_t)kEstGroup * kEstStage * (3 * 8 + 3 * 4);
+constexpr size_t kEstStageBytes = (size_t)kEstGroup * kEstStage * (3 * 8 + 3 * 4);
+// and each warp's tile of 32 later records (slack, far, thr, bar, bl); three CTAs with
+// their views fit an SM
+constexpr size_t kEstTileBytes = 32 * (3 * 8 + 2 * 4);
+constexpr size_t kEstSmem = kEstStageBytes + kEstWarps * kEstTileBytes;
 
 // The walk's fields of an instance's leading records, in shared memory.
 struct KvStage {
@@ -788,29 +792,19 @@ struct KvView {
     Div32 dv;  // division by bs
 };
 
-// Record t of the view; past the records of a finished instance, an empty batch.
-__device__ __forceinline__ void kv_record(const KvView &v, const KvStage &st, int t, long long &slack,
-                                          long long &far, long long &thr, int &bar, int &bl) {
-    if (t < v.ns) {
-        slack = st.slack[t];
-        far = st.far[t];
-        thr = st.thr[t];
-        bar = st.bar[t];
-        bl = st.bl[t];
-    } else if (t < v.nrec) {
-        const KvRec *r = v.rec + t;
-        slack = __ldg(&r->slack);
-        far = __ldg(&r->far);
-        thr = __ldg(&r->thr);
-        bar = __ldg(&r->bar);
-        bl = __ldg(&r->bl);
-    } else {
-        slack = kHuge;
-        far = v.nb;
-        thr = kHuge;
-        bar = v.B;
-        bl = v.B;
-    }
+// A warp's tile of 32 consecutive records past the staged ones (the walk's fields).
+struct KvTile {
+    long long *slack, *far, *thr;
+    int32_t *bar, *bl;
+};
+__device__ __forceinline__ KvTile kv_tile(unsigned char *smem, int w) {
+    KvTile tl;
+    tl.slack = reinterpret_cast<long long *>(smem + kEstStageBytes + (size_t)w * kEstTileBytes);
+    tl.far = tl.slack + 32;
+    tl.thr = tl.far + 32;
+    tl.bar = reinterpret_cast<int32_t *>(tl.thr + 32);
+    tl.bl = tl.bar + 32;
+    return tl;
 }
 
 // first index in [lo, lo + n) whose value is >= p, in a nondecreasing array
@@ -827,76 +821,131 @@ __device__ __forceinline__ int kv_lower_bound(const int32_t *a, int lo, int n, i
     return lo;
 }
 
-// One (query, instance) candidate: its features and first-token record, or an error.
-// The query waits (pre = p) until the first record whose admission bound reaches p,
-// found by binary search over the bounds' running maximum; from there it holds ctx
-// tokens in `held` blocks and pre still to prefill.  In a batch it is preempted if
-// the residents' scan leaves a slack below its blocks, or if its own tokens need more
-// blocks than are free to it (it is the last running request: it preempts itself);
-// a preempted query recomputes its whole context and may be readmitted in the same
-// batch.  Token counts stay below p + 2 <= 2^31.
+// A candidate's walk: whether it runs, its prefill left, its context, the blocks it
+// holds and its own Eq. 9 features so far.
+struct KvWalk {
+    bool run;
+    int pre, ctx, held;
+    long long o1, o2, o3, o4;
+};
+
+// One batch (record) of a candidate's walk; true if its first token falls in it.  A
+// running query is preempted if the residents' scan leaves a slack below its blocks,
+// or if its own tokens need more blocks than are free to it (it is the last running
+// request: it preempts itself); a preempted query recomputes its whole context and may
+// be readmitted in the same batch.  Token counts stay below p + 2 <= 2^31.
 template <int MODE>
-__device__ int kv_candidate(const KvView &v, const KvStage &st, int p, long long F[5], int &lt) {
-    int lo;
-    if (v.ns > 0 && st.pmx[v.ns - 1] >= p) lo = kv_lower_bound(st.pmx, 0, v.ns, p);
-    else lo = kv_lower_bound(v.pmx, v.ns, v.nrec - v.ns, p);
-    if (lo == v.nrec && !v.done) return kETraj;
-    // after the records the instance is empty; the query then needs at most
-    // ceil(p / B) + 2 batches
-    const int limit = v.nrec + (v.done ? (p / v.B + 3) : 0);
-    bool run = false;
-    int pre = p, ctx = 0, held = 0;
-    long long o1 = 0, o2 = 0, o3 = 0, o4 = 0;
-    int t = lo;
-    for (;; ++t) {
-        if (t >= limit) return kETraj;
-        long long slack, far, thr;
-        int bar, bl;
-        kv_record(v, st, t, slack, far, thr, bar, bl);
-        if (run) {
-            if (slack < held) {  // a resident needs the query's blocks
-                pre += ctx;
-                ctx = 0;
-                held = 0;
-                run = false;
-            } else if (bar > 0) {
-                const int x = pre > 0 ? min(pre, bar) : 1;
-                const int nh = dblk(v.dv, ctx + x);
-                if (nh > far) {  // its own tokens do not fit: it preempts itself
-                    pre += ctx;
-                    ctx = 0;
-                    held = 0;
-                    run = false;
-                } else {
-                    held = nh;
-                    if (pre > 0) {
-                        o1 += x;
-                        o4 += (long long)x * ctx + (long long)x * (x + 1) / 2;
-                        ctx += x;
-                        pre -= x;
-                        if (pre == 0 && MODE == 1) break;
-                    } else {
-                        o2 += 1;
-                        o3 += ctx;
-                        break;
-                    }
-                    continue;
-                }
+__device__ __forceinline__ bool kv_step(KvWalk &w, const Div32 &dv, long long slack, long long far, long long thr,
+                                        int bar, int bl) {
+    if (w.run) {
+        if (slack < w.held) {  // a resident needs the query's blocks
+            w.pre += w.ctx;
+            w.ctx = 0;
+            w.held = 0;
+            w.run = false;
+        } else if (bar > 0) {
+            const int x = w.pre > 0 ? min(w.pre, bar) : 1;
+            const int nh = dblk(dv, w.ctx + x);
+            if (nh > far) {  // its own tokens do not fit: it preempts itself
+                w.pre += w.ctx;
+                w.ctx = 0;
+                w.held = 0;
+                w.run = false;
             } else {
-                continue;  // no budget reached the query this batch
+                w.held = nh;
+                if (w.pre > 0) {
+                    w.o1 += x;
+                    w.o4 += (long long)x * w.ctx + (long long)x * (x + 1) / 2;
+                    w.ctx += x;
+                    w.pre -= x;
+                    return w.pre == 0 && MODE == 1;
+                }
+                w.o2 += 1;
+                w.o3 += w.ctx;
+                return true;
             }
-        }
-        if (pre <= thr) {  // admission (pre == p while waiting)
-            const int x = min(pre, bl);
-            held = dblk(v.dv, x);
-            o1 += x;
-            o4 += (long long)x * (x + 1) / 2;
-            ctx = x;
-            pre -= x;
-            run = true;
-            if (pre == 0 && MODE == 1) break;
+        } else {
+            return false;  // no budget reached the query this batch
         }
     }
+    if (w.pre <= thr) {  // admission (pre == p while waiting)
+        const int x = min(w.pre, bl);
+        w.held = dblk(dv, x);
+        w.o1 += x;
+        w.o4 += (long long)x * (x + 1) / 2;
+        w.ctx = x;
+        w.pre -= x;
+        w.run = true;
+        return w.pre == 0 && MODE == 1;
+    }
+    return false;
+}
+
+// The (query, instance) candidates of a warp's lanes (one instance, `live`: the lane
+// has one), called by all 32 lanes: each candidate's features and first-token record,
+// or an error.  The query waits (pre = p) until the first record whose admission bound
+// reaches p, found by binary search over the bounds' running maximum (the staged part
+// in shared memory, the rest in global memory), and is followed from there record by
+// record to its first token: through the staged records alone, then through the warp's
+// tile, which holds the 32 records from the least one a lane still needs (one load of
+// 32 records for the warp instead of one dependent load per record and lane).
+template <int MODE>
+__device__ int kv_candidate(const KvView &v, const KvStage &st, const KvTile &tl, int lane, bool live, int p,
+                            long long F[5], int &lt) {
+    int err = 0, t = 0;
+    KvWalk w = {false, p, 0, 0, 0, 0, 0, 0};
+    bool fin = !live;
+    if (live) {
+        int lo;
+        if (v.ns > 0 && st.pmx[v.ns - 1] >= p) lo = kv_lower_bound(st.pmx, 0, v.ns, p);
+        else lo = kv_lower_bound(v.pmx, v.ns, v.nrec - v.ns, p);
+        if (lo == v.nrec && !v.done) {
+            err = kETraj;
+            fin = true;
+        }
+        for (t = lo; !fin && t < v.ns;) {
+            if (kv_step<MODE>(w, v.dv, st.slack[t], st.far[t], st.thr[t], st.bar[t], st.bl[t])) fin = true;
+            else ++t;
+        }
+    }
+    // after the records the instance is empty; the query then needs at most
+    // ceil(p / B) + 2 batches
+    const int limit = live ? v.nrec + (v.done ? (p / v.B + 3) : 0) : 0;
+    for (;;) {
+        if (__ballot_sync(kFull, !fin) == 0u) break;
+        const int base = __reduce_min_sync(kFull, fin ? 0x7fffffff : t);  // >= ns
+        {
+            const int r = base + lane;
+            long long sl = kHuge, fa = v.nb, th = kHuge;  // past the records: an empty batch
+            int ba = v.B, bb = v.B;
+            if (r < v.nrec) {
+                const KvRec *rr = v.rec + r;
+                sl = __ldg(&rr->slack);
+                fa = __ldg(&rr->far);
+                th = __ldg(&rr->thr);
+                ba = __ldg(&rr->bar);
+                bb = __ldg(&rr->bl);
+            }
+            tl.slack[lane] = sl;
+            tl.far[lane] = fa;
+            tl.thr[lane] = th;
+            tl.bar[lane] = ba;
+            tl.bl[lane] = bb;
+        }
+        __syncwarp();
+        while (!fin && t < base + 32) {
+            if (t >= limit) {
+                err = kETraj;
+                fin = true;
+                break;
+            }
+            const int k = t - base;
+            if (kv_step<MODE>(w, v.dv, tl.slack[k], tl.far[k], tl.thr[k], tl.bar[k], tl.bl[k])) fin = true;
+            else ++t;
+        }
+        __syncwarp();  // the tile is read before the next one is written
+    }
+    if (!live || err) return err;
     lt = t;
     const int tc = min(t, v.nrec - 1);
     long long cf[4] = {0, 0, 0, 0};
@@ -905,10 +954,10 @@ __device__ int kv_candidate(const KvView &v, const KvStage &st, int p, long long
         for (int k = 0; k < 4; ++k) cf[k] = __ldg(&r->cf[k]);
     }
     F[0] = v.fcum[0] + t + 1;
-    F[1] = v.fcum[1] + cf[0] + o1;
-    F[2] = v.fcum[2] + cf[1] + o2;
-    F[3] = v.fcum[3] + cf[2] + o3;
-    F[4] = v.fcum[4] + cf[3] + o4;
+    F[1] = v.fcum[1] + cf[0] + w.o1;
+    F[2] = v.fcum[2] + cf[1] + w.o2;
+    F[3] = v.fcum[3] + cf[2] + w.o3;
+    F[4] = v.fcum[4] + cf[3] + w.o4;
     return 0;
 }
 
@@ -1086,7 +1135,9 @@ __global__ void __launch_bounds__(kEstWarps * 32, 3) k_kv_estimate(const KvEst a
     const int gy = gridDim.y;
     const int ng = min(kEstGroup, (c.I - (int)blockIdx.y + gy - 1) / gy);
     const int active = load_acquire(&a.ctl->active);
-    for (int gw = w; gw < ng; gw += kEstWarps) {  // warp w stages instances w, w + 8, ...
+    // the group's views, a thread each
+    if ((int)threadIdx.x < ng) {
+        const int gw = threadIdx.x;
         const int j = gw * gy + blockIdx.y;
         KvView v;
         v.nb = a.kv.nb[j];
@@ -1108,42 +1159,47 @@ __global__ void __launch_bounds__(kEstWarps * 32, 3) k_kv_estimate(const KvEst a
             v.rec = sb.kvr + (size_t)j * a.kv.horizon;
             v.pmx = sb.kvp + (size_t)j * a.kv.horizon;
             v.ns = min(v.nrec, kEstStage);
-            const KvStage st = kv_stage(est_smem, gw);
-            // the loads of the staged fields issued before their stores (one memory
-            // round trip)
-            constexpr int kPer = (kEstStage + 31) / 32;
-            {
-                constexpr int h = 0;
-                long long f_sl[kPer], f_fa[kPer], f_th[kPer];
-                int f_ba[kPer], f_bl[kPer], f_pm[kPer];
+        }
+        sv[gw] = v;
+    }
+    __syncthreads();
+    // the walk's fields of the instances' leading records, staged by every thread of the
+    // CTA in rounds whose loads are all issued before their stores
+    if (active >= 0) {
+        constexpr int kRound = 4;
+        constexpr int kAll = kEstGroup * kEstStage;
+        for (int r0 = 0; r0 < kAll; r0 += kRound * kEstWarps * 32) {
+            long long f_sl[kRound], f_fa[kRound], f_th[kRound];
+            int f_ba[kRound], f_bl[kRound], f_pm[kRound];
 #pragma unroll
-                for (int k = 0; k < kPer; ++k) {
-                    const int t = lane + 32 * (k + h * kPer);
-                    if (t < v.ns) {
-                        const KvRec *r = v.rec + t;
-                        f_sl[k] = __ldg(&r->slack);
-                        f_fa[k] = __ldg(&r->far);
-                        f_th[k] = __ldg(&r->thr);
-                        f_ba[k] = __ldg(&r->bar);
-                        f_bl[k] = __ldg(&r->bl);
-                        f_pm[k] = __ldg(v.pmx + t);
-                    }
+            for (int k = 0; k < kRound; ++k) {
+                const int idx = r0 + (int)threadIdx.x + k * kEstWarps * 32;
+                const int gw = idx / kEstStage, t = idx - gw * kEstStage;
+                if (gw < ng && t < sv[gw].ns) {
+                    const KvRec *r = sv[gw].rec + t;
+                    f_sl[k] = __ldg(&r->slack);
+                    f_fa[k] = __ldg(&r->far);
+                    f_th[k] = __ldg(&r->thr);
+                    f_ba[k] = __ldg(&r->bar);
+                    f_bl[k] = __ldg(&r->bl);
+                    f_pm[k] = __ldg(sv[gw].pmx + t);
                 }
+            }
 #pragma unroll
-                for (int k = 0; k < kPer; ++k) {
-                    const int t = lane + 32 * (k + h * kPer);
-                    if (t < v.ns) {
-                        st.slack[t] = f_sl[k];
-                        st.far[t] = f_fa[k];
-                        st.thr[t] = f_th[k];
-                        st.bar[t] = f_ba[k];
-                        st.bl[t] = f_bl[k];
-                        st.pmx[t] = f_pm[k];
-                    }
+            for (int k = 0; k < kRound; ++k) {
+                const int idx = r0 + (int)threadIdx.x + k * kEstWarps * 32;
+                const int gw = idx / kEstStage, t = idx - gw * kEstStage;
+                if (gw < ng && t < sv[gw].ns) {
+                    const KvStage st = kv_stage(est_smem, gw);
+                    st.slack[t] = f_sl[k];
+                    st.far[t] = f_fa[k];
+                    st.thr[t] = f_th[k];
+                    st.bar[t] = f_ba[k];
+                    st.bl[t] = f_bl[k];
+                    st.pmx[t] = f_pm[k];
                 }
             }
         }
-        if (lane == 0) sv[gw] = v;
     }
     __syncthreads();
     // the work: one query per distinct prompt length, or every query, by length
@@ -1178,17 +1234,22 @@ __global__ void __launch_bounds__(kEstWarps * 32, 3) k_kv_estimate(const KvEst a
         const int i = i_cur, p = p_cur;
         int i_nx, p_nx;
         fetch(it_next, i_nx, p_nx);
+        // every lane of the warp takes part in the walks (their record tiles)
+        const KvView &v = sv[g];
+        long long F[5] = {-1, -1, -1, -1, -1};
+        int lt = -1;
+        int err = 0;
+        // a query with one output token: its prompt below the context limit and
+        // its first token within the instance's blocks
         if (i >= 0) {
-            const KvView &v = sv[g];
-            long long F[5] = {-1, -1, -1, -1, -1};
-            int lt = -1;
-            int err;
-            // a query with one output token: its prompt below the context limit and
-            // its first token within the instance's blocks
             if (active < 0) err = kENoState;
             else if (!(p >= 1 && p <= c.pmax && (long long)p < v.mctx && kv_blocks32(p + 1, v.bs) <= v.nb))
                 err = kEInval;
-            else err = kv_candidate<MODE>(v, kv_stage(est_smem, g), p, F, lt);
+        }
+        const int werr = kv_candidate<MODE>(v, kv_stage(est_smem, g), kv_tile(est_smem, w), lane,
+                                            i >= 0 && err == 0, p, F, lt);
+        if (err == 0) err = werr;
+        if (i >= 0) {
             float tt = kNaN;
             if (err) {
                 record_status(a.ctl, err);
