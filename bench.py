@@ -706,8 +706,8 @@ def run_kv(args, dev, wl, flush):
                                    "k_kv_estimate, k_kv_expand)", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                          "frac": ach / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs, copy)",
                          "algorithmic_bytes": nbytes, "traffic": None,
-                         "note": "the call's six kernels together; k_kv_estimate alone read 4.92 MB and wrote "
-                                 "0.19 MB per launch (ncu); the load is one dependency chain per instance"}}
+                         "note": "the call's six kernels together; k_kv_estimate alone read 2.35 MB and wrote "
+                                 "0.85 MB per launch (ncu); the load is one dependency chain per instance"}}
 
 
 def run_avgcase(args, dev, wl, flush):
