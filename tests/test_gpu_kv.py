@@ -149,6 +149,44 @@ def test_horizon_exceeded():
     rt.close()
 
 
+def test_long_walks_across_record_tiles():
+    # pool256 under the bench's limits: a candidate whose first token comes more than
+    # 84 batches after the earliest one on its instance walked past the 52 staged
+    # leading records and through two or more of the warp's 32-record tiles; those
+    # candidates match the oracle exactly.  With a horizon of 40 records (below the
+    # staged count) a walk past an unfinished instance's records is cut (NaN, LR_ETRAJ)
+    # and the others still match.
+    wl = W.make_workload("pool256")
+    limits = W.kv_limits(wl, 11, block_sizes=(16,))
+    rng = np.random.default_rng(9)
+    for horizon in (4096, 40):
+        rt = make(wl, limits, horizon=horizon)
+        t, fb, F = gpu_estimate(rt, wl)
+        status = rt.status()
+        rt.close()
+        cut = np.isnan(t)
+        assert (fb[cut] == -1).all() and (F[cut] == -1).all()
+        assert status == (R().LR_ETRAJ if cut.any() else R().LR_OK)
+        fbm = np.where(cut, np.iinfo(np.int32).max, fb)
+        far = np.where(cut, -1, fb - fbm.min(axis=0, keepdims=True))
+        # one query per (prompt length, instance): the other queries' rows are copies
+        _, first = np.unique(wl.prompt_len, return_index=True)
+        sub = far[first]
+        qi, cj = np.nonzero(sub > 84)
+        if horizon == 4096:
+            assert len(qi) > 50
+        else:
+            qi, cj = np.nonzero(~cut[first])
+            assert cut.any() and len(qi) > 0
+        pick = rng.choice(len(qi), min(len(qi), 1500), replace=False)
+        cq, cj = first[qi[pick]], cj[pick]
+        st, eF, elt, et, _ = oracle.estimate_matrix_kv(wl, *limits, cand_q=cq, cand_j=cj)
+        assert (st == 0).all()
+        np.testing.assert_array_equal(F[cq, cj], eF)
+        np.testing.assert_array_equal(fb[cq, cj], elt)
+        np.testing.assert_array_equal(bits(t[cq, cj]), bits(et))
+
+
 def test_invalid_snapshot_keeps_the_live_one():
     wl = W.small_workload(63, num_instances=9, num_models=2, num_queries=20, budget_range=(8, 96), min_gap=8)
     bs, nb, mc = W.kv_limits(wl, 9, block_sizes=(4,))
