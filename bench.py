@@ -275,9 +275,10 @@ def run_gpu(args):
 
     # End to end, as a serving loop runs it: every step copies its snapshot and queries
     # from pinned host memory, ingests and routes them (K1 || K2 as above) and copies
-    # the routing result back to pinned host memory, which the host reads.  Two device
-    # buffer sets alternate, so step k+1's upload (copy stream) overlaps step k's
-    # compute; a step's time runs from after its L2 flush to its result's arrival.
+    # the routing result back to pinned host memory, which the host reads.  NB buffer
+    # sets rotate, so step k+1's upload (copy stream) overlaps step k's compute, and the
+    # host waits for each step's result HOST_LAG steps later (NB > HOST_LAG keeps that
+    # result's host buffer from being overwritten before it is read).
     # The step's inputs (snapshot arrays, then prompts, predicted lengths and accuracies)
     # sit in one pinned host buffer and arrive with one copy; the routing results go back
     # with one copy too (one large copy moves ~200 GB/s here, ten separate ones far less).
@@ -295,18 +296,19 @@ def run_gpu(args):
         return v[:len(state)], v[len(state):]
 
     res_keys = ("assign", "util", "ttft_chosen")
-    dev_in = [torch.empty(int(offs[-1]), dtype=torch.int32, device=dev) for _ in range(2)]
+    NB, HOST_LAG = 3, 2
+    dev_in = [torch.empty(int(offs[-1]), dtype=torch.int32, device=dev) for _ in range(NB)]
     bufs = [views(f) for f in dev_in]
-    dev_out = [torch.empty(3 * Q, dtype=torch.int32, device=dev) for _ in range(2)]
+    dev_out = [torch.empty(3 * Q, dtype=torch.int32, device=dev) for _ in range(NB)]
     outs = [{"assign": f[:Q].view(1, Q), "util": f[Q:2 * Q].view(torch.float32).view(1, Q),
              "ttft_chosen": f[2 * Q:].view(torch.float32).view(1, Q)} for f in dev_out]
-    host_out_flat = [torch.empty(3 * Q, dtype=torch.int32).pin_memory() for _ in range(2)]
+    host_out_flat = [torch.empty(3 * Q, dtype=torch.int32).pin_memory() for _ in range(NB)]
     host_outs = [{"assign": f[:Q].view(1, Q)} for f in host_out_flat]
     h2d = int(offs[-1]) * 4
     d2h = 3 * Q * 4
     copy_stream = torch.cuda.Stream(device=dev)
     g_up, g_step = [], []
-    for b in range(2):
+    for b in range(NB):
         dst, dqq = bufs[b]
 
         def upload(b=b):
@@ -338,32 +340,33 @@ def run_gpu(args):
         # `steps` pipelined steps with no L2 flush inside the loop (each step's inputs
         # arrive by their own host->device copy).  Three streams: uploads, compute and
         # read-backs, so that step k's read-back and step k+1's upload overlap step
-        # k+1's compute.  Returns the span from the first upload's issue to the last
-        # result's arrival in host memory, and each step's latency from its upload's
-        # issue to its result's arrival.
+        # k+1's compute; the host waits for step k - HOST_LAG's result after issuing
+        # step k.  Returns the span from the first upload's issue to the last result's
+        # arrival in host memory, and each step's latency from its upload's issue to
+        # its result's arrival.
         ev_up0 = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
         ev1 = [torch.cuda.Event() for _ in range(steps)]          # compute done
         ev2 = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]  # result in host memory
         up = [torch.cuda.Event() for _ in range(steps)]
         for k in range(steps):
-            b = k & 1
-            if k >= 2:
-                copy_stream.wait_event(ev1[k - 2])  # step k-2 has read buffer set b's inputs
+            b = k % NB
+            if k >= NB:
+                copy_stream.wait_event(ev1[k - NB])  # step k-NB has read buffer set b's inputs
             ev_up0[k].record(copy_stream)
             with torch.cuda.stream(copy_stream):
                 g_up[b].replay()
             up[k].record(copy_stream)
             stream.wait_event(up[k])
-            if k >= 2:
-                stream.wait_event(ev2[k - 2])  # step k-2's results have left buffer set b
+            if k >= NB:
+                stream.wait_event(ev2[k - NB])  # step k-NB's results have left buffer set b
             g_step[b].replay()
             ev1[k].record(stream)
             d2h_stream.wait_event(ev1[k])
             with torch.cuda.stream(d2h_stream):
                 host_out_flat[b].copy_(dev_out[b], non_blocking=True)
             ev2[k].record(d2h_stream)
-            if k >= 1:
-                ev2[k - 1].synchronize()  # the host has the previous step's result
+            if k >= HOST_LAG:
+                ev2[k - HOST_LAG].synchronize()  # the host has step k-HOST_LAG's result
         torch.cuda.synchronize()
         return ev_up0[0].elapsed_time(ev2[-1]), [ev_up0[k].elapsed_time(ev2[k]) for k in range(steps)]
 
@@ -371,8 +374,8 @@ def run_gpu(args):
     KE = max(3, min(K, 2000))
     e2e_span, e2e_lat = run_e2e(KE)
     e2e_mean = _max_over_ranks(e2e_span / KE, world)
-    host_out = host_outs[(KE - 1) & 1]
-    out = outs[(KE - 1) & 1]
+    host_out = host_outs[(KE - 1) % NB]
+    out = outs[(KE - 1) % NB]
     assert rt.status() == R.LR_OK
     ok = torch.equal(host_out["assign"].to(dev), out["assign"])
     if not ok:
@@ -430,9 +433,9 @@ def run_gpu(args):
                     "note": "through the public API (lr_load_state + lr_route): per step the snapshot and "
                             "queries are copied from pinned host memory on an upload stream (one packed copy), "
                             "ingested and routed (K1 || K2), and the result copied back to pinned host memory "
-                            "on a read-back stream (one copy), which the host reads one step later; two device "
-                            "buffer sets alternate, so a step's upload and the previous step's read-back overlap "
-                            "its compute.  ms_per_step = span from the first upload's issue to the last result's "
+                            f"on a read-back stream (one copy), which the host waits for {HOST_LAG} steps later; "
+                            f"{NB} device and host buffer sets rotate, so a step's upload and the previous step's "
+                            "read-back overlap its compute.  ms_per_step = span from the first upload's issue to the last result's "
                             "arrival / steps (no L2 flush inside the loop: every step's inputs arrive by copy); "
                             "latency = a step's upload issue to its result's arrival"},
             "gpu_launches": 2 * K, "clocks": clocks, "wall_s_timed_region": t_wall,
