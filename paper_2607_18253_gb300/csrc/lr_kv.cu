@@ -781,7 +781,8 @@ __device__ __forceinline__ KvStage kv_stage(unsigned char *smem, int g) {
 }
 
 // One instance as the estimate reads it: the first `ns` records (with their admission
-// maxima) from shared memory, the rest from global memory.
+// maxima) from shared memory; later records through the warp's tile, and their
+// admission maxima and the residents' features from global memory.
 struct KvView {
     const KvRec *rec;
     const int32_t *pmx;
